@@ -1,0 +1,311 @@
+"""ctypes wrapper of the plain C oracle (gracekv_oracle.c).
+
+TEST INFRASTRUCTURE ONLY: tests/, __graft_entry__.smoke() and bench.py's
+CPU-baseline leg use it to check and time against the CUDA path.  It shares
+nothing with the CUDA library; inputs are widened to float64 exactly.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import dataclasses
+import os
+import subprocess
+from typing import Optional
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+SRC = os.path.join(HERE, "gracekv_oracle.c")
+LIB = os.path.join(HERE, "liboracle.so")
+
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc (no fast-math, no FMA contraction)."""
+    if force or not os.path.exists(LIB) or os.path.getmtime(LIB) < max(
+            os.path.getmtime(SRC), os.path.getmtime(os.path.join(HERE, "gracekv_oracle.h"))):
+        tmp = LIB + f".tmp{os.getpid()}"
+        subprocess.check_call(["gcc", "-O2", "-ffp-contract=off", "-fno-fast-math", "-std=c11",
+                               "-shared", "-fPIC", "-o", tmp, SRC, "-lm"])
+        os.replace(tmp, LIB)
+    return LIB
+
+
+class Params(C.Structure):
+    _fields_ = [
+        ("L", C.c_int32), ("G", C.c_int32), ("Hq", C.c_int32), ("T", C.c_int32),
+        ("d", C.c_int32), ("W", C.c_int32),
+        ("ctx_start", C.c_int32), ("ctx_end", C.c_int32), ("recent", C.c_int32),
+        ("rope_base", C.c_double),
+        ("n_min", C.c_int32), ("n_max", C.c_int32), ("n0", C.c_int32),
+        ("lambda_stab", C.c_double), ("lambda_s", C.c_double), ("lambda_d", C.c_double),
+        ("lambda_n", C.c_double), ("c_cut", C.c_double),
+        ("seg_layers", C.c_int32 * 8), ("n_seg_layers", C.c_int32),
+        ("windows", C.c_int32 * 4), ("n_windows", C.c_int32),
+        ("k_cand", C.c_int32),
+        ("lambda_kappa", C.c_double), ("lambda_Z", C.c_double), ("lambda_M", C.c_double),
+        ("eps", C.c_double), ("base_frac", C.c_double),
+        ("disp_mode", C.c_int32),
+    ]
+
+
+_NODE_I32 = ["lg", "slot", "a", "b", "parent", "child0", "nchild", "form", "cost"]
+_NODE_F64 = ["D", "Ddrop", "R", "U", "kappa", "kscale", "m_cut", "m_form", "m_topk", "m_ext"]
+
+
+class Nodes(C.Structure):
+    _fields_ = ([("cap", C.c_int64), ("count", C.c_int64)]
+                + [(n, C.POINTER(C.c_int32)) for n in _NODE_I32]
+                + [(n, C.POINTER(C.c_double)) for n in _NODE_F64])
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        build()
+        _lib = C.CDLL(LIB)
+    return _lib
+
+
+def _p(a, t):
+    return a.ctypes.data_as(C.POINTER(t))
+
+
+def _f64(x) -> np.ndarray:
+    if x is None:
+        return None
+    if hasattr(x, "detach"):
+        x = x.detach().to("cpu").double().numpy()
+    return np.ascontiguousarray(np.asarray(x, dtype=np.float64))
+
+
+PAPER_DEFAULTS = dict(
+    recent=32, n_min=16, n_max=128, n0=64, lambda_stab=0.25, lambda_s=0.15,
+    lambda_d=0.25, lambda_n=0.10, c_cut=1.0, windows=(4, 8, 16), k_cand=16,
+    lambda_kappa=0.05, lambda_Z=0.25, lambda_M=0.75, eps=1e-6, base_frac=0.1,
+    seg_layers=(), disp_mode=0)
+
+
+def make_params(L, G, Hq, T, d, W, rope_base, ctx_start=0, ctx_end=None, **kw) -> Params:
+    o = dict(PAPER_DEFAULTS)
+    o.update(kw)
+    p = Params()
+    p.L, p.G, p.Hq, p.T, p.d, p.W = L, G, Hq, T, d, W
+    p.ctx_start = ctx_start
+    p.ctx_end = T if ctx_end is None else ctx_end
+    p.recent = o["recent"]
+    p.rope_base = float(rope_base)
+    p.n_min, p.n_max, p.n0 = o["n_min"], o["n_max"], o["n0"]
+    p.lambda_stab, p.lambda_s = o["lambda_stab"], o["lambda_s"]
+    p.lambda_d, p.lambda_n, p.c_cut = o["lambda_d"], o["lambda_n"], o["c_cut"]
+    sl = tuple(o["seg_layers"])
+    for i, v in enumerate(sl):
+        p.seg_layers[i] = v
+    p.n_seg_layers = len(sl)
+    for i, v in enumerate(o["windows"]):
+        p.windows[i] = v
+    p.n_windows = len(o["windows"])
+    p.k_cand = o["k_cand"]
+    p.lambda_kappa, p.lambda_Z, p.lambda_M = o["lambda_kappa"], o["lambda_Z"], o["lambda_M"]
+    p.eps, p.base_frac = o["eps"], o["base_frac"]
+    p.disp_mode = o["disp_mode"]
+    return p
+
+
+def budget(p: Params, B_total: int):
+    r = C.c_int32()
+    bf = C.c_int64()
+    rc = lib().orc_budget(C.byref(p), C.c_int64(B_total), C.byref(r), C.byref(bf))
+    if rc:
+        raise ValueError(f"budget rejected (rc={rc})")
+    return r.value, bf.value
+
+
+def curvature(p: Params, V, hidden=None):
+    V = _f64(V)
+    hid = _f64(hidden)
+    Dh = 0 if hid is None else hid.shape[-1]
+    kap = np.zeros(p.T)
+    nl = p.n_seg_layers or len({min(int(np.floor(r * p.L)), p.L - 1) for r in (0.33, 0.5, 0.67)})
+    klw = np.zeros((p.T, nl * p.n_windows))
+    rc = lib().orc_curvature(C.byref(p), _p(V, C.c_double),
+                             None if hid is None else _p(hid, C.c_double), C.c_int32(Dh),
+                             _p(kap, C.c_double), _p(klw, C.c_double))
+    assert rc == 0, rc
+    return kap, klw
+
+
+def robust_z(a):
+    a = _f64(a)
+    z = np.zeros_like(a)
+    rc = lib().orc_robust_z(_p(a, C.c_double), C.c_int32(a.size), _p(z, C.c_double))
+    assert rc == 0
+    return z
+
+
+def segment(p: Params, V, hidden=None, surprisal=None):
+    V = _f64(V)
+    hid = _f64(hidden)
+    sur = _f64(surprisal)
+    Dh = 0 if hid is None else hid.shape[-1]
+    N = p.ctx_end - p.recent - p.ctx_start
+    kap = np.zeros(p.T)
+    b = np.zeros(p.T)
+    cap = N + 2
+    starts = np.zeros(cap + 1, dtype=np.int32)
+    J = C.c_int32()
+    best = np.full(N + 1, -np.inf)
+    second = np.full(N + 1, -np.inf)
+    rc = lib().orc_segment(C.byref(p), _p(V, C.c_double),
+                           None if hid is None else _p(hid, C.c_double), C.c_int32(Dh),
+                           None if sur is None else _p(sur, C.c_double),
+                           _p(kap, C.c_double), _p(b, C.c_double), _p(starts, C.c_int32),
+                           C.c_int32(cap), C.byref(J), _p(best, C.c_double), _p(second, C.c_double))
+    assert rc == 0, rc
+    return dict(kappa=kap, b=b, slot_starts=starts[:J.value + 1].copy(), dp_best=best,
+                dp_second=second)
+
+
+def row_stats(p: Params, Q, K):
+    Q, K = _f64(Q), _f64(K)
+    n = p.L * p.Hq * p.W
+    m, Z, ZC = np.zeros(n), np.zeros(n), np.zeros(n)
+    rc = lib().orc_row_stats(C.byref(p), _p(Q, C.c_double), _p(K, C.c_double),
+                             _p(m, C.c_double), _p(Z, C.c_double), _p(ZC, C.c_double))
+    assert rc == 0
+    sh = (p.L, p.Hq, p.W)
+    return m.reshape(sh), Z.reshape(sh), ZC.reshape(sh)
+
+
+def token_values(p: Params, Q, K, m, Z):
+    Q, K = _f64(Q), _f64(K)
+    m, Z = _f64(m), _f64(Z)
+    Nc = p.ctx_end - p.recent - p.ctx_start
+    r = np.zeros(p.L * p.G * Nc)
+    rc = lib().orc_token_values(C.byref(p), _p(Q, C.c_double), _p(K, C.c_double),
+                                _p(m, C.c_double), _p(Z, C.c_double), _p(r, C.c_double))
+    assert rc == 0
+    return r.reshape(p.L, p.G, Nc)
+
+
+def eval_interval(p: Params, K, V, Q, m, Z, rtok, l, g, a, b):
+    K, V, Q, m, Z, rtok = map(_f64, (K, V, Q, m, Z, rtok))
+    D, Dd, lm = C.c_double(), C.c_double(), C.c_double()
+    pos = C.c_int32()
+    kt, vt = np.zeros(p.d), np.zeros(p.d)
+    rc = lib().orc_eval_interval(C.byref(p), _p(K, C.c_double), _p(V, C.c_double),
+                                 _p(Q, C.c_double), _p(m, C.c_double), _p(Z, C.c_double),
+                                 _p(rtok, C.c_double), *(C.c_int32(int(v)) for v in (l, g, a, b)),
+                                 C.byref(D), C.byref(Dd),
+                                 _p(kt, C.c_double), _p(vt, C.c_double), C.byref(pos),
+                                 C.byref(lm))
+    assert rc == 0
+    return dict(D=D.value, Ddrop=Dd.value, ktil=kt, vtil=vt, pos=pos.value, logm=lm.value)
+
+
+@dataclasses.dataclass
+class Trees:
+    nodes: dict           # field -> array (length count)
+    unit_Uadd: np.ndarray  # [L*G*J]
+    unit_root: np.ndarray  # [L*G*J]
+    n_slots: int
+    _keep: tuple = ()
+
+    def struct(self) -> Nodes:
+        ns = Nodes()
+        n = len(self.nodes["a"])
+        ns.cap = n
+        ns.count = n
+        for f in _NODE_I32:
+            setattr(ns, f, _p(self.nodes[f], C.c_int32))
+        for f in _NODE_F64:
+            setattr(ns, f, _p(self.nodes[f], C.c_double))
+        return ns
+
+
+def build_trees(p: Params, K, V, Q, kappa, slot_starts, m, Z, rtok, omega=None) -> Trees:
+    K, V, Q, kappa, m, Z, rtok, om = map(_f64, (K, V, Q, kappa, m, Z, rtok, omega))
+    ss = np.ascontiguousarray(np.asarray(slot_starts, dtype=np.int32))
+    J = len(ss) - 1
+    Nc = p.ctx_end - p.recent - p.ctx_start
+    cap = p.L * p.G * 2 * Nc + 8
+    arr = {f: np.zeros(cap, dtype=np.int32) for f in _NODE_I32}
+    arr.update({f: np.zeros(cap) for f in _NODE_F64})
+    ns = Nodes()
+    ns.cap = cap
+    for f in _NODE_I32:
+        setattr(ns, f, _p(arr[f], C.c_int32))
+    for f in _NODE_F64:
+        setattr(ns, f, _p(arr[f], C.c_double))
+    uadd = np.zeros(p.L * p.G * J)
+    uroot = np.zeros(p.L * p.G * J, dtype=np.int64)
+    rc = lib().orc_build_trees(C.byref(p), _p(K, C.c_double), _p(V, C.c_double),
+                               _p(Q, C.c_double), None if om is None else _p(om, C.c_double),
+                               _p(kappa, C.c_double), _p(ss, C.c_int32), C.c_int32(J),
+                               _p(m, C.c_double), _p(Z, C.c_double), _p(rtok, C.c_double),
+                               C.byref(ns), _p(uadd, C.c_double), _p(uroot, C.c_int64))
+    assert rc == 0, rc
+    n = ns.count
+    return Trees({f: arr[f][:n].copy() for f in arr}, uadd, uroot, J)
+
+
+def allocate(p: Params, B_free: int, tr: Trees):
+    ns = tr.struct()
+    nu = len(tr.unit_Uadd)
+    add_sel = np.zeros(nu, dtype=np.uint8)
+    split_sel = np.zeros(len(tr.nodes["a"]), dtype=np.uint8)
+    used = C.c_int64()
+    rc = lib().orc_allocate(C.byref(p), C.c_int64(B_free), C.c_int32(tr.n_slots), C.byref(ns),
+                            _p(tr.unit_Uadd, C.c_double), _p(tr.unit_root, C.c_int64),
+                            _p(add_sel, C.c_uint8), _p(split_sel, C.c_uint8), C.byref(used))
+    assert rc == 0
+    return add_sel, split_sel, used.value
+
+
+def gather(p: Params, K, V, rtok, tr: Trees, add_sel, split_sel, cap: int):
+    K, V, rtok = map(_f64, (K, V, rtok))
+    ns = tr.struct()
+    Ko = np.zeros((cap, p.d))
+    Vo = np.zeros((cap, p.d))
+    pos = np.zeros(cap, dtype=np.int32)
+    lm = np.zeros(cap)
+    lo = np.zeros(cap, dtype=np.int32)
+    hi = np.zeros(cap, dtype=np.int32)
+    off = np.zeros(p.L * p.G + 1, dtype=np.int64)
+    ne = C.c_int64()
+    rc = lib().orc_gather(C.byref(p), _p(K, C.c_double), _p(V, C.c_double),
+                          _p(rtok, C.c_double), C.c_int32(tr.n_slots), C.byref(ns),
+                          _p(tr.unit_root, C.c_int64), _p(add_sel, C.c_uint8),
+                          _p(split_sel, C.c_uint8), C.c_int64(cap), _p(Ko, C.c_double),
+                          _p(Vo, C.c_double), _p(pos, C.c_int32), _p(lm, C.c_double),
+                          _p(lo, C.c_int32), _p(hi, C.c_int32), _p(off, C.c_int64), C.byref(ne))
+    assert rc == 0, rc
+    E = ne.value
+    return dict(K=Ko[:E], V=Vo[:E], pos=pos[:E], log_m=lm[:E], src_lo=lo[:E], src_hi=hi[:E],
+                offsets=off)
+
+
+def run(K, V, Q, B_total: int, rope_base: float, *, ctx_start=0, ctx_end=None, omega=None,
+        surprisal=None, hidden=None, slot_starts=None, **overrides) -> dict:
+    """Whole compression pass on the oracle; returns every intermediate."""
+    L, G, T, d = K.shape
+    Hq, W = Q.shape[1], Q.shape[2]
+    p = make_params(L, G, Hq, T, d, W, rope_base, ctx_start, ctx_end, **overrides)
+    r_eff, B_free = budget(p, B_total)
+    p.recent = r_eff
+    K64, V64, Q64 = _f64(K), _f64(V), _f64(Q)
+    if slot_starts is None:
+        seg = segment(p, V64, hidden, surprisal)
+    else:
+        kap, _ = curvature(p, V64, hidden)
+        seg = dict(kappa=kap, b=None, slot_starts=np.asarray(slot_starts, np.int32) + p.ctx_start,
+                   dp_best=None, dp_second=None)
+    m, Z, ZC = row_stats(p, Q64, K64)
+    rtok = token_values(p, Q64, K64, m, Z)
+    tr = build_trees(p, K64, V64, Q64, seg["kappa"], seg["slot_starts"], m, Z, rtok, omega)
+    add_sel, split_sel, used = allocate(p, B_free, tr)
+    cap = B_total + L * G * (T - (p.ctx_end - p.ctx_start)) + 16
+    cache = gather(p, K64, V64, rtok, tr, add_sel, split_sel, cap)
+    return dict(params=p, r_eff=r_eff, B_free=B_free, seg=seg, m=m, Z=Z, ZC=ZC, rtok=rtok,
+                trees=tr, add_sel=add_sel, split_sel=split_sel, used=used, cache=cache)

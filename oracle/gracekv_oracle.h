@@ -1,0 +1,123 @@
+/*
+ * gracekv_oracle.h -- plain CPU oracle of the GraceKV prefill-time compression
+ * pass (arxiv 2608.07001, "Every Cache Entry Earns Its Place").
+ *
+ * TEST INFRASTRUCTURE ONLY.  This oracle exists to check the CUDA path; only
+ * tests/, __graft_entry__.smoke() and bench.py's CPU-baseline leg may load it.
+ * It shares no code, header, table or helper with the CUDA library.
+ *
+ * Everything is single-threaded fp64 arithmetic on the exact input values
+ * (bf16/fp32 inputs are widened to double by the caller), written as plain
+ * loops that follow the paper's definitions in the paper's order:
+ *
+ *   budget            Sec. App. A.1, Eq. (app_total_budget), (app_free_budget)
+ *   curvature         App. B.2, Eqs. (app_hidden_normalization) ..
+ *                     (app_stabilized_curvature)
+ *   boundary score    App. B.2, Eqs. (app_robust_z), (app_mad), (app_boundary_score)
+ *   DP segmentation   App. B.3, Eqs. (app_adjacent_difference) ..
+ *                     (app_terminal_predecessor)
+ *   row statistics    App. A.3 "Prototype distortion" (max-logit shift),
+ *                     App. A.4 Eq. (app_attention_probability)
+ *   token values      App. A.4 Eqs. (app_direct_relevance), (app_bottom_up_value)
+ *   prototypes        App. A.3 Eqs. (app_rope_prototype), (app_value_prototype),
+ *                     (app_effective_multiplicity)
+ *   distortion        App. A.3 Eqs. (app_original_attention_stats) ..
+ *                     (app_node_and_drop_distortion)
+ *   refinement        App. A.3 Eqs. (app_binary_split) .. (app_split_choice),
+ *                     App. B.4 Eq. (app_tree_split_candidates)
+ *   gains / costs     App. A.5 Eqs. (app_operation_gains) .. (app_unit_utility)
+ *   greedy allocation App. A.5 Stage II, App. C.3 (max-priority queue)
+ *   packing           App. A.5 "Frontier updates and physical packing"
+ *
+ * Readings of silent or ambiguous passages (each also listed in the design doc):
+ *   R1  trajectory h^(l)_t = concat_g v^(l,g)_t unless hidden states are given;
+ *       surprisal defaults to 0; omega defaults to 1; lambda_graph = 0.
+ *   R2  visible range of every probe = [0, T); probes = the W observation
+ *       queries; distortion probe u uses query head H(g)[u mod |H(g)|].
+ *   R3  b_i rewards a cut between positions i and i+1.
+ *   R4  median = lower median (rank floor((n-1)/2)).
+ *   R5  DP ties -> first maximum in ascending predecessor a.
+ *   R6  split candidates: top-K positions t in [a, b-2] by kappa (ties: lower
+ *       t), cut xi = t+1, plus midpoint xi = a + floor(n/2); kappa-hat is the
+ *       min-max normalisation of kappa over [a, b-2] (0 when flat); cut ties
+ *       -> smallest xi; extraction p* = argmax R_tok (ties: lower t);
+ *       binary wins a rho tie.
+ *   R7  normalisation of the mass weight = the probe's full partition over
+ *       [0, T) with the same max-logit shift.
+ *   R8  epsilon = 1e-6 wherever the paper writes epsilon without a value.
+ *   R9  p_v = round half to even of the mean position.
+ *   R10 single-token intervals store the original K/V, p = t, m = 1, D = 0.
+ *   R11 RoPE: half-split pairs (i, i + d/2), theta_i = base^(-2i/d),
+ *       RoPE^-1(k, t) = RoPE(k, -t); base 0 means keys carry no rotation.
+ *   R12 gains are clamped at 0; heap order (U desc, unit asc, a asc, b desc);
+ *       an unaffordable pop is discarded for good.
+ *
+ * Parity is pinned for every function here (see tests/test_oracle_*.py);
+ * no function is "parity unpinned".
+ */
+#ifndef GRACEKV_ORACLE_H
+#define GRACEKV_ORACLE_H
+#include <stdint.h>
+
+typedef struct {
+    int32_t L, G, Hq, T, d, W;
+    int32_t ctx_start, ctx_end;   /* context [c_s, c_e) inside [0, T) */
+    int32_t recent;               /* requested recent window r */
+    double rope_base;             /* 0: keys carry no RoPE */
+    int32_t n_min, n_max, n0;
+    double lambda_stab, lambda_s, lambda_d, lambda_n, c_cut;
+    int32_t seg_layers[8];
+    int32_t n_seg_layers;
+    int32_t windows[4];
+    int32_t n_windows;
+    int32_t k_cand;
+    double lambda_kappa, lambda_Z, lambda_M, eps, base_frac;
+    int32_t disp_mode;            /* 0: definition, 1: paper's prefix form */
+} orc_params;
+
+/* Per-node records of all trees (flat, capacity = L*G*2*N_c). */
+typedef struct {
+    int64_t cap;
+    int64_t count;      /* out */
+    int32_t *lg, *slot, *a, *b, *parent, *child0, *nchild, *form, *cost;
+    double *D, *Ddrop, *R, *U, *kappa, *kscale;
+    double *m_cut, *m_form, *m_topk, *m_ext;
+} orc_nodes;
+
+int orc_budget(const orc_params *p, int64_t B_total, int32_t *r_eff, int64_t *B_free);
+
+int orc_curvature(const orc_params *p, const double *V, const double *hidden, int32_t Dh,
+                  double *kappa_out, double *kappa_lw_out);
+int orc_robust_z(const double *a, int32_t n, double *z);
+int orc_segment(const orc_params *p, const double *V, const double *hidden, int32_t Dh,
+                const double *surprisal, double *kappa_out, double *b_out,
+                int32_t *slot_starts, int32_t cap, int32_t *n_slots,
+                double *dp_best, double *dp_second);
+
+int orc_row_stats(const orc_params *p, const double *Q, const double *K,
+                  double *m, double *Z, double *ZC);
+int orc_token_values(const orc_params *p, const double *Q, const double *K,
+                     const double *m, const double *Z, double *rtok);
+
+int orc_eval_interval(const orc_params *p, const double *K, const double *V,
+                      const double *Q, const double *m, const double *Z,
+                      const double *rtok, int32_t l, int32_t g, int32_t a, int32_t b,
+                      double *D, double *Ddrop, double *ktil, double *vtil,
+                      int32_t *pos, double *logm);
+
+int orc_build_trees(const orc_params *p, const double *K, const double *V, const double *Q,
+                    const double *omega, const double *kappa, const int32_t *slot_starts,
+                    int32_t n_slots, const double *m, const double *Z, const double *rtok,
+                    orc_nodes *nodes, double *unit_Uadd, int64_t *unit_root);
+
+int orc_allocate(const orc_params *p, int64_t B_free, int32_t n_slots,
+                 const orc_nodes *nodes, const double *unit_Uadd, const int64_t *unit_root,
+                 uint8_t *add_sel, uint8_t *split_sel, int64_t *used);
+
+int orc_gather(const orc_params *p, const double *K, const double *V, const double *rtok,
+               int32_t n_slots, const orc_nodes *nodes, const int64_t *unit_root,
+               const uint8_t *add_sel, const uint8_t *split_sel, int64_t cap,
+               double *K_out, double *V_out, int32_t *pos, double *log_m,
+               int32_t *src_lo, int32_t *src_hi, int64_t *offsets, int64_t *n_entries);
+
+#endif
