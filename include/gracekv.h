@@ -1,0 +1,198 @@
+/*
+ * gracekv.h -- C ABI of the GraceKV prefill-time KV-cache compression pass
+ * (arxiv 2608.07001, "Every Cache Entry Earns Its Place: Global Allocation of
+ * Resolution and Coverage for KV Cache Compression"), implemented as
+ * hand-written CUDA kernels for sm_103a (GB300).
+ *
+ * The pass follows the problem statement of Sec. 3.1 / App. A.1: after one
+ * prefill, the cache K, V of every layer l and KV head g is compressed into a
+ * ragged cache of at most B_total entries (one entry = one stored K/V pair).
+ * Four calls, in this order, on one context:
+ *
+ *   gracekv_segment      curvature-guided slot partition      (App. B.2-B.3)
+ *   gracekv_build_trees  prototype trees, node values, gains  (App. A.3-A.5)
+ *   gracekv_allocate     global greedy Add/Split allocation   (App. A.5, C.3)
+ *   gracekv_gather       ragged compressed cache + index map  (App. A.5)
+ *
+ * Conventions for every call:
+ *   - Tensor arguments are DEVICE pointers to contiguous row-major arrays owned
+ *     by the caller; the library never frees or retains them past the call.
+ *     Arguments named *_host are host pointers.
+ *   - K and V have layout [L][G][T][d] (G = number of KV heads); Q (the
+ *     observation-window queries, placed after the input at positions
+ *     T..T+W-1, all seeing [0, T)) has layout [L][Hq][W][d]; query head h
+ *     belongs to KV head h / (Hq / G).  Element type = params.dtype
+ *     (fp32 or bf16) for K, V, Q, K_out and V_out.
+ *   - `stream` is a cudaStream_t passed as void*; work is enqueued on it.
+ *     Calls that return a host count (*_host) synchronise that stream once.
+ *   - Every call returns a gkv_status and never aborts or throws.  A CUDA
+ *     error makes the context sticky-failed (GKV_ECUDA on every later call);
+ *     gracekv_last_error() describes the first failure.
+ *   - Calls out of order return GKV_ESTATE without enqueuing work.
+ *   - A context and its workspace belong to one device (the device current
+ *     at gracekv_create); calls on one context must not overlap.
+ */
+#ifndef GRACEKV_H
+#define GRACEKV_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define GRACEKV_ABI_VERSION 1
+
+typedef enum {
+    GKV_OK = 0,
+    GKV_EINVAL = 1,        /* bad shape, pointer or hyper-parameter */
+    GKV_EBUDGET = 2,       /* budget cannot hold L*G*4 recent entries, or no context left */
+    GKV_ENOMEM = 3,        /* device workspace allocation failed */
+    GKV_ECUDA = 4,         /* a CUDA call failed (context is now sticky-failed) */
+    GKV_ETIMEOUT = 5,      /* a bounded device-side wait gave up */
+    GKV_ENONFINITE = 6,    /* a NaN/Inf input or intermediate was found */
+    GKV_ESTATE = 7,        /* call out of order, or context already failed */
+    GKV_EUNSUPPORTED = 8,  /* valid per the paper but not built here (see message) */
+    GKV_ECAPACITY = 9      /* an output buffer is too small */
+} gkv_status;
+
+typedef enum { GKV_F32 = 0, GKV_BF16 = 1 } gkv_dtype;
+
+typedef struct gracekv_ctx gracekv_ctx;
+
+/*
+ * Shapes and hyper-parameters.  Defaults (gracekv_default_params) are the
+ * paper's: App. A.1 (recent window 32), App. B.2 (windows {4,8,16},
+ * lambda_stab 0.25, lambda_s 0.15, segmentation layers at relative depths
+ * 0.33/0.50/0.67), App. B.3 (n_min 16, n_max 128, n0 64, lambda_d 0.25,
+ * lambda_n 0.10, c_cut 1.0), App. A.3 (K = 16 split candidates, lambda_kappa
+ * 0.05, lambda_Z 0.25, lambda_M 0.75, value base 0.1), epsilon 1e-6.
+ */
+typedef struct {
+    int32_t L, G, Hq, T, d, W;     /* layers, KV heads, query heads, tokens, head dim, probes */
+    int32_t dtype;                 /* gkv_dtype of K, V, Q, K_out, V_out */
+    int32_t ctx_start, ctx_end;    /* context [c_s, c_e) inside [0, T) (App. A.1) */
+    int32_t recent;                /* requested recent window r (shrinks to fit the budget) */
+    int64_t budget;                /* B_total = floor(L G N_ctx / x), App. A.1 Eq. app_total_budget */
+    double rope_base;              /* RoPE base of the keys (0: keys carry no RoPE) */
+    int32_t n_min, n_max, n0;      /* slot length bounds and target (App. B.3) */
+    double lambda_stab, lambda_s, lambda_d, lambda_n, c_cut;
+    int32_t seg_layers[8];         /* explicit segmentation layers, or n_seg_layers = 0 */
+    int32_t n_seg_layers;          /*   for the relative-depth rule of App. B.2 */
+    int32_t windows[4];            /* curvature window scales (App. B.2) */
+    int32_t n_windows;
+    int32_t k_cand;                /* top-K curvature split candidates (App. B.4) */
+    double lambda_kappa, lambda_Z, lambda_M, eps, base_frac;
+    double lambda_graph;           /* multi-hop weight: only 0 is built (GKV_EUNSUPPORTED) */
+    double alpha_floor;            /* singleton-floor cap: only 0 is built (GKV_EUNSUPPORTED) */
+} gkv_params;
+
+/* Fill *p with the paper's defaults; shapes and budget are left zero.  Host only. */
+gkv_status gracekv_default_params(gkv_params *p);
+
+/* B_total = floor(L * G * n_ctx / x) for compression ratio x >= 1
+ * (App. A.1 Eq. app_total_budget).  Returns -1 for invalid arguments.  Host only. */
+int64_t gracekv_budget_for_ratio(int32_t L, int32_t G, int32_t n_ctx, double x);
+
+/* Validate *p, resolve the recent window against the budget (r = 32, shrunk to
+ * floor(B_total / (L G)) when L G r > B_total, never below 4: App. A.1) and
+ * allocate the device workspace on the current device.  On success *out owns
+ * it; release with gracekv_destroy.  Errors: GKV_EINVAL, GKV_EBUDGET,
+ * GKV_EUNSUPPORTED (lambda_graph != 0, alpha_floor != 0, d not in {64, 128},
+ * W > 64, ...), GKV_ENOMEM, GKV_ECUDA. */
+gkv_status gracekv_create(const gkv_params *p, gracekv_ctx **out);
+void gracekv_destroy(gracekv_ctx *ctx);
+const char *gracekv_last_error(const gracekv_ctx *ctx);
+const char *gracekv_status_string(gkv_status s);
+
+/* Resolved quantities: effective recent window r, compressible length
+ * N_c = c_e - r - c_s, free budget B_free = B_total - L G r (App. A.1
+ * Eq. app_free_budget), and the number of slots of the last segmentation. */
+gkv_status gracekv_query(const gracekv_ctx *ctx, int32_t *recent, int32_t *n_c,
+                         int64_t *b_free, int32_t *n_slots);
+
+/*
+ * Stage 1 -- curvature-guided segmentation (App. B.2-B.3).
+ * Trajectory h^(l)_t = concat_g V[l][g][t][:] at the segmentation layers
+ * (or `hidden` [n_seg][T][Dh] fp32 when given), multi-scale curvature
+ * (Eq. app_local_curvature), stabilised curvature (Eq.
+ * app_stabilized_curvature), robust-z boundary score (Eq. app_boundary_score,
+ * surprisal [T] fp32 optional, 0 when NULL), and the length-constrained DP
+ * (Eq. app_dp_recurrence with the terminal relaxation of Eq.
+ * app_terminal_predecessor) over the compressible region [c_s, c_e - r).
+ * Outputs: slot_starts (device, [cap + 1] int32, absolute positions,
+ * slot_starts[J] = c_e - r), *n_slots_host = J (synchronises `stream`),
+ * kappa (device, nullable, [T] fp32 stabilised curvature).
+ * Errors: GKV_EINVAL, GKV_ECAPACITY (J > cap), GKV_ENONFINITE, GKV_ECUDA.
+ */
+gkv_status gracekv_segment(gracekv_ctx *ctx, const void *V, const float *hidden, int32_t Dh,
+                           const float *surprisal, int32_t *slot_starts, int32_t cap,
+                           int32_t *n_slots_host, float *kappa, void *stream);
+
+/*
+ * Stage 2 -- prototype trees (App. A.3), token and node values (App. A.4),
+ * gains (App. A.5 Eq. app_operation_gains).  Requires a prior
+ * gracekv_segment (its curvature drives the split candidates).  If
+ * slot_starts (device, [n_slots + 1] int32 absolute) is non-NULL it replaces
+ * the segmentation's slots (externally supplied partition of [c_s, c_e - r));
+ * omega (device [L][G] fp32, nullable = all ones) is the head sensitivity.
+ * Row statistics (max logit, partition over [0, T), partition over the
+ * compressible region) are computed for every probe row (l, h, u); the trees
+ * stay in the context's workspace.  Errors: GKV_EINVAL, GKV_ESTATE,
+ * GKV_EUNSUPPORTED (a slot longer than 128 tokens), GKV_ECUDA.
+ */
+gkv_status gracekv_build_trees(gracekv_ctx *ctx, const void *K, const void *V, const void *Q,
+                               const float *omega, const int32_t *slot_starts, int32_t n_slots,
+                               void *stream);
+
+/*
+ * Stage 3 -- global greedy allocation (App. A.5 Stage II, App. C.3): the
+ * result equals a max-priority queue keyed by U = Delta / c with order
+ * (U desc, unit (l, g, j) asc, node (a asc, b desc)), seeded with every Add,
+ * discarding unaffordable pops, under B_free.  *n_entries_host receives the
+ * number of cache entries E = L G (T - N_c) + used (synchronises `stream`).
+ * Errors: GKV_ESTATE, GKV_ENONFINITE, GKV_ECUDA.
+ */
+gkv_status gracekv_allocate(gracekv_ctx *ctx, int64_t *n_entries_host, void *stream);
+
+/*
+ * Stage 4 -- packing (App. A.5 "Frontier updates and physical packing").
+ * Per (l, g), in this order: prefix tokens [0, c_s), the frontier nodes of
+ * every covered slot in ascending position, the recent window and the
+ * suffix [c_e - r, T).  Non-singleton nodes store (ktil, vtil, p, log m_eff)
+ * (Eqs. app_rope_prototype, app_value_prototype,
+ * app_effective_multiplicity); single tokens store their original K/V bits,
+ * position and log m = 0.  Outputs (device): K_out, V_out [cap][d] dtype,
+ * pos [cap] int32, log_m [cap] fp32, src_lo / src_hi [cap] int32 (the token
+ * interval each entry covers), offsets [L G + 1] int64 (entry range of each
+ * (l, g)).  cap must be >= the count returned by gracekv_allocate.
+ * Errors: GKV_ESTATE, GKV_ECAPACITY, GKV_ECUDA.
+ */
+gkv_status gracekv_gather(gracekv_ctx *ctx, const void *K, const void *V, void *K_out,
+                          void *V_out, int32_t *pos, float *log_m, int32_t *src_lo,
+                          int32_t *src_hi, int64_t *offsets, int64_t cap, void *stream);
+
+/*
+ * Introspection for tests and tools (not needed to compress).  Copies the
+ * current trees and selection to caller-owned HOST arrays (synchronises
+ * `stream`).  Node records of all units are packed unit after unit, unit
+ * order (l, g, j); within a unit in creation (breadth-first) order.
+ *   unit_first [L G J + 1] int64: node range of each unit
+ *   unit_Uadd, unit_Ddrop [L G J] fp32; add_sel [L G J] uint8
+ *   per node (capacity node_cap): a, b, child0 (index within the unit, -1 for
+ *   leaves), nchild, cost int32; D, R, U, kappa fp32; split_sel uint8
+ *   row stats (nullable) [L][Hq][W] fp32: max logit, Z over [0,T), Z over C
+ *   rtok (nullable) [L][G][N_c] fp32 token values
+ * *n_nodes_host receives the node count (GKV_ECAPACITY if > node_cap).
+ */
+gkv_status gracekv_export(gracekv_ctx *ctx, int64_t node_cap, int64_t *n_nodes_host,
+                          int64_t *unit_first, float *unit_Uadd, float *unit_Ddrop,
+                          uint8_t *add_sel, int32_t *a, int32_t *b, int32_t *child0,
+                          int32_t *nchild, int32_t *cost, float *D, float *R, float *U,
+                          float *kappa, uint8_t *split_sel, float *row_m, float *row_Z,
+                          float *row_ZC, float *rtok, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

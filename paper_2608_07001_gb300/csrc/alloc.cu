@@ -1,0 +1,348 @@
+// alloc.cu -- stage 3 of the GraceKV pass: global greedy Add/Split allocation
+// (App. A.5 Stage II, App. C.3), computed on the device without a priority
+// queue.
+//
+// The heap of the paper pops ops in non-increasing order of their bottleneck
+// key kappa(op) = min(U(op), kappa(op that exposed it)) (kappa(Add) = U(Add)):
+// an op is exposed only after its creator, and a child whose U exceeds its
+// creator's key is popped right after it.  Hence, with tau the cost-weighted
+// threshold cost{kappa > tau} <= B_free < cost{kappa >= tau}:
+//   1. every op with kappa > tau is executed (they fit and are
+//      prerequisite-closed, since kappa never increases down a path);
+//   2. ops with kappa == tau are executed in the heap's order, which visits
+//      units in ascending order and, inside a unit, follows the unit's own
+//      queue (U desc, a asc, b desc); an op that does not fit the remaining
+//      budget is discarded with its subtree (App. C.3);
+//   3. if one budget unit is left, the best exposed cost-1 op under the heap's
+//      order (U desc, unit asc, a asc, b desc) takes it.
+// Ties in U are therefore resolved exactly as the heap resolves them.
+//
+// Kernels: alloc_hist (cost-weighted histogram of the 32-bit keys, three
+// passes of 11/11/10 bits), alloc_scan (pick the digit, one block), alloc_mark
+// (main set + units holding ties), alloc_ties (one block, units in order),
+// alloc_end_max / alloc_end_key / alloc_end_pick (endgame).
+#include "gkv_internal.cuh"
+
+#include <algorithm>
+
+namespace gkv {
+namespace {
+
+// alloc_state layout (unsigned long long)
+enum { ST_PREFIX = 0, ST_ABOVE, ST_ALL, ST_R, ST_ENDU, ST_ENDKEY, ST_TOTAL, ST_USED, ST_N };
+
+struct AllocArgs {
+    int64_t n_units, n_nodes;
+    const float *u_U;        // Add keys (kappa = U)
+    const float *nd_kappa;
+    const int8_t *nd_cost;
+    const float *nd_U;
+    const int32_t *nd_a, *nd_b, *nd_parent, *nd_unit, *nd_child0;
+    const int8_t *nd_nchild;
+    const int32_t *u_nnodes;
+    const int32_t *slots;
+    int J, LG, cs, Nc;
+    uint8_t *u_sel, *nd_sel;
+    int32_t *u_flag;
+    unsigned long long *hist, *st;
+    int64_t B_free;
+    int *status;
+};
+
+__device__ __forceinline__ bool op_key(const AllocArgs &A, int64_t i, uint32_t &key, int &cost) {
+    if (i < A.n_units) {
+        float x = A.u_U[i];
+        key = __float_as_uint(x);
+        cost = 1;
+        if (!(x >= 0.f) || isinf(x)) atomicOr(A.status, 8);
+        return true;
+    }
+    int64_t v = i - A.n_units;
+    int c = A.nd_cost[v];
+    if (c <= 0) return false;
+    float x = A.nd_kappa[v];
+    if (!(x >= 0.f) || isinf(x)) atomicOr(A.status, 8);
+    key = __float_as_uint(x);
+    cost = c;
+    return true;
+}
+
+__global__ void alloc_hist_kernel(AllocArgs A, int shift, int nbits, uint32_t mask) {
+    __shared__ unsigned int sh[2048];
+    const int nbin = 1 << nbits;
+    for (int b = threadIdx.x; b < nbin; b += blockDim.x) sh[b] = 0;
+    __syncthreads();
+    const uint32_t prefix = (uint32_t)A.st[ST_PREFIX];
+    const int64_t n = A.n_units + A.n_nodes;
+    unsigned long long tot = 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        uint32_t key;
+        int cost;
+        if (!op_key(A, i, key, cost)) continue;
+        tot += cost;
+        if ((key & mask) != prefix) continue;
+        atomicAdd(&sh[(key >> shift) & (nbin - 1)], (unsigned)cost);
+    }
+    __syncthreads();
+    for (int b = threadIdx.x; b < nbin; b += blockDim.x)
+        if (sh[b]) atomicAdd(&A.hist[b], (unsigned long long)sh[b]);
+    if (shift == 21) {   // first pass: total cost of all ops
+        tot = (unsigned long long)warp_sum((double)tot);
+        if ((threadIdx.x & 31) == 0 && tot) atomicAdd(&A.st[ST_TOTAL], tot);
+    }
+}
+
+__global__ void alloc_scan_kernel(AllocArgs A, int shift, int nbits) {
+    if (threadIdx.x != 0) return;
+    const int nbin = 1 << nbits;
+    unsigned long long above = A.st[ST_ABOVE];
+    const unsigned long long B = (unsigned long long)A.B_free;
+    if (shift == 21 && A.st[ST_TOTAL] <= B) {
+        A.st[ST_ALL] = 1;
+    }
+    if (A.st[ST_ALL]) {
+        for (int b = 0; b < nbin; b++) A.hist[b] = 0;
+        return;
+    }
+    int pick = 0;
+    for (int b = nbin - 1; b >= 0; b--) {
+        unsigned long long h = A.hist[b];
+        if (above + h > B) { pick = b; break; }
+        above += h;
+    }
+    A.st[ST_PREFIX] |= ((unsigned long long)pick << shift);
+    A.st[ST_ABOVE] = above;
+    for (int b = 0; b < nbin; b++) A.hist[b] = 0;
+}
+
+// Main set (kappa > tau, or everything when it fits) and units holding ties.
+__global__ void alloc_mark_kernel(AllocArgs A) {
+    const bool all = A.st[ST_ALL] != 0;
+    const uint32_t tau = (uint32_t)A.st[ST_PREFIX];
+    const int64_t n = A.n_units + A.n_nodes;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        uint32_t key;
+        int cost;
+        if (!op_key(A, i, key, cost)) continue;
+        uint8_t s = (all || key > tau) ? 1 : 0;
+        if (i < A.n_units) {
+            A.u_sel[i] = s;
+            if (!all && key == tau) A.u_flag[i] = 1;
+        } else {
+            int64_t v = i - A.n_units;
+            A.nd_sel[v] = s;
+            if (!all && key == tau) A.u_flag[A.nd_unit[v]] = 1;
+        }
+    }
+}
+
+// Node index base of unit uid.
+__device__ __forceinline__ int64_t unit_base(const AllocArgs &A, int64_t uid) {
+    int lg = (int)(uid / A.J), j = (int)(uid - (int64_t)lg * A.J);
+    return node_base(lg, A.slots[j], A.cs, A.Nc);
+}
+
+// One block: walk the units in ascending order; thread 0 replays every unit
+// that holds tie ops with the unit's own queue.
+__global__ void __launch_bounds__(1024) alloc_ties_kernel(AllocArgs A) {
+    __shared__ int list[1024];
+    __shared__ int nlist;
+    __shared__ long long Rs;
+    __shared__ short parent[2 * kMaxUnit];
+    if (threadIdx.x == 0) {
+        const bool all = A.st[ST_ALL] != 0;
+        long long above = (long long)A.st[ST_ABOVE];
+        Rs = all ? (long long)A.B_free - (long long)A.st[ST_TOTAL] : (long long)A.B_free - above;
+    }
+    __syncthreads();
+    if (A.st[ST_ALL]) {
+        if (threadIdx.x == 0) A.st[ST_R] = 0, A.st[ST_USED] = A.st[ST_TOTAL];
+        return;
+    }
+    const uint32_t tau = (uint32_t)A.st[ST_PREFIX];
+    for (int64_t base = 0; base < A.n_units && Rs > 0; base += 1024) {
+        // ordered compaction of flagged units in [base, base + 1024)
+        int64_t uid = base + threadIdx.x;
+        bool f = uid < A.n_units && A.u_flag[uid];
+        if (threadIdx.x == 0) nlist = 0;
+        __syncthreads();
+        unsigned bal = __ballot_sync(0xffffffffu, f);
+        __shared__ int wcnt[32];
+        if ((threadIdx.x & 31) == 0) wcnt[threadIdx.x >> 5] = __popc(bal);
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            int acc = 0;
+            for (int w = 0; w < 32; w++) { int c = wcnt[w]; wcnt[w] = acc; acc += c; }
+            nlist = acc;
+        }
+        __syncthreads();
+        if (f) list[wcnt[threadIdx.x >> 5] + __popc(bal & ((1u << (threadIdx.x & 31)) - 1))] = (int)(uid - base);
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            for (int q = 0; q < nlist && Rs > 0; q++) {
+                int64_t u = base + list[q];
+                int64_t nb = unit_base(A, u);
+                int nn = A.u_nnodes[u];
+                for (int k = 0; k < nn; k++) parent[k] = -1;
+                for (int k = 0; k < nn; k++) {
+                    int c0 = A.nd_child0[nb + k], nc = A.nd_nchild[nb + k];
+                    for (int x = 0; x < nc; x++) parent[c0 + x] = (short)k;
+                }
+                // the unit's queue restricted to tie ops; -1 stands for the Add
+                for (;;) {
+                    int best = -2;
+                    float bu = 0.f;
+                    int ba = 0, bb = 0;
+                    // Add
+                    if (A.u_sel[u] == 0 && __float_as_uint(A.u_U[u]) == tau) {
+                        best = -1; bu = A.u_U[u]; ba = A.nd_a[nb]; bb = A.nd_b[nb];
+                    }
+                    for (int k = 0; k < nn; k++) {
+                        int64_t v = nb + k;
+                        if (A.nd_cost[v] <= 0 || A.nd_sel[v] != 0) continue;
+                        if (__float_as_uint(A.nd_kappa[v]) != tau) continue;
+                        bool exposed = parent[k] < 0 ? A.u_sel[u] == 1 : A.nd_sel[nb + parent[k]] == 1;
+                        if (!exposed) continue;
+                        float uu = A.nd_U[v];
+                        int aa = A.nd_a[v], bbb = A.nd_b[v];
+                        bool better = best == -2 || uu > bu || (uu == bu && (aa < ba || (aa == ba && bbb > bb)));
+                        if (better) { best = k; bu = uu; ba = aa; bb = bbb; }
+                    }
+                    if (best == -2 || Rs <= 0) break;
+                    int cost = best == -1 ? 1 : A.nd_cost[nb + best];
+                    uint8_t s = cost > Rs ? 2 : 1;     // 2 = discarded (subtree never exposed)
+                    if (s == 1) Rs -= cost;
+                    if (best == -1) A.u_sel[u] = s;
+                    else A.nd_sel[nb + best] = s;
+                }
+            }
+        }
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) A.st[ST_R] = (unsigned long long)Rs;
+}
+
+// Endgame: when exactly one budget unit is left, the best exposed cost-1 op.
+__device__ __forceinline__ bool end_cand(const AllocArgs &A, int64_t i, float &U,
+                                         unsigned long long &key) {
+    if (i < A.n_units) {
+        if (A.u_sel[i] != 0) return false;
+        int64_t nb = unit_base(A, i);
+        U = A.u_U[i];
+        int a = A.nd_a[nb], b = A.nd_b[nb];
+        key = ((unsigned long long)i << 37) | ((unsigned long long)a << 17) | (0x1FFFFull - (unsigned)(b - a));
+        return true;
+    }
+    int64_t v = i - A.n_units;
+    if (A.nd_cost[v] != 1 || A.nd_sel[v] != 0) return false;
+    int32_t p = A.nd_parent[v];
+    bool exposed = p < 0 ? A.u_sel[-2 - p] == 1 : A.nd_sel[p] == 1;
+    if (!exposed) return false;
+    U = A.nd_U[v];
+    int a = A.nd_a[v], b = A.nd_b[v];
+    key = ((unsigned long long)A.nd_unit[v] << 37) | ((unsigned long long)a << 17) |
+          (0x1FFFFull - (unsigned)(b - a));
+    return true;
+}
+
+__global__ void alloc_end_max_kernel(AllocArgs A) {
+    if (A.st[ST_R] != 1) return;
+    const int64_t n = A.n_units + A.n_nodes;
+    unsigned best = 0;
+    bool any = false;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        float U;
+        unsigned long long k;
+        if (!end_cand(A, i, U, k)) continue;
+        unsigned b = __float_as_uint(U) + 1u;     // +1: distinguish "no candidate" (0)
+        if (!any || b > best) best = b;
+        any = true;
+    }
+    if (any) atomicMax(reinterpret_cast<unsigned long long *>(&A.st[ST_ENDU]), (unsigned long long)best);
+}
+
+__global__ void alloc_end_key_kernel(AllocArgs A) {
+    if (A.st[ST_R] != 1 || A.st[ST_ENDU] == 0) return;
+    const unsigned target = (unsigned)A.st[ST_ENDU] - 1u;
+    const int64_t n = A.n_units + A.n_nodes;
+    unsigned long long best = ~0ull;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        float U;
+        unsigned long long k;
+        if (!end_cand(A, i, U, k)) continue;
+        if (__float_as_uint(U) != target) continue;
+        if (k < best) best = k;
+    }
+    if (best != ~0ull) atomicMin(&A.st[ST_ENDKEY], best);
+}
+
+__global__ void alloc_end_pick_kernel(AllocArgs A) {
+    const int64_t n = A.n_units + A.n_nodes;
+    const bool go = A.st[ST_R] == 1 && A.st[ST_ENDU] != 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        if (!go) break;
+        float U;
+        unsigned long long k;
+        if (!end_cand(A, i, U, k)) continue;
+        if (k != A.st[ST_ENDKEY] || __float_as_uint(U) + 1u != (unsigned)A.st[ST_ENDU]) continue;
+        if (i < A.n_units) A.u_sel[i] = 1;
+        else A.nd_sel[i - A.n_units] = 1;
+    }
+}
+
+__global__ void alloc_final_kernel(AllocArgs A) {
+    if (threadIdx.x) return;
+    long long R = (long long)A.st[ST_R];
+    if (!A.st[ST_ALL] && R == 1 && A.st[ST_ENDU] != 0) R = 0;
+    A.st[ST_R] = (unsigned long long)R;
+    if (!A.st[ST_ALL]) A.st[ST_USED] = (unsigned long long)(A.B_free - R);
+}
+
+__global__ void alloc_init_kernel(unsigned long long *st, unsigned long long *hist) {
+    int i = threadIdx.x;
+    if (i < ST_N) st[i] = (i == ST_ENDKEY) ? ~0ull : 0ull;
+    for (int b = i; b < 2048; b += blockDim.x) hist[b] = 0;
+}
+
+}  // namespace
+
+cudaError_t launch_allocate(Ctx &c, int J, cudaStream_t s) {
+    Workspace &w = c.w;
+    AllocArgs A;
+    A.n_units = (int64_t)c.p.L * c.p.G * J;
+    A.n_nodes = c.node_cap;
+    A.u_U = w.u_Uadd; A.nd_kappa = w.nd_kappa; A.nd_cost = w.nd_cost; A.nd_U = w.nd_U;
+    A.nd_a = w.nd_a; A.nd_b = w.nd_b; A.nd_parent = w.nd_parent; A.nd_unit = w.nd_unit;
+    A.nd_child0 = w.nd_child0; A.nd_nchild = w.nd_nchild; A.u_nnodes = w.u_nnodes;
+    A.slots = w.slots;
+    A.J = J; A.LG = c.p.L * c.p.G; A.cs = c.p.ctx_start; A.Nc = c.Nc;
+    A.u_sel = w.u_sel; A.nd_sel = w.nd_sel; A.u_flag = w.u_count;
+    A.hist = w.hist; A.st = w.alloc_state; A.B_free = c.B_free; A.status = w.dev_int + 1;
+    cudaMemsetAsync(w.u_count, 0, sizeof(int32_t) * A.n_units, s);
+    alloc_init_kernel<<<1, 256, 0, s>>>(w.alloc_state, w.hist);
+    const int64_t n = A.n_units + A.n_nodes;
+    int blocks = (int)std::min<int64_t>((n + 255) / 256, (int64_t)c.num_sms * 8);
+    if (blocks < 1) blocks = 1;
+    const int shifts[3] = {21, 10, 0};
+    const int bits[3] = {11, 11, 10};
+    uint32_t mask = 0;
+    for (int ps = 0; ps < 3; ps++) {
+        alloc_hist_kernel<<<blocks, 256, 0, s>>>(A, shifts[ps], bits[ps], mask);
+        alloc_scan_kernel<<<1, 32, 0, s>>>(A, shifts[ps], bits[ps]);
+        mask |= ((1u << bits[ps]) - 1u) << shifts[ps];
+    }
+    alloc_mark_kernel<<<blocks, 256, 0, s>>>(A);
+    alloc_ties_kernel<<<1, 1024, 0, s>>>(A);
+    alloc_end_max_kernel<<<blocks, 256, 0, s>>>(A);
+    alloc_end_key_kernel<<<blocks, 256, 0, s>>>(A);
+    alloc_end_pick_kernel<<<blocks, 256, 0, s>>>(A);
+    alloc_final_kernel<<<1, 32, 0, s>>>(A);
+    return cudaGetLastError();
+}
+
+}  // namespace gkv

@@ -1,0 +1,426 @@
+// api.cu -- the C ABI of include/gracekv.h: parameter validation, budget
+// resolution (App. A.1), workspace ownership and the stage state machine.
+#include "gkv_internal.cuh"
+
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <vector>
+
+using gkv::Ctx;
+
+struct gracekv_ctx {
+    Ctx c;
+    std::vector<void *> allocs;
+};
+
+namespace {
+
+// Device status bits (dev_int[1]).
+enum : int { ST_NONFINITE_KAPPA = 1, ST_NONFINITE_ROWS = 2, ST_LONG_SLOT = 4, ST_NONFINITE_GAIN = 8,
+             ST_BAD_SLOTS = 16 };
+
+gkv_status fail(gracekv_ctx *x, gkv_status s, const char *msg) {
+    if (x) {
+        if (x->c.err.empty()) x->c.err = msg;
+        if (s == GKV_ECUDA) x->c.sticky = GKV_ECUDA;
+    }
+    return s;
+}
+
+gkv_status cuda_fail(gracekv_ctx *x, cudaError_t e, const char *where) {
+    char buf[256];
+    snprintf(buf, sizeof buf, "%s: %s", where, cudaGetErrorString(e));
+    if (x && x->c.err.empty()) x->c.err = buf;
+    if (x) x->c.sticky = GKV_ECUDA;
+    return GKV_ECUDA;
+}
+
+template <typename T>
+bool dalloc(gracekv_ctx *x, T **p, size_t n) {
+    void *q = nullptr;
+    if (n == 0) n = 1;
+    if (cudaMalloc(&q, n * sizeof(T)) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    x->allocs.push_back(q);
+    *p = static_cast<T *>(q);
+    return true;
+}
+
+gkv_status check_status(gracekv_ctx *x, int st) {
+    if (st & ST_BAD_SLOTS) return fail(x, GKV_EINVAL, "supplied slot starts are not a partition of [c_s, c_e - r) into slots of 1..128 tokens");
+    if (st & ST_LONG_SLOT) return fail(x, GKV_EUNSUPPORTED, "a slot is longer than 128 tokens (unit kernel limit)");
+    if (st & ST_NONFINITE_KAPPA) return fail(x, GKV_ENONFINITE, "non-finite curvature (NaN/Inf in the trajectory)");
+    if (st & ST_NONFINITE_ROWS) return fail(x, GKV_ENONFINITE, "non-finite attention row statistics (NaN/Inf in K or Q)");
+    if (st & ST_NONFINITE_GAIN) return fail(x, GKV_ENONFINITE, "non-finite gain (NaN/Inf in K, V, Q or omega)");
+    return GKV_OK;
+}
+
+gkv_status ready(gracekv_ctx *x, int need_stage) {
+    if (!x) return GKV_EINVAL;
+    if (x->c.sticky != GKV_OK) return GKV_ESTATE;
+    if (x->c.stage < need_stage) return fail(x, GKV_ESTATE, "call out of order");
+    return GKV_OK;
+}
+
+__global__ void validate_slots_kernel(const int32_t *s, int J, int cs, int cend, int *status) {
+    int j = blockIdx.x * blockDim.x + threadIdx.x;
+    if (j >= J) return;
+    int a = s[j], b = s[j + 1];
+    bool bad = b - a < 1 || (j == 0 && a != cs) || (j == J - 1 && b != cend);
+    if (bad) atomicOr(status, ST_BAD_SLOTS);
+    else if (b - a > gkv::kMaxUnit) atomicOr(status, ST_LONG_SLOT);
+}
+
+}  // namespace
+
+extern "C" {
+
+gkv_status gracekv_default_params(gkv_params *p) {
+    if (!p) return GKV_EINVAL;
+    memset(p, 0, sizeof *p);
+    p->dtype = GKV_BF16;
+    p->recent = 32;                                    // App. A.1
+    p->n_min = 16; p->n_max = 128; p->n0 = 64;         // App. B.3
+    p->lambda_stab = 0.25; p->lambda_s = 0.15;         // App. B.2
+    p->lambda_d = 0.25; p->lambda_n = 0.10; p->c_cut = 1.0;
+    p->n_seg_layers = 0;                               // depths 0.33 / 0.50 / 0.67
+    p->windows[0] = 4; p->windows[1] = 8; p->windows[2] = 16; p->n_windows = 3;
+    p->k_cand = 16; p->lambda_kappa = 0.05;            // App. A.3, B.4
+    p->lambda_Z = 0.25; p->lambda_M = 0.75;
+    p->eps = 1e-6; p->base_frac = 0.1;
+    p->lambda_graph = 0.0; p->alpha_floor = 0.0;
+    p->ctx_start = 0; p->ctx_end = -1;                 // -1: T
+    return GKV_OK;
+}
+
+int64_t gracekv_budget_for_ratio(int32_t L, int32_t G, int32_t n_ctx, double x) {
+    if (L <= 0 || G <= 0 || n_ctx <= 0 || !(x >= 1.0)) return -1;
+    double n = (double)L * G * n_ctx;
+    if (x == std::floor(x) && x < 9.0e15) return (int64_t)L * G * n_ctx / (int64_t)x;
+    return (int64_t)std::floor(n / x);
+}
+
+const char *gracekv_status_string(gkv_status s) {
+    switch (s) {
+        case GKV_OK: return "ok";
+        case GKV_EINVAL: return "invalid argument";
+        case GKV_EBUDGET: return "budget too small";
+        case GKV_ENOMEM: return "out of device memory";
+        case GKV_ECUDA: return "CUDA error";
+        case GKV_ETIMEOUT: return "device wait timed out";
+        case GKV_ENONFINITE: return "non-finite value";
+        case GKV_ESTATE: return "call out of order or context failed";
+        case GKV_EUNSUPPORTED: return "unsupported configuration";
+        case GKV_ECAPACITY: return "output capacity too small";
+    }
+    return "unknown status";
+}
+
+const char *gracekv_last_error(const gracekv_ctx *x) {
+    if (!x) return "null context";
+    return x->c.err.c_str();
+}
+
+void gracekv_destroy(gracekv_ctx *x) {
+    if (!x) return;
+    for (void *p : x->allocs) cudaFree(p);
+    delete x;
+}
+
+gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
+    if (!pin || !out) return GKV_EINVAL;
+    *out = nullptr;
+    gkv_params p = *pin;
+    if (p.ctx_end < 0) p.ctx_end = p.T;
+    if (p.L <= 0 || p.G <= 0 || p.Hq <= 0 || p.T <= 0 || p.d <= 0 || p.W <= 0 || p.Hq % p.G)
+        return GKV_EINVAL;
+    if (p.dtype != GKV_F32 && p.dtype != GKV_BF16) return GKV_EINVAL;
+    if (p.ctx_start < 0 || p.ctx_end > p.T || p.ctx_start >= p.ctx_end) return GKV_EINVAL;
+    if (p.n_min < 1 || p.n_max < p.n_min || p.n0 < 1) return GKV_EINVAL;
+    if (p.n_windows < 1 || p.n_windows > gkv::kMaxWindows) return GKV_EINVAL;
+    for (int i = 0; i < p.n_windows; i++)
+        if (p.windows[i] < 1 || p.windows[i] > 16) return GKV_EINVAL;
+    if (p.n_seg_layers < 0 || p.n_seg_layers > gkv::kMaxSegLayers) return GKV_EINVAL;
+    for (int i = 0; i < p.n_seg_layers; i++)
+        if (p.seg_layers[i] < 0 || p.seg_layers[i] >= p.L) return GKV_EINVAL;
+    if (p.k_cand < 1 || p.k_cand > 16) return GKV_EINVAL;
+    if (!(p.eps > 0) || !(p.base_frac >= 0)) return GKV_EINVAL;
+    if (p.lambda_graph != 0.0 || p.alpha_floor != 0.0) return GKV_EUNSUPPORTED;
+    if ((p.d != 64 && p.d != 128) || p.W > 64 || p.n_max > gkv::kMaxUnit ||
+        (int64_t)p.G * p.d > 2048)
+        return GKV_EUNSUPPORTED;
+    // recent window (App. A.1): r = 32, shrunk to floor(B / (L G)) when it does
+    // not fit, never below 4; the compressible region must stay non-empty.
+    int64_t LG = (int64_t)p.L * p.G;
+    int64_t r = p.recent;
+    if (r < 0) return GKV_EINVAL;
+    if (LG * r > p.budget) {
+        r = p.budget / LG;
+        if (r < 4) return GKV_EBUDGET;
+    }
+    int64_t Nc = (int64_t)p.ctx_end - r - p.ctx_start;
+    if (Nc < 1) return GKV_EBUDGET;
+    if (Nc + 1 + 4096 > 227 * 1024) return GKV_EUNSUPPORTED;   // DP keeps lengths in shared memory
+
+    gracekv_ctx *x = new (std::nothrow) gracekv_ctx();
+    if (!x) return GKV_ENOMEM;
+    Ctx &c = x->c;
+    c.p = p;
+    c.r = (int32_t)r;
+    c.Nc = (int32_t)Nc;
+    c.c_end = p.ctx_end - c.r;
+    c.B_free = p.budget - LG * r;
+    c.nwin = p.n_windows;
+    if (p.n_seg_layers > 0) {
+        c.nseg = p.n_seg_layers;
+        for (int i = 0; i < c.nseg; i++) c.seg_layers[i] = p.seg_layers[i];
+    } else {   // App. B.2 Eq. app_seg_layers
+        const double rho[3] = {0.33, 0.50, 0.67};
+        c.nseg = 0;
+        for (double q : rho) {
+            int l = (int)std::floor(q * p.L);
+            if (l > p.L - 1) l = p.L - 1;
+            bool dup = false;
+            for (int i = 0; i < c.nseg; i++) dup |= c.seg_layers[i] == l;
+            if (!dup) c.seg_layers[c.nseg++] = l;
+        }
+    }
+    if (cudaGetDevice(&c.device) != cudaSuccess) {
+        delete x;
+        return GKV_ECUDA;
+    }
+    cudaDeviceGetAttribute(&c.num_sms, cudaDevAttrMultiProcessorCount, c.device);
+    const int Rg = (p.Hq / p.G) * p.W;
+    const int64_t base = LG * ((Rg + 63) / 64);
+    c.n_chunks = (int)std::max<int64_t>(1, std::min<int64_t>((4 * c.num_sms + base - 1) / base,
+                                                             std::max(1, p.T / 256)));
+    c.node_cap = LG * 2 * Nc;
+    const int nb = p.n_max - p.n_min + 1;
+    const int64_t nrow = (int64_t)p.L * p.Hq * p.W;
+    gkv::Workspace &w = c.w;
+    bool ok = dalloc(x, &w.rope, (size_t)p.T * (p.d / 2)) &&
+              dalloc(x, &w.inv_norm, (size_t)c.nseg * p.T) &&
+              dalloc(x, &w.nrm2, (size_t)c.nseg * p.T) &&
+              dalloc(x, &w.klw, (size_t)c.nseg * c.nwin * p.T) &&
+              dalloc(x, &w.kappa, (size_t)p.T) && dalloc(x, &w.bscore, (size_t)p.T) &&
+              dalloc(x, &w.zbuf, (size_t)p.T) && dalloc(x, &w.p2, (size_t)Nc + 1) &&
+              dalloc(x, &w.ew, (size_t)(Nc + 1) * nb) && dalloc(x, &w.ewt, (size_t)p.n_max + 1) &&
+              dalloc(x, &w.dpF, (size_t)Nc + 1) && dalloc(x, &w.slots, (size_t)Nc + 2) &&
+              dalloc(x, &w.dev_int, 16) &&
+              dalloc(x, &w.row_m, (size_t)nrow) && dalloc(x, &w.row_Z, (size_t)nrow) &&
+              dalloc(x, &w.row_ZC, (size_t)nrow) && dalloc(x, &w.rowp, (size_t)3 * nrow * c.n_chunks) &&
+              dalloc(x, &w.rtok, (size_t)LG * Nc) &&
+              dalloc(x, &w.nd_a, (size_t)c.node_cap) && dalloc(x, &w.nd_b, (size_t)c.node_cap) &&
+              dalloc(x, &w.nd_child0, (size_t)c.node_cap) && dalloc(x, &w.nd_parent, (size_t)c.node_cap) &&
+              dalloc(x, &w.nd_unit, (size_t)c.node_cap) && dalloc(x, &w.nd_nchild, (size_t)c.node_cap) &&
+              dalloc(x, &w.nd_cost, (size_t)c.node_cap) && dalloc(x, &w.nd_D, (size_t)c.node_cap) &&
+              dalloc(x, &w.nd_R, (size_t)c.node_cap) && dalloc(x, &w.nd_U, (size_t)c.node_cap) &&
+              dalloc(x, &w.nd_kappa, (size_t)c.node_cap) && dalloc(x, &w.nd_sel, (size_t)c.node_cap) &&
+              dalloc(x, &w.hist, 2048) && dalloc(x, &w.alloc_state, 16);
+    if (!ok) {
+        gracekv_destroy(x);
+        return GKV_ENOMEM;
+    }
+    cudaError_t e = cudaMemset(w.nd_cost, 0, (size_t)c.node_cap);
+    if (e == cudaSuccess) e = cudaMemset(w.dev_int, 0, 16 * sizeof(int));
+    if (e == cudaSuccess) e = gkv::launch_rope_table(c, 0);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) {
+        gracekv_destroy(x);
+        return GKV_ECUDA;
+    }
+    *out = x;
+    return GKV_OK;
+}
+
+gkv_status gracekv_query(const gracekv_ctx *x, int32_t *recent, int32_t *n_c, int64_t *b_free,
+                         int32_t *n_slots) {
+    if (!x) return GKV_EINVAL;
+    if (recent) *recent = x->c.r;
+    if (n_c) *n_c = x->c.Nc;
+    if (b_free) *b_free = x->c.B_free;
+    if (n_slots) *n_slots = x->c.J;
+    return GKV_OK;
+}
+
+gkv_status gracekv_segment(gracekv_ctx *x, const void *V, const float *hidden, int32_t Dh,
+                           const float *surprisal, int32_t *slot_starts, int32_t cap,
+                           int32_t *n_slots_host, float *kappa, void *stream) {
+    gkv_status st = ready(x, 0);
+    if (st) return st;
+    Ctx &c = x->c;
+    if (!V || !slot_starts || !n_slots_host || cap < 1) return fail(x, GKV_EINVAL, "segment: null argument");
+    if (hidden && (Dh <= 0 || Dh > 2048)) return fail(x, GKV_EINVAL, "segment: hidden dim must be in [1, 2048]");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaMemsetAsync(c.w.dev_int, 0, 16 * sizeof(int), s);
+    if (e == cudaSuccess) e = gkv::launch_segment(c, V, hidden, hidden ? Dh : 0, surprisal, kappa, s);
+    if (e != cudaSuccess) return cuda_fail(x, e, "segment launch");
+    int h[2];
+    e = cudaMemcpyAsync(h, c.w.dev_int, 2 * sizeof(int), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(x, e, "segment");
+    st = check_status(x, h[1]);
+    if (st) return st;
+    if (h[0] <= 0) return fail(x, GKV_EINVAL, "segmentation found no partition");
+    *n_slots_host = h[0];
+    if (h[0] > cap) return fail(x, GKV_ECAPACITY, "segment: more slots than cap");
+    e = cudaMemcpyAsync(slot_starts, c.w.slots, (size_t)(h[0] + 1) * sizeof(int32_t),
+                        cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(x, e, "segment copy");
+    c.J = h[0];
+    c.stage = 1;
+    return GKV_OK;
+}
+
+gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, const void *Q,
+                               const float *omega, const int32_t *slot_starts, int32_t n_slots,
+                               void *stream) {
+    gkv_status st = ready(x, 1);
+    if (st) return st;
+    Ctx &c = x->c;
+    if (!K || !V || !Q) return fail(x, GKV_EINVAL, "build_trees: null tensor");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e;
+    if (slot_starts) {
+        if (n_slots < 1 || n_slots > c.Nc) return fail(x, GKV_EINVAL, "build_trees: bad n_slots");
+        e = cudaMemcpyAsync(c.w.slots, slot_starts, (size_t)(n_slots + 1) * sizeof(int32_t),
+                            cudaMemcpyDeviceToDevice, s);
+        int h = 0;
+        if (e == cudaSuccess) e = cudaMemsetAsync(c.w.dev_int + 1, 0, sizeof(int), s);
+        if (e == cudaSuccess) {
+            validate_slots_kernel<<<(n_slots + 255) / 256, 256, 0, s>>>(c.w.slots, n_slots, c.p.ctx_start,
+                                                                          c.c_end, c.w.dev_int + 1);
+            e = cudaGetLastError();
+        }
+        if (e == cudaSuccess) e = cudaMemcpyAsync(&h, c.w.dev_int + 1, sizeof(int), cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+        if (e != cudaSuccess) return cuda_fail(x, e, "build_trees slots");
+        st = check_status(x, h);
+        if (st) return st;
+        c.J = n_slots;
+    }
+    const int J = c.J;
+    const int64_t nu = (int64_t)c.p.L * c.p.G * J;
+    gkv::Workspace &w = c.w;
+    if (nu > w.units_cap) {   // grows only when a partition has more slots than any before
+        int64_t cap = std::max<int64_t>(nu, w.units_cap * 2);
+        bool ok = dalloc(x, &w.u_nnodes, cap) && dalloc(x, &w.u_Uadd, cap) &&
+                  dalloc(x, &w.u_Ddrop, cap) && dalloc(x, &w.u_sel, cap) &&
+                  dalloc(x, &w.u_count, cap) && dalloc(x, &w.u_off, cap);
+        if (!ok) return fail(x, GKV_ENOMEM, "build_trees: unit arrays");
+        w.units_cap = cap;
+    }
+    e = gkv::launch_row_stats(c, K, Q, s);
+    if (e == cudaSuccess) e = gkv::launch_token_values(c, K, Q, s);
+    if (e == cudaSuccess) e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, s);
+    if (e != cudaSuccess) return cuda_fail(x, e, "build_trees launch");
+    c.stage = 2;
+    return GKV_OK;
+}
+
+gkv_status gracekv_allocate(gracekv_ctx *x, int64_t *n_entries_host, void *stream) {
+    gkv_status st = ready(x, 2);
+    if (st) return st;
+    Ctx &c = x->c;
+    if (!n_entries_host) return fail(x, GKV_EINVAL, "allocate: null argument");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = gkv::launch_allocate(c, c.J, s);
+    if (e != cudaSuccess) return cuda_fail(x, e, "allocate launch");
+    unsigned long long used = 0;
+    int h = 0;
+    e = cudaMemcpyAsync(&used, c.w.alloc_state + 7, sizeof used, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&h, c.w.dev_int + 1, sizeof(int), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(x, e, "allocate");
+    st = check_status(x, h);
+    if (st) return st;
+    const int64_t LG = (int64_t)c.p.L * c.p.G;
+    c.used = (int64_t)used;
+    *n_entries_host = LG * (c.p.T - c.Nc) + c.used;
+    c.stage = 3;
+    return GKV_OK;
+}
+
+gkv_status gracekv_gather(gracekv_ctx *x, const void *K, const void *V, void *K_out, void *V_out,
+                          int32_t *pos, float *log_m, int32_t *src_lo, int32_t *src_hi,
+                          int64_t *offsets, int64_t cap, void *stream) {
+    gkv_status st = ready(x, 3);
+    if (st) return st;
+    Ctx &c = x->c;
+    if (!K || !V || !K_out || !V_out || !pos || !log_m || !src_lo || !src_hi || !offsets)
+        return fail(x, GKV_EINVAL, "gather: null argument");
+    const int64_t LG = (int64_t)c.p.L * c.p.G;
+    if (cap < LG * (c.p.T - c.Nc) + c.used) return fail(x, GKV_ECAPACITY, "gather: cap below the entry count");
+    cudaError_t e = gkv::launch_gather(c, K, V, c.w.slots, c.J, K_out, V_out, pos, log_m, src_lo,
+                                       src_hi, offsets, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(x, e, "gather launch");
+    return GKV_OK;
+}
+
+gkv_status gracekv_export(gracekv_ctx *x, int64_t node_cap, int64_t *n_nodes_host, int64_t *unit_first,
+                          float *unit_Uadd, float *unit_Ddrop, uint8_t *add_sel, int32_t *a, int32_t *b,
+                          int32_t *child0, int32_t *nchild, int32_t *cost, float *D, float *R, float *U,
+                          float *kappa, uint8_t *split_sel, float *row_m, float *row_Z, float *row_ZC,
+                          float *rtok, void *stream) {
+    gkv_status st = ready(x, 2);
+    if (st) return st;
+    Ctx &c = x->c;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int64_t LG = (int64_t)c.p.L * c.p.G, J = c.J, nu = LG * J;
+    const gkv::Workspace &w = c.w;
+    std::vector<int32_t> slots(J + 1), nn(nu);
+    std::vector<int32_t> ha(c.node_cap), hb(c.node_cap), hc(c.node_cap);
+    std::vector<int8_t> hn(c.node_cap), hk(c.node_cap);
+    std::vector<float> hD(c.node_cap), hR(c.node_cap), hU(c.node_cap), hK(c.node_cap);
+    std::vector<uint8_t> hs(c.node_cap);
+    cudaError_t e = cudaStreamSynchronize(s);
+#define CP(dst, src, n) if (e == cudaSuccess) e = cudaMemcpy(dst, src, (n) * sizeof(*(dst)), cudaMemcpyDeviceToHost)
+    CP(slots.data(), w.slots, J + 1);
+    CP(nn.data(), w.u_nnodes, nu);
+    CP(ha.data(), w.nd_a, c.node_cap); CP(hb.data(), w.nd_b, c.node_cap);
+    CP(hc.data(), w.nd_child0, c.node_cap); CP(hn.data(), w.nd_nchild, c.node_cap);
+    CP(hk.data(), w.nd_cost, c.node_cap); CP(hD.data(), w.nd_D, c.node_cap);
+    CP(hR.data(), w.nd_R, c.node_cap); CP(hU.data(), w.nd_U, c.node_cap);
+    CP(hK.data(), w.nd_kappa, c.node_cap); CP(hs.data(), w.nd_sel, c.node_cap);
+    if (unit_Uadd) CP(unit_Uadd, w.u_Uadd, nu);
+    if (unit_Ddrop) CP(unit_Ddrop, w.u_Ddrop, nu);
+    if (add_sel) CP(add_sel, w.u_sel, nu);
+    const int64_t nrow = (int64_t)c.p.L * c.p.Hq * c.p.W;
+    if (row_m) CP(row_m, w.row_m, nrow);
+    if (row_Z) CP(row_Z, w.row_Z, nrow);
+    if (row_ZC) CP(row_ZC, w.row_ZC, nrow);
+    if (rtok) CP(rtok, w.rtok, LG * c.Nc);
+#undef CP
+    if (e != cudaSuccess) return cuda_fail(x, e, "export");
+    int64_t k = 0;
+    for (int64_t uid = 0; uid < nu; uid++) {
+        int lg = (int)(uid / J), j = (int)(uid % J);
+        int64_t nb = gkv::node_base(lg, slots[j], c.p.ctx_start, c.Nc);
+        if (unit_first) unit_first[uid] = k;
+        for (int q = 0; q < nn[uid]; q++, k++) {
+            if (k >= node_cap) continue;
+            int64_t v = nb + q;
+            if (a) a[k] = ha[v];
+            if (b) b[k] = hb[v];
+            if (child0) child0[k] = hc[v];
+            if (nchild) nchild[k] = hn[v];
+            if (cost) cost[k] = hk[v];
+            if (D) D[k] = hD[v];
+            if (R) R[k] = hR[v];
+            if (U) U[k] = hU[v];
+            if (kappa) kappa[k] = hK[v];
+            if (split_sel) split_sel[k] = c.stage >= 3 ? hs[v] : 0;
+        }
+    }
+    if (unit_first) unit_first[nu] = k;
+    *n_nodes_host = k;
+    if (k > node_cap) return fail(x, GKV_ECAPACITY, "export: node_cap too small");
+    return GKV_OK;
+}
+
+}  // extern "C"

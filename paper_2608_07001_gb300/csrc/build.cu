@@ -1,0 +1,653 @@
+// build.cu -- stage 2 of the GraceKV pass: one prototype tree per
+// layer-KV-head-slot unit (App. A.2 atomic units), built level by level by one
+// CTA that keeps the whole slot in shared memory.
+//
+// Per unit (l, g, j), slot [sa, sb), n <= 128 tokens:
+//   E[u][t] = exp(q_u . k_t / sqrt d - m_u)   distortion probe u uses query
+//             head H(g)[u mod |H(g)|] (App. A.3, GQA round robin), m_u its
+//             max logit over [0, T)
+//   k_circ_t = RoPE^-1(k_t, t)                 (Eq. app_rope_prototype)
+// For every node I = [a, b) of a level, the candidate children are prefixes
+// [a, xi) and suffixes [xi, b) of I for the binary cuts X_v (top-16 positions
+// by curvature in [a, b-2], cut xi = t + 1, plus the midpoint; App. B.4
+// Eq. app_tree_split_candidates) and the two sides of the salient-token
+// extraction at p* = argmax R_tok (Eq. app_extract_split).  For each
+// candidate J the prototype (ktil, vtil, m_eff; Eqs. app_rope_prototype,
+// app_value_prototype, app_effective_multiplicity) is formed by direct sums
+// over J; then one forward and one backward scan over the level's tokens
+// accumulate Z_u(J) and M_u(J) (Eq. app_original_attention_stats) for every
+// probe and evaluate D_u (Eq. app_probe_distortion) at each candidate end,
+// weighted by the attention mass Z_u(J) / Z_u (Eq.
+// app_node_and_drop_distortion).  The refinement form follows Eqs.
+// app_binary_split .. app_split_choice; gains, costs and utilities follow
+// Eqs. app_operation_gains .. app_unit_utility (clamped at 0); each Split op
+// also gets its bottleneck key kappa = min(U, kappa of the op that created
+// the node), which the allocator's threshold select uses.
+#include "gkv_internal.cuh"
+
+namespace gkv {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+constexpr int kNCmax = 48;       // candidate intervals per batch (at least 2*17+3 = 37 per node)
+constexpr int kNB = 32;          // nodes per batch
+constexpr int kMaxCuts = 18;     // K + midpoint, K <= 16 (+1 spare)
+constexpr int kMaxNodes = 2 * kMaxUnit;
+
+struct BuildArgs {
+    const void *K, *V, *Q;
+    const int32_t *slots;
+    const float2 *rope;
+    const double *kappa;
+    const float *rtok, *row_m, *row_Z, *omega;
+    int L, G, Hq, T, d, W, gq, cs, Nc, J, k_cand;
+    float inv_sqrt_d, lamZ, lamM, eps;
+    double lam_kappa, base_frac, eps_d;
+    // outputs
+    int32_t *nd_a, *nd_b, *nd_child0, *nd_parent, *nd_unit;
+    int8_t *nd_nchild, *nd_cost;
+    float *nd_D, *nd_R, *nd_U, *nd_kappa;
+    uint8_t *nd_sel;
+    int32_t *u_nnodes;
+    float *u_Uadd, *u_Ddrop;
+    uint8_t *u_sel;
+    int *status;
+};
+
+struct NodeS {
+    int a, b, parent, child0, nchild;
+    double D, R;
+    float kin;       // bottleneck key of the op that created the node
+};
+
+struct BatchNode {
+    int node;
+    int ncut;
+    int cut[kMaxCuts];      // local cut positions xi (ascending)
+    int pidx[kMaxCuts];     // candidate index of [a, xi) (-1: single token)
+    int sidx[kMaxCuts];     // candidate index of [xi, b) (-1: single token)
+    int pstar, eL, eR, whole;
+    int pre_b, pre_e, suf_b, suf_e;   // candidate ranges (prefixes ascending end,
+                                      // suffixes descending start)
+    double kmin, kmax;
+    int nchild, ca[3], cb[3];
+    double cD[3];
+};
+
+struct Cand {
+    int a, b;        // local interval
+    float meff;
+};
+
+__device__ __forceinline__ int round_half_even_mid(int a, int b) {
+    int s = a + b - 1;
+    if ((s & 1) == 0) return s >> 1;
+    int lo = (s - 1) >> 1;
+    return (lo & 1) == 0 ? lo : lo + 1;
+}
+
+template <int DH, int NW, typename Tin>
+struct Smem {
+    static constexpr int NCH = kThreads / NW;
+    static constexpr int CH = DH / NCH;
+    // fp32 slots of d = 128 with 64 probes leave room for 38 candidates only
+    static constexpr int NC = (DH == 128 && NW == 64 && sizeof(Tin) == 4) ? 38 : kNCmax;
+    static_assert(NC >= 37, "one node needs up to 2 * 17 + 3 candidate intervals");
+    float kc[kMaxUnit][DH];
+    Tin vv[kMaxUnit][DH];
+    float E[NW][kMaxUnit];
+    float ktil[NC][DH];
+    float vtil[NC][DH];
+    float Rt[kMaxUnit];
+    float kn[kMaxUnit];
+    double kap[kMaxUnit];
+    float redD[NC][kWarps];
+    float redP[NC][kWarps];
+    Cand cand[NC];
+    NodeS nodes[kMaxNodes];
+    BatchNode bn[kNB];
+    short lvl[2][kMaxNodes];
+    int nlvl[2];
+    int nnodes;
+    int batch_n, batch_next, ncand;
+};
+
+template <int DH, int NW, typename Tin>
+__global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
+    using S = Smem<DH, NW, Tin>;
+    constexpr int NCH = S::NCH, CH = S::CH, HALF = DH / 2;
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    S &sm = *reinterpret_cast<S *>(smem_raw);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int LG = A.L * A.G;
+    const int j = blockIdx.x / LG, lg = blockIdx.x - j * LG;
+    const int l = lg / A.G, g = lg - l * A.G;
+    const int sa = A.slots[j], sb = A.slots[j + 1];
+    const int n = sb - sa;
+    const int64_t uid = (int64_t)lg * A.J + j;
+    const int64_t nbase = node_base(lg, sa, A.cs, A.Nc);
+    if (n < 1 || n > kMaxUnit) {
+        if (tid == 0) atomicOr(A.status, 4);
+        return;
+    }
+    const Tin *Kp = static_cast<const Tin *>(A.K) + ((size_t)lg * A.T + sa) * DH;
+    const Tin *Vp = static_cast<const Tin *>(A.V) + ((size_t)lg * A.T + sa) * DH;
+    const float om = A.omega ? A.omega[lg] : 1.0f;
+
+    // ---- load the slot ------------------------------------------------------
+    for (int e = tid * 8; e < n * DH; e += kThreads * 8) {
+        Vec8<Tin> kx, vx;
+        kx.load(Kp + e);
+        vx.load(Vp + e);
+        int t = e / DH, i = e - t * DH;
+#pragma unroll
+        for (int q = 0; q < 8; q++) {
+            sm.kc[t][i + q] = kx.v[q];
+            sm.vv[t][i + q] = (Tin)vx.v[q];
+        }
+    }
+    for (int t = tid; t < n; t += kThreads) {
+        sm.kap[t] = A.kappa[sa + t];
+        sm.Rt[t] = A.rtok[(size_t)lg * A.Nc + (sa - A.cs) + t];
+    }
+    // probe registers: thread (u, c) owns chunk c of probe u
+    const int u = tid / NCH, c = tid - u * NCH;
+    const bool pact = u < A.W;
+    float qreg[CH];
+    float mu = 0.f, invZ = 0.f;
+    {
+        const int h = g * A.gq + (u % A.gq);
+        const size_t row = ((size_t)l * A.Hq + h) * A.W + u;
+        if (pact) {
+            const Tin *qp = static_cast<const Tin *>(A.Q) + row * DH + c * CH;
+#pragma unroll
+            for (int k = 0; k < CH; k += 8) {
+                Vec8<Tin> x;
+                x.load(qp + k);
+#pragma unroll
+                for (int q = 0; q < 8; q++) qreg[k + q] = x.v[q];
+            }
+            mu = A.row_m[row];
+            invZ = 1.0f / A.row_Z[row];
+        } else {
+#pragma unroll
+            for (int k = 0; k < CH; k++) qreg[k] = 0.f;
+        }
+    }
+    __syncthreads();
+
+    // ---- E[u][t] from the raw (post-RoPE) keys -------------------------------
+    for (int t = 0; t < n; t++) {
+        float x = 0.f;
+#pragma unroll
+        for (int k = 0; k < CH; k++) x = fmaf(qreg[k], sm.kc[t][c * CH + k], x);
+#pragma unroll
+        for (int o = 1; o < NCH; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+        if (c == 0) sm.E[u][t] = pact ? expf(x * A.inv_sqrt_d - mu) : 0.f;
+    }
+    __syncthreads();
+    // ---- k_circ = RoPE^-1(k, t) ----------------------------------------------
+    for (int e = tid; e < n * HALF; e += kThreads) {
+        int t = e / HALF, i = e - t * HALF;
+        float2 cs = A.rope[(size_t)(sa + t) * HALF + i];
+        float x = sm.kc[t][i], y = sm.kc[t][i + HALF];
+        sm.kc[t][i] = x * cs.x + y * cs.y;
+        sm.kc[t][i + HALF] = y * cs.x - x * cs.y;
+    }
+    __syncthreads();
+    for (int t = warp; t < n; t += kWarps) {
+        float s = 0.f;
+        for (int i = lane; i < DH; i += 32) s = fmaf(sm.kc[t][i], sm.kc[t][i], s);
+        s = warp_sum(s);
+        if (lane == 0) sm.kn[t] = sqrtf(s);
+    }
+    // ---- root -----------------------------------------------------------------
+    if (warp == 0) {
+        double r = 0.0;
+        for (int t = lane; t < n; t += 32) r += sm.Rt[t];
+        r = warp_sum(r);
+        if (lane == 0) {
+            NodeS &nd = sm.nodes[0];
+            nd.a = 0; nd.b = n; nd.parent = -1; nd.child0 = -1; nd.nchild = 0;
+            nd.D = 0.0; nd.R = r; nd.kin = 0.f;
+            sm.nnodes = 1;
+            sm.lvl[0][0] = 0;
+            sm.nlvl[0] = 1;
+            A.nd_a[nbase] = sa; A.nd_b[nbase] = sb; A.nd_R[nbase] = (float)r;
+            A.nd_parent[nbase] = (int32_t)(-2 - uid);
+            A.nd_unit[nbase] = (int32_t)uid;
+        }
+    }
+    __syncthreads();
+
+    int cur = 0;
+    while (sm.nlvl[cur] > 0) {
+        const int nl = sm.nlvl[cur];
+        if (tid == 0) { sm.nlvl[cur ^ 1] = 0; sm.batch_next = 0; }
+        __syncthreads();
+        while (sm.batch_next < nl) {
+            // ---- batch assignment (thread 0) --------------------------------
+            if (tid == 0) {
+                int nb = 0, used = 0, k = sm.batch_next;
+                while (k < nl && nb < kNB) {
+                    int v = sm.lvl[cur][k];
+                    int nv = sm.nodes[v].b - sm.nodes[v].a;
+                    int ub = (v == 0 ? 1 : 0) + (nv >= 3 ? 2 * min(A.k_cand + 1, nv - 1) + 2 : 0);
+                    if (used + ub > S::NC) break;
+                    sm.bn[nb].node = v;
+                    sm.bn[nb].pre_b = used;
+                    used += ub;
+                    nb++;
+                    k++;
+                }
+                sm.batch_n = nb;
+                sm.batch_next = k;
+                sm.ncand = used;
+            }
+            __syncthreads();
+            const int nb = sm.batch_n;
+            // ---- phase A: cut candidates per node (warp per node) ------------
+            for (int bi = warp; bi < nb; bi += kWarps) {
+                BatchNode &B = sm.bn[bi];
+                const int v = B.node;
+                const int a = sm.nodes[v].a, b = sm.nodes[v].b, nv = b - a;
+                // top-K by curvature over positions [a, b-2] (ties: lower t)
+                unsigned sel[kMaxUnit / 32];
+                double kmin = INFINITY, kmax = -INFINITY;
+#pragma unroll
+                for (int w = 0; w < kMaxUnit / 32; w++) {
+                    int t = a + w * 32 + lane;
+                    bool in = t <= b - 2;
+                    bool s = false;
+                    if (in) {
+                        double kt = sm.kap[t];
+                        kmin = fmin(kmin, kt);
+                        kmax = fmax(kmax, kt);
+                        int rank = 0;
+                        for (int q = a; q <= b - 2; q++) {
+                            double kq = sm.kap[q];
+                            rank += (kq > kt) || (kq == kt && q < t);
+                        }
+                        s = rank < A.k_cand || t == a + nv / 2 - 1;   // + midpoint
+                    }
+                    sel[w] = __ballot_sync(0xffffffffu, s);
+                }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) {
+                    kmin = fmin(kmin, __shfl_xor_sync(0xffffffffu, kmin, o));
+                    kmax = fmax(kmax, __shfl_xor_sync(0xffffffffu, kmax, o));
+                }
+                // salient token p* = argmax R_tok over [a, b) (ties: lower t)
+                float rb = -INFINITY;
+                int pb = 0x7fffffff;
+                for (int t = a + lane; t < b; t += 32) {
+                    float r = sm.Rt[t];
+                    if (r > rb) { rb = r; pb = t; }
+                }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) {
+                    float r2 = __shfl_xor_sync(0xffffffffu, rb, o);
+                    int p2 = __shfl_xor_sync(0xffffffffu, pb, o);
+                    if (r2 > rb || (r2 == rb && p2 < pb)) { rb = r2; pb = p2; }
+                }
+                if (lane == 0) {
+                    B.kmin = kmin;
+                    B.kmax = kmax;
+                    B.pstar = pb;
+                    B.ncut = 0;
+                    B.eL = B.eR = B.whole = -1;
+                    int k = B.pre_b;
+                    const bool cands = nv >= 3;
+                    if (cands) {
+                        for (int w = 0; w < kMaxUnit / 32; w++) {
+                            unsigned m = sel[w];
+                            while (m) {
+                                int bit = __ffs(m) - 1;
+                                m &= m - 1;
+                                B.cut[B.ncut++] = a + w * 32 + bit + 1;
+                            }
+                        }
+                        // prefixes in ascending end: cuts merged with the extraction's left side
+                        bool el_done = !(pb - a >= 2);
+                        for (int q = 0; q < B.ncut; q++) {
+                            int xi = B.cut[q];
+                            if (!el_done && pb <= xi) {
+                                if (pb == xi) { B.eL = -2 - q; }   // same interval as cut q
+                                else { sm.cand[k] = {a, pb, 0.f}; B.eL = k++; }
+                                el_done = true;
+                            }
+                            if (xi - a >= 2) { sm.cand[k] = {a, xi, 0.f}; B.pidx[q] = k++; }
+                            else B.pidx[q] = -1;
+                        }
+                        if (!el_done) { sm.cand[k] = {a, pb, 0.f}; B.eL = k++; }
+                        if (B.eL <= -2) B.eL = B.pidx[-2 - B.eL];
+                    }
+                    if (v == 0) { sm.cand[k] = {a, b, 0.f}; B.whole = k++; }
+                    B.pre_e = k;
+                    B.suf_b = k;
+                    if (cands) {
+                        // suffixes in descending start: cuts (descending) merged with p*+1
+                        int er = pb + 1;
+                        bool er_done = !(b - er >= 2);
+                        for (int q = B.ncut - 1; q >= 0; q--) {
+                            int xi = B.cut[q];
+                            if (!er_done && er >= xi) {
+                                if (er == xi) B.eR = -2 - q;
+                                else { sm.cand[k] = {er, b, 0.f}; B.eR = k++; }
+                                er_done = true;
+                            }
+                            if (b - xi >= 2) { sm.cand[k] = {xi, b, 0.f}; B.sidx[q] = k++; }
+                            else B.sidx[q] = -1;
+                        }
+                        if (!er_done) { sm.cand[k] = {er, b, 0.f}; B.eR = k++; }
+                        if (B.eR <= -2) B.eR = B.sidx[-2 - B.eR];
+                    }
+                    B.suf_e = k;
+                }
+            }
+            __syncthreads();
+            // ---- phase B: prototype of every candidate (warp per candidate) ----
+            for (int bi = 0; bi < nb; bi++) {
+                const BatchNode &B = sm.bn[bi];
+                for (int k = B.pre_b + warp; k < B.suf_e; k += kWarps) {
+                    const int ja = sm.cand[k].a, jb = sm.cand[k].b, nJ = jb - ja;
+                    double rs = 0.0, ks = 0.0;
+                    for (int t = ja + lane; t < jb; t += 32) { rs += sm.Rt[t]; ks += sm.kn[t]; }
+                    rs = warp_sum(rs);
+                    ks = warp_sum(ks);
+                    const float beta = (float)(A.base_frac * (rs / nJ));
+                    const double wsum = rs + nJ * (double)beta;
+                    const float winv = (float)(1.0 / (wsum + A.eps_d));
+                    const float ninv = 1.0f / (float)nJ;
+                    const int p = round_half_even_mid(sa + ja, sa + jb);   // absolute positions
+                    float mu2 = 0.f;
+                    for (int i = lane; i < HALF; i += 32) {
+                        float m0 = 0.f, m1 = 0.f, v0 = 0.f, v1 = 0.f;
+                        for (int t = ja; t < jb; t++) {
+                            m0 += sm.kc[t][i];
+                            m1 += sm.kc[t][i + HALF];
+                            float wt = sm.Rt[t] + beta;
+                            v0 = fmaf(wt, to_f(sm.vv[t][i]), v0);
+                            v1 = fmaf(wt, to_f(sm.vv[t][i + HALF]), v1);
+                        }
+                        m0 *= ninv;
+                        m1 *= ninv;
+                        mu2 = fmaf(m0, m0, fmaf(m1, m1, mu2));
+                        float2 cs = A.rope[(size_t)p * HALF + i];
+                        sm.ktil[k][i] = m0 * cs.x - m1 * cs.y;
+                        sm.ktil[k][i + HALF] = m0 * cs.y + m1 * cs.x;
+                        sm.vtil[k][i] = v0 * winv;
+                        sm.vtil[k][i + HALF] = v1 * winv;
+                    }
+                    mu2 = warp_sum(mu2);
+                    if (lane == 0) {
+                        double coh = sqrt((double)mu2) / (ks / nJ + A.eps_d);
+                        double me = nJ * coh * coh;
+                        sm.cand[k].meff = (float)(me < 1.0 ? 1.0 : (me > nJ ? (double)nJ : me));
+                    }
+                }
+            }
+            __syncthreads();
+            // ---- phase C: probe scans --------------------------------------------
+            auto evaluate = [&](int k, float Z, const float *M) {
+                float x = 0.f;
+#pragma unroll
+                for (int q = 0; q < CH; q++) x = fmaf(qreg[q], sm.ktil[k][c * CH + q], x);
+#pragma unroll
+                for (int o = 1; o < NCH; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+                const float zt = sm.cand[k].meff * expf(x * A.inv_sqrt_d - mu);
+                float res = 0.f, mm = 0.f;
+#pragma unroll
+                for (int q = 0; q < CH; q++) {
+                    float df = M[q] - zt * sm.vtil[k][c * CH + q];
+                    res = fmaf(df, df, res);
+                    mm = fmaf(M[q], M[q], mm);
+                }
+#pragma unroll
+                for (int o = 1; o < NCH; o <<= 1) {
+                    res += __shfl_xor_sync(0xffffffffu, res, o);
+                    mm += __shfl_xor_sync(0xffffffffu, mm, o);
+                }
+                float pd = 0.f, pp = 0.f;
+                if (pact) {
+                    float dz = Z - zt;
+                    float Du = A.lamZ * (dz * dz) / (Z * Z + A.eps) + A.lamM * res / (mm + A.eps);
+                    pp = Z * invZ;
+                    pd = pp * Du;
+                }
+#pragma unroll
+                for (int o = NCH; o < 32; o <<= 1) {
+                    pd += __shfl_xor_sync(0xffffffffu, pd, o);
+                    pp += __shfl_xor_sync(0xffffffffu, pp, o);
+                }
+                if (lane == 0) { sm.redD[k][warp] = pd; sm.redP[k][warp] = pp; }
+            };
+            for (int bi = 0; bi < nb; bi++) {
+                const BatchNode &B = sm.bn[bi];
+                if (B.pre_e == B.pre_b && B.suf_e == B.suf_b) continue;
+                const int a = sm.nodes[B.node].a, b = sm.nodes[B.node].b;
+                float M[CH];
+                float Z = 0.f;
+                // forward: prefixes [a, end) in ascending end
+                int k = B.pre_b;
+                if (k < B.pre_e) {
+#pragma unroll
+                    for (int q = 0; q < CH; q++) M[q] = 0.f;
+                    for (int t = a; t < b && k < B.pre_e; t++) {
+                        const float e = sm.E[u][t];
+                        Z += e;
+#pragma unroll
+                        for (int q = 0; q < CH; q++) M[q] = fmaf(e, to_f(sm.vv[t][c * CH + q]), M[q]);
+                        while (k < B.pre_e && sm.cand[k].b == t + 1) { evaluate(k, Z, M); k++; }
+                    }
+                }
+                // backward: suffixes [start, b) in descending start
+                k = B.suf_b;
+                if (k < B.suf_e) {
+                    Z = 0.f;
+#pragma unroll
+                    for (int q = 0; q < CH; q++) M[q] = 0.f;
+                    for (int t = b - 1; t >= a && k < B.suf_e; t--) {
+                        const float e = sm.E[u][t];
+                        Z += e;
+#pragma unroll
+                        for (int q = 0; q < CH; q++) M[q] = fmaf(e, to_f(sm.vv[t][c * CH + q]), M[q]);
+                        while (k < B.suf_e && sm.cand[k].a == t) { evaluate(k, Z, M); k++; }
+                    }
+                }
+            }
+            __syncthreads();
+            // ---- phase D1: decisions (warp per node, lane 0) --------------------
+            for (int bi = warp; bi < nb; bi += kWarps) {
+                if (lane) continue;
+                BatchNode &B = sm.bn[bi];
+                NodeS &nd = sm.nodes[B.node];
+                const int a = nd.a, b = nd.b, nv = b - a;
+                auto Dc = [&](int k) -> double {
+                    double s = 0.0;
+                    for (int w = 0; w < kWarps; w++) s += sm.redD[k][w];
+                    return s / A.W;
+                };
+                if (B.whole >= 0) {   // root: D, Ddrop, Add gain (Eq. app_operation_gains)
+                    double Pd = 0.0;
+                    for (int w = 0; w < kWarps; w++) Pd += sm.redP[B.whole][w];
+                    Pd /= A.W;
+                    double D = nv >= 2 ? Dc(B.whole) : 0.0;
+                    nd.D = D;
+                    double gain = (double)om * nd.R * (Pd - D);
+                    if (gain < 0.0) gain = 0.0;
+                    nd.kin = (float)gain;
+                    A.u_Uadd[uid] = (float)gain;
+                    A.u_Ddrop[uid] = (float)Pd;
+                    A.nd_D[nbase] = (float)D;
+                }
+                B.nchild = 0;
+                if (nv < 2) continue;
+                const double DI = nd.D;
+                if (nv == 2) {
+                    B.nchild = 2;
+                    B.ca[0] = a; B.cb[0] = a + 1; B.cD[0] = 0.0;
+                    B.ca[1] = a + 1; B.cb[1] = b; B.cD[1] = 0.0;
+                    continue;
+                }
+                // binary cut: max G_bin, ties -> smallest xi
+                double best = -INFINITY, bL = 0, bR = 0;
+                int bxi = -1;
+                for (int q = 0; q < B.ncut; q++) {
+                    int xi = B.cut[q];
+                    double DL = B.pidx[q] >= 0 ? Dc(B.pidx[q]) : 0.0;
+                    double DR = B.sidx[q] >= 0 ? Dc(B.sidx[q]) : 0.0;
+                    double kh = B.kmax > B.kmin ? (sm.kap[xi - 1] - B.kmin) / (B.kmax - B.kmin) : 0.0;
+                    double gb = ((DI - DL) - DR) + A.lam_kappa * kh;
+                    if (gb > best) { best = gb; bxi = xi; bL = DL; bR = DR; }
+                }
+                // extraction at p*
+                const int ps = B.pstar;
+                int ea[3], eb[3], ne = 0;
+                double eD[3];
+                if (ps > a) { ea[ne] = a; eb[ne] = ps; eD[ne] = ps - a >= 2 ? Dc(B.eL) : 0.0; ne++; }
+                ea[ne] = ps; eb[ne] = ps + 1; eD[ne] = 0.0; ne++;
+                if (ps + 1 < b) { ea[ne] = ps + 1; eb[ne] = b; eD[ne] = b - ps - 1 >= 2 ? Dc(B.eR) : 0.0; ne++; }
+                double gext = DI;
+                for (int q = 0; q < ne; q++) gext -= eD[q];
+                const double rho_ext = gext / (ne - 1);
+                if (rho_ext > best) {
+                    B.nchild = ne;
+                    for (int q = 0; q < ne; q++) { B.ca[q] = ea[q]; B.cb[q] = eb[q]; B.cD[q] = eD[q]; }
+                } else {
+                    B.nchild = 2;
+                    B.ca[0] = a; B.cb[0] = bxi; B.cD[0] = bL;
+                    B.ca[1] = bxi; B.cb[1] = b; B.cD[1] = bR;
+                }
+            }
+            __syncthreads();
+            // ---- child numbering (deterministic, breadth-first) ----------------
+            if (tid == 0) {
+                int cnt = sm.nnodes;
+                for (int bi = 0; bi < nb; bi++) {
+                    BatchNode &B = sm.bn[bi];
+                    NodeS &nd = sm.nodes[B.node];
+                    nd.nchild = B.nchild;
+                    nd.child0 = B.nchild ? cnt : -1;
+                    cnt += B.nchild;
+                }
+                sm.nnodes = cnt;
+            }
+            __syncthreads();
+            // ---- phase D2: children, gains, keys (warp per node) ----------------
+            for (int bi = warp; bi < nb; bi += kWarps) {
+                const BatchNode &B = sm.bn[bi];
+                NodeS &nd = sm.nodes[B.node];
+                const int64_t gv = nbase + B.node;
+                if (B.nchild == 0) {
+                    if (lane == 0) {
+                        A.nd_child0[gv] = -1; A.nd_nchild[gv] = 0; A.nd_cost[gv] = 0;
+                        A.nd_U[gv] = 0.f; A.nd_kappa[gv] = 0.f; A.nd_sel[gv] = 0;
+                    }
+                    continue;
+                }
+                double dsum = 0.0, rch[3];
+                for (int q = 0; q < B.nchild; q++) {
+                    double r = 0.0;
+                    for (int t = B.ca[q] + lane; t < B.cb[q]; t += 32) r += sm.Rt[t];
+                    rch[q] = warp_sum(r);
+                    dsum += B.cD[q];
+                }
+                if (lane == 0) {
+                    const int cost = B.nchild - 1;
+                    double gain = (double)om * nd.R * (nd.D - dsum);
+                    if (gain < 0.0) gain = 0.0;
+                    float U = (float)(gain / cost);
+                    float kap = fminf(U, nd.kin);
+                    A.nd_child0[gv] = nd.child0; A.nd_nchild[gv] = (int8_t)B.nchild;
+                    A.nd_cost[gv] = (int8_t)cost; A.nd_U[gv] = U; A.nd_kappa[gv] = kap;
+                    A.nd_sel[gv] = 0;
+                    int nxt = cur ^ 1;
+                    for (int q = 0; q < B.nchild; q++) {
+                        int ci = nd.child0 + q;
+                        NodeS &ch = sm.nodes[ci];
+                        ch.a = B.ca[q]; ch.b = B.cb[q]; ch.parent = B.node;
+                        ch.child0 = -1; ch.nchild = 0; ch.D = B.cD[q]; ch.R = rch[q]; ch.kin = kap;
+                        const int64_t gc = nbase + ci;
+                        A.nd_a[gc] = sa + ch.a; A.nd_b[gc] = sa + ch.b;
+                        A.nd_parent[gc] = (int32_t)gv; A.nd_unit[gc] = (int32_t)uid;
+                        A.nd_D[gc] = (float)ch.D; A.nd_R[gc] = (float)ch.R;
+                        A.nd_child0[gc] = -1; A.nd_nchild[gc] = 0; A.nd_cost[gc] = 0;
+                        A.nd_U[gc] = 0.f; A.nd_kappa[gc] = 0.f; A.nd_sel[gc] = 0;
+                        if (ch.b - ch.a >= 2) {
+                            int pos = atomicAdd(&sm.nlvl[nxt], 1);
+                            sm.lvl[nxt][pos] = (short)ci;
+                        }
+                    }
+                }
+            }
+            __syncthreads();
+        }
+        // keep the next level in creation order (atomic appends may permute it)
+        if (tid == 0) {
+            int nx = cur ^ 1, m = sm.nlvl[nx];
+            for (int x = 1; x < m; x++) {
+                short v = sm.lvl[nx][x];
+                int y = x - 1;
+                while (y >= 0 && sm.lvl[nx][y] > v) { sm.lvl[nx][y + 1] = sm.lvl[nx][y]; y--; }
+                sm.lvl[nx][y + 1] = v;
+            }
+        }
+        __syncthreads();
+        cur ^= 1;
+    }
+    if (tid == 0) {
+        A.u_nnodes[uid] = sm.nnodes;
+        A.u_sel[uid] = 0;
+    }
+    // unused node slots of the unit carry cost 0 (no op)
+    for (int k = sm.nnodes + tid; k < 2 * n; k += kThreads) A.nd_cost[nbase + k] = 0;
+}
+
+template <int DH, int NW, typename Tin>
+cudaError_t launch_t(Ctx &c, BuildArgs &A, int J, cudaStream_t s) {
+    using S = Smem<DH, NW, Tin>;
+    static_assert(sizeof(S) <= 227 * 1024, "unit kernel shared memory above the per-CTA limit");
+    size_t sm = sizeof(S);
+    cudaError_t e = cudaFuncSetAttribute(unit_build_kernel<DH, NW, Tin>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    unsigned grid = (unsigned)((int64_t)J * c.p.L * c.p.G);
+    unit_build_kernel<DH, NW, Tin><<<grid, kThreads, sm, s>>>(A);
+    return cudaGetLastError();
+}
+
+template <typename Tin>
+cudaError_t launch_dt(Ctx &c, BuildArgs &A, int J, cudaStream_t s) {
+    int nw = c.p.W <= 32 ? 32 : 64;
+    if (c.p.d == 128) return nw == 32 ? launch_t<128, 32, Tin>(c, A, J, s) : launch_t<128, 64, Tin>(c, A, J, s);
+    return nw == 32 ? launch_t<64, 32, Tin>(c, A, J, s) : launch_t<64, 64, Tin>(c, A, J, s);
+}
+
+}  // namespace
+
+cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *Q,
+                              const float *omega, const int32_t *slots, int J, cudaStream_t s) {
+    const gkv_params &p = c.p;
+    BuildArgs A;
+    A.K = K; A.V = V; A.Q = Q;
+    A.slots = slots; A.rope = c.w.rope; A.kappa = c.w.kappa;
+    A.rtok = c.w.rtok; A.row_m = c.w.row_m; A.row_Z = c.w.row_Z; A.omega = omega;
+    A.L = p.L; A.G = p.G; A.Hq = p.Hq; A.T = p.T; A.d = p.d; A.W = p.W; A.gq = p.Hq / p.G;
+    A.cs = p.ctx_start; A.Nc = c.Nc; A.J = J; A.k_cand = p.k_cand;
+    A.inv_sqrt_d = (float)(1.0 / sqrt((double)p.d));
+    A.lamZ = (float)p.lambda_Z; A.lamM = (float)p.lambda_M; A.eps = (float)p.eps;
+    A.lam_kappa = p.lambda_kappa; A.base_frac = p.base_frac; A.eps_d = p.eps;
+    A.nd_a = c.w.nd_a; A.nd_b = c.w.nd_b; A.nd_child0 = c.w.nd_child0;
+    A.nd_parent = c.w.nd_parent; A.nd_unit = c.w.nd_unit;
+    A.nd_nchild = c.w.nd_nchild; A.nd_cost = c.w.nd_cost;
+    A.nd_D = c.w.nd_D; A.nd_R = c.w.nd_R; A.nd_U = c.w.nd_U; A.nd_kappa = c.w.nd_kappa;
+    A.nd_sel = c.w.nd_sel;
+    A.u_nnodes = c.w.u_nnodes; A.u_Uadd = c.w.u_Uadd; A.u_Ddrop = c.w.u_Ddrop; A.u_sel = c.w.u_sel;
+    A.status = c.w.dev_int + 1;
+    if (p.dtype == GKV_BF16) return launch_dt<__nv_bfloat16>(c, A, J, s);
+    return launch_dt<float>(c, A, J, s);
+}
+
+}  // namespace gkv

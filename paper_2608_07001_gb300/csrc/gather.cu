@@ -1,0 +1,265 @@
+// gather.cu -- stage 4 of the GraceKV pass: packing of the retained frontier
+// into a ragged cache (App. A.5 "Frontier updates and physical packing").
+//
+// A node is on the frontier when the op that created it was executed (the
+// Add for a root, the parent's Split otherwise) and its own Split was not.
+// Per (l, g) the cache holds, in ascending position: the prefix [0, c_s),
+// the frontier nodes of every covered slot, then the recent window and the
+// suffix [c_e - r, T).  Single tokens keep their original K/V bits, position
+// and log m = 0; other nodes store the prototype (ktil, vtil, p, log m_eff) of
+// Eqs. app_rope_prototype, app_value_prototype, app_effective_multiplicity,
+// recomputed here from K, V and the token values.
+//
+// Kernels: gather_count (frontier entries per unit), gather_scan (one block,
+// ordered exclusive scan -> per-unit and per-(l, g) offsets), gather_units
+// (warp per unit, depth-first in ascending position), gather_tokens
+// (prefix / recent / suffix copies).
+#include "gkv_internal.cuh"
+
+namespace gkv {
+namespace {
+
+struct GatherArgs {
+    const void *K, *V;
+    const float *rtok;
+    const float2 *rope;
+    const int32_t *slots;
+    const int32_t *nd_a, *nd_b, *nd_child0;
+    const int8_t *nd_nchild;
+    const uint8_t *nd_sel, *u_sel;
+    const int32_t *u_nnodes;
+    int32_t *u_count;
+    int64_t *u_off;
+    int L, G, T, d, J, cs, cend, Nc;
+    double base_frac, eps;
+    void *K_out, *V_out;
+    int32_t *pos, *src_lo, *src_hi;
+    float *log_m;
+    int64_t *offsets;
+};
+
+__device__ __forceinline__ int round_half_even_mid(int a, int b) {
+    int s = a + b - 1;
+    if ((s & 1) == 0) return s >> 1;
+    int lo = (s - 1) >> 1;
+    return (lo & 1) == 0 ? lo : lo + 1;
+}
+
+__device__ __forceinline__ void store(float *p, float x) { *p = x; }
+__device__ __forceinline__ void store(__nv_bfloat16 *p, float x) { *p = __float2bfloat16_rn(x); }
+
+__global__ void gather_count_kernel(GatherArgs A) {
+    int64_t nu = (int64_t)A.L * A.G * A.J;
+    int64_t uid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (uid >= nu) return;
+    int lg = (int)(uid / A.J), j = (int)(uid - (int64_t)lg * A.J);
+    int cnt = 0;
+    if (A.u_sel[uid] == 1) {
+        int64_t nb = node_base(lg, A.slots[j], A.cs, A.Nc);
+        int nn = A.u_nnodes[uid];
+        // frontier count = 1 + sum over executed splits of (|child| - 1)
+        cnt = 1;
+        for (int k = 0; k < nn; k++)
+            if (A.nd_sel[nb + k] == 1) cnt += A.nd_nchild[nb + k] - 1;
+    }
+    A.u_count[uid] = cnt;
+}
+
+// Ordered exclusive scan of the per-unit counts; unit offsets include the
+// prefix tokens of its (l, g) and the prefix + tail tokens of earlier (l, g).
+__global__ void __launch_bounds__(1024) gather_scan_kernel(GatherArgs A) {
+    __shared__ long long part[1024];
+    const int64_t nu = (int64_t)A.L * A.G * A.J;
+    const int tid = threadIdx.x;
+    const int64_t per = (nu + 1023) / 1024;
+    const int64_t b = tid * per, e = b + per < nu ? b + per : nu;
+    long long s = 0;
+    for (int64_t i = b; i < e; i++) s += A.u_count[i];
+    part[tid] = s;
+    __syncthreads();
+    if (tid == 0) {
+        long long acc = 0;
+        for (int k = 0; k < 1024; k++) { long long v = part[k]; part[k] = acc; acc += v; }
+    }
+    __syncthreads();
+    const long long extra = (long long)A.cs + (A.T - A.cend);   // uncompressed entries per (l, g)
+    long long acc = part[tid];
+    for (int64_t i = b; i < e; i++) {
+        int lg = (int)(i / A.J), j = (int)(i - (int64_t)lg * A.J);
+        long long off = acc + (long long)lg * extra + A.cs;
+        A.u_off[i] = off;
+        if (j == 0) A.offsets[lg] = off - A.cs;
+        acc += A.u_count[i];
+    }
+    if (tid == 1023) A.offsets[A.L * A.G] = acc + (long long)A.L * A.G * extra;
+    if (nu == 0 && tid == 0)
+        for (int lg = 0; lg <= A.L * A.G; lg++) A.offsets[lg] = (long long)lg * extra;
+}
+
+template <typename Tin>
+__device__ void emit_node(const GatherArgs &A, int lg, int a, int b, int64_t e, int lane) {
+    const int d = A.d, half = d / 2;
+    const Tin *K = static_cast<const Tin *>(A.K) + (size_t)lg * A.T * d;
+    const Tin *V = static_cast<const Tin *>(A.V) + (size_t)lg * A.T * d;
+    Tin *Ko = static_cast<Tin *>(A.K_out) + (size_t)e * d;
+    Tin *Vo = static_cast<Tin *>(A.V_out) + (size_t)e * d;
+    const int n = b - a;
+    if (n == 1) {
+        for (int i = lane; i < d; i += 32) {
+            Ko[i] = K[(size_t)a * d + i];
+            Vo[i] = V[(size_t)a * d + i];
+        }
+        if (lane == 0) { A.pos[e] = a; A.log_m[e] = 0.f; A.src_lo[e] = a; A.src_hi[e] = b; }
+        return;
+    }
+    const float *R = A.rtok + (size_t)lg * A.Nc - A.cs;
+    double rs = 0.0;
+    for (int t = a + lane; t < b; t += 32) rs += R[t];
+    rs = warp_sum(rs);
+    const float beta = (float)(A.base_frac * (rs / n));
+    const double wsum = rs + n * (double)beta;
+    const float winv = (float)(1.0 / (wsum + A.eps));
+    const float ninv = 1.0f / (float)n;
+    const int p = round_half_even_mid(a, b);
+    // mean of the inverse-rotated keys and the mean of their norms
+    double knorm = 0.0;
+    float mu2 = 0.f;
+    constexpr int kMaxPairs = 4;   // d / 2 / 32 <= 2 for d <= 128 (4 for 256)
+    float m0[kMaxPairs], m1[kMaxPairs];
+#pragma unroll
+    for (int q = 0; q < kMaxPairs; q++) m0[q] = m1[q] = 0.f;
+    for (int t = a; t < b; t++) {
+        float nn = 0.f;
+#pragma unroll
+        for (int q = 0; q < kMaxPairs; q++) {
+            int i = lane + 32 * q;
+            if (i >= half) break;
+            float2 cs = A.rope[(size_t)t * half + i];
+            float x = to_f(K[(size_t)t * d + i]), y = to_f(K[(size_t)t * d + i + half]);
+            float kx = x * cs.x + y * cs.y, ky = y * cs.x - x * cs.y;
+            m0[q] += kx;
+            m1[q] += ky;
+            nn = fmaf(kx, kx, fmaf(ky, ky, nn));
+        }
+        nn = warp_sum(nn);
+        knorm += sqrt((double)nn);
+    }
+#pragma unroll
+    for (int q = 0; q < kMaxPairs; q++) {
+        int i = lane + 32 * q;
+        if (i >= half) break;
+        float u0 = m0[q] * ninv, u1 = m1[q] * ninv;
+        mu2 = fmaf(u0, u0, fmaf(u1, u1, mu2));
+        float2 cs = A.rope[(size_t)p * half + i];
+        store(Ko + i, u0 * cs.x - u1 * cs.y);
+        store(Ko + i + half, u0 * cs.y + u1 * cs.x);
+        float v0 = 0.f, v1 = 0.f;
+        for (int t = a; t < b; t++) {
+            float wt = R[t] + beta;
+            v0 = fmaf(wt, to_f(V[(size_t)t * d + i]), v0);
+            v1 = fmaf(wt, to_f(V[(size_t)t * d + i + half]), v1);
+        }
+        store(Vo + i, v0 * winv);
+        store(Vo + i + half, v1 * winv);
+    }
+    mu2 = warp_sum(mu2);
+    if (lane == 0) {
+        double coh = sqrt((double)mu2) / (knorm / n + A.eps);
+        double me = n * coh * coh;
+        me = me < 1.0 ? 1.0 : (me > n ? (double)n : me);
+        A.pos[e] = p;
+        A.log_m[e] = (float)log(me);
+        A.src_lo[e] = a;
+        A.src_hi[e] = b;
+    }
+}
+
+// Warp per unit: depth-first traversal of the executed splits, children in
+// ascending position, so frontier nodes come out in ascending position.
+template <typename Tin>
+__global__ void gather_units_kernel(GatherArgs A) {
+    __shared__ short stack[8][kMaxUnit + 4];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t nu = (int64_t)A.L * A.G * A.J;
+    const int64_t uid = (int64_t)blockIdx.x * 8 + warp;
+    if (uid >= nu || A.u_sel[uid] != 1) return;
+    const int lg = (int)(uid / A.J), j = (int)(uid - (int64_t)lg * A.J);
+    const int64_t nb = node_base(lg, A.slots[j], A.cs, A.Nc);
+    int64_t e = A.u_off[uid];
+    short *st = stack[warp];
+    int sp = 0;                      // stack owned by lane 0
+    if (lane == 0) st[sp++] = 0;
+    for (;;) {
+        int k = -1;
+        if (lane == 0) {
+            while (sp > 0) {
+                int x = st[--sp];
+                int64_t v = nb + x;
+                if (A.nd_sel[v] == 1) {
+                    int c0 = A.nd_child0[v], nc = A.nd_nchild[v];
+                    for (int q = nc - 1; q >= 0; q--) st[sp++] = (short)(c0 + q);   // leftmost on top
+                    continue;
+                }
+                k = x;
+                break;
+            }
+        }
+        k = __shfl_sync(0xffffffffu, k, 0);
+        if (k < 0) break;
+        emit_node<Tin>(A, lg, A.nd_a[nb + k], A.nd_b[nb + k], e, lane);
+        e++;
+    }
+}
+
+template <typename Tin>
+__global__ void gather_tokens_kernel(GatherArgs A) {
+    const int lg = blockIdx.y;
+    const int ntail = A.T - A.cend;
+    const int k = blockIdx.x * 8 + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (k >= A.cs + ntail) return;
+    int t;
+    int64_t e;
+    if (k < A.cs) { t = k; e = A.offsets[lg] + k; }
+    else { t = A.cend + (k - A.cs); e = A.offsets[lg + 1] - ntail + (k - A.cs); }
+    const Tin *K = static_cast<const Tin *>(A.K) + ((size_t)lg * A.T + t) * A.d;
+    const Tin *V = static_cast<const Tin *>(A.V) + ((size_t)lg * A.T + t) * A.d;
+    Tin *Ko = static_cast<Tin *>(A.K_out) + (size_t)e * A.d;
+    Tin *Vo = static_cast<Tin *>(A.V_out) + (size_t)e * A.d;
+    for (int i = lane; i < A.d; i += 32) { Ko[i] = K[i]; Vo[i] = V[i]; }
+    if (lane == 0) { A.pos[e] = t; A.log_m[e] = 0.f; A.src_lo[e] = t; A.src_hi[e] = t + 1; }
+}
+
+}  // namespace
+
+cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *slots, int J,
+                          void *K_out, void *V_out, int32_t *pos, float *log_m,
+                          int32_t *src_lo, int32_t *src_hi, int64_t *offsets, cudaStream_t s) {
+    GatherArgs A;
+    A.K = K; A.V = V; A.rtok = c.w.rtok; A.rope = c.w.rope; A.slots = slots;
+    A.nd_a = c.w.nd_a; A.nd_b = c.w.nd_b; A.nd_child0 = c.w.nd_child0; A.nd_nchild = c.w.nd_nchild;
+    A.nd_sel = c.w.nd_sel; A.u_sel = c.w.u_sel; A.u_nnodes = c.w.u_nnodes;
+    A.u_count = c.w.u_count; A.u_off = c.w.u_off;
+    A.L = c.p.L; A.G = c.p.G; A.T = c.p.T; A.d = c.p.d; A.J = J; A.cs = c.p.ctx_start;
+    A.cend = c.c_end; A.Nc = c.Nc; A.base_frac = c.p.base_frac; A.eps = c.p.eps;
+    A.K_out = K_out; A.V_out = V_out; A.pos = pos; A.log_m = log_m; A.src_lo = src_lo;
+    A.src_hi = src_hi; A.offsets = offsets;
+    const int64_t nu = (int64_t)c.p.L * c.p.G * J;
+    gather_count_kernel<<<(unsigned)((nu + 255) / 256), 256, 0, s>>>(A);
+    gather_scan_kernel<<<1, 1024, 0, s>>>(A);
+    const bool bf = c.p.dtype == GKV_BF16;
+    unsigned gu = (unsigned)((nu + 7) / 8);
+    if (gu) {
+        if (bf) gather_units_kernel<__nv_bfloat16><<<gu, 256, 0, s>>>(A);
+        else gather_units_kernel<float><<<gu, 256, 0, s>>>(A);
+    }
+    int ntok = c.p.ctx_start + (c.p.T - c.c_end);
+    if (ntok > 0) {
+        dim3 g((ntok + 7) / 8, c.p.L * c.p.G);
+        if (bf) gather_tokens_kernel<__nv_bfloat16><<<g, 256, 0, s>>>(A);
+        else gather_tokens_kernel<float><<<g, 256, 0, s>>>(A);
+    }
+    return cudaGetLastError();
+}
+
+}  // namespace gkv

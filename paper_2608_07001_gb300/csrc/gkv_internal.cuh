@@ -1,0 +1,154 @@
+// gkv_internal.cuh -- internal declarations shared by the CUDA translation
+// units of the GraceKV compression library (context, workspace, launchers,
+// small device helpers).  Not part of the public ABI (include/gracekv.h).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+#include <string>
+
+#include "../../include/gracekv.h"
+
+namespace gkv {
+
+constexpr int kMaxUnit = 128;      // longest slot a unit kernel holds in shared memory
+constexpr int kMaxSegLayers = 8;
+constexpr int kMaxWindows = 4;
+
+// ---------------------------------------------------------------------------
+// Workspace owned by a context.  All arrays are device memory.
+// ---------------------------------------------------------------------------
+struct Workspace {
+    // RoPE rotation table: (cos, sin)(t * theta_i) for t in [0, T), i < d/2.
+    float2 *rope = nullptr;
+    // segmentation
+    float *inv_norm = nullptr;     // [n_seg][T] 1 / max(||h_t||, eps)
+    float *nrm2 = nullptr;         // [n_seg][T] ||hbar_t||^2
+    double *klw = nullptr;         // [n_seg * n_win][T] curvature per (layer, window)
+    double *kappa = nullptr;       // [T] stabilised curvature
+    double *bscore = nullptr;      // [T] boundary score
+    double *zbuf = nullptr;        // [T] scratch for robust z
+    double *p2 = nullptr;          // [N_c + 1] prefix of sum_l ||d_t||^2
+    double *ew = nullptr;          // [(N_c + 1) * nb] DP edge weights (len n_min..n_max)
+    double *ewt = nullptr;         // [n_max + 1] terminal edge weights (len 1..n_max) at i = N_c
+    double *dpF = nullptr;         // [N_c + 1] DP values
+    int32_t *slots = nullptr;      // [N_c + 2] slot starts (absolute)
+    int32_t *dev_int = nullptr;    // [8] small device scalars (J, status, ...)
+    unsigned long long *sel_state = nullptr;   // radix-select state for the median
+    // row statistics and token values
+    float *row_m = nullptr, *row_Z = nullptr, *row_ZC = nullptr;  // [L*Hq*W]
+    float *rowp = nullptr;         // [3][L*Hq*W][n_chunks] pass-A partials
+    float *rtok = nullptr;         // [L*G*N_c]
+    // node records, indexed lg*2*N_c + 2*(slot start - c_s) + k
+    int32_t *nd_a = nullptr, *nd_b = nullptr, *nd_child0 = nullptr;
+    int32_t *nd_parent = nullptr;  // global index of the parent; roots: -2 - unit id
+    int32_t *nd_unit = nullptr;    // unit id lg * J + j
+    int8_t *nd_nchild = nullptr, *nd_cost = nullptr;
+    float *nd_D = nullptr, *nd_R = nullptr, *nd_U = nullptr, *nd_kappa = nullptr;
+    uint8_t *nd_sel = nullptr;     // split selected (1), discarded tie (2)
+    // per-unit arrays (capacity units_cap), unit id = lg * J + j
+    int64_t units_cap = 0;
+    int32_t *u_nnodes = nullptr;
+    float *u_Uadd = nullptr, *u_Ddrop = nullptr;
+    uint8_t *u_sel = nullptr;      // Add selected (1), discarded tie (2)
+    int32_t *u_count = nullptr;    // frontier entries per unit
+    int64_t *u_off = nullptr;      // entry offset of each unit's frontier
+    int32_t *u_list = nullptr;     // compacted unit ids (ties)
+    int32_t *u_blk = nullptr;      // per-block counts for compaction / scans
+    int64_t *u_blk64 = nullptr;
+    // allocation
+    unsigned long long *hist = nullptr;        // [2048] cost-weighted histogram
+    unsigned long long *alloc_state = nullptr; // see alloc.cu
+};
+
+struct Ctx {
+    gkv_params p;
+    int device = 0;
+    int num_sms = 148;
+    int32_t r = 0, Nc = 0, c_end = 0, nseg = 0, nwin = 0;
+    int32_t seg_layers[kMaxSegLayers];
+    int64_t B_free = 0;
+    int64_t used = 0;              // budget spent by the last allocation
+    int32_t J = 0;                 // slots of the last segmentation / build
+    int stage = 0;                 // 0 created, 1 segmented, 2 built, 3 allocated
+    gkv_status sticky = GKV_OK;
+    std::string err;
+    Workspace w;
+    int64_t node_cap = 0;          // L*G*2*N_c
+    int n_chunks = 0;              // pass-A chunks per row
+};
+
+// ---------------------------------------------------------------------------
+// Device helpers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float to_f(float x) { return x; }
+__device__ __forceinline__ float to_f(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+template <typename T> struct Vec8;   // 8 consecutive elements
+template <> struct Vec8<float> {
+    float v[8];
+    __device__ __forceinline__ void load(const float *p) {
+        float4 a = reinterpret_cast<const float4 *>(p)[0];
+        float4 b = reinterpret_cast<const float4 *>(p)[1];
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+        v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    }
+};
+template <> struct Vec8<__nv_bfloat16> {
+    float v[8];
+    __device__ __forceinline__ void load(const __nv_bfloat16 *p) {
+        uint4 u = reinterpret_cast<const uint4 *>(p)[0];
+        const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&u);
+#pragma unroll
+        for (int i = 0; i < 4; i++) {
+            float2 f = __bfloat1622float2(h[i]);
+            v[2 * i] = f.x;
+            v[2 * i + 1] = f.y;
+        }
+    }
+};
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ double warp_sum(double v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+
+// Monotone 32-bit key of a non-negative float (larger value -> larger key).
+__device__ __forceinline__ uint32_t fkey(float x) { return __float_as_uint(x); }
+
+// ---------------------------------------------------------------------------
+// Launchers (each returns the launch error, cudaSuccess otherwise)
+// ---------------------------------------------------------------------------
+cudaError_t launch_rope_table(Ctx &c, cudaStream_t s);
+
+cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
+                           const float *surprisal, float *kappa_out, cudaStream_t s);
+
+cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t s);
+cudaError_t launch_token_values(Ctx &c, const void *K, const void *Q, cudaStream_t s);
+cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *Q,
+                              const float *omega, const int32_t *slots, int J, cudaStream_t s);
+
+cudaError_t launch_allocate(Ctx &c, int J, cudaStream_t s);
+cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *slots, int J,
+                          void *K_out, void *V_out, int32_t *pos, float *log_m,
+                          int32_t *src_lo, int32_t *src_hi, int64_t *offsets, cudaStream_t s);
+
+// Node index base of slot j of (l, g).
+__host__ __device__ __forceinline__ int64_t node_base(int lg, int slot_start, int cs, int Nc) {
+    return (int64_t)lg * 2 * Nc + 2 * (int64_t)(slot_start - cs);
+}
+
+}  // namespace gkv

@@ -1,0 +1,273 @@
+// score.cu -- observation-query x key score passes of the GraceKV pass.
+//
+//   rope_table     (cos, sin)(t theta_i), theta_i = base^(-2i/d), built in fp64
+//                  (RoPE convention: half-split pairs (i, i + d/2)).
+//   row_stats      pass A: for every probe row r = (l, h, u) the max logit
+//                  m_r = max_t q.k_t / sqrt(d) over the visible range [0, T),
+//                  Z_r = sum_t exp(x - m_r) and Z^C_r = the same sum over the
+//                  compressible context C (App. A.3 max-logit shift; App. A.4
+//                  Eq. app_attention_probability denominators).
+//   token_values   pass B: s_t = sum_r exp(x_rt - m_r) / Z_r over the rows of
+//                  KV head g, shat_t = s_t / (sum_r Z^C_r / Z_r + eps) for t in C
+//                  (App. A.4 Eqs. app_direct_relevance, app_bottom_up_value with
+//                  lambda_graph = 0).
+//
+// Both passes contract a [rows x d] query block with [tokens x d] keys in
+// 64 x 64 tiles (FFMA, fp32 accumulation of the exact bf16/fp32 inputs).
+#include "gkv_internal.cuh"
+
+namespace gkv {
+namespace {
+
+__global__ void rope_table_kernel(int T, int d, double base, float2 *tab) {
+    int half = d / 2;
+    int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= (int64_t)T * half) return;
+    int t = (int)(e / half), i = (int)(e - (int64_t)t * half);
+    if (base == 0.0) {
+        tab[e] = make_float2(1.f, 0.f);
+        return;
+    }
+    double theta = pow(base, -2.0 * (double)i / (double)d);
+    double s, c;
+    sincos((double)t * theta, &s, &c);
+    tab[e] = make_float2((float)c, (float)s);
+}
+
+constexpr int kTR = 64;   // rows per tile
+constexpr int kTT = 64;   // tokens per tile
+constexpr int kKC = 32;   // head-dim chunk
+
+struct ScoreArgs {
+    int L, G, Hq, T, d, W, gq, Rg, cs, cend, Nc;
+    float inv_sqrt_d;
+};
+
+// Accumulate the 64 x 64 score tile of (rows rbase.., tokens tbase..) into
+// acc[i][j] (row ty + 16 i, token tx + 16 j); Qs / Ks are [kKC][64] staging.
+template <typename Tin>
+__device__ __forceinline__ void score_tile(const Tin *Qblk, const Tin *Kblk, int nrows, int ntok,
+                                           int d, float *Qs, float *Ks, float acc[4][4]) {
+    const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+#pragma unroll
+    for (int i = 0; i < 4; i++)
+#pragma unroll
+        for (int j = 0; j < 4; j++) acc[i][j] = 0.f;
+    for (int k0 = 0; k0 < d; k0 += kKC) {
+        __syncthreads();
+        for (int e = tid; e < kTR * kKC; e += 256) {
+            int r = e / kKC, k = e - r * kKC;
+            Qs[k * kTR + r] = (r < nrows && k0 + k < d) ? to_f(Qblk[(size_t)r * d + k0 + k]) : 0.f;
+            Ks[k * kTT + r] = (r < ntok && k0 + k < d) ? to_f(Kblk[(size_t)r * d + k0 + k]) : 0.f;
+        }
+        __syncthreads();
+#pragma unroll 8
+        for (int k = 0; k < kKC; k++) {
+            float q[4], kv[4];
+#pragma unroll
+            for (int i = 0; i < 4; i++) q[i] = Qs[k * kTR + ty + 16 * i];
+#pragma unroll
+            for (int j = 0; j < 4; j++) kv[j] = Ks[k * kTT + tx + 16 * j];
+#pragma unroll
+            for (int i = 0; i < 4; i++)
+#pragma unroll
+                for (int j = 0; j < 4; j++) acc[i][j] = fmaf(q[i], kv[j], acc[i][j]);
+        }
+    }
+}
+
+// Pass A.  grid = (token chunks, row tiles, L*G); writes per-chunk partials.
+template <typename Tin>
+__global__ void __launch_bounds__(256) row_stats_kernel(const Tin *K, const Tin *Q, ScoreArgs a,
+                                                        int chunk, int nchunks, float *part) {
+    __shared__ float Qs[kKC * kTR], Ks[kKC * kTT];
+    const int lg = blockIdx.z, l = lg / a.G, g = lg - l * a.G;
+    const int r0 = blockIdx.y * kTR;
+    const int t_begin = blockIdx.x * chunk, t_end = min(a.T, t_begin + chunk);
+    const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+    const Tin *Qblk = Q + ((size_t)(l * a.Hq + g * a.gq) * a.W + r0) * a.d;
+    const Tin *Kl = K + (size_t)lg * a.T * a.d;
+    const int nrows = min(kTR, a.Rg - r0);
+    float m[4], z[4], zc[4];
+#pragma unroll
+    for (int i = 0; i < 4; i++) { m[i] = -INFINITY; z[i] = 0.f; zc[i] = 0.f; }
+    for (int t0 = t_begin; t0 < t_end; t0 += kTT) {
+        int ntok = min(kTT, t_end - t0);
+        float acc[4][4];
+        score_tile(Qblk, Kl + (size_t)t0 * a.d, nrows, ntok, a.d, Qs, Ks, acc);
+#pragma unroll
+        for (int i = 0; i < 4; i++) {
+            float x[4], tm = -INFINITY;
+#pragma unroll
+            for (int j = 0; j < 4; j++) {
+                x[j] = (tx + 16 * j < ntok) ? acc[i][j] * a.inv_sqrt_d : -INFINITY;
+                tm = fmaxf(tm, x[j]);
+            }
+#pragma unroll
+            for (int o = 1; o < 16; o <<= 1) tm = fmaxf(tm, __shfl_xor_sync(0xffffffffu, tm, o));
+            float nm = fmaxf(m[i], tm);
+            float sz = 0.f, szc = 0.f;
+#pragma unroll
+            for (int j = 0; j < 4; j++) {
+                int t = t0 + tx + 16 * j;
+                if (tx + 16 * j < ntok) {
+                    float e = expf(x[j] - nm);
+                    sz += e;
+                    if (t >= a.cs && t < a.cend) szc += e;
+                }
+            }
+#pragma unroll
+            for (int o = 1; o < 16; o <<= 1) {
+                sz += __shfl_xor_sync(0xffffffffu, sz, o);
+                szc += __shfl_xor_sync(0xffffffffu, szc, o);
+            }
+            float sc = (m[i] == -INFINITY) ? 0.f : expf(m[i] - nm);
+            z[i] = z[i] * sc + sz;
+            zc[i] = zc[i] * sc + szc;
+            m[i] = nm;
+        }
+    }
+    if (tx == 0) {
+        const int nrow_all = a.L * a.Hq * a.W;
+#pragma unroll
+        for (int i = 0; i < 4; i++) {
+            int r = ty + 16 * i;
+            if (r >= nrows) continue;
+            size_t row = (size_t)(l * a.Hq + g * a.gq) * a.W + r0 + r;   // index into [L][Hq][W]
+            part[((size_t)0 * nrow_all + row) * nchunks + blockIdx.x] = m[i];
+            part[((size_t)1 * nrow_all + row) * nchunks + blockIdx.x] = z[i];
+            part[((size_t)2 * nrow_all + row) * nchunks + blockIdx.x] = zc[i];
+        }
+    }
+}
+
+__global__ void row_combine_kernel(const float *part, int nrow, int nchunks, float *rm, float *rz,
+                                   float *rzc, int *status) {
+    int row = blockIdx.x * blockDim.x + threadIdx.x;
+    if (row >= nrow) return;
+    const float *pm = part + (size_t)row * nchunks;
+    const float *pz = part + ((size_t)nrow + row) * nchunks;
+    const float *pc = part + ((size_t)2 * nrow + row) * nchunks;
+    float M = -INFINITY;
+    for (int c = 0; c < nchunks; c++) M = fmaxf(M, pm[c]);
+    double Z = 0.0, ZC = 0.0;
+    for (int c = 0; c < nchunks; c++) {
+        if (pm[c] == -INFINITY) continue;
+        double s = exp((double)pm[c] - (double)M);
+        Z += pz[c] * s;
+        ZC += pc[c] * s;
+    }
+    if (!isfinite(M) || !isfinite(Z)) atomicOr(status, 2);
+    rm[row] = M;
+    rz[row] = (float)Z;
+    rzc[row] = (float)ZC;
+}
+
+// Pass B.  grid = (token tiles over C, L*G).  Loops over the row tiles of the
+// KV head, accumulating s_t for the 64 tokens of the tile.
+template <typename Tin>
+__global__ void __launch_bounds__(256) token_values_kernel(const Tin *K, const Tin *Q, ScoreArgs a,
+                                                           const float *rm, const float *rz,
+                                                           const float *rzc, float eps,
+                                                           float *rtok) {
+    __shared__ float Qs[kKC * kTR], Ks[kKC * kTT];
+    __shared__ float colpart[16][kTT];
+    __shared__ float rowm[kTR], rowiz[kTR];
+    __shared__ double scale_s;
+    const int lg = blockIdx.y, l = lg / a.G, g = lg - l * a.G;
+    const int t0 = a.cs + blockIdx.x * kTT;
+    const int ntok = min(kTT, a.cend - t0);
+    const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+    const size_t rowbase = (size_t)(l * a.Hq + g * a.gq) * a.W;
+    if (tid < 32) {
+        double s = 0.0;
+        for (int r = tid; r < a.Rg; r += 32) s += (double)rzc[rowbase + r] / (double)rz[rowbase + r];
+        s = warp_sum(s);
+        if (tid == 0) scale_s = 1.0 / (s + (double)eps);
+    }
+    float s_tok[4] = {0.f, 0.f, 0.f, 0.f};
+    const Tin *Kl = K + ((size_t)lg * a.T + t0) * a.d;
+    for (int r0 = 0; r0 < a.Rg; r0 += kTR) {
+        int nrows = min(kTR, a.Rg - r0);
+        __syncthreads();
+        if (tid < kTR) {
+            bool ok = tid < nrows;
+            rowm[tid] = ok ? rm[rowbase + r0 + tid] : 0.f;
+            rowiz[tid] = ok ? 1.0f / rz[rowbase + r0 + tid] : 0.f;
+        }
+        float acc[4][4];
+        score_tile(Q + (rowbase + r0) * a.d, Kl, nrows, ntok, a.d, Qs, Ks, acc);
+#pragma unroll
+        for (int i = 0; i < 4; i++) {
+            int r = ty + 16 * i;
+            if (r >= nrows) continue;
+#pragma unroll
+            for (int j = 0; j < 4; j++)
+                s_tok[j] += expf(acc[i][j] * a.inv_sqrt_d - rowm[r]) * rowiz[r];
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < 4; j++) colpart[ty][tx + 16 * j] = s_tok[j];
+    __syncthreads();
+    if (tid < ntok) {
+        float s = 0.f;
+        for (int q = 0; q < 16; q++) s += colpart[q][tid];
+        rtok[(size_t)lg * a.Nc + (t0 - a.cs) + tid] = (float)((double)s * scale_s);
+    }
+}
+
+ScoreArgs make_args(const Ctx &c) {
+    ScoreArgs a;
+    a.L = c.p.L; a.G = c.p.G; a.Hq = c.p.Hq; a.T = c.p.T; a.d = c.p.d; a.W = c.p.W;
+    a.gq = c.p.Hq / c.p.G;
+    a.Rg = a.gq * a.W;
+    a.cs = c.p.ctx_start;
+    a.cend = c.c_end;
+    a.Nc = c.Nc;
+    a.inv_sqrt_d = (float)(1.0 / sqrt((double)c.p.d));
+    return a;
+}
+
+}  // namespace
+
+cudaError_t launch_rope_table(Ctx &c, cudaStream_t s) {
+    int64_t n = (int64_t)c.p.T * (c.p.d / 2);
+    rope_table_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(c.p.T, c.p.d, c.p.rope_base, c.w.rope);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t s) {
+    ScoreArgs a = make_args(c);
+    int chunk = (c.p.T + c.n_chunks - 1) / c.n_chunks;
+    chunk = (chunk + kTT - 1) / kTT * kTT;
+    dim3 grid(c.n_chunks, (a.Rg + kTR - 1) / kTR, a.L * a.G);
+    if (c.p.dtype == GKV_BF16)
+        row_stats_kernel<<<grid, 256, 0, s>>>(static_cast<const __nv_bfloat16 *>(K),
+                                              static_cast<const __nv_bfloat16 *>(Q), a, chunk,
+                                              c.n_chunks, c.w.rowp);
+    else
+        row_stats_kernel<<<grid, 256, 0, s>>>(static_cast<const float *>(K),
+                                              static_cast<const float *>(Q), a, chunk, c.n_chunks,
+                                              c.w.rowp);
+    int nrow = a.L * a.Hq * a.W;
+    row_combine_kernel<<<(nrow + 255) / 256, 256, 0, s>>>(c.w.rowp, nrow, c.n_chunks, c.w.row_m,
+                                                          c.w.row_Z, c.w.row_ZC, c.w.dev_int + 1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_token_values(Ctx &c, const void *K, const void *Q, cudaStream_t s) {
+    ScoreArgs a = make_args(c);
+    dim3 grid((c.Nc + kTT - 1) / kTT, a.L * a.G);
+    float eps = (float)c.p.eps;
+    if (c.p.dtype == GKV_BF16)
+        token_values_kernel<<<grid, 256, 0, s>>>(static_cast<const __nv_bfloat16 *>(K),
+                                                 static_cast<const __nv_bfloat16 *>(Q), a,
+                                                 c.w.row_m, c.w.row_Z, c.w.row_ZC, eps, c.w.rtok);
+    else
+        token_values_kernel<<<grid, 256, 0, s>>>(static_cast<const float *>(K),
+                                                 static_cast<const float *>(Q), a, c.w.row_m,
+                                                 c.w.row_Z, c.w.row_ZC, eps, c.w.rtok);
+    return cudaGetLastError();
+}
+
+}  // namespace gkv

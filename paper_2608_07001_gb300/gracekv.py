@@ -1,0 +1,259 @@
+"""Python binding of the GraceKV compression library (include/gracekv.h).
+
+Argument marshalling only: every step of the compression pass runs in the
+CUDA kernels of libgracekv.so.  Tensors are torch CUDA tensors (device
+memory); calls are enqueued on the current torch stream.  There is no CPU
+fallback: importing this module fails if the library is missing.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import dataclasses
+import os
+from typing import Optional
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIBPATH = os.path.join(_HERE, "libgracekv.so")
+
+GKV_OK, GKV_EINVAL, GKV_EBUDGET, GKV_ENOMEM, GKV_ECUDA, GKV_ETIMEOUT = 0, 1, 2, 3, 4, 5
+GKV_ENONFINITE, GKV_ESTATE, GKV_EUNSUPPORTED, GKV_ECAPACITY = 6, 7, 8, 9
+GKV_F32, GKV_BF16 = 0, 1
+
+
+class GkvParams(C.Structure):
+    _fields_ = [
+        ("L", C.c_int32), ("G", C.c_int32), ("Hq", C.c_int32), ("T", C.c_int32),
+        ("d", C.c_int32), ("W", C.c_int32), ("dtype", C.c_int32),
+        ("ctx_start", C.c_int32), ("ctx_end", C.c_int32), ("recent", C.c_int32),
+        ("budget", C.c_int64), ("rope_base", C.c_double),
+        ("n_min", C.c_int32), ("n_max", C.c_int32), ("n0", C.c_int32),
+        ("lambda_stab", C.c_double), ("lambda_s", C.c_double), ("lambda_d", C.c_double),
+        ("lambda_n", C.c_double), ("c_cut", C.c_double),
+        ("seg_layers", C.c_int32 * 8), ("n_seg_layers", C.c_int32),
+        ("windows", C.c_int32 * 4), ("n_windows", C.c_int32),
+        ("k_cand", C.c_int32),
+        ("lambda_kappa", C.c_double), ("lambda_Z", C.c_double), ("lambda_M", C.c_double),
+        ("eps", C.c_double), ("base_frac", C.c_double),
+        ("lambda_graph", C.c_double), ("alpha_floor", C.c_double),
+    ]
+
+
+class GraceKVError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"gracekv status {status}: {msg}")
+        self.status = status
+
+
+_lib = None
+
+EXPORTED = ["gracekv_default_params", "gracekv_budget_for_ratio", "gracekv_create",
+            "gracekv_destroy", "gracekv_last_error", "gracekv_status_string", "gracekv_query",
+            "gracekv_segment", "gracekv_build_trees", "gracekv_allocate", "gracekv_gather",
+            "gracekv_export"]
+
+
+def lib() -> C.CDLL:
+    """Load libgracekv.so (built by __graft_entry__.build()); raises if absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIBPATH):
+        raise ImportError(f"{LIBPATH} is missing: build it with __graft_entry__.build()")
+    L = C.CDLL(LIBPATH)
+    vp, i32, i64 = C.c_void_p, C.c_int32, C.c_int64
+    L.gracekv_default_params.argtypes = [C.POINTER(GkvParams)]
+    L.gracekv_budget_for_ratio.argtypes = [i32, i32, i32, C.c_double]
+    L.gracekv_budget_for_ratio.restype = i64
+    L.gracekv_create.argtypes = [C.POINTER(GkvParams), C.POINTER(vp)]
+    L.gracekv_destroy.argtypes = [vp]
+    L.gracekv_destroy.restype = None
+    L.gracekv_last_error.argtypes = [vp]
+    L.gracekv_last_error.restype = C.c_char_p
+    L.gracekv_status_string.argtypes = [C.c_int]
+    L.gracekv_status_string.restype = C.c_char_p
+    L.gracekv_query.argtypes = [vp, C.POINTER(i32), C.POINTER(i32), C.POINTER(i64), C.POINTER(i32)]
+    L.gracekv_segment.argtypes = [vp, vp, vp, i32, vp, vp, i32, C.POINTER(i32), vp, vp]
+    L.gracekv_build_trees.argtypes = [vp, vp, vp, vp, vp, vp, i32, vp]
+    L.gracekv_allocate.argtypes = [vp, C.POINTER(i64), vp]
+    L.gracekv_gather.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, i64, vp]
+    L.gracekv_export.argtypes = [vp, i64, C.POINTER(i64)] + [vp] * 18 + [vp]
+    _lib = L
+    return L
+
+
+def gracekv_default_params() -> GkvParams:
+    p = GkvParams()
+    lib().gracekv_default_params(C.byref(p))
+    return p
+
+
+def gracekv_budget_for_ratio(L: int, G: int, n_ctx: int, x: float) -> int:
+    return int(lib().gracekv_budget_for_ratio(L, G, n_ctx, float(x)))
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if not t.is_cuda or not t.is_contiguous():
+        raise ValueError("tensors must be contiguous CUDA tensors")
+    return C.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return C.c_void_p(s.cuda_stream)
+
+
+def make_params(L, G, Hq, T, d, W, *, dtype, budget, rope_base, ctx_start=0, ctx_end=None,
+                **overrides) -> GkvParams:
+    p = gracekv_default_params()
+    p.L, p.G, p.Hq, p.T, p.d, p.W = L, G, Hq, T, d, W
+    p.dtype = GKV_BF16 if dtype in (torch.bfloat16, "bf16") else GKV_F32
+    p.ctx_start = ctx_start
+    p.ctx_end = T if ctx_end is None else ctx_end
+    p.budget = int(budget)
+    p.rope_base = float(rope_base)
+    for k, v in overrides.items():
+        if k == "windows":
+            for i, w in enumerate(v):
+                p.windows[i] = w
+            p.n_windows = len(v)
+        elif k == "seg_layers":
+            for i, w in enumerate(v):
+                p.seg_layers[i] = w
+            p.n_seg_layers = len(v)
+        else:
+            setattr(p, k, v)
+    return p
+
+
+class Context:
+    """Owns a gracekv_ctx; the four stage calls follow the C ABI one to one."""
+
+    def __init__(self, params: GkvParams):
+        self.params = params
+        h = C.c_void_p()
+        st = lib().gracekv_create(C.byref(params), C.byref(h))
+        if st != GKV_OK:
+            raise GraceKVError(st, lib().gracekv_status_string(st).decode())
+        self.h = h
+        r, nc, bf, js = C.c_int32(), C.c_int32(), C.c_int64(), C.c_int32()
+        lib().gracekv_query(self.h, C.byref(r), C.byref(nc), C.byref(bf), C.byref(js))
+        self.recent, self.n_c, self.b_free = r.value, nc.value, bf.value
+
+    def close(self):
+        if getattr(self, "h", None):
+            lib().gracekv_destroy(self.h)
+            self.h = None
+
+    __del__ = close
+
+    def _check(self, st: int):
+        if st != GKV_OK:
+            msg = lib().gracekv_last_error(self.h).decode()
+            raise GraceKVError(st, msg or lib().gracekv_status_string(st).decode())
+
+    def gracekv_segment(self, V, slot_starts, hidden=None, surprisal=None, kappa=None, stream=None) -> int:
+        n = C.c_int32()
+        Dh = 0 if hidden is None else hidden.shape[-1]
+        self._check(lib().gracekv_segment(self.h, _ptr(V), _ptr(hidden), Dh, _ptr(surprisal),
+                                          _ptr(slot_starts), slot_starts.numel() - 1, C.byref(n),
+                                          _ptr(kappa), _stream(stream)))
+        return n.value
+
+    def gracekv_build_trees(self, K, V, Q, omega=None, slot_starts=None, n_slots=0, stream=None):
+        self._check(lib().gracekv_build_trees(self.h, _ptr(K), _ptr(V), _ptr(Q), _ptr(omega),
+                                              _ptr(slot_starts), n_slots, _stream(stream)))
+
+    def gracekv_allocate(self, stream=None) -> int:
+        n = C.c_int64()
+        self._check(lib().gracekv_allocate(self.h, C.byref(n), _stream(stream)))
+        return n.value
+
+    def gracekv_gather(self, K, V, out: "Cache", stream=None):
+        self._check(lib().gracekv_gather(self.h, _ptr(K), _ptr(V), _ptr(out.K), _ptr(out.V),
+                                         _ptr(out.pos), _ptr(out.log_m), _ptr(out.src_lo),
+                                         _ptr(out.src_hi), _ptr(out.offsets), out.K.shape[0],
+                                         _stream(stream)))
+
+    def gracekv_export(self, node_cap: Optional[int] = None, stream=None) -> dict:
+        """Host copy of the trees and selection (introspection for tests)."""
+        import numpy as np
+        p = self.params
+        js = C.c_int32()
+        lib().gracekv_query(self.h, None, None, None, C.byref(js))
+        J = js.value
+        nu = p.L * p.G * J
+        cap = node_cap or p.L * p.G * 2 * self.n_c
+        nrow = p.L * p.Hq * p.W
+        arr = dict(unit_first=np.zeros(nu + 1, np.int64), unit_Uadd=np.zeros(nu, np.float32),
+                   unit_Ddrop=np.zeros(nu, np.float32), add_sel=np.zeros(nu, np.uint8),
+                   a=np.zeros(cap, np.int32), b=np.zeros(cap, np.int32),
+                   child0=np.zeros(cap, np.int32), nchild=np.zeros(cap, np.int32),
+                   cost=np.zeros(cap, np.int32), D=np.zeros(cap, np.float32),
+                   R=np.zeros(cap, np.float32), U=np.zeros(cap, np.float32),
+                   kappa=np.zeros(cap, np.float32), split_sel=np.zeros(cap, np.uint8),
+                   row_m=np.zeros(nrow, np.float32), row_Z=np.zeros(nrow, np.float32),
+                   row_ZC=np.zeros(nrow, np.float32), rtok=np.zeros(p.L * p.G * self.n_c, np.float32))
+        order = ["unit_first", "unit_Uadd", "unit_Ddrop", "add_sel", "a", "b", "child0", "nchild",
+                 "cost", "D", "R", "U", "kappa", "split_sel", "row_m", "row_Z", "row_ZC", "rtok"]
+        nn = C.c_int64()
+        self._check(lib().gracekv_export(self.h, cap, C.byref(nn),
+                                         *[C.c_void_p(arr[k].ctypes.data) for k in order],
+                                         _stream(stream)))
+        n = nn.value
+        for k in ["a", "b", "child0", "nchild", "cost", "D", "R", "U", "kappa", "split_sel"]:
+            arr[k] = arr[k][:n]
+        arr["J"] = J
+        return arr
+
+
+@dataclasses.dataclass
+class Cache:
+    """Ragged compressed cache (device tensors, capacity rows)."""
+    K: torch.Tensor
+    V: torch.Tensor
+    pos: torch.Tensor
+    log_m: torch.Tensor
+    src_lo: torch.Tensor
+    src_hi: torch.Tensor
+    offsets: torch.Tensor
+
+    @staticmethod
+    def empty(cap: int, d: int, LG: int, dtype, device="cuda") -> "Cache":
+        i32 = dict(dtype=torch.int32, device=device)
+        return Cache(torch.empty(cap, d, dtype=dtype, device=device),
+                     torch.empty(cap, d, dtype=dtype, device=device),
+                     torch.empty(cap, **i32), torch.empty(cap, dtype=torch.float32, device=device),
+                     torch.empty(cap, **i32), torch.empty(cap, **i32),
+                     torch.empty(LG + 1, dtype=torch.int64, device=device))
+
+
+class Compressor:
+    """Runs the four stages on one context with preallocated outputs."""
+
+    def __init__(self, params: GkvParams, device="cuda"):
+        self.ctx = Context(params)
+        p = params
+        self.params = p
+        dt = torch.bfloat16 if p.dtype == GKV_BF16 else torch.float32
+        self.slots = torch.empty(self.ctx.n_c + 2, dtype=torch.int32, device=device)
+        self.kappa = torch.empty(p.T, dtype=torch.float32, device=device)
+        cap = p.budget + p.L * p.G * (p.T - (p.ctx_end - p.ctx_start)) + 8
+        self.cache = Cache.empty(cap, p.d, p.L * p.G, dt, device)
+        self.n_slots = 0
+        self.n_entries = 0
+
+    def __call__(self, K, V, Q, omega=None, hidden=None, surprisal=None, slot_starts=None,
+                 stream=None) -> "Cache":
+        c = self.ctx
+        self.n_slots = c.gracekv_segment(V, self.slots, hidden, surprisal, self.kappa, stream)
+        if slot_starts is not None:
+            c.gracekv_build_trees(K, V, Q, omega, slot_starts, slot_starts.numel() - 1, stream)
+        else:
+            c.gracekv_build_trees(K, V, Q, omega, None, 0, stream)
+        self.n_entries = c.gracekv_allocate(stream)
+        c.gracekv_gather(K, V, self.cache, stream)
+        return self.cache

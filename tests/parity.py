@@ -1,0 +1,213 @@
+"""GPU-vs-oracle comparison helpers (test infrastructure).
+
+run_gpu runs the four C-ABI stages on the device; run_oracle runs the CPU
+oracle on the same inputs; compare() checks, stage by stage:
+
+  slot starts          bit-exact (or a DP near-tie on the oracle's path)
+  curvature            |kappa_gpu - kappa_oracle| <= KAPPA_ATOL
+  row stats / values   relative tolerances ROW_RTOL / RTOK_RTOL
+  tree topology        exact per unit; a differing refinement decision is
+                       allowed only where the oracle's margin at that node is
+                       below NEAR_TIE (1e-6 relative) -- the unit is then
+                       excluded from the remaining checks and counted
+  D, U                 relative to the magnitude of the terms they are
+                       formed from (D_RTOL, U_RTOL)
+  selection            exact for units with identical trees, except ops whose
+                       oracle key is within NEAR_TIE of the threshold (counted)
+  cache                positions / intervals / offsets exact; single tokens
+                       bit-exact; prototypes within PROTO_RTOL[dtype]
+                       (vector-relative), log m within LOGM_ATOL
+
+Tolerances follow from fp32 arithmetic on exact bf16/fp32 inputs: logits
+and window sums carry ~1e-6 relative rounding, which bounds curvature,
+statistics and prototype errors; the distortion D is a ratio of squared
+differences and is compared at 1e-3 relative to its own magnitude.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle as O
+from paper_2608_07001_gb300 import gracekv as gk
+
+NEAR_TIE = 1e-6
+KAPPA_ATOL = 2e-5
+ROW_RTOL = 2e-5
+RTOK_RTOL = 1e-4
+D_RTOL = 1e-3
+U_RTOL = 1e-3
+PROTO_RTOL = {torch.float32: 1e-5, torch.bfloat16: 2e-2}
+LOGM_ATOL = 1e-4
+
+
+def run_gpu(K, V, Q, B, rope_base, *, ctx_start=0, ctx_end=None, omega=None, hidden=None,
+            surprisal=None, slot_starts=None, **ov):
+    L, G, T, d = K.shape
+    Hq, W = Q.shape[1], Q.shape[2]
+    p = gk.make_params(L, G, Hq, T, d, W, dtype=K.dtype, budget=B, rope_base=rope_base,
+                       ctx_start=ctx_start, ctx_end=ctx_end, **ov)
+    comp = gk.Compressor(p)
+    dev = lambda t: None if t is None else torch.as_tensor(t).cuda().contiguous()
+    Kc, Vc, Qc = dev(K), dev(V), dev(Q)
+    om = None if omega is None else dev(torch.as_tensor(omega, dtype=torch.float32))
+    hid = None if hidden is None else dev(torch.as_tensor(hidden, dtype=torch.float32))
+    sur = None if surprisal is None else dev(torch.as_tensor(surprisal, dtype=torch.float32))
+    ss = None
+    if slot_starts is not None:
+        ss = dev(torch.as_tensor(np.asarray(slot_starts) + ctx_start, dtype=torch.int32))
+    cache = comp(Kc, Vc, Qc, omega=om, hidden=hid, surprisal=sur, slot_starts=ss)
+    torch.cuda.synchronize()
+    ex = comp.ctx.gracekv_export()
+    E = comp.n_entries
+    c = {k: getattr(cache, k)[:E].cpu() for k in ("K", "V", "pos", "log_m", "src_lo", "src_hi")}
+    c["offsets"] = cache.offsets.cpu().numpy()
+    J = ex["J"]
+    slots = (ss.cpu().numpy() if ss is not None else comp.slots[:comp.n_slots + 1].cpu().numpy())
+    return dict(comp=comp, slots=slots, seg_slots=comp.slots[:comp.n_slots + 1].cpu().numpy(),
+                kappa=comp.kappa.cpu().numpy(), export=ex, cache=c, E=E, J=J,
+                recent=comp.ctx.recent, b_free=comp.ctx.b_free)
+
+
+def run_oracle(K, V, Q, B, rope_base, *, ctx_start=0, ctx_end=None, omega=None, hidden=None,
+               surprisal=None, slot_starts=None, **ov):
+    return O.run(K, V, Q, B, rope_base, ctx_start=ctx_start, ctx_end=ctx_end, omega=omega,
+                 hidden=hidden, surprisal=surprisal, slot_starts=slot_starts, **ov)
+
+
+def oracle_tau(o):
+    """Cost-weighted threshold of the oracle's bottleneck keys (fp64)."""
+    tr = o["trees"]
+    nd = tr.nodes
+    keys = np.concatenate([tr.unit_Uadd, nd["kappa"][nd["cost"] > 0]])
+    cost = np.concatenate([np.ones(len(tr.unit_Uadd)), nd["cost"][nd["cost"] > 0]])
+    order = np.argsort(-keys, kind="stable")
+    cum = np.cumsum(cost[order])
+    B = o["B_free"]
+    if cum[-1] <= B:
+        return -np.inf
+    k = np.searchsorted(cum, B, side="right")
+    return keys[order][k]
+
+
+def compare(g, o, dtype, report=None, require_exact_selection=True):
+    rep = {} if report is None else report
+    # -------- segmentation --------------------------------------------------
+    og = o["seg"]["slot_starts"]
+    rep["kappa_maxerr"] = float(np.max(np.abs(g["kappa"] - o["seg"]["kappa"])))
+    assert rep["kappa_maxerr"] <= KAPPA_ATOL, rep["kappa_maxerr"]
+    if o["seg"]["dp_best"] is not None:
+        same = np.array_equal(g["seg_slots"], og)
+        if not same:
+            best, second = o["seg"]["dp_best"], o["seg"]["dp_second"]
+            ends = og[1:] - og[0]
+            m = np.abs(best[ends] - second[ends]) / np.maximum(np.abs(best[ends]), 1e-300)
+            rep["dp_near_tie"] = float(m.min())
+            assert m.min() < NEAR_TIE, f"slot starts differ without an oracle near-tie (min margin {m.min():.3e})"
+            return rep
+    assert np.array_equal(g["slots"], og), "slots used by the trees differ"
+    # -------- row statistics and token values --------------------------------
+    ex = g["export"]
+    for k, ok in (("row_m", "m"), ("row_Z", "Z"), ("row_ZC", "ZC")):
+        a, b = ex[k], o[ok].reshape(-1)
+        err = np.abs(a - b) / np.maximum(np.abs(b), 1e-30 if k != "row_m" else 1.0)
+        rep[k + "_relerr"] = float(err.max())
+        assert err.max() <= ROW_RTOL * (1 if k == "row_m" else 10), (k, err.max())
+    rt = o["rtok"].reshape(-1)
+    err = np.abs(ex["rtok"] - rt) / np.maximum(np.abs(rt), 1e-3 * rt.max())
+    rep["rtok_relerr"] = float(err.max())
+    assert err.max() <= RTOK_RTOL, err.max()
+    # -------- trees ---------------------------------------------------------
+    tr = o["trees"]
+    ond = tr.nodes
+    roots = list(tr.unit_root) + [len(ond["a"])]
+    uf = ex["unit_first"]
+    nu = len(tr.unit_root)
+    assert len(uf) == nu + 1
+    excluded = set()
+    worst_D = worst_U = 0.0
+    for u in range(nu):
+        gs, ge = uf[u], uf[u + 1]
+        os_, oe = roots[u], roots[u + 1]
+        ga, gb, gn = ex["a"][gs:ge], ex["b"][gs:ge], ex["nchild"][gs:ge]
+        oa, ob, on = ond["a"][os_:oe], ond["b"][os_:oe], ond["nchild"][os_:oe]
+        if not (len(ga) == len(oa) and np.array_equal(ga, oa) and np.array_equal(gb, ob)
+                and np.array_equal(gn, on)):
+            # first node whose children differ: its decision margins decide
+            k = 0
+            n = min(len(ga), len(oa))
+            while k < n and ga[k] == oa[k] and gb[k] == ob[k]:
+                gc = ex["child0"][gs + k]
+                oc = ond["child0"][os_ + k] - os_
+                if gn[k] != on[k] or (gn[k] and (not np.array_equal(
+                        ga[gc:gc + gn[k]], oa[oc:oc + on[k]]) or not np.array_equal(
+                        gb[gc:gc + gn[k]], ob[oc:oc + on[k]]))):
+                    break
+                k += 1
+            v = os_ + k
+            margin = min(ond["m_cut"][v], ond["m_form"][v], ond["m_topk"][v], ond["m_ext"][v])
+            assert margin < NEAR_TIE, (f"unit {u}: tree differs at node [{oa[k]},{ob[k]}) "
+                                       f"without a near-tie (oracle margin {margin:.3e})")
+            excluded.add(u)
+            continue
+        oD, gD = ond["D"][os_:oe], ex["D"][gs:ge]
+        eD = np.abs(gD - oD) / np.maximum(np.abs(oD), 1e-30)
+        eD[oD == 0] = np.abs(gD[oD == 0])
+        worst_D = max(worst_D, float(eD.max()))
+        scale = np.maximum(ond["R"][os_:oe] * np.maximum(np.abs(oD), 1e-300), 1e-300)
+        # U is relative to R * max(D(v), sum D(children)) / cost
+        oU = ond["U"][os_:oe]
+        cst = np.maximum(ond["cost"][os_:oe], 1)
+        eU = np.abs(ex["U"][gs:ge] - oU) / (scale / cst)
+        worst_U = max(worst_U, float(eU.max()))
+    rep["units"] = nu
+    rep["units_excluded_near_tie"] = len(excluded)
+    rep["D_relerr"] = worst_D
+    rep["U_relerr"] = worst_U
+    assert worst_D <= D_RTOL, worst_D
+    assert worst_U <= U_RTOL, worst_U
+    # -------- selection -----------------------------------------------------
+    tau = oracle_tau(o)
+    mism = exempt = 0
+    for u in range(nu):
+        if u in excluded:
+            continue
+        gs, os_ = uf[u], roots[u]
+        n = uf[u + 1] - gs
+        if int(ex["add_sel"][u] == 1) != int(o["add_sel"][u]):
+            mism += 1
+            if abs(tr.unit_Uadd[u] - tau) <= NEAR_TIE * max(abs(tau), 1e-300):
+                exempt += 1
+        gsel = (ex["split_sel"][gs:gs + n] == 1).astype(int)
+        osel = o["split_sel"][os_:os_ + n].astype(int)
+        for k in np.nonzero(gsel != osel)[0]:
+            mism += 1
+            v = os_ + k
+            if abs(ond["kappa"][v] - tau) <= NEAR_TIE * max(ond["kscale"][v], abs(tau), 1e-300):
+                exempt += 1
+    rep["selection_mismatch"] = mism
+    rep["selection_exempt"] = exempt
+    if require_exact_selection:
+        assert mism == 0 or (mism - exempt) <= 1, rep   # one endgame op may follow an exempt flip
+    if mism or excluded:
+        return rep
+    # -------- cache ----------------------------------------------------------
+    oc, gc = o["cache"], g["cache"]
+    assert g["E"] == len(oc["pos"])
+    assert np.array_equal(gc["offsets"], oc["offsets"])
+    for k in ("pos", "src_lo", "src_hi"):
+        assert np.array_equal(gc[k].numpy(), oc[k]), k
+    single = (oc["src_hi"] - oc["src_lo"]) == 1
+    for k in ("K", "V"):
+        gv = gc[k].double().numpy()
+        assert np.array_equal(gv[single], oc[k][single]), f"single-token {k} not bit-exact"
+        if (~single).any():
+            rel = (np.linalg.norm(gv[~single] - oc[k][~single], axis=1)
+                   / np.maximum(np.linalg.norm(oc[k][~single], axis=1), 1e-30))
+            rep[f"proto_{k}_relerr"] = float(rel.max())
+            assert rel.max() <= PROTO_RTOL[dtype], (k, rel.max())
+    lm = np.abs(gc["log_m"].double().numpy() - oc["log_m"])
+    rep["logm_abserr"] = float(lm.max())
+    assert lm.max() <= LOGM_ATOL
+    assert np.all(gc["log_m"].numpy()[single] == 0.0)
+    return rep

@@ -1,0 +1,153 @@
+"""CUDA path vs CPU oracle on seeded inputs (through the C ABI)."""
+import json
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2608_07001_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    import __graft_entry__ as g
+    g.build()
+    assert torch.cuda.is_available()
+
+
+def _run(inp_K, inp_V, inp_Q, B, base, **kw):
+    from tests import parity as P
+    g = P.run_gpu(inp_K, inp_V, inp_Q, B, base, **kw)
+    o = P.run_oracle(inp_K, inp_V, inp_Q, B, base, **kw)
+    return P, g, o
+
+
+def test_pr1_parity():
+    # PR1: 1 layer x 2 KV heads x d 128, T = 1024, fp32, 8x (B_total = 256)
+    w = synth.WORKLOADS["pr1"]
+    x = synth.make_inputs(w)
+    B = (1 * 2 * 1024) // 8
+    P, g, o = _run(x.K, x.V, x.Q, B, w.rope_base)
+    rep = P.compare(g, o, torch.float32)
+    print("pr1", json.dumps(rep))
+    assert g["E"] == 256 and g["recent"] == 32
+
+
+def test_ragged_bf16_gqa_parity():
+    # small-model shapes (d 64, 4 query heads per KV head, 64 probes, bf16) on a
+    # 2-layer slice with a ragged T = 1000; several slots, tiles and tails.
+    w = synth.WORKLOADS["small"]
+    x = synth.make_inputs(w, layers=[0, 1], heads=[0, 1], T=1000)
+    L, G, T, d = x.K.shape
+    B = (L * G * T) // 8
+    P, g, o = _run(x.K, x.V, x.Q, B, w.rope_base)
+    rep = P.compare(g, o, torch.bfloat16)
+    print("ragged_bf16", json.dumps(rep))
+
+
+@pytest.mark.parametrize("x_ratio", [2, 16])
+def test_budget_sweep_bf16(x_ratio):
+    w = synth.WORKLOADS["small"]
+    x = synth.make_inputs(w, layers=[3], heads=[2, 5], T=1536, W=32)
+    L, G, T, d = x.K.shape
+    B = (L * G * T) // x_ratio
+    P, g, o = _run(x.K, x.V, x.Q, B, w.rope_base)
+    rep = P.compare(g, o, torch.bfloat16)
+    print(f"x={x_ratio}", json.dumps(rep))
+
+
+def test_fullkv_identity_is_bit_exact():
+    # x = 1: every tree expands to its leaves; the cache is the input (App. C.5)
+    w = synth.WORKLOADS["pr1"]
+    x = synth.make_inputs(w, T=640)
+    L, G, T, d = x.K.shape
+    from tests import parity as P
+    g = P.run_gpu(x.K, x.V, x.Q, L * G * T, w.rope_base)
+    c = g["cache"]
+    assert g["E"] == L * G * T
+    for lg in range(L * G):
+        lo, hi = c["offsets"][lg], c["offsets"][lg + 1]
+        assert np.array_equal(c["pos"][lo:hi].numpy(), np.arange(T))
+        assert torch.equal(c["K"][lo:hi], x.K[lg // G, lg % G])
+        assert torch.equal(c["V"][lo:hi], x.V[lg // G, lg % G])
+        assert torch.all(c["log_m"][lo:hi] == 0)
+
+
+def test_context_prefix_suffix_parity():
+    w = synth.WORKLOADS["pr1"]
+    x = synth.make_inputs(w, T=700)
+    L, G, T, d = x.K.shape
+    cs, ce = 37, 650
+    B = (L * G * (ce - cs)) // 6
+    P, g, o = _run(x.K, x.V, x.Q, B, w.rope_base, ctx_start=cs, ctx_end=ce)
+    rep = P.compare(g, o, torch.float32)
+    print("ctx", json.dumps(rep))
+    c = g["cache"]
+    for lg in range(L * G):
+        lo, hi = c["offsets"][lg], c["offsets"][lg + 1]
+        assert np.array_equal(c["pos"][lo:lo + cs].numpy(), np.arange(cs))
+        assert np.array_equal(c["pos"][hi - (T - ce + g["recent"]):hi].numpy(),
+                              np.arange(ce - g["recent"], T))
+
+
+def test_supplied_slots_hidden_surprisal_omega():
+    w = synth.WORKLOADS["small"]
+    x = synth.make_inputs(w, layers=[0], heads=[0, 1, 2], T=900, W=16)
+    L, G, T, d = x.K.shape
+    rng = np.random.default_rng(5)
+    N = T - 32
+    lens = []
+    while sum(lens) < N:                      # includes single-token slots
+        lens.append(int(rng.integers(1, 129)))
+    lens[-1] -= sum(lens) - N
+    lens = [n for n in lens if n > 0]
+    starts = np.concatenate([[0], np.cumsum(lens)])
+    hidden = rng.normal(size=(1, T, 48)).astype(np.float32)
+    surprisal = np.abs(rng.normal(size=T)).astype(np.float32)
+    surprisal[0] = 0
+    omega = rng.uniform(0.5, 1.5, size=L * G).astype(np.float32)
+    B = (L * G * T) // 5
+    P, g, o = _run(x.K, x.V, x.Q, B, w.rope_base, slot_starts=starts, hidden=hidden,
+                   surprisal=surprisal, omega=omega)
+    rep = P.compare(g, o, torch.bfloat16)
+    print("supplied", json.dumps(rep))
+
+
+def test_errors_are_reported_not_trapped():
+    from paper_2608_07001_gb300 import gracekv as gk
+    w = synth.WORKLOADS["pr1"]
+    x = synth.make_inputs(w, T=300)
+    L, G, T, d = x.K.shape
+    p = gk.make_params(L, G, 2, T, d, 32, dtype=torch.float32, budget=100, rope_base=w.rope_base)
+    ctx = gk.Context(p)
+    K, V, Q = x.K.cuda(), x.V.cuda(), x.Q.cuda()
+    with pytest.raises(gk.GraceKVError) as e:          # out of order
+        ctx.gracekv_allocate()
+    assert e.value.status == gk.GKV_ESTATE
+    slots = torch.empty(T, dtype=torch.int32, device="cuda")
+    ctx.gracekv_segment(V, slots)
+    bad = torch.tensor([0, 200, T - 32], dtype=torch.int32, device="cuda")   # slot of 200 tokens
+    with pytest.raises(gk.GraceKVError) as e:
+        ctx.gracekv_build_trees(K, V, Q, None, bad, 2)
+    assert e.value.status == gk.GKV_EUNSUPPORTED
+    bad = torch.tensor([0, 50, 40, T - 32], dtype=torch.int32, device="cuda")
+    with pytest.raises(gk.GraceKVError) as e:
+        ctx.gracekv_build_trees(K, V, Q, None, bad, 3)
+    assert e.value.status == gk.GKV_EINVAL
+    Vn = V.clone()
+    Vn[0, 0, 17, 3] = float("nan")
+    ctx2 = gk.Context(p)
+    with pytest.raises(gk.GraceKVError) as e:
+        ctx2.gracekv_segment(Vn, slots)
+    assert e.value.status == gk.GKV_ENONFINITE
+    Kn = K.clone()
+    Kn[0, 1, 5, 0] = float("inf")
+    ctx3 = gk.Context(p)
+    ctx3.gracekv_segment(V, slots)
+    ctx3.gracekv_build_trees(Kn, V, Q)
+    with pytest.raises(gk.GraceKVError) as e:
+        ctx3.gracekv_allocate()
+    assert e.value.status == gk.GKV_ENONFINITE
