@@ -1,0 +1,317 @@
+#!/usr/bin/env python3
+"""Benchmark of the GraceKV compression pass on GB300.
+
+One step = the whole pass (segment, build trees, allocate, gather) over one
+synthetic request of the workload, inputs resident in HBM.  Default workload:
+Llama-3-8B-shaped cache, 32 layers x 8 KV heads x 128K tokens x d 128, bf16,
+64 observation queries, 32x compression (B_total = L G T / 32).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload NAME] [--ratio X] [--no-e2e]
+
+Under torchrun each rank compresses its own request on its own GPU (independent
+requests, no collective): value = requests x T tokens / max-over-ranks time.
+--impl reference times the CPU oracle (the paper's definitions in plain C,
+single thread) on a bounded sample of the same workload and extrapolates its
+tokens/s linearly in L*G*T.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np
+import torch
+
+METRIC = "context tokens compressed/sec per GB300 and % of HBM roofline (vs CPU oracle)"
+PEAK_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                 "sm_max_mhz": 2070.0}
+N_SMS = 152
+FP32_LANES = 128
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d, "measured"
+    return PEAK_FALLBACK, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle sampling during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu: int):
+        self.gpu = gpu
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+def cpu_baseline(w, ratio: float, T_s: int = 1536):
+    """Oracle on one layer x one KV head x T_s tokens of the workload's recipe."""
+    import oracle as O
+    from paper_2608_07001_gb300 import synth
+    x = synth.make_inputs(w, layers=[0], heads=[0], T=T_s)
+    L1, G1, T1, d = x.K.shape
+    B = max(int(L1 * G1 * T1 // ratio), 4 * L1 * G1 + 1)
+    t0 = time.perf_counter()
+    O.run(x.K, x.V, x.Q, B, w.rope_base)
+    dt = time.perf_counter() - t0
+    # linear extrapolation in L*G*T: tokens/s = T / (dt * L * G * T / T_s)
+    value = T_s / (dt * w.L * w.G)
+    sample = (f"oracle pipeline on 1 layer x 1 KV head x {T_s} tokens "
+              f"({dt:.1f} s), extrapolated linearly to {w.L} x {w.G} x {w.T}")
+    return value, dt, sample
+
+
+def run_reference(args, w):
+    """Reference arm: the CPU oracle, timed on the host cores."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    vals = []
+    for i in range(args.warmup + args.steps):
+        v, dt, sample = cpu_baseline(w, args.ratio, T_s=args.ref_tokens)
+        if i >= args.warmup:
+            vals.append((v, dt))
+    value = statistics.median(v for v, _ in vals)
+    ms = statistics.median(dt for _, dt in vals) * 1e3 * (w.L * w.G * w.T / args.ref_tokens)
+    out = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+           "data": "synthetic", "impl": "reference",
+           "config": workload_config(w, args.ratio),
+           "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                            "sample": sample},
+           "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0}}
+    print(json.dumps(out))
+
+
+def workload_config(w, ratio):
+    return {"workload": f"{w.name}@{int(ratio)}x", "L": w.L, "G": w.G, "Hq": w.Hq, "d": w.d,
+            "T": w.T, "W": w.W, "ratio": ratio, "dtype": w.dtype,
+            "l2": "inputs larger than L2 (no flush needed)"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llama128k")
+    ap.add_argument("--ratio", type=float, default=32.0)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--ref-tokens", type=int, default=1024)
+    args = ap.parse_args()
+
+    from paper_2608_07001_gb300 import synth
+    w = synth.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, w)
+        return
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    from paper_2608_07001_gb300 import gracekv as gk
+    dev = torch.device("cuda", local)
+    x = synth.make_inputs(w, device=dev)
+    K, V, Q = x.K, x.V, x.Q
+    L, G, T, d = K.shape
+    B = gk.gracekv_budget_for_ratio(L, G, T, args.ratio)
+    p = gk.make_params(L, G, Q.shape[1], T, d, Q.shape[2], dtype=K.dtype, budget=B,
+                       rope_base=w.rope_base)
+    comp = gk.Compressor(p, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    for _ in range(args.warmup):
+        comp(K, V, Q)
+    comp.ctx.gracekv_profile(True)
+    comp.ctx.gracekv_stats()
+    _, launches0, _ = comp.ctx.gracekv_stats()
+    barrier()
+    clk = ClockSampler(local)
+    clk.start()
+    time.sleep(0.3)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        comp(K, V, Q)
+    e1.record(stream)
+    barrier()
+    clocks = clk.stop()
+    ms_total = e0.elapsed_time(e1)
+    stage_ms, launches1, work = comp.ctx.gracekv_stats()
+    comp.ctx.gracekv_profile(False)
+    t = torch.tensor([ms_total], device=dev, dtype=torch.float64)
+    if dist is not None:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms_total = float(t.item())
+    ms_step = ms_total / args.steps
+    value = world * T * args.steps / (ms_total / 1e3)
+    E = comp.n_entries
+
+    # ---- roofline ----------------------------------------------------------------
+    pk, pk_kind = peaks()
+    elem = 2 if K.dtype == torch.bfloat16 else 4
+    floor_bytes = L * G * T * 2 * d * elem + E * (2 * d * elem + 16)
+    hbm = {"floor_bytes": floor_bytes, "achieved_gbs": floor_bytes / (ms_step / 1e3) / 1e9,
+           "peak_gbs": pk["hbm_gbs"], "peak_kind": pk_kind}
+    hbm["frac"] = hbm["achieved_gbs"] / hbm["peak_gbs"]
+    per_step = {k: v / args.steps for k, v in stage_ms.items()}
+    dom = max(per_step, key=per_step.get)
+    Wp = Q.shape[2]
+    if dom == "unit_trees":
+        # probe scans (W*d FMA per token step), candidate evaluation (logit,
+        # residual and ||M||^2: 4 W d FMA), prototype sums (3 d per token),
+        # probe weights of every token (W d FMA)
+        flops = (2 * Wp * d * work["scan_steps"] + 8 * Wp * d * work["cand_evals"]
+                 + 6 * d * work["cand_len_sum"] + 2 * Wp * d * L * G * comp.ctx.n_c)
+        peak = N_SMS * FP32_LANES * 2 * pk.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+        ach = flops / (per_step[dom] / 1e3) / 1e12
+        roof = {"kernel": "unit_build_kernel", "bound": "alu", "achieved": ach, "peak": peak,
+                "unit": "TFLOP/s", "frac": ach / peak, "traffic": None,
+                "peak_basis": f"{N_SMS} SMs x {FP32_LANES} fp32 lanes x 2 x max SM clock"}
+    elif dom in ("row_stats", "token_values"):
+        flops = 2 * L * Q.shape[1] * Wp * d * (T if dom == "row_stats" else comp.ctx.n_c)
+        peak = N_SMS * FP32_LANES * 2 * pk.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+        ach = flops / (per_step[dom] / 1e3) / 1e12
+        roof = {"kernel": dom, "bound": "alu", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
+                "frac": ach / peak, "traffic": None}
+    else:
+        byt = L * G * T * 2 * d * elem if dom == "gather" else floor_bytes
+        ach = byt / (per_step[dom] / 1e3) / 1e9
+        roof = {"kernel": dom, "bound": "hbm", "achieved": ach, "peak": pk["hbm_gbs"],
+                "unit": "GB/s", "frac": ach / pk["hbm_gbs"], "traffic": None}
+
+    # ---- end to end through the C ABI with host buffers ---------------------------
+    e2e = None
+    if not args.no_e2e:
+        Kh = torch.empty_like(K, device="cpu").pin_memory()
+        Vh = torch.empty_like(V, device="cpu").pin_memory()
+        Qh = torch.empty_like(Q, device="cpu").pin_memory()
+        Kh.copy_(K); Vh.copy_(V); Qh.copy_(Q)
+        Kd, Vd, Qd = torch.empty_like(K), torch.empty_like(V), torch.empty_like(Q)
+        c = comp.cache
+        outs = [torch.empty_like(t, device="cpu").pin_memory()
+                for t in (c.K, c.V, c.pos, c.log_m, c.src_lo, c.src_hi, c.offsets)]
+
+        def e2e_step():
+            Kd.copy_(Kh, non_blocking=True); Vd.copy_(Vh, non_blocking=True)
+            Qd.copy_(Qh, non_blocking=True)
+            comp(Kd, Vd, Qd)
+            n = comp.n_entries
+            for o, t_ in zip(outs, (c.K, c.V, c.pos, c.log_m, c.src_lo, c.src_hi)):
+                o[:n].copy_(t_[:n], non_blocking=True)
+            outs[-1].copy_(c.offsets, non_blocking=True)
+            return n
+
+        e2e_step()
+        barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            n = e2e_step()
+        barrier()
+        dt = time.perf_counter() - t0
+        tt = torch.tensor([dt], device=dev, dtype=torch.float64)
+        if dist is not None:
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        dt = float(tt.item())
+        h2d = sum(t_.numel() * t_.element_size() for t_ in (K, V, Q))
+        d2h = n * (2 * d * elem + 16) + c.offsets.numel() * 8
+        e2e = {"value": world * T * args.e2e_steps / dt, "unit": "tokens/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        v, dt, sample = cpu_baseline(w, args.ratio)
+        cpu = {"value": v, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": sample}
+
+    if rank == 0:
+        out = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+               "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+               "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+               "dtype": "bf16" if K.dtype == torch.bfloat16 else "f32", "data": "synthetic",
+               "config": dict(workload_config(w, args.ratio), B_total=B, entries=E,
+                              slots=comp.n_slots, parallelism=f"replicas{world}"),
+               "roofline": roof, "hbm_pass": hbm, "stages_ms": per_step, "tree_work": work,
+               "cpu_baseline": cpu, "e2e": e2e,
+               "gpu_launches": launches1 - launches0, "clocks": clocks}
+        print(json.dumps(out))
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

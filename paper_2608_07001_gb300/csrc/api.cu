@@ -128,6 +128,7 @@ const char *gracekv_last_error(const gracekv_ctx *x) {
 
 void gracekv_destroy(gracekv_ctx *x) {
     if (!x) return;
+    for (cudaEvent_t e : x->c.ev_pool) cudaEventDestroy(e);
     for (void *p : x->allocs) cudaFree(p);
     delete x;
 }
@@ -221,7 +222,7 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
               dalloc(x, &w.nd_cost, (size_t)c.node_cap) && dalloc(x, &w.nd_D, (size_t)c.node_cap) &&
               dalloc(x, &w.nd_R, (size_t)c.node_cap) && dalloc(x, &w.nd_U, (size_t)c.node_cap) &&
               dalloc(x, &w.nd_kappa, (size_t)c.node_cap) && dalloc(x, &w.nd_sel, (size_t)c.node_cap) &&
-              dalloc(x, &w.hist, 2048) && dalloc(x, &w.alloc_state, 16);
+              dalloc(x, &w.hist, 2048) && dalloc(x, &w.alloc_state, 16) && dalloc(x, &w.work, 4);
     if (!ok) {
         gracekv_destroy(x);
         return GKV_ENOMEM;
@@ -258,7 +259,10 @@ gkv_status gracekv_segment(gracekv_ctx *x, const void *V, const float *hidden, i
     if (hidden && (Dh <= 0 || Dh > 2048)) return fail(x, GKV_EINVAL, "segment: hidden dim must be in [1, 2048]");
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t e = cudaMemsetAsync(c.w.dev_int, 0, 16 * sizeof(int), s);
-    if (e == cudaSuccess) e = gkv::launch_segment(c, V, hidden, hidden ? Dh : 0, surprisal, kappa, s);
+    if (e == cudaSuccess) {
+        gkv::StageTimer tm(c, 0, s);
+        e = gkv::launch_segment(c, V, hidden, hidden ? Dh : 0, surprisal, kappa, s);
+    }
     if (e != cudaSuccess) return cuda_fail(x, e, "segment launch");
     int h[2];
     e = cudaMemcpyAsync(h, c.w.dev_int, 2 * sizeof(int), cudaMemcpyDeviceToHost, s);
@@ -295,6 +299,7 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
         if (e == cudaSuccess) {
             validate_slots_kernel<<<(n_slots + 255) / 256, 256, 0, s>>>(c.w.slots, n_slots, c.p.ctx_start,
                                                                           c.c_end, c.w.dev_int + 1);
+            c.launches += 1;
             e = cudaGetLastError();
         }
         if (e == cudaSuccess) e = cudaMemcpyAsync(&h, c.w.dev_int + 1, sizeof(int), cudaMemcpyDeviceToHost, s);
@@ -315,9 +320,18 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
         if (!ok) return fail(x, GKV_ENOMEM, "build_trees: unit arrays");
         w.units_cap = cap;
     }
-    e = gkv::launch_row_stats(c, K, Q, s);
-    if (e == cudaSuccess) e = gkv::launch_token_values(c, K, Q, s);
-    if (e == cudaSuccess) e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, s);
+    {
+        gkv::StageTimer tm(c, 1, s);
+        e = gkv::launch_row_stats(c, K, Q, s);
+    }
+    if (e == cudaSuccess) {
+        gkv::StageTimer tm(c, 2, s);
+        e = gkv::launch_token_values(c, K, Q, s);
+    }
+    if (e == cudaSuccess) {
+        gkv::StageTimer tm(c, 3, s);
+        e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, s);
+    }
     if (e != cudaSuccess) return cuda_fail(x, e, "build_trees launch");
     c.stage = 2;
     return GKV_OK;
@@ -329,7 +343,11 @@ gkv_status gracekv_allocate(gracekv_ctx *x, int64_t *n_entries_host, void *strea
     Ctx &c = x->c;
     if (!n_entries_host) return fail(x, GKV_EINVAL, "allocate: null argument");
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    cudaError_t e = gkv::launch_allocate(c, c.J, s);
+    cudaError_t e;
+    {
+        gkv::StageTimer tm(c, 4, s);
+        e = gkv::launch_allocate(c, c.J, s);
+    }
     if (e != cudaSuccess) return cuda_fail(x, e, "allocate launch");
     unsigned long long used = 0;
     int h = 0;
@@ -356,8 +374,12 @@ gkv_status gracekv_gather(gracekv_ctx *x, const void *K, const void *V, void *K_
         return fail(x, GKV_EINVAL, "gather: null argument");
     const int64_t LG = (int64_t)c.p.L * c.p.G;
     if (cap < LG * (c.p.T - c.Nc) + c.used) return fail(x, GKV_ECAPACITY, "gather: cap below the entry count");
-    cudaError_t e = gkv::launch_gather(c, K, V, c.w.slots, c.J, K_out, V_out, pos, log_m, src_lo,
-                                       src_hi, offsets, static_cast<cudaStream_t>(stream));
+    cudaError_t e;
+    {
+        gkv::StageTimer tm(c, 5, static_cast<cudaStream_t>(stream));
+        e = gkv::launch_gather(c, K, V, c.w.slots, c.J, K_out, V_out, pos, log_m, src_lo, src_hi,
+                               offsets, static_cast<cudaStream_t>(stream));
+    }
     if (e != cudaSuccess) return cuda_fail(x, e, "gather launch");
     return GKV_OK;
 }
@@ -420,6 +442,42 @@ gkv_status gracekv_export(gracekv_ctx *x, int64_t node_cap, int64_t *n_nodes_hos
     if (unit_first) unit_first[nu] = k;
     *n_nodes_host = k;
     if (k > node_cap) return fail(x, GKV_ECAPACITY, "export: node_cap too small");
+    return GKV_OK;
+}
+
+gkv_status gracekv_profile(gracekv_ctx *x, int32_t enable) {
+    if (!x) return GKV_EINVAL;
+    x->c.profile = enable != 0;
+    x->c.ev_used = 0;
+    x->c.ev_stage.clear();
+    return GKV_OK;
+}
+
+gkv_status gracekv_stats(gracekv_ctx *x, float *stage_ms, int32_t n_stages, int64_t *launches,
+                         uint64_t *work, int32_t n_work) {
+    if (!x) return GKV_EINVAL;
+    Ctx &c = x->c;
+    if (launches) *launches = c.launches;
+    if (work && n_work > 0) {
+        unsigned long long h[4] = {0, 0, 0, 0};
+        cudaError_t e = cudaMemcpy(h, c.w.work, sizeof h, cudaMemcpyDeviceToHost);
+        if (e != cudaSuccess) return cuda_fail(x, e, "stats");
+        for (int i = 0; i < n_work; i++) work[i] = i < 4 ? h[i] : 0;
+    }
+    if (stage_ms) {
+        for (int i = 0; i < n_stages; i++) stage_ms[i] = 0.f;
+        for (size_t k = 0; k < c.ev_stage.size(); k++) {
+            cudaEvent_t e0 = c.ev_pool[2 * k], e1 = c.ev_pool[2 * k + 1];
+            cudaError_t e = cudaEventSynchronize(e1);
+            float ms = 0.f;
+            if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, e0, e1);
+            if (e != cudaSuccess) return cuda_fail(x, e, "stats");
+            int st = c.ev_stage[k];
+            if (st >= 0 && st < n_stages) stage_ms[st] += ms;
+        }
+    }
+    c.ev_used = 0;
+    c.ev_stage.clear();
     return GKV_OK;
 }
 

@@ -53,6 +53,7 @@ struct BuildArgs {
     float *u_Uadd, *u_Ddrop;
     uint8_t *u_sel;
     int *status;
+    unsigned long long *work;
 };
 
 struct NodeS {
@@ -187,6 +188,30 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
         if (c == 0) sm.E[u][t] = pact ? expf(x * A.inv_sqrt_d - mu) : 0.f;
     }
     __syncthreads();
+    // Non-finite probe weights or token values (NaN/Inf in K, Q or the row
+    // statistics) make every decision of the unit meaningless: record the
+    // unit as a single uncovered leaf with zero gain and flag the error, which
+    // the host reports as GKV_ENONFINITE at the allocation's count sync.
+    {
+        bool bad = false;
+        for (int e = tid; e < n * NW; e += kThreads) {
+            float v = sm.E[e / n][e % n];
+            bad |= !isfinite(v);
+        }
+        for (int t = tid; t < n; t += kThreads) bad |= !isfinite(sm.Rt[t]);
+        if (__syncthreads_or(bad)) {
+            if (tid == 0) {
+                atomicOr(A.status, 8);
+                A.nd_a[nbase] = sa; A.nd_b[nbase] = sb; A.nd_R[nbase] = 0.f; A.nd_D[nbase] = 0.f;
+                A.nd_parent[nbase] = (int32_t)(-2 - uid); A.nd_unit[nbase] = (int32_t)uid;
+                A.nd_child0[nbase] = -1; A.nd_nchild[nbase] = 0; A.nd_U[nbase] = 0.f;
+                A.nd_kappa[nbase] = 0.f; A.nd_sel[nbase] = 0;
+                A.u_nnodes[uid] = 1; A.u_Uadd[uid] = 0.f; A.u_Ddrop[uid] = 0.f; A.u_sel[uid] = 0;
+            }
+            for (int k = tid; k < 2 * n; k += kThreads) A.nd_cost[nbase + k] = 0;
+            return;
+        }
+    }
     // ---- k_circ = RoPE^-1(k, t) ----------------------------------------------
     for (int e = tid; e < n * HALF; e += kThreads) {
         int t = e / HALF, i = e - t * HALF;
@@ -221,6 +246,7 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
     }
     __syncthreads();
 
+    unsigned long long w_scan = 0, w_eval = 0, w_len = 0;   // thread 0's work counters
     int cur = 0;
     while (sm.nlvl[cur] > 0) {
         const int nl = sm.nlvl[cur];
@@ -291,6 +317,7 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
                     int p2 = __shfl_xor_sync(0xffffffffu, pb, o);
                     if (r2 > rb || (r2 == rb && p2 < pb)) { rb = r2; pb = p2; }
                 }
+                if (pb < a || pb >= b) pb = a;   // only reachable with non-finite values
                 if (lane == 0) {
                     B.kmin = kmin;
                     B.kmax = kmax;
@@ -305,7 +332,8 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
                             while (m) {
                                 int bit = __ffs(m) - 1;
                                 m &= m - 1;
-                                B.cut[B.ncut++] = a + w * 32 + bit + 1;
+                                if (B.ncut < min(A.k_cand + 1, nv - 1))
+                                    B.cut[B.ncut++] = a + w * 32 + bit + 1;
                             }
                         }
                         // prefixes in ascending end: cuts merged with the extraction's left side
@@ -427,6 +455,13 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
                 const BatchNode &B = sm.bn[bi];
                 if (B.pre_e == B.pre_b && B.suf_e == B.suf_b) continue;
                 const int a = sm.nodes[B.node].a, b = sm.nodes[B.node].b;
+                if (tid == 0) {
+                    int pe = B.pre_e > B.pre_b ? sm.cand[B.pre_e - 1].b : a;   // forward scan stops here
+                    int ss = B.suf_e > B.suf_b ? sm.cand[B.suf_e - 1].a : b;   // backward scan stops here
+                    w_scan += (pe - a) + (b - ss);
+                    w_eval += B.suf_e - B.pre_b;
+                    for (int k = B.pre_b; k < B.suf_e; k++) w_len += sm.cand[k].b - sm.cand[k].a;
+                }
                 float M[CH];
                 float Z = 0.f;
                 // forward: prefixes [a, end) in ascending end
@@ -511,6 +546,11 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
                 if (ps + 1 < b) { ea[ne] = ps + 1; eb[ne] = b; eD[ne] = b - ps - 1 >= 2 ? Dc(B.eR) : 0.0; ne++; }
                 double gext = DI;
                 for (int q = 0; q < ne; q++) gext -= eD[q];
+                if (bxi < 0) {   // only reachable with non-finite gains
+                    bxi = B.cut[0];
+                    bL = B.pidx[0] >= 0 ? Dc(B.pidx[0]) : 0.0;
+                    bR = B.sidx[0] >= 0 ? Dc(B.sidx[0]) : 0.0;
+                }
                 const double rho_ext = gext / (ne - 1);
                 if (rho_ext > best) {
                     B.nchild = ne;
@@ -600,6 +640,10 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
     if (tid == 0) {
         A.u_nnodes[uid] = sm.nnodes;
         A.u_sel[uid] = 0;
+        atomicAdd(&A.work[0], w_scan);
+        atomicAdd(&A.work[1], w_eval);
+        atomicAdd(&A.work[2], w_len);
+        atomicAdd(&A.work[3], 1ull);
     }
     // unused node slots of the unit carry cost 0 (no op)
     for (int k = sm.nnodes + tid; k < 2 * n; k += kThreads) A.nd_cost[nbase + k] = 0;
@@ -615,6 +659,7 @@ cudaError_t launch_t(Ctx &c, BuildArgs &A, int J, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     unsigned grid = (unsigned)((int64_t)J * c.p.L * c.p.G);
     unit_build_kernel<DH, NW, Tin><<<grid, kThreads, sm, s>>>(A);
+    c.launches += 1;
     return cudaGetLastError();
 }
 
@@ -646,6 +691,8 @@ cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *
     A.nd_sel = c.w.nd_sel;
     A.u_nnodes = c.w.u_nnodes; A.u_Uadd = c.w.u_Uadd; A.u_Ddrop = c.w.u_Ddrop; A.u_sel = c.w.u_sel;
     A.status = c.w.dev_int + 1;
+    A.work = c.w.work;
+    cudaMemsetAsync(c.w.work, 0, 4 * sizeof(unsigned long long), s);
     if (p.dtype == GKV_BF16) return launch_dt<__nv_bfloat16>(c, A, J, s);
     return launch_dt<float>(c, A, J, s);
 }

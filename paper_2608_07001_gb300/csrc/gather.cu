@@ -254,6 +254,7 @@ cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *s
         else gather_units_kernel<float><<<gu, 256, 0, s>>>(A);
     }
     int ntok = c.p.ctx_start + (c.p.T - c.c_end);
+    c.launches += 2 + (gu ? 1 : 0) + (ntok > 0 ? 1 : 0);
     if (ntok > 0) {
         dim3 g((ntok + 7) / 8, c.p.L * c.p.G);
         if (bf) gather_tokens_kernel<__nv_bfloat16><<<g, 256, 0, s>>>(A);

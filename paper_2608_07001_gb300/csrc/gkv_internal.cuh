@@ -7,6 +7,7 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 #include <string>
+#include <vector>
 
 #include "../../include/gracekv.h"
 
@@ -60,6 +61,7 @@ struct Workspace {
     // allocation
     unsigned long long *hist = nullptr;        // [2048] cost-weighted histogram
     unsigned long long *alloc_state = nullptr; // see alloc.cu
+    unsigned long long *work = nullptr;        // [4] tree-building work counters
 };
 
 struct Ctx {
@@ -77,6 +79,38 @@ struct Ctx {
     Workspace w;
     int64_t node_cap = 0;          // L*G*2*N_c
     int n_chunks = 0;              // pass-A chunks per row
+    // measurement
+    int64_t launches = 0;          // kernels launched (host count)
+    bool profile = false;
+    std::vector<cudaEvent_t> ev_pool;          // recorded (begin, end) pairs
+    std::vector<int> ev_stage;                 // stage of each pair
+    size_t ev_used = 0;
+};
+
+// RAII helper: records a (begin, end) event pair around a kernel group when
+// profiling is on.
+struct StageTimer {
+    Ctx &c;
+    cudaStream_t s;
+    cudaEvent_t e1 = nullptr;
+    StageTimer(Ctx &c_, int stage, cudaStream_t s_) : c(c_), s(s_) {
+        if (!c.profile) return;
+        if (c.ev_used + 2 > c.ev_pool.size()) {
+            for (int k = 0; k < 64; k++) {
+                cudaEvent_t e;
+                if (cudaEventCreate(&e) != cudaSuccess) return;
+                c.ev_pool.push_back(e);
+            }
+        }
+        cudaEvent_t e0 = c.ev_pool[c.ev_used];
+        e1 = c.ev_pool[c.ev_used + 1];
+        c.ev_used += 2;
+        c.ev_stage.push_back(stage);
+        cudaEventRecord(e0, s);
+    }
+    ~StageTimer() {
+        if (e1) cudaEventRecord(e1, s);
+    }
 };
 
 // ---------------------------------------------------------------------------

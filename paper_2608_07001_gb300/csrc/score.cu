@@ -252,6 +252,7 @@ cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t 
     int nrow = a.L * a.Hq * a.W;
     row_combine_kernel<<<(nrow + 255) / 256, 256, 0, s>>>(c.w.rowp, nrow, c.n_chunks, c.w.row_m,
                                                           c.w.row_Z, c.w.row_ZC, c.w.dev_int + 1);
+    c.launches += 2;
     return cudaGetLastError();
 }
 
@@ -267,6 +268,7 @@ cudaError_t launch_token_values(Ctx &c, const void *K, const void *Q, cudaStream
         token_values_kernel<<<grid, 256, 0, s>>>(static_cast<const float *>(K),
                                                  static_cast<const float *>(Q), a, c.w.row_m,
                                                  c.w.row_Z, c.w.row_ZC, eps, c.w.rtok);
+    c.launches += 1;
     return cudaGetLastError();
 }
 

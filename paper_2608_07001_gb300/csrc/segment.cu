@@ -667,6 +667,7 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
     cudaFuncSetAttribute(seg_dp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smd);
     seg_dp_kernel<<<1, 1024, smd, s>>>(w.ew, w.ewt, N, p.n_min, p.n_max, p.ctx_start, w.dpF,
                                        w.slots, w.dev_int);
+    c.launches += 8 + (surprisal ? 2 : 0) + (N > 1 ? 1 : 0);
     return cudaGetLastError();
 }
 

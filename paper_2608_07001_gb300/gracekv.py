@@ -51,7 +51,7 @@ _lib = None
 EXPORTED = ["gracekv_default_params", "gracekv_budget_for_ratio", "gracekv_create",
             "gracekv_destroy", "gracekv_last_error", "gracekv_status_string", "gracekv_query",
             "gracekv_segment", "gracekv_build_trees", "gracekv_allocate", "gracekv_gather",
-            "gracekv_export"]
+            "gracekv_export", "gracekv_profile", "gracekv_stats"]
 
 
 def lib() -> C.CDLL:
@@ -79,6 +79,8 @@ def lib() -> C.CDLL:
     L.gracekv_allocate.argtypes = [vp, C.POINTER(i64), vp]
     L.gracekv_gather.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, i64, vp]
     L.gracekv_export.argtypes = [vp, i64, C.POINTER(i64)] + [vp] * 18 + [vp]
+    L.gracekv_profile.argtypes = [vp, i32]
+    L.gracekv_stats.argtypes = [vp, vp, i32, C.POINTER(i64), vp, i32]
     _lib = L
     return L
 
@@ -177,6 +179,22 @@ class Context:
                                          _ptr(out.pos), _ptr(out.log_m), _ptr(out.src_lo),
                                          _ptr(out.src_hi), _ptr(out.offsets), out.K.shape[0],
                                          _stream(stream)))
+
+    STAGES = ("segment", "row_stats", "token_values", "unit_trees", "allocate", "gather")
+
+    def gracekv_profile(self, enable: bool = True):
+        self._check(lib().gracekv_profile(self.h, int(enable)))
+
+    def gracekv_stats(self):
+        """(per-stage ms since the last call, kernels launched so far, tree work counters)."""
+        import numpy as np
+        ms = np.zeros(len(self.STAGES), np.float32)
+        work = np.zeros(4, np.uint64)
+        n = C.c_int64()
+        self._check(lib().gracekv_stats(self.h, C.c_void_p(ms.ctypes.data), len(ms), C.byref(n),
+                                        C.c_void_p(work.ctypes.data), 4))
+        names = ("scan_steps", "cand_evals", "cand_len_sum", "units")
+        return dict(zip(self.STAGES, ms.tolist())), n.value, dict(zip(names, map(int, work)))
 
     def gracekv_export(self, node_cap: Optional[int] = None, stream=None) -> dict:
         """Host copy of the trees and selection (introspection for tests)."""
