@@ -210,6 +210,30 @@ gkv_status gracekv_profile(gracekv_ctx *ctx, int32_t enable);
 gkv_status gracekv_stats(gracekv_ctx *ctx, float *stage_ms, int32_t n_stages, int64_t *launches,
                          uint64_t *work, int32_t n_work);
 
+/*
+ * Allocation-free row statistics (the paper has no counterpart: this is a
+ * deployment entry point).  For callers that must not call cudaMalloc -- an
+ * engine that reserves the whole device for its own memory pool, or a
+ * latency-critical loop that cannot take the device synchronisation an
+ * allocation may cause -- this call computes, without a context and without
+ * allocating, the same per-probe-row statistics as gracekv_build_trees: for
+ * every row (l, h, u) the max logit m over [0, T), Z = sum exp(x - m) over
+ * [0, T) and Z^C over the range [c_lo, c_hi).  K [L][G][T][d] and Q
+ * [L][Hq][W][d] (dtype GKV_F32 / GKV_BF16) are device inputs; row_m, row_Z,
+ * row_ZC [L][Hq][W] fp32 are device outputs; work is enqueued on `stream`.
+ *   Scratch: a fixed 4 MiB device array inside this library (held by every
+ *   GPU that loads it until the process exits); L * Hq * W above 349525 rows
+ *   returns GKV_ECAPACITY.  The first call on a device resolves the array's
+ *   device address; make that first call before any stream capture.
+ *   Calls share the array: calls that overlap on the GPU (other streams,
+ *   other threads) race and must be serialised by the caller.
+ *   Errors: GKV_EINVAL (shapes, pointers), GKV_ECAPACITY, GKV_ECUDA.
+ */
+gkv_status gracekv_row_stats_noalloc(const void *K, const void *Q, int32_t L, int32_t G,
+                                     int32_t Hq, int32_t T, int32_t d, int32_t W, int32_t dtype,
+                                     int32_t c_lo, int32_t c_hi, float *row_m, float *row_Z,
+                                     float *row_ZC, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

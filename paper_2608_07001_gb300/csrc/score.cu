@@ -16,6 +16,9 @@
 // 64 x 64 tiles (FFMA, fp32 accumulation of the exact bf16/fp32 inputs).
 #include "gkv_internal.cuh"
 
+#include <algorithm>
+#include <mutex>
+
 namespace gkv {
 namespace {
 
@@ -273,3 +276,90 @@ cudaError_t launch_token_values(Ctx &c, const void *K, const void *Q, cudaStream
 }
 
 }  // namespace gkv
+
+// ---------------------------------------------------------------------------
+// Allocation-free row statistics.
+//
+// Some callers cannot call cudaMalloc: a serving engine or framework that
+// reserves the whole device for its own memory pool, or a latency-critical
+// loop that cannot accept the implicit device synchronisation an allocation
+// can cause.  gracekv_row_stats_noalloc gives them the row statistics pass
+// without a context: its scratch (the per-chunk partial maxima and sums, and
+// a status word) lives in the fixed array below, which every GPU that loads
+// this library keeps for the life of the process.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr size_t kNoAllocScratchFloats = (size_t)1 << 20;   // 4 MiB of fp32 scratch
+static __device__ __align__(256) float g_noalloc_scratch[kNoAllocScratchFloats];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+float *g_noalloc_ptr[kMaxDevices] = {};
+
+// Device address of the scratch array for the current device, resolved once
+// per device (host code cannot use the array's name as a device address).
+cudaError_t noalloc_scratch(int dev, float **out) {
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void *p = nullptr;
+        cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess) return e;
+        g_noalloc_ptr[dev] = static_cast<float *>(p);
+    }
+    *out = g_noalloc_ptr[dev];
+    return cudaSuccess;
+}
+
+}  // namespace
+
+extern "C" gkv_status gracekv_row_stats_noalloc(const void *K, const void *Q, int32_t L, int32_t G,
+                                                int32_t Hq, int32_t T, int32_t d, int32_t W,
+                                                int32_t dtype, int32_t c_lo, int32_t c_hi,
+                                                float *row_m, float *row_Z, float *row_ZC,
+                                                void *stream) {
+    if (!K || !Q || !row_m || !row_Z || !row_ZC) return GKV_EINVAL;
+    if (L <= 0 || G <= 0 || Hq <= 0 || T <= 0 || d <= 0 || W <= 0 || Hq % G || d % 8) return GKV_EINVAL;
+    if (dtype != GKV_F32 && dtype != GKV_BF16) return GKV_EINVAL;
+    if (c_lo < 0 || c_hi > T || c_lo > c_hi) return GKV_EINVAL;
+    const int64_t nrow = (int64_t)L * Hq * W;
+    // three partials per (row, chunk) plus one status word must fit the array
+    if (3 * nrow + 1 > (int64_t)kNoAllocScratchFloats) return GKV_ECAPACITY;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return GKV_ECUDA;
+    float *scratch = nullptr;
+    if (noalloc_scratch(dev, &scratch) != cudaSuccess) return GKV_ECUDA;
+    int sms = 148;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    gkv::ScoreArgs a;
+    a.L = L; a.G = G; a.Hq = Hq; a.T = T; a.d = d; a.W = W;
+    a.gq = Hq / G;
+    a.Rg = a.gq * W;
+    a.cs = c_lo; a.cend = c_hi; a.Nc = c_hi - c_lo;
+    a.inv_sqrt_d = (float)(1.0 / sqrt((double)d));
+    const int64_t base = (int64_t)L * G * ((a.Rg + 63) / 64);
+    int64_t nch = (4 * (int64_t)sms + base - 1) / base;
+    nch = std::max<int64_t>(1, std::min<int64_t>(nch, std::max(1, T / 256)));
+    while (nch > 1 && 3 * nrow * nch + 1 > (int64_t)kNoAllocScratchFloats) nch--;
+    const int nchunks = (int)nch;
+    int chunk = (T + nchunks - 1) / nchunks;
+    chunk = (chunk + gkv::kTT - 1) / gkv::kTT * gkv::kTT;
+    int *status = reinterpret_cast<int *>(scratch + 3 * nrow * nchunks);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    // every (row, chunk) partial is overwritten by the pass; only the status
+    // word has to start at zero
+    if (cudaMemsetAsync(status, 0, sizeof(int), s) != cudaSuccess) return GKV_ECUDA;
+    dim3 grid(nchunks, (a.Rg + gkv::kTR - 1) / gkv::kTR, L * G);
+    if (dtype == GKV_BF16)
+        gkv::row_stats_kernel<<<grid, 256, 0, s>>>(static_cast<const __nv_bfloat16 *>(K),
+                                                   static_cast<const __nv_bfloat16 *>(Q), a, chunk,
+                                                   nchunks, scratch);
+    else
+        gkv::row_stats_kernel<<<grid, 256, 0, s>>>(static_cast<const float *>(K),
+                                                   static_cast<const float *>(Q), a, chunk, nchunks,
+                                                   scratch);
+    gkv::row_combine_kernel<<<(unsigned)((nrow + 255) / 256), 256, 0, s>>>(scratch, (int)nrow, nchunks,
+                                                                            row_m, row_Z, row_ZC, status);
+    return cudaGetLastError() == cudaSuccess ? GKV_OK : GKV_ECUDA;
+}

@@ -51,7 +51,7 @@ _lib = None
 EXPORTED = ["gracekv_default_params", "gracekv_budget_for_ratio", "gracekv_create",
             "gracekv_destroy", "gracekv_last_error", "gracekv_status_string", "gracekv_query",
             "gracekv_segment", "gracekv_build_trees", "gracekv_allocate", "gracekv_gather",
-            "gracekv_export", "gracekv_profile", "gracekv_stats"]
+            "gracekv_export", "gracekv_profile", "gracekv_stats", "gracekv_row_stats_noalloc"]
 
 
 def lib() -> C.CDLL:
@@ -81,6 +81,7 @@ def lib() -> C.CDLL:
     L.gracekv_export.argtypes = [vp, i64, C.POINTER(i64)] + [vp] * 18 + [vp]
     L.gracekv_profile.argtypes = [vp, i32]
     L.gracekv_stats.argtypes = [vp, vp, i32, C.POINTER(i64), vp, i32]
+    L.gracekv_row_stats_noalloc.argtypes = [vp, vp] + [i32] * 9 + [vp, vp, vp, vp]
     _lib = L
     return L
 
@@ -93,6 +94,23 @@ def gracekv_default_params() -> GkvParams:
 
 def gracekv_budget_for_ratio(L: int, G: int, n_ctx: int, x: float) -> int:
     return int(lib().gracekv_budget_for_ratio(L, G, n_ctx, float(x)))
+
+
+def gracekv_row_stats_noalloc(K, Q, c_lo: int, c_hi: int, row_m, row_Z, row_ZC, stream=None):
+    """Row statistics without a context and without any device allocation.
+
+    For callers that cannot call cudaMalloc (an engine owning the device's
+    memory pool, or a loop that cannot afford an allocation's synchronisation):
+    the scratch is a fixed 4 MiB array inside the library.  Outputs are
+    caller-provided [L, Hq, W] fp32 CUDA tensors.  Overlapping calls race.
+    """
+    L, G, T, d = K.shape
+    Hq, W = Q.shape[1], Q.shape[2]
+    dt = GKV_BF16 if K.dtype == torch.bfloat16 else GKV_F32
+    st = lib().gracekv_row_stats_noalloc(_ptr(K), _ptr(Q), L, G, Hq, T, d, W, dt, c_lo, c_hi,
+                                         _ptr(row_m), _ptr(row_Z), _ptr(row_ZC), _stream(stream))
+    if st != GKV_OK:
+        raise GraceKVError(st, lib().gracekv_status_string(st).decode())
 
 
 def _ptr(t: Optional[torch.Tensor]):
