@@ -309,9 +309,8 @@ __global__ void alloc_init_kernel(unsigned long long *st, unsigned long long *hi
     for (int b = i; b < 2048; b += blockDim.x) hist[b] = 0;
 }
 
-}  // namespace
 
-cudaError_t launch_allocate(Ctx &c, int J, cudaStream_t s) {
+AllocArgs make_args(Ctx &c, int J) {
     Workspace &w = c.w;
     AllocArgs A;
     A.n_units = (int64_t)c.p.L * c.p.G * J;
@@ -323,11 +322,32 @@ cudaError_t launch_allocate(Ctx &c, int J, cudaStream_t s) {
     A.J = J; A.LG = c.p.L * c.p.G; A.cs = c.p.ctx_start; A.Nc = c.Nc;
     A.u_sel = w.u_sel; A.nd_sel = w.nd_sel; A.u_flag = w.u_count;
     A.hist = w.hist; A.st = w.alloc_state; A.B_free = c.B_free; A.status = w.dev_int + 1;
-    cudaMemsetAsync(w.u_count, 0, sizeof(int32_t) * A.n_units, s);
-    alloc_init_kernel<<<1, 256, 0, s>>>(w.alloc_state, w.hist);
-    const int64_t n = A.n_units + A.n_nodes;
+    return A;
+}
+
+int grid_for(const Ctx &c, int64_t n) {
     int blocks = (int)std::min<int64_t>((n + 255) / 256, (int64_t)c.num_sms * 8);
-    if (blocks < 1) blocks = 1;
+    return blocks < 1 ? 1 : blocks;
+}
+
+// Units with a pending node whose creator key is >= tau (all of them when
+// every op built so far fits the budget).
+__global__ void prune_list_kernel(const float *u_pend, int64_t n_units,
+                                  const unsigned long long *st, int32_t *list, int *count) {
+    int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= n_units) return;
+    float p = u_pend[i];
+    if (!(p >= 0.f)) return;   // -1: no pending node
+    const bool all = st[ST_ALL] != 0;
+    if (all || __float_as_uint(p) >= (uint32_t)st[ST_PREFIX]) list[atomicAdd(count, 1)] = (int32_t)i;
+}
+
+}  // namespace
+
+cudaError_t launch_threshold(Ctx &c, int J, cudaStream_t s) {
+    AllocArgs A = make_args(c, J);
+    alloc_init_kernel<<<1, 256, 0, s>>>(c.w.alloc_state, c.w.hist);
+    const int blocks = grid_for(c, A.n_units + A.n_nodes);
     const int shifts[3] = {21, 10, 0};
     const int bits[3] = {11, 11, 10};
     uint32_t mask = 0;
@@ -336,13 +356,34 @@ cudaError_t launch_allocate(Ctx &c, int J, cudaStream_t s) {
         alloc_scan_kernel<<<1, 32, 0, s>>>(A, shifts[ps], bits[ps]);
         mask |= ((1u << bits[ps]) - 1u) << shifts[ps];
     }
+    c.launches += 7;
+    return cudaGetLastError();
+}
+
+cudaError_t launch_prune_list(Ctx &c, int J, int32_t *list, int *count, cudaStream_t s) {
+    const int64_t nu = (int64_t)c.p.L * c.p.G * J;
+    cudaError_t e = cudaMemsetAsync(count, 0, sizeof(int), s);
+    if (e != cudaSuccess) return e;
+    prune_list_kernel<<<(unsigned)((nu + 255) / 256), 256, 0, s>>>(c.w.u_pend, nu, c.w.alloc_state,
+                                                                    list, count);
+    c.launches += 1;
+    return cudaGetLastError();
+}
+
+cudaError_t launch_allocate(Ctx &c, int J, cudaStream_t s) {
+    Workspace &w = c.w;
+    AllocArgs A = make_args(c, J);
+    cudaMemsetAsync(w.u_count, 0, sizeof(int32_t) * A.n_units, s);
+    cudaError_t e = launch_threshold(c, J, s);
+    if (e != cudaSuccess) return e;
+    const int blocks = grid_for(c, A.n_units + A.n_nodes);
     alloc_mark_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_ties_kernel<<<1, 1024, 0, s>>>(A);
     alloc_end_max_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_end_key_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_end_pick_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_final_kernel<<<1, 32, 0, s>>>(A);
-    c.launches += 13;
+    c.launches += 6;
     return cudaGetLastError();
 }
 

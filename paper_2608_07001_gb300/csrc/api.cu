@@ -316,7 +316,8 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
         int64_t cap = std::max<int64_t>(nu, w.units_cap * 2);
         bool ok = dalloc(x, &w.u_nnodes, cap) && dalloc(x, &w.u_Uadd, cap) &&
                   dalloc(x, &w.u_Ddrop, cap) && dalloc(x, &w.u_sel, cap) &&
-                  dalloc(x, &w.u_count, cap) && dalloc(x, &w.u_off, cap);
+                  dalloc(x, &w.u_count, cap) && dalloc(x, &w.u_off, cap) &&
+                  dalloc(x, &w.u_pend, cap) && dalloc(x, &w.u_list, cap);
         if (!ok) return fail(x, GKV_ENOMEM, "build_trees: unit arrays");
         w.units_cap = cap;
     }
@@ -328,9 +329,37 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
         gkv::StageTimer tm(c, 2, s);
         e = gkv::launch_token_values(c, K, Q, s);
     }
+    // Trees: roots and their splits for every unit, then pruned resumption
+    // (see build.cu): only pending nodes whose creator key reaches the
+    // threshold of the ops built so far are evaluated.
+    if (e == cudaSuccess) e = cudaMemsetAsync(w.work, 0, 4 * sizeof(unsigned long long), s);
     if (e == cudaSuccess) {
         gkv::StageTimer tm(c, 3, s);
-        e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, s);
+        e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 0, 1, 0.f, nullptr, 0, s);
+    }
+    for (int it = 0; e == cudaSuccess; it++) {
+        struct { int count; unsigned long long prefix, all; } h = {0, 0, 0};
+        {
+            gkv::StageTimer tm(c, 3, s);
+            e = gkv::launch_threshold(c, J, s);
+            if (e == cudaSuccess) e = gkv::launch_prune_list(c, J, w.u_list, w.dev_int + 2, s);
+        }
+        if (e == cudaSuccess) e = cudaMemcpyAsync(&h.count, w.dev_int + 2, sizeof(int), cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(&h.prefix, w.alloc_state, 2 * sizeof(unsigned long long),
+                                                  cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(&h.all, w.alloc_state + 2, sizeof(unsigned long long),
+                                                  cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+        if (e != cudaSuccess || h.count == 0) break;
+        uint32_t bits = (uint32_t)h.prefix;
+        float tau;
+        memcpy(&tau, &bits, sizeof tau);
+        if (h.all) tau = -INFINITY;
+        // everything built so far fits: nothing can be pruned yet, go deeper at once
+        const int levels = h.all ? 4 * gkv::kMaxUnit : 2;
+        gkv::StageTimer tm(c, 3, s);
+        e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 1, levels, tau, w.u_list, h.count, s);
+        c.build_passes = it + 2;
     }
     if (e != cudaSuccess) return cuda_fail(x, e, "build_trees launch");
     c.stage = 2;
@@ -398,7 +427,8 @@ gkv_status gracekv_export(gracekv_ctx *x, int64_t node_cap, int64_t *n_nodes_hos
     std::vector<int32_t> slots(J + 1), nn(nu);
     std::vector<int32_t> ha(c.node_cap), hb(c.node_cap), hc(c.node_cap);
     std::vector<int8_t> hn(c.node_cap), hk(c.node_cap);
-    std::vector<float> hD(c.node_cap), hR(c.node_cap), hU(c.node_cap), hK(c.node_cap);
+    std::vector<double> hD(c.node_cap);
+    std::vector<float> hR(c.node_cap), hU(c.node_cap), hK(c.node_cap);
     std::vector<uint8_t> hs(c.node_cap);
     cudaError_t e = cudaStreamSynchronize(s);
 #define CP(dst, src, n) if (e == cudaSuccess) e = cudaMemcpy(dst, src, (n) * sizeof(*(dst)), cudaMemcpyDeviceToHost)
@@ -432,7 +462,7 @@ gkv_status gracekv_export(gracekv_ctx *x, int64_t node_cap, int64_t *n_nodes_hos
             if (child0) child0[k] = hc[v];
             if (nchild) nchild[k] = hn[v];
             if (cost) cost[k] = hk[v];
-            if (D) D[k] = hD[v];
+            if (D) D[k] = (float)hD[v];
             if (R) R[k] = hR[v];
             if (U) U[k] = hU[v];
             if (kappa) kappa[k] = hK[v];

@@ -3,7 +3,7 @@
 // CTA that keeps the whole slot in shared memory.
 //
 // Per unit (l, g, j), slot [sa, sb), n <= 128 tokens:
-//   E[u][t] = exp(q_u . k_t / sqrt d - m_u)   distortion probe u uses query
+//   E[t][u] = exp(q_u . k_t / sqrt d - m_u)   distortion probe u uses query
 //             head H(g)[u mod |H(g)|] (App. A.3, GQA round robin), m_u its
 //             max logit over [0, T)
 //   k_circ_t = RoPE^-1(k_t, t)                 (Eq. app_rope_prototype)
@@ -23,15 +23,21 @@
 // Eqs. app_operation_gains .. app_unit_utility (clamped at 0); each Split op
 // also gets its bottleneck key kappa = min(U, kappa of the op that created
 // the node), which the allocator's threshold select uses.
+//
+// Pruned construction.  A launch evaluates at most `max_levels` levels; the
+// nodes below stay pending (child count -1, no Split op yet) and each unit
+// reports the largest key of the ops that created its pending nodes.  The
+// host then computes the allocation threshold tau over the ops built so far
+// -- tau can only grow as ops are added, so it never exceeds the final
+// threshold -- and resumes only the pending nodes whose creator has a key
+// >= tau: a node whose creator's key is below the final threshold never
+// reaches the frontier before the allocation stops, so its own Split is never
+// needed.  Resuming repeats until no pending node qualifies.
 #include "gkv_internal.cuh"
 
 namespace gkv {
 namespace {
 
-constexpr int kThreads = 256;
-constexpr int kWarps = kThreads / 32;
-constexpr int kNCmax = 48;       // candidate intervals per batch (at least 2*17+3 = 37 per node)
-constexpr int kNB = 32;          // nodes per batch
 constexpr int kMaxCuts = 18;     // K + midpoint, K <= 16 (+1 spare)
 constexpr int kMaxNodes = 2 * kMaxUnit;
 
@@ -44,30 +50,37 @@ struct BuildArgs {
     int L, G, Hq, T, d, W, gq, cs, Nc, J, k_cand;
     float inv_sqrt_d, lamZ, lamM, eps;
     double lam_kappa, base_frac, eps_d;
+    // pruning
+    int resume;                  // 0: build from the root, 1: resume pending nodes
+    int max_levels;              // levels evaluated by this launch
+    float tau;                   // resume: evaluate pending nodes whose creator key >= tau
+    const int32_t *unit_list;    // resume: units to process (blockIdx.x indexes it)
     // outputs
     int32_t *nd_a, *nd_b, *nd_child0, *nd_parent, *nd_unit;
     int8_t *nd_nchild, *nd_cost;
-    float *nd_D, *nd_R, *nd_U, *nd_kappa;
+    double *nd_D;
+    float *nd_R, *nd_U, *nd_kappa;
     uint8_t *nd_sel;
     int32_t *u_nnodes;
-    float *u_Uadd, *u_Ddrop;
+    float *u_Uadd, *u_Ddrop, *u_pend;
     uint8_t *u_sel;
     int *status;
     unsigned long long *work;
 };
 
 struct NodeS {
-    int a, b, parent, child0, nchild;
+    short a, b, parent, child0;
+    signed char nchild;          // -1: pending (not evaluated)
+    float kin;                   // bottleneck key of the op that created the node
     double D, R;
-    float kin;       // bottleneck key of the op that created the node
 };
 
 struct BatchNode {
     int node;
     int ncut;
-    int cut[kMaxCuts];      // local cut positions xi (ascending)
-    int pidx[kMaxCuts];     // candidate index of [a, xi) (-1: single token)
-    int sidx[kMaxCuts];     // candidate index of [xi, b) (-1: single token)
+    short cut[kMaxCuts];     // local cut positions xi (ascending)
+    short pidx[kMaxCuts];    // candidate index of [a, xi) (-1: single token)
+    short sidx[kMaxCuts];    // candidate index of [xi, b) (-1: single token)
     int pstar, eL, eR, whole;
     int pre_b, pre_e, suf_b, suf_e;   // candidate ranges (prefixes ascending end,
                                       // suffixes descending start)
@@ -81,6 +94,17 @@ struct Cand {
     float meff;
 };
 
+// Order-preserving 64-bit key of a double (larger value -> larger key), so
+// that curvature ranks compare exactly like the fp64 values with integer ops.
+__device__ __forceinline__ unsigned long long okey(double x) {
+    unsigned long long u = (unsigned long long)__double_as_longlong(x);
+    return (u >> 63) ? ~u : (u | 0x8000000000000000ull);
+}
+__device__ __forceinline__ double okey_inv(unsigned long long k) {
+    unsigned long long u = (k >> 63) ? (k & 0x7fffffffffffffffull) : ~k;
+    return __longlong_as_double((long long)u);
+}
+
 __device__ __forceinline__ int round_half_even_mid(int a, int b) {
     int s = a + b - 1;
     if ((s & 1) == 0) return s >> 1;
@@ -88,41 +112,54 @@ __device__ __forceinline__ int round_half_even_mid(int a, int b) {
     return (lo & 1) == 0 ? lo : lo + 1;
 }
 
-template <int DH, int NW, typename Tin>
+template <int DH, int NW, typename Tin, int NT>
 struct Smem {
-    static constexpr int NCH = kThreads / NW;
-    static constexpr int CH = DH / NCH;
-    // fp32 slots of d = 128 with 64 probes leave room for 38 candidates only
-    static constexpr int NC = (DH == 128 && NW == 64 && sizeof(Tin) == 4) ? 38 : kNCmax;
-    static_assert(NC >= 37, "one node needs up to 2 * 17 + 3 candidate intervals");
+    static constexpr int NWARPS = NT / 32;
+    static constexpr int NCH = NT / NW;      // threads per probe
+    static constexpr int CH = DH / NCH;      // elements per thread
+    // candidate capacity: at least 2*17+3 = 37 (one node); less where the slot
+    // arrays are fp32 with 64 probes
+    static constexpr int NC = (DH == 128 && NW == 64 && sizeof(Tin) == 4) ? 37 : 48;
+    static constexpr int NB = (DH == 128 && NW == 64 && sizeof(Tin) == 4) ? 24 : 32;
     float kc[kMaxUnit][DH];
     Tin vv[kMaxUnit][DH];
-    float E[NW][kMaxUnit];
+    float E[kMaxUnit][NW];
     float ktil[NC][DH];
     float vtil[NC][DH];
     float Rt[kMaxUnit];
     float kn[kMaxUnit];
-    double kap[kMaxUnit];
-    float redD[NC][kWarps];
-    float redP[NC][kWarps];
+    unsigned long long kap[kMaxUnit];   // order-preserving keys of the curvature
+    float redD[NC][NWARPS];
+    float redP[NC][NWARPS];
+    double candD[NC], candP[NC];        // per-candidate D and drop mass
     Cand cand[NC];
     NodeS nodes[kMaxNodes];
-    BatchNode bn[kNB];
+    BatchNode bn[NB];
     short lvl[2][kMaxNodes];
     int nlvl[2];
     int nnodes;
-    int batch_n, batch_next, ncand;
+    int batch_n, batch_next;
+    float pend;
 };
 
-template <int DH, int NW, typename Tin>
-__global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
-    using S = Smem<DH, NW, Tin>;
-    constexpr int NCH = S::NCH, CH = S::CH, HALF = DH / 2;
+template <int DH, int NW, typename Tin, int NT>
+__global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
+    using S = Smem<DH, NW, Tin, NT>;
+    constexpr int NCH = S::NCH, CH = S::CH, HALF = DH / 2, NWARPS = S::NWARPS;
+    static_assert(NCH <= 32 && (32 % NCH) == 0 && CH >= 1, "probe layout");
     extern __shared__ __align__(16) unsigned char smem_raw[];
     S &sm = *reinterpret_cast<S *>(smem_raw);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int LG = A.L * A.G;
-    const int j = blockIdx.x / LG, lg = blockIdx.x - j * LG;
+    int j, lg;
+    if (A.resume) {
+        const int uidr = A.unit_list[blockIdx.x];
+        lg = uidr / A.J;
+        j = uidr - lg * A.J;
+    } else {
+        j = blockIdx.x / LG;   // slot-major: the units of a slot share its table rows
+        lg = blockIdx.x - j * LG;
+    }
     const int l = lg / A.G, g = lg - l * A.G;
     const int sa = A.slots[j], sb = A.slots[j + 1];
     const int n = sb - sa;
@@ -137,7 +174,7 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
     const float om = A.omega ? A.omega[lg] : 1.0f;
 
     // ---- load the slot ------------------------------------------------------
-    for (int e = tid * 8; e < n * DH; e += kThreads * 8) {
+    for (int e = tid * 8; e < n * DH; e += NT * 8) {
         Vec8<Tin> kx, vx;
         kx.load(Kp + e);
         vx.load(Vp + e);
@@ -148,11 +185,11 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
             sm.vv[t][i + q] = (Tin)vx.v[q];
         }
     }
-    for (int t = tid; t < n; t += kThreads) {
-        sm.kap[t] = A.kappa[sa + t];
+    for (int t = tid; t < n; t += NT) {
+        sm.kap[t] = okey(A.kappa[sa + t]);
         sm.Rt[t] = A.rtok[(size_t)lg * A.Nc + (sa - A.cs) + t];
     }
-    // probe registers: thread (u, c) owns chunk c of probe u
+    // probe registers: thread (u, c) owns elements c + NCH q of probe u
     const int u = tid / NCH, c = tid - u * NCH;
     const bool pact = u < A.W;
     float qreg[CH];
@@ -161,31 +198,26 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
         const int h = g * A.gq + (u % A.gq);
         const size_t row = ((size_t)l * A.Hq + h) * A.W + u;
         if (pact) {
-            const Tin *qp = static_cast<const Tin *>(A.Q) + row * DH + c * CH;
+            const Tin *qp = static_cast<const Tin *>(A.Q) + row * DH;
 #pragma unroll
-            for (int k = 0; k < CH; k += 8) {
-                Vec8<Tin> x;
-                x.load(qp + k);
-#pragma unroll
-                for (int q = 0; q < 8; q++) qreg[k + q] = x.v[q];
-            }
+            for (int q = 0; q < CH; q++) qreg[q] = to_f(qp[c + NCH * q]);
             mu = A.row_m[row];
             invZ = 1.0f / A.row_Z[row];
         } else {
 #pragma unroll
-            for (int k = 0; k < CH; k++) qreg[k] = 0.f;
+            for (int q = 0; q < CH; q++) qreg[q] = 0.f;
         }
     }
     __syncthreads();
 
-    // ---- E[u][t] from the raw (post-RoPE) keys -------------------------------
+    // ---- E[t][u] from the raw (post-RoPE) keys -------------------------------
     for (int t = 0; t < n; t++) {
         float x = 0.f;
 #pragma unroll
-        for (int k = 0; k < CH; k++) x = fmaf(qreg[k], sm.kc[t][c * CH + k], x);
+        for (int q = 0; q < CH; q++) x = fmaf(qreg[q], sm.kc[t][c + NCH * q], x);
 #pragma unroll
         for (int o = 1; o < NCH; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-        if (c == 0) sm.E[u][t] = pact ? expf(x * A.inv_sqrt_d - mu) : 0.f;
+        if (c == 0) sm.E[t][u] = pact ? expf(x * A.inv_sqrt_d - mu) : 0.f;
     }
     __syncthreads();
     // Non-finite probe weights or token values (NaN/Inf in K, Q or the row
@@ -194,26 +226,24 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
     // the host reports as GKV_ENONFINITE at the allocation's count sync.
     {
         bool bad = false;
-        for (int e = tid; e < n * NW; e += kThreads) {
-            float v = sm.E[e / n][e % n];
-            bad |= !isfinite(v);
-        }
-        for (int t = tid; t < n; t += kThreads) bad |= !isfinite(sm.Rt[t]);
+        for (int e = tid; e < n * NW; e += NT) bad |= !isfinite(sm.E[e / NW][e % NW]);
+        for (int t = tid; t < n; t += NT) bad |= !isfinite(sm.Rt[t]);
         if (__syncthreads_or(bad)) {
             if (tid == 0) {
                 atomicOr(A.status, 8);
-                A.nd_a[nbase] = sa; A.nd_b[nbase] = sb; A.nd_R[nbase] = 0.f; A.nd_D[nbase] = 0.f;
+                A.nd_a[nbase] = sa; A.nd_b[nbase] = sb; A.nd_R[nbase] = 0.f; A.nd_D[nbase] = 0.0;
                 A.nd_parent[nbase] = (int32_t)(-2 - uid); A.nd_unit[nbase] = (int32_t)uid;
                 A.nd_child0[nbase] = -1; A.nd_nchild[nbase] = 0; A.nd_U[nbase] = 0.f;
                 A.nd_kappa[nbase] = 0.f; A.nd_sel[nbase] = 0;
                 A.u_nnodes[uid] = 1; A.u_Uadd[uid] = 0.f; A.u_Ddrop[uid] = 0.f; A.u_sel[uid] = 0;
+                A.u_pend[uid] = -1.f;
             }
-            for (int k = tid; k < 2 * n; k += kThreads) A.nd_cost[nbase + k] = 0;
+            for (int k = tid; k < 2 * n; k += NT) A.nd_cost[nbase + k] = 0;
             return;
         }
     }
     // ---- k_circ = RoPE^-1(k, t) ----------------------------------------------
-    for (int e = tid; e < n * HALF; e += kThreads) {
+    for (int e = tid; e < n * HALF; e += NT) {
         int t = e / HALF, i = e - t * HALF;
         float2 cs = A.rope[(size_t)(sa + t) * HALF + i];
         float x = sm.kc[t][i], y = sm.kc[t][i + HALF];
@@ -221,45 +251,96 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
         sm.kc[t][i + HALF] = y * cs.x - x * cs.y;
     }
     __syncthreads();
-    for (int t = warp; t < n; t += kWarps) {
+    for (int t = warp; t < n; t += NWARPS) {
         float s = 0.f;
         for (int i = lane; i < DH; i += 32) s = fmaf(sm.kc[t][i], sm.kc[t][i], s);
         s = warp_sum(s);
         if (lane == 0) sm.kn[t] = sqrtf(s);
     }
-    // ---- root -----------------------------------------------------------------
-    if (warp == 0) {
-        double r = 0.0;
-        for (int t = lane; t < n; t += 32) r += sm.Rt[t];
-        r = warp_sum(r);
-        if (lane == 0) {
-            NodeS &nd = sm.nodes[0];
-            nd.a = 0; nd.b = n; nd.parent = -1; nd.child0 = -1; nd.nchild = 0;
-            nd.D = 0.0; nd.R = r; nd.kin = 0.f;
-            sm.nnodes = 1;
-            sm.lvl[0][0] = 0;
-            sm.nlvl[0] = 1;
-            A.nd_a[nbase] = sa; A.nd_b[nbase] = sb; A.nd_R[nbase] = (float)r;
-            A.nd_parent[nbase] = (int32_t)(-2 - uid);
-            A.nd_unit[nbase] = (int32_t)uid;
+    // ---- tree state: a fresh root, or the unit's records so far --------------
+    if (!A.resume) {
+        if (warp == 0) {
+            double r = 0.0;
+            for (int t = lane; t < n; t += 32) r += sm.Rt[t];
+            r = warp_sum(r);
+            if (lane == 0) {
+                NodeS &nd = sm.nodes[0];
+                nd.a = 0; nd.b = (short)n; nd.parent = -1; nd.child0 = -1; nd.nchild = 0;
+                nd.D = 0.0; nd.R = r; nd.kin = 0.f;
+                sm.nnodes = 1;
+                sm.lvl[0][0] = 0;
+                sm.nlvl[0] = 1;
+                sm.pend = -1.f;
+                A.nd_a[nbase] = sa; A.nd_b[nbase] = sb; A.nd_R[nbase] = (float)r;
+                A.nd_parent[nbase] = (int32_t)(-2 - uid);
+                A.nd_unit[nbase] = (int32_t)uid;
+            }
+        }
+    } else {
+        const int nn = A.u_nnodes[uid];
+        for (int k = tid; k < nn; k += NT) {
+            const int64_t v = nbase + k;
+            NodeS &nd = sm.nodes[k];
+            nd.a = (short)(A.nd_a[v] - sa);
+            nd.b = (short)(A.nd_b[v] - sa);
+            int32_t pg = A.nd_parent[v];
+            nd.parent = pg < 0 ? (short)-1 : (short)(pg - nbase);
+            nd.child0 = (short)A.nd_child0[v];
+            nd.nchild = A.nd_nchild[v];
+            nd.D = A.nd_D[v];
+            nd.R = 0.0;
+            nd.kin = pg < 0 ? A.u_Uadd[uid] : A.nd_kappa[pg];
+        }
+        if (tid == 0) { sm.nnodes = nn; sm.nlvl[0] = 0; sm.pend = -1.f; }
+        __syncthreads();
+        if (tid == 0) {   // pending nodes that qualify, in creation order
+            for (int k = 0; k < nn; k++) {
+                const NodeS &nd = sm.nodes[k];
+                if (nd.nchild != -1) continue;
+                if (nd.kin >= A.tau) sm.lvl[0][sm.nlvl[0]++] = (short)k;
+                else sm.pend = fmaxf(sm.pend, nd.kin);
+            }
+        }
+        __syncthreads();
+        for (int q = warp; q < sm.nlvl[0]; q += NWARPS) {   // node values of the resumed nodes
+            NodeS &nd = sm.nodes[sm.lvl[0][q]];
+            double r = 0.0;
+            for (int t = nd.a + lane; t < nd.b; t += 32) r += sm.Rt[t];
+            r = warp_sum(r);
+            if (lane == 0) nd.R = r;
         }
     }
     __syncthreads();
 
     unsigned long long w_scan = 0, w_eval = 0, w_len = 0;   // thread 0's work counters
     int cur = 0;
+    int levels_left = A.max_levels;
     while (sm.nlvl[cur] > 0) {
         const int nl = sm.nlvl[cur];
+        if (levels_left == 0) {   // depth limit: the level's nodes stay pending
+            if (tid == 0) {
+                float pm = sm.pend;
+                for (int k = 0; k < nl; k++) {
+                    const int v = sm.lvl[cur][k];
+                    A.nd_nchild[nbase + v] = -1;
+                    pm = fmaxf(pm, sm.nodes[v].kin);
+                }
+                sm.pend = pm;
+            }
+            break;
+        }
+        levels_left--;
         if (tid == 0) { sm.nlvl[cur ^ 1] = 0; sm.batch_next = 0; }
         __syncthreads();
         while (sm.batch_next < nl) {
             // ---- batch assignment (thread 0) --------------------------------
             if (tid == 0) {
                 int nb = 0, used = 0, k = sm.batch_next;
-                while (k < nl && nb < kNB) {
+                while (k < nl && nb < S::NB) {
                     int v = sm.lvl[cur][k];
                     int nv = sm.nodes[v].b - sm.nodes[v].a;
-                    int ub = (v == 0 ? 1 : 0) + (nv >= 3 ? 2 * min(A.k_cand + 1, nv - 1) + 2 : 0);
+                    bool root = v == 0 && !A.resume;
+                    int ub = (root ? 1 : 0) + (nv >= 3 ? 2 * min(A.k_cand + 1, nv - 1) + 2 : 0);
                     if (used + ub > S::NC) break;
                     sm.bn[nb].node = v;
                     sm.bn[nb].pre_b = used;
@@ -269,30 +350,29 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
                 }
                 sm.batch_n = nb;
                 sm.batch_next = k;
-                sm.ncand = used;
             }
             __syncthreads();
             const int nb = sm.batch_n;
             // ---- phase A: cut candidates per node (warp per node) ------------
-            for (int bi = warp; bi < nb; bi += kWarps) {
+            for (int bi = warp; bi < nb; bi += NWARPS) {
                 BatchNode &B = sm.bn[bi];
                 const int v = B.node;
                 const int a = sm.nodes[v].a, b = sm.nodes[v].b, nv = b - a;
                 // top-K by curvature over positions [a, b-2] (ties: lower t)
                 unsigned sel[kMaxUnit / 32];
-                double kmin = INFINITY, kmax = -INFINITY;
+                unsigned long long kmin = ~0ull, kmax = 0ull;
 #pragma unroll
                 for (int w = 0; w < kMaxUnit / 32; w++) {
                     int t = a + w * 32 + lane;
                     bool in = t <= b - 2;
                     bool s = false;
                     if (in) {
-                        double kt = sm.kap[t];
-                        kmin = fmin(kmin, kt);
-                        kmax = fmax(kmax, kt);
+                        const unsigned long long kt = sm.kap[t];
+                        kmin = min(kmin, kt);
+                        kmax = max(kmax, kt);
                         int rank = 0;
                         for (int q = a; q <= b - 2; q++) {
-                            double kq = sm.kap[q];
+                            const unsigned long long kq = sm.kap[q];
                             rank += (kq > kt) || (kq == kt && q < t);
                         }
                         s = rank < A.k_cand || t == a + nv / 2 - 1;   // + midpoint
@@ -301,8 +381,8 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
                 }
 #pragma unroll
                 for (int o = 16; o > 0; o >>= 1) {
-                    kmin = fmin(kmin, __shfl_xor_sync(0xffffffffu, kmin, o));
-                    kmax = fmax(kmax, __shfl_xor_sync(0xffffffffu, kmax, o));
+                    kmin = min(kmin, __shfl_xor_sync(0xffffffffu, kmin, o));
+                    kmax = max(kmax, __shfl_xor_sync(0xffffffffu, kmax, o));
                 }
                 // salient token p* = argmax R_tok over [a, b) (ties: lower t)
                 float rb = -INFINITY;
@@ -319,8 +399,8 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
                 }
                 if (pb < a || pb >= b) pb = a;   // only reachable with non-finite values
                 if (lane == 0) {
-                    B.kmin = kmin;
-                    B.kmax = kmax;
+                    B.kmin = nv >= 2 ? okey_inv(kmin) : 0.0;
+                    B.kmax = nv >= 2 ? okey_inv(kmax) : 0.0;
                     B.pstar = pb;
                     B.ncut = 0;
                     B.eL = B.eR = B.whole = -1;
@@ -333,7 +413,7 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
                                 int bit = __ffs(m) - 1;
                                 m &= m - 1;
                                 if (B.ncut < min(A.k_cand + 1, nv - 1))
-                                    B.cut[B.ncut++] = a + w * 32 + bit + 1;
+                                    B.cut[B.ncut++] = (short)(a + w * 32 + bit + 1);
                             }
                         }
                         // prefixes in ascending end: cuts merged with the extraction's left side
@@ -345,13 +425,13 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
                                 else { sm.cand[k] = {a, pb, 0.f}; B.eL = k++; }
                                 el_done = true;
                             }
-                            if (xi - a >= 2) { sm.cand[k] = {a, xi, 0.f}; B.pidx[q] = k++; }
+                            if (xi - a >= 2) { sm.cand[k] = {a, xi, 0.f}; B.pidx[q] = (short)k++; }
                             else B.pidx[q] = -1;
                         }
                         if (!el_done) { sm.cand[k] = {a, pb, 0.f}; B.eL = k++; }
                         if (B.eL <= -2) B.eL = B.pidx[-2 - B.eL];
                     }
-                    if (v == 0) { sm.cand[k] = {a, b, 0.f}; B.whole = k++; }
+                    if (v == 0 && !A.resume) { sm.cand[k] = {a, b, 0.f}; B.whole = k++; }
                     B.pre_e = k;
                     B.suf_b = k;
                     if (cands) {
@@ -365,7 +445,7 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
                                 else { sm.cand[k] = {er, b, 0.f}; B.eR = k++; }
                                 er_done = true;
                             }
-                            if (b - xi >= 2) { sm.cand[k] = {xi, b, 0.f}; B.sidx[q] = k++; }
+                            if (b - xi >= 2) { sm.cand[k] = {xi, b, 0.f}; B.sidx[q] = (short)k++; }
                             else B.sidx[q] = -1;
                         }
                         if (!er_done) { sm.cand[k] = {er, b, 0.f}; B.eR = k++; }
@@ -378,16 +458,16 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
             // ---- phase B: prototype of every candidate (warp per candidate) ----
             for (int bi = 0; bi < nb; bi++) {
                 const BatchNode &B = sm.bn[bi];
-                for (int k = B.pre_b + warp; k < B.suf_e; k += kWarps) {
+                for (int k = B.pre_b + warp; k < B.suf_e; k += NWARPS) {
                     const int ja = sm.cand[k].a, jb = sm.cand[k].b, nJ = jb - ja;
-                    double rs = 0.0, ks = 0.0;
+                    float rs = 0.f, ks = 0.f;
                     for (int t = ja + lane; t < jb; t += 32) { rs += sm.Rt[t]; ks += sm.kn[t]; }
                     rs = warp_sum(rs);
                     ks = warp_sum(ks);
-                    const float beta = (float)(A.base_frac * (rs / nJ));
-                    const double wsum = rs + nJ * (double)beta;
-                    const float winv = (float)(1.0 / (wsum + A.eps_d));
                     const float ninv = 1.0f / (float)nJ;
+                    const float beta = (float)A.base_frac * (rs * ninv);
+                    const float wsum = rs + (float)nJ * beta;
+                    const float winv = 1.0f / (wsum + A.eps);
                     const int p = round_half_even_mid(sa + ja, sa + jb);   // absolute positions
                     float mu2 = 0.f;
                     for (int i = lane; i < HALF; i += 32) {
@@ -410,9 +490,9 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
                     }
                     mu2 = warp_sum(mu2);
                     if (lane == 0) {
-                        double coh = sqrt((double)mu2) / (ks / nJ + A.eps_d);
-                        double me = nJ * coh * coh;
-                        sm.cand[k].meff = (float)(me < 1.0 ? 1.0 : (me > nJ ? (double)nJ : me));
+                        const float coh = sqrtf(mu2) / (ks * ninv + A.eps);
+                        const float me = (float)nJ * coh * coh;
+                        sm.cand[k].meff = me < 1.0f ? 1.0f : (me > (float)nJ ? (float)nJ : me);
                     }
                 }
             }
@@ -421,14 +501,14 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
             auto evaluate = [&](int k, float Z, const float *M) {
                 float x = 0.f;
 #pragma unroll
-                for (int q = 0; q < CH; q++) x = fmaf(qreg[q], sm.ktil[k][c * CH + q], x);
+                for (int q = 0; q < CH; q++) x = fmaf(qreg[q], sm.ktil[k][c + NCH * q], x);
 #pragma unroll
                 for (int o = 1; o < NCH; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
                 const float zt = sm.cand[k].meff * expf(x * A.inv_sqrt_d - mu);
                 float res = 0.f, mm = 0.f;
 #pragma unroll
                 for (int q = 0; q < CH; q++) {
-                    float df = M[q] - zt * sm.vtil[k][c * CH + q];
+                    float df = M[q] - zt * sm.vtil[k][c + NCH * q];
                     res = fmaf(df, df, res);
                     mm = fmaf(M[q], M[q], mm);
                 }
@@ -470,10 +550,10 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
 #pragma unroll
                     for (int q = 0; q < CH; q++) M[q] = 0.f;
                     for (int t = a; t < b && k < B.pre_e; t++) {
-                        const float e = sm.E[u][t];
+                        const float e = sm.E[t][u];
                         Z += e;
 #pragma unroll
-                        for (int q = 0; q < CH; q++) M[q] = fmaf(e, to_f(sm.vv[t][c * CH + q]), M[q]);
+                        for (int q = 0; q < CH; q++) M[q] = fmaf(e, to_f(sm.vv[t][c + NCH * q]), M[q]);
                         while (k < B.pre_e && sm.cand[k].b == t + 1) { evaluate(k, Z, M); k++; }
                     }
                 }
@@ -484,72 +564,92 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
 #pragma unroll
                     for (int q = 0; q < CH; q++) M[q] = 0.f;
                     for (int t = b - 1; t >= a && k < B.suf_e; t--) {
-                        const float e = sm.E[u][t];
+                        const float e = sm.E[t][u];
                         Z += e;
 #pragma unroll
-                        for (int q = 0; q < CH; q++) M[q] = fmaf(e, to_f(sm.vv[t][c * CH + q]), M[q]);
+                        for (int q = 0; q < CH; q++) M[q] = fmaf(e, to_f(sm.vv[t][c + NCH * q]), M[q]);
                         while (k < B.suf_e && sm.cand[k].a == t) { evaluate(k, Z, M); k++; }
                     }
                 }
             }
             __syncthreads();
-            // ---- phase D1: decisions (warp per node, lane 0) --------------------
-            for (int bi = warp; bi < nb; bi += kWarps) {
-                if (lane) continue;
+            // ---- per-candidate D and drop mass (thread per candidate) ------------
+            for (int k = tid; k < sm.bn[nb - 1].suf_e; k += NT) {
+                double d = 0.0, pp = 0.0;
+#pragma unroll
+                for (int w = 0; w < NWARPS; w++) { d += sm.redD[k][w]; pp += sm.redP[k][w]; }
+                sm.candD[k] = d / A.W;
+                sm.candP[k] = pp / A.W;
+            }
+            __syncthreads();
+            // ---- phase D1: decisions (warp per node) ------------------------------
+            for (int bi = warp; bi < nb; bi += NWARPS) {
                 BatchNode &B = sm.bn[bi];
                 NodeS &nd = sm.nodes[B.node];
                 const int a = nd.a, b = nd.b, nv = b - a;
-                auto Dc = [&](int k) -> double {
-                    double s = 0.0;
-                    for (int w = 0; w < kWarps; w++) s += sm.redD[k][w];
-                    return s / A.W;
-                };
-                if (B.whole >= 0) {   // root: D, Ddrop, Add gain (Eq. app_operation_gains)
-                    double Pd = 0.0;
-                    for (int w = 0; w < kWarps; w++) Pd += sm.redP[B.whole][w];
-                    Pd /= A.W;
-                    double D = nv >= 2 ? Dc(B.whole) : 0.0;
+                if (B.whole >= 0 && lane == 0) {   // root: D, Ddrop, Add gain (Eq. app_operation_gains)
+                    const double Pd = sm.candP[B.whole];
+                    const double D = nv >= 2 ? sm.candD[B.whole] : 0.0;
                     nd.D = D;
                     double gain = (double)om * nd.R * (Pd - D);
                     if (gain < 0.0) gain = 0.0;
                     nd.kin = (float)gain;
                     A.u_Uadd[uid] = (float)gain;
                     A.u_Ddrop[uid] = (float)Pd;
-                    A.nd_D[nbase] = (float)D;
+                    A.nd_D[nbase] = D;
                 }
-                B.nchild = 0;
-                if (nv < 2) continue;
-                const double DI = nd.D;
-                if (nv == 2) {
-                    B.nchild = 2;
-                    B.ca[0] = a; B.cb[0] = a + 1; B.cD[0] = 0.0;
-                    B.ca[1] = a + 1; B.cb[1] = b; B.cD[1] = 0.0;
+                __syncwarp();
+                if (nv < 3) {
+                    if (lane == 0) {
+                        B.nchild = 0;
+                        if (nv == 2) {
+                            B.nchild = 2;
+                            B.ca[0] = a; B.cb[0] = a + 1; B.cD[0] = 0.0;
+                            B.ca[1] = a + 1; B.cb[1] = b; B.cD[1] = 0.0;
+                        }
+                    }
                     continue;
                 }
-                // binary cut: max G_bin, ties -> smallest xi
-                double best = -INFINITY, bL = 0, bR = 0;
+                const double DI = nd.D;
+                // binary cut: lane q evaluates cut q; max G_bin, ties -> smallest xi
+                double best = -INFINITY;
+                int bq = 0x7fffffff;
+                if (lane < B.ncut) {
+                    const int xi = B.cut[lane];
+                    const double DL = B.pidx[lane] >= 0 ? sm.candD[B.pidx[lane]] : 0.0;
+                    const double DR = B.sidx[lane] >= 0 ? sm.candD[B.sidx[lane]] : 0.0;
+                    const double kh = B.kmax > B.kmin
+                                          ? (okey_inv(sm.kap[xi - 1]) - B.kmin) / (B.kmax - B.kmin) : 0.0;
+                    best = ((DI - DL) - DR) + A.lam_kappa * kh;
+                    bq = lane;
+                }
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) {
+                    double ov = __shfl_xor_sync(0xffffffffu, best, o);
+                    int oq = __shfl_xor_sync(0xffffffffu, bq, o);
+                    if (ov > best || (ov == best && oq < bq)) { best = ov; bq = oq; }
+                }
+                if (lane) continue;
                 int bxi = -1;
-                for (int q = 0; q < B.ncut; q++) {
-                    int xi = B.cut[q];
-                    double DL = B.pidx[q] >= 0 ? Dc(B.pidx[q]) : 0.0;
-                    double DR = B.sidx[q] >= 0 ? Dc(B.sidx[q]) : 0.0;
-                    double kh = B.kmax > B.kmin ? (sm.kap[xi - 1] - B.kmin) / (B.kmax - B.kmin) : 0.0;
-                    double gb = ((DI - DL) - DR) + A.lam_kappa * kh;
-                    if (gb > best) { best = gb; bxi = xi; bL = DL; bR = DR; }
+                double bL = 0, bR = 0;
+                if (bq < B.ncut && best > -INFINITY) {
+                    bxi = B.cut[bq];
+                    bL = B.pidx[bq] >= 0 ? sm.candD[B.pidx[bq]] : 0.0;
+                    bR = B.sidx[bq] >= 0 ? sm.candD[B.sidx[bq]] : 0.0;
                 }
                 // extraction at p*
                 const int ps = B.pstar;
                 int ea[3], eb[3], ne = 0;
                 double eD[3];
-                if (ps > a) { ea[ne] = a; eb[ne] = ps; eD[ne] = ps - a >= 2 ? Dc(B.eL) : 0.0; ne++; }
+                if (ps > a) { ea[ne] = a; eb[ne] = ps; eD[ne] = ps - a >= 2 ? sm.candD[B.eL] : 0.0; ne++; }
                 ea[ne] = ps; eb[ne] = ps + 1; eD[ne] = 0.0; ne++;
-                if (ps + 1 < b) { ea[ne] = ps + 1; eb[ne] = b; eD[ne] = b - ps - 1 >= 2 ? Dc(B.eR) : 0.0; ne++; }
+                if (ps + 1 < b) { ea[ne] = ps + 1; eb[ne] = b; eD[ne] = b - ps - 1 >= 2 ? sm.candD[B.eR] : 0.0; ne++; }
                 double gext = DI;
                 for (int q = 0; q < ne; q++) gext -= eD[q];
                 if (bxi < 0) {   // only reachable with non-finite gains
                     bxi = B.cut[0];
-                    bL = B.pidx[0] >= 0 ? Dc(B.pidx[0]) : 0.0;
-                    bR = B.sidx[0] >= 0 ? Dc(B.sidx[0]) : 0.0;
+                    bL = B.pidx[0] >= 0 ? sm.candD[B.pidx[0]] : 0.0;
+                    bR = B.sidx[0] >= 0 ? sm.candD[B.sidx[0]] : 0.0;
                 }
                 const double rho_ext = gext / (ne - 1);
                 if (rho_ext > best) {
@@ -562,21 +662,21 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
                 }
             }
             __syncthreads();
-            // ---- child numbering (deterministic, breadth-first) ----------------
+            // ---- child numbering (deterministic, creation order) ----------------
             if (tid == 0) {
                 int cnt = sm.nnodes;
                 for (int bi = 0; bi < nb; bi++) {
                     BatchNode &B = sm.bn[bi];
                     NodeS &nd = sm.nodes[B.node];
-                    nd.nchild = B.nchild;
-                    nd.child0 = B.nchild ? cnt : -1;
+                    nd.nchild = (signed char)B.nchild;
+                    nd.child0 = B.nchild ? (short)cnt : (short)-1;
                     cnt += B.nchild;
                 }
                 sm.nnodes = cnt;
             }
             __syncthreads();
             // ---- phase D2: children, gains, keys (warp per node) ----------------
-            for (int bi = warp; bi < nb; bi += kWarps) {
+            for (int bi = warp; bi < nb; bi += NWARPS) {
                 const BatchNode &B = sm.bn[bi];
                 NodeS &nd = sm.nodes[B.node];
                 const int64_t gv = nbase + B.node;
@@ -607,12 +707,12 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
                     for (int q = 0; q < B.nchild; q++) {
                         int ci = nd.child0 + q;
                         NodeS &ch = sm.nodes[ci];
-                        ch.a = B.ca[q]; ch.b = B.cb[q]; ch.parent = B.node;
+                        ch.a = (short)B.ca[q]; ch.b = (short)B.cb[q]; ch.parent = (short)B.node;
                         ch.child0 = -1; ch.nchild = 0; ch.D = B.cD[q]; ch.R = rch[q]; ch.kin = kap;
                         const int64_t gc = nbase + ci;
                         A.nd_a[gc] = sa + ch.a; A.nd_b[gc] = sa + ch.b;
                         A.nd_parent[gc] = (int32_t)gv; A.nd_unit[gc] = (int32_t)uid;
-                        A.nd_D[gc] = (float)ch.D; A.nd_R[gc] = (float)ch.R;
+                        A.nd_D[gc] = ch.D; A.nd_R[gc] = (float)ch.R;
                         A.nd_child0[gc] = -1; A.nd_nchild[gc] = 0; A.nd_cost[gc] = 0;
                         A.nd_U[gc] = 0.f; A.nd_kappa[gc] = 0.f; A.nd_sel[gc] = 0;
                         if (ch.b - ch.a >= 2) {
@@ -637,43 +737,48 @@ __global__ void __launch_bounds__(kThreads, 1) unit_build_kernel(BuildArgs A) {
         __syncthreads();
         cur ^= 1;
     }
+    __syncthreads();
     if (tid == 0) {
         A.u_nnodes[uid] = sm.nnodes;
-        A.u_sel[uid] = 0;
+        A.u_pend[uid] = sm.pend;
+        if (!A.resume) A.u_sel[uid] = 0;
         atomicAdd(&A.work[0], w_scan);
         atomicAdd(&A.work[1], w_eval);
         atomicAdd(&A.work[2], w_len);
         atomicAdd(&A.work[3], 1ull);
     }
     // unused node slots of the unit carry cost 0 (no op)
-    for (int k = sm.nnodes + tid; k < 2 * n; k += kThreads) A.nd_cost[nbase + k] = 0;
+    if (!A.resume)
+        for (int k = sm.nnodes + tid; k < 2 * n; k += NT) A.nd_cost[nbase + k] = 0;
 }
 
 template <int DH, int NW, typename Tin>
-cudaError_t launch_t(Ctx &c, BuildArgs &A, int J, cudaStream_t s) {
-    using S = Smem<DH, NW, Tin>;
+cudaError_t launch_t(Ctx &c, BuildArgs &A, unsigned grid, cudaStream_t s) {
+    constexpr int NT = 512;
+    using S = Smem<DH, NW, Tin, NT>;
     static_assert(sizeof(S) <= 227 * 1024, "unit kernel shared memory above the per-CTA limit");
     size_t sm = sizeof(S);
-    cudaError_t e = cudaFuncSetAttribute(unit_build_kernel<DH, NW, Tin>,
+    cudaError_t e = cudaFuncSetAttribute(unit_build_kernel<DH, NW, Tin, NT>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
-    unsigned grid = (unsigned)((int64_t)J * c.p.L * c.p.G);
-    unit_build_kernel<DH, NW, Tin><<<grid, kThreads, sm, s>>>(A);
+    unit_build_kernel<DH, NW, Tin, NT><<<grid, NT, sm, s>>>(A);
     c.launches += 1;
     return cudaGetLastError();
 }
 
 template <typename Tin>
-cudaError_t launch_dt(Ctx &c, BuildArgs &A, int J, cudaStream_t s) {
+cudaError_t launch_dt(Ctx &c, BuildArgs &A, unsigned grid, cudaStream_t s) {
     int nw = c.p.W <= 32 ? 32 : 64;
-    if (c.p.d == 128) return nw == 32 ? launch_t<128, 32, Tin>(c, A, J, s) : launch_t<128, 64, Tin>(c, A, J, s);
-    return nw == 32 ? launch_t<64, 32, Tin>(c, A, J, s) : launch_t<64, 64, Tin>(c, A, J, s);
+    if (c.p.d == 128) return nw == 32 ? launch_t<128, 32, Tin>(c, A, grid, s) : launch_t<128, 64, Tin>(c, A, grid, s);
+    return nw == 32 ? launch_t<64, 32, Tin>(c, A, grid, s) : launch_t<64, 64, Tin>(c, A, grid, s);
 }
 
 }  // namespace
 
 cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *Q,
-                              const float *omega, const int32_t *slots, int J, cudaStream_t s) {
+                              const float *omega, const int32_t *slots, int J, int resume,
+                              int max_levels, float tau, const int32_t *unit_list, int n_list,
+                              cudaStream_t s) {
     const gkv_params &p = c.p;
     BuildArgs A;
     A.K = K; A.V = V; A.Q = Q;
@@ -684,17 +789,20 @@ cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *
     A.inv_sqrt_d = (float)(1.0 / sqrt((double)p.d));
     A.lamZ = (float)p.lambda_Z; A.lamM = (float)p.lambda_M; A.eps = (float)p.eps;
     A.lam_kappa = p.lambda_kappa; A.base_frac = p.base_frac; A.eps_d = p.eps;
+    A.resume = resume; A.max_levels = max_levels; A.tau = tau; A.unit_list = unit_list;
     A.nd_a = c.w.nd_a; A.nd_b = c.w.nd_b; A.nd_child0 = c.w.nd_child0;
     A.nd_parent = c.w.nd_parent; A.nd_unit = c.w.nd_unit;
     A.nd_nchild = c.w.nd_nchild; A.nd_cost = c.w.nd_cost;
     A.nd_D = c.w.nd_D; A.nd_R = c.w.nd_R; A.nd_U = c.w.nd_U; A.nd_kappa = c.w.nd_kappa;
     A.nd_sel = c.w.nd_sel;
     A.u_nnodes = c.w.u_nnodes; A.u_Uadd = c.w.u_Uadd; A.u_Ddrop = c.w.u_Ddrop; A.u_sel = c.w.u_sel;
+    A.u_pend = c.w.u_pend;
     A.status = c.w.dev_int + 1;
     A.work = c.w.work;
-    cudaMemsetAsync(c.w.work, 0, 4 * sizeof(unsigned long long), s);
-    if (p.dtype == GKV_BF16) return launch_dt<__nv_bfloat16>(c, A, J, s);
-    return launch_dt<float>(c, A, J, s);
+    unsigned grid = resume ? (unsigned)n_list : (unsigned)((int64_t)J * p.L * p.G);
+    if (grid == 0) return cudaSuccess;
+    if (p.dtype == GKV_BF16) return launch_dt<__nv_bfloat16>(c, A, grid, s);
+    return launch_dt<float>(c, A, grid, s);
 }
 
 }  // namespace gkv

@@ -46,12 +46,15 @@ struct Workspace {
     int32_t *nd_parent = nullptr;  // global index of the parent; roots: -2 - unit id
     int32_t *nd_unit = nullptr;    // unit id lg * J + j
     int8_t *nd_nchild = nullptr, *nd_cost = nullptr;
-    float *nd_D = nullptr, *nd_R = nullptr, *nd_U = nullptr, *nd_kappa = nullptr;
+    double *nd_D = nullptr;        // distortion D(I_v) of every node (fp64 so that resumed
+                                   // nodes see exactly the value their parent computed)
+    float *nd_R = nullptr, *nd_U = nullptr, *nd_kappa = nullptr;
     uint8_t *nd_sel = nullptr;     // split selected (1), discarded tie (2)
     // per-unit arrays (capacity units_cap), unit id = lg * J + j
     int64_t units_cap = 0;
     int32_t *u_nnodes = nullptr;
     float *u_Uadd = nullptr, *u_Ddrop = nullptr;
+    float *u_pend = nullptr;       // largest creator key of the unit's pending nodes (-1: none)
     uint8_t *u_sel = nullptr;      // Add selected (1), discarded tie (2)
     int32_t *u_count = nullptr;    // frontier entries per unit
     int64_t *u_off = nullptr;      // entry offset of each unit's frontier
@@ -81,6 +84,7 @@ struct Ctx {
     int n_chunks = 0;              // pass-A chunks per row
     // measurement
     int64_t launches = 0;          // kernels launched (host count)
+    int build_passes = 1;          // unit-kernel launches of the last build (pruning passes)
     bool profile = false;
     std::vector<cudaEvent_t> ev_pool;          // recorded (begin, end) pairs
     std::vector<int> ev_stage;                 // stage of each pair
@@ -173,7 +177,13 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
 cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t s);
 cudaError_t launch_token_values(Ctx &c, const void *K, const void *Q, cudaStream_t s);
 cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *Q,
-                              const float *omega, const int32_t *slots, int J, cudaStream_t s);
+                              const float *omega, const int32_t *slots, int J, int resume,
+                              int max_levels, float tau, const int32_t *unit_list, int n_list,
+                              cudaStream_t s);
+// Allocation threshold tau over the ops built so far (alloc_state prefix /
+// all-fit flag), and the list of units whose pending nodes qualify (key >= tau).
+cudaError_t launch_threshold(Ctx &c, int J, cudaStream_t s);
+cudaError_t launch_prune_list(Ctx &c, int J, int32_t *list, int *count, cudaStream_t s);
 
 cudaError_t launch_allocate(Ctx &c, int J, cudaStream_t s);
 cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *slots, int J,

@@ -118,6 +118,9 @@ def compare(g, o, dtype, report=None, require_exact_selection=True):
     rep["rtok_relerr"] = float(err.max())
     assert err.max() <= RTOK_RTOL, err.max()
     # -------- trees ---------------------------------------------------------
+    # The GPU builds trees lazily (pending nodes, child count -1, are the ones
+    # the allocation can never reach); every node it built must be the
+    # oracle's node of the same interval, with the same children.
     tr = o["trees"]
     ond = tr.nodes
     roots = list(tr.unit_root) + [len(ond["a"])]
@@ -126,65 +129,75 @@ def compare(g, o, dtype, report=None, require_exact_selection=True):
     assert len(uf) == nu + 1
     excluded = set()
     worst_D = worst_U = 0.0
+    tau = oracle_tau(o)
+    mism = exempt = pruned = pending = 0
     for u in range(nu):
         gs, ge = uf[u], uf[u + 1]
         os_, oe = roots[u], roots[u + 1]
-        ga, gb, gn = ex["a"][gs:ge], ex["b"][gs:ge], ex["nchild"][gs:ge]
-        oa, ob, on = ond["a"][os_:oe], ond["b"][os_:oe], ond["nchild"][os_:oe]
-        if not (len(ga) == len(oa) and np.array_equal(ga, oa) and np.array_equal(gb, ob)
-                and np.array_equal(gn, on)):
-            # first node whose children differ: its decision margins decide
-            k = 0
-            n = min(len(ga), len(oa))
-            while k < n and ga[k] == oa[k] and gb[k] == ob[k]:
-                gc = ex["child0"][gs + k]
-                oc = ond["child0"][os_ + k] - os_
-                if gn[k] != on[k] or (gn[k] and (not np.array_equal(
-                        ga[gc:gc + gn[k]], oa[oc:oc + on[k]]) or not np.array_equal(
-                        gb[gc:gc + gn[k]], ob[oc:oc + on[k]]))):
-                    break
-                k += 1
-            v = os_ + k
+        okey = {(int(ond["a"][v]), int(ond["b"][v])): v for v in range(os_, oe)}
+        seen = set()
+        bad_node = None
+        for k in range(gs, ge):
+            key = (int(ex["a"][k]), int(ex["b"][k]))
+            assert key in okey, f"unit {u}: GPU node {key} is not a node of the oracle's tree"
+            v = okey[key]
+            seen.add(v)
+            gn = int(ex["nchild"][k])
+            if gn == -1:
+                pending += 1
+                continue
+            on = int(ond["nchild"][v])
+            gch = [(int(ex["a"][gs + ex["child0"][k] + q]), int(ex["b"][gs + ex["child0"][k] + q]))
+                   for q in range(gn)]
+            och = [(int(ond["a"][ond["child0"][v] + q]), int(ond["b"][ond["child0"][v] + q]))
+                   for q in range(on)]
+            if gch != och:
+                bad_node = v
+                break
+        if bad_node is not None:
+            v = bad_node
             margin = min(ond["m_cut"][v], ond["m_form"][v], ond["m_topk"][v], ond["m_ext"][v])
-            assert margin < NEAR_TIE, (f"unit {u}: tree differs at node [{oa[k]},{ob[k]}) "
+            assert margin < NEAR_TIE, (f"unit {u}: tree differs at node [{ond['a'][v]},{ond['b'][v]}) "
                                        f"without a near-tie (oracle margin {margin:.3e})")
             excluded.add(u)
             continue
-        oD, gD = ond["D"][os_:oe], ex["D"][gs:ge]
-        eD = np.abs(gD - oD) / np.maximum(np.abs(oD), 1e-30)
-        eD[oD == 0] = np.abs(gD[oD == 0])
-        worst_D = max(worst_D, float(eD.max()))
-        scale = np.maximum(ond["R"][os_:oe] * np.maximum(np.abs(oD), 1e-300), 1e-300)
-        # U is relative to R * max(D(v), sum D(children)) / cost
-        oU = ond["U"][os_:oe]
-        cst = np.maximum(ond["cost"][os_:oe], 1)
-        eU = np.abs(ex["U"][gs:ge] - oU) / (scale / cst)
-        worst_U = max(worst_U, float(eU.max()))
-    rep["units"] = nu
-    rep["units_excluded_near_tie"] = len(excluded)
-    rep["D_relerr"] = worst_D
-    rep["U_relerr"] = worst_U
-    assert worst_D <= D_RTOL, worst_D
-    assert worst_U <= U_RTOL, worst_U
-    # -------- selection -----------------------------------------------------
-    tau = oracle_tau(o)
-    mism = exempt = 0
-    for u in range(nu):
-        if u in excluded:
-            continue
-        gs, os_ = uf[u], roots[u]
-        n = uf[u + 1] - gs
+        # values of the built nodes
+        for k in range(gs, ge):
+            v = okey[(int(ex["a"][k]), int(ex["b"][k]))]
+            oD, gD = ond["D"][v], ex["D"][k]
+            eD = abs(gD - oD) / abs(oD) if oD != 0 else abs(gD)
+            worst_D = max(worst_D, eD)
+            if ex["nchild"][k] > 0:
+                scale = max(ond["R"][v] * max(abs(oD), 1e-300), 1e-300) / max(ond["cost"][v], 1)
+                worst_U = max(worst_U, abs(ex["U"][k] - ond["U"][v]) / scale)
+        # selection: Add, then every split the GPU built or pruned
         if int(ex["add_sel"][u] == 1) != int(o["add_sel"][u]):
             mism += 1
             if abs(tr.unit_Uadd[u] - tau) <= NEAR_TIE * max(abs(tau), 1e-300):
                 exempt += 1
-        gsel = (ex["split_sel"][gs:gs + n] == 1).astype(int)
-        osel = o["split_sel"][os_:os_ + n].astype(int)
-        for k in np.nonzero(gsel != osel)[0]:
-            mism += 1
-            v = os_ + k
-            if abs(ond["kappa"][v] - tau) <= NEAR_TIE * max(ond["kscale"][v], abs(tau), 1e-300):
-                exempt += 1
+        for v in range(os_, oe):
+            if v not in seen:
+                pruned += 1
+                assert o["split_sel"][v] == 0, f"unit {u}: a pruned node's split was selected by the heap"
+                continue
+        for k in range(gs, ge):
+            v = okey[(int(ex["a"][k]), int(ex["b"][k]))]
+            gsel = int(ex["split_sel"][k] == 1)
+            if ex["nchild"][k] == -1:
+                assert o["split_sel"][v] == 0, f"unit {u}: a pending node's split was selected by the heap"
+                continue
+            if gsel != int(o["split_sel"][v]):
+                mism += 1
+                if abs(ond["kappa"][v] - tau) <= NEAR_TIE * max(ond["kscale"][v], abs(tau), 1e-300):
+                    exempt += 1
+    rep["units"] = nu
+    rep["units_excluded_near_tie"] = len(excluded)
+    rep["nodes_pending"] = pending
+    rep["nodes_pruned"] = pruned
+    rep["D_relerr"] = worst_D
+    rep["U_relerr"] = worst_U
+    assert worst_D <= D_RTOL, worst_D
+    assert worst_U <= U_RTOL, worst_U
     rep["selection_mismatch"] = mism
     rep["selection_exempt"] = exempt
     if require_exact_selection:
