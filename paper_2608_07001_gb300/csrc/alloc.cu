@@ -93,27 +93,53 @@ __global__ void alloc_hist_kernel(AllocArgs A, int shift, int nbits, uint32_t ma
     }
 }
 
-__global__ void alloc_scan_kernel(AllocArgs A, int shift, int nbits) {
-    if (threadIdx.x != 0) return;
+// Pick the digit of this pass: scanning bins from the top, the bin where the
+// cost of higher keys first exceeds B_free.  One block of 1024 threads; thread
+// t owns bins nbin-1-2t and nbin-2-2t.
+__global__ void __launch_bounds__(1024) alloc_scan_kernel(AllocArgs A, int shift, int nbits) {
+    __shared__ unsigned long long wsum[32];
     const int nbin = 1 << nbits;
-    unsigned long long above = A.st[ST_ABOVE];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const unsigned long long B = (unsigned long long)A.B_free;
-    if (shift == 21 && A.st[ST_TOTAL] <= B) {
-        A.st[ST_ALL] = 1;
+    const bool all = (shift == 21) ? (A.st[ST_TOTAL] <= B) : (A.st[ST_ALL] != 0);
+    const int b0 = nbin - 1 - 2 * tid, b1 = b0 - 1;
+    unsigned long long h0 = b0 >= 0 ? A.hist[b0] : 0ull, h1 = b1 >= 0 ? A.hist[b1] : 0ull;
+    // exclusive scan of (h0 + h1) over threads, in descending bin order
+    unsigned long long x = h0 + h1, incl = x;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        unsigned long long y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
     }
-    if (A.st[ST_ALL]) {
-        for (int b = 0; b < nbin; b++) A.hist[b] = 0;
-        return;
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        unsigned long long v = wsum[lane], iv = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            unsigned long long y = __shfl_up_sync(0xffffffffu, iv, o);
+            if (lane >= o) iv += y;
+        }
+        wsum[lane] = iv - v;   // exclusive prefix of warp totals
     }
-    int pick = 0;
-    for (int b = nbin - 1; b >= 0; b--) {
-        unsigned long long h = A.hist[b];
-        if (above + h > B) { pick = b; break; }
-        above += h;
+    __syncthreads();
+    const unsigned long long above = A.st[ST_ABOVE];
+    const unsigned long long before = above + wsum[warp] + (incl - x);
+    __syncthreads();
+    if (all) {
+        if (tid == 0 && shift == 21) A.st[ST_ALL] = 1;
+    } else {
+        // the crossing bin is unique: above + cost(higher bins) <= B < ... + h
+        if (b0 >= 0 && before <= B && before + h0 > B) {
+            A.st[ST_PREFIX] |= ((unsigned long long)b0 << shift);
+            A.st[ST_ABOVE] = before;
+        } else if (b1 >= 0 && before + h0 <= B && before + h0 + h1 > B) {
+            A.st[ST_PREFIX] |= ((unsigned long long)b1 << shift);
+            A.st[ST_ABOVE] = before + h0;
+        }
     }
-    A.st[ST_PREFIX] |= ((unsigned long long)pick << shift);
-    A.st[ST_ABOVE] = above;
-    for (int b = 0; b < nbin; b++) A.hist[b] = 0;
+    if (b0 >= 0) A.hist[b0] = 0;
+    if (b1 >= 0) A.hist[b1] = 0;
 }
 
 // Main set (kappa > tau, or everything when it fits) and units holding ties.
@@ -353,7 +379,7 @@ cudaError_t launch_threshold(Ctx &c, int J, cudaStream_t s) {
     uint32_t mask = 0;
     for (int ps = 0; ps < 3; ps++) {
         alloc_hist_kernel<<<blocks, 256, 0, s>>>(A, shifts[ps], bits[ps], mask);
-        alloc_scan_kernel<<<1, 32, 0, s>>>(A, shifts[ps], bits[ps]);
+        alloc_scan_kernel<<<1, 1024, 0, s>>>(A, shifts[ps], bits[ps]);
         mask |= ((1u << bits[ps]) - 1u) << shifts[ps];
     }
     c.launches += 7;

@@ -31,8 +31,8 @@ struct Workspace {
     double *bscore = nullptr;      // [T] boundary score
     double *zbuf = nullptr;        // [T] scratch for robust z
     double *p2 = nullptr;          // [N_c + 1] prefix of sum_l ||d_t||^2
-    double *ew = nullptr;          // [(N_c + 1) * nb] DP edge weights (len n_min..n_max)
-    double *ewt = nullptr;         // [n_max + 1] terminal edge weights (len 1..n_max) at i = N_c
+    float2 *ew = nullptr;          // [(N_c + 1) * nb] DP edge weights (len n_min..n_max), (hi, lo) pairs
+    float2 *ewt = nullptr;         // [n_max + 1] terminal edge weights (len 1..n_max) at i = N_c
     double *dpF = nullptr;         // [N_c + 1] DP values
     int32_t *slots = nullptr;      // [N_c + 2] slot starts (absolute)
     int32_t *dev_int = nullptr;    // [8] small device scalars (J, status, ...)

@@ -219,6 +219,243 @@ __global__ void __launch_bounds__(256) token_values_kernel(const Tin *K, const T
     }
 }
 
+// ---------------------------------------------------------------------------
+// Tensor-core (bf16 mma.sync m16n8k16, fp32 accumulation) versions of both
+// passes for bf16 inputs: products of bf16 values are exact, sums are fp32.
+// 16 warps per CTA, warp w owns probe rows 16 w .. 16 w + 15 of the KV head
+// (its Q fragments stay in registers); 64-token key tiles are staged in
+// shared memory (row stride d + 8 halves: conflict-free fragment reads) with
+// cp.async double buffering.  Exponentials run in base 2 on pre-scaled logits.
+// ---------------------------------------------------------------------------
+constexpr int kMT = 64;           // tokens per tile
+constexpr int kMmaWarps = 16;
+constexpr float kLog2e = 1.4426950408889634f;
+
+__device__ __forceinline__ void mma_bf16(float c[4], const uint32_t a[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+        "{%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};\n"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ void cp_async16(void *smem, const void *gmem, bool pred) {
+    unsigned s = (unsigned)__cvta_generic_to_shared(smem);
+    int n = pred ? 16 : 0;   // zero-fill past the end
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(s), "l"(gmem), "r"(n));
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N)); }
+
+// Stage tokens [t0, t0 + 64) of K (row-major [T][DH]) into a padded tile.
+template <int DH>
+__device__ __forceinline__ void stage_tile(__nv_bfloat16 *tile, const __nv_bfloat16 *Kl, int t0, int tend) {
+    constexpr int CPR = DH / 8;            // 16-byte chunks per row
+    for (int e = threadIdx.x; e < kMT * CPR; e += blockDim.x) {
+        int r = e / CPR, cc = e - r * CPR;
+        int t = t0 + r;
+        bool ok = t < tend;
+        const __nv_bfloat16 *src = Kl + (size_t)(ok ? t : t0) * DH + cc * 8;
+        cp_async16(tile + r * (DH + 8) + cc * 8, src, ok);
+    }
+}
+
+// Load the A fragments of rows [r0, r0 + 16) of a row-major [rows][DH] block.
+template <int DH>
+__device__ __forceinline__ void load_qfrag(uint32_t qa[DH / 16][4], const __nv_bfloat16 *Qrows, int lane) {
+    const int r = lane >> 2, k = 2 * (lane & 3);
+#pragma unroll
+    for (int ks = 0; ks < DH / 16; ks++) {
+        const __nv_bfloat16 *p0 = Qrows + (size_t)r * DH + ks * 16 + k;
+        const __nv_bfloat16 *p1 = Qrows + (size_t)(r + 8) * DH + ks * 16 + k;
+        qa[ks][0] = *reinterpret_cast<const uint32_t *>(p0);
+        qa[ks][1] = *reinterpret_cast<const uint32_t *>(p1);
+        qa[ks][2] = *reinterpret_cast<const uint32_t *>(p0 + 8);
+        qa[ks][3] = *reinterpret_cast<const uint32_t *>(p1 + 8);
+    }
+}
+
+// Scores of the warp's 16 rows against the 64 tokens of a staged tile.
+template <int DH>
+__device__ __forceinline__ void tile_scores(float c[8][4], const uint32_t qa[DH / 16][4],
+                                            const __nv_bfloat16 *tile, int lane) {
+    const int n = lane >> 2, k = 2 * (lane & 3);
+#pragma unroll
+    for (int nt = 0; nt < 8; nt++) {
+        c[nt][0] = c[nt][1] = c[nt][2] = c[nt][3] = 0.f;
+        const __nv_bfloat16 *row = tile + (nt * 8 + n) * (DH + 8) + k;
+#pragma unroll
+        for (int ks = 0; ks < DH / 16; ks++) {
+            uint32_t b0 = *reinterpret_cast<const uint32_t *>(row + ks * 16);
+            uint32_t b1 = *reinterpret_cast<const uint32_t *>(row + ks * 16 + 8);
+            mma_bf16(c[nt], qa[ks], b0, b1);
+        }
+    }
+}
+
+// Pass A on tensor cores.  grid = (token chunks, 1, L*G); rows = 16 * warps.
+template <int DH>
+__global__ void __launch_bounds__(kMmaWarps * 32) row_stats_mma_kernel(
+        const __nv_bfloat16 *K, const __nv_bfloat16 *Q, ScoreArgs a, int chunk, int nchunks,
+        float *part) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    __nv_bfloat16 *tiles = reinterpret_cast<__nv_bfloat16 *>(smem_raw);   // [2][64][DH + 8]
+    const int lg = blockIdx.z, l = lg / a.G, g = lg - l * a.G;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int t_begin = blockIdx.x * chunk, t_end = min(a.T, t_begin + chunk);
+    const __nv_bfloat16 *Kl = K + (size_t)lg * a.T * DH;
+    const size_t rowbase = (size_t)(l * a.Hq + g * a.gq) * a.W;
+    const bool wact = warp * 16 < a.Rg;
+    uint32_t qa[DH / 16][4];
+    if (wact) load_qfrag<DH>(qa, Q + (rowbase + warp * 16) * DH, lane);
+    const float scale = a.inv_sqrt_d * kLog2e;     // logits in base-2 units
+    float m[2] = {-INFINITY, -INFINITY}, z[2] = {0.f, 0.f}, zc[2] = {0.f, 0.f};
+    const int ntile = (t_end - t_begin + kMT - 1) / kMT;
+    if (ntile > 0) stage_tile<DH>(tiles, Kl, t_begin, t_end);
+    cp_async_commit();
+    for (int it = 0; it < ntile; it++) {
+        const int t0 = t_begin + it * kMT;
+        if (it + 1 < ntile) stage_tile<DH>(tiles + ((it + 1) & 1) * kMT * (DH + 8), Kl, t0 + kMT, t_end);
+        cp_async_commit();
+        cp_async_wait<1>();
+        __syncthreads();
+        if (wact) {
+            float c[8][4];
+            tile_scores<DH>(c, qa, tiles + (it & 1) * kMT * (DH + 8), lane);
+#pragma unroll
+            for (int h = 0; h < 2; h++) {          // h = 0: row lane/4, h = 1: row lane/4 + 8
+                float tm = -INFINITY;
+#pragma unroll
+                for (int nt = 0; nt < 8; nt++)
+#pragma unroll
+                    for (int q = 0; q < 2; q++) {
+                        int t = t0 + nt * 8 + 2 * (lane & 3) + q;
+                        float x = c[nt][2 * h + q] * scale;
+                        c[nt][2 * h + q] = x;
+                        if (t < t_end) tm = fmaxf(tm, x);
+                    }
+                tm = fmaxf(tm, __shfl_xor_sync(0xffffffffu, tm, 1));
+                tm = fmaxf(tm, __shfl_xor_sync(0xffffffffu, tm, 2));
+                const float nm = fmaxf(m[h], tm);
+                float sz = 0.f, szc = 0.f;
+#pragma unroll
+                for (int nt = 0; nt < 8; nt++)
+#pragma unroll
+                    for (int q = 0; q < 2; q++) {
+                        int t = t0 + nt * 8 + 2 * (lane & 3) + q;
+                        if (t < t_end) {
+                            float e = exp2f(c[nt][2 * h + q] - nm);
+                            sz += e;
+                            if (t >= a.cs && t < a.cend) szc += e;
+                        }
+                    }
+                sz += __shfl_xor_sync(0xffffffffu, sz, 1);
+                sz += __shfl_xor_sync(0xffffffffu, sz, 2);
+                szc += __shfl_xor_sync(0xffffffffu, szc, 1);
+                szc += __shfl_xor_sync(0xffffffffu, szc, 2);
+                const float sc = m[h] == -INFINITY ? 0.f : exp2f(m[h] - nm);
+                z[h] = z[h] * sc + sz;
+                zc[h] = zc[h] * sc + szc;
+                m[h] = nm;
+            }
+        }
+        __syncthreads();
+    }
+    if (wact && (lane & 3) == 0) {
+        const int nrow_all = a.L * a.Hq * a.W;
+#pragma unroll
+        for (int h = 0; h < 2; h++) {
+            const size_t row = rowbase + warp * 16 + (lane >> 2) + 8 * h;
+            part[((size_t)0 * nrow_all + row) * nchunks + blockIdx.x] =
+                m[h] == -INFINITY ? -INFINITY : m[h] * (1.0f / kLog2e);
+            part[((size_t)1 * nrow_all + row) * nchunks + blockIdx.x] = z[h];
+            part[((size_t)2 * nrow_all + row) * nchunks + blockIdx.x] = zc[h];
+        }
+    }
+}
+
+// Pass B on tensor cores.  grid = (token chunks over C, L*G).
+template <int DH>
+__global__ void __launch_bounds__(kMmaWarps * 32) token_values_mma_kernel(
+        const __nv_bfloat16 *K, const __nv_bfloat16 *Q, ScoreArgs a, int chunk, const float *rm,
+        const float *rz, const float *rzc, float eps, float *rtok) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    __nv_bfloat16 *tiles = reinterpret_cast<__nv_bfloat16 *>(smem_raw);   // [2][64][DH + 8]
+    float *colpart = reinterpret_cast<float *>(tiles + 2 * kMT * (DH + 8));  // [16][64]
+    __shared__ double scale_s;
+    const int lg = blockIdx.y, l = lg / a.G, g = lg - l * a.G;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int t_begin = a.cs + blockIdx.x * chunk, t_end = min(a.cend, t_begin + chunk);
+    const __nv_bfloat16 *Kl = K + (size_t)lg * a.T * DH;
+    const size_t rowbase = (size_t)(l * a.Hq + g * a.gq) * a.W;
+    const bool wact = warp * 16 < a.Rg;
+    if (warp == 0) {
+        double sum = 0.0;
+        for (int r = lane; r < a.Rg; r += 32) sum += (double)rzc[rowbase + r] / (double)rz[rowbase + r];
+        sum = warp_sum(sum);
+        if (lane == 0) scale_s = 1.0 / (sum + (double)eps);
+    }
+    uint32_t qa[DH / 16][4];
+    float rmh[2] = {0.f, 0.f}, rih[2] = {0.f, 0.f};
+    if (wact) {
+        load_qfrag<DH>(qa, Q + (rowbase + warp * 16) * DH, lane);
+#pragma unroll
+        for (int h = 0; h < 2; h++) {
+            const size_t row = rowbase + warp * 16 + (lane >> 2) + 8 * h;
+            rmh[h] = rm[row] * kLog2e;
+            rih[h] = 1.0f / rz[row];
+        }
+    }
+    const float scale = a.inv_sqrt_d * kLog2e;
+    const int ntile = (t_end - t_begin + kMT - 1) / kMT;
+    if (ntile > 0) stage_tile<DH>(tiles, Kl, t_begin, t_end);
+    cp_async_commit();
+    for (int it = 0; it < ntile; it++) {
+        const int t0 = t_begin + it * kMT;
+        if (it + 1 < ntile) stage_tile<DH>(tiles + ((it + 1) & 1) * kMT * (DH + 8), Kl, t0 + kMT, t_end);
+        cp_async_commit();
+        cp_async_wait<1>();
+        __syncthreads();
+        float col[16];
+#pragma unroll
+        for (int q = 0; q < 16; q++) col[q] = 0.f;
+        if (wact) {
+            float c[8][4];
+            tile_scores<DH>(c, qa, tiles + (it & 1) * kMT * (DH + 8), lane);
+#pragma unroll
+            for (int nt = 0; nt < 8; nt++)
+#pragma unroll
+                for (int q = 0; q < 2; q++)
+                    col[2 * nt + q] = exp2f(c[nt][q] * scale - rmh[0]) * rih[0] +
+                                      exp2f(c[nt][2 + q] * scale - rmh[1]) * rih[1];
+        }
+#pragma unroll
+        for (int q = 0; q < 16; q++) {
+            float v = col[q];
+            v += __shfl_xor_sync(0xffffffffu, v, 4);
+            v += __shfl_xor_sync(0xffffffffu, v, 8);
+            v += __shfl_xor_sync(0xffffffffu, v, 16);
+            col[q] = v;
+        }
+        if (lane < 4) {
+#pragma unroll
+            for (int nt = 0; nt < 8; nt++)
+#pragma unroll
+                for (int q = 0; q < 2; q++) colpart[warp * kMT + nt * 8 + 2 * lane + q] = col[2 * nt + q];
+        }
+        __syncthreads();
+        if (threadIdx.x < kMT) {
+            const int t = t0 + threadIdx.x;
+            if (t < t_end) {
+                float sum = 0.f;
+                for (int w = 0; w < kMmaWarps; w++) sum += colpart[w * kMT + threadIdx.x];
+                rtok[(size_t)lg * a.Nc + (t - a.cs)] = (float)((double)sum * scale_s);
+            }
+        }
+    }
+}
+
 ScoreArgs make_args(const Ctx &c) {
     ScoreArgs a;
     a.L = c.p.L; a.G = c.p.G; a.Hq = c.p.Hq; a.T = c.p.T; a.d = c.p.d; a.W = c.p.W;
@@ -239,10 +476,43 @@ cudaError_t launch_rope_table(Ctx &c, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+bool use_mma(const Ctx &c, const ScoreArgs &a) {
+    return c.p.dtype == GKV_BF16 && (c.p.d == 64 || c.p.d == 128) && a.Rg % 16 == 0 &&
+           a.Rg <= 16 * kMmaWarps;
+}
+
+template <int DH>
+void launch_mma_a(const Ctx &c, const ScoreArgs &a, const void *K, const void *Q, int chunk, cudaStream_t s) {
+    size_t sm = 2 * kMT * (DH + 8) * sizeof(__nv_bfloat16);
+    dim3 grid(c.n_chunks, 1, a.L * a.G);
+    row_stats_mma_kernel<DH><<<grid, kMmaWarps * 32, sm, s>>>(
+        static_cast<const __nv_bfloat16 *>(K), static_cast<const __nv_bfloat16 *>(Q), a, chunk,
+        c.n_chunks, c.w.rowp);
+}
+
+template <int DH>
+void launch_mma_b(const Ctx &c, const ScoreArgs &a, const void *K, const void *Q, int chunk, float eps,
+                  cudaStream_t s) {
+    size_t sm = 2 * kMT * (DH + 8) * sizeof(__nv_bfloat16) + kMmaWarps * kMT * sizeof(float);
+    dim3 grid((c.Nc + chunk - 1) / chunk, a.L * a.G);
+    token_values_mma_kernel<DH><<<grid, kMmaWarps * 32, sm, s>>>(
+        static_cast<const __nv_bfloat16 *>(K), static_cast<const __nv_bfloat16 *>(Q), a, chunk,
+        c.w.row_m, c.w.row_Z, c.w.row_ZC, eps, c.w.rtok);
+}
+
 cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t s) {
     ScoreArgs a = make_args(c);
     int chunk = (c.p.T + c.n_chunks - 1) / c.n_chunks;
     chunk = (chunk + kTT - 1) / kTT * kTT;
+    if (use_mma(c, a)) {
+        if (c.p.d == 128) launch_mma_a<128>(c, a, K, Q, chunk, s);
+        else launch_mma_a<64>(c, a, K, Q, chunk, s);
+        int nrow = a.L * a.Hq * a.W;
+        row_combine_kernel<<<(nrow + 255) / 256, 256, 0, s>>>(c.w.rowp, nrow, c.n_chunks, c.w.row_m,
+                                                              c.w.row_Z, c.w.row_ZC, c.w.dev_int + 1);
+        c.launches += 2;
+        return cudaGetLastError();
+    }
     dim3 grid(c.n_chunks, (a.Rg + kTR - 1) / kTR, a.L * a.G);
     if (c.p.dtype == GKV_BF16)
         row_stats_kernel<<<grid, 256, 0, s>>>(static_cast<const __nv_bfloat16 *>(K),
@@ -263,6 +533,16 @@ cudaError_t launch_token_values(Ctx &c, const void *K, const void *Q, cudaStream
     ScoreArgs a = make_args(c);
     dim3 grid((c.Nc + kTT - 1) / kTT, a.L * a.G);
     float eps = (float)c.p.eps;
+    if (use_mma(c, a)) {
+        // about 4 CTAs of 16 warps per SM-pass over the compressible region
+        int64_t want = 4LL * c.num_sms;
+        int64_t per = std::max<int64_t>(1, ((int64_t)a.L * a.G * c.Nc) / want);
+        int chunk = (int)std::min<int64_t>(std::max<int64_t>(kMT, (per + kMT - 1) / kMT * kMT), 4096);
+        if (c.p.d == 128) launch_mma_b<128>(c, a, K, Q, chunk, eps, s);
+        else launch_mma_b<64>(c, a, K, Q, chunk, eps, s);
+        c.launches += 1;
+        return cudaGetLastError();
+    }
     if (c.p.dtype == GKV_BF16)
         token_values_kernel<<<grid, 256, 0, s>>>(static_cast<const __nv_bfloat16 *>(K),
                                                  static_cast<const __nv_bfloat16 *>(Q), a,

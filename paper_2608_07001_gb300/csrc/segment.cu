@@ -27,6 +27,27 @@ namespace {
 
 constexpr double kEps = 1e-6;   // App. B.2: epsilon of the normalisations and of robust z
 
+// Double-float numbers (value = hi + lo, |lo| <= ulp(hi) / 2): the DP state is
+// carried in ~48-bit precision on the fp32 units, because fp64 throughput on
+// GB300 is very low.  Additions use the error-free two-sum of Knuth.
+struct df2 {
+    float hi, lo;
+};
+__device__ __forceinline__ float2 df_split(double x) {
+    float hi = (float)x;
+    return make_float2(hi, (float)(x - (double)hi));
+}
+__device__ __forceinline__ df2 df_add(df2 a, float2 b) {
+    float s = a.hi + b.x;
+    float bb = s - a.hi;
+    float e = (a.hi - (s - bb)) + (b.x - bb);
+    e += a.lo + b.y;
+    float hi = s + e;
+    return df2{hi, e - (hi - s)};
+}
+__device__ __forceinline__ bool df_gt(df2 a, df2 b) { return a.hi > b.hi || (a.hi == b.hi && a.lo > b.lo); }
+__device__ __forceinline__ bool df_eq(df2 a, df2 b) { return a.hi == b.hi && a.lo == b.lo; }
+
 // Element (channel c of the trajectory) of h^(l)_t: concat over KV heads of V.
 template <typename Tin>
 __device__ __forceinline__ float traj_elem(const Tin *V, const float *hidden, int Dh, int G,
@@ -355,7 +376,7 @@ template <typename Tin>
 __global__ void __launch_bounds__(256) seg_band_kernel(const Tin *V, const float *hidden, BandArgs b,
                                                        const float *inv_norm, const float *nrm2,
                                                        const double *p2, const double *bscore,
-                                                       double *ew) {
+                                                       float2 *ew) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const SegArgs &a = b.s;
     const int nb = b.n_max - b.n_min + 1;
@@ -430,7 +451,8 @@ __global__ void __launch_bounds__(256) seg_band_kernel(const Tin *V, const float
         if (len < b.n_min || len > b.n_max) continue;
         double w;
         if (ap < 0) {
-            w = -INFINITY;
+            ew[(size_t)i * nb + (len - b.n_min)] = make_float2(-INFINITY, 0.f);
+            continue;
         } else {
             int nS = len - 1;
             double disp = 0.0;
@@ -442,7 +464,7 @@ __global__ void __launch_bounds__(256) seg_band_kernel(const Tin *V, const float
             double pen = (double)(len - b.n0) / b.n0;
             w = gam - b.lambda_d * disp - b.lambda_n * pen * pen;
         }
-        ew[(size_t)i * nb + (len - b.n_min)] = w;
+        ew[(size_t)i * nb + (len - b.n_min)] = df_split(w);
     }
 }
 
@@ -450,14 +472,14 @@ __global__ void __launch_bounds__(256) seg_band_kernel(const Tin *V, const float
 template <typename Tin>
 __global__ void seg_band_terminal_kernel(const Tin *V, const float *hidden, BandArgs b,
                                          const float *inv_norm, const float *nrm2,
-                                         const double *p2, const double *bscore, double *ewt) {
+                                         const double *p2, const double *bscore, float2 *ewt) {
     const SegArgs &a = b.s;
     int len = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32 + 1;
     int lane = threadIdx.x & 31;
     if (len > b.n_max) return;
     int i = a.N, ep = i - 1, ap = i - len;
     if (ap < 0) {
-        if (lane == 0) ewt[len] = -INFINITY;
+        if (lane == 0) ewt[len] = make_float2(-INFINITY, 0.f);
         return;
     }
     double sd = 0.0;
@@ -477,7 +499,7 @@ __global__ void seg_band_terminal_kernel(const Tin *V, const float *hidden, Band
     if (nS >= 2) disp = ((p2[ep] - p2[ap]) - sd / nS) / (double)(nS - 1) / a.nseg;
     double gam = ap == 0 ? 0.0 : bscore[a.cs + ap - 1] - b.c_cut;
     double pen = (double)(len - b.n0) / b.n0;
-    ewt[len] = gam - b.lambda_d * disp - b.lambda_n * pen * pen;
+    ewt[len] = df_split(gam - b.lambda_d * disp - b.lambda_n * pen * pen);
 }
 
 // ---------------------------------------------------------------------------
@@ -491,24 +513,25 @@ constexpr int kDpRing = 256;
 constexpr int kDpEp = 16;
 constexpr int kDpTpe = 64;
 
-__device__ __forceinline__ bool better(double v, int a, double bv, int ba) {
-    return v > bv || (v == bv && a < ba);
+__device__ __forceinline__ bool better(df2 v, int a, df2 bv, int ba) {
+    return df_gt(v, bv) || (df_eq(v, bv) && a < ba);
 }
 
-__global__ void __launch_bounds__(1024) seg_dp_kernel(const double *ew, const double *ewt, int N,
+__global__ void __launch_bounds__(1024) seg_dp_kernel(const float2 *ew, const float2 *ewt, int N,
                                                       int n_min, int n_max, int cs, double *Fout,
                                                       int32_t *slots, int *dev_int) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
-    double *ring = reinterpret_cast<double *>(smem_raw);                 // [kDpRing]
-    double *rv = ring + kDpRing;                                         // [32] per-warp best value
+    df2 *ring = reinterpret_cast<df2 *>(smem_raw);                       // [kDpRing]
+    df2 *rv = ring + kDpRing;                                            // [32] per-warp best value
     int *ra = reinterpret_cast<int *>(rv + 32);                          // [32] per-warp best a
     uint8_t *lenarr = reinterpret_cast<uint8_t *>(ra + 32);              // [N + 1]
     const int nb = n_max - n_min + 1;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int k = tid / kDpTpe, sub = tid % kDpTpe;
     const int step = min(n_min, kDpEp);
+    const df2 NEG = df2{-INFINITY, 0.f};
     if (tid == 0) {
-        ring[0] = 0.0;
+        ring[0] = df2{0.f, 0.f};
         Fout[0] = 0.0;
         lenarr[0] = 0;
     }
@@ -516,52 +539,55 @@ __global__ void __launch_bounds__(1024) seg_dp_kernel(const double *ew, const do
     for (int i0 = 1; i0 <= N; i0 += step) {
         int i = i0 + k;
         bool act = k < step && i <= N;
-        double best = -INFINITY;
+        df2 best = NEG;
         int ba = 0x7fffffff;
         if (act) {
             for (int len = n_min + sub; len <= n_max; len += kDpTpe) {
                 int a = i - len;
                 if (a < 0) break;
-                double fa = ring[a % kDpRing];
-                if (fa == -INFINITY) continue;
-                double v = fa + ew[(size_t)i * nb + (len - n_min)];
+                df2 fa = ring[a % kDpRing];
+                if (fa.hi == -INFINITY) continue;
+                float2 w = ew[(size_t)i * nb + (len - n_min)];
+                df2 v = df_add(fa, w);
                 if (better(v, a, best, ba)) { best = v; ba = a; }
             }
         }
         // reduce over the 64 threads of the endpoint (2 warps)
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
-            double ov = __shfl_xor_sync(0xffffffffu, best, o);
+            df2 ov;
+            ov.hi = __shfl_xor_sync(0xffffffffu, best.hi, o);
+            ov.lo = __shfl_xor_sync(0xffffffffu, best.lo, o);
             int oa = __shfl_xor_sync(0xffffffffu, ba, o);
             if (better(ov, oa, best, ba)) { best = ov; ba = oa; }
         }
         if (lane == 0) { rv[warp] = best; ra[warp] = ba; }
         __syncthreads();
         if (sub == 0 && act) {
-            double v2 = rv[warp + 1];
+            df2 v2 = rv[warp + 1];
             int a2 = ra[warp + 1];
             if (better(v2, a2, best, ba)) { best = v2; ba = a2; }
             ring[i % kDpRing] = best;
-            Fout[i] = best;
-            lenarr[i] = best == -INFINITY ? 0 : (uint8_t)(i - ba);
+            Fout[i] = (double)best.hi + (double)best.lo;
+            lenarr[i] = best.hi == -INFINITY ? 0 : (uint8_t)(i - ba);
         }
         __syncthreads();
     }
-    if (tid == 0 && ring[N % kDpRing] == -INFINITY) {
+    if (tid == 0 && ring[N % kDpRing].hi == -INFINITY) {
         // terminal relaxation (Eq. app_terminal_predecessor): 1 <= N - a <= n_max,
         // read after every F[< N] has been written
-        double best = -INFINITY;
+        df2 best = NEG;
         int ba = 0x7fffffff;
         for (int len = 1; len <= n_max; len++) {
             int a = N - len;
             if (a < 0) break;
-            double fa = ring[a % kDpRing];
-            if (fa == -INFINITY) continue;
-            double v = fa + ewt[len];
+            df2 fa = ring[a % kDpRing];
+            if (fa.hi == -INFINITY || ewt[len].x == -INFINITY) continue;
+            df2 v = df_add(fa, ewt[len]);
             if (better(v, a, best, ba)) { best = v; ba = a; }
         }
-        Fout[N] = best;
-        lenarr[N] = best == -INFINITY ? 0 : (uint8_t)(N - ba);
+        Fout[N] = (double)best.hi + (double)best.lo;
+        lenarr[N] = best.hi == -INFINITY ? 0 : (uint8_t)(N - ba);
     }
     if (tid == 0) {
         int J = 0, ok = 1;
@@ -661,7 +687,7 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
         seg_band_kernel<<<gb, 256, smb, s>>>(Vf, hidden, b, w.inv_norm, w.nrm2, w.p2, w.bscore, w.ew);
         seg_band_terminal_kernel<<<(p.n_max + 7) / 8, 256, 0, s>>>(Vf, hidden, b, w.inv_norm, w.nrm2, w.p2, w.bscore, w.ewt);
     }
-    size_t smd = kDpRing * 8 + 32 * 8 + 32 * 4 + (size_t)(N + 1);
+    size_t smd = kDpRing * sizeof(df2) + 32 * sizeof(df2) + 32 * 4 + (size_t)(N + 1);
     smd = (smd + 15) & ~(size_t)15;
     if (smd > 227 * 1024) return cudaErrorInvalidConfiguration;
     cudaFuncSetAttribute(seg_dp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smd);
