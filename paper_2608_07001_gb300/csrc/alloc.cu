@@ -358,14 +358,25 @@ int grid_for(const Ctx &c, int64_t n) {
 
 // Units with a pending node whose creator key is >= tau (all of them when
 // every op built so far fits the budget).
-__global__ void prune_list_kernel(const float *u_pend, int64_t n_units,
+__global__ void prune_list_kernel(const float *u_pend, const int32_t *slots, int J, int64_t n_units,
                                   const unsigned long long *st, int32_t *list, int *count) {
     int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= n_units) return;
     float p = u_pend[i];
     if (!(p >= 0.f)) return;   // -1: no pending node
     const bool all = st[ST_ALL] != 0;
-    if (all || __float_as_uint(p) >= (uint32_t)st[ST_PREFIX]) list[atomicAdd(count, 1)] = (int32_t)i;
+    if (all || __float_as_uint(p) >= (uint32_t)st[ST_PREFIX]) {
+        const int j = (int)(i % J);
+        if (slots[j + 1] - slots[j] <= kShortUnit) list[atomicAdd(count, 1)] = (int32_t)i;
+        else list[n_units - 1 - atomicAdd(count + 1, 1)] = (int32_t)i;
+    }
+}
+
+__global__ void slot_classes_kernel(const int32_t *slots, int J, int32_t *list, int *count) {
+    int j = blockIdx.x * blockDim.x + threadIdx.x;
+    if (j >= J) return;
+    if (slots[j + 1] - slots[j] <= kShortUnit) list[atomicAdd(count, 1)] = j;
+    else list[J - 1 - atomicAdd(count + 1, 1)] = j;
 }
 
 }  // namespace
@@ -386,12 +397,22 @@ cudaError_t launch_threshold(Ctx &c, int J, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-cudaError_t launch_prune_list(Ctx &c, int J, int32_t *list, int *count, cudaStream_t s) {
+cudaError_t launch_prune_list(Ctx &c, const int32_t *slots, int J, int32_t *list, int *count,
+                              cudaStream_t s) {
     const int64_t nu = (int64_t)c.p.L * c.p.G * J;
-    cudaError_t e = cudaMemsetAsync(count, 0, sizeof(int), s);
+    cudaError_t e = cudaMemsetAsync(count, 0, 2 * sizeof(int), s);
     if (e != cudaSuccess) return e;
-    prune_list_kernel<<<(unsigned)((nu + 255) / 256), 256, 0, s>>>(c.w.u_pend, nu, c.w.alloc_state,
-                                                                    list, count);
+    prune_list_kernel<<<(unsigned)((nu + 255) / 256), 256, 0, s>>>(c.w.u_pend, slots, J, nu,
+                                                                    c.w.alloc_state, list, count);
+    c.launches += 1;
+    return cudaGetLastError();
+}
+
+cudaError_t launch_slot_classes(Ctx &c, const int32_t *slots, int J, int32_t *list, int *count,
+                                cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(count, 0, 2 * sizeof(int), s);
+    if (e != cudaSuccess) return e;
+    slot_classes_kernel<<<(J + 255) / 256, 256, 0, s>>>(slots, J, list, count);
     c.launches += 1;
     return cudaGetLastError();
 }

@@ -334,23 +334,33 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
     // threshold of the ops built so far are evaluated.
     if (e == cudaSuccess) e = cudaMemsetAsync(w.work, 0, 4 * sizeof(unsigned long long), s);
     if (e == cudaSuccess) {
-        gkv::StageTimer tm(c, 3, s);
-        e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 0, 1, 0.f, nullptr, 0, s);
+        int cnt[2] = {0, 0};
+        {
+            gkv::StageTimer tm(c, 3, s);
+            e = gkv::launch_slot_classes(c, w.slots, J, w.u_list, w.dev_int + 2, s);
+        }
+        if (e == cudaSuccess) e = cudaMemcpyAsync(cnt, w.dev_int + 2, 2 * sizeof(int), cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+        if (e == cudaSuccess) {
+            gkv::StageTimer tm(c, 3, s);
+            e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 0, 1, 0.f, w.u_list, cnt[0],
+                                       w.u_list + (J - cnt[1]), cnt[1], s);
+        }
     }
     for (int it = 0; e == cudaSuccess; it++) {
-        struct { int count; unsigned long long prefix, all; } h = {0, 0, 0};
+        struct { int count[2]; unsigned long long prefix, all; } h = {{0, 0}, 0, 0};
         {
             gkv::StageTimer tm(c, 3, s);
             e = gkv::launch_threshold(c, J, s);
-            if (e == cudaSuccess) e = gkv::launch_prune_list(c, J, w.u_list, w.dev_int + 2, s);
+            if (e == cudaSuccess) e = gkv::launch_prune_list(c, w.slots, J, w.u_list, w.dev_int + 2, s);
         }
-        if (e == cudaSuccess) e = cudaMemcpyAsync(&h.count, w.dev_int + 2, sizeof(int), cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(h.count, w.dev_int + 2, 2 * sizeof(int), cudaMemcpyDeviceToHost, s);
         if (e == cudaSuccess) e = cudaMemcpyAsync(&h.prefix, w.alloc_state, 2 * sizeof(unsigned long long),
                                                   cudaMemcpyDeviceToHost, s);
         if (e == cudaSuccess) e = cudaMemcpyAsync(&h.all, w.alloc_state + 2, sizeof(unsigned long long),
                                                   cudaMemcpyDeviceToHost, s);
         if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-        if (e != cudaSuccess || h.count == 0) break;
+        if (e != cudaSuccess || h.count[0] + h.count[1] == 0) break;
         uint32_t bits = (uint32_t)h.prefix;
         float tau;
         memcpy(&tau, &bits, sizeof tau);
@@ -358,7 +368,8 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
         // everything built so far fits: nothing can be pruned yet, go deeper at once
         const int levels = h.all ? 4 * gkv::kMaxUnit : 2;
         gkv::StageTimer tm(c, 3, s);
-        e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 1, levels, tau, w.u_list, h.count, s);
+        e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 1, levels, tau, w.u_list, h.count[0],
+                                   w.u_list + (nu - h.count[1]), h.count[1], s);
         c.build_passes = it + 2;
     }
     if (e != cudaSuccess) return cuda_fail(x, e, "build_trees launch");

@@ -14,15 +14,15 @@
 // extraction at p* = argmax R_tok (Eq. app_extract_split).  For each
 // candidate J the prototype (ktil, vtil, m_eff; Eqs. app_rope_prototype,
 // app_value_prototype, app_effective_multiplicity) is formed by direct sums
-// over J; then one forward and one backward scan over the level's tokens
-// accumulate Z_u(J) and M_u(J) (Eq. app_original_attention_stats) for every
-// probe and evaluate D_u (Eq. app_probe_distortion) at each candidate end,
-// weighted by the attention mass Z_u(J) / Z_u (Eq.
-// app_node_and_drop_distortion).  The refinement form follows Eqs.
-// app_binary_split .. app_split_choice; gains, costs and utilities follow
-// Eqs. app_operation_gains .. app_unit_utility (clamped at 0); each Split op
-// also gets its bottleneck key kappa = min(U, kappa of the op that created
-// the node), which the allocator's threshold select uses.
+// over J; then a forward scan (prefixes) and a backward scan (suffixes) over
+// the node's tokens accumulate Z_u(J) and M_u(J) (Eq.
+// app_original_attention_stats) for every probe and evaluate D_u (Eq.
+// app_probe_distortion) at each candidate end, weighted by the attention mass
+// Z_u(J) / Z_u (Eq. app_node_and_drop_distortion).  The refinement form
+// follows Eqs. app_binary_split .. app_split_choice; gains, costs and
+// utilities follow Eqs. app_operation_gains .. app_unit_utility (clamped at
+// 0); each Split op also gets its bottleneck key kappa = min(U, kappa of the
+// op that created the node), which the allocator's threshold select uses.
 //
 // Pruned construction.  A launch evaluates at most `max_levels` levels; the
 // nodes below stay pending (child count -1, no Split op yet) and each unit
@@ -33,13 +33,20 @@
 // >= tau: a node whose creator's key is below the final threshold never
 // reaches the frontier before the allocation stops, so its own Split is never
 // needed.  Resuming repeats until no pending node qualifies.
+//
+// Layout.  256 threads; thread (u, c) owns probe u and the 8-element chunks
+// c, c + NCH, c + 2 NCH, ... of every d-vector, so that its shared-memory
+// reads are 16-byte vectors and the lanes of a warp never share a bank.
+// Slots of up to 64 tokens use a 64-token instance whose footprint allows two
+// CTAs per SM; longer slots use the 128-token instance.
 #include "gkv_internal.cuh"
 
 namespace gkv {
 namespace {
 
 constexpr int kMaxCuts = 18;     // K + midpoint, K <= 16 (+1 spare)
-constexpr int kMaxNodes = 2 * kMaxUnit;
+constexpr int kNT = 256;         // threads per CTA
+constexpr int kNCD = 24;         // candidate intervals per direction and batch (>= 17 + 2)
 
 struct BuildArgs {
     const void *K, *V, *Q;
@@ -49,12 +56,12 @@ struct BuildArgs {
     const float *rtok, *row_m, *row_Z, *omega;
     int L, G, Hq, T, d, W, gq, cs, Nc, J, k_cand;
     float inv_sqrt_d, lamZ, lamM, eps;
-    double lam_kappa, base_frac, eps_d;
-    // pruning
+    double lam_kappa, base_frac;
+    // work list: fresh launches index (slot list entry, lg), resume launches units
     int resume;                  // 0: build from the root, 1: resume pending nodes
     int max_levels;              // levels evaluated by this launch
     float tau;                   // resume: evaluate pending nodes whose creator key >= tau
-    const int32_t *unit_list;    // resume: units to process (blockIdx.x indexes it)
+    const int32_t *list;         // fresh: slot indices; resume: unit ids
     // outputs
     int32_t *nd_a, *nd_b, *nd_child0, *nd_parent, *nd_unit;
     int8_t *nd_nchild, *nd_cost;
@@ -82,8 +89,9 @@ struct BatchNode {
     short pidx[kMaxCuts];    // candidate index of [a, xi) (-1: single token)
     short sidx[kMaxCuts];    // candidate index of [xi, b) (-1: single token)
     int pstar, eL, eR, whole;
-    int pre_b, pre_e, suf_b, suf_e;   // candidate ranges (prefixes ascending end,
-                                      // suffixes descending start)
+    int pre_b, pre_e, suf_b, suf_e;   // prefixes (ascending end) in [0, NCD),
+                                      // suffixes (descending start) in [NCD, 2 NCD)
+    int pre_r, suf_r;                 // ends of the reserved candidate ranges
     double kmin, kmax;
     int nchild, ca[3], cb[3];
     double cD[3];
@@ -112,60 +120,75 @@ __device__ __forceinline__ int round_half_even_mid(int a, int b) {
     return (lo & 1) == 0 ? lo : lo + 1;
 }
 
-template <int DH, int NW, typename Tin, int NT>
+// 8 consecutive elements of a shared-memory row as floats (one or two 16-byte loads).
+__device__ __forceinline__ void ld8(const float *p, float v[8]) {
+    float4 a = reinterpret_cast<const float4 *>(p)[0], b = reinterpret_cast<const float4 *>(p)[1];
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+__device__ __forceinline__ void ld8(const __nv_bfloat16 *p, float v[8]) {
+    uint4 u = reinterpret_cast<const uint4 *>(p)[0];
+    const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&u);
+#pragma unroll
+    for (int i = 0; i < 4; i++) {
+        float2 f = __bfloat1622float2(h[i]);
+        v[2 * i] = f.x;
+        v[2 * i + 1] = f.y;
+    }
+}
+
+template <int DH, int NW, typename Tin, int NMAX>
 struct Smem {
-    static constexpr int NWARPS = NT / 32;
-    static constexpr int NCH = NT / NW;      // threads per probe
+    static constexpr int NWARPS = kNT / 32;
+    static constexpr int NCH = kNT / NW;     // threads per probe
     static constexpr int CH = DH / NCH;      // elements per thread
-    // candidate capacity: at least 2*17+3 = 37 (one node); less where the slot
-    // arrays are fp32 with 64 probes
-    static constexpr int NC = (DH == 128 && NW == 64 && sizeof(Tin) == 4) ? 37 : 48;
-    static constexpr int NB = (DH == 128 && NW == 64 && sizeof(Tin) == 4) ? 24 : 32;
-    float kc[kMaxUnit][DH];
-    Tin vv[kMaxUnit][DH];
-    float E[kMaxUnit][NW];
-    float ktil[NC][DH];
-    float vtil[NC][DH];
-    float Rt[kMaxUnit];
-    float kn[kMaxUnit];
-    unsigned long long kap[kMaxUnit];   // order-preserving keys of the curvature
-    float redD[NC][NWARPS];
-    float redP[NC][NWARPS];
-    double candD[NC], candP[NC];        // per-candidate D and drop mass
-    Cand cand[NC];
-    NodeS nodes[kMaxNodes];
+    static constexpr int NQ = CH / 8;        // 8-element chunks per thread
+    static constexpr int NB = 32;            // nodes per batch
+    static constexpr int MAXNODES = 2 * NMAX;
+    float kc[NMAX][DH];
+    Tin vv[NMAX][DH];
+    float E[NMAX][NW];
+    float ktil[kNCD][DH];                    // prototypes of one direction at a time
+    float vtil[kNCD][DH];
+    float Rt[NMAX];
+    float kn[NMAX];
+    unsigned long long kap[NMAX];            // order-preserving keys of the curvature
+    float redD[2 * kNCD][NWARPS];
+    float redP[2 * kNCD][NWARPS];
+    double candD[2 * kNCD], candP[2 * kNCD]; // per-candidate D and drop mass
+    Cand cand[2 * kNCD];
+    NodeS nodes[MAXNODES];
     BatchNode bn[NB];
-    short lvl[2][kMaxNodes];
+    short lvl[2][MAXNODES];
     int nlvl[2];
     int nnodes;
-    int batch_n, batch_next;
+    int batch_n, batch_next, batch_pre, batch_suf;
     float pend;
 };
 
-template <int DH, int NW, typename Tin, int NT>
-__global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
-    using S = Smem<DH, NW, Tin, NT>;
-    constexpr int NCH = S::NCH, CH = S::CH, HALF = DH / 2, NWARPS = S::NWARPS;
-    static_assert(NCH <= 32 && (32 % NCH) == 0 && CH >= 1, "probe layout");
+template <int DH, int NW, typename Tin, int NMAX>
+__global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(BuildArgs A) {
+    using S = Smem<DH, NW, Tin, NMAX>;
+    constexpr int NCH = S::NCH, CH = S::CH, NQ = S::NQ, HALF = DH / 2, NWARPS = S::NWARPS;
+    static_assert(NCH <= 32 && (32 % NCH) == 0 && CH % 8 == 0, "probe layout");
     extern __shared__ __align__(16) unsigned char smem_raw[];
     S &sm = *reinterpret_cast<S *>(smem_raw);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int LG = A.L * A.G;
     int j, lg;
     if (A.resume) {
-        const int uidr = A.unit_list[blockIdx.x];
+        const int uidr = A.list[blockIdx.x];
         lg = uidr / A.J;
         j = uidr - lg * A.J;
     } else {
-        j = blockIdx.x / LG;   // slot-major: the units of a slot share its table rows
-        lg = blockIdx.x - j * LG;
+        j = A.list[blockIdx.x / LG];   // slot-major: the units of a slot share its table rows
+        lg = blockIdx.x % LG;
     }
     const int l = lg / A.G, g = lg - l * A.G;
     const int sa = A.slots[j], sb = A.slots[j + 1];
     const int n = sb - sa;
     const int64_t uid = (int64_t)lg * A.J + j;
     const int64_t nbase = node_base(lg, sa, A.cs, A.Nc);
-    if (n < 1 || n > kMaxUnit) {
+    if (n < 1 || n > NMAX) {
         if (tid == 0) atomicOr(A.status, 4);
         return;
     }
@@ -174,7 +197,7 @@ __global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
     const float om = A.omega ? A.omega[lg] : 1.0f;
 
     // ---- load the slot ------------------------------------------------------
-    for (int e = tid * 8; e < n * DH; e += NT * 8) {
+    for (int e = tid * 8; e < n * DH; e += kNT * 8) {
         Vec8<Tin> kx, vx;
         kx.load(Kp + e);
         vx.load(Vp + e);
@@ -185,11 +208,11 @@ __global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
             sm.vv[t][i + q] = (Tin)vx.v[q];
         }
     }
-    for (int t = tid; t < n; t += NT) {
+    for (int t = tid; t < n; t += kNT) {
         sm.kap[t] = okey(A.kappa[sa + t]);
         sm.Rt[t] = A.rtok[(size_t)lg * A.Nc + (sa - A.cs) + t];
     }
-    // probe registers: thread (u, c) owns elements c + NCH q of probe u
+    // probe registers: thread (u, c) owns chunks c + NCH q of probe u
     const int u = tid / NCH, c = tid - u * NCH;
     const bool pact = u < A.W;
     float qreg[CH];
@@ -200,7 +223,12 @@ __global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
         if (pact) {
             const Tin *qp = static_cast<const Tin *>(A.Q) + row * DH;
 #pragma unroll
-            for (int q = 0; q < CH; q++) qreg[q] = to_f(qp[c + NCH * q]);
+            for (int q = 0; q < NQ; q++) {
+                Vec8<Tin> x;
+                x.load(qp + 8 * (c + NCH * q));
+#pragma unroll
+                for (int r = 0; r < 8; r++) qreg[8 * q + r] = x.v[r];
+            }
             mu = A.row_m[row];
             invZ = 1.0f / A.row_Z[row];
         } else {
@@ -214,7 +242,12 @@ __global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
     for (int t = 0; t < n; t++) {
         float x = 0.f;
 #pragma unroll
-        for (int q = 0; q < CH; q++) x = fmaf(qreg[q], sm.kc[t][c + NCH * q], x);
+        for (int q = 0; q < NQ; q++) {
+            float kv[8];
+            ld8(&sm.kc[t][8 * (c + NCH * q)], kv);
+#pragma unroll
+            for (int r = 0; r < 8; r++) x = fmaf(qreg[8 * q + r], kv[r], x);
+        }
 #pragma unroll
         for (int o = 1; o < NCH; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
         if (c == 0) sm.E[t][u] = pact ? expf(x * A.inv_sqrt_d - mu) : 0.f;
@@ -226,8 +259,8 @@ __global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
     // the host reports as GKV_ENONFINITE at the allocation's count sync.
     {
         bool bad = false;
-        for (int e = tid; e < n * NW; e += NT) bad |= !isfinite(sm.E[e / NW][e % NW]);
-        for (int t = tid; t < n; t += NT) bad |= !isfinite(sm.Rt[t]);
+        for (int e = tid; e < n * NW; e += kNT) bad |= !isfinite(sm.E[e / NW][e % NW]);
+        for (int t = tid; t < n; t += kNT) bad |= !isfinite(sm.Rt[t]);
         if (__syncthreads_or(bad)) {
             if (tid == 0) {
                 atomicOr(A.status, 8);
@@ -238,12 +271,12 @@ __global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
                 A.u_nnodes[uid] = 1; A.u_Uadd[uid] = 0.f; A.u_Ddrop[uid] = 0.f; A.u_sel[uid] = 0;
                 A.u_pend[uid] = -1.f;
             }
-            for (int k = tid; k < 2 * n; k += NT) A.nd_cost[nbase + k] = 0;
+            for (int k = tid; k < 2 * n; k += kNT) A.nd_cost[nbase + k] = 0;
             return;
         }
     }
     // ---- k_circ = RoPE^-1(k, t) ----------------------------------------------
-    for (int e = tid; e < n * HALF; e += NT) {
+    for (int e = tid; e < n * HALF; e += kNT) {
         int t = e / HALF, i = e - t * HALF;
         float2 cs = A.rope[(size_t)(sa + t) * HALF + i];
         float x = sm.kc[t][i], y = sm.kc[t][i + HALF];
@@ -278,7 +311,7 @@ __global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
         }
     } else {
         const int nn = A.u_nnodes[uid];
-        for (int k = tid; k < nn; k += NT) {
+        for (int k = tid; k < nn; k += kNT) {
             const int64_t v = nbase + k;
             NodeS &nd = sm.nodes[k];
             nd.a = (short)(A.nd_a[v] - sa);
@@ -313,6 +346,125 @@ __global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
     __syncthreads();
 
     unsigned long long w_scan = 0, w_eval = 0, w_len = 0;   // thread 0's work counters
+
+    // Prototypes of the batch's prefix (or suffix) candidates, warp per
+    // candidate; reserved entries a node did not use are empty and skipped.
+    auto prototypes = [&](bool suffix) {
+        const int kb = suffix ? kNCD : 0, ke = suffix ? kNCD + sm.batch_suf : sm.batch_pre;
+        for (int k = kb + warp; k < ke; k += NWARPS) {
+            const int row = k - kb;
+            const int ja = sm.cand[k].a, jb = sm.cand[k].b, nJ = jb - ja;
+            if (nJ <= 0) continue;
+            float rs = 0.f, ks = 0.f;
+            for (int t = ja + lane; t < jb; t += 32) { rs += sm.Rt[t]; ks += sm.kn[t]; }
+            rs = warp_sum(rs);
+            ks = warp_sum(ks);
+            const float ninv = 1.0f / (float)nJ;
+            const float beta = (float)A.base_frac * (rs * ninv);
+            const float wsum = rs + (float)nJ * beta;
+            const float winv = 1.0f / (wsum + A.eps);
+            const int p = round_half_even_mid(sa + ja, sa + jb);   // absolute positions
+            float mu2 = 0.f;
+            for (int i = lane; i < HALF; i += 32) {
+                float m0 = 0.f, m1 = 0.f, v0 = 0.f, v1 = 0.f;
+                for (int t = ja; t < jb; t++) {
+                    m0 += sm.kc[t][i];
+                    m1 += sm.kc[t][i + HALF];
+                    float wt = sm.Rt[t] + beta;
+                    v0 = fmaf(wt, to_f(sm.vv[t][i]), v0);
+                    v1 = fmaf(wt, to_f(sm.vv[t][i + HALF]), v1);
+                }
+                m0 *= ninv;
+                m1 *= ninv;
+                mu2 = fmaf(m0, m0, fmaf(m1, m1, mu2));
+                float2 cs = A.rope[(size_t)p * HALF + i];
+                sm.ktil[row][i] = m0 * cs.x - m1 * cs.y;
+                sm.ktil[row][i + HALF] = m0 * cs.y + m1 * cs.x;
+                sm.vtil[row][i] = v0 * winv;
+                sm.vtil[row][i + HALF] = v1 * winv;
+            }
+            mu2 = warp_sum(mu2);
+            if (lane == 0) {
+                const float coh = sqrtf(mu2) / (ks * ninv + A.eps);
+                const float me = (float)nJ * coh * coh;
+                sm.cand[k].meff = me < 1.0f ? 1.0f : (me > (float)nJ ? (float)nJ : me);
+            }
+        }
+    };
+    // D_u of candidate k (prototype row `row`) from the probe statistics Z, M
+    // of its interval; per-warp partial sums of pi_u D_u and pi_u.
+    auto evaluate = [&](int k, int row, float Z, const float *M) {
+        float x = 0.f;
+#pragma unroll
+        for (int q = 0; q < NQ; q++) {
+            float kv[8];
+            ld8(&sm.ktil[row][8 * (c + NCH * q)], kv);
+#pragma unroll
+            for (int r = 0; r < 8; r++) x = fmaf(qreg[8 * q + r], kv[r], x);
+        }
+#pragma unroll
+        for (int o = 1; o < NCH; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+        const float zt = sm.cand[k].meff * expf(x * A.inv_sqrt_d - mu);
+        float res = 0.f, mm = 0.f;
+#pragma unroll
+        for (int q = 0; q < NQ; q++) {
+            float vt[8];
+            ld8(&sm.vtil[row][8 * (c + NCH * q)], vt);
+#pragma unroll
+            for (int r = 0; r < 8; r++) {
+                const float mv = M[8 * q + r];
+                const float df = mv - zt * vt[r];
+                res = fmaf(df, df, res);
+                mm = fmaf(mv, mv, mm);
+            }
+        }
+#pragma unroll
+        for (int o = 1; o < NCH; o <<= 1) {
+            res += __shfl_xor_sync(0xffffffffu, res, o);
+            mm += __shfl_xor_sync(0xffffffffu, mm, o);
+        }
+        float pd = 0.f, pp = 0.f;
+        if (pact) {
+            const float dz = Z - zt;
+            const float Du = A.lamZ * (dz * dz) / (Z * Z + A.eps) + A.lamM * res / (mm + A.eps);
+            pp = Z * invZ;
+            pd = pp * Du;
+        }
+#pragma unroll
+        for (int o = NCH; o < 32; o <<= 1) {
+            pd += __shfl_xor_sync(0xffffffffu, pd, o);
+            pp += __shfl_xor_sync(0xffffffffu, pp, o);
+        }
+        if (lane == 0) { sm.redD[k][warp] = pd; sm.redP[k][warp] = pp; }
+    };
+    // Probe scan of one node in one direction, evaluating its candidates.
+    auto scan = [&](const BatchNode &B, bool suffix) {
+        const int a = sm.nodes[B.node].a, b = sm.nodes[B.node].b;
+        int k = suffix ? B.suf_b : B.pre_b;
+        const int ke = suffix ? B.suf_e : B.pre_e;
+        if (k >= ke) return;
+        float M[CH];
+        float Z = 0.f;
+#pragma unroll
+        for (int q = 0; q < CH; q++) M[q] = 0.f;
+        for (int s = 0; s < b - a && k < ke; s++) {
+            const int t = suffix ? b - 1 - s : a + s;
+            const float e = sm.E[t][u];
+            Z += e;
+#pragma unroll
+            for (int q = 0; q < NQ; q++) {
+                float vv[8];
+                ld8(&sm.vv[t][8 * (c + NCH * q)], vv);
+#pragma unroll
+                for (int r = 0; r < 8; r++) M[8 * q + r] = fmaf(e, vv[r], M[8 * q + r]);
+            }
+            while (k < ke && (suffix ? sm.cand[k].a == t : sm.cand[k].b == t + 1)) {
+                evaluate(k, suffix ? k - kNCD : k, Z, M);
+                k++;
+            }
+        }
+    };
+
     int cur = 0;
     int levels_left = A.max_levels;
     while (sm.nlvl[cur] > 0) {
@@ -335,21 +487,28 @@ __global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
         while (sm.batch_next < nl) {
             // ---- batch assignment (thread 0) --------------------------------
             if (tid == 0) {
-                int nb = 0, used = 0, k = sm.batch_next;
+                int nb = 0, upre = 0, usuf = 0, k = sm.batch_next;
                 while (k < nl && nb < S::NB) {
-                    int v = sm.lvl[cur][k];
-                    int nv = sm.nodes[v].b - sm.nodes[v].a;
-                    bool root = v == 0 && !A.resume;
-                    int ub = (root ? 1 : 0) + (nv >= 3 ? 2 * min(A.k_cand + 1, nv - 1) + 2 : 0);
-                    if (used + ub > S::NC) break;
+                    const int v = sm.lvl[cur][k];
+                    const int nv = sm.nodes[v].b - sm.nodes[v].a;
+                    const bool root = v == 0 && !A.resume;
+                    const int nc = nv >= 3 ? min(A.k_cand + 1, nv - 1) + 1 : 0;
+                    const int bp = nc + (root ? 1 : 0), bs = nc;
+                    if (upre + bp > kNCD || usuf + bs > kNCD) break;
                     sm.bn[nb].node = v;
-                    sm.bn[nb].pre_b = used;
-                    used += ub;
+                    sm.bn[nb].pre_b = upre;
+                    sm.bn[nb].suf_b = kNCD + usuf;
+                    upre += bp;
+                    usuf += bs;
+                    sm.bn[nb].pre_r = upre;
+                    sm.bn[nb].suf_r = kNCD + usuf;
                     nb++;
                     k++;
                 }
                 sm.batch_n = nb;
                 sm.batch_next = k;
+                sm.batch_pre = upre;
+                sm.batch_suf = usuf;
             }
             __syncthreads();
             const int nb = sm.batch_n;
@@ -359,10 +518,10 @@ __global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
                 const int v = B.node;
                 const int a = sm.nodes[v].a, b = sm.nodes[v].b, nv = b - a;
                 // top-K by curvature over positions [a, b-2] (ties: lower t)
-                unsigned sel[kMaxUnit / 32];
+                unsigned sel[NMAX / 32];
                 unsigned long long kmin = ~0ull, kmax = 0ull;
 #pragma unroll
-                for (int w = 0; w < kMaxUnit / 32; w++) {
+                for (int w = 0; w < NMAX / 32; w++) {
                     int t = a + w * 32 + lane;
                     bool in = t <= b - 2;
                     bool s = false;
@@ -407,7 +566,7 @@ __global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
                     int k = B.pre_b;
                     const bool cands = nv >= 3;
                     if (cands) {
-                        for (int w = 0; w < kMaxUnit / 32; w++) {
+                        for (int w = 0; w < NMAX / 32; w++) {
                             unsigned m = sel[w];
                             while (m) {
                                 int bit = __ffs(m) - 1;
@@ -433,7 +592,7 @@ __global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
                     }
                     if (v == 0 && !A.resume) { sm.cand[k] = {a, b, 0.f}; B.whole = k++; }
                     B.pre_e = k;
-                    B.suf_b = k;
+                    k = B.suf_b;
                     if (cands) {
                         // suffixes in descending start: cuts (descending) merged with p*+1
                         int er = pb + 1;
@@ -452,129 +611,34 @@ __global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
                         if (B.eR <= -2) B.eR = B.sidx[-2 - B.eR];
                     }
                     B.suf_e = k;
+                    for (int q = B.pre_e; q < B.pre_r; q++) sm.cand[q] = {0, 0, 0.f};
+                    for (int q = B.suf_e; q < B.suf_r; q++) sm.cand[q] = {0, 0, 0.f};
                 }
             }
             __syncthreads();
-            // ---- phase B: prototype of every candidate (warp per candidate) ----
-            for (int bi = 0; bi < nb; bi++) {
-                const BatchNode &B = sm.bn[bi];
-                for (int k = B.pre_b + warp; k < B.suf_e; k += NWARPS) {
-                    const int ja = sm.cand[k].a, jb = sm.cand[k].b, nJ = jb - ja;
-                    float rs = 0.f, ks = 0.f;
-                    for (int t = ja + lane; t < jb; t += 32) { rs += sm.Rt[t]; ks += sm.kn[t]; }
-                    rs = warp_sum(rs);
-                    ks = warp_sum(ks);
-                    const float ninv = 1.0f / (float)nJ;
-                    const float beta = (float)A.base_frac * (rs * ninv);
-                    const float wsum = rs + (float)nJ * beta;
-                    const float winv = 1.0f / (wsum + A.eps);
-                    const int p = round_half_even_mid(sa + ja, sa + jb);   // absolute positions
-                    float mu2 = 0.f;
-                    for (int i = lane; i < HALF; i += 32) {
-                        float m0 = 0.f, m1 = 0.f, v0 = 0.f, v1 = 0.f;
-                        for (int t = ja; t < jb; t++) {
-                            m0 += sm.kc[t][i];
-                            m1 += sm.kc[t][i + HALF];
-                            float wt = sm.Rt[t] + beta;
-                            v0 = fmaf(wt, to_f(sm.vv[t][i]), v0);
-                            v1 = fmaf(wt, to_f(sm.vv[t][i + HALF]), v1);
-                        }
-                        m0 *= ninv;
-                        m1 *= ninv;
-                        mu2 = fmaf(m0, m0, fmaf(m1, m1, mu2));
-                        float2 cs = A.rope[(size_t)p * HALF + i];
-                        sm.ktil[k][i] = m0 * cs.x - m1 * cs.y;
-                        sm.ktil[k][i + HALF] = m0 * cs.y + m1 * cs.x;
-                        sm.vtil[k][i] = v0 * winv;
-                        sm.vtil[k][i + HALF] = v1 * winv;
-                    }
-                    mu2 = warp_sum(mu2);
-                    if (lane == 0) {
-                        const float coh = sqrtf(mu2) / (ks * ninv + A.eps);
-                        const float me = (float)nJ * coh * coh;
-                        sm.cand[k].meff = me < 1.0f ? 1.0f : (me > (float)nJ ? (float)nJ : me);
-                    }
-                }
-            }
-            __syncthreads();
-            // ---- phase C: probe scans --------------------------------------------
-            auto evaluate = [&](int k, float Z, const float *M) {
-                float x = 0.f;
-#pragma unroll
-                for (int q = 0; q < CH; q++) x = fmaf(qreg[q], sm.ktil[k][c + NCH * q], x);
-#pragma unroll
-                for (int o = 1; o < NCH; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-                const float zt = sm.cand[k].meff * expf(x * A.inv_sqrt_d - mu);
-                float res = 0.f, mm = 0.f;
-#pragma unroll
-                for (int q = 0; q < CH; q++) {
-                    float df = M[q] - zt * sm.vtil[k][c + NCH * q];
-                    res = fmaf(df, df, res);
-                    mm = fmaf(M[q], M[q], mm);
-                }
-#pragma unroll
-                for (int o = 1; o < NCH; o <<= 1) {
-                    res += __shfl_xor_sync(0xffffffffu, res, o);
-                    mm += __shfl_xor_sync(0xffffffffu, mm, o);
-                }
-                float pd = 0.f, pp = 0.f;
-                if (pact) {
-                    float dz = Z - zt;
-                    float Du = A.lamZ * (dz * dz) / (Z * Z + A.eps) + A.lamM * res / (mm + A.eps);
-                    pp = Z * invZ;
-                    pd = pp * Du;
-                }
-#pragma unroll
-                for (int o = NCH; o < 32; o <<= 1) {
-                    pd += __shfl_xor_sync(0xffffffffu, pd, o);
-                    pp += __shfl_xor_sync(0xffffffffu, pp, o);
-                }
-                if (lane == 0) { sm.redD[k][warp] = pd; sm.redP[k][warp] = pp; }
-            };
-            for (int bi = 0; bi < nb; bi++) {
-                const BatchNode &B = sm.bn[bi];
-                if (B.pre_e == B.pre_b && B.suf_e == B.suf_b) continue;
-                const int a = sm.nodes[B.node].a, b = sm.nodes[B.node].b;
-                if (tid == 0) {
-                    int pe = B.pre_e > B.pre_b ? sm.cand[B.pre_e - 1].b : a;   // forward scan stops here
-                    int ss = B.suf_e > B.suf_b ? sm.cand[B.suf_e - 1].a : b;   // backward scan stops here
+            if (tid == 0) {
+                for (int bi = 0; bi < nb; bi++) {
+                    const BatchNode &B = sm.bn[bi];
+                    const int a = sm.nodes[B.node].a, b = sm.nodes[B.node].b;
+                    const int pe = B.pre_e > B.pre_b ? sm.cand[B.pre_e - 1].b : a;   // forward scan end
+                    const int ss = B.suf_e > B.suf_b ? sm.cand[B.suf_e - 1].a : b;   // backward scan end
                     w_scan += (pe - a) + (b - ss);
-                    w_eval += B.suf_e - B.pre_b;
-                    for (int k = B.pre_b; k < B.suf_e; k++) w_len += sm.cand[k].b - sm.cand[k].a;
-                }
-                float M[CH];
-                float Z = 0.f;
-                // forward: prefixes [a, end) in ascending end
-                int k = B.pre_b;
-                if (k < B.pre_e) {
-#pragma unroll
-                    for (int q = 0; q < CH; q++) M[q] = 0.f;
-                    for (int t = a; t < b && k < B.pre_e; t++) {
-                        const float e = sm.E[t][u];
-                        Z += e;
-#pragma unroll
-                        for (int q = 0; q < CH; q++) M[q] = fmaf(e, to_f(sm.vv[t][c + NCH * q]), M[q]);
-                        while (k < B.pre_e && sm.cand[k].b == t + 1) { evaluate(k, Z, M); k++; }
-                    }
-                }
-                // backward: suffixes [start, b) in descending start
-                k = B.suf_b;
-                if (k < B.suf_e) {
-                    Z = 0.f;
-#pragma unroll
-                    for (int q = 0; q < CH; q++) M[q] = 0.f;
-                    for (int t = b - 1; t >= a && k < B.suf_e; t--) {
-                        const float e = sm.E[t][u];
-                        Z += e;
-#pragma unroll
-                        for (int q = 0; q < CH; q++) M[q] = fmaf(e, to_f(sm.vv[t][c + NCH * q]), M[q]);
-                        while (k < B.suf_e && sm.cand[k].a == t) { evaluate(k, Z, M); k++; }
-                    }
+                    w_eval += (B.pre_e - B.pre_b) + (B.suf_e - B.suf_b);
+                    for (int k = B.pre_b; k < B.pre_e; k++) w_len += sm.cand[k].b - sm.cand[k].a;
+                    for (int k = B.suf_b; k < B.suf_e; k++) w_len += sm.cand[k].b - sm.cand[k].a;
                 }
             }
+            // ---- phases B/C: prefixes, then suffixes ---------------------------
+            prototypes(false);
+            __syncthreads();
+            for (int bi = 0; bi < nb; bi++) scan(sm.bn[bi], false);
+            __syncthreads();
+            prototypes(true);
+            __syncthreads();
+            for (int bi = 0; bi < nb; bi++) scan(sm.bn[bi], true);
             __syncthreads();
             // ---- per-candidate D and drop mass (thread per candidate) ------------
-            for (int k = tid; k < sm.bn[nb - 1].suf_e; k += NT) {
+            for (int k = tid; k < 2 * kNCD; k += kNT) {
                 double d = 0.0, pp = 0.0;
 #pragma unroll
                 for (int w = 0; w < NWARPS; w++) { d += sm.redD[k][w]; pp += sm.redP[k][w]; }
@@ -749,36 +813,37 @@ __global__ void __launch_bounds__(NT, 1) unit_build_kernel(BuildArgs A) {
     }
     // unused node slots of the unit carry cost 0 (no op)
     if (!A.resume)
-        for (int k = sm.nnodes + tid; k < 2 * n; k += NT) A.nd_cost[nbase + k] = 0;
+        for (int k = sm.nnodes + tid; k < 2 * n; k += kNT) A.nd_cost[nbase + k] = 0;
 }
 
-template <int DH, int NW, typename Tin>
+template <int DH, int NW, typename Tin, int NMAX>
 cudaError_t launch_t(Ctx &c, BuildArgs &A, unsigned grid, cudaStream_t s) {
-    constexpr int NT = 512;
-    using S = Smem<DH, NW, Tin, NT>;
+    using S = Smem<DH, NW, Tin, NMAX>;
     static_assert(sizeof(S) <= 227 * 1024, "unit kernel shared memory above the per-CTA limit");
+    if (grid == 0) return cudaSuccess;
     size_t sm = sizeof(S);
-    cudaError_t e = cudaFuncSetAttribute(unit_build_kernel<DH, NW, Tin, NT>,
+    cudaError_t e = cudaFuncSetAttribute(unit_build_kernel<DH, NW, Tin, NMAX>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
-    unit_build_kernel<DH, NW, Tin, NT><<<grid, NT, sm, s>>>(A);
+    unit_build_kernel<DH, NW, Tin, NMAX><<<grid, kNT, sm, s>>>(A);
     c.launches += 1;
     return cudaGetLastError();
 }
 
-template <typename Tin>
+template <typename Tin, int NMAX>
 cudaError_t launch_dt(Ctx &c, BuildArgs &A, unsigned grid, cudaStream_t s) {
     int nw = c.p.W <= 32 ? 32 : 64;
-    if (c.p.d == 128) return nw == 32 ? launch_t<128, 32, Tin>(c, A, grid, s) : launch_t<128, 64, Tin>(c, A, grid, s);
-    return nw == 32 ? launch_t<64, 32, Tin>(c, A, grid, s) : launch_t<64, 64, Tin>(c, A, grid, s);
+    if (c.p.d == 128)
+        return nw == 32 ? launch_t<128, 32, Tin, NMAX>(c, A, grid, s) : launch_t<128, 64, Tin, NMAX>(c, A, grid, s);
+    return nw == 32 ? launch_t<64, 32, Tin, NMAX>(c, A, grid, s) : launch_t<64, 64, Tin, NMAX>(c, A, grid, s);
 }
 
 }  // namespace
 
 cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *Q,
                               const float *omega, const int32_t *slots, int J, int resume,
-                              int max_levels, float tau, const int32_t *unit_list, int n_list,
-                              cudaStream_t s) {
+                              int max_levels, float tau, const int32_t *list_short, int n_short,
+                              const int32_t *list_long, int n_long, cudaStream_t s) {
     const gkv_params &p = c.p;
     BuildArgs A;
     A.K = K; A.V = V; A.Q = Q;
@@ -788,8 +853,8 @@ cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *
     A.cs = p.ctx_start; A.Nc = c.Nc; A.J = J; A.k_cand = p.k_cand;
     A.inv_sqrt_d = (float)(1.0 / sqrt((double)p.d));
     A.lamZ = (float)p.lambda_Z; A.lamM = (float)p.lambda_M; A.eps = (float)p.eps;
-    A.lam_kappa = p.lambda_kappa; A.base_frac = p.base_frac; A.eps_d = p.eps;
-    A.resume = resume; A.max_levels = max_levels; A.tau = tau; A.unit_list = unit_list;
+    A.lam_kappa = p.lambda_kappa; A.base_frac = p.base_frac;
+    A.resume = resume; A.max_levels = max_levels; A.tau = tau;
     A.nd_a = c.w.nd_a; A.nd_b = c.w.nd_b; A.nd_child0 = c.w.nd_child0;
     A.nd_parent = c.w.nd_parent; A.nd_unit = c.w.nd_unit;
     A.nd_nchild = c.w.nd_nchild; A.nd_cost = c.w.nd_cost;
@@ -799,10 +864,16 @@ cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *
     A.u_pend = c.w.u_pend;
     A.status = c.w.dev_int + 1;
     A.work = c.w.work;
-    unsigned grid = resume ? (unsigned)n_list : (unsigned)((int64_t)J * p.L * p.G);
-    if (grid == 0) return cudaSuccess;
-    if (p.dtype == GKV_BF16) return launch_dt<__nv_bfloat16>(c, A, grid, s);
-    return launch_dt<float>(c, A, grid, s);
+    const unsigned LG = (unsigned)(p.L * p.G);
+    const bool bf = p.dtype == GKV_BF16;
+    // short slots (<= 64 tokens) on the two-CTA-per-SM instance, the rest on the 128-token one
+    A.list = list_short;
+    unsigned g1 = resume ? (unsigned)n_short : (unsigned)n_short * LG;
+    cudaError_t e = bf ? launch_dt<__nv_bfloat16, 64>(c, A, g1, s) : launch_dt<float, 64>(c, A, g1, s);
+    if (e != cudaSuccess) return e;
+    A.list = list_long;
+    unsigned g2 = resume ? (unsigned)n_long : (unsigned)n_long * LG;
+    return bf ? launch_dt<__nv_bfloat16, kMaxUnit>(c, A, g2, s) : launch_dt<float, kMaxUnit>(c, A, g2, s);
 }
 
 }  // namespace gkv

@@ -176,14 +176,25 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
 
 cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t s);
 cudaError_t launch_token_values(Ctx &c, const void *K, const void *Q, cudaStream_t s);
+// Slots of at most kShortUnit tokens run on the unit kernel instance that fits
+// two CTAs per SM; the work lists hold them (slot indices for a fresh build,
+// unit ids for a resumed one) separately from the longer ones.
+constexpr int kShortUnit = 64;
 cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *Q,
                               const float *omega, const int32_t *slots, int J, int resume,
-                              int max_levels, float tau, const int32_t *unit_list, int n_list,
-                              cudaStream_t s);
+                              int max_levels, float tau, const int32_t *list_short, int n_short,
+                              const int32_t *list_long, int n_long, cudaStream_t s);
+// Slot indices split by length class: short ones at list[0, count[0]), long
+// ones at list[J - count[1], J).
+cudaError_t launch_slot_classes(Ctx &c, const int32_t *slots, int J, int32_t *list, int *count,
+                                cudaStream_t s);
 // Allocation threshold tau over the ops built so far (alloc_state prefix /
-// all-fit flag), and the list of units whose pending nodes qualify (key >= tau).
+// all-fit flag), and the units whose pending nodes qualify (key >= tau),
+// split by slot length class: short units at list[0, count[0]), long units at
+// list[n_units - count[1], n_units).
 cudaError_t launch_threshold(Ctx &c, int J, cudaStream_t s);
-cudaError_t launch_prune_list(Ctx &c, int J, int32_t *list, int *count, cudaStream_t s);
+cudaError_t launch_prune_list(Ctx &c, const int32_t *slots, int J, int32_t *list, int *count,
+                              cudaStream_t s);
 
 cudaError_t launch_allocate(Ctx &c, int J, cudaStream_t s);
 cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *slots, int J,
