@@ -143,8 +143,10 @@ def run_reference(args, w):
     print(json.dumps(out))
 
 
-def workload_config(w, ratio):
-    return {"workload": f"{w.name}@{int(ratio)}x", "L": w.L, "G": w.G, "Hq": w.Hq, "d": w.d,
+def workload_config(w, ratio, L=None):
+    L = w.L if L is None else L
+    name = w.name if L == w.L else f"{w.name}[{L} layers]"
+    return {"workload": f"{name}@{int(ratio)}x", "L": L, "G": w.G, "Hq": w.Hq, "d": w.d,
             "T": w.T, "W": w.W, "ratio": ratio, "dtype": w.dtype,
             "l2": "inputs larger than L2 (no flush needed)"}
 
@@ -161,6 +163,8 @@ def main():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--ref-tokens", type=int, default=1024)
+    ap.add_argument("--layers", type=int, default=0,
+                    help="compress only the first N layers (small cases for profiler captures)")
     args = ap.parse_args()
 
     from paper_2608_07001_gb300 import synth
@@ -180,7 +184,8 @@ def main():
 
     from paper_2608_07001_gb300 import gracekv as gk
     dev = torch.device("cuda", local)
-    x = synth.make_inputs(w, device=dev)
+    layers = list(range(args.layers)) if args.layers > 0 else None
+    x = synth.make_inputs(w, device=dev, layers=layers)
     K, V, Q = x.K, x.V, x.Q
     L, G, T, d = K.shape
     B = gk.gracekv_budget_for_ratio(L, G, T, args.ratio)
@@ -303,7 +308,7 @@ def main():
                "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
                "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                "dtype": "bf16" if K.dtype == torch.bfloat16 else "f32", "data": "synthetic",
-               "config": dict(workload_config(w, args.ratio), B_total=B, entries=E,
+               "config": dict(workload_config(w, args.ratio, L), B_total=B, entries=E,
                               slots=comp.n_slots, parallelism=f"replicas{world}"),
                "roofline": roof, "hbm_pass": hbm, "stages_ms": per_step, "tree_work": work,
                "cpu_baseline": cpu, "e2e": e2e,
