@@ -41,6 +41,8 @@
 // CTAs per SM; longer slots use the 128-token instance.
 #include "gkv_internal.cuh"
 
+#include <type_traits>
+
 namespace gkv {
 namespace {
 
@@ -91,14 +93,14 @@ struct BatchNode {
     int pstar, eL, eR, whole;
     int pre_b, pre_e, suf_b, suf_e;   // prefixes (ascending end) in [0, NCD),
                                       // suffixes (descending start) in [NCD, 2 NCD)
-    int pre_r, suf_r;                 // ends of the reserved candidate ranges
+    int pre_r, suf_r;                 // ends of the reserved ranges (unused entries empty)
     double kmin, kmax;
     int nchild, ca[3], cb[3];
     double cD[3];
 };
 
 struct Cand {
-    int a, b;        // local interval
+    int a, b;        // local interval (a == b: unused entry)
     float meff;
 };
 
@@ -136,6 +138,28 @@ __device__ __forceinline__ void ld8(const __nv_bfloat16 *p, float v[8]) {
     }
 }
 
+// N consecutive elements of a shared-memory row as floats (N = 1 or 2).
+template <int N>
+__device__ __forceinline__ void ld_pairs(const float *p, float v[N]) {
+    if constexpr (N == 2) {
+        const float2 x = *reinterpret_cast<const float2 *>(p);
+        v[0] = x.x; v[1] = x.y;
+    } else {
+#pragma unroll
+        for (int j = 0; j < N; j++) v[j] = p[j];
+    }
+}
+template <int N>
+__device__ __forceinline__ void ld_pairs(const __nv_bfloat16 *p, float v[N]) {
+    if constexpr (N == 2) {
+        const float2 x = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(p));
+        v[0] = x.x; v[1] = x.y;
+    } else {
+#pragma unroll
+        for (int j = 0; j < N; j++) v[j] = __bfloat162float(p[j]);
+    }
+}
+
 template <int DH, int NW, typename Tin, int NMAX>
 struct Smem {
     static constexpr int NWARPS = kNT / 32;
@@ -161,7 +185,8 @@ struct Smem {
     short lvl[2][MAXNODES];
     int nlvl[2];
     int nnodes;
-    int batch_n, batch_next, batch_pre, batch_suf;
+    int batch_n, batch_next, batch_pre, batch_suf;   // candidate entries reserved per direction
+    unsigned long long wcnt[kNT / 32][3];   // per-warp work counters
     float pend;
 };
 
@@ -239,18 +264,65 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     __syncthreads();
 
     // ---- E[t][u] from the raw (post-RoPE) keys -------------------------------
-    for (int t = 0; t < n; t++) {
-        float x = 0.f;
+    if constexpr (std::is_same<Tin, __nv_bfloat16>::value) {
+        // Tensor cores: logits = Q_probes (NW x DH) . K_slot^T, one 16x8 tile
+        // per (probe block, token block); warp w keeps probe block w % MT.
+        constexpr int MT = NW / 16, WSTEP = NWARPS / MT;
+        const int gr = lane >> 2, c2 = 2 * (lane & 3);
+        const int mt = warp % MT;
+        const int u0 = mt * 16 + gr, u1 = u0 + 8;
+        const __nv_bfloat16 *Qb = static_cast<const __nv_bfloat16 *>(A.Q);
+        const size_t r0 = ((size_t)l * A.Hq + g * A.gq + u0 % A.gq) * A.W + u0;
+        const size_t r1 = ((size_t)l * A.Hq + g * A.gq + u1 % A.gq) * A.W + u1;
+        const bool ok0 = u0 < A.W, ok1 = u1 < A.W;
+        uint32_t qa[DH / 16][4];
 #pragma unroll
-        for (int q = 0; q < NQ; q++) {
-            float kv[8];
-            ld8(&sm.kc[t][8 * (c + NCH * q)], kv);
-#pragma unroll
-            for (int r = 0; r < 8; r++) x = fmaf(qreg[8 * q + r], kv[r], x);
+        for (int ks = 0; ks < DH / 16; ks++) {
+            const __nv_bfloat16 *p0 = Qb + r0 * DH + ks * 16 + c2, *p1 = Qb + r1 * DH + ks * 16 + c2;
+            qa[ks][0] = ok0 ? *reinterpret_cast<const uint32_t *>(p0) : 0u;
+            qa[ks][1] = ok1 ? *reinterpret_cast<const uint32_t *>(p1) : 0u;
+            qa[ks][2] = ok0 ? *reinterpret_cast<const uint32_t *>(p0 + 8) : 0u;
+            qa[ks][3] = ok1 ? *reinterpret_cast<const uint32_t *>(p1 + 8) : 0u;
         }
+        const float m0 = ok0 ? A.row_m[r0] : 0.f, m1 = ok1 ? A.row_m[r1] : 0.f;
+        const int ntn = (n + 7) / 8;
+        for (int nt = warp / MT; nt < ntn; nt += WSTEP) {
+            float acc[4] = {0.f, 0.f, 0.f, 0.f};
+            const float *kr = &sm.kc[nt * 8 + gr][c2];
 #pragma unroll
-        for (int o = 1; o < NCH; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-        if (c == 0) sm.E[t][u] = pact ? expf(x * A.inv_sqrt_d - mu) : 0.f;
+            for (int ks = 0; ks < DH / 16; ks++) {
+                const float2 x0 = *reinterpret_cast<const float2 *>(kr + ks * 16);
+                const float2 x1 = *reinterpret_cast<const float2 *>(kr + ks * 16 + 8);
+                mma_bf16(acc, qa[ks], pack_bf16x2(x0.x, x0.y), pack_bf16x2(x1.x, x1.y));
+            }
+            const int t0 = nt * 8 + c2;
+            if (t0 < n) {
+                sm.E[t0][u0] = ok0 ? expf(acc[0] * A.inv_sqrt_d - m0) : 0.f;
+                sm.E[t0][u1] = ok1 ? expf(acc[2] * A.inv_sqrt_d - m1) : 0.f;
+            }
+            if (t0 + 1 < n) {
+                sm.E[t0 + 1][u0] = ok0 ? expf(acc[1] * A.inv_sqrt_d - m0) : 0.f;
+                sm.E[t0 + 1][u1] = ok1 ? expf(acc[3] * A.inv_sqrt_d - m1) : 0.f;
+            }
+        }
+    } else {
+        for (int t = 0; t < n; t++) {
+            float xs[NQ];
+#pragma unroll
+            for (int q = 0; q < NQ; q++) {
+                float kv[8];
+                ld8(&sm.kc[t][8 * (c + NCH * q)], kv);
+                xs[q] = 0.f;
+#pragma unroll
+                for (int r = 0; r < 8; r++) xs[q] = fmaf(qreg[8 * q + r], kv[r], xs[q]);
+            }
+            float x = xs[0];
+#pragma unroll
+            for (int q = 1; q < NQ; q++) x += xs[q];
+#pragma unroll
+            for (int o = 1; o < NCH; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+            if (c == 0) sm.E[t][u] = pact ? expf(x * A.inv_sqrt_d - mu) : 0.f;
+        }
     }
     __syncthreads();
     // Non-finite probe weights or token values (NaN/Inf in K, Q or the row
@@ -345,7 +417,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     }
     __syncthreads();
 
-    unsigned long long w_scan = 0, w_eval = 0, w_len = 0;   // thread 0's work counters
+    unsigned long long w_scan = 0, w_eval = 0, w_len = 0;   // work counters (lane 0 of each warp)
 
     // Prototypes of the batch's prefix (or suffix) candidates, warp per
     // candidate; reserved entries a node did not use are empty and skipped.
@@ -364,24 +436,38 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             const float wsum = rs + (float)nJ * beta;
             const float winv = 1.0f / (wsum + A.eps);
             const int p = round_half_even_mid(sa + ja, sa + jb);   // absolute positions
-            float mu2 = 0.f;
-            for (int i = lane; i < HALF; i += 32) {
-                float m0 = 0.f, m1 = 0.f, v0 = 0.f, v1 = 0.f;
-                for (int t = ja; t < jb; t++) {
-                    m0 += sm.kc[t][i];
-                    m1 += sm.kc[t][i + HALF];
-                    float wt = sm.Rt[t] + beta;
-                    v0 = fmaf(wt, to_f(sm.vv[t][i]), v0);
-                    v1 = fmaf(wt, to_f(sm.vv[t][i + HALF]), v1);
+            // lane owns the rotation pairs (i, i + d/2), i = PPL lane + j
+            constexpr int PPL = HALF / 32;
+            const int i0 = lane * PPL;
+            float m0[PPL], m1[PPL], v0[PPL], v1[PPL];
+#pragma unroll
+            for (int j = 0; j < PPL; j++) m0[j] = m1[j] = v0[j] = v1[j] = 0.f;
+#pragma unroll 2
+            for (int t = ja; t < jb; t++) {
+                float k0[PPL], k1[PPL], x0[PPL], x1[PPL];
+                ld_pairs<PPL>(&sm.kc[t][i0], k0);
+                ld_pairs<PPL>(&sm.kc[t][i0 + HALF], k1);
+                ld_pairs<PPL>(&sm.vv[t][i0], x0);
+                ld_pairs<PPL>(&sm.vv[t][i0 + HALF], x1);
+                const float wt = sm.Rt[t] + beta;
+#pragma unroll
+                for (int j = 0; j < PPL; j++) {
+                    m0[j] += k0[j];
+                    m1[j] += k1[j];
+                    v0[j] = fmaf(wt, x0[j], v0[j]);
+                    v1[j] = fmaf(wt, x1[j], v1[j]);
                 }
-                m0 *= ninv;
-                m1 *= ninv;
-                mu2 = fmaf(m0, m0, fmaf(m1, m1, mu2));
-                float2 cs = A.rope[(size_t)p * HALF + i];
-                sm.ktil[row][i] = m0 * cs.x - m1 * cs.y;
-                sm.ktil[row][i + HALF] = m0 * cs.y + m1 * cs.x;
-                sm.vtil[row][i] = v0 * winv;
-                sm.vtil[row][i + HALF] = v1 * winv;
+            }
+            float mu2 = 0.f;
+#pragma unroll
+            for (int j = 0; j < PPL; j++) {
+                const float a0 = m0[j] * ninv, a1 = m1[j] * ninv;
+                mu2 = fmaf(a0, a0, fmaf(a1, a1, mu2));
+                const float2 cs = A.rope[(size_t)p * HALF + i0 + j];
+                sm.ktil[row][i0 + j] = a0 * cs.x - a1 * cs.y;
+                sm.ktil[row][i0 + j + HALF] = a0 * cs.y + a1 * cs.x;
+                sm.vtil[row][i0 + j] = v0[j] * winv;
+                sm.vtil[row][i0 + j + HALF] = v1[j] * winv;
             }
             mu2 = warp_sum(mu2);
             if (lane == 0) {
@@ -394,30 +480,45 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     // D_u of candidate k (prototype row `row`) from the probe statistics Z, M
     // of its interval; per-warp partial sums of pi_u D_u and pi_u.
     auto evaluate = [&](int k, int row, float Z, const float *M) {
-        float x = 0.f;
+        float xs[2 * NQ];
 #pragma unroll
         for (int q = 0; q < NQ; q++) {
             float kv[8];
             ld8(&sm.ktil[row][8 * (c + NCH * q)], kv);
+            float x0 = 0.f, x1 = 0.f;
 #pragma unroll
-            for (int r = 0; r < 8; r++) x = fmaf(qreg[8 * q + r], kv[r], x);
+            for (int r = 0; r < 8; r += 2) {
+                x0 = fmaf(qreg[8 * q + r], kv[r], x0);
+                x1 = fmaf(qreg[8 * q + r + 1], kv[r + 1], x1);
+            }
+            xs[2 * q] = x0;
+            xs[2 * q + 1] = x1;
         }
+        float x = 0.f;
+#pragma unroll
+        for (int q = 0; q < 2 * NQ; q++) x += xs[q];
 #pragma unroll
         for (int o = 1; o < NCH; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
         const float zt = sm.cand[k].meff * expf(x * A.inv_sqrt_d - mu);
-        float res = 0.f, mm = 0.f;
+        float rq[NQ], mq[NQ];
 #pragma unroll
         for (int q = 0; q < NQ; q++) {
             float vt[8];
             ld8(&sm.vtil[row][8 * (c + NCH * q)], vt);
+            float r0 = 0.f, m0 = 0.f;
 #pragma unroll
             for (int r = 0; r < 8; r++) {
                 const float mv = M[8 * q + r];
                 const float df = mv - zt * vt[r];
-                res = fmaf(df, df, res);
-                mm = fmaf(mv, mv, mm);
+                r0 = fmaf(df, df, r0);
+                m0 = fmaf(mv, mv, m0);
             }
+            rq[q] = r0;
+            mq[q] = m0;
         }
+        float res = 0.f, mm = 0.f;
+#pragma unroll
+        for (int q = 0; q < NQ; q++) { res += rq[q]; mm += mq[q]; }
 #pragma unroll
         for (int o = 1; o < NCH; o <<= 1) {
             res += __shfl_xor_sync(0xffffffffu, res, o);
@@ -611,23 +712,18 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                         if (B.eR <= -2) B.eR = B.sidx[-2 - B.eR];
                     }
                     B.suf_e = k;
-                    for (int q = B.pre_e; q < B.pre_r; q++) sm.cand[q] = {0, 0, 0.f};
-                    for (int q = B.suf_e; q < B.suf_r; q++) sm.cand[q] = {0, 0, 0.f};
+                    for (int q = B.pre_e; q < B.pre_r; q++) sm.cand[q].a = sm.cand[q].b = 0;
+                    for (int q = B.suf_e; q < B.suf_r; q++) sm.cand[q].a = sm.cand[q].b = 0;
+                    // work counters: tokens swept, candidates evaluated, their lengths
+                    const int pe = B.pre_e > B.pre_b ? sm.cand[B.pre_e - 1].b : a;
+                    const int ss = B.suf_e > B.suf_b ? sm.cand[B.suf_e - 1].a : b;
+                    w_scan += (pe - a) + (b - ss);
+                    w_eval += (B.pre_e - B.pre_b) + (B.suf_e - B.suf_b);
+                    for (int q = B.pre_b; q < B.pre_e; q++) w_len += sm.cand[q].b - sm.cand[q].a;
+                    for (int q = B.suf_b; q < B.suf_e; q++) w_len += sm.cand[q].b - sm.cand[q].a;
                 }
             }
             __syncthreads();
-            if (tid == 0) {
-                for (int bi = 0; bi < nb; bi++) {
-                    const BatchNode &B = sm.bn[bi];
-                    const int a = sm.nodes[B.node].a, b = sm.nodes[B.node].b;
-                    const int pe = B.pre_e > B.pre_b ? sm.cand[B.pre_e - 1].b : a;   // forward scan end
-                    const int ss = B.suf_e > B.suf_b ? sm.cand[B.suf_e - 1].a : b;   // backward scan end
-                    w_scan += (pe - a) + (b - ss);
-                    w_eval += (B.pre_e - B.pre_b) + (B.suf_e - B.suf_b);
-                    for (int k = B.pre_b; k < B.pre_e; k++) w_len += sm.cand[k].b - sm.cand[k].a;
-                    for (int k = B.suf_b; k < B.suf_e; k++) w_len += sm.cand[k].b - sm.cand[k].a;
-                }
-            }
             // ---- phases B/C: prefixes, then suffixes ---------------------------
             prototypes(false);
             __syncthreads();
@@ -801,14 +897,18 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         __syncthreads();
         cur ^= 1;
     }
+    if (lane == 0) { sm.wcnt[warp][0] = w_scan; sm.wcnt[warp][1] = w_eval; sm.wcnt[warp][2] = w_len; }
     __syncthreads();
     if (tid == 0) {
         A.u_nnodes[uid] = sm.nnodes;
         A.u_pend[uid] = sm.pend;
         if (!A.resume) A.u_sel[uid] = 0;
-        atomicAdd(&A.work[0], w_scan);
-        atomicAdd(&A.work[1], w_eval);
-        atomicAdd(&A.work[2], w_len);
+        unsigned long long tot[3] = {0, 0, 0};
+        for (int w = 0; w < NWARPS; w++)
+            for (int q = 0; q < 3; q++) tot[q] += sm.wcnt[w][q];
+        atomicAdd(&A.work[0], tot[0]);
+        atomicAdd(&A.work[1], tot[1]);
+        atomicAdd(&A.work[2], tot[2]);
         atomicAdd(&A.work[3], 1ull);
     }
     // unused node slots of the unit carry cost 0 (no op)

@@ -163,6 +163,23 @@ __device__ __forceinline__ float warp_max(float v) {
     return v;
 }
 
+// D += A B on the tensor cores: one m16n8k16 tile, bf16 operands (exact
+// products), fp32 accumulation.  a: row-major 16x16 fragment, b0/b1: the
+// column-major 16x8 fragment, c: the 16x8 accumulator (PTX ISA fragment
+// layouts for mma.m16n8k16 with .bf16 operands).
+__device__ __forceinline__ void mma_bf16(float c[4], const uint32_t a[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+        "{%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};\n"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+// Two floats (exactly representable in bf16) packed as a bf16x2 operand word.
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t *>(&h);
+}
+
 // Monotone 32-bit key of a non-negative float (larger value -> larger key).
 __device__ __forceinline__ uint32_t fkey(float x) { return __float_as_uint(x); }
 

@@ -231,14 +231,6 @@ constexpr int kMT = 64;           // tokens per tile
 constexpr int kMmaWarps = 16;
 constexpr float kLog2e = 1.4426950408889634f;
 
-__device__ __forceinline__ void mma_bf16(float c[4], const uint32_t a[4], uint32_t b0, uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
-        "{%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};\n"
-        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-
 __device__ __forceinline__ void cp_async16(void *smem, const void *gmem, bool pred) {
     unsigned s = (unsigned)__cvta_generic_to_shared(smem);
     int n = pred ? 16 : 0;   // zero-fill past the end
