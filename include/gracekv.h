@@ -23,6 +23,9 @@
  *     T..T+W-1, all seeing [0, T)) has layout [L][Hq][W][d]; query head h
  *     belongs to KV head h / (Hq / G).  Element type = params.dtype
  *     (fp32 or bf16) for K, V, Q, K_out and V_out.
+ *   - K, V, Q, K_out and V_out must start on a 16-byte boundary (they are
+ *     read and written as 16-byte vectors); int32/float arrays on 4 bytes,
+ *     int64 arrays on 8.  A misaligned pointer returns GKV_EINVAL.
  *   - `stream` is a cudaStream_t passed as void*; work is enqueued on it.
  *     Calls that return a host count (*_host) synchronise that stream once.
  *   - Every call returns a gkv_status and never aborts or throws.  A CUDA
@@ -114,7 +117,8 @@ gkv_status gracekv_query(const gracekv_ctx *ctx, int32_t *recent, int32_t *n_c,
 /*
  * Stage 1 -- curvature-guided segmentation (App. B.2-B.3).
  * Trajectory h^(l)_t = concat_g V[l][g][t][:] at the segmentation layers
- * (or `hidden` [n_seg][T][Dh] fp32 when given), multi-scale curvature
+ * (or `hidden` [n_seg][T][Dh] fp32 when given, Dh a multiple of 8 up to
+ * 2048, 16-byte aligned), multi-scale curvature
  * (Eq. app_local_curvature), stabilised curvature (Eq.
  * app_stabilized_curvature), robust-z boundary score (Eq. app_boundary_score,
  * surprisal [T] fp32 optional, 0 when NULL), and the length-constrained DP

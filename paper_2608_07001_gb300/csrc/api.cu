@@ -249,6 +249,13 @@ gkv_status gracekv_query(const gracekv_ctx *x, int32_t *recent, int32_t *n_c, in
     return GKV_OK;
 }
 
+// Device tensors are read and written as 16-byte vectors (8-byte for the
+// float2 tables), so their base addresses must be 16-byte aligned; index and
+// scalar arrays need their natural alignment.
+static bool al16(const void *p) { return p && (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+static bool al4(const void *p) { return !p || (reinterpret_cast<uintptr_t>(p) & 3u) == 0; }
+static bool al8(const void *p) { return !p || (reinterpret_cast<uintptr_t>(p) & 7u) == 0; }
+
 gkv_status gracekv_segment(gracekv_ctx *x, const void *V, const float *hidden, int32_t Dh,
                            const float *surprisal, int32_t *slot_starts, int32_t cap,
                            int32_t *n_slots_host, float *kappa, void *stream) {
@@ -256,7 +263,10 @@ gkv_status gracekv_segment(gracekv_ctx *x, const void *V, const float *hidden, i
     if (st) return st;
     Ctx &c = x->c;
     if (!V || !slot_starts || !n_slots_host || cap < 1) return fail(x, GKV_EINVAL, "segment: null argument");
-    if (hidden && (Dh <= 0 || Dh > 2048)) return fail(x, GKV_EINVAL, "segment: hidden dim must be in [1, 2048]");
+    if (!al16(V) || (hidden && !al16(hidden)) || !al4(surprisal) || !al4(slot_starts) || !al4(kappa))
+        return fail(x, GKV_EINVAL, "segment: misaligned pointer (V and hidden need 16 bytes, the others 4)");
+    if (hidden && (Dh <= 0 || Dh > 2048 || Dh % 8))
+        return fail(x, GKV_EINVAL, "segment: hidden dim must be a multiple of 8 in [8, 2048]");
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t e = cudaMemsetAsync(c.w.dev_int, 0, 16 * sizeof(int), s);
     if (e == cudaSuccess) {
@@ -288,6 +298,8 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
     if (st) return st;
     Ctx &c = x->c;
     if (!K || !V || !Q) return fail(x, GKV_EINVAL, "build_trees: null tensor");
+    if (!al16(K) || !al16(V) || !al16(Q) || !al4(omega) || !al4(slot_starts))
+        return fail(x, GKV_EINVAL, "build_trees: misaligned pointer (K, V, Q need 16 bytes)");
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t e;
     if (slot_starts) {
@@ -412,6 +424,9 @@ gkv_status gracekv_gather(gracekv_ctx *x, const void *K, const void *V, void *K_
     Ctx &c = x->c;
     if (!K || !V || !K_out || !V_out || !pos || !log_m || !src_lo || !src_hi || !offsets)
         return fail(x, GKV_EINVAL, "gather: null argument");
+    if (!al16(K) || !al16(V) || !al16(K_out) || !al16(V_out) || !al4(pos) || !al4(log_m) ||
+        !al4(src_lo) || !al4(src_hi) || !al8(offsets))
+        return fail(x, GKV_EINVAL, "gather: misaligned pointer (K, V, K_out, V_out need 16 bytes)");
     const int64_t LG = (int64_t)c.p.L * c.p.G;
     if (cap < LG * (c.p.T - c.Nc) + c.used) return fail(x, GKV_ECAPACITY, "gather: cap below the entry count");
     cudaError_t e;

@@ -45,8 +45,6 @@ __device__ __forceinline__ int round_half_even_mid(int a, int b) {
     return (lo & 1) == 0 ? lo : lo + 1;
 }
 
-__device__ __forceinline__ void store(float *p, float x) { *p = x; }
-__device__ __forceinline__ void store(__nv_bfloat16 *p, float x) { *p = __float2bfloat16_rn(x); }
 
 __global__ void gather_count_kernel(GatherArgs A) {
     int64_t nu = (int64_t)A.L * A.G * A.J;
@@ -96,79 +94,156 @@ __global__ void __launch_bounds__(1024) gather_scan_kernel(GatherArgs A) {
         for (int lg = 0; lg <= A.L * A.G; lg++) A.offsets[lg] = (long long)lg * extra;
 }
 
-template <typename Tin>
+// 8 consecutive elements copied bit for bit.
+__device__ __forceinline__ void copy8(__nv_bfloat16 *dst, const __nv_bfloat16 *src) {
+    *reinterpret_cast<uint4 *>(dst) = *reinterpret_cast<const uint4 *>(src);
+}
+__device__ __forceinline__ void copy8(float *dst, const float *src) {
+    reinterpret_cast<uint4 *>(dst)[0] = reinterpret_cast<const uint4 *>(src)[0];
+    reinterpret_cast<uint4 *>(dst)[1] = reinterpret_cast<const uint4 *>(src)[1];
+}
+__device__ __forceinline__ void store8(__nv_bfloat16 *dst, const float v[8]) {
+    uint4 u;
+    __nv_bfloat162 *h = reinterpret_cast<__nv_bfloat162 *>(&u);
+#pragma unroll
+    for (int j = 0; j < 4; j++) h[j] = __floats2bfloat162_rn(v[2 * j], v[2 * j + 1]);
+    *reinterpret_cast<uint4 *>(dst) = u;
+}
+__device__ __forceinline__ void store8(float *dst, const float v[8]) {
+    reinterpret_cast<float4 *>(dst)[0] = make_float4(v[0], v[1], v[2], v[3]);
+    reinterpret_cast<float4 *>(dst)[1] = make_float4(v[4], v[5], v[6], v[7]);
+}
+
+// One frontier node [a, b) of head lg -> cache entry e (one warp).  Rows are
+// read as 8-element chunks, LPR = d / 8 lanes per row and 32 / LPR rows per
+// step; the chunk holding elements i .. i+7 of the first half and the one
+// holding i + d/2 .. of the second half sit PX = LPR / 2 lanes apart, so the
+// rotation partner comes from a shuffle.  All arithmetic is fp32.
+template <typename Tin, int DH>
 __device__ void emit_node(const GatherArgs &A, int lg, int a, int b, int64_t e, int lane) {
-    const int d = A.d, half = d / 2;
-    const Tin *K = static_cast<const Tin *>(A.K) + (size_t)lg * A.T * d;
-    const Tin *V = static_cast<const Tin *>(A.V) + (size_t)lg * A.T * d;
-    Tin *Ko = static_cast<Tin *>(A.K_out) + (size_t)e * d;
-    Tin *Vo = static_cast<Tin *>(A.V_out) + (size_t)e * d;
+    constexpr int HALF = DH / 2, LPR = DH / 8, RPW = 32 / LPR, PX = LPR / 2;
+    const int r = lane / LPR, c = lane - r * LPR;
+    const bool hi = c >= PX;                   // chunk in the second half
+    const int i0 = 8 * (c - (hi ? PX : 0));    // pair index of the chunk's first element
+    const Tin *K = static_cast<const Tin *>(A.K) + (size_t)lg * A.T * DH;
+    const Tin *V = static_cast<const Tin *>(A.V) + (size_t)lg * A.T * DH;
+    Tin *Ko = static_cast<Tin *>(A.K_out) + (size_t)e * DH;
+    Tin *Vo = static_cast<Tin *>(A.V_out) + (size_t)e * DH;
     const int n = b - a;
-    if (n == 1) {
-        for (int i = lane; i < d; i += 32) {
-            Ko[i] = K[(size_t)a * d + i];
-            Vo[i] = V[(size_t)a * d + i];
+    if (n == 1) {   // single token: original bits, p = t, log m = 0
+        if (lane < LPR) {
+            copy8(Ko + 8 * c, K + (size_t)a * DH + 8 * c);
+            copy8(Vo + 8 * c, V + (size_t)a * DH + 8 * c);
         }
         if (lane == 0) { A.pos[e] = a; A.log_m[e] = 0.f; A.src_lo[e] = a; A.src_hi[e] = b; }
         return;
     }
     const float *R = A.rtok + (size_t)lg * A.Nc - A.cs;
-    double rs = 0.0;
+    float rs = 0.f;
     for (int t = a + lane; t < b; t += 32) rs += R[t];
     rs = warp_sum(rs);
-    const float beta = (float)(A.base_frac * (rs / n));
-    const double wsum = rs + n * (double)beta;
-    const float winv = (float)(1.0 / (wsum + A.eps));
     const float ninv = 1.0f / (float)n;
+    const float beta = (float)A.base_frac * (rs * ninv);
+    const float winv = 1.0f / (rs + (float)n * beta + (float)A.eps);
+    float mk[8], mv[8], kn = 0.f;
+#pragma unroll
+    for (int j = 0; j < 8; j++) mk[j] = mv[j] = 0.f;
+    constexpr int U = 2;   // row groups whose loads are issued together
+    for (int t0 = a; t0 < b; t0 += U * RPW) {
+        Vec8<Tin> kx[U], vx[U];
+        float4 cs[U][4];
+        float wt[U];
+        bool ok[U];
+#pragma unroll
+        for (int g = 0; g < U; g++) {
+            const int t = t0 + g * RPW + r;
+            ok[g] = t < b;
+            if (ok[g]) {
+                kx[g].load(K + (size_t)t * DH + 8 * c);
+                vx[g].load(V + (size_t)t * DH + 8 * c);
+                const float4 *cs4 = reinterpret_cast<const float4 *>(A.rope + (size_t)t * HALF + i0);
+#pragma unroll
+                for (int j2 = 0; j2 < 4; j2++) cs[g][j2] = cs4[j2];
+                wt[g] = R[t] + beta;
+            } else {
+#pragma unroll
+                for (int j = 0; j < 8; j++) kx[g].v[j] = vx[g].v[j] = 0.f;
+#pragma unroll
+                for (int j2 = 0; j2 < 4; j2++) cs[g][j2] = make_float4(0.f, 0.f, 0.f, 0.f);
+                wt[g] = 0.f;
+            }
+        }
+#pragma unroll
+        for (int g = 0; g < U; g++) {
+            float y[8], nn = 0.f;
+#pragma unroll
+            for (int j = 0; j < 8; j++) {
+                y[j] = __shfl_xor_sync(0xffffffffu, kx[g].v[j], PX);
+                nn = fmaf(kx[g].v[j], kx[g].v[j], nn);
+            }
+#pragma unroll
+            for (int o = 1; o < LPR; o <<= 1) nn += __shfl_xor_sync(0xffffffffu, nn, o);
+            if (ok[g] && c == 0) kn += sqrtf(nn);   // |k_circ_t| = |k_t| (RoPE is a rotation)
+#pragma unroll
+            for (int j2 = 0; j2 < 4; j2++) {
+                const float4 q = cs[g][j2];          // (cos, sin) of pairs i0 + 2 j2, i0 + 2 j2 + 1
+                const float cc[2] = {q.x, q.z}, sn[2] = {q.y, q.w};
+#pragma unroll
+                for (int h = 0; h < 2; h++) {
+                    const int j = 2 * j2 + h;
+                    // RoPE^-1(k, t): x' = x cos + y sin, y' = y cos - x sin (rows past b add 0)
+                    mk[j] += hi ? fmaf(kx[g].v[j], cc[h], -y[j] * sn[h]) : fmaf(kx[g].v[j], cc[h], y[j] * sn[h]);
+                    mv[j] = fmaf(wt[g], vx[g].v[j], mv[j]);
+                }
+            }
+        }
+    }
+    // combine the row groups
+#pragma unroll
+    for (int o = LPR; o < 32; o <<= 1) {
+#pragma unroll
+        for (int j = 0; j < 8; j++) {
+            mk[j] += __shfl_xor_sync(0xffffffffu, mk[j], o);
+            mv[j] += __shfl_xor_sync(0xffffffffu, mv[j], o);
+        }
+        kn += __shfl_xor_sync(0xffffffffu, kn, o);
+    }
+    kn = __shfl_sync(0xffffffffu, kn, 0);
     const int p = round_half_even_mid(a, b);
-    // mean of the inverse-rotated keys and the mean of their norms
-    double knorm = 0.0;
-    float mu2 = 0.f;
-    constexpr int kMaxPairs = 4;   // d / 2 / 32 <= 2 for d <= 128 (4 for 256)
-    float m0[kMaxPairs], m1[kMaxPairs];
+    float u[8], pu[8], mu2 = 0.f;
 #pragma unroll
-    for (int q = 0; q < kMaxPairs; q++) m0[q] = m1[q] = 0.f;
-    for (int t = a; t < b; t++) {
-        float nn = 0.f;
-#pragma unroll
-        for (int q = 0; q < kMaxPairs; q++) {
-            int i = lane + 32 * q;
-            if (i >= half) break;
-            float2 cs = A.rope[(size_t)t * half + i];
-            float x = to_f(K[(size_t)t * d + i]), y = to_f(K[(size_t)t * d + i + half]);
-            float kx = x * cs.x + y * cs.y, ky = y * cs.x - x * cs.y;
-            m0[q] += kx;
-            m1[q] += ky;
-            nn = fmaf(kx, kx, fmaf(ky, ky, nn));
-        }
-        nn = warp_sum(nn);
-        knorm += sqrt((double)nn);
+    for (int j = 0; j < 8; j++) {
+        u[j] = mk[j] * ninv;
+        mu2 = fmaf(u[j], u[j], mu2);
     }
 #pragma unroll
-    for (int q = 0; q < kMaxPairs; q++) {
-        int i = lane + 32 * q;
-        if (i >= half) break;
-        float u0 = m0[q] * ninv, u1 = m1[q] * ninv;
-        mu2 = fmaf(u0, u0, fmaf(u1, u1, mu2));
-        float2 cs = A.rope[(size_t)p * half + i];
-        store(Ko + i, u0 * cs.x - u1 * cs.y);
-        store(Ko + i + half, u0 * cs.y + u1 * cs.x);
-        float v0 = 0.f, v1 = 0.f;
-        for (int t = a; t < b; t++) {
-            float wt = R[t] + beta;
-            v0 = fmaf(wt, to_f(V[(size_t)t * d + i]), v0);
-            v1 = fmaf(wt, to_f(V[(size_t)t * d + i + half]), v1);
+    for (int o = 1; o < LPR; o <<= 1) mu2 += __shfl_xor_sync(0xffffffffu, mu2, o);
+#pragma unroll
+    for (int j = 0; j < 8; j++) pu[j] = __shfl_xor_sync(0xffffffffu, u[j], PX);
+    if (lane < LPR) {
+        const float4 *cs4 = reinterpret_cast<const float4 *>(A.rope + (size_t)p * HALF + i0);
+        float ko[8], vo[8];
+#pragma unroll
+        for (int j2 = 0; j2 < 4; j2++) {
+            const float4 q = cs4[j2];
+            const float cc[2] = {q.x, q.z}, sn[2] = {q.y, q.w};
+#pragma unroll
+            for (int h = 0; h < 2; h++) {
+                const int j = 2 * j2 + h;
+                // RoPE(mu, p): x' = x cos - y sin, y' = x sin + y cos
+                ko[j] = hi ? fmaf(u[j], cc[h], pu[j] * sn[h]) : fmaf(u[j], cc[h], -pu[j] * sn[h]);
+                vo[j] = mv[j] * winv;
+            }
         }
-        store(Vo + i, v0 * winv);
-        store(Vo + i + half, v1 * winv);
+        store8(Ko + 8 * c, ko);
+        store8(Vo + 8 * c, vo);
     }
-    mu2 = warp_sum(mu2);
     if (lane == 0) {
-        double coh = sqrt((double)mu2) / (knorm / n + A.eps);
-        double me = n * coh * coh;
-        me = me < 1.0 ? 1.0 : (me > n ? (double)n : me);
+        const float coh = sqrtf(mu2) / (kn * ninv + (float)A.eps);
+        float me = (float)n * coh * coh;
+        me = me < 1.0f ? 1.0f : (me > (float)n ? (float)n : me);
         A.pos[e] = p;
-        A.log_m[e] = (float)log(me);
+        A.log_m[e] = logf(me);
         A.src_lo[e] = a;
         A.src_hi[e] = b;
     }
@@ -176,8 +251,8 @@ __device__ void emit_node(const GatherArgs &A, int lg, int a, int b, int64_t e, 
 
 // Warp per unit: depth-first traversal of the executed splits, children in
 // ascending position, so frontier nodes come out in ascending position.
-template <typename Tin>
-__global__ void gather_units_kernel(GatherArgs A) {
+template <typename Tin, int DH>
+__global__ void __launch_bounds__(256, 2) gather_units_kernel(GatherArgs A) {
     __shared__ short stack[8][kMaxUnit + 4];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t nu = (int64_t)A.L * A.G * A.J;
@@ -206,7 +281,7 @@ __global__ void gather_units_kernel(GatherArgs A) {
         }
         k = __shfl_sync(0xffffffffu, k, 0);
         if (k < 0) break;
-        emit_node<Tin>(A, lg, A.nd_a[nb + k], A.nd_b[nb + k], e, lane);
+        emit_node<Tin, DH>(A, lg, A.nd_a[nb + k], A.nd_b[nb + k], e, lane);
         e++;
     }
 }
@@ -250,8 +325,13 @@ cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *s
     const bool bf = c.p.dtype == GKV_BF16;
     unsigned gu = (unsigned)((nu + 7) / 8);
     if (gu) {
-        if (bf) gather_units_kernel<__nv_bfloat16><<<gu, 256, 0, s>>>(A);
-        else gather_units_kernel<float><<<gu, 256, 0, s>>>(A);
+        if (c.p.d == 128) {
+            if (bf) gather_units_kernel<__nv_bfloat16, 128><<<gu, 256, 0, s>>>(A);
+            else gather_units_kernel<float, 128><<<gu, 256, 0, s>>>(A);
+        } else {
+            if (bf) gather_units_kernel<__nv_bfloat16, 64><<<gu, 256, 0, s>>>(A);
+            else gather_units_kernel<float, 64><<<gu, 256, 0, s>>>(A);
+        }
     }
     int ntok = c.p.ctx_start + (c.p.T - c.c_end);
     c.launches += 2 + (gu ? 1 : 0) + (ntok > 0 ? 1 : 0);

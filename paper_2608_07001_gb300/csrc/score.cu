@@ -231,15 +231,6 @@ constexpr int kMT = 64;           // tokens per tile
 constexpr int kMmaWarps = 16;
 constexpr float kLog2e = 1.4426950408889634f;
 
-__device__ __forceinline__ void cp_async16(void *smem, const void *gmem, bool pred) {
-    unsigned s = (unsigned)__cvta_generic_to_shared(smem);
-    int n = pred ? 16 : 0;   // zero-fill past the end
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(s), "l"(gmem), "r"(n));
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N)); }
-
 // Stage tokens [t0, t0 + 64) of K (row-major [T][DH]) into a padded tile.
 template <int DH>
 __device__ __forceinline__ void stage_tile(__nv_bfloat16 *tile, const __nv_bfloat16 *Kl, int t0, int tend) {
@@ -592,6 +583,10 @@ extern "C" gkv_status gracekv_row_stats_noalloc(const void *K, const void *Q, in
                                                 float *row_m, float *row_Z, float *row_ZC,
                                                 void *stream) {
     if (!K || !Q || !row_m || !row_Z || !row_ZC) return GKV_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(K) & 15u) || (reinterpret_cast<uintptr_t>(Q) & 15u) ||
+        (reinterpret_cast<uintptr_t>(row_m) & 3u) || (reinterpret_cast<uintptr_t>(row_Z) & 3u) ||
+        (reinterpret_cast<uintptr_t>(row_ZC) & 3u))
+        return GKV_EINVAL;
     if (L <= 0 || G <= 0 || Hq <= 0 || T <= 0 || d <= 0 || W <= 0 || Hq % G || d % 8) return GKV_EINVAL;
     if (dtype != GKV_F32 && dtype != GKV_BF16) return GKV_EINVAL;
     if (c_lo < 0 || c_hi > T || c_lo > c_hi) return GKV_EINVAL;

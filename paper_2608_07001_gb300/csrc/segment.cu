@@ -74,7 +74,7 @@ __global__ void seg_norm_kernel(const Tin *V, const float *hidden, SegArgs a, fl
     int lane = threadIdx.x & 31;
     if (t >= a.T) return;
     int l = a.layers[li];
-    double s = 0.0;
+    float s = 0.f;
     if (!hidden && (a.d % 8) == 0) {
         for (int c = lane * 8; c < a.D; c += 256) {
             int g = c / a.d, i = c - g * a.d;
@@ -88,127 +88,146 @@ __global__ void seg_norm_kernel(const Tin *V, const float *hidden, SegArgs a, fl
     } else {
         for (int c = lane; c < a.D; c += 32) {
             float x = traj_elem(V, hidden, a.Dh, a.G, a.T, a.d, l, li, t, c);
-            s += (double)x * x;
+            s = fmaf(x, x, s);
         }
     }
     s = warp_sum(s);
     if (lane == 0) {
-        double n = sqrt(s);
-        double den = n > kEps ? n : kEps;
-        inv_norm[(size_t)li * a.T + t] = (float)(1.0 / den);
-        nrm2[(size_t)li * a.T + t] = (float)(s / (den * den));
+        const float n = sqrtf(s);
+        const float den = n > (float)kEps ? n : (float)kEps;
+        inv_norm[(size_t)li * a.T + t] = 1.0f / den;
+        nrm2[(size_t)li * a.T + t] = s / (den * den);
     }
 }
 
 // ---------------------------------------------------------------------------
-// Curvature.  Block = 256 threads, tile of PT positions of one layer.  The
-// raw rows [i0 - 16, i0 + PT + 16) are staged in shared memory; every thread
-// owns channels c = tid, tid + 256, ... and slides the window sums of its
-// channels along the tile; per position the 9 dot products (3 windows x
-// {||d-||^2, ||d+||^2, d-.d+}, up to 4 windows) are reduced per warp into shared memory and
-// combined across warps once per tile.
+// Curvature.  Block = 256 threads = 256 consecutive positions (one per
+// thread) of one segmentation layer.  The trajectory channels are staged in
+// chunks of kCurvCC channels, already normalised (hbar = h / max(|h|, eps)),
+// channel-major in shared memory so that the threads of a warp read
+// consecutive rows.  Each thread forms its window sums directly (running sums
+// outward from its position, left window [i-w+1, i], right window [i+1, i+w])
+// and accumulates |d-|^2, |d+|^2 and d-.d+ over all channels in registers: no
+// cross-thread reduction.
 // ---------------------------------------------------------------------------
-constexpr int kHalo = 16;
+constexpr int kHalo = 16;                       // largest window
+constexpr int kCurvPT = 256;                    // positions per block
+constexpr int kCurvRows = kCurvPT + 2 * kHalo;  // staged rows
+constexpr int kCurvRS = kCurvRows + 1;          // row stride (odd: 2-way staging conflicts at most)
+constexpr int kCurvCC = 64;                     // channels per stage
+constexpr size_t kCurvSmem = ((size_t)kCurvCC * kCurvRS + kCurvRows) * sizeof(float);
 
+// 8 consecutive trajectory channels c .. c+7 (c % 8 == 0) of row t, or zeros
+// outside [0, T).
 template <typename Tin>
+__device__ __forceinline__ void traj_load8(const Tin *V, const float *hidden, const SegArgs &a,
+                                           int l, int li, int t, int c, float v[8]) {
+    if (t < 0 || t >= a.T) {
+#pragma unroll
+        for (int j = 0; j < 8; j++) v[j] = 0.f;
+        return;
+    }
+    if (hidden) {
+        const float4 *p = reinterpret_cast<const float4 *>(hidden + ((size_t)li * a.T + t) * a.Dh + c);
+        const float4 x = p[0], y = p[1];
+        v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w; v[4] = y.x; v[5] = y.y; v[6] = y.z; v[7] = y.w;
+        return;
+    }
+    const int g = c / a.d, i = c - g * a.d;
+    Vec8<Tin> x;
+    x.load(V + (((size_t)l * a.G + g) * a.T + t) * a.d + i);
+#pragma unroll
+    for (int j = 0; j < 8; j++) v[j] = x.v[j];
+}
+
+template <typename Tin, bool kDefaultWindows>
 __global__ void __launch_bounds__(256) seg_curv_kernel(const Tin *V, const float *hidden,
                                                        SegArgs a, const float *inv_norm,
-                                                       int PT, double *klw) {
+                                                       double *klw) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
-    const int li = blockIdx.y;
-    const int l = a.layers[li];
-    const int i0 = blockIdx.x * PT;
-    const int rows = PT + 2 * kHalo;
-    const int row0 = i0 - kHalo;
-    float *inv_s = reinterpret_cast<float *>(smem_raw);                       // [rows]
-    float *red = inv_s + rows;                                                // [PT][8][12]
-    Tin *hraw = reinterpret_cast<Tin *>(red + (size_t)PT * 8 * 12);           // [rows][D]
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    for (int r = tid; r < rows; r += 256) {
-        int t = row0 + r;
+    float *P = reinterpret_cast<float *>(smem_raw);   // [kCurvCC][kCurvRS] normalised values
+    float *inv_s = P + (size_t)kCurvCC * kCurvRS;     // [kCurvRows]
+    const int li = blockIdx.y, l = a.layers[li];
+    const int i0 = blockIdx.x * kCurvPT, row0 = i0 - kHalo;
+    const int tid = threadIdx.x;
+    for (int r = tid; r < kCurvRows; r += 256) {
+        const int t = row0 + r;
         inv_s[r] = (t >= 0 && t < a.T) ? inv_norm[(size_t)li * a.T + t] : 0.f;
     }
-    for (size_t e = tid; e < (size_t)rows * a.D; e += 256) {
-        int r = (int)(e / a.D), c = (int)(e - (size_t)r * a.D);
-        int t = row0 + r;
-        float x = (t >= 0 && t < a.T) ? traj_elem(V, hidden, a.Dh, a.G, a.T, a.d, l, li, t, c) : 0.f;
-        hraw[e] = (Tin)x;
-    }
-    __syncthreads();
-    auto H = [&](int r, int c) -> float { return to_f(hraw[(size_t)r * a.D + c]) * inv_s[r]; };
-
     const int nw = a.nwin;
-    const int npos = min(PT, a.T - i0);
-    constexpr int kMaxCh = 8;                      // D <= 2048
-    float SL[kMaxCh][kMaxWindows], SR[kMaxCh][kMaxWindows];
-    const int nch = (a.D - tid + 255) / 256;
+    int wv[kMaxWindows];
+    float inv_w[kMaxWindows];
 #pragma unroll
-    for (int k = 0; k < kMaxCh; k++) {
-        if (k >= nch) break;
-        int c = tid + 256 * k;
-#pragma unroll
-        for (int wi = 0; wi < kMaxWindows; wi++) {
-            float sl = 0.f, sr = 0.f;
-            if (wi < nw) {
-                int w = a.windows[wi];
-                for (int tau = 0; tau < w; tau++) sl += H(kHalo - tau, c);
-                for (int tau = 1; tau <= w; tau++) sr += H(kHalo + tau, c);
-            }
-            SL[k][wi] = sl;
-            SR[k][wi] = sr;
-        }
+    for (int wi = 0; wi < kMaxWindows; wi++) {
+        wv[wi] = kDefaultWindows ? (4 << wi) : a.windows[wi];
+        inv_w[wi] = 1.0f / (float)wv[wi];
     }
-    for (int p = 0; p < npos; p++) {
-        const int rr = kHalo + p;       // row of position i0 + p
-        float acc[kMaxWindows][3];
+    float acc[kMaxWindows][3];
 #pragma unroll
-        for (int wi = 0; wi < kMaxWindows; wi++) acc[wi][0] = acc[wi][1] = acc[wi][2] = 0.f;
+    for (int wi = 0; wi < kMaxWindows; wi++) acc[wi][0] = acc[wi][1] = acc[wi][2] = 0.f;
+    const int R = tid + kHalo;   // staged row of this thread's position
+    for (int c0 = 0; c0 < a.D; c0 += kCurvCC) {
+        const int nq = min(kCurvCC, a.D - c0) >> 3;   // 8-channel chunks in this stage
+        __syncthreads();
+        for (int e = tid; e < kCurvRows * nq; e += 256) {
+            const int r = e / nq, q = e - r * nq;
+            float v[8];
+            traj_load8(V, hidden, a, l, li, row0 + r, c0 + 8 * q, v);
+            const float sc = inv_s[r];
 #pragma unroll
-        for (int k = 0; k < kMaxCh; k++) {
-            if (k >= nch) break;
-            int c = tid + 256 * k;
-            float hi = H(rr, c);
+            for (int j = 0; j < 8; j++) P[(size_t)(8 * q + j) * kCurvRS + r] = v[j] * sc;
+        }
+        __syncthreads();
+        for (int c = 0; c < 8 * nq; c++) {
+            const float *row = P + (size_t)c * kCurvRS + R;
+            const float h = row[0];
+            float sl = h, sr = 0.f;
+            float SL[kMaxWindows], SR[kMaxWindows];
+#pragma unroll
+            for (int wi = 0; wi < kMaxWindows; wi++) SL[wi] = SR[wi] = 0.f;
+#pragma unroll
+            for (int tau = 1; tau <= kHalo; tau++) {
+                // left sum over tau' < tau, right sum over 1 .. tau
+                if (kDefaultWindows) {
+                    if (tau == 4) SL[0] = sl;
+                    if (tau == 8) SL[1] = sl;
+                    if (tau == 16) SL[2] = sl;
+                } else {
+#pragma unroll
+                    for (int wi = 0; wi < kMaxWindows; wi++) SL[wi] = wv[wi] == tau ? sl : SL[wi];
+                }
+                if (tau < kHalo) sl += row[-tau];
+                sr += row[tau];
+                if (kDefaultWindows) {
+                    if (tau == 4) SR[0] = sr;
+                    if (tau == 8) SR[1] = sr;
+                    if (tau == 16) SR[2] = sr;
+                } else {
+#pragma unroll
+                    for (int wi = 0; wi < kMaxWindows; wi++) SR[wi] = wv[wi] == tau ? sr : SR[wi];
+                }
+            }
 #pragma unroll
             for (int wi = 0; wi < kMaxWindows; wi++) {
                 if (wi >= nw) break;
-                int w = a.windows[wi];
-                if (p > 0) {   // slide from position p-1 to p
-                    SL[k][wi] += hi - H(rr - w, c);
-                    SR[k][wi] += H(rr + w, c) - hi;
-                }
-                float inv_w = 1.0f / (float)w;
-                float dm = hi - SL[k][wi] * inv_w;
-                float dp = SR[k][wi] * inv_w - hi;
+                const float dm = h - SL[wi] * inv_w[wi];   // h_i - mean of the left window
+                const float dp = SR[wi] * inv_w[wi] - h;   // mean of the right window - h_i
                 acc[wi][0] = fmaf(dm, dm, acc[wi][0]);
                 acc[wi][1] = fmaf(dp, dp, acc[wi][1]);
                 acc[wi][2] = fmaf(dm, dp, acc[wi][2]);
             }
         }
-#pragma unroll
-        for (int wi = 0; wi < kMaxWindows; wi++) {
-            if (wi >= nw) break;
-#pragma unroll
-            for (int q = 0; q < 3; q++) {
-                float v = warp_sum(acc[wi][q]);
-                if (lane == 0) red[((size_t)p * 8 + warp) * 12 + wi * 3 + q] = v;
-            }
-        }
     }
-    __syncthreads();
-    for (int e = tid; e < npos * nw; e += 256) {
-        int p = e / nw, wi = e - p * nw;
-        int i = i0 + p, w = a.windows[wi];
-        double nm = 0, np_ = 0, dt = 0;
-        for (int q = 0; q < 8; q++) {
-            const float *rp = red + ((size_t)p * 8 + q) * 12 + wi * 3;
-            nm += rp[0];
-            np_ += rp[1];
-            dt += rp[2];
-        }
+    const int i = i0 + tid;
+    if (i >= a.T) return;
+#pragma unroll
+    for (int wi = 0; wi < kMaxWindows; wi++) {
+        if (wi >= nw) break;
+        const int w = wv[wi];
         double k = 0.0;
         if (i >= w && i < a.T - w) {
-            double x = sqrt(nm), y = sqrt(np_);
-            k = 1.0 - dt / ((x > kEps ? x : kEps) * (y > kEps ? y : kEps));
+            const double x = sqrt((double)acc[wi][0]), y = sqrt((double)acc[wi][1]);
+            k = 1.0 - (double)acc[wi][2] / ((x > kEps ? x : kEps) * (y > kEps ? y : kEps));
         }
         klw[((size_t)li * nw + wi) * a.T + i] = k;
     }
@@ -317,15 +336,18 @@ __global__ void seg_dd_kernel(const Tin *V, const float *hidden, SegArgs a, cons
         int p0 = a.cs + t, p1 = p0 + 1;
         float i0 = inv_norm[(size_t)li * a.T + p0], i1 = inv_norm[(size_t)li * a.T + p1];
         float f = 0.f;
-        for (int c = lane; c < a.D; c += 32) {
-            float x0 = traj_elem(V, hidden, a.Dh, a.G, a.T, a.d, l, li, p0, c) * i0;
-            float x1 = traj_elem(V, hidden, a.Dh, a.G, a.T, a.d, l, li, p1, c) * i1;
-            float df = x1 - x0;
-            f = fmaf(df, df, f);
+        for (int c = lane * 8; c < a.D; c += 256) {
+            float x0[8], x1[8];
+            traj_load8(V, hidden, a, l, li, p0, c, x0);
+            traj_load8(V, hidden, a, l, li, p1, c, x1);
+#pragma unroll
+            for (int j = 0; j < 8; j++) {
+                const float df = x1[j] * i1 - x0[j] * i0;
+                f = fmaf(df, df, f);
+            }
         }
-        s += (double)f;
+        s += (double)warp_sum(f);
     }
-    s = warp_sum(s);
     if (lane == 0) dd[t] = s;
 }
 
@@ -468,6 +490,155 @@ __global__ void __launch_bounds__(256) seg_band_kernel(const Tin *V, const float
     }
 }
 
+// Tensor-core version for bf16 V trajectories.  Block = 64 endpoints (rows
+// e' = E0 .. E0 + 63) x their predecessor band (columns a = a0 .. a0 + ncol - 1,
+// ncol = 64 + nb - 1).  The raw bf16 rows are staged 64 channels at a time
+// with cp.async (double buffered, row stride 72 halves: conflict-free fragment
+// reads) and multiplied with mma.sync m16n8k16 (exact bf16 products, fp32
+// sums); after each segmentation layer the Gram entries are folded into
+// |hbar_e - hbar_a|^2 = |hbar_e|^2 + |hbar_a|^2 - 2 inv_e inv_a (h_e . h_a).
+// Warp w owns row tile w % 4 and every other column tile of that row tile's
+// band (the column tiles [2 mt, (16 mt + 15 + nb - 1) / 8]).
+// ---------------------------------------------------------------------------
+constexpr int kBM = 64;               // endpoints per block
+constexpr int kBK = 64;               // channels per stage
+constexpr int kBStride = kBK + 8;     // staged row stride (halves)
+constexpr int kBNtW = 9;              // column tiles per warp: ceil(18 / 2) for nb <= 128
+
+__host__ __device__ constexpr int band_ncol_tiles(int nb) { return (kBM + nb - 1 + 7) / 8; }
+__host__ __device__ constexpr size_t band_mma_smem(int nb) {
+    return (size_t)2 * (kBM + 8 * band_ncol_tiles(nb)) * kBStride * sizeof(__nv_bfloat16) +
+           (size_t)2 * (kBM + 8 * band_ncol_tiles(nb)) * sizeof(float);
+}
+
+__global__ void __launch_bounds__(256) seg_band_mma_kernel(const __nv_bfloat16 *V, BandArgs b,
+                                                           const float *inv_norm, const float *nrm2,
+                                                           const double *p2, const double *bscore,
+                                                           float2 *ew) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const SegArgs &a = b.s;
+    const int nb = b.n_max - b.n_min + 1;
+    const int nct = band_ncol_tiles(nb);
+    const int nrs = kBM + 8 * nct;                      // staged rows: A rows, then B rows
+    __nv_bfloat16 *stg = reinterpret_cast<__nv_bfloat16 *>(smem_raw);   // [2][nrs][kBStride]
+    float *inv_r = reinterpret_cast<float *>(stg + (size_t)2 * nrs * kBStride);   // [nrs]
+    float *nrm_r = inv_r + nrs;                                                    // [nrs]
+    const int E0 = blockIdx.x * kBM;
+    const int a0 = E0 + 1 - b.n_max;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int gr = lane >> 2, c2 = 2 * (lane & 3);
+    const int mt = warp & 3, hw = warp >> 2;
+    const int nt_lo = 2 * mt, nt_hi = min(nct - 1, (16 * mt + 15 + nb - 1) / 8);
+    // relative position (index into the compressible region) of staged row r
+    auto rel = [&](int r) { return r < kBM ? E0 + r : a0 + (r - kBM); };
+    auto valid = [&](int x) { return x >= 0 && x < a.N; };
+
+    float acc[kBNtW][4], sd[kBNtW][4];
+#pragma unroll
+    for (int q = 0; q < kBNtW; q++)
+#pragma unroll
+        for (int h = 0; h < 4; h++) acc[q][h] = sd[q][h] = 0.f;
+
+    const int nchunk = a.D / kBK;
+    const int nstage = a.nseg * nchunk;
+    auto stage = [&](int st) {
+        const int li = st / nchunk, c0 = (st - li * nchunk) * kBK;
+        const int l = a.layers[li], g = c0 / a.d, i = c0 - g * a.d;
+        __nv_bfloat16 *dst = stg + (size_t)(st & 1) * nrs * kBStride;
+        for (int e = tid; e < nrs * (kBK / 8); e += 256) {
+            const int r = e >> 3, q = e & 7;
+            const int x = rel(r);
+            const bool ok = valid(x);
+            const __nv_bfloat16 *src = V + (((size_t)l * a.G + g) * a.T + a.cs + (ok ? x : 0)) * a.d + i + 8 * q;
+            cp_async16(dst + (size_t)r * kBStride + 8 * q, src, ok);
+        }
+        cp_async_commit();
+    };
+    stage(0);
+    for (int st = 0; st < nstage; st++) {
+        const int li = st / nchunk, ch = st - li * nchunk;
+        if (ch == 0) {   // this layer's norms of the staged rows
+            for (int r = tid; r < nrs; r += 256) {
+                const int x = rel(r);
+                const bool ok = valid(x);
+                inv_r[r] = ok ? inv_norm[(size_t)li * a.T + a.cs + x] : 0.f;
+                nrm_r[r] = ok ? nrm2[(size_t)li * a.T + a.cs + x] : 0.f;
+            }
+        }
+        if (st + 1 < nstage) {
+            stage(st + 1);
+            cp_async_wait<1>();
+        } else {
+            cp_async_wait<0>();
+        }
+        __syncthreads();
+        const __nv_bfloat16 *As = stg + (size_t)(st & 1) * nrs * kBStride;
+        const __nv_bfloat16 *Bs = As + (size_t)kBM * kBStride;
+#pragma unroll
+        for (int ks = 0; ks < kBK / 16; ks++) {
+            uint32_t af[4];
+            const __nv_bfloat16 *ar = As + (size_t)(16 * mt + gr) * kBStride + ks * 16 + c2;
+            af[0] = *reinterpret_cast<const uint32_t *>(ar);
+            af[1] = *reinterpret_cast<const uint32_t *>(ar + 8 * kBStride);
+            af[2] = *reinterpret_cast<const uint32_t *>(ar + 8);
+            af[3] = *reinterpret_cast<const uint32_t *>(ar + 8 * kBStride + 8);
+#pragma unroll
+            for (int q = 0; q < kBNtW; q++) {
+                const int nt = nt_lo + 2 * q + hw;
+                if (nt > nt_hi) break;
+                const __nv_bfloat16 *br = Bs + (size_t)(nt * 8 + gr) * kBStride + ks * 16 + c2;
+                mma_bf16(acc[q], af, *reinterpret_cast<const uint32_t *>(br),
+                         *reinterpret_cast<const uint32_t *>(br + 8));
+            }
+        }
+        if (ch == nchunk - 1) {   // fold this layer: sd += |hbar_e|^2 + |hbar_a|^2 - 2 hbar_e . hbar_a
+#pragma unroll
+            for (int q = 0; q < kBNtW; q++) {
+                const int nt = nt_lo + 2 * q + hw;
+                if (nt > nt_hi) break;
+#pragma unroll
+                for (int h = 0; h < 4; h++) {
+                    const int row = 16 * mt + gr + (h >= 2 ? 8 : 0);
+                    const int col = nt * 8 + c2 + (h & 1);
+                    const float ie = inv_r[row], ne = nrm_r[row];
+                    const float ia = inv_r[kBM + col], na = nrm_r[kBM + col];
+                    sd[q][h] += ne + na - 2.f * (ie * ia * acc[q][h]);
+                    acc[q][h] = 0.f;
+                }
+            }
+        }
+        __syncthreads();   // buffer st & 1 and the norms are reused
+    }
+    // edge weights for endpoint i = ep + 1 and len = i - ap
+#pragma unroll
+    for (int q = 0; q < kBNtW; q++) {
+        const int nt = nt_lo + 2 * q + hw;
+        if (nt > nt_hi) break;
+#pragma unroll
+        for (int h = 0; h < 4; h++) {
+            const int row = 16 * mt + gr + (h >= 2 ? 8 : 0);
+            const int col = nt * 8 + c2 + (h & 1);
+            const int ep = E0 + row, ap = a0 + col;
+            if (ep >= a.N) continue;
+            const int i = ep + 1, len = i - ap;
+            if (len < b.n_min || len > b.n_max) continue;
+            if (ap < 0) {
+                ew[(size_t)i * nb + (len - b.n_min)] = make_float2(-INFINITY, 0.f);
+                continue;
+            }
+            const int nS = len - 1;
+            double disp = 0.0;
+            if (nS >= 2) {
+                const double s2 = p2[ep] - p2[ap];     // sum_{t=ap}^{ep-1} ||d_t||^2
+                disp = (s2 - (double)sd[q][h] / nS) / (double)(nS - 1) / a.nseg;
+            }
+            const double gam = ap == 0 ? 0.0 : bscore[a.cs + ap - 1] - b.c_cut;
+            const double pen = (double)(len - b.n0) / b.n0;
+            ew[(size_t)i * nb + (len - b.n_min)] = df_split(gam - b.lambda_d * disp - b.lambda_n * pen * pen);
+        }
+    }
+}
+
 // Terminal relaxation weights at i = N: len in [1, n_max]; warp per len.
 template <typename Tin>
 __global__ void seg_band_terminal_kernel(const Tin *V, const float *hidden, BandArgs b,
@@ -503,31 +674,32 @@ __global__ void seg_band_terminal_kernel(const Tin *V, const float *hidden, Band
 }
 
 // ---------------------------------------------------------------------------
-// DP: one block of 1024 threads.  Endpoints are processed 16 (or n_min, if
-// smaller) at a time: F[i..i+nb-1] only read F[< i] because i - a >= n_min.
-// 64 threads per endpoint reduce its candidates (value desc, a asc).  The
-// chosen slot length of every endpoint is kept in shared memory (uint8) so
-// the backtracking runs without global round trips.
+// DP: one block, one warp per endpoint.  Endpoints are processed 16 (or n_min,
+// if smaller) at a time: F[i..i+15] only read F[< i] because i - a >= n_min,
+// so one barrier per step suffices.  Lane handles the lengths n_min + lane +
+// 32 j; the warp reduces its candidates (value desc, a asc) with shuffles.
+// The edge weights of the next kDpPD steps are prefetched into registers
+// (they do not depend on F).  The chosen slot length of every endpoint is
+// kept in shared memory (uint8) so the backtracking runs without global
+// round trips.
 // ---------------------------------------------------------------------------
 constexpr int kDpRing = 256;
-constexpr int kDpEp = 16;
-constexpr int kDpTpe = 64;
+constexpr int kDpEp = 16;    // endpoints per step (warps)
+constexpr int kDpPD = 6;     // steps of edge weights in flight
+constexpr int kDpLen = 4;    // lengths per lane: n_max - n_min + 1 <= 128
 
 __device__ __forceinline__ bool better(df2 v, int a, df2 bv, int ba) {
     return df_gt(v, bv) || (df_eq(v, bv) && a < ba);
 }
 
-__global__ void __launch_bounds__(1024) seg_dp_kernel(const float2 *ew, const float2 *ewt, int N,
-                                                      int n_min, int n_max, int cs, double *Fout,
-                                                      int32_t *slots, int *dev_int) {
+__global__ void __launch_bounds__(kDpEp * 32) seg_dp_kernel(const float2 *ew, const float2 *ewt, int N,
+                                                            int n_min, int n_max, int cs, double *Fout,
+                                                            int32_t *slots, int *dev_int) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     df2 *ring = reinterpret_cast<df2 *>(smem_raw);                       // [kDpRing]
-    df2 *rv = ring + kDpRing;                                            // [32] per-warp best value
-    int *ra = reinterpret_cast<int *>(rv + 32);                          // [32] per-warp best a
-    uint8_t *lenarr = reinterpret_cast<uint8_t *>(ra + 32);              // [N + 1]
+    uint8_t *lenarr = reinterpret_cast<uint8_t *>(ring + kDpRing);       // [N + 1]
     const int nb = n_max - n_min + 1;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int k = tid / kDpTpe, sub = tid % kDpTpe;
+    const int tid = threadIdx.x, lane = tid & 31, k = tid >> 5;
     const int step = min(n_min, kDpEp);
     const df2 NEG = df2{-INFINITY, 0.f};
     if (tid == 0) {
@@ -535,38 +707,49 @@ __global__ void __launch_bounds__(1024) seg_dp_kernel(const float2 *ew, const fl
         Fout[0] = 0.0;
         lenarr[0] = 0;
     }
+    float2 wb[kDpPD][kDpLen];
+    auto load_w = [&](int i, float2 out[kDpLen]) {
+#pragma unroll
+        for (int j = 0; j < kDpLen; j++) {
+            const int len = n_min + lane + 32 * j;
+            out[j] = (k < step && i <= N && len <= n_max) ? ew[(size_t)i * nb + (len - n_min)]
+                                                          : make_float2(-INFINITY, 0.f);
+        }
+    };
+#pragma unroll
+    for (int q = 0; q < kDpPD; q++) load_w(1 + q * step + k, wb[q]);
     __syncthreads();
     for (int i0 = 1; i0 <= N; i0 += step) {
-        int i = i0 + k;
-        bool act = k < step && i <= N;
+        const int i = i0 + k;
+        const bool act = k < step && i <= N;
         df2 best = NEG;
         int ba = 0x7fffffff;
         if (act) {
-            for (int len = n_min + sub; len <= n_max; len += kDpTpe) {
-                int a = i - len;
-                if (a < 0) break;
-                df2 fa = ring[a % kDpRing];
+#pragma unroll
+            for (int j = 0; j < kDpLen; j++) {
+                const int len = n_min + lane + 32 * j;
+                const int a = i - len;
+                if (len > n_max || a < 0) break;
+                const df2 fa = ring[a % kDpRing];
                 if (fa.hi == -INFINITY) continue;
-                float2 w = ew[(size_t)i * nb + (len - n_min)];
-                df2 v = df_add(fa, w);
+                const df2 v = df_add(fa, wb[0][j]);
                 if (better(v, a, best, ba)) { best = v; ba = a; }
             }
         }
-        // reduce over the 64 threads of the endpoint (2 warps)
+#pragma unroll
+        for (int q = 0; q + 1 < kDpPD; q++)
+#pragma unroll
+            for (int j = 0; j < kDpLen; j++) wb[q][j] = wb[q + 1][j];
+        load_w(i0 + kDpPD * step + k, wb[kDpPD - 1]);
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
             df2 ov;
             ov.hi = __shfl_xor_sync(0xffffffffu, best.hi, o);
             ov.lo = __shfl_xor_sync(0xffffffffu, best.lo, o);
-            int oa = __shfl_xor_sync(0xffffffffu, ba, o);
+            const int oa = __shfl_xor_sync(0xffffffffu, ba, o);
             if (better(ov, oa, best, ba)) { best = ov; ba = oa; }
         }
-        if (lane == 0) { rv[warp] = best; ra[warp] = ba; }
-        __syncthreads();
-        if (sub == 0 && act) {
-            df2 v2 = rv[warp + 1];
-            int a2 = ra[warp + 1];
-            if (better(v2, a2, best, ba)) { best = v2; ba = a2; }
+        if (lane == 0 && act) {
             ring[i % kDpRing] = best;
             Fout[i] = (double)best.hi + (double)best.lo;
             lenarr[i] = best.hi == -INFINITY ? 0 : (uint8_t)(i - ba);
@@ -634,25 +817,29 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
     if (bf) seg_norm_kernel<<<gn, 256, 0, s>>>(Vb, hidden, a, w.inv_norm, w.nrm2);
     else seg_norm_kernel<<<gn, 256, 0, s>>>(Vf, hidden, a, w.inv_norm, w.nrm2);
 
-    // curvature tile: staged raw rows (input element type, fp32 for hidden
-    // states) + inverse norms + per-warp reductions
-    const bool stage_bf = bf && !hidden;
-    const size_t esz = stage_bf ? 2 : 4;
-    const size_t budget = 224 * 1024;
-    int PT = 64;
-    auto cur_smem = [&](int pt) {
-        return (size_t)(pt + 2 * kHalo) * 4 + (size_t)pt * 8 * 12 * 4 + (size_t)(pt + 2 * kHalo) * a.D * esz;
-    };
-    while (PT > 8 && cur_smem(PT) > budget) PT /= 2;
-    if (cur_smem(PT) > budget) return cudaErrorInvalidConfiguration;
-    size_t sm = cur_smem(PT);
-    dim3 gc((p.T + PT - 1) / PT, c.nseg);
-    if (stage_bf) {
-        cudaFuncSetAttribute(seg_curv_kernel<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-        seg_curv_kernel<<<gc, 256, sm, s>>>(Vb, hidden, a, w.inv_norm, PT, w.klw);
-    } else {
-        cudaFuncSetAttribute(seg_curv_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-        seg_curv_kernel<<<gc, 256, sm, s>>>(bf ? nullptr : Vf, hidden, a, w.inv_norm, PT, w.klw);
+    // curvature: one thread per position, staged normalised channels
+    {
+        const bool defw = c.nwin == 3 && p.windows[0] == 4 && p.windows[1] == 8 && p.windows[2] == 16;
+        dim3 gc((p.T + kCurvPT - 1) / kCurvPT, c.nseg);
+        const int sm = (int)kCurvSmem;
+        if (bf && !hidden) {
+            if (defw) {
+                cudaFuncSetAttribute(seg_curv_kernel<__nv_bfloat16, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+                seg_curv_kernel<__nv_bfloat16, true><<<gc, 256, sm, s>>>(Vb, hidden, a, w.inv_norm, w.klw);
+            } else {
+                cudaFuncSetAttribute(seg_curv_kernel<__nv_bfloat16, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+                seg_curv_kernel<__nv_bfloat16, false><<<gc, 256, sm, s>>>(Vb, hidden, a, w.inv_norm, w.klw);
+            }
+        } else {
+            const float *Vx = bf ? nullptr : Vf;
+            if (defw) {
+                cudaFuncSetAttribute(seg_curv_kernel<float, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+                seg_curv_kernel<float, true><<<gc, 256, sm, s>>>(Vx, hidden, a, w.inv_norm, w.klw);
+            } else {
+                cudaFuncSetAttribute(seg_curv_kernel<float, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+                seg_curv_kernel<float, false><<<gc, 256, sm, s>>>(Vx, hidden, a, w.inv_norm, w.klw);
+            }
+        }
     }
     seg_combine_kernel<<<(p.T + 255) / 256, 256, 0, s>>>(w.klw, c.nseg * c.nwin, p.T, p.lambda_stab,
                                                           w.kappa, kappa_out, w.dev_int + 1);
@@ -680,18 +867,24 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
     if (ncol > 8 * 24) return cudaErrorInvalidConfiguration;
     size_t smb = (size_t)(kRB + ncol) * kKC * 4;
     int gb = (N + kRB - 1) / kRB;
-    if (bf) {
+    if (bf && !hidden && a.D % kBK == 0 && a.d % kBK == 0 && nb <= 128) {
+        const int gm = (N + kBM - 1) / kBM;
+        const int smm = (int)band_mma_smem(nb);
+        cudaFuncSetAttribute(seg_band_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smm);
+        seg_band_mma_kernel<<<gm, 256, smm, s>>>(Vb, b, w.inv_norm, w.nrm2, w.p2, w.bscore, w.ew);
+        seg_band_terminal_kernel<<<(p.n_max + 7) / 8, 256, 0, s>>>(Vb, hidden, b, w.inv_norm, w.nrm2, w.p2, w.bscore, w.ewt);
+    } else if (bf) {
         seg_band_kernel<<<gb, 256, smb, s>>>(Vb, hidden, b, w.inv_norm, w.nrm2, w.p2, w.bscore, w.ew);
         seg_band_terminal_kernel<<<(p.n_max + 7) / 8, 256, 0, s>>>(Vb, hidden, b, w.inv_norm, w.nrm2, w.p2, w.bscore, w.ewt);
     } else {
         seg_band_kernel<<<gb, 256, smb, s>>>(Vf, hidden, b, w.inv_norm, w.nrm2, w.p2, w.bscore, w.ew);
         seg_band_terminal_kernel<<<(p.n_max + 7) / 8, 256, 0, s>>>(Vf, hidden, b, w.inv_norm, w.nrm2, w.p2, w.bscore, w.ewt);
     }
-    size_t smd = kDpRing * sizeof(df2) + 32 * sizeof(df2) + 32 * 4 + (size_t)(N + 1);
+    size_t smd = kDpRing * sizeof(df2) + (size_t)(N + 1);
     smd = (smd + 15) & ~(size_t)15;
-    if (smd > 227 * 1024) return cudaErrorInvalidConfiguration;
+    if (smd > 227 * 1024 || nb > 32 * kDpLen) return cudaErrorInvalidConfiguration;
     cudaFuncSetAttribute(seg_dp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smd);
-    seg_dp_kernel<<<1, 1024, smd, s>>>(w.ew, w.ewt, N, p.n_min, p.n_max, p.ctx_start, w.dpF,
+    seg_dp_kernel<<<1, kDpEp * 32, smd, s>>>(w.ew, w.ewt, N, p.n_min, p.n_max, p.ctx_start, w.dpF,
                                        w.slots, w.dev_int);
     c.launches += 8 + (surprisal ? 2 : 0) + (N > 1 ? 1 : 0);
     return cudaGetLastError();

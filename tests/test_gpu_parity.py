@@ -128,6 +128,13 @@ def test_errors_are_reported_not_trapped():
         ctx.gracekv_allocate()
     assert e.value.status == gk.GKV_ESTATE
     slots = torch.empty(T, dtype=torch.int32, device="cuda")
+    # a view starting one element past a 16-byte boundary is rejected on the host
+    buf = torch.empty(V.numel() + 8, dtype=V.dtype, device="cuda")
+    Vm = buf[1:1 + V.numel()].view(V.shape)
+    Vm.copy_(V)
+    with pytest.raises(gk.GraceKVError) as e:
+        ctx.gracekv_segment(Vm, slots)
+    assert e.value.status == gk.GKV_EINVAL
     ctx.gracekv_segment(V, slots)
     bad = torch.tensor([0, 200, T - 32], dtype=torch.int32, device="cuda")   # slot of 200 tokens
     with pytest.raises(gk.GraceKVError) as e:
