@@ -167,6 +167,23 @@ def segment(p: Params, V, hidden=None, surprisal=None):
                 dp_second=second)
 
 
+def dp_weights(p: Params, V, b, a_rel, i_rel, hidden=None):
+    """Edge weights w(a, i) of the segmentation DP for the given position pairs."""
+    V = _f64(V)
+    hid = _f64(hidden)
+    bb = _f64(b)
+    Dh = 0 if hid is None else hid.shape[-1]
+    a_ = np.ascontiguousarray(np.asarray(a_rel, dtype=np.int32))
+    i_ = np.ascontiguousarray(np.asarray(i_rel, dtype=np.int32))
+    w = np.zeros(len(a_))
+    rc = lib().orc_dp_weights(C.byref(p), _p(V, C.c_double),
+                              None if hid is None else _p(hid, C.c_double), C.c_int32(Dh),
+                              _p(bb, C.c_double), C.c_int32(len(a_)), _p(a_, C.c_int32),
+                              _p(i_, C.c_int32), _p(w, C.c_double))
+    assert rc == 0, rc
+    return w
+
+
 def row_stats(p: Params, Q, K):
     Q, K = _f64(Q), _f64(K)
     n = p.L * p.Hq * p.W

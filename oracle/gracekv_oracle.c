@@ -357,6 +357,58 @@ int orc_segment(const orc_params *p, const double *V, const double *hidden, int3
 }
 
 /* ------------------------------------------------------------------------ */
+/* DP edge weights w(a, i) = Gamma(a) - lambda_d Disp([a, i)) - lambda_n      */
+/* ((i - a - n0) / n0)^2 of Eq. (app_dp_recurrence), for given pairs of       */
+/* region-relative positions 0 <= a < i <= N, with the boundary score b given */
+/* (b[cs + a - 1] enters Gamma(a), a > 0).  Same Disp as orc_segment.  Used   */
+/* to check the optimality of a partition locally at sizes where the full DP  */
+/* is too slow.                                                               */
+/* ------------------------------------------------------------------------ */
+int orc_dp_weights(const orc_params *p, const double *V, const double *hidden, int32_t Dh,
+                   const double *b, int32_t n, const int32_t *a_rel, const int32_t *i_rel,
+                   double *w_out)
+{
+    int T = p->T;
+    int cs = p->ctx_start;
+    int N = p->ctx_end - p->recent - cs;
+    if (N < 1) return ORC_EINVAL;
+    for (int k = 0; k < n; k++)
+        if (a_rel[k] < 0 || i_rel[k] <= a_rel[k] || i_rel[k] > N) return ORC_EINVAL;
+    int32_t layers[8];
+    int nl = seg_layers(p, layers);
+    int D = hidden ? Dh : p->G * p->d;
+    disp_ctx c;
+    c.nl = nl; c.D = D; c.cs = cs; c.N = N; c.T = T; c.mode = p->disp_mode;
+    c.hb = (double *)malloc(sizeof(double) * (size_t)nl * T * D);
+    c.pref2 = (double *)calloc((size_t)nl * N, sizeof(double));
+    c.tmp = (double *)malloc(sizeof(double) * D);
+    if (!c.hb || !c.pref2 || !c.tmp) {
+        free(c.hb); free(c.pref2); free(c.tmp);
+        return ORC_ENOMEM;
+    }
+    for (int li = 0; li < nl; li++) {
+        double *hb = c.hb + (size_t)li * T * D;
+        trajectory(p, V, hidden, Dh, li, layers[li], hb, D);
+        double *pr = c.pref2 + (size_t)li * N;
+        pr[0] = 0.0;
+        for (int t = 1; t < N; t++) {
+            double s = 0.0;
+            for (int k = 0; k < D; k++)
+                s += sqr(hb[(size_t)(cs + t) * D + k] - hb[(size_t)(cs + t - 1) * D + k]);
+            pr[t] = pr[t - 1] + s;
+        }
+    }
+    for (int k = 0; k < n; k++) {
+        int a = a_rel[k], i = i_rel[k];
+        double gamma = a == 0 ? 0.0 : b[cs + a - 1] - p->c_cut;
+        w_out[k] = gamma - p->lambda_d * disp(&c, a, i)
+                   - p->lambda_n * sqr((double)(i - a - p->n0) / p->n0);
+    }
+    free(c.hb); free(c.pref2); free(c.tmp);
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------------------ */
 /* Row statistics.  For every probe row (l, h, u) and key t in the visible    */
 /* range [0, T) (reading R2): x = q . k_t / sqrt(d); m = max_t x (the          */
 /* max-logit shift of App. A.3 "Prototype distortion"); Z = sum exp(x - m)    */

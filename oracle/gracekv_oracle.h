@@ -94,6 +94,10 @@ int orc_segment(const orc_params *p, const double *V, const double *hidden, int3
                 int32_t *slot_starts, int32_t cap, int32_t *n_slots,
                 double *dp_best, double *dp_second);
 
+int orc_dp_weights(const orc_params *p, const double *V, const double *hidden, int32_t Dh,
+                   const double *b, int32_t n, const int32_t *a_rel, const int32_t *i_rel,
+                   double *w_out);
+
 int orc_row_stats(const orc_params *p, const double *Q, const double *K,
                   double *m, double *Z, double *ZC);
 int orc_token_values(const orc_params *p, const double *Q, const double *K,

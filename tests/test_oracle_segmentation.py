@@ -211,6 +211,29 @@ def test_dp_matches_exhaustive_enumeration(oracle_lib, seed, N, n_min, n_max, n0
     assert list(seg["slot_starts"] - cs) == arg
 
 
+@pytest.mark.parametrize("disp_mode", [0, 1])
+def test_dp_weights_match_numpy_and_sum_to_dp_value(oracle_lib, disp_mode):
+    # w(a, i) = Gamma(a) - lambda_d Disp([a, i)) - lambda_n ((i-a-n0)/n0)^2, Eq. (app_dp_recurrence):
+    # each weight against numpy's sample variance of the differences, and the
+    # weights along the DP's own partition add up to its optimum F[N].
+    rng = np.random.default_rng(11)
+    cs, N, r = 3, 60, 4
+    T = cs + N + r + 2
+    V = rng.normal(size=(1, 2, T, 5))
+    p = O.make_params(1, 2, 2, T, 5, 1, 0.0, ctx_start=cs, ctx_end=T - 2, recent=r,
+                      n_min=4, n_max=12, n0=8, windows=(2, 3), disp_mode=disp_mode)
+    seg = O.segment(p, V)
+    b, hb = seg["b"], _traj(V)
+    pairs = [(a, i) for a in range(0, N - 1, 3) for i in range(a + 1, min(N, a + 14) + 1, 2)]
+    w = O.dp_weights(p, V, b, [x for x, _ in pairs], [y for _, y in pairs])
+    ref = [(b[cs + a - 1] - 1.0 if a > 0 else 0.0) - 0.25 * _disp_lib(hb, cs, a, i)
+           - 0.10 * ((i - a - 8) / 8) ** 2 for a, i in pairs]
+    np.testing.assert_allclose(w, ref, rtol=1e-10, atol=1e-10)
+    ss = seg["slot_starts"] - cs
+    w_path = O.dp_weights(p, V, b, ss[:-1], ss[1:])
+    np.testing.assert_allclose(w_path.sum(), seg["dp_best"][N], rtol=1e-12, atol=1e-12)
+
+
 def test_dp_dispersion_forms_agree(oracle_lib):
     # Eq. (app_layer_dispersion) vs the equivalent form Eq. (app_prefix_dispersion)
     rng = np.random.default_rng(9)
