@@ -29,7 +29,7 @@
  *   greedy allocation App. A.5 Stage II, App. C.3 (max-priority queue)
  *   packing           App. A.5 "Frontier updates and physical packing"
  *
- * Readings of silent or ambiguous passages (each also listed in the design doc):
+ * Readings of silent or ambiguous passages:
  *   R1  trajectory h^(l)_t = concat_g v^(l,g)_t unless hidden states are given;
  *       surprisal defaults to 0; omega defaults to 1; lambda_graph = 0.
  *   R2  visible range of every probe = [0, T); probes = the W observation
