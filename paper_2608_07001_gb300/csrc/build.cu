@@ -658,69 +658,83 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     if (r2 > rb || (r2 == rb && p2 < pb)) { rb = r2; pb = p2; }
                 }
                 if (pb < a || pb >= b) pb = a;   // only reachable with non-finite values
+                // Candidate lists, lane-parallel (ranks from ballots): cuts xi in
+                // ascending order; prefixes [a, xi) (xi - a >= 2) and the
+                // extraction's left side [a, p*) in ascending end, then the whole
+                // node (fresh roots); suffixes [xi, b) (b - xi >= 2) and the right
+                // side [p*+1, b) in descending start.  A side equal to a cut's
+                // interval shares its candidate.
+                const unsigned FULL = 0xffffffffu;
+                const bool cands = nv >= 3;
+                const int maxc = cands ? min(A.k_cand + 1, nv - 1) : 0;
+                int ncut = 0;
+#pragma unroll
+                for (int w = 0; w < NMAX / 32; w++) {
+                    const unsigned m = sel[w];
+                    const int q = ncut + __popc(m & ((1u << lane) - 1u));
+                    if (((m >> lane) & 1u) && q < maxc) B.cut[q] = (short)(a + w * 32 + lane + 1);
+                    ncut += __popc(m);
+                }
+                ncut = min(ncut, maxc);
+                __syncwarp();
+                const bool hq = lane < ncut;
+                const int xi = hq ? B.cut[lane] : 0;
+                const unsigned lt = (1u << lane) - 1u, gt = ~((2u << lane) - 1u);
+                // prefixes
+                const bool pv = hq && xi - a >= 2;
+                const unsigned pm = __ballot_sync(FULL, pv);
+                const unsigned pbm = __ballot_sync(FULL, hq && xi == pb);
+                const bool el_cand = cands && pb - a >= 2;
+                const bool el_sep = el_cand && pbm == 0u;
+                const int pidx = pv ? B.pre_b + __popc(pm & lt) + (el_sep && pb < xi ? 1 : 0) : -1;
+                const int eL_sep = B.pre_b + __popc(__ballot_sync(FULL, pv && xi < pb));
+                const int eL_cut = __shfl_sync(FULL, pidx, pbm ? __ffs(pbm) - 1 : 0);
+                if (hq) B.pidx[lane] = (short)pidx;
+                if (pv) sm.cand[pidx] = {a, xi, 0.f};
+                // suffixes
+                const int er = pb + 1;
+                const bool sv = hq && b - xi >= 2;
+                const unsigned smk = __ballot_sync(FULL, sv);
+                const unsigned erm = __ballot_sync(FULL, hq && xi == er);
+                const bool er_cand = cands && b - er >= 2;
+                const bool er_sep = er_cand && erm == 0u;
+                const int sidx = sv ? B.suf_b + __popc(smk & gt) + (er_sep && er > xi ? 1 : 0) : -1;
+                const int eR_sep = B.suf_b + __popc(__ballot_sync(FULL, sv && xi > er));
+                const int eR_cut = __shfl_sync(FULL, sidx, erm ? __ffs(erm) - 1 : 0);
+                if (hq) B.sidx[lane] = (short)sidx;
+                if (sv) sm.cand[sidx] = {xi, b, 0.f};
+                // work counters: tokens swept, candidates evaluated, their lengths
+                int len = (pv ? xi - a : 0) + (sv ? b - xi : 0);
+                int pe = pv ? xi : a, ss = sv ? xi : b;
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) {
+                    len += __shfl_xor_sync(FULL, len, o);
+                    pe = max(pe, __shfl_xor_sync(FULL, pe, o));
+                    ss = min(ss, __shfl_xor_sync(FULL, ss, o));
+                }
                 if (lane == 0) {
                     B.kmin = nv >= 2 ? okey_inv(kmin) : 0.0;
                     B.kmax = nv >= 2 ? okey_inv(kmax) : 0.0;
                     B.pstar = pb;
-                    B.ncut = 0;
-                    B.eL = B.eR = B.whole = -1;
-                    int k = B.pre_b;
-                    const bool cands = nv >= 3;
-                    if (cands) {
-                        for (int w = 0; w < NMAX / 32; w++) {
-                            unsigned m = sel[w];
-                            while (m) {
-                                int bit = __ffs(m) - 1;
-                                m &= m - 1;
-                                if (B.ncut < min(A.k_cand + 1, nv - 1))
-                                    B.cut[B.ncut++] = (short)(a + w * 32 + bit + 1);
-                            }
-                        }
-                        // prefixes in ascending end: cuts merged with the extraction's left side
-                        bool el_done = !(pb - a >= 2);
-                        for (int q = 0; q < B.ncut; q++) {
-                            int xi = B.cut[q];
-                            if (!el_done && pb <= xi) {
-                                if (pb == xi) { B.eL = -2 - q; }   // same interval as cut q
-                                else { sm.cand[k] = {a, pb, 0.f}; B.eL = k++; }
-                                el_done = true;
-                            }
-                            if (xi - a >= 2) { sm.cand[k] = {a, xi, 0.f}; B.pidx[q] = (short)k++; }
-                            else B.pidx[q] = -1;
-                        }
-                        if (!el_done) { sm.cand[k] = {a, pb, 0.f}; B.eL = k++; }
-                        if (B.eL <= -2) B.eL = B.pidx[-2 - B.eL];
-                    }
-                    if (v == 0 && !A.resume) { sm.cand[k] = {a, b, 0.f}; B.whole = k++; }
+                    B.ncut = ncut;
+                    B.eL = el_sep ? eL_sep : (el_cand ? eL_cut : -1);
+                    if (el_sep) sm.cand[eL_sep] = {a, pb, 0.f};
+                    int k = B.pre_b + __popc(pm) + (el_sep ? 1 : 0);
+                    const bool whole = v == 0 && !A.resume;
+                    B.whole = -1;
+                    if (whole) { sm.cand[k] = {a, b, 0.f}; B.whole = k++; }
                     B.pre_e = k;
-                    k = B.suf_b;
-                    if (cands) {
-                        // suffixes in descending start: cuts (descending) merged with p*+1
-                        int er = pb + 1;
-                        bool er_done = !(b - er >= 2);
-                        for (int q = B.ncut - 1; q >= 0; q--) {
-                            int xi = B.cut[q];
-                            if (!er_done && er >= xi) {
-                                if (er == xi) B.eR = -2 - q;
-                                else { sm.cand[k] = {er, b, 0.f}; B.eR = k++; }
-                                er_done = true;
-                            }
-                            if (b - xi >= 2) { sm.cand[k] = {xi, b, 0.f}; B.sidx[q] = (short)k++; }
-                            else B.sidx[q] = -1;
-                        }
-                        if (!er_done) { sm.cand[k] = {er, b, 0.f}; B.eR = k++; }
-                        if (B.eR <= -2) B.eR = B.sidx[-2 - B.eR];
-                    }
-                    B.suf_e = k;
+                    B.eR = er_sep ? eR_sep : (er_cand ? eR_cut : -1);
+                    if (er_sep) sm.cand[eR_sep] = {er, b, 0.f};
+                    B.suf_e = B.suf_b + __popc(smk) + (er_sep ? 1 : 0);
                     for (int q = B.pre_e; q < B.pre_r; q++) sm.cand[q].a = sm.cand[q].b = 0;
                     for (int q = B.suf_e; q < B.suf_r; q++) sm.cand[q].a = sm.cand[q].b = 0;
-                    // work counters: tokens swept, candidates evaluated, their lengths
-                    const int pe = B.pre_e > B.pre_b ? sm.cand[B.pre_e - 1].b : a;
-                    const int ss = B.suf_e > B.suf_b ? sm.cand[B.suf_e - 1].a : b;
+                    if (el_sep) { pe = max(pe, pb); len += pb - a; }
+                    if (er_sep) { ss = min(ss, er); len += b - er; }
+                    if (whole) { pe = b; len += b - a; }
                     w_scan += (pe - a) + (b - ss);
                     w_eval += (B.pre_e - B.pre_b) + (B.suf_e - B.suf_b);
-                    for (int q = B.pre_b; q < B.pre_e; q++) w_len += sm.cand[q].b - sm.cand[q].a;
-                    for (int q = B.suf_b; q < B.suf_e; q++) w_len += sm.cand[q].b - sm.cand[q].a;
+                    w_len += len;
                 }
             }
             __syncthreads();
