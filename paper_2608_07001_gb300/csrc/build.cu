@@ -138,6 +138,19 @@ __device__ __forceinline__ void ld8(const __nv_bfloat16 *p, float v[8]) {
     }
 }
 
+// 8 consecutive elements of a shared-memory row as 4 float pairs.
+__device__ __forceinline__ void ld8x2(const float *p, float2 v[4]) {
+    const float4 a = reinterpret_cast<const float4 *>(p)[0], b = reinterpret_cast<const float4 *>(p)[1];
+    v[0] = make_float2(a.x, a.y); v[1] = make_float2(a.z, a.w);
+    v[2] = make_float2(b.x, b.y); v[3] = make_float2(b.z, b.w);
+}
+__device__ __forceinline__ void ld8x2(const __nv_bfloat16 *p, float2 v[4]) {
+    const uint4 u = reinterpret_cast<const uint4 *>(p)[0];
+    const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&u);
+#pragma unroll
+    for (int i = 0; i < 4; i++) v[i] = __bfloat1622float2(h[i]);
+}
+
 // N consecutive elements of a shared-memory row as floats (N = 1 or 2).
 template <int N>
 __device__ __forceinline__ void ld_pairs(const float *p, float v[N]) {
@@ -240,7 +253,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     // probe registers: thread (u, c) owns chunks c + NCH q of probe u
     const int u = tid / NCH, c = tid - u * NCH;
     const bool pact = u < A.W;
-    float qreg[CH];
+    float2 qreg[CH / 2];   // the thread's q chunks as element pairs
     float mu = 0.f, invZ = 0.f;
     {
         const int h = g * A.gq + (u % A.gq);
@@ -252,13 +265,13 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 Vec8<Tin> x;
                 x.load(qp + 8 * (c + NCH * q));
 #pragma unroll
-                for (int r = 0; r < 8; r++) qreg[8 * q + r] = x.v[r];
+                for (int r = 0; r < 4; r++) qreg[4 * q + r] = make_float2(x.v[2 * r], x.v[2 * r + 1]);
             }
             mu = A.row_m[row];
             invZ = 1.0f / A.row_Z[row];
         } else {
 #pragma unroll
-            for (int q = 0; q < CH; q++) qreg[q] = 0.f;
+            for (int q = 0; q < CH / 2; q++) qreg[q] = make_float2(0.f, 0.f);
         }
     }
     __syncthreads();
@@ -307,18 +320,18 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         }
     } else {
         for (int t = 0; t < n; t++) {
-            float xs[NQ];
+            float2 xs[NQ];
 #pragma unroll
             for (int q = 0; q < NQ; q++) {
-                float kv[8];
-                ld8(&sm.kc[t][8 * (c + NCH * q)], kv);
-                xs[q] = 0.f;
+                float2 kv[4];
+                ld8x2(&sm.kc[t][8 * (c + NCH * q)], kv);
+                xs[q] = make_float2(0.f, 0.f);
 #pragma unroll
-                for (int r = 0; r < 8; r++) xs[q] = fmaf(qreg[8 * q + r], kv[r], xs[q]);
+                for (int r = 0; r < 4; r++) xs[q] = ffma2(qreg[4 * q + r], kv[r], xs[q]);
             }
-            float x = xs[0];
+            float x = 0.f;
 #pragma unroll
-            for (int q = 1; q < NQ; q++) x += xs[q];
+            for (int q = 0; q < NQ; q++) x += xs[q].x + xs[q].y;
 #pragma unroll
             for (int o = 1; o < NCH; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
             if (c == 0) sm.E[t][u] = pact ? expf(x * A.inv_sqrt_d - mu) : 0.f;
@@ -479,46 +492,36 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     };
     // D_u of candidate k (prototype row `row`) from the probe statistics Z, M
     // of its interval; per-warp partial sums of pi_u D_u and pi_u.
-    auto evaluate = [&](int k, int row, float Z, const float *M) {
-        float xs[2 * NQ];
-#pragma unroll
-        for (int q = 0; q < NQ; q++) {
-            float kv[8];
-            ld8(&sm.ktil[row][8 * (c + NCH * q)], kv);
-            float x0 = 0.f, x1 = 0.f;
-#pragma unroll
-            for (int r = 0; r < 8; r += 2) {
-                x0 = fmaf(qreg[8 * q + r], kv[r], x0);
-                x1 = fmaf(qreg[8 * q + r + 1], kv[r + 1], x1);
-            }
-            xs[2 * q] = x0;
-            xs[2 * q + 1] = x1;
-        }
+    auto evaluate = [&](int k, int row, float Z, const float2 *M) {
         float x = 0.f;
 #pragma unroll
-        for (int q = 0; q < 2 * NQ; q++) x += xs[q];
+        for (int q = 0; q < NQ; q++) {
+            float2 kv[4];
+            ld8x2(&sm.ktil[row][8 * (c + NCH * q)], kv);
+            float2 xa = make_float2(0.f, 0.f);
+#pragma unroll
+            for (int r = 0; r < 4; r++) xa = ffma2(qreg[4 * q + r], kv[r], xa);
+            x += xa.x + xa.y;
+        }
 #pragma unroll
         for (int o = 1; o < NCH; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
         const float zt = sm.cand[k].meff * expf(x * A.inv_sqrt_d - mu);
-        float rq[NQ], mq[NQ];
-#pragma unroll
-        for (int q = 0; q < NQ; q++) {
-            float vt[8];
-            ld8(&sm.vtil[row][8 * (c + NCH * q)], vt);
-            float r0 = 0.f, m0 = 0.f;
-#pragma unroll
-            for (int r = 0; r < 8; r++) {
-                const float mv = M[8 * q + r];
-                const float df = mv - zt * vt[r];
-                r0 = fmaf(df, df, r0);
-                m0 = fmaf(mv, mv, m0);
-            }
-            rq[q] = r0;
-            mq[q] = m0;
-        }
+        const float2 nz = make_float2(-zt, -zt);
         float res = 0.f, mm = 0.f;
 #pragma unroll
-        for (int q = 0; q < NQ; q++) { res += rq[q]; mm += mq[q]; }
+        for (int q = 0; q < NQ; q++) {
+            float2 vt[4];
+            ld8x2(&sm.vtil[row][8 * (c + NCH * q)], vt);
+            float2 r2 = make_float2(0.f, 0.f), m2 = make_float2(0.f, 0.f);
+#pragma unroll
+            for (int r = 0; r < 4; r++) {
+                const float2 df = ffma2(nz, vt[r], M[4 * q + r]);   // M - zt vtil
+                r2 = ffma2(df, df, r2);
+                m2 = ffma2(M[4 * q + r], M[4 * q + r], m2);
+            }
+            res += r2.x + r2.y;
+            mm += m2.x + m2.y;
+        }
 #pragma unroll
         for (int o = 1; o < NCH; o <<= 1) {
             res += __shfl_xor_sync(0xffffffffu, res, o);
@@ -544,20 +547,21 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         int k = suffix ? B.suf_b : B.pre_b;
         const int ke = suffix ? B.suf_e : B.pre_e;
         if (k >= ke) return;
-        float M[CH];
+        float2 M[CH / 2];
         float Z = 0.f;
 #pragma unroll
-        for (int q = 0; q < CH; q++) M[q] = 0.f;
+        for (int q = 0; q < CH / 2; q++) M[q] = make_float2(0.f, 0.f);
         for (int s = 0; s < b - a && k < ke; s++) {
             const int t = suffix ? b - 1 - s : a + s;
             const float e = sm.E[t][u];
+            const float2 e2 = make_float2(e, e);
             Z += e;
 #pragma unroll
             for (int q = 0; q < NQ; q++) {
-                float vv[8];
-                ld8(&sm.vv[t][8 * (c + NCH * q)], vv);
+                float2 vv[4];
+                ld8x2(&sm.vv[t][8 * (c + NCH * q)], vv);
 #pragma unroll
-                for (int r = 0; r < 8; r++) M[8 * q + r] = fmaf(e, vv[r], M[8 * q + r]);
+                for (int r = 0; r < 4; r++) M[4 * q + r] = ffma2(e2, vv[r], M[4 * q + r]);
             }
             while (k < ke && (suffix ? sm.cand[k].a == t : sm.cand[k].b == t + 1)) {
                 evaluate(k, suffix ? k - kNCD : k, Z, M);
