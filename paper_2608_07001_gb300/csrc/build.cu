@@ -48,7 +48,7 @@ namespace {
 
 constexpr int kMaxCuts = 18;     // K + midpoint, K <= 16 (+1 spare)
 constexpr int kNT = 256;         // threads per CTA
-constexpr int kNCD = 24;         // candidate intervals per direction and batch (>= 17 + 2)
+constexpr int kNCD = 19;         // candidate intervals per direction and batch: 17 cuts + p* side + whole node
 
 struct BuildArgs {
     const void *K, *V, *Q;
@@ -78,18 +78,18 @@ struct BuildArgs {
 };
 
 struct NodeS {
+    double D;
+    float kin;                   // bottleneck key of the op that created the node
     short a, b, parent, child0;
     signed char nchild;          // -1: pending (not evaluated)
-    float kin;                   // bottleneck key of the op that created the node
-    double D, R;
 };
 
 struct BatchNode {
     int node;
     int ncut;
-    short cut[kMaxCuts];     // local cut positions xi (ascending)
-    short pidx[kMaxCuts];    // candidate index of [a, xi) (-1: single token)
-    short sidx[kMaxCuts];    // candidate index of [xi, b) (-1: single token)
+    int8_t cut[kMaxCuts];    // local cut positions xi (ascending)
+    int8_t pidx[kMaxCuts];   // candidate index of [a, xi) (-1: single token)
+    int8_t sidx[kMaxCuts];   // candidate index of [xi, b) (-1: single token)
     int pstar, eL, eR, whole;
     int pre_b, pre_e, suf_b, suf_e;   // prefixes (ascending end) in [0, NCD),
                                       // suffixes (descending start) in [NCD, 2 NCD)
@@ -179,10 +179,10 @@ struct Smem {
     static constexpr int NCH = kNT / NW;     // threads per probe
     static constexpr int CH = DH / NCH;      // elements per thread
     static constexpr int NQ = CH / 8;        // 8-element chunks per thread
-    static constexpr int NB = 32;            // nodes per batch
+    static constexpr int NB = 16;            // nodes per batch
     static constexpr int MAXNODES = 2 * NMAX;
     float kc[NMAX][DH];
-    Tin vv[NMAX][DH];
+    float vv[NMAX][DH];                      // values, converted once to fp32
     float E[NMAX][NW];
     float ktil[kNCD][DH];                    // prototypes of one direction at a time
     float vtil[kNCD][DH];
@@ -201,6 +201,7 @@ struct Smem {
     int batch_n, batch_next, batch_pre, batch_suf;   // candidate entries reserved per direction
     unsigned long long wcnt[kNT / 32][3];   // per-warp work counters
     float pend;
+    double rootR;                            // R of a fresh root
 };
 
 template <int DH, int NW, typename Tin, int NMAX>
@@ -243,7 +244,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
 #pragma unroll
         for (int q = 0; q < 8; q++) {
             sm.kc[t][i + q] = kx.v[q];
-            sm.vv[t][i + q] = (Tin)vx.v[q];
+            sm.vv[t][i + q] = vx.v[q];
         }
     }
     for (int t = tid; t < n; t += kNT) {
@@ -384,7 +385,8 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             if (lane == 0) {
                 NodeS &nd = sm.nodes[0];
                 nd.a = 0; nd.b = (short)n; nd.parent = -1; nd.child0 = -1; nd.nchild = 0;
-                nd.D = 0.0; nd.R = r; nd.kin = 0.f;
+                nd.D = 0.0; nd.kin = 0.f;
+                sm.rootR = r;
                 sm.nnodes = 1;
                 sm.lvl[0][0] = 0;
                 sm.nlvl[0] = 1;
@@ -406,7 +408,6 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             nd.child0 = (short)A.nd_child0[v];
             nd.nchild = A.nd_nchild[v];
             nd.D = A.nd_D[v];
-            nd.R = 0.0;
             nd.kin = pg < 0 ? A.u_Uadd[uid] : A.nd_kappa[pg];
         }
         if (tid == 0) { sm.nnodes = nn; sm.nlvl[0] = 0; sm.pend = -1.f; }
@@ -418,14 +419,6 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 if (nd.kin >= A.tau) sm.lvl[0][sm.nlvl[0]++] = (short)k;
                 else sm.pend = fmaxf(sm.pend, nd.kin);
             }
-        }
-        __syncthreads();
-        for (int q = warp; q < sm.nlvl[0]; q += NWARPS) {   // node values of the resumed nodes
-            NodeS &nd = sm.nodes[sm.lvl[0][q]];
-            double r = 0.0;
-            for (int t = nd.a + lane; t < nd.b; t += 32) r += sm.Rt[t];
-            r = warp_sum(r);
-            if (lane == 0) nd.R = r;
         }
     }
     __syncthreads();
@@ -492,48 +485,49 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     };
     // D_u of candidate k (prototype row `row`) from the probe statistics Z, M
     // of its interval; per-warp partial sums of pi_u D_u and pi_u.
+    const float inv_sqrt_d = A.inv_sqrt_d, lamZ = A.lamZ, lamM = A.lamM, epsf = A.eps;
     auto evaluate = [&](int k, int row, float Z, const float2 *M) {
-        float x = 0.f;
+        // two packed accumulators per sum (even / odd chunks), reduced once
+        float2 xs[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
         for (int q = 0; q < NQ; q++) {
             float2 kv[4];
             ld8x2(&sm.ktil[row][8 * (c + NCH * q)], kv);
-            float2 xa = make_float2(0.f, 0.f);
 #pragma unroll
-            for (int r = 0; r < 4; r++) xa = ffma2(qreg[4 * q + r], kv[r], xa);
-            x += xa.x + xa.y;
+            for (int r = 0; r < 4; r++) xs[q & 1] = ffma2(qreg[4 * q + r], kv[r], xs[q & 1]);
         }
+        float x = (xs[0].x + xs[0].y) + (xs[1].x + xs[1].y);
 #pragma unroll
         for (int o = 1; o < NCH; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-        const float zt = sm.cand[k].meff * expf(x * A.inv_sqrt_d - mu);
+        const float zt = sm.cand[k].meff * expf(x * inv_sqrt_d - mu);
         const float2 nz = make_float2(-zt, -zt);
-        float res = 0.f, mm = 0.f;
+        float2 rs2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+        float2 ms2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
         for (int q = 0; q < NQ; q++) {
             float2 vt[4];
             ld8x2(&sm.vtil[row][8 * (c + NCH * q)], vt);
-            float2 r2 = make_float2(0.f, 0.f), m2 = make_float2(0.f, 0.f);
 #pragma unroll
             for (int r = 0; r < 4; r++) {
                 const float2 df = ffma2(nz, vt[r], M[4 * q + r]);   // M - zt vtil
-                r2 = ffma2(df, df, r2);
-                m2 = ffma2(M[4 * q + r], M[4 * q + r], m2);
+                rs2[q & 1] = ffma2(df, df, rs2[q & 1]);
+                ms2[q & 1] = ffma2(M[4 * q + r], M[4 * q + r], ms2[q & 1]);
             }
-            res += r2.x + r2.y;
-            mm += m2.x + m2.y;
         }
+        float res = (rs2[0].x + rs2[0].y) + (rs2[1].x + rs2[1].y);
+        float mm = (ms2[0].x + ms2[0].y) + (ms2[1].x + ms2[1].y);
 #pragma unroll
         for (int o = 1; o < NCH; o <<= 1) {
             res += __shfl_xor_sync(0xffffffffu, res, o);
             mm += __shfl_xor_sync(0xffffffffu, mm, o);
         }
-        float pd = 0.f, pp = 0.f;
-        if (pact) {
-            const float dz = Z - zt;
-            const float Du = A.lamZ * (dz * dz) / (Z * Z + A.eps) + A.lamM * res / (mm + A.eps);
-            pp = Z * invZ;
-            pd = pp * Du;
-        }
+        // D_u (Eq. app_probe_distortion), weighted by the probe's attention
+        // mass; probes past W have E = 0 and invZ = 0, so they add nothing.
+        // Fast division: at most 2 ulp, far below the distortion tolerance.
+        const float dz = Z - zt;
+        const float Du = lamZ * __fdividef(dz * dz, fmaf(Z, Z, epsf)) + lamM * __fdividef(res, mm + epsf);
+        float pp = Z * invZ;
+        float pd = pp * Du;
 #pragma unroll
         for (int o = NCH; o < 32; o <<= 1) {
             pd += __shfl_xor_sync(0xffffffffu, pd, o);
@@ -676,7 +670,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 for (int w = 0; w < NMAX / 32; w++) {
                     const unsigned m = sel[w];
                     const int q = ncut + __popc(m & ((1u << lane) - 1u));
-                    if (((m >> lane) & 1u) && q < maxc) B.cut[q] = (short)(a + w * 32 + lane + 1);
+                    if (((m >> lane) & 1u) && q < maxc) B.cut[q] = (int8_t)(a + w * 32 + lane + 1);
                     ncut += __popc(m);
                 }
                 ncut = min(ncut, maxc);
@@ -693,7 +687,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 const int pidx = pv ? B.pre_b + __popc(pm & lt) + (el_sep && pb < xi ? 1 : 0) : -1;
                 const int eL_sep = B.pre_b + __popc(__ballot_sync(FULL, pv && xi < pb));
                 const int eL_cut = __shfl_sync(FULL, pidx, pbm ? __ffs(pbm) - 1 : 0);
-                if (hq) B.pidx[lane] = (short)pidx;
+                if (hq) B.pidx[lane] = (int8_t)pidx;
                 if (pv) sm.cand[pidx] = {a, xi, 0.f};
                 // suffixes
                 const int er = pb + 1;
@@ -705,7 +699,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 const int sidx = sv ? B.suf_b + __popc(smk & gt) + (er_sep && er > xi ? 1 : 0) : -1;
                 const int eR_sep = B.suf_b + __popc(__ballot_sync(FULL, sv && xi > er));
                 const int eR_cut = __shfl_sync(FULL, sidx, erm ? __ffs(erm) - 1 : 0);
-                if (hq) B.sidx[lane] = (short)sidx;
+                if (hq) B.sidx[lane] = (int8_t)sidx;
                 if (sv) sm.cand[sidx] = {xi, b, 0.f};
                 // work counters: tokens swept, candidates evaluated, their lengths
                 int len = (pv ? xi - a : 0) + (sv ? b - xi : 0);
@@ -769,7 +763,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     const double Pd = sm.candP[B.whole];
                     const double D = nv >= 2 ? sm.candD[B.whole] : 0.0;
                     nd.D = D;
-                    double gain = (double)om * nd.R * (Pd - D);
+                    double gain = (double)om * sm.rootR * (Pd - D);
                     if (gain < 0.0) gain = 0.0;
                     nd.kin = (float)gain;
                     A.u_Uadd[uid] = (float)gain;
@@ -865,16 +859,17 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     }
                     continue;
                 }
-                double dsum = 0.0, rch[3];
+                double dsum = 0.0, rch[3], rnode = 0.0;   // R of the node = sum over its children
                 for (int q = 0; q < B.nchild; q++) {
                     double r = 0.0;
                     for (int t = B.ca[q] + lane; t < B.cb[q]; t += 32) r += sm.Rt[t];
                     rch[q] = warp_sum(r);
+                    rnode += rch[q];
                     dsum += B.cD[q];
                 }
                 if (lane == 0) {
                     const int cost = B.nchild - 1;
-                    double gain = (double)om * nd.R * (nd.D - dsum);
+                    double gain = (double)om * rnode * (nd.D - dsum);
                     if (gain < 0.0) gain = 0.0;
                     float U = (float)(gain / cost);
                     float kap = fminf(U, nd.kin);
@@ -886,11 +881,11 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                         int ci = nd.child0 + q;
                         NodeS &ch = sm.nodes[ci];
                         ch.a = (short)B.ca[q]; ch.b = (short)B.cb[q]; ch.parent = (short)B.node;
-                        ch.child0 = -1; ch.nchild = 0; ch.D = B.cD[q]; ch.R = rch[q]; ch.kin = kap;
+                        ch.child0 = -1; ch.nchild = 0; ch.D = B.cD[q]; ch.kin = kap;
                         const int64_t gc = nbase + ci;
                         A.nd_a[gc] = sa + ch.a; A.nd_b[gc] = sa + ch.b;
                         A.nd_parent[gc] = (int32_t)gv; A.nd_unit[gc] = (int32_t)uid;
-                        A.nd_D[gc] = ch.D; A.nd_R[gc] = (float)ch.R;
+                        A.nd_D[gc] = ch.D; A.nd_R[gc] = (float)rch[q];
                         A.nd_child0[gc] = -1; A.nd_nchild[gc] = 0; A.nd_cost[gc] = 0;
                         A.nd_U[gc] = 0.f; A.nd_kappa[gc] = 0.f; A.nd_sel[gc] = 0;
                         if (ch.b - ch.a >= 2) {
