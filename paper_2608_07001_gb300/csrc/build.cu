@@ -535,8 +535,10 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         }
         if (lane == 0) { sm.redD[k][warp] = pd; sm.redP[k][warp] = pp; }
     };
-    // Probe scan of one node in one direction, evaluating its candidates.
-    auto scan = [&](const BatchNode &B, bool suffix) {
+    // Probe scan of one node in one direction (SUF: suffixes, descending),
+    // evaluating each candidate when the running sums reach its far end.
+    auto scan = [&](const BatchNode &B, auto SUF) {
+        constexpr bool suffix = decltype(SUF)::value;
         const int a = sm.nodes[B.node].a, b = sm.nodes[B.node].b;
         int k = suffix ? B.suf_b : B.pre_b;
         const int ke = suffix ? B.suf_e : B.pre_e;
@@ -545,8 +547,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         float Z = 0.f;
 #pragma unroll
         for (int q = 0; q < CH / 2; q++) M[q] = make_float2(0.f, 0.f);
-        for (int s = 0; s < b - a && k < ke; s++) {
-            const int t = suffix ? b - 1 - s : a + s;
+        auto add = [&](int t) {
             const float e = sm.E[t][u];
             const float2 e2 = make_float2(e, e);
             Z += e;
@@ -557,9 +558,19 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
 #pragma unroll
                 for (int r = 0; r < 4; r++) M[4 * q + r] = ffma2(e2, vv[r], M[4 * q + r]);
             }
-            while (k < ke && (suffix ? sm.cand[k].a == t : sm.cand[k].b == t + 1)) {
-                evaluate(k, suffix ? k - kNCD : k, Z, M);
-                k++;
+        };
+        int t = suffix ? b - 1 : a;   // next token to add
+        for (; k < ke; k++) {
+            if (suffix) {
+                const int stop = sm.cand[k].a;   // candidates in descending start, all >= a
+#pragma unroll 1
+                for (; t >= stop; t--) add(t);
+                evaluate(k, k - kNCD, Z, M);
+            } else {
+                const int stop = sm.cand[k].b;   // candidates in ascending end, all <= b
+#pragma unroll 1
+                for (; t < stop; t++) add(t);
+                evaluate(k, k, Z, M);
             }
         }
     };
@@ -739,11 +750,11 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             // ---- phases B/C: prefixes, then suffixes ---------------------------
             prototypes(false);
             __syncthreads();
-            for (int bi = 0; bi < nb; bi++) scan(sm.bn[bi], false);
+            for (int bi = 0; bi < nb; bi++) scan(sm.bn[bi], std::false_type());
             __syncthreads();
             prototypes(true);
             __syncthreads();
-            for (int bi = 0; bi < nb; bi++) scan(sm.bn[bi], true);
+            for (int bi = 0; bi < nb; bi++) scan(sm.bn[bi], std::true_type());
             __syncthreads();
             // ---- per-candidate D and drop mass (thread per candidate) ------------
             for (int k = tid; k < 2 * kNCD; k += kNT) {
