@@ -34,9 +34,10 @@
 // reaches the frontier before the allocation stops, so its own Split is never
 // needed.  Resuming repeats until no pending node qualifies.
 //
-// Layout.  256 threads; thread (u, c) owns probe u and the 8-element chunks
-// c, c + NCH, c + 2 NCH, ... of every d-vector, so that its shared-memory
-// reads are 16-byte vectors and the lanes of a warp never share a bank.
+// Layout.  256 threads; thread (p, c) owns the probes p and p + 32 and the
+// elements 4 c + 32 g + j (j < 4) of every d-vector: each value, prototype or
+// key chunk it reads from shared memory serves two probes, and 8 consecutive
+// threads read 128 contiguous bytes (one wavefront, no bank conflicts).
 // Slots of up to 64 tokens use a 64-token instance whose footprint allows two
 // CTAs per SM; longer slots use the 128-token instance.
 #include "gkv_internal.cuh"
@@ -48,6 +49,8 @@ namespace {
 
 constexpr int kMaxCuts = 18;     // K + midpoint, K <= 16 (+1 spare)
 constexpr int kNT = 256;         // threads per CTA
+constexpr int kNPP = 32;         // probe pairs: thread handles probes p and p + 32 (W <= 64)
+constexpr int kNCL = 8;          // threads per probe pair (4-element groups, interleaved)
 constexpr int kNCD = 19;         // candidate intervals per direction and batch: 17 cuts + p* side + whole node
 
 struct BuildArgs {
@@ -138,6 +141,15 @@ __device__ __forceinline__ void ld8(const __nv_bfloat16 *p, float v[8]) {
     }
 }
 
+// 4 consecutive elements (8- or 16-byte aligned) as floats.
+__device__ __forceinline__ float4 ld4(const float *p) { return *reinterpret_cast<const float4 *>(p); }
+__device__ __forceinline__ float4 ld4(const __nv_bfloat16 *p) {
+    const uint2 u = *reinterpret_cast<const uint2 *>(p);
+    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&u.x));
+    const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&u.y));
+    return make_float4(a.x, a.y, b.x, b.y);
+}
+
 // 8 consecutive elements of a shared-memory row as 4 float pairs.
 __device__ __forceinline__ void ld8x2(const float *p, float2 v[4]) {
     const float4 a = reinterpret_cast<const float4 *>(p)[0], b = reinterpret_cast<const float4 *>(p)[1];
@@ -173,17 +185,14 @@ __device__ __forceinline__ void ld_pairs(const __nv_bfloat16 *p, float v[N]) {
     }
 }
 
-template <int DH, int NW, typename Tin, int NMAX>
+template <int DH, typename Tin, int NMAX>
 struct Smem {
     static constexpr int NWARPS = kNT / 32;
-    static constexpr int NCH = kNT / NW;     // threads per probe
-    static constexpr int CH = DH / NCH;      // elements per thread
-    static constexpr int NQ = CH / 8;        // 8-element chunks per thread
     static constexpr int NB = 16;            // nodes per batch
     static constexpr int MAXNODES = 2 * NMAX;
     float kc[NMAX][DH];
     float vv[NMAX][DH];                      // values, converted once to fp32
-    float E[NMAX][NW];
+    float2 E[NMAX][kNPP];                    // probe weights of probes (p, p + 32)
     float ktil[kNCD][DH];                    // prototypes of one direction at a time
     float vtil[kNCD][DH];
     float Rt[NMAX];
@@ -204,11 +213,12 @@ struct Smem {
     double rootR;                            // R of a fresh root
 };
 
-template <int DH, int NW, typename Tin, int NMAX>
+template <int DH, typename Tin, int NMAX>
 __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(BuildArgs A) {
-    using S = Smem<DH, NW, Tin, NMAX>;
-    constexpr int NCH = S::NCH, CH = S::CH, NQ = S::NQ, HALF = DH / 2, NWARPS = S::NWARPS;
-    static_assert(NCH <= 32 && (32 % NCH) == 0 && CH % 8 == 0, "probe layout");
+    using S = Smem<DH, Tin, NMAX>;
+    // thread (p, c): probes p and p + 32, elements 4 c + 32 g + j (g < NG, j < 4)
+    constexpr int HALF = DH / 2, NWARPS = S::NWARPS, NG = DH / (4 * kNCL), CH = 4 * NG;
+    static_assert(kNPP * kNCL == kNT && DH % (4 * kNCL) == 0, "probe layout");
     extern __shared__ __align__(16) unsigned char smem_raw[];
     S &sm = *reinterpret_cast<S *>(smem_raw);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -251,37 +261,41 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         sm.kap[t] = okey(A.kappa[sa + t]);
         sm.Rt[t] = A.rtok[(size_t)lg * A.Nc + (sa - A.cs) + t];
     }
-    // probe registers: thread (u, c) owns chunks c + NCH q of probe u
-    const int u = tid / NCH, c = tid - u * NCH;
-    const bool pact = u < A.W;
-    float2 qreg[CH / 2];   // the thread's q chunks as element pairs
-    float mu = 0.f, invZ = 0.f;
-    {
-        const int h = g * A.gq + (u % A.gq);
-        const size_t row = ((size_t)l * A.Hq + h) * A.W + u;
-        if (pact) {
-            const Tin *qp = static_cast<const Tin *>(A.Q) + row * DH;
+    // probe registers: thread (pp, c) owns probes pp and pp + 32, elements
+    // 4 c + 32 g + j, so that 8 consecutive threads read 128 contiguous bytes
+    const int pp = tid / kNCL, c = tid - pp * kNCL;
+    float2 qa0[CH / 2], qa1[CH / 2];   // q of the two probes as element pairs
+    float mu0 = 0.f, mu1 = 0.f, invZ0 = 0.f, invZ1 = 0.f;
 #pragma unroll
-            for (int q = 0; q < NQ; q++) {
-                Vec8<Tin> x;
-                x.load(qp + 8 * (c + NCH * q));
+    for (int h = 0; h < 2; h++) {
+        const int u = pp + kNPP * h;
+        float2 *qd = h ? qa1 : qa0;
+        if (u < A.W) {
+            const size_t row = ((size_t)l * A.Hq + g * A.gq + (u % A.gq)) * A.W + u;
+            const Tin *qp = static_cast<const Tin *>(A.Q) + row * DH + 4 * c;
 #pragma unroll
-                for (int r = 0; r < 4; r++) qreg[4 * q + r] = make_float2(x.v[2 * r], x.v[2 * r + 1]);
+            for (int gi = 0; gi < NG; gi++) {
+                float4 x = ld4(qp + 32 * gi);
+                qd[2 * gi] = make_float2(x.x, x.y);
+                qd[2 * gi + 1] = make_float2(x.z, x.w);
             }
-            mu = A.row_m[row];
-            invZ = 1.0f / A.row_Z[row];
+            (h ? mu1 : mu0) = A.row_m[row];
+            (h ? invZ1 : invZ0) = 1.0f / A.row_Z[row];
         } else {
 #pragma unroll
-            for (int q = 0; q < CH / 2; q++) qreg[q] = make_float2(0.f, 0.f);
+            for (int q = 0; q < CH / 2; q++) qd[q] = make_float2(0.f, 0.f);
         }
     }
     __syncthreads();
 
     // ---- E[t][u] from the raw (post-RoPE) keys -------------------------------
+    // Probe u is stored at E[t][u % 32].x (u < 32) or .y (u >= 32).
+    float *Ef = reinterpret_cast<float *>(&sm.E[0][0]);
+    auto eidx = [](int t, int u) { return t * 2 * kNPP + 2 * (u & (kNPP - 1)) + (u >> 5); };
     if constexpr (std::is_same<Tin, __nv_bfloat16>::value) {
-        // Tensor cores: logits = Q_probes (NW x DH) . K_slot^T, one 16x8 tile
-        // per (probe block, token block); warp w keeps probe block w % MT.
-        constexpr int MT = NW / 16, WSTEP = NWARPS / MT;
+        // Tensor cores: logits = Q_probes (64 x DH) . K_slot^T, one 16x8 tile
+        // per (probe block, token block); warp w keeps probe block w % 4.
+        constexpr int MT = 4, WSTEP = NWARPS / MT;
         const int gr = lane >> 2, c2 = 2 * (lane & 3);
         const int mt = warp % MT;
         const int u0 = mt * 16 + gr, u1 = u0 + 8;
@@ -311,31 +325,33 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             }
             const int t0 = nt * 8 + c2;
             if (t0 < n) {
-                sm.E[t0][u0] = ok0 ? expf(acc[0] * A.inv_sqrt_d - m0) : 0.f;
-                sm.E[t0][u1] = ok1 ? expf(acc[2] * A.inv_sqrt_d - m1) : 0.f;
+                Ef[eidx(t0, u0)] = ok0 ? expf(acc[0] * A.inv_sqrt_d - m0) : 0.f;
+                Ef[eidx(t0, u1)] = ok1 ? expf(acc[2] * A.inv_sqrt_d - m1) : 0.f;
             }
             if (t0 + 1 < n) {
-                sm.E[t0 + 1][u0] = ok0 ? expf(acc[1] * A.inv_sqrt_d - m0) : 0.f;
-                sm.E[t0 + 1][u1] = ok1 ? expf(acc[3] * A.inv_sqrt_d - m1) : 0.f;
+                Ef[eidx(t0 + 1, u0)] = ok0 ? expf(acc[1] * A.inv_sqrt_d - m0) : 0.f;
+                Ef[eidx(t0 + 1, u1)] = ok1 ? expf(acc[3] * A.inv_sqrt_d - m1) : 0.f;
             }
         }
     } else {
         for (int t = 0; t < n; t++) {
-            float2 xs[NQ];
+            float2 x0 = make_float2(0.f, 0.f), x1 = make_float2(0.f, 0.f);
 #pragma unroll
-            for (int q = 0; q < NQ; q++) {
-                float2 kv[4];
-                ld8x2(&sm.kc[t][8 * (c + NCH * q)], kv);
-                xs[q] = make_float2(0.f, 0.f);
-#pragma unroll
-                for (int r = 0; r < 4; r++) xs[q] = ffma2(qreg[4 * q + r], kv[r], xs[q]);
+            for (int gi = 0; gi < NG; gi++) {
+                const float4 kv = *reinterpret_cast<const float4 *>(&sm.kc[t][4 * c + 32 * gi]);
+                const float2 ka = make_float2(kv.x, kv.y), kb = make_float2(kv.z, kv.w);
+                x0 = ffma2(qa0[2 * gi], ka, x0); x0 = ffma2(qa0[2 * gi + 1], kb, x0);
+                x1 = ffma2(qa1[2 * gi], ka, x1); x1 = ffma2(qa1[2 * gi + 1], kb, x1);
             }
-            float x = 0.f;
+            float y0 = x0.x + x0.y, y1 = x1.x + x1.y;
 #pragma unroll
-            for (int q = 0; q < NQ; q++) x += xs[q].x + xs[q].y;
-#pragma unroll
-            for (int o = 1; o < NCH; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-            if (c == 0) sm.E[t][u] = pact ? expf(x * A.inv_sqrt_d - mu) : 0.f;
+            for (int o = 1; o < kNCL; o <<= 1) {
+                y0 += __shfl_xor_sync(0xffffffffu, y0, o);
+                y1 += __shfl_xor_sync(0xffffffffu, y1, o);
+            }
+            if (c == 0)
+                sm.E[t][pp] = make_float2(pp < A.W ? expf(y0 * A.inv_sqrt_d - mu0) : 0.f,
+                                          pp + kNPP < A.W ? expf(y1 * A.inv_sqrt_d - mu1) : 0.f);
         }
     }
     __syncthreads();
@@ -345,7 +361,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     // the host reports as GKV_ENONFINITE at the allocation's count sync.
     {
         bool bad = false;
-        for (int e = tid; e < n * NW; e += kNT) bad |= !isfinite(sm.E[e / NW][e % NW]);
+        for (int e = tid; e < n * 2 * kNPP; e += kNT) bad |= !isfinite(Ef[e]);
         for (int t = tid; t < n; t += kNT) bad |= !isfinite(sm.Rt[t]);
         if (__syncthreads_or(bad)) {
             if (tid == 0) {
@@ -486,54 +502,69 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     // D_u of candidate k (prototype row `row`) from the probe statistics Z, M
     // of its interval; per-warp partial sums of pi_u D_u and pi_u.
     const float inv_sqrt_d = A.inv_sqrt_d, lamZ = A.lamZ, lamM = A.lamM, epsf = A.eps;
-    auto evaluate = [&](int k, int row, float Z, const float2 *M) {
-        // two packed accumulators per sum (even / odd chunks), reduced once
-        float2 xs[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+    // D_u of candidate k (prototype row `row`) for the thread's two probes from
+    // their running statistics Z, M; per-warp partial sums of pi_u D_u and pi_u.
+    auto evaluate = [&](int k, int row, float Z0, float Z1, const float2 *M0, const float2 *M1) {
+        float2 kt[CH / 2];
 #pragma unroll
-        for (int q = 0; q < NQ; q++) {
-            float2 kv[4];
-            ld8x2(&sm.ktil[row][8 * (c + NCH * q)], kv);
-#pragma unroll
-            for (int r = 0; r < 4; r++) xs[q & 1] = ffma2(qreg[4 * q + r], kv[r], xs[q & 1]);
+        for (int gi = 0; gi < NG; gi++) {
+            const float4 x = *reinterpret_cast<const float4 *>(&sm.ktil[row][4 * c + 32 * gi]);
+            kt[2 * gi] = make_float2(x.x, x.y);
+            kt[2 * gi + 1] = make_float2(x.z, x.w);
         }
-        float x = (xs[0].x + xs[0].y) + (xs[1].x + xs[1].y);
+        float2 xa = make_float2(0.f, 0.f), xb = make_float2(0.f, 0.f);
 #pragma unroll
-        for (int o = 1; o < NCH; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-        const float zt = sm.cand[k].meff * expf(x * inv_sqrt_d - mu);
-        const float2 nz = make_float2(-zt, -zt);
-        float2 rs2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-        float2 ms2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+        for (int q = 0; q < CH / 2; q++) {
+            xa = ffma2(qa0[q], kt[q], xa);
+            xb = ffma2(qa1[q], kt[q], xb);
+        }
+        float x0 = xa.x + xa.y, x1 = xb.x + xb.y;
 #pragma unroll
-        for (int q = 0; q < NQ; q++) {
-            float2 vt[4];
-            ld8x2(&sm.vtil[row][8 * (c + NCH * q)], vt);
+        for (int o = 1; o < kNCL; o <<= 1) {
+            x0 += __shfl_xor_sync(0xffffffffu, x0, o);
+            x1 += __shfl_xor_sync(0xffffffffu, x1, o);
+        }
+        const float me = sm.cand[k].meff;
+        const float zt0 = me * expf(x0 * inv_sqrt_d - mu0), zt1 = me * expf(x1 * inv_sqrt_d - mu1);
+        const float2 nz0 = make_float2(-zt0, -zt0), nz1 = make_float2(-zt1, -zt1);
+        float2 r0 = make_float2(0.f, 0.f), r1 = r0, m0 = r0, m1 = r0;
 #pragma unroll
-            for (int r = 0; r < 4; r++) {
-                const float2 df = ffma2(nz, vt[r], M[4 * q + r]);   // M - zt vtil
-                rs2[q & 1] = ffma2(df, df, rs2[q & 1]);
-                ms2[q & 1] = ffma2(M[4 * q + r], M[4 * q + r], ms2[q & 1]);
+        for (int gi = 0; gi < NG; gi++) {
+            const float4 x = *reinterpret_cast<const float4 *>(&sm.vtil[row][4 * c + 32 * gi]);
+            const float2 va = make_float2(x.x, x.y), vb = make_float2(x.z, x.w);
+#pragma unroll
+            for (int h = 0; h < 2; h++) {
+                const int q = 2 * gi + h;
+                const float2 vt = h ? vb : va;
+                const float2 d0 = ffma2(nz0, vt, M0[q]), d1 = ffma2(nz1, vt, M1[q]);   // M - zt vtil
+                r0 = ffma2(d0, d0, r0);
+                r1 = ffma2(d1, d1, r1);
+                m0 = ffma2(M0[q], M0[q], m0);
+                m1 = ffma2(M1[q], M1[q], m1);
             }
         }
-        float res = (rs2[0].x + rs2[0].y) + (rs2[1].x + rs2[1].y);
-        float mm = (ms2[0].x + ms2[0].y) + (ms2[1].x + ms2[1].y);
+        float res0 = r0.x + r0.y, res1 = r1.x + r1.y, mm0 = m0.x + m0.y, mm1 = m1.x + m1.y;
 #pragma unroll
-        for (int o = 1; o < NCH; o <<= 1) {
-            res += __shfl_xor_sync(0xffffffffu, res, o);
-            mm += __shfl_xor_sync(0xffffffffu, mm, o);
+        for (int o = 1; o < kNCL; o <<= 1) {
+            res0 += __shfl_xor_sync(0xffffffffu, res0, o);
+            res1 += __shfl_xor_sync(0xffffffffu, res1, o);
+            mm0 += __shfl_xor_sync(0xffffffffu, mm0, o);
+            mm1 += __shfl_xor_sync(0xffffffffu, mm1, o);
         }
         // D_u (Eq. app_probe_distortion), weighted by the probe's attention
         // mass; probes past W have E = 0 and invZ = 0, so they add nothing.
         // Fast division: at most 2 ulp, far below the distortion tolerance.
-        const float dz = Z - zt;
-        const float Du = lamZ * __fdividef(dz * dz, fmaf(Z, Z, epsf)) + lamM * __fdividef(res, mm + epsf);
-        float pp = Z * invZ;
-        float pd = pp * Du;
+        const float dz0 = Z0 - zt0, dz1 = Z1 - zt1;
+        const float D0 = lamZ * __fdividef(dz0 * dz0, fmaf(Z0, Z0, epsf)) + lamM * __fdividef(res0, mm0 + epsf);
+        const float D1 = lamZ * __fdividef(dz1 * dz1, fmaf(Z1, Z1, epsf)) + lamM * __fdividef(res1, mm1 + epsf);
+        const float p0 = Z0 * invZ0, p1 = Z1 * invZ1;
+        float pd = fmaf(p0, D0, p1 * D1), pw = p0 + p1;
 #pragma unroll
-        for (int o = NCH; o < 32; o <<= 1) {
+        for (int o = kNCL; o < 32; o <<= 1) {
             pd += __shfl_xor_sync(0xffffffffu, pd, o);
-            pp += __shfl_xor_sync(0xffffffffu, pp, o);
+            pw += __shfl_xor_sync(0xffffffffu, pw, o);
         }
-        if (lane == 0) { sm.redD[k][warp] = pd; sm.redP[k][warp] = pp; }
+        if (lane == 0) { sm.redD[k][warp] = pd; sm.redP[k][warp] = pw; }
     };
     // Probe scan of one node in one direction (SUF: suffixes, descending),
     // evaluating each candidate when the running sums reach its far end.
@@ -543,20 +574,23 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         int k = suffix ? B.suf_b : B.pre_b;
         const int ke = suffix ? B.suf_e : B.pre_e;
         if (k >= ke) return;
-        float2 M[CH / 2];
-        float Z = 0.f;
+        float2 M0[CH / 2], M1[CH / 2];
+        float Z0 = 0.f, Z1 = 0.f;
 #pragma unroll
-        for (int q = 0; q < CH / 2; q++) M[q] = make_float2(0.f, 0.f);
+        for (int q = 0; q < CH / 2; q++) M0[q] = M1[q] = make_float2(0.f, 0.f);
         auto add = [&](int t) {
-            const float e = sm.E[t][u];
-            const float2 e2 = make_float2(e, e);
-            Z += e;
+            const float2 e = sm.E[t][pp];
+            const float2 e0 = make_float2(e.x, e.x), e1 = make_float2(e.y, e.y);
+            Z0 += e.x;
+            Z1 += e.y;
 #pragma unroll
-            for (int q = 0; q < NQ; q++) {
-                float2 vv[4];
-                ld8x2(&sm.vv[t][8 * (c + NCH * q)], vv);
-#pragma unroll
-                for (int r = 0; r < 4; r++) M[4 * q + r] = ffma2(e2, vv[r], M[4 * q + r]);
+            for (int gi = 0; gi < NG; gi++) {
+                const float4 x = *reinterpret_cast<const float4 *>(&sm.vv[t][4 * c + 32 * gi]);
+                const float2 va = make_float2(x.x, x.y), vb = make_float2(x.z, x.w);
+                M0[2 * gi] = ffma2(e0, va, M0[2 * gi]);
+                M0[2 * gi + 1] = ffma2(e0, vb, M0[2 * gi + 1]);
+                M1[2 * gi] = ffma2(e1, va, M1[2 * gi]);
+                M1[2 * gi + 1] = ffma2(e1, vb, M1[2 * gi + 1]);
             }
         };
         int t = suffix ? b - 1 : a;   // next token to add
@@ -565,12 +599,12 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 const int stop = sm.cand[k].a;   // candidates in descending start, all >= a
 #pragma unroll 1
                 for (; t >= stop; t--) add(t);
-                evaluate(k, k - kNCD, Z, M);
+                evaluate(k, k - kNCD, Z0, Z1, M0, M1);
             } else {
                 const int stop = sm.cand[k].b;   // candidates in ascending end, all <= b
 #pragma unroll 1
                 for (; t < stop; t++) add(t);
-                evaluate(k, k, Z, M);
+                evaluate(k, k, Z0, Z1, M0, M1);
             }
         }
     };
@@ -940,26 +974,23 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         for (int k = sm.nnodes + tid; k < 2 * n; k += kNT) A.nd_cost[nbase + k] = 0;
 }
 
-template <int DH, int NW, typename Tin, int NMAX>
+template <int DH, typename Tin, int NMAX>
 cudaError_t launch_t(Ctx &c, BuildArgs &A, unsigned grid, cudaStream_t s) {
-    using S = Smem<DH, NW, Tin, NMAX>;
+    using S = Smem<DH, Tin, NMAX>;
     static_assert(sizeof(S) <= 227 * 1024, "unit kernel shared memory above the per-CTA limit");
     if (grid == 0) return cudaSuccess;
     size_t sm = sizeof(S);
-    cudaError_t e = cudaFuncSetAttribute(unit_build_kernel<DH, NW, Tin, NMAX>,
+    cudaError_t e = cudaFuncSetAttribute(unit_build_kernel<DH, Tin, NMAX>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
-    unit_build_kernel<DH, NW, Tin, NMAX><<<grid, kNT, sm, s>>>(A);
+    unit_build_kernel<DH, Tin, NMAX><<<grid, kNT, sm, s>>>(A);
     c.launches += 1;
     return cudaGetLastError();
 }
 
 template <typename Tin, int NMAX>
 cudaError_t launch_dt(Ctx &c, BuildArgs &A, unsigned grid, cudaStream_t s) {
-    int nw = c.p.W <= 32 ? 32 : 64;
-    if (c.p.d == 128)
-        return nw == 32 ? launch_t<128, 32, Tin, NMAX>(c, A, grid, s) : launch_t<128, 64, Tin, NMAX>(c, A, grid, s);
-    return nw == 32 ? launch_t<64, 32, Tin, NMAX>(c, A, grid, s) : launch_t<64, 64, Tin, NMAX>(c, A, grid, s);
+    return c.p.d == 128 ? launch_t<128, Tin, NMAX>(c, A, grid, s) : launch_t<64, Tin, NMAX>(c, A, grid, s);
 }
 
 }  // namespace
