@@ -31,7 +31,7 @@ struct Workspace {
     double *bscore = nullptr;      // [T] boundary score
     double *zbuf = nullptr;        // [T] scratch for robust z
     double *p2 = nullptr;          // [N_c + 1] prefix of sum_l ||d_t||^2
-    float2 *ew = nullptr;          // [(N_c + 1) * nb] DP edge weights (len n_min..n_max), (hi, lo) pairs
+    float *ew = nullptr;           // [(N_c + 1) * nbp] DP edge weights (len n_min..n_max), rows padded to 4
     float2 *ewt = nullptr;         // [n_max + 1] terminal edge weights (len 1..n_max) at i = N_c
     double *dpF = nullptr;         // [N_c + 1] DP values
     int32_t *slots = nullptr;      // [N_c + 2] slot starts (absolute)

@@ -391,6 +391,10 @@ struct BandArgs {
     double lambda_d, lambda_n, c_cut;
 };
 
+// Row stride of the DP edge weights: n_max - n_min + 1 floats padded to a
+// multiple of 4, so that every row starts on a 16-byte boundary.
+__host__ __device__ constexpr int dp_row(int nb) { return (nb + 3) & ~3; }
+
 constexpr int kRB = 32;
 constexpr int kKC = 32;   // channel chunk
 
@@ -398,10 +402,10 @@ template <typename Tin>
 __global__ void __launch_bounds__(256) seg_band_kernel(const Tin *V, const float *hidden, BandArgs b,
                                                        const float *inv_norm, const float *nrm2,
                                                        const double *p2, const double *bscore,
-                                                       float2 *ew) {
+                                                       float *ew) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const SegArgs &a = b.s;
-    const int nb = b.n_max - b.n_min + 1;
+    const int nb = b.n_max - b.n_min + 1, nbp = dp_row(nb);
     const int ncol = kRB + nb - 1;                   // predecessors a in [E0+1-n_max, E0+RB-n_min]
     float *As = reinterpret_cast<float *>(smem_raw); // [kKC][kRB] (conflict-free reads)
     float *Bs = As + kRB * kKC;                      // [ncol][kKC]
@@ -473,7 +477,7 @@ __global__ void __launch_bounds__(256) seg_band_kernel(const Tin *V, const float
         if (len < b.n_min || len > b.n_max) continue;
         double w;
         if (ap < 0) {
-            ew[(size_t)i * nb + (len - b.n_min)] = make_float2(-INFINITY, 0.f);
+            ew[(size_t)i * nbp + (len - b.n_min)] = -INFINITY;
             continue;
         } else {
             int nS = len - 1;
@@ -486,7 +490,7 @@ __global__ void __launch_bounds__(256) seg_band_kernel(const Tin *V, const float
             double pen = (double)(len - b.n0) / b.n0;
             w = gam - b.lambda_d * disp - b.lambda_n * pen * pen;
         }
-        ew[(size_t)i * nb + (len - b.n_min)] = df_split(w);
+        ew[(size_t)i * nbp + (len - b.n_min)] = (float)w;
     }
 }
 
@@ -514,10 +518,10 @@ __host__ __device__ constexpr size_t band_mma_smem(int nb) {
 __global__ void __launch_bounds__(256) seg_band_mma_kernel(const __nv_bfloat16 *V, BandArgs b,
                                                            const float *inv_norm, const float *nrm2,
                                                            const double *p2, const double *bscore,
-                                                           float2 *ew) {
+                                                           float *ew) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const SegArgs &a = b.s;
-    const int nb = b.n_max - b.n_min + 1;
+    const int nb = b.n_max - b.n_min + 1, nbp = dp_row(nb);
     const int nct = band_ncol_tiles(nb);
     const int nrs = kBM + 8 * nct;                      // staged rows: A rows, then B rows
     __nv_bfloat16 *stg = reinterpret_cast<__nv_bfloat16 *>(smem_raw);   // [2][nrs][kBStride]
@@ -623,7 +627,7 @@ __global__ void __launch_bounds__(256) seg_band_mma_kernel(const __nv_bfloat16 *
             const int i = ep + 1, len = i - ap;
             if (len < b.n_min || len > b.n_max) continue;
             if (ap < 0) {
-                ew[(size_t)i * nb + (len - b.n_min)] = make_float2(-INFINITY, 0.f);
+                ew[(size_t)i * nbp + (len - b.n_min)] = -INFINITY;
                 continue;
             }
             const int nS = len - 1;
@@ -634,7 +638,7 @@ __global__ void __launch_bounds__(256) seg_band_mma_kernel(const __nv_bfloat16 *
             }
             const double gam = ap == 0 ? 0.0 : bscore[a.cs + ap - 1] - b.c_cut;
             const double pen = (double)(len - b.n0) / b.n0;
-            ew[(size_t)i * nb + (len - b.n_min)] = df_split(gam - b.lambda_d * disp - b.lambda_n * pen * pen);
+            ew[(size_t)i * nbp + (len - b.n_min)] = (float)(gam - b.lambda_d * disp - b.lambda_n * pen * pen);
         }
     }
 }
@@ -678,27 +682,34 @@ __global__ void seg_band_terminal_kernel(const Tin *V, const float *hidden, Band
 // if smaller) at a time: F[i..i+15] only read F[< i] because i - a >= n_min,
 // so one barrier per step suffices.  Lane handles the lengths n_min + lane +
 // 32 j; the warp reduces its candidates (value desc, a asc) with shuffles.
-// The edge weights of the next kDpPD steps are prefetched into registers
-// (they do not depend on F).  The chosen slot length of every endpoint is
-// kept in shared memory (uint8) so the backtracking runs without global
-// round trips.
+// The edge weights do not depend on F: each warp streams its own endpoint
+// rows kDpPD steps ahead into a private shared-memory ring with cp.async.
+// The chosen slot length of every endpoint is kept in shared memory (uint8)
+// so the backtracking runs without global round trips.  The state F is a
+// double-float; the edge weights are fp32 (their rounding, ~1e-7 of a weight,
+// is far below the DP's near-tie margin).
 // ---------------------------------------------------------------------------
 constexpr int kDpRing = 256;
 constexpr int kDpEp = 16;    // endpoints per step (warps)
-constexpr int kDpPD = 6;     // steps of edge weights in flight
+constexpr int kDpPD = 8;     // steps of edge weights in flight per warp
 constexpr int kDpLen = 4;    // lengths per lane: n_max - n_min + 1 <= 128
+
+__host__ __device__ constexpr size_t dp_smem(int N, int nb) {
+    return (size_t)kDpRing * 8 + (size_t)kDpEp * kDpPD * dp_row(nb) * 4 + (((size_t)N + 1 + 15) & ~(size_t)15);
+}
 
 __device__ __forceinline__ bool better(df2 v, int a, df2 bv, int ba) {
     return df_gt(v, bv) || (df_eq(v, bv) && a < ba);
 }
 
-__global__ void __launch_bounds__(kDpEp * 32) seg_dp_kernel(const float2 *ew, const float2 *ewt, int N,
+__global__ void __launch_bounds__(kDpEp * 32) seg_dp_kernel(const float *ew, const float2 *ewt, int N,
                                                             int n_min, int n_max, int cs, double *Fout,
                                                             int32_t *slots, int *dev_int) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
-    df2 *ring = reinterpret_cast<df2 *>(smem_raw);                       // [kDpRing]
-    uint8_t *lenarr = reinterpret_cast<uint8_t *>(ring + kDpRing);       // [N + 1]
-    const int nb = n_max - n_min + 1;
+    const int nb = n_max - n_min + 1, nbp = dp_row(nb);
+    df2 *ring = reinterpret_cast<df2 *>(smem_raw);                                   // [kDpRing]
+    float *wbuf = reinterpret_cast<float *>(ring + kDpRing);                         // [kDpEp][kDpPD][nbp]
+    uint8_t *lenarr = reinterpret_cast<uint8_t *>(wbuf + (size_t)kDpEp * kDpPD * nbp);   // [N + 1]
     const int tid = threadIdx.x, lane = tid & 31, k = tid >> 5;
     const int step = min(n_min, kDpEp);
     const df2 NEG = df2{-INFINITY, 0.f};
@@ -707,21 +718,24 @@ __global__ void __launch_bounds__(kDpEp * 32) seg_dp_kernel(const float2 *ew, co
         Fout[0] = 0.0;
         lenarr[0] = 0;
     }
-    float2 wb[kDpPD][kDpLen];
-    auto load_w = [&](int i, float2 out[kDpLen]) {
-#pragma unroll
-        for (int j = 0; j < kDpLen; j++) {
-            const int len = n_min + lane + 32 * j;
-            out[j] = (k < step && i <= N && len <= n_max) ? ew[(size_t)i * nb + (len - n_min)]
-                                                          : make_float2(-INFINITY, 0.f);
-        }
+    float *mybuf = wbuf + (size_t)k * kDpPD * nbp;
+    // row of endpoint i into stage q of this warp's ring (16-byte chunks)
+    auto fetch = [&](int i, int q) {
+        const bool ok = k < step && i <= N;
+        for (int c4 = lane; c4 < nbp / 4; c4 += 32)
+            cp_async16(mybuf + (size_t)q * nbp + 4 * c4, ew + (size_t)(ok ? i : 0) * nbp + 4 * c4, ok);
+        cp_async_commit();
     };
 #pragma unroll
-    for (int q = 0; q < kDpPD; q++) load_w(1 + q * step + k, wb[q]);
+    for (int q = 0; q < kDpPD; q++) fetch(1 + q * step + k, q);
     __syncthreads();
+    int q = 0;
     for (int i0 = 1; i0 <= N; i0 += step) {
         const int i = i0 + k;
         const bool act = k < step && i <= N;
+        cp_async_wait<kDpPD - 1>();   // this step's row (the oldest group) has landed
+        __syncwarp();
+        const float *wr = mybuf + (size_t)q * nbp;
         df2 best = NEG;
         int ba = 0x7fffffff;
         if (act) {
@@ -732,15 +746,13 @@ __global__ void __launch_bounds__(kDpEp * 32) seg_dp_kernel(const float2 *ew, co
                 if (len > n_max || a < 0) break;
                 const df2 fa = ring[a % kDpRing];
                 if (fa.hi == -INFINITY) continue;
-                const df2 v = df_add(fa, wb[0][j]);
+                const df2 v = df_add(fa, make_float2(wr[len - n_min], 0.f));
                 if (better(v, a, best, ba)) { best = v; ba = a; }
             }
         }
-#pragma unroll
-        for (int q = 0; q + 1 < kDpPD; q++)
-#pragma unroll
-            for (int j = 0; j < kDpLen; j++) wb[q][j] = wb[q + 1][j];
-        load_w(i0 + kDpPD * step + k, wb[kDpPD - 1]);
+        __syncwarp();
+        fetch(i0 + kDpPD * step + k, q);   // reuse the stage for kDpPD steps ahead
+        q = q + 1 == kDpPD ? 0 : q + 1;
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
             df2 ov;
@@ -756,6 +768,7 @@ __global__ void __launch_bounds__(kDpEp * 32) seg_dp_kernel(const float2 *ew, co
         }
         __syncthreads();
     }
+    cp_async_wait<0>();
     if (tid == 0 && ring[N % kDpRing].hi == -INFINITY) {
         // terminal relaxation (Eq. app_terminal_predecessor): 1 <= N - a <= n_max,
         // read after every F[< N] has been written
@@ -880,8 +893,7 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
         seg_band_kernel<<<gb, 256, smb, s>>>(Vf, hidden, b, w.inv_norm, w.nrm2, w.p2, w.bscore, w.ew);
         seg_band_terminal_kernel<<<(p.n_max + 7) / 8, 256, 0, s>>>(Vf, hidden, b, w.inv_norm, w.nrm2, w.p2, w.bscore, w.ewt);
     }
-    size_t smd = kDpRing * sizeof(df2) + (size_t)(N + 1);
-    smd = (smd + 15) & ~(size_t)15;
+    const size_t smd = dp_smem(N, nb);
     if (smd > 227 * 1024 || nb > 32 * kDpLen) return cudaErrorInvalidConfiguration;
     cudaFuncSetAttribute(seg_dp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smd);
     seg_dp_kernel<<<1, kDpEp * 32, smd, s>>>(w.ew, w.ewt, N, p.n_min, p.n_max, p.ctx_start, w.dpF,
