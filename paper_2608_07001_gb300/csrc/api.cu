@@ -211,7 +211,7 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
               dalloc(x, &w.kappa, (size_t)p.T) && dalloc(x, &w.bscore, (size_t)p.T) &&
               dalloc(x, &w.zbuf, (size_t)p.T) && dalloc(x, &w.p2, (size_t)Nc + 1) &&
               dalloc(x, &w.ew, (size_t)(Nc + 1) * ((nb + 3) & ~3)) && dalloc(x, &w.ewt, (size_t)p.n_max + 1) &&
-              dalloc(x, &w.dpF, (size_t)Nc + 1) && dalloc(x, &w.slots, (size_t)Nc + 2) &&
+              dalloc(x, &w.slots, (size_t)Nc + 2) &&
               dalloc(x, &w.dev_int, 16) &&
               dalloc(x, &w.row_m, (size_t)nrow) && dalloc(x, &w.row_Z, (size_t)nrow) &&
               dalloc(x, &w.row_ZC, (size_t)nrow) && dalloc(x, &w.rowp, (size_t)3 * nrow * c.n_chunks) &&

@@ -33,7 +33,6 @@ struct Workspace {
     double *p2 = nullptr;          // [N_c + 1] prefix of sum_l ||d_t||^2
     float *ew = nullptr;           // [(N_c + 1) * nbp] DP edge weights (len n_min..n_max), rows padded to 4
     float2 *ewt = nullptr;         // [n_max + 1] terminal edge weights (len 1..n_max) at i = N_c
-    double *dpF = nullptr;         // [N_c + 1] DP values
     int32_t *slots = nullptr;      // [N_c + 2] slot starts (absolute)
     int32_t *dev_int = nullptr;    // [8] small device scalars (J, status, ...)
     unsigned long long *sel_state = nullptr;   // radix-select state for the median

@@ -703,7 +703,7 @@ __device__ __forceinline__ bool better(df2 v, int a, df2 bv, int ba) {
 }
 
 __global__ void __launch_bounds__(kDpEp * 32) seg_dp_kernel(const float *ew, const float2 *ewt, int N,
-                                                            int n_min, int n_max, int cs, double *Fout,
+                                                            int n_min, int n_max, int cs,
                                                             int32_t *slots, int *dev_int) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int nb = n_max - n_min + 1, nbp = dp_row(nb);
@@ -715,7 +715,6 @@ __global__ void __launch_bounds__(kDpEp * 32) seg_dp_kernel(const float *ew, con
     const df2 NEG = df2{-INFINITY, 0.f};
     if (tid == 0) {
         ring[0] = df2{0.f, 0.f};
-        Fout[0] = 0.0;
         lenarr[0] = 0;
     }
     float *mybuf = wbuf + (size_t)k * kDpPD * nbp;
@@ -736,20 +735,25 @@ __global__ void __launch_bounds__(kDpEp * 32) seg_dp_kernel(const float *ew, con
         cp_async_wait<kDpPD - 1>();   // this step's row (the oldest group) has landed
         __syncwarp();
         const float *wr = mybuf + (size_t)q * nbp;
-        df2 best = NEG;
-        int ba = 0x7fffffff;
-        if (act) {
+        // the lane's candidates are independent: form them all, then keep the best
+        df2 v[kDpLen];
+        int av[kDpLen];
 #pragma unroll
-            for (int j = 0; j < kDpLen; j++) {
-                const int len = n_min + lane + 32 * j;
-                const int a = i - len;
-                if (len > n_max || a < 0) break;
-                const df2 fa = ring[a % kDpRing];
-                if (fa.hi == -INFINITY) continue;
-                const df2 v = df_add(fa, make_float2(wr[len - n_min], 0.f));
-                if (better(v, a, best, ba)) { best = v; ba = a; }
-            }
+        for (int j = 0; j < kDpLen; j++) {
+            const int len = n_min + lane + 32 * j;
+            const int a = i - len;
+            const bool ok = act && len <= n_max && a >= 0;
+            const df2 fa = ring[ok ? (a & (kDpRing - 1)) : 0];
+            const float w = wr[ok ? len - n_min : 0];
+            const bool live = ok && fa.hi != -INFINITY;
+            v[j] = live ? df_add(fa, make_float2(w, 0.f)) : NEG;
+            av[j] = live ? a : 0x7fffffff;
         }
+        df2 best = v[0];
+        int ba = av[0];
+#pragma unroll
+        for (int j = 1; j < kDpLen; j++)
+            if (better(v[j], av[j], best, ba)) { best = v[j]; ba = av[j]; }
         __syncwarp();
         fetch(i0 + kDpPD * step + k, q);   // reuse the stage for kDpPD steps ahead
         q = q + 1 == kDpPD ? 0 : q + 1;
@@ -763,7 +767,6 @@ __global__ void __launch_bounds__(kDpEp * 32) seg_dp_kernel(const float *ew, con
         }
         if (lane == 0 && act) {
             ring[i % kDpRing] = best;
-            Fout[i] = (double)best.hi + (double)best.lo;
             lenarr[i] = best.hi == -INFINITY ? 0 : (uint8_t)(i - ba);
         }
         __syncthreads();
@@ -782,7 +785,6 @@ __global__ void __launch_bounds__(kDpEp * 32) seg_dp_kernel(const float *ew, con
             df2 v = df_add(fa, ewt[len]);
             if (better(v, a, best, ba)) { best = v; ba = a; }
         }
-        Fout[N] = (double)best.hi + (double)best.lo;
         lenarr[N] = best.hi == -INFINITY ? 0 : (uint8_t)(N - ba);
     }
     if (tid == 0) {
@@ -896,8 +898,8 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
     const size_t smd = dp_smem(N, nb);
     if (smd > 227 * 1024 || nb > 32 * kDpLen) return cudaErrorInvalidConfiguration;
     cudaFuncSetAttribute(seg_dp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smd);
-    seg_dp_kernel<<<1, kDpEp * 32, smd, s>>>(w.ew, w.ewt, N, p.n_min, p.n_max, p.ctx_start, w.dpF,
-                                       w.slots, w.dev_int);
+    seg_dp_kernel<<<1, kDpEp * 32, smd, s>>>(w.ew, w.ewt, N, p.n_min, p.n_max, p.ctx_start,
+                                             w.slots, w.dev_int);
     c.launches += 8 + (surprisal ? 2 : 0) + (N > 1 ? 1 : 0);
     return cudaGetLastError();
 }
