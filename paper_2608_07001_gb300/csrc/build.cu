@@ -790,20 +790,24 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             __syncthreads();
             for (int bi = 0; bi < nb; bi++) scan(sm.bn[bi], std::true_type());
             __syncthreads();
-            // ---- per-candidate D and drop mass (thread per candidate) ------------
-            for (int k = tid; k < 2 * kNCD; k += kNT) {
-                double d = 0.0, pp = 0.0;
-#pragma unroll
-                for (int w = 0; w < NWARPS; w++) { d += sm.redD[k][w]; pp += sm.redP[k][w]; }
-                sm.candD[k] = d / A.W;
-                sm.candP[k] = pp / A.W;
-            }
-            __syncthreads();
-            // ---- phase D1: decisions (warp per node) ------------------------------
+            // ---- phase D1: candidate sums and decisions (warp per node) -------------
             for (int bi = warp; bi < nb; bi += NWARPS) {
                 BatchNode &B = sm.bn[bi];
                 NodeS &nd = sm.nodes[B.node];
                 const int a = nd.a, b = nd.b, nv = b - a;
+                // D and drop mass of this node's candidates: mean over the W probes
+                // of the per-warp partial sums
+                const double invW = 1.0 / A.W;
+                for (int k = lane; k < 2 * kNCD; k += 32) {
+                    const bool mine = k < kNCD ? (k >= B.pre_b && k < B.pre_e) : (k >= B.suf_b && k < B.suf_e);
+                    if (!mine) continue;
+                    double d = 0.0, pw = 0.0;
+#pragma unroll
+                    for (int w = 0; w < NWARPS; w++) { d += sm.redD[k][w]; pw += sm.redP[k][w]; }
+                    sm.candD[k] = d * invW;
+                    sm.candP[k] = pw * invW;
+                }
+                __syncwarp();
                 if (B.whole >= 0 && lane == 0) {   // root: D, Ddrop, Add gain (Eq. app_operation_gains)
                     const double Pd = sm.candP[B.whole];
                     const double D = nv >= 2 ? sm.candD[B.whole] : 0.0;
@@ -829,14 +833,14 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 }
                 const double DI = nd.D;
                 // binary cut: lane q evaluates cut q; max G_bin, ties -> smallest xi
+                const double krange = B.kmax > B.kmin ? 1.0 / (B.kmax - B.kmin) : 0.0;
                 double best = -INFINITY;
                 int bq = 0x7fffffff;
                 if (lane < B.ncut) {
                     const int xi = B.cut[lane];
                     const double DL = B.pidx[lane] >= 0 ? sm.candD[B.pidx[lane]] : 0.0;
                     const double DR = B.sidx[lane] >= 0 ? sm.candD[B.sidx[lane]] : 0.0;
-                    const double kh = B.kmax > B.kmin
-                                          ? (okey_inv(sm.kap[xi - 1]) - B.kmin) / (B.kmax - B.kmin) : 0.0;
+                    const double kh = (okey_inv(sm.kap[xi - 1]) - B.kmin) * krange;
                     best = ((DI - DL) - DR) + A.lam_kappa * kh;
                     bq = lane;
                 }
@@ -868,7 +872,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     bL = B.pidx[0] >= 0 ? sm.candD[B.pidx[0]] : 0.0;
                     bR = B.sidx[0] >= 0 ? sm.candD[B.sidx[0]] : 0.0;
                 }
-                const double rho_ext = gext / (ne - 1);
+                const double rho_ext = ne == 3 ? 0.5 * gext : gext;   // G_ext / (|children| - 1), exact
                 if (rho_ext > best) {
                     B.nchild = ne;
                     for (int q = 0; q < ne; q++) { B.ca[q] = ea[q]; B.cb[q] = eb[q]; B.cD[q] = eD[q]; }
@@ -879,66 +883,69 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 }
             }
             __syncthreads();
-            // ---- child numbering (deterministic, creation order) ----------------
-            if (tid == 0) {
-                int cnt = sm.nnodes;
-                for (int bi = 0; bi < nb; bi++) {
-                    BatchNode &B = sm.bn[bi];
-                    NodeS &nd = sm.nodes[B.node];
-                    nd.nchild = (signed char)B.nchild;
-                    nd.child0 = B.nchild ? (short)cnt : (short)-1;
-                    cnt += B.nchild;
-                }
-                sm.nnodes = cnt;
-            }
-            __syncthreads();
-            // ---- phase D2: children, gains, keys (warp per node) ----------------
+            // ---- phase D2: numbering, children, gains, keys (warp per node) --------
+            // Child indices are deterministic: the batch's nodes in order, after the
+            // nodes created before this batch.
             for (int bi = warp; bi < nb; bi += NWARPS) {
                 const BatchNode &B = sm.bn[bi];
                 NodeS &nd = sm.nodes[B.node];
                 const int64_t gv = nbase + B.node;
-                if (B.nchild == 0) {
+                int before = lane < bi ? sm.bn[lane].nchild : 0;
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) before += __shfl_xor_sync(0xffffffffu, before, o);
+                const int nch = B.nchild;
+                const int child0 = nch ? sm.nnodes + before : -1;
+                if (nch == 0) {
                     if (lane == 0) {
+                        nd.nchild = 0; nd.child0 = -1;
                         A.nd_child0[gv] = -1; A.nd_nchild[gv] = 0; A.nd_cost[gv] = 0;
                         A.nd_U[gv] = 0.f; A.nd_kappa[gv] = 0.f; A.nd_sel[gv] = 0;
                     }
                     continue;
                 }
-                double dsum = 0.0, rch[3], rnode = 0.0;   // R of the node = sum over its children
-                for (int q = 0; q < B.nchild; q++) {
+                double rch[3] = {0.0, 0.0, 0.0};
+                for (int q = 0; q < nch; q++) {
                     double r = 0.0;
                     for (int t = B.ca[q] + lane; t < B.cb[q]; t += 32) r += sm.Rt[t];
                     rch[q] = warp_sum(r);
-                    rnode += rch[q];
-                    dsum += B.cD[q];
                 }
+                const double rnode = (rch[0] + rch[1]) + rch[2];   // R of the node = sum over its children
+                const double dsum = (B.cD[0] + B.cD[1]) + (nch == 3 ? B.cD[2] : 0.0);
+                const int cost = nch - 1;
+                double gain = (double)om * rnode * (nd.D - dsum);
+                if (gain < 0.0) gain = 0.0;
+                const float U = (float)(gain / cost);
+                const float kap = fminf(U, nd.kin);
                 if (lane == 0) {
-                    const int cost = B.nchild - 1;
-                    double gain = (double)om * rnode * (nd.D - dsum);
-                    if (gain < 0.0) gain = 0.0;
-                    float U = (float)(gain / cost);
-                    float kap = fminf(U, nd.kin);
-                    A.nd_child0[gv] = nd.child0; A.nd_nchild[gv] = (int8_t)B.nchild;
+                    nd.nchild = (signed char)nch;
+                    nd.child0 = (short)child0;
+                    A.nd_child0[gv] = child0; A.nd_nchild[gv] = (int8_t)nch;
                     A.nd_cost[gv] = (int8_t)cost; A.nd_U[gv] = U; A.nd_kappa[gv] = kap;
                     A.nd_sel[gv] = 0;
-                    int nxt = cur ^ 1;
-                    for (int q = 0; q < B.nchild; q++) {
-                        int ci = nd.child0 + q;
-                        NodeS &ch = sm.nodes[ci];
-                        ch.a = (short)B.ca[q]; ch.b = (short)B.cb[q]; ch.parent = (short)B.node;
-                        ch.child0 = -1; ch.nchild = 0; ch.D = B.cD[q]; ch.kin = kap;
-                        const int64_t gc = nbase + ci;
-                        A.nd_a[gc] = sa + ch.a; A.nd_b[gc] = sa + ch.b;
-                        A.nd_parent[gc] = (int32_t)gv; A.nd_unit[gc] = (int32_t)uid;
-                        A.nd_D[gc] = ch.D; A.nd_R[gc] = (float)rch[q];
-                        A.nd_child0[gc] = -1; A.nd_nchild[gc] = 0; A.nd_cost[gc] = 0;
-                        A.nd_U[gc] = 0.f; A.nd_kappa[gc] = 0.f; A.nd_sel[gc] = 0;
-                        if (ch.b - ch.a >= 2) {
-                            int pos = atomicAdd(&sm.nlvl[nxt], 1);
-                            sm.lvl[nxt][pos] = (short)ci;
-                        }
+                }
+                if (lane < nch) {   // lane q writes child q
+                    const int q = lane, ci = child0 + q;
+                    const double rq = q == 0 ? rch[0] : (q == 1 ? rch[1] : rch[2]);
+                    NodeS &ch = sm.nodes[ci];
+                    ch.a = (short)B.ca[q]; ch.b = (short)B.cb[q]; ch.parent = (short)B.node;
+                    ch.child0 = -1; ch.nchild = 0; ch.D = B.cD[q]; ch.kin = kap;
+                    const int64_t gc = nbase + ci;
+                    A.nd_a[gc] = sa + B.ca[q]; A.nd_b[gc] = sa + B.cb[q];
+                    A.nd_parent[gc] = (int32_t)gv; A.nd_unit[gc] = (int32_t)uid;
+                    A.nd_D[gc] = B.cD[q]; A.nd_R[gc] = (float)rq;
+                    A.nd_child0[gc] = -1; A.nd_nchild[gc] = 0; A.nd_cost[gc] = 0;
+                    A.nd_U[gc] = 0.f; A.nd_kappa[gc] = 0.f; A.nd_sel[gc] = 0;
+                    if (B.cb[q] - B.ca[q] >= 2) {
+                        const int pos = atomicAdd(&sm.nlvl[cur ^ 1], 1);
+                        sm.lvl[cur ^ 1][pos] = (short)ci;
                     }
                 }
+            }
+            __syncthreads();
+            if (tid == 0) {   // nodes created by this batch (read by the next batch's D2)
+                int total = 0;
+                for (int bi = 0; bi < nb; bi++) total += sm.bn[bi].nchild;
+                sm.nnodes += total;
             }
             __syncthreads();
         }
