@@ -74,22 +74,27 @@ __global__ void alloc_hist_kernel(AllocArgs A, int shift, int nbits, uint32_t ma
     __syncthreads();
     const uint32_t prefix = (uint32_t)A.st[ST_PREFIX];
     const int64_t n = A.n_units + A.n_nodes;
-    unsigned long long tot = 0;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
-         i += (int64_t)gridDim.x * blockDim.x) {
-        uint32_t key;
-        int cost;
-        if (!op_key(A, i, key, cost)) continue;
-        tot += cost;
-        if ((key & mask) != prefix) continue;
-        atomicAdd(&sh[(key >> shift) & (nbin - 1)], (unsigned)cost);
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    unsigned int tot = 0;
+    // whole warps iterate together so that equal bins can be combined first
+    // (keys cluster in few bins: one shared atomic per distinct bin and warp)
+    for (int64_t i0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); i0 < n; i0 += stride) {
+        const int64_t i = i0 + (threadIdx.x & 31);
+        uint32_t key = 0;
+        int cost = 0;
+        const bool op = i < n && op_key(A, i, key, cost);
+        tot += op ? cost : 0;
+        const int bin = op && (key & mask) == prefix ? (int)((key >> shift) & (nbin - 1)) : -1;
+        const unsigned grp = __match_any_sync(0xffffffffu, bin);
+        const unsigned sum = __reduce_add_sync(grp, (unsigned)cost);
+        if (bin >= 0 && (threadIdx.x & 31) == __ffs(grp) - 1) atomicAdd(&sh[bin], sum);
     }
     __syncthreads();
     for (int b = threadIdx.x; b < nbin; b += blockDim.x)
         if (sh[b]) atomicAdd(&A.hist[b], (unsigned long long)sh[b]);
     if (shift == 21) {   // first pass: total cost of all ops
-        tot = (unsigned long long)warp_sum((double)tot);
-        if ((threadIdx.x & 31) == 0 && tot) atomicAdd(&A.st[ST_TOTAL], tot);
+        tot = __reduce_add_sync(0xffffffffu, tot);
+        if ((threadIdx.x & 31) == 0 && tot) atomicAdd(&A.st[ST_TOTAL], (unsigned long long)tot);
     }
 }
 
