@@ -378,7 +378,7 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
         memcpy(&tau, &bits, sizeof tau);
         if (h.all) tau = -INFINITY;
         // everything built so far fits: nothing can be pruned yet, go deeper at once
-        const int levels = h.all ? 4 * gkv::kMaxUnit : 2;
+        const int levels = h.all ? 4 * gkv::kMaxUnit : 1;
         gkv::StageTimer tm(c, 3, s);
         e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 1, levels, tau, w.u_list, h.count[0],
                                    w.u_list + (nu - h.count[1]), h.count[1], s);
