@@ -364,17 +364,75 @@ int grid_for(const Ctx &c, int64_t n) {
 // Units with a pending node whose creator key is >= tau (all of them when
 // every op built so far fits the budget).
 __global__ void prune_list_kernel(const float *u_pend, const int32_t *slots, int J, int64_t n_units,
-                                  const unsigned long long *st, int32_t *list, int *count) {
+                                  const unsigned long long *st, const float *cut, int32_t *list,
+                                  int *count, unsigned long long *potential) {
     int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= n_units) return;
     float p = u_pend[i];
     if (!(p >= 0.f)) return;   // -1: no pending node
     const bool all = st[ST_ALL] != 0;
-    if (all || __float_as_uint(p) >= (uint32_t)st[ST_PREFIX]) {
+    const bool above = all || __float_as_uint(p) >= (uint32_t)st[ST_PREFIX];
+    if (above) {   // cost of expanding the unit completely: n - 1 entries at most
+        const int j = (int)(i % J);
+        atomicAdd(potential, (unsigned long long)(slots[j + 1] - slots[j] - 1));
+    }
+    if (above && p >= *cut) {
         const int j = (int)(i % J);
         if (slots[j + 1] - slots[j] <= kShortUnit) list[atomicAdd(count, 1)] = (int32_t)i;
         else list[n_units - 1 - atomicAdd(count + 1, 1)] = (int32_t)i;
     }
+}
+
+// Histogram (top 16 bits of the non-negative float keys) of the largest
+// pending key bound of every unit that reaches the threshold.
+constexpr int kPendBins = 1 << 16;
+__global__ void pend_hist_kernel(const float *u_pend, int64_t n_units, const unsigned long long *st,
+                                 unsigned int *hist) {
+    int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= n_units) return;
+    const float p = u_pend[i];
+    if (!(p >= 0.f)) return;
+    const bool all = st[ST_ALL] != 0;
+    if (all || __float_as_uint(p) >= (uint32_t)st[ST_PREFIX]) atomicAdd(&hist[__float_as_uint(p) >> 16], 1u);
+}
+
+// One block of 1024 threads: thread t owns the 64 bins below kPendBins - 64 t;
+// the bin where the count of larger-or-equal bounds first reaches m gives the cut.
+__global__ void __launch_bounds__(1024) pend_cut_kernel(const unsigned int *hist, int m, float *cut,
+                                                        unsigned int *n_qual) {
+    __shared__ unsigned int wsum[32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int hi = kPendBins - 64 * tid;   // bins [hi - 64, hi), descending
+    unsigned int own = 0;
+    for (int b = hi - 1; b >= hi - 64; b--) own += hist[b];
+    unsigned int incl = own;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const unsigned int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        unsigned int w = wsum[lane], wi = w;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const unsigned int y = __shfl_up_sync(0xffffffffu, wi, o);
+            if (lane >= o) wi += y;
+        }
+        wsum[lane] = wi - w;   // exclusive over warps
+    }
+    __syncthreads();
+    const unsigned int before = wsum[warp] + incl - own;   // bounds in bins >= hi
+    if (tid == 1023) *n_qual = before + own;
+    if (before < (unsigned)m && before + own >= (unsigned)m) {
+        unsigned int acc = before;
+        for (int b = hi - 1; b >= hi - 64; b--) {
+            acc += hist[b];
+            if (acc >= (unsigned)m) { *cut = __uint_as_float((unsigned)b << 16); break; }
+        }
+    }
+    if (tid == 1023 && before + own < (unsigned)m) *cut = -INFINITY;   // fewer than m qualify: no cut
 }
 
 __global__ void slot_classes_kernel(const int32_t *slots, int J, int32_t *list, int *count) {
@@ -406,10 +464,23 @@ cudaError_t launch_prune_list(Ctx &c, const int32_t *slots, int J, int32_t *list
                               cudaStream_t s) {
     const int64_t nu = (int64_t)c.p.L * c.p.G * J;
     cudaError_t e = cudaMemsetAsync(count, 0, 2 * sizeof(int), s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(c.w.pend_pot, 0, sizeof(unsigned long long), s);
     if (e != cudaSuccess) return e;
     prune_list_kernel<<<(unsigned)((nu + 255) / 256), 256, 0, s>>>(c.w.u_pend, slots, J, nu,
-                                                                    c.w.alloc_state, list, count);
+                                                                    c.w.alloc_state, c.w.pend_cut, list,
+                                                                    count, c.w.pend_pot);
     c.launches += 1;
+    return cudaGetLastError();
+}
+
+cudaError_t launch_pend_cut(Ctx &c, int J, int m, float *cut, unsigned int *n_qual, cudaStream_t s) {
+    const int64_t nu = (int64_t)c.p.L * c.p.G * J;
+    cudaError_t e = cudaMemsetAsync(c.w.pend_hist, 0, sizeof(unsigned int) * kPendBins, s);
+    if (e != cudaSuccess) return e;
+    pend_hist_kernel<<<(unsigned)((nu + 255) / 256), 256, 0, s>>>(c.w.u_pend, nu, c.w.alloc_state,
+                                                                   c.w.pend_hist);
+    pend_cut_kernel<<<1, 1024, 0, s>>>(c.w.pend_hist, m, cut, n_qual);
+    c.launches += 2;
     return cudaGetLastError();
 }
 

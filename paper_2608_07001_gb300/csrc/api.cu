@@ -222,7 +222,9 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
               dalloc(x, &w.nd_cost, (size_t)c.node_cap) && dalloc(x, &w.nd_D, (size_t)c.node_cap) &&
               dalloc(x, &w.nd_R, (size_t)c.node_cap) && dalloc(x, &w.nd_U, (size_t)c.node_cap) &&
               dalloc(x, &w.nd_kappa, (size_t)c.node_cap) && dalloc(x, &w.nd_sel, (size_t)c.node_cap) &&
-              dalloc(x, &w.hist, 2048) && dalloc(x, &w.alloc_state, 16) && dalloc(x, &w.work, 4);
+              dalloc(x, &w.hist, 2048) && dalloc(x, &w.alloc_state, 16) && dalloc(x, &w.work, 4) &&
+              dalloc(x, &w.pend_hist, 1 << 16) && dalloc(x, &w.pend_cut, 1) && dalloc(x, &w.pend_n, 1) &&
+              dalloc(x, &w.pend_pot, 1);
     if (!ok) {
         gracekv_destroy(x);
         return GKV_ENOMEM;
@@ -341,9 +343,22 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
         gkv::StageTimer tm(c, 2, s);
         e = gkv::launch_token_values(c, K, Q, s);
     }
-    // Trees: roots and their splits for every unit, then pruned resumption
-    // (see build.cu): only pending nodes whose creator key reaches the
-    // threshold of the ops built so far are evaluated.
+    // Trees (build.cu).  Every op's key is bounded before it is built: a pending
+    // node's split key is at most min(creator key, omega R D).  Each pass derives
+    // the threshold tau of the ops built so far (a lower bound of the final one)
+    // and expands one level of the pending nodes whose bound reaches it, until
+    // none does; nodes left pending can never be selected.  When the budget is
+    // smaller than the number of units, the first launch evaluates only the
+    // roots' own distortion (their Add ops) and later passes expand the units
+    // with the largest bounds first, about 32768 at a time, so that tau rises
+    // before weaker units are considered; otherwise it evaluates every root's
+    // split at once.  When the budget left provably covers the complete
+    // expansion of every unit that reaches tau, those trees are built to the end.
+    const bool root_only = c.B_free < nu;
+    const int pass_units = 32768;
+    static const float kNoCut = -INFINITY;
+    if (e == cudaSuccess && !root_only)
+        e = cudaMemcpyAsync(w.pend_cut, &kNoCut, sizeof(float), cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = cudaMemsetAsync(w.work, 0, 4 * sizeof(unsigned long long), s);
     if (e == cudaSuccess) {
         int cnt[2] = {0, 0};
@@ -355,15 +370,21 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
         if (e == cudaSuccess) e = cudaStreamSynchronize(s);
         if (e == cudaSuccess) {
             gkv::StageTimer tm(c, 3, s);
-            e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 0, 1, 0.f, w.u_list, cnt[0],
+            e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 0, root_only ? 1 : 0, 1, 0.f, w.u_list, cnt[0],
                                        w.u_list + (J - cnt[1]), cnt[1], s);
         }
     }
     for (int it = 0; e == cudaSuccess; it++) {
-        struct { int count[2]; unsigned long long prefix, all; } h = {{0, 0}, 0, 0};
+        struct {
+            int count[2];
+            unsigned long long prefix, all, total, pot;
+            float cut;
+            unsigned int nqual;
+        } h = {{0, 0}, 0, 0, 0, 0, 0.f, 0};
         {
             gkv::StageTimer tm(c, 3, s);
             e = gkv::launch_threshold(c, J, s);
+            if (e == cudaSuccess && root_only) e = gkv::launch_pend_cut(c, J, pass_units, w.pend_cut, w.pend_n, s);
             if (e == cudaSuccess) e = gkv::launch_prune_list(c, w.slots, J, w.u_list, w.dev_int + 2, s);
         }
         if (e == cudaSuccess) e = cudaMemcpyAsync(h.count, w.dev_int + 2, 2 * sizeof(int), cudaMemcpyDeviceToHost, s);
@@ -371,17 +392,25 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
                                                   cudaMemcpyDeviceToHost, s);
         if (e == cudaSuccess) e = cudaMemcpyAsync(&h.all, w.alloc_state + 2, sizeof(unsigned long long),
                                                   cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(&h.cut, w.pend_cut, sizeof(float), cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(&h.nqual, w.pend_n, sizeof(unsigned int), cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(&h.total, w.alloc_state + 6, sizeof(unsigned long long),
+                                                  cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(&h.pot, w.pend_pot, sizeof(unsigned long long),
+                                                  cudaMemcpyDeviceToHost, s);
         if (e == cudaSuccess) e = cudaStreamSynchronize(s);
         if (e != cudaSuccess || h.count[0] + h.count[1] == 0) break;
         uint32_t bits = (uint32_t)h.prefix;
         float tau;
         memcpy(&tau, &bits, sizeof tau);
         if (h.all) tau = -INFINITY;
-        // everything built so far fits: nothing can be pruned yet, go deeper at once
-        const int levels = h.all ? 4 * gkv::kMaxUnit : 1;
+        const float tau_eff = fmaxf(tau, h.cut);
+        // everything built so far fits and few units remain: expand them fully at once
+        const bool fits = h.all && (long long)c.B_free - (long long)h.total >= (long long)h.pot;
+        const int levels = fits ? 4 * gkv::kMaxUnit : 1;
         gkv::StageTimer tm(c, 3, s);
-        e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 1, levels, tau, w.u_list, h.count[0],
-                                   w.u_list + (nu - h.count[1]), h.count[1], s);
+        e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 1, 0, levels, tau_eff, w.u_list,
+                                   h.count[0], w.u_list + (nu - h.count[1]), h.count[1], s);
         c.build_passes = it + 2;
     }
     if (e != cudaSuccess) return cuda_fail(x, e, "build_trees launch");

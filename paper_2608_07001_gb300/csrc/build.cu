@@ -64,8 +64,9 @@ struct BuildArgs {
     double lam_kappa, base_frac;
     // work list: fresh launches index (slot list entry, lg), resume launches units
     int resume;                  // 0: build from the root, 1: resume pending nodes
+    int root_only;               // fresh: evaluate only the root's own distortion (split stays pending)
     int max_levels;              // levels evaluated by this launch
-    float tau;                   // resume: evaluate pending nodes whose creator key >= tau
+    float tau;                   // resume: evaluate pending nodes whose key bound >= tau
     const int32_t *list;         // fresh: slot indices; resume: unit ids
     // outputs
     int32_t *nd_a, *nd_b, *nd_child0, *nd_parent, *nd_unit;
@@ -106,6 +107,15 @@ struct Cand {
     int a, b;        // local interval (a == b: unused entry)
     float meff;
 };
+
+// Upper bound of a split's utility: U = omega R (D - sum D_children) / cost
+// <= omega R D, since every D >= 0 and cost >= 1 (Eqs. app_operation_gains,
+// app_unit_utility).  Rounded up, so that fp32 rounding never makes a bound
+// fall below the utility it bounds.
+__device__ __forceinline__ float key_bound(double x) {
+    const float f = (float)x;
+    return f + fabsf(f) * 1e-6f;
+}
 
 // Order-preserving 64-bit key of a double (larger value -> larger key), so
 // that curvature ranks compare exactly like the fp64 values with integer ops.
@@ -414,6 +424,8 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         }
     } else {
         const int nn = A.u_nnodes[uid];
+        float *bnd_stage = &sm.redD[0][0];   // scratch until the first evaluation
+        static_assert(sizeof(sm.redD) >= sizeof(float) * S::MAXNODES, "bound staging");
         for (int k = tid; k < nn; k += kNT) {
             const int64_t v = nbase + k;
             NodeS &nd = sm.nodes[k];
@@ -425,15 +437,15 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             nd.nchild = A.nd_nchild[v];
             nd.D = A.nd_D[v];
             nd.kin = pg < 0 ? A.u_Uadd[uid] : A.nd_kappa[pg];
+            bnd_stage[k] = nd.nchild == -1 ? A.nd_U[v] : -1.f;   // key bound of a pending node
         }
         if (tid == 0) { sm.nnodes = nn; sm.nlvl[0] = 0; sm.pend = -1.f; }
         __syncthreads();
         if (tid == 0) {   // pending nodes that qualify, in creation order
             for (int k = 0; k < nn; k++) {
-                const NodeS &nd = sm.nodes[k];
-                if (nd.nchild != -1) continue;
-                if (nd.kin >= A.tau) sm.lvl[0][sm.nlvl[0]++] = (short)k;
-                else sm.pend = fmaxf(sm.pend, nd.kin);
+                if (sm.nodes[k].nchild != -1) continue;
+                if (bnd_stage[k] >= A.tau) sm.lvl[0][sm.nlvl[0]++] = (short)k;
+                else sm.pend = fmaxf(sm.pend, bnd_stage[k]);
             }
         }
     }
@@ -619,7 +631,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 for (int k = 0; k < nl; k++) {
                     const int v = sm.lvl[cur][k];
                     A.nd_nchild[nbase + v] = -1;
-                    pm = fmaxf(pm, sm.nodes[v].kin);
+                    pm = fmaxf(pm, A.nd_U[nbase + v]);   // the key bound written at its creation
                 }
                 sm.pend = pm;
             }
@@ -636,7 +648,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     const int v = sm.lvl[cur][k];
                     const int nv = sm.nodes[v].b - sm.nodes[v].a;
                     const bool root = v == 0 && !A.resume;
-                    const int nc = nv >= 3 ? min(A.k_cand + 1, nv - 1) + 1 : 0;
+                    const int nc = (nv >= 3 && !(root && A.root_only)) ? min(A.k_cand + 1, nv - 1) + 1 : 0;
                     const int bp = nc + (root ? 1 : 0), bs = nc;
                     if (upre + bp > kNCD || usuf + bs > kNCD) break;
                     sm.bn[nb].node = v;
@@ -661,13 +673,14 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 BatchNode &B = sm.bn[bi];
                 const int v = B.node;
                 const int a = sm.nodes[v].a, b = sm.nodes[v].b, nv = b - a;
+                const bool ronly = v == 0 && !A.resume && A.root_only;   // only the node's own distortion
                 // top-K by curvature over positions [a, b-2] (ties: lower t)
                 unsigned sel[NMAX / 32];
                 unsigned long long kmin = ~0ull, kmax = 0ull;
 #pragma unroll
                 for (int w = 0; w < NMAX / 32; w++) {
                     int t = a + w * 32 + lane;
-                    bool in = t <= b - 2;
+                    bool in = !ronly && t <= b - 2;
                     bool s = false;
                     if (in) {
                         const unsigned long long kt = sm.kap[t];
@@ -708,7 +721,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 // side [p*+1, b) in descending start.  A side equal to a cut's
                 // interval shares its candidate.
                 const unsigned FULL = 0xffffffffu;
-                const bool cands = nv >= 3;
+                const bool cands = nv >= 3 && !ronly;
                 const int maxc = cands ? min(A.k_cand + 1, nv - 1) : 0;
                 int ncut = 0;
 #pragma unroll
@@ -820,6 +833,10 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     A.nd_D[nbase] = D;
                 }
                 __syncwarp();
+                if (A.root_only && B.whole >= 0 && nv >= 2) {   // its split is decided later
+                    if (lane == 0) B.nchild = -1;
+                    continue;
+                }
                 if (nv < 3) {
                     if (lane == 0) {
                         B.nchild = 0;
@@ -890,10 +907,20 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 const BatchNode &B = sm.bn[bi];
                 NodeS &nd = sm.nodes[B.node];
                 const int64_t gv = nbase + B.node;
-                int before = lane < bi ? sm.bn[lane].nchild : 0;
+                int before = lane < bi ? max(sm.bn[lane].nchild, 0) : 0;
 #pragma unroll
                 for (int o = 16; o > 0; o >>= 1) before += __shfl_xor_sync(0xffffffffu, before, o);
                 const int nch = B.nchild;
+                if (nch < 0) {   // pending root: its split key is at most min(U_add, omega R D)
+                    if (lane == 0) {
+                        const float bnd = fminf(nd.kin, key_bound((double)om * sm.rootR * nd.D));
+                        nd.nchild = -1; nd.child0 = -1;
+                        A.nd_child0[gv] = -1; A.nd_nchild[gv] = -1; A.nd_cost[gv] = 0;
+                        A.nd_U[gv] = bnd; A.nd_kappa[gv] = 0.f; A.nd_sel[gv] = 0;
+                        atomicMax(reinterpret_cast<int *>(&sm.pend), __float_as_int(bnd));
+                    }
+                    continue;
+                }
                 const int child0 = nch ? sm.nnodes + before : -1;
                 if (nch == 0) {
                     if (lane == 0) {
@@ -934,7 +961,9 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     A.nd_parent[gc] = (int32_t)gv; A.nd_unit[gc] = (int32_t)uid;
                     A.nd_D[gc] = B.cD[q]; A.nd_R[gc] = (float)rq;
                     A.nd_child0[gc] = -1; A.nd_nchild[gc] = 0; A.nd_cost[gc] = 0;
-                    A.nd_U[gc] = 0.f; A.nd_kappa[gc] = 0.f; A.nd_sel[gc] = 0;
+                    // until the child is evaluated, nd_U holds the bound of its split key
+                    A.nd_U[gc] = B.cb[q] - B.ca[q] >= 2 ? fminf(kap, key_bound((double)om * rq * B.cD[q])) : 0.f;
+                    A.nd_kappa[gc] = 0.f; A.nd_sel[gc] = 0;
                     if (B.cb[q] - B.ca[q] >= 2) {
                         const int pos = atomicAdd(&sm.nlvl[cur ^ 1], 1);
                         sm.lvl[cur ^ 1][pos] = (short)ci;
@@ -944,7 +973,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             __syncthreads();
             if (tid == 0) {   // nodes created by this batch (read by the next batch's D2)
                 int total = 0;
-                for (int bi = 0; bi < nb; bi++) total += sm.bn[bi].nchild;
+                for (int bi = 0; bi < nb; bi++) total += max(sm.bn[bi].nchild, 0);
                 sm.nnodes += total;
             }
             __syncthreads();
@@ -1004,7 +1033,7 @@ cudaError_t launch_dt(Ctx &c, BuildArgs &A, unsigned grid, cudaStream_t s) {
 
 cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *Q,
                               const float *omega, const int32_t *slots, int J, int resume,
-                              int max_levels, float tau, const int32_t *list_short, int n_short,
+                              int root_only, int max_levels, float tau, const int32_t *list_short, int n_short,
                               const int32_t *list_long, int n_long, cudaStream_t s) {
     const gkv_params &p = c.p;
     BuildArgs A;
@@ -1016,7 +1045,7 @@ cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *
     A.inv_sqrt_d = (float)(1.0 / sqrt((double)p.d));
     A.lamZ = (float)p.lambda_Z; A.lamM = (float)p.lambda_M; A.eps = (float)p.eps;
     A.lam_kappa = p.lambda_kappa; A.base_frac = p.base_frac;
-    A.resume = resume; A.max_levels = max_levels; A.tau = tau;
+    A.resume = resume; A.root_only = root_only; A.max_levels = max_levels; A.tau = tau;
     A.nd_a = c.w.nd_a; A.nd_b = c.w.nd_b; A.nd_child0 = c.w.nd_child0;
     A.nd_parent = c.w.nd_parent; A.nd_unit = c.w.nd_unit;
     A.nd_nchild = c.w.nd_nchild; A.nd_cost = c.w.nd_cost;

@@ -53,7 +53,7 @@ struct Workspace {
     int64_t units_cap = 0;
     int32_t *u_nnodes = nullptr;
     float *u_Uadd = nullptr, *u_Ddrop = nullptr;
-    float *u_pend = nullptr;       // largest creator key of the unit's pending nodes (-1: none)
+    float *u_pend = nullptr;       // largest key bound of the unit's pending nodes (-1: none)
     uint8_t *u_sel = nullptr;      // Add selected (1), discarded tie (2)
     int32_t *u_count = nullptr;    // frontier entries per unit
     int64_t *u_off = nullptr;      // entry offset of each unit's frontier
@@ -64,6 +64,11 @@ struct Workspace {
     unsigned long long *hist = nullptr;        // [2048] cost-weighted histogram
     unsigned long long *alloc_state = nullptr; // see alloc.cu
     unsigned long long *work = nullptr;        // [4] tree-building work counters
+    // bound-ordered expansion of pending nodes
+    unsigned int *pend_hist = nullptr;         // [65536] units per bound bin
+    float *pend_cut = nullptr;                 // [1] lower bound of the next pass
+    unsigned int *pend_n = nullptr;            // [1] units that reach the threshold
+    unsigned long long *pend_pot = nullptr;    // [1] entries a full expansion of those units could take
 };
 
 struct Ctx {
@@ -221,19 +226,26 @@ cudaError_t launch_token_values(Ctx &c, const void *K, const void *Q, cudaStream
 constexpr int kShortUnit = 64;
 cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *Q,
                               const float *omega, const int32_t *slots, int J, int resume,
-                              int max_levels, float tau, const int32_t *list_short, int n_short,
-                              const int32_t *list_long, int n_long, cudaStream_t s);
+                              int root_only, int max_levels, float tau, const int32_t *list_short,
+                              int n_short, const int32_t *list_long, int n_long, cudaStream_t s);
 // Slot indices split by length class: short ones at list[0, count[0]), long
 // ones at list[J - count[1], J).
 cudaError_t launch_slot_classes(Ctx &c, const int32_t *slots, int J, int32_t *list, int *count,
                                 cudaStream_t s);
 // Allocation threshold tau over the ops built so far (alloc_state prefix /
-// all-fit flag), and the units whose pending nodes qualify (key >= tau),
-// split by slot length class: short units at list[0, count[0]), long units at
-// list[n_units - count[1], n_units).
+// all-fit flag), and the units whose largest pending key bound reaches
+// max(tau, cut), split by slot length class: short units at list[0, count[0]),
+// long units at list[n_units - count[1], n_units); *pend_pot receives the
+// entries a complete expansion of every unit reaching tau could take.
 cudaError_t launch_threshold(Ctx &c, int J, cudaStream_t s);
 cudaError_t launch_prune_list(Ctx &c, const int32_t *slots, int J, int32_t *list, int *count,
                               cudaStream_t s);
+// Bound-ordered expansion: among the units whose largest pending key bound
+// reaches the threshold, the cut that keeps about `m` of them (the lower edge
+// of the bin of the m-th largest bound; -inf when fewer qualify), written to
+// *cut, with the number that qualify at the threshold in *n_qual.  The prune
+// list then uses max(threshold, *cut).
+cudaError_t launch_pend_cut(Ctx &c, int J, int m, float *cut, unsigned int *n_qual, cudaStream_t s);
 
 cudaError_t launch_allocate(Ctx &c, int J, cudaStream_t s);
 cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *slots, int J,
