@@ -205,6 +205,8 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
     const int64_t nrow = (int64_t)p.L * p.Hq * p.W;
     gkv::Workspace &w = c.w;
     bool ok = dalloc(x, &w.rope, (size_t)p.T * (p.d / 2)) &&
+              dalloc(x, &w.rope_rel, (size_t)(2 * gkv::kMaxUnit - 1) * (p.d / 2)) &&
+              dalloc(x, &w.ent, (size_t)p.budget + (size_t)p.L * p.G * (p.T - Nc)) &&
               dalloc(x, &w.inv_norm, (size_t)c.nseg * p.T) &&
               dalloc(x, &w.nrm2, (size_t)c.nseg * p.T) &&
               dalloc(x, &w.klw, (size_t)c.nseg * c.nwin * p.T) &&

@@ -11,10 +11,14 @@
 // recomputed here from K, V and the token values.
 //
 // Kernels: gather_count (frontier entries per unit), gather_scan (one block,
-// ordered exclusive scan -> per-unit and per-(l, g) offsets), gather_units
-// (warp per unit, depth-first in ascending position), gather_tokens
-// (prefix / recent / suffix copies).
+// ordered exclusive scan -> per-unit and per-(l, g) offsets), gather_list
+// (warp per unit, depth-first in ascending position: entry descriptors by
+// output position), gather_emit (persistent warps, one entry at a time:
+// prototypes or single-token copies), gather_tokens (prefix / recent / suffix
+// copies).
 #include "gkv_internal.cuh"
+
+#include <algorithm>
 
 namespace gkv {
 namespace {
@@ -23,6 +27,8 @@ struct GatherArgs {
     const void *K, *V;
     const float *rtok;
     const float2 *rope;
+    const float2 *rope_rel;    // [2 kMaxUnit - 1][d/2]: rotation by the offset p - t
+    int4 *ent;                 // [entries]: (a, b, lg, 1) of every frontier entry, by output position
     const int32_t *slots;
     const int32_t *nd_a, *nd_b, *nd_child0;
     const int8_t *nd_nchild;
@@ -116,12 +122,16 @@ __device__ __forceinline__ void store8(float *dst, const float v[8]) {
 
 // One frontier node [a, b) of head lg -> cache entry e (one warp).  Rows are
 // read as 8-element chunks, LPR = d / 8 lanes per row and 32 / LPR rows per
-// step; the chunk holding elements i .. i+7 of the first half and the one
-// holding i + d/2 .. of the second half sit PX = LPR / 2 lanes apart, so the
-// rotation partner comes from a shuffle.  All arithmetic is fp32.
+// group, U groups in flight; the chunk holding elements i .. i+7 of the first
+// half and the one holding i + d/2 .. of the second half sit PX = LPR / 2
+// lanes apart, so the rotation partner comes from a shuffle.  The key
+// prototype RoPE(mean_t RoPE^-1(k_t, t), p) is formed as mean_t of k_t rotated
+// by p - t (rotations compose), from a table of the 2 n_max - 1 offsets; its
+// norm equals the norm of the mean inverse-rotated key.  The value prototype
+// uses sum_t (R_t + beta) v_t = sum R v + beta sum v.  All arithmetic is fp32.
 template <typename Tin, int DH>
 __device__ void emit_node(const GatherArgs &A, int lg, int a, int b, int64_t e, int lane) {
-    constexpr int HALF = DH / 2, LPR = DH / 8, RPW = 32 / LPR, PX = LPR / 2;
+    constexpr int HALF = DH / 2, LPR = DH / 8, RPW = 32 / LPR, PX = LPR / 2, U = 3;
     const int r = lane / LPR, c = lane - r * LPR;
     const bool hi = c >= PX;                   // chunk in the second half
     const int i0 = 8 * (c - (hi ? PX : 0));    // pair index of the chunk's first element
@@ -139,38 +149,27 @@ __device__ void emit_node(const GatherArgs &A, int lg, int a, int b, int64_t e, 
         return;
     }
     const float *R = A.rtok + (size_t)lg * A.Nc - A.cs;
-    float rs = 0.f;
-    for (int t = a + lane; t < b; t += 32) rs += R[t];
-    rs = warp_sum(rs);
-    const float ninv = 1.0f / (float)n;
-    const float beta = (float)A.base_frac * (rs * ninv);
-    const float winv = 1.0f / (rs + (float)n * beta + (float)A.eps);
-    float mk[8], mv[8], kn = 0.f;
+    const int p = round_half_even_mid(a, b);
+    float mk[8], sv[8], srv[8], kn = 0.f, rs = 0.f;
 #pragma unroll
-    for (int j = 0; j < 8; j++) mk[j] = mv[j] = 0.f;
-    constexpr int U = 2;   // row groups whose loads are issued together
+    for (int j = 0; j < 8; j++) mk[j] = sv[j] = srv[j] = 0.f;
     for (int t0 = a; t0 < b; t0 += U * RPW) {
         Vec8<Tin> kx[U], vx[U];
-        float4 cs[U][4];
-        float wt[U];
-        bool ok[U];
+        float rr[U];
+        int tt[U];
 #pragma unroll
-        for (int g = 0; g < U; g++) {
+        for (int g = 0; g < U; g++) {   // issue every group's loads first
             const int t = t0 + g * RPW + r;
-            ok[g] = t < b;
-            if (ok[g]) {
+            const bool ok = t < b;
+            tt[g] = ok ? t : b - 1;
+            if (ok) {
                 kx[g].load(K + (size_t)t * DH + 8 * c);
                 vx[g].load(V + (size_t)t * DH + 8 * c);
-                const float4 *cs4 = reinterpret_cast<const float4 *>(A.rope + (size_t)t * HALF + i0);
-#pragma unroll
-                for (int j2 = 0; j2 < 4; j2++) cs[g][j2] = cs4[j2];
-                wt[g] = R[t] + beta;
+                rr[g] = R[t];
             } else {
 #pragma unroll
                 for (int j = 0; j < 8; j++) kx[g].v[j] = vx[g].v[j] = 0.f;
-#pragma unroll
-                for (int j2 = 0; j2 < 4; j2++) cs[g][j2] = make_float4(0.f, 0.f, 0.f, 0.f);
-                wt[g] = 0.f;
+                rr[g] = 0.f;
             }
         }
 #pragma unroll
@@ -183,17 +182,21 @@ __device__ void emit_node(const GatherArgs &A, int lg, int a, int b, int64_t e, 
             }
 #pragma unroll
             for (int o = 1; o < LPR; o <<= 1) nn += __shfl_xor_sync(0xffffffffu, nn, o);
-            if (ok[g] && c == 0) kn += sqrtf(nn);   // |k_circ_t| = |k_t| (RoPE is a rotation)
+            if (c == 0) kn += sqrtf(nn);   // |k_t| (rows past b are zero)
+            rs += rr[g];
+            const float4 *cs4 = reinterpret_cast<const float4 *>(
+                A.rope_rel + (size_t)(p - tt[g] + kMaxUnit - 1) * HALF + i0);
 #pragma unroll
             for (int j2 = 0; j2 < 4; j2++) {
-                const float4 q = cs[g][j2];          // (cos, sin) of pairs i0 + 2 j2, i0 + 2 j2 + 1
+                const float4 q = cs4[j2];          // (cos, sin) of pairs i0 + 2 j2, i0 + 2 j2 + 1
                 const float cc[2] = {q.x, q.z}, sn[2] = {q.y, q.w};
 #pragma unroll
                 for (int h = 0; h < 2; h++) {
                     const int j = 2 * j2 + h;
-                    // RoPE^-1(k, t): x' = x cos + y sin, y' = y cos - x sin (rows past b add 0)
-                    mk[j] += hi ? fmaf(kx[g].v[j], cc[h], -y[j] * sn[h]) : fmaf(kx[g].v[j], cc[h], y[j] * sn[h]);
-                    mv[j] = fmaf(wt[g], vx[g].v[j], mv[j]);
+                    // rotation by p - t: x' = x cos - y sin, y' = x sin + y cos
+                    mk[j] += hi ? fmaf(kx[g].v[j], cc[h], y[j] * sn[h]) : fmaf(kx[g].v[j], cc[h], -y[j] * sn[h]);
+                    sv[j] += vx[g].v[j];
+                    srv[j] = fmaf(rr[g], vx[g].v[j], srv[j]);
                 }
             }
         }
@@ -204,37 +207,26 @@ __device__ void emit_node(const GatherArgs &A, int lg, int a, int b, int64_t e, 
 #pragma unroll
         for (int j = 0; j < 8; j++) {
             mk[j] += __shfl_xor_sync(0xffffffffu, mk[j], o);
-            mv[j] += __shfl_xor_sync(0xffffffffu, mv[j], o);
+            sv[j] += __shfl_xor_sync(0xffffffffu, sv[j], o);
+            srv[j] += __shfl_xor_sync(0xffffffffu, srv[j], o);
         }
         kn += __shfl_xor_sync(0xffffffffu, kn, o);
+        rs += __shfl_xor_sync(0xffffffffu, rs, o);
     }
     kn = __shfl_sync(0xffffffffu, kn, 0);
-    const int p = round_half_even_mid(a, b);
-    float u[8], pu[8], mu2 = 0.f;
+    const float ninv = 1.0f / (float)n;
+    const float beta = (float)A.base_frac * (rs * ninv);
+    const float winv = 1.0f / (rs + (float)n * beta + (float)A.eps);
+    float ko[8], vo[8], mu2 = 0.f;
 #pragma unroll
     for (int j = 0; j < 8; j++) {
-        u[j] = mk[j] * ninv;
-        mu2 = fmaf(u[j], u[j], mu2);
+        ko[j] = mk[j] * ninv;
+        vo[j] = fmaf(beta, sv[j], srv[j]) * winv;
+        mu2 = fmaf(ko[j], ko[j], mu2);
     }
 #pragma unroll
     for (int o = 1; o < LPR; o <<= 1) mu2 += __shfl_xor_sync(0xffffffffu, mu2, o);
-#pragma unroll
-    for (int j = 0; j < 8; j++) pu[j] = __shfl_xor_sync(0xffffffffu, u[j], PX);
     if (lane < LPR) {
-        const float4 *cs4 = reinterpret_cast<const float4 *>(A.rope + (size_t)p * HALF + i0);
-        float ko[8], vo[8];
-#pragma unroll
-        for (int j2 = 0; j2 < 4; j2++) {
-            const float4 q = cs4[j2];
-            const float cc[2] = {q.x, q.z}, sn[2] = {q.y, q.w};
-#pragma unroll
-            for (int h = 0; h < 2; h++) {
-                const int j = 2 * j2 + h;
-                // RoPE(mu, p): x' = x cos - y sin, y' = x sin + y cos
-                ko[j] = hi ? fmaf(u[j], cc[h], pu[j] * sn[h]) : fmaf(u[j], cc[h], -pu[j] * sn[h]);
-                vo[j] = mv[j] * winv;
-            }
-        }
         store8(Ko + 8 * c, ko);
         store8(Vo + 8 * c, vo);
     }
@@ -249,40 +241,42 @@ __device__ void emit_node(const GatherArgs &A, int lg, int a, int b, int64_t e, 
     }
 }
 
-// Warp per unit: depth-first traversal of the executed splits, children in
-// ascending position, so frontier nodes come out in ascending position.
-template <typename Tin, int DH>
-__global__ void __launch_bounds__(256, 2) gather_units_kernel(GatherArgs A) {
+// Frontier entries of every covered unit in ascending position (warp per
+// unit, depth-first over the executed splits, children in ascending
+// position): the descriptor of each entry goes to its output position.
+__global__ void gather_list_kernel(GatherArgs A) {
     __shared__ short stack[8][kMaxUnit + 4];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t nu = (int64_t)A.L * A.G * A.J;
     const int64_t uid = (int64_t)blockIdx.x * 8 + warp;
-    if (uid >= nu || A.u_sel[uid] != 1) return;
+    if (uid >= nu || A.u_sel[uid] != 1 || lane != 0) return;
     const int lg = (int)(uid / A.J), j = (int)(uid - (int64_t)lg * A.J);
     const int64_t nb = node_base(lg, A.slots[j], A.cs, A.Nc);
     int64_t e = A.u_off[uid];
     short *st = stack[warp];
-    int sp = 0;                      // stack owned by lane 0
-    if (lane == 0) st[sp++] = 0;
-    for (;;) {
-        int k = -1;
-        if (lane == 0) {
-            while (sp > 0) {
-                int x = st[--sp];
-                int64_t v = nb + x;
-                if (A.nd_sel[v] == 1) {
-                    int c0 = A.nd_child0[v], nc = A.nd_nchild[v];
-                    for (int q = nc - 1; q >= 0; q--) st[sp++] = (short)(c0 + q);   // leftmost on top
-                    continue;
-                }
-                k = x;
-                break;
-            }
+    int sp = 0;
+    st[sp++] = 0;
+    while (sp > 0) {
+        const int x = st[--sp];
+        const int64_t v = nb + x;
+        if (A.nd_sel[v] == 1) {
+            const int c0 = A.nd_child0[v], nc = A.nd_nchild[v];
+            for (int q = nc - 1; q >= 0; q--) st[sp++] = (short)(c0 + q);   // leftmost on top
+            continue;
         }
-        k = __shfl_sync(0xffffffffu, k, 0);
-        if (k < 0) break;
-        emit_node<Tin, DH>(A, lg, A.nd_a[nb + k], A.nd_b[nb + k], e, lane);
-        e++;
+        A.ent[e++] = make_int4(A.nd_a[v], A.nd_b[v], lg, 1);
+    }
+}
+
+// Prototypes of the listed entries: persistent warps, one entry at a time.
+template <typename Tin, int DH>
+__global__ void __launch_bounds__(256, 2) gather_emit_kernel(GatherArgs A, int64_t n_ent) {
+    const int lane = threadIdx.x & 31;
+    const int64_t nw = (int64_t)gridDim.x * 8;
+    for (int64_t e = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5); e < n_ent; e += nw) {
+        const int4 en = A.ent[e];
+        if (en.w == 0) continue;   // prefix / recent / suffix token (gather_tokens)
+        emit_node<Tin, DH>(A, en.z, en.x, en.y, e, lane);
     }
 }
 
@@ -311,7 +305,8 @@ cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *s
                           void *K_out, void *V_out, int32_t *pos, float *log_m,
                           int32_t *src_lo, int32_t *src_hi, int64_t *offsets, cudaStream_t s) {
     GatherArgs A;
-    A.K = K; A.V = V; A.rtok = c.w.rtok; A.rope = c.w.rope; A.slots = slots;
+    A.K = K; A.V = V; A.rtok = c.w.rtok; A.rope = c.w.rope; A.rope_rel = c.w.rope_rel; A.ent = c.w.ent;
+    A.slots = slots;
     A.nd_a = c.w.nd_a; A.nd_b = c.w.nd_b; A.nd_child0 = c.w.nd_child0; A.nd_nchild = c.w.nd_nchild;
     A.nd_sel = c.w.nd_sel; A.u_sel = c.w.u_sel; A.u_nnodes = c.w.u_nnodes;
     A.u_count = c.w.u_count; A.u_off = c.w.u_off;
@@ -324,17 +319,23 @@ cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *s
     gather_scan_kernel<<<1, 1024, 0, s>>>(A);
     const bool bf = c.p.dtype == GKV_BF16;
     unsigned gu = (unsigned)((nu + 7) / 8);
+    // descriptors by output position; positions of uncompressed tokens stay 0
+    const int64_t n_ent = c.p.L * (int64_t)c.p.G * (c.p.T - c.Nc) + c.used;
+    cudaError_t me = cudaMemsetAsync(A.ent, 0, sizeof(int4) * (size_t)n_ent, s);
+    if (me != cudaSuccess) return me;
     if (gu) {
+        gather_list_kernel<<<gu, 256, 0, s>>>(A);
+        const unsigned ge = (unsigned)std::min<int64_t>((n_ent + 7) / 8, (int64_t)c.num_sms * 2 * 8);
         if (c.p.d == 128) {
-            if (bf) gather_units_kernel<__nv_bfloat16, 128><<<gu, 256, 0, s>>>(A);
-            else gather_units_kernel<float, 128><<<gu, 256, 0, s>>>(A);
+            if (bf) gather_emit_kernel<__nv_bfloat16, 128><<<ge, 256, 0, s>>>(A, n_ent);
+            else gather_emit_kernel<float, 128><<<ge, 256, 0, s>>>(A, n_ent);
         } else {
-            if (bf) gather_units_kernel<__nv_bfloat16, 64><<<gu, 256, 0, s>>>(A);
-            else gather_units_kernel<float, 64><<<gu, 256, 0, s>>>(A);
+            if (bf) gather_emit_kernel<__nv_bfloat16, 64><<<ge, 256, 0, s>>>(A, n_ent);
+            else gather_emit_kernel<float, 64><<<ge, 256, 0, s>>>(A, n_ent);
         }
     }
     int ntok = c.p.ctx_start + (c.p.T - c.c_end);
-    c.launches += 2 + (gu ? 1 : 0) + (ntok > 0 ? 1 : 0);
+    c.launches += 2 + (gu ? 2 : 0) + (ntok > 0 ? 1 : 0);
     if (ntok > 0) {
         dim3 g((ntok + 7) / 8, c.p.L * c.p.G);
         if (bf) gather_tokens_kernel<__nv_bfloat16><<<g, 256, 0, s>>>(A);

@@ -23,6 +23,8 @@ constexpr int kMaxWindows = 4;
 struct Workspace {
     // RoPE rotation table: (cos, sin)(t * theta_i) for t in [0, T), i < d/2.
     float2 *rope = nullptr;
+    float2 *rope_rel = nullptr;    // [2 kMaxUnit - 1][d/2] rotations by the offsets -(kMaxUnit-1)..kMaxUnit-1
+    int4 *ent = nullptr;           // [B_total + L G (T - N_c)] frontier entry descriptors of the gather
     // segmentation
     float *inv_norm = nullptr;     // [n_seg][T] 1 / max(||h_t||, eps)
     float *nrm2 = nullptr;         // [n_seg][T] ||hbar_t||^2

@@ -22,11 +22,13 @@
 namespace gkv {
 namespace {
 
-__global__ void rope_table_kernel(int T, int d, double base, float2 *tab) {
+// (cos, sin) of the rotation angle (t0 + row) theta_i, theta_i = base^(-2i/d).
+__global__ void rope_table_kernel(int T, int d, double base, float2 *tab, int t0) {
     int half = d / 2;
     int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (e >= (int64_t)T * half) return;
     int t = (int)(e / half), i = (int)(e - (int64_t)t * half);
+    t += t0;
     if (base == 0.0) {
         tab[e] = make_float2(1.f, 0.f);
         return;
@@ -455,7 +457,11 @@ ScoreArgs make_args(const Ctx &c) {
 
 cudaError_t launch_rope_table(Ctx &c, cudaStream_t s) {
     int64_t n = (int64_t)c.p.T * (c.p.d / 2);
-    rope_table_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(c.p.T, c.p.d, c.p.rope_base, c.w.rope);
+    rope_table_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(c.p.T, c.p.d, c.p.rope_base, c.w.rope, 0);
+    // rotations by the offsets -(kMaxUnit - 1) .. kMaxUnit - 1 (prototype position minus token position)
+    int64_t nr = (int64_t)(2 * kMaxUnit - 1) * (c.p.d / 2);
+    rope_table_kernel<<<(unsigned)((nr + 255) / 256), 256, 0, s>>>(2 * kMaxUnit - 1, c.p.d, c.p.rope_base,
+                                                                   c.w.rope_rel, -(kMaxUnit - 1));
     return cudaGetLastError();
 }
 
