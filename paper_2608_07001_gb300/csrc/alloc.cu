@@ -73,28 +73,57 @@ __global__ void alloc_hist_kernel(AllocArgs A, int shift, int nbits, uint32_t ma
     for (int b = threadIdx.x; b < nbin; b += blockDim.x) sh[b] = 0;
     __syncthreads();
     const uint32_t prefix = (uint32_t)A.st[ST_PREFIX];
-    const int64_t n = A.n_units + A.n_nodes;
+    const int lane = threadIdx.x & 31;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t w0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31);
     unsigned int tot = 0;
-    // whole warps iterate together so that equal bins can be combined first
+    // whole warps consume items together so that equal bins are combined first
     // (keys cluster in few bins: one shared atomic per distinct bin and warp)
-    for (int64_t i0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); i0 < n; i0 += stride) {
-        const int64_t i = i0 + (threadIdx.x & 31);
-        uint32_t key = 0;
-        int cost = 0;
-        const bool op = i < n && op_key(A, i, key, cost);
+    auto consume = [&](bool op, uint32_t key, int cost) {
         tot += op ? cost : 0;
         const int bin = op && (key & mask) == prefix ? (int)((key >> shift) & (nbin - 1)) : -1;
         const unsigned grp = __match_any_sync(0xffffffffu, bin);
-        const unsigned sum = __reduce_add_sync(grp, (unsigned)cost);
-        if (bin >= 0 && (threadIdx.x & 31) == __ffs(grp) - 1) atomicAdd(&sh[bin], sum);
+        const unsigned sum = __reduce_add_sync(grp, (unsigned)(op ? cost : 0));
+        if (bin >= 0 && lane == __ffs(grp) - 1) atomicAdd(&sh[bin], sum);
+    };
+    for (int64_t i0 = w0; i0 < A.n_units; i0 += stride) {   // Add ops, cost 1
+        const int64_t i = i0 + lane;
+        const bool in = i < A.n_units;
+        const float x = in ? A.u_U[i] : 0.f;
+        if (in && (!(x >= 0.f) || isinf(x))) atomicOr(A.status, 8);
+        consume(in, __float_as_uint(x), 1);
+    }
+    // Split ops: 4 node slots per thread and step (one 32-bit load of their
+    // costs, one 16-byte load of their keys when any is an op)
+    const int64_t nq = A.n_nodes / 4;
+    for (int64_t q0 = w0; q0 < nq; q0 += stride) {
+        const int64_t q = q0 + lane;
+        const uint32_t cw = q < nq ? reinterpret_cast<const uint32_t *>(A.nd_cost)[q] : 0u;
+        float4 kv = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (cw) kv = reinterpret_cast<const float4 *>(A.nd_kappa)[q];
+        const float ks[4] = {kv.x, kv.y, kv.z, kv.w};
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            const int c = (int)(int8_t)(cw >> (8 * j));
+            const bool op = c > 0;
+            if (op && (!(ks[j] >= 0.f) || isinf(ks[j]))) atomicOr(A.status, 8);
+            consume(op, __float_as_uint(ks[j]), c);
+        }
+    }
+    if (blockIdx.x == 0 && threadIdx.x < 32) {   // the last n_nodes % 4 slots
+        const int64_t v = 4 * nq + lane;
+        const bool in = v < A.n_nodes;
+        const int c = in ? (int)A.nd_cost[v] : 0;
+        const float x = c > 0 ? A.nd_kappa[v] : 0.f;
+        if (c > 0 && (!(x >= 0.f) || isinf(x))) atomicOr(A.status, 8);
+        consume(c > 0, __float_as_uint(x), c);
     }
     __syncthreads();
     for (int b = threadIdx.x; b < nbin; b += blockDim.x)
         if (sh[b]) atomicAdd(&A.hist[b], (unsigned long long)sh[b]);
     if (shift == 21) {   // first pass: total cost of all ops
         tot = __reduce_add_sync(0xffffffffu, tot);
-        if ((threadIdx.x & 31) == 0 && tot) atomicAdd(&A.st[ST_TOTAL], (unsigned long long)tot);
+        if (lane == 0 && tot) atomicAdd(&A.st[ST_TOTAL], (unsigned long long)tot);
     }
 }
 
