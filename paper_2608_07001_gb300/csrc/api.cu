@@ -20,7 +20,7 @@ namespace {
 
 // Device status bits (dev_int[1]).
 enum : int { ST_NONFINITE_KAPPA = 1, ST_NONFINITE_ROWS = 2, ST_LONG_SLOT = 4, ST_NONFINITE_GAIN = 8,
-             ST_BAD_SLOTS = 16 };
+             ST_BAD_SLOTS = 16, ST_PIPE_TIMEOUT = gkv::kStPipeTimeout };
 
 gkv_status fail(gracekv_ctx *x, gkv_status s, const char *msg) {
     if (x) {
@@ -52,6 +52,7 @@ bool dalloc(gracekv_ctx *x, T **p, size_t n) {
 }
 
 gkv_status check_status(gracekv_ctx *x, int st) {
+    if (st & ST_PIPE_TIMEOUT) return fail(x, GKV_ECUDA, "a tensor-core pipeline wait timed out");
     if (st & ST_BAD_SLOTS) return fail(x, GKV_EINVAL, "supplied slot starts are not a partition of [c_s, c_e - r) into slots of 1..128 tokens");
     if (st & ST_LONG_SLOT) return fail(x, GKV_EUNSUPPORTED, "a slot is longer than 128 tokens (unit kernel limit)");
     if (st & ST_NONFINITE_KAPPA) return fail(x, GKV_ENONFINITE, "non-finite curvature (NaN/Inf in the trajectory)");
@@ -200,6 +201,7 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
     const int64_t base = LG * ((Rg + 63) / 64);
     c.n_chunks = (int)std::max<int64_t>(1, std::min<int64_t>((4 * c.num_sms + base - 1) / base,
                                                              std::max(1, p.T / 256)));
+    if (gkv::use_tc(c)) c.n_chunks = std::max(c.n_chunks, gkv::tc_row_chunks(c));
     c.node_cap = LG * 2 * Nc;
     const int nb = p.n_max - p.n_min + 1;
     const int64_t nrow = (int64_t)p.L * p.Hq * p.W;

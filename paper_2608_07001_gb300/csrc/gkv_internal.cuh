@@ -13,7 +13,8 @@
 
 namespace gkv {
 
-constexpr int kMaxUnit = 128;      // longest slot a unit kernel holds in shared memory
+constexpr int kMaxUnit = 128;
+constexpr int kStPipeTimeout = 32;   // status bit: a bounded wait of a tensor-core pipeline gave up      // longest slot a unit kernel holds in shared memory
 constexpr int kMaxSegLayers = 8;
 constexpr int kMaxWindows = 4;
 
@@ -221,6 +222,12 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
                            const float *surprisal, float *kappa_out, cudaStream_t s);
 
 cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t s);
+// tcgen05 score passes (score_tc.cu): applicable to bf16, d in {64, 128}, at
+// most 256 probe rows per KV head; row-statistics partials per row = tc_row_chunks.
+bool use_tc(const Ctx &c);
+int tc_row_chunks(const Ctx &c);
+cudaError_t launch_row_stats_tc(Ctx &c, const void *K, const void *Q, cudaStream_t s);
+cudaError_t launch_token_values_tc(Ctx &c, const void *K, const void *Q, cudaStream_t s);
 cudaError_t launch_token_values(Ctx &c, const void *K, const void *Q, cudaStream_t s);
 // Slots of at most kShortUnit tokens run on the unit kernel instance that fits
 // two CTAs per SM; the work lists hold them (slot indices for a fresh build,

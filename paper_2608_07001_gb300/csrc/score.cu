@@ -12,8 +12,10 @@
 //                  (App. A.4 Eqs. app_direct_relevance, app_bottom_up_value with
 //                  lambda_graph = 0).
 //
-// Both passes contract a [rows x d] query block with [tokens x d] keys in
-// 64 x 64 tiles (FFMA, fp32 accumulation of the exact bf16/fp32 inputs).
+// Both passes contract a [rows x d] query block with [tokens x d] keys.  bf16
+// inputs with d in {64, 128} run on the tcgen05 tensor cores (score_tc.cu);
+// other bf16 shapes on mma.sync tiles below; fp32 inputs in 64 x 64 FFMA tiles.
+// All accumulate in fp32 from exact products of the inputs.
 #include "gkv_internal.cuh"
 
 #include <algorithm>
@@ -491,6 +493,15 @@ void launch_mma_b(const Ctx &c, const ScoreArgs &a, const void *K, const void *Q
 
 cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t s) {
     ScoreArgs a = make_args(c);
+    if (use_tc(c)) {   // tcgen05 pass (score_tc.cu), then the same combine
+        cudaError_t e = launch_row_stats_tc(c, K, Q, s);
+        if (e != cudaSuccess) return e;
+        int nrow = a.L * a.Hq * a.W;
+        row_combine_kernel<<<(nrow + 255) / 256, 256, 0, s>>>(c.w.rowp, nrow, tc_row_chunks(c), c.w.row_m,
+                                                              c.w.row_Z, c.w.row_ZC, c.w.dev_int + 1);
+        c.launches += 1;
+        return cudaGetLastError();
+    }
     int chunk = (c.p.T + c.n_chunks - 1) / c.n_chunks;
     chunk = (chunk + kTT - 1) / kTT * kTT;
     if (use_mma(c, a)) {
@@ -522,6 +533,7 @@ cudaError_t launch_token_values(Ctx &c, const void *K, const void *Q, cudaStream
     ScoreArgs a = make_args(c);
     dim3 grid((c.Nc + kTT - 1) / kTT, a.L * a.G);
     float eps = (float)c.p.eps;
+    if (use_tc(c)) return launch_token_values_tc(c, K, Q, s);
     if (use_mma(c, a)) {
         // about 4 CTAs of 16 warps per SM-pass over the compressible region
         int64_t want = 4LL * c.num_sms;
