@@ -219,6 +219,7 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
               dalloc(x, &w.dev_int, 16) &&
               dalloc(x, &w.row_m, (size_t)nrow) && dalloc(x, &w.row_Z, (size_t)nrow) &&
               dalloc(x, &w.row_ZC, (size_t)nrow) && dalloc(x, &w.rowp, (size_t)3 * nrow * c.n_chunks) &&
+              dalloc(x, &w.row_mneg, (size_t)nrow) && dalloc(x, &w.lg_scale, (size_t)LG) &&
               dalloc(x, &w.rtok, (size_t)LG * Nc) &&
               dalloc(x, &w.nd_a, (size_t)c.node_cap) && dalloc(x, &w.nd_b, (size_t)c.node_cap) &&
               dalloc(x, &w.nd_child0, (size_t)c.node_cap) && dalloc(x, &w.nd_parent, (size_t)c.node_cap) &&
@@ -486,7 +487,7 @@ gkv_status gracekv_export(gracekv_ctx *x, int64_t node_cap, int64_t *n_nodes_hos
     std::vector<int32_t> slots(J + 1), nn(nu);
     std::vector<int32_t> ha(c.node_cap), hb(c.node_cap), hc(c.node_cap);
     std::vector<int8_t> hn(c.node_cap), hk(c.node_cap);
-    std::vector<double> hD(c.node_cap);
+    std::vector<float> hD(c.node_cap);
     std::vector<float> hR(c.node_cap), hU(c.node_cap), hK(c.node_cap);
     std::vector<uint8_t> hs(c.node_cap);
     cudaError_t e = cudaStreamSynchronize(s);
@@ -521,7 +522,7 @@ gkv_status gracekv_export(gracekv_ctx *x, int64_t node_cap, int64_t *n_nodes_hos
             if (child0) child0[k] = hc[v];
             if (nchild) nchild[k] = hn[v];
             if (cost) cost[k] = hk[v];
-            if (D) D[k] = (float)hD[v];
+            if (D) D[k] = hD[v];
             if (R) R[k] = hR[v];
             if (U) U[k] = hU[v];
             if (kappa) kappa[k] = hK[v];

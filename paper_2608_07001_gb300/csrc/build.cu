@@ -61,7 +61,7 @@ struct BuildArgs {
     const float *rtok, *row_m, *row_Z, *omega;
     int L, G, Hq, T, d, W, gq, cs, Nc, J, k_cand;
     float inv_sqrt_d, lamZ, lamM, eps;
-    double lam_kappa, base_frac;
+    float lam_kappa, base_frac;
     // work list: fresh launches index (slot list entry, lg), resume launches units
     int resume;                  // 0: build from the root, 1: resume pending nodes
     int root_only;               // fresh: evaluate only the root's own distortion (split stays pending)
@@ -71,7 +71,7 @@ struct BuildArgs {
     // outputs
     int32_t *nd_a, *nd_b, *nd_child0, *nd_parent, *nd_unit;
     int8_t *nd_nchild, *nd_cost;
-    double *nd_D;
+    float *nd_D;
     float *nd_R, *nd_U, *nd_kappa;
     uint8_t *nd_sel;
     int32_t *u_nnodes;
@@ -82,7 +82,7 @@ struct BuildArgs {
 };
 
 struct NodeS {
-    double D;
+    float D;
     float kin;                   // bottleneck key of the op that created the node
     short a, b, parent, child0;
     signed char nchild;          // -1: pending (not evaluated)
@@ -98,9 +98,10 @@ struct BatchNode {
     int pre_b, pre_e, suf_b, suf_e;   // prefixes (ascending end) in [0, NCD),
                                       // suffixes (descending start) in [NCD, 2 NCD)
     int pre_r, suf_r;                 // ends of the reserved ranges (unused entries empty)
-    double kmin, kmax;
+    double kmin;             // smallest curvature over the node's cut positions
+    float krange;            // 1 / (largest - smallest), 0 when they are equal
     int nchild, ca[3], cb[3];
-    double cD[3];
+    float cD[3];
 };
 
 struct Cand {
@@ -110,11 +111,12 @@ struct Cand {
 
 // Upper bound of a split's utility: U = omega R (D - sum D_children) / cost
 // <= omega R D, since every D >= 0 and cost >= 1 (Eqs. app_operation_gains,
-// app_unit_utility).  Rounded up, so that fp32 rounding never makes a bound
-// fall below the utility it bounds.
-__device__ __forceinline__ float key_bound(double x) {
-    const float f = (float)x;
-    return f + fabsf(f) * 1e-6f;
+// app_unit_utility).  Rounded up by 1e-5 of its value: the R that the bound
+// uses (one fp32 sum over the node's tokens) and the R of the later gain (the
+// sum of its children's sums) differ by at most ~1.3e-6 of R, and the products
+// add a few ulp, so rounding never makes a bound fall below the utility it bounds.
+__device__ __forceinline__ float key_bound(float x) {
+    return x + fabsf(x) * 1e-5f;
 }
 
 // Order-preserving 64-bit key of a double (larger value -> larger key), so
@@ -210,7 +212,7 @@ struct Smem {
     unsigned long long kap[NMAX];            // order-preserving keys of the curvature
     float redD[2 * kNCD][NWARPS];
     float redP[2 * kNCD][NWARPS];
-    double candD[2 * kNCD], candP[2 * kNCD]; // per-candidate D and drop mass
+    float candD[2 * kNCD], candP[2 * kNCD];  // per-candidate D and drop mass
     Cand cand[2 * kNCD];
     NodeS nodes[MAXNODES];
     BatchNode bn[NB];
@@ -220,7 +222,7 @@ struct Smem {
     int batch_n, batch_next, batch_pre, batch_suf;   // candidate entries reserved per direction
     unsigned long long wcnt[kNT / 32][3];   // per-warp work counters
     float pend;
-    double rootR;                            // R of a fresh root
+    float rootR;                             // R of a fresh root
 };
 
 template <int DH, typename Tin, int NMAX>
@@ -376,7 +378,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         if (__syncthreads_or(bad)) {
             if (tid == 0) {
                 atomicOr(A.status, 8);
-                A.nd_a[nbase] = sa; A.nd_b[nbase] = sb; A.nd_R[nbase] = 0.f; A.nd_D[nbase] = 0.0;
+                A.nd_a[nbase] = sa; A.nd_b[nbase] = sb; A.nd_R[nbase] = 0.f; A.nd_D[nbase] = 0.f;
                 A.nd_parent[nbase] = (int32_t)(-2 - uid); A.nd_unit[nbase] = (int32_t)uid;
                 A.nd_child0[nbase] = -1; A.nd_nchild[nbase] = 0; A.nd_U[nbase] = 0.f;
                 A.nd_kappa[nbase] = 0.f; A.nd_sel[nbase] = 0;
@@ -405,13 +407,13 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     // ---- tree state: a fresh root, or the unit's records so far --------------
     if (!A.resume) {
         if (warp == 0) {
-            double r = 0.0;
+            float r = 0.f;
             for (int t = lane; t < n; t += 32) r += sm.Rt[t];
             r = warp_sum(r);
             if (lane == 0) {
                 NodeS &nd = sm.nodes[0];
                 nd.a = 0; nd.b = (short)n; nd.parent = -1; nd.child0 = -1; nd.nchild = 0;
-                nd.D = 0.0; nd.kin = 0.f;
+                nd.D = 0.f; nd.kin = 0.f;
                 sm.rootR = r;
                 sm.nnodes = 1;
                 sm.lvl[0][0] = 0;
@@ -769,8 +771,9 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     ss = min(ss, __shfl_xor_sync(FULL, ss, o));
                 }
                 if (lane == 0) {
-                    B.kmin = nv >= 2 ? okey_inv(kmin) : 0.0;
-                    B.kmax = nv >= 2 ? okey_inv(kmax) : 0.0;
+                    const double kmn = nv >= 2 ? okey_inv(kmin) : 0.0, kmx = nv >= 2 ? okey_inv(kmax) : 0.0;
+                    B.kmin = kmn;
+                    B.krange = kmx > kmn ? 1.0f / (float)(kmx - kmn) : 0.f;
                     B.pstar = pb;
                     B.ncut = ncut;
                     B.eL = el_sep ? eL_sep : (el_cand ? eL_cut : -1);
@@ -810,11 +813,11 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 const int a = nd.a, b = nd.b, nv = b - a;
                 // D and drop mass of this node's candidates: mean over the W probes
                 // of the per-warp partial sums
-                const double invW = 1.0 / A.W;
+                const float invW = 1.0f / A.W;
                 for (int k = lane; k < 2 * kNCD; k += 32) {
                     const bool mine = k < kNCD ? (k >= B.pre_b && k < B.pre_e) : (k >= B.suf_b && k < B.suf_e);
                     if (!mine) continue;
-                    double d = 0.0, pw = 0.0;
+                    float d = 0.f, pw = 0.f;
 #pragma unroll
                     for (int w = 0; w < NWARPS; w++) { d += sm.redD[k][w]; pw += sm.redP[k][w]; }
                     sm.candD[k] = d * invW;
@@ -822,14 +825,14 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 }
                 __syncwarp();
                 if (B.whole >= 0 && lane == 0) {   // root: D, Ddrop, Add gain (Eq. app_operation_gains)
-                    const double Pd = sm.candP[B.whole];
-                    const double D = nv >= 2 ? sm.candD[B.whole] : 0.0;
+                    const float Pd = sm.candP[B.whole];
+                    const float D = nv >= 2 ? sm.candD[B.whole] : 0.f;
                     nd.D = D;
-                    double gain = (double)om * sm.rootR * (Pd - D);
-                    if (gain < 0.0) gain = 0.0;
-                    nd.kin = (float)gain;
-                    A.u_Uadd[uid] = (float)gain;
-                    A.u_Ddrop[uid] = (float)Pd;
+                    float gain = om * sm.rootR * (Pd - D);
+                    if (gain < 0.f) gain = 0.f;
+                    nd.kin = gain;
+                    A.u_Uadd[uid] = gain;
+                    A.u_Ddrop[uid] = Pd;
                     A.nd_D[nbase] = D;
                 }
                 __syncwarp();
@@ -842,54 +845,55 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                         B.nchild = 0;
                         if (nv == 2) {
                             B.nchild = 2;
-                            B.ca[0] = a; B.cb[0] = a + 1; B.cD[0] = 0.0;
-                            B.ca[1] = a + 1; B.cb[1] = b; B.cD[1] = 0.0;
+                            B.ca[0] = a; B.cb[0] = a + 1; B.cD[0] = 0.f;
+                            B.ca[1] = a + 1; B.cb[1] = b; B.cD[1] = 0.f;
                         }
                     }
                     continue;
                 }
-                const double DI = nd.D;
+                const float DI = nd.D;
                 // binary cut: lane q evaluates cut q; max G_bin, ties -> smallest xi
-                const double krange = B.kmax > B.kmin ? 1.0 / (B.kmax - B.kmin) : 0.0;
-                double best = -INFINITY;
+                float best = -INFINITY;
                 int bq = 0x7fffffff;
                 if (lane < B.ncut) {
                     const int xi = B.cut[lane];
-                    const double DL = B.pidx[lane] >= 0 ? sm.candD[B.pidx[lane]] : 0.0;
-                    const double DR = B.sidx[lane] >= 0 ? sm.candD[B.sidx[lane]] : 0.0;
-                    const double kh = (okey_inv(sm.kap[xi - 1]) - B.kmin) * krange;
+                    const float DL = B.pidx[lane] >= 0 ? sm.candD[B.pidx[lane]] : 0.f;
+                    const float DR = B.sidx[lane] >= 0 ? sm.candD[B.sidx[lane]] : 0.f;
+                    // normalised curvature: the difference is taken in fp64 (the
+                    // curvatures may be close), the rest in fp32
+                    const float kh = (float)(okey_inv(sm.kap[xi - 1]) - B.kmin) * B.krange;
                     best = ((DI - DL) - DR) + A.lam_kappa * kh;
                     bq = lane;
                 }
 #pragma unroll
                 for (int o = 16; o > 0; o >>= 1) {
-                    double ov = __shfl_xor_sync(0xffffffffu, best, o);
+                    float ov = __shfl_xor_sync(0xffffffffu, best, o);
                     int oq = __shfl_xor_sync(0xffffffffu, bq, o);
                     if (ov > best || (ov == best && oq < bq)) { best = ov; bq = oq; }
                 }
                 if (lane) continue;
                 int bxi = -1;
-                double bL = 0, bR = 0;
+                float bL = 0.f, bR = 0.f;
                 if (bq < B.ncut && best > -INFINITY) {
                     bxi = B.cut[bq];
-                    bL = B.pidx[bq] >= 0 ? sm.candD[B.pidx[bq]] : 0.0;
-                    bR = B.sidx[bq] >= 0 ? sm.candD[B.sidx[bq]] : 0.0;
+                    bL = B.pidx[bq] >= 0 ? sm.candD[B.pidx[bq]] : 0.f;
+                    bR = B.sidx[bq] >= 0 ? sm.candD[B.sidx[bq]] : 0.f;
                 }
                 // extraction at p*
                 const int ps = B.pstar;
                 int ea[3], eb[3], ne = 0;
-                double eD[3];
-                if (ps > a) { ea[ne] = a; eb[ne] = ps; eD[ne] = ps - a >= 2 ? sm.candD[B.eL] : 0.0; ne++; }
-                ea[ne] = ps; eb[ne] = ps + 1; eD[ne] = 0.0; ne++;
-                if (ps + 1 < b) { ea[ne] = ps + 1; eb[ne] = b; eD[ne] = b - ps - 1 >= 2 ? sm.candD[B.eR] : 0.0; ne++; }
-                double gext = DI;
+                float eD[3];
+                if (ps > a) { ea[ne] = a; eb[ne] = ps; eD[ne] = ps - a >= 2 ? sm.candD[B.eL] : 0.f; ne++; }
+                ea[ne] = ps; eb[ne] = ps + 1; eD[ne] = 0.f; ne++;
+                if (ps + 1 < b) { ea[ne] = ps + 1; eb[ne] = b; eD[ne] = b - ps - 1 >= 2 ? sm.candD[B.eR] : 0.f; ne++; }
+                float gext = DI;
                 for (int q = 0; q < ne; q++) gext -= eD[q];
                 if (bxi < 0) {   // only reachable with non-finite gains
                     bxi = B.cut[0];
-                    bL = B.pidx[0] >= 0 ? sm.candD[B.pidx[0]] : 0.0;
-                    bR = B.sidx[0] >= 0 ? sm.candD[B.sidx[0]] : 0.0;
+                    bL = B.pidx[0] >= 0 ? sm.candD[B.pidx[0]] : 0.f;
+                    bR = B.sidx[0] >= 0 ? sm.candD[B.sidx[0]] : 0.f;
                 }
-                const double rho_ext = ne == 3 ? 0.5 * gext : gext;   // G_ext / (|children| - 1), exact
+                const float rho_ext = ne == 3 ? 0.5f * gext : gext;   // G_ext / (|children| - 1), exact
                 if (rho_ext > best) {
                     B.nchild = ne;
                     for (int q = 0; q < ne; q++) { B.ca[q] = ea[q]; B.cb[q] = eb[q]; B.cD[q] = eD[q]; }
@@ -913,7 +917,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 const int nch = B.nchild;
                 if (nch < 0) {   // pending root: its split key is at most min(U_add, omega R D)
                     if (lane == 0) {
-                        const float bnd = fminf(nd.kin, key_bound((double)om * sm.rootR * nd.D));
+                        const float bnd = fminf(nd.kin, key_bound(om * sm.rootR * nd.D));
                         nd.nchild = -1; nd.child0 = -1;
                         A.nd_child0[gv] = -1; A.nd_nchild[gv] = -1; A.nd_cost[gv] = 0;
                         A.nd_U[gv] = bnd; A.nd_kappa[gv] = 0.f; A.nd_sel[gv] = 0;
@@ -930,18 +934,18 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     }
                     continue;
                 }
-                double rch[3] = {0.0, 0.0, 0.0};
+                float rch[3] = {0.f, 0.f, 0.f};
                 for (int q = 0; q < nch; q++) {
-                    double r = 0.0;
+                    float r = 0.f;
                     for (int t = B.ca[q] + lane; t < B.cb[q]; t += 32) r += sm.Rt[t];
                     rch[q] = warp_sum(r);
                 }
-                const double rnode = (rch[0] + rch[1]) + rch[2];   // R of the node = sum over its children
-                const double dsum = (B.cD[0] + B.cD[1]) + (nch == 3 ? B.cD[2] : 0.0);
+                const float rnode = (rch[0] + rch[1]) + rch[2];   // R of the node = sum over its children
+                const float dsum = (B.cD[0] + B.cD[1]) + (nch == 3 ? B.cD[2] : 0.f);
                 const int cost = nch - 1;
-                double gain = (double)om * rnode * (nd.D - dsum);
-                if (gain < 0.0) gain = 0.0;
-                const float U = (float)(gain / cost);
+                float gain = om * rnode * (nd.D - dsum);
+                if (gain < 0.f) gain = 0.f;
+                const float U = cost == 2 ? 0.5f * gain : gain;
                 const float kap = fminf(U, nd.kin);
                 if (lane == 0) {
                     nd.nchild = (signed char)nch;
@@ -952,7 +956,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 }
                 if (lane < nch) {   // lane q writes child q
                     const int q = lane, ci = child0 + q;
-                    const double rq = q == 0 ? rch[0] : (q == 1 ? rch[1] : rch[2]);
+                    const float rq = q == 0 ? rch[0] : (q == 1 ? rch[1] : rch[2]);
                     NodeS &ch = sm.nodes[ci];
                     ch.a = (short)B.ca[q]; ch.b = (short)B.cb[q]; ch.parent = (short)B.node;
                     ch.child0 = -1; ch.nchild = 0; ch.D = B.cD[q]; ch.kin = kap;
@@ -962,7 +966,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     A.nd_D[gc] = B.cD[q]; A.nd_R[gc] = (float)rq;
                     A.nd_child0[gc] = -1; A.nd_nchild[gc] = 0; A.nd_cost[gc] = 0;
                     // until the child is evaluated, nd_U holds the bound of its split key
-                    A.nd_U[gc] = B.cb[q] - B.ca[q] >= 2 ? fminf(kap, key_bound((double)om * rq * B.cD[q])) : 0.f;
+                    A.nd_U[gc] = B.cb[q] - B.ca[q] >= 2 ? fminf(kap, key_bound(om * rq * B.cD[q])) : 0.f;
                     A.nd_kappa[gc] = 0.f; A.nd_sel[gc] = 0;
                     if (B.cb[q] - B.ca[q] >= 2) {
                         const int pos = atomicAdd(&sm.nlvl[cur ^ 1], 1);

@@ -42,14 +42,16 @@ struct Workspace {
     // row statistics and token values
     float *row_m = nullptr, *row_Z = nullptr, *row_ZC = nullptr;  // [L*Hq*W]
     float *rowp = nullptr;         // [3][L*Hq*W][n_chunks] pass-A partials
+    float *row_mneg = nullptr;     // [L*Hq*W] -(m log2 e + log2 Z): pass-B exponent offset
+    double *lg_scale = nullptr;    // [L*G] pass-B normaliser 1 / (sum_r Z^C_r / Z_r + eps)
     float *rtok = nullptr;         // [L*G*N_c]
     // node records, indexed lg*2*N_c + 2*(slot start - c_s) + k
     int32_t *nd_a = nullptr, *nd_b = nullptr, *nd_child0 = nullptr;
     int32_t *nd_parent = nullptr;  // global index of the parent; roots: -2 - unit id
     int32_t *nd_unit = nullptr;    // unit id lg * J + j
     int8_t *nd_nchild = nullptr, *nd_cost = nullptr;
-    double *nd_D = nullptr;        // distortion D(I_v) of every node (fp64 so that resumed
-                                   // nodes see exactly the value their parent computed)
+    float *nd_D = nullptr;         // distortion D(I_v) of every node (resumed nodes read
+                                   // exactly the value their parent computed)
     float *nd_R = nullptr, *nd_U = nullptr, *nd_kappa = nullptr;
     uint8_t *nd_sel = nullptr;     // split selected (1), discarded tie (2)
     // per-unit arrays (capacity units_cap), unit id = lg * J + j

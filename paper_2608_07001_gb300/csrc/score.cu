@@ -148,8 +148,10 @@ __global__ void __launch_bounds__(256) row_stats_kernel(const Tin *K, const Tin 
     }
 }
 
+// Combines the per-chunk partials of every row; rmneg (nullable) receives
+// -(m_r log2 e + log2 Z_r), the base-2 exponent offset of exp(x - m_r) / Z_r.
 __global__ void row_combine_kernel(const float *part, int nrow, int nchunks, float *rm, float *rz,
-                                   float *rzc, int *status) {
+                                   float *rzc, int *status, float *rmneg) {
     int row = blockIdx.x * blockDim.x + threadIdx.x;
     if (row >= nrow) return;
     const float *pm = part + (size_t)row * nchunks;
@@ -168,6 +170,18 @@ __global__ void row_combine_kernel(const float *part, int nrow, int nchunks, flo
     rm[row] = M;
     rz[row] = (float)Z;
     rzc[row] = (float)ZC;
+    if (rmneg) rmneg[row] = (float)(-((double)M * 1.4426950408889634 + log2((double)(float)Z)));
+}
+
+// Pass-B normaliser of every KV head: 1 / (sum_r Z^C_r / Z_r + eps) over its rows.
+__global__ void lg_scale_kernel(const float *rz, const float *rzc, int G, int Hq, int W, int gq, double eps,
+                                double *out) {
+    const int lg = blockIdx.x, l = lg / G, g = lg - l * G;
+    const size_t rowbase = (size_t)(l * Hq + g * gq) * W;
+    double s = 0.0;
+    for (int r = threadIdx.x; r < gq * W; r += 32) s += (double)rzc[rowbase + r] / (double)rz[rowbase + r];
+    s = warp_sum(s);
+    if (threadIdx.x == 0) out[lg] = 1.0 / (s + eps);
 }
 
 // Pass B.  grid = (token tiles over C, L*G).  Loops over the row tiles of the
@@ -498,7 +512,10 @@ cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t 
         if (e != cudaSuccess) return e;
         int nrow = a.L * a.Hq * a.W;
         row_combine_kernel<<<(nrow + 255) / 256, 256, 0, s>>>(c.w.rowp, nrow, tc_row_chunks(c), c.w.row_m,
-                                                              c.w.row_Z, c.w.row_ZC, c.w.dev_int + 1);
+                                                              c.w.row_Z, c.w.row_ZC, c.w.dev_int + 1, c.w.row_mneg);
+        lg_scale_kernel<<<a.L * a.G, 32, 0, s>>>(c.w.row_Z, c.w.row_ZC, a.G, a.Hq, a.W, a.gq, (double)c.p.eps,
+                                                  c.w.lg_scale);
+        c.launches += 1;
         c.launches += 1;
         return cudaGetLastError();
     }
@@ -509,7 +526,7 @@ cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t 
         else launch_mma_a<64>(c, a, K, Q, chunk, s);
         int nrow = a.L * a.Hq * a.W;
         row_combine_kernel<<<(nrow + 255) / 256, 256, 0, s>>>(c.w.rowp, nrow, c.n_chunks, c.w.row_m,
-                                                              c.w.row_Z, c.w.row_ZC, c.w.dev_int + 1);
+                                                              c.w.row_Z, c.w.row_ZC, c.w.dev_int + 1, nullptr);
         c.launches += 2;
         return cudaGetLastError();
     }
@@ -524,7 +541,7 @@ cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t 
                                               c.w.rowp);
     int nrow = a.L * a.Hq * a.W;
     row_combine_kernel<<<(nrow + 255) / 256, 256, 0, s>>>(c.w.rowp, nrow, c.n_chunks, c.w.row_m,
-                                                          c.w.row_Z, c.w.row_ZC, c.w.dev_int + 1);
+                                                          c.w.row_Z, c.w.row_ZC, c.w.dev_int + 1, nullptr);
     c.launches += 2;
     return cudaGetLastError();
 }
@@ -645,6 +662,6 @@ extern "C" gkv_status gracekv_row_stats_noalloc(const void *K, const void *Q, in
                                                    static_cast<const float *>(Q), a, chunk, nchunks,
                                                    scratch);
     gkv::row_combine_kernel<<<(unsigned)((nrow + 255) / 256), 256, 0, s>>>(scratch, (int)nrow, nchunks,
-                                                                            row_m, row_Z, row_ZC, status);
+                                                                            row_m, row_Z, row_ZC, status, nullptr);
     return cudaGetLastError() == cudaSuccess ? GKV_OK : GKV_ECUDA;
 }

@@ -56,7 +56,6 @@ struct TcArgs {
     int chunk_tiles, nch;    // tiles per block, blocks per (l, g)
     int nq;                  // probe rows staged: 128 * halves (pass A) or the padded width N (pass B)
     float scale;             // log2(e) / sqrt(d)
-    float eps;
 };
 
 __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
@@ -79,7 +78,7 @@ struct TcBars {
 template <int DH, int MODE>
 __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
         const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CUtensorMap mapQ, TcArgs a,
-        const float *rm, const float *rz, const float *rzc, float *part, float *rtok, int *status) {
+        const float *rmneg, const double *lg_scale, float *part, float *rtok, int *status) {
     constexpr int NKB = DH / 64;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char *sbase = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -89,7 +88,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
     unsigned char *Ks = sbase + (size_t)NKB * QR * 128;     // [stage][NKB][128][128 B]
     __shared__ TcBars sb;
     __shared__ __align__(16) float mneg[256];   // pass B: -(m_r log2 e + log2 Z_r), -inf past the rows
-    __shared__ double scale_s;
+    __shared__ float scale_s;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int lg = blockIdx.y, l = lg / a.G, g = lg - l * a.G;
@@ -116,20 +115,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
         tc::fence_barrier_init();
     }
     if (MODE == 1) {
-        for (int r = threadIdx.x; r < 256; r += kTcThreads) {
-            float v = -INFINITY;
-            if (r < a.Rg) {
-                const double m2 = (double)rm[rowbase + r] * 1.4426950408889634 + log2((double)rz[rowbase + r]);
-                v = (float)(-m2);
-            }
-            mneg[r] = v;
-        }
-        if (warp == kTcWarpTma) {
-            double sum = 0.0;
-            for (int r = lane; r < a.Rg; r += 32) sum += (double)rzc[rowbase + r] / (double)rz[rowbase + r];
-            sum = warp_sum(sum);
-            if (lane == 0) scale_s = 1.0 / (sum + (double)a.eps);
-        }
+        for (int r = threadIdx.x; r < 256; r += kTcThreads) mneg[r] = r < a.Rg ? rmneg[rowbase + r] : -INFINITY;
+        if (threadIdx.x == 0) scale_s = (float)lg_scale[lg];
     }
     if (warp == kTcWarpMma) {
         tc::tmem_alloc(tc::smem_u32(&sb.tbase), tcols);
@@ -335,7 +322,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
             }
             const float s = (acc0.x + acc0.y) + (acc1.x + acc1.y);
             const int t = t_begin + i * kTcTile + q * 32 + lane;
-            if (t < t_end) rtok[(size_t)lg * a.Nc + (t - a.cs)] = (float)((double)s * scale_s);
+            if (t < t_end) rtok[(size_t)lg * a.Nc + (t - a.cs)] = s * scale_s;
         }
     }
     tc::tc_fence_before();
@@ -382,7 +369,7 @@ size_t tc_smem(int DH, int nq) {
 
 template <int DH, int MODE>
 cudaError_t launch_tc(const TcArgs &a, int LG, const void *K, const void *Q, int64_t krows, int64_t qrows,
-                      const float *rm, const float *rz, const float *rzc, float *part, float *rtok, int *status,
+                      const float *rmneg, const double *lg_scale, float *part, float *rtok, int *status,
                       cudaStream_t s) {
     CUtensorMap mk, mq;
     if (!make_map(&mk, K, krows, DH) || !make_map(&mq, Q, qrows, DH)) return cudaErrorNotSupported;
@@ -391,7 +378,7 @@ cudaError_t launch_tc(const TcArgs &a, int LG, const void *K, const void *Q, int
                                          (int)tc_smem(DH, 256));
     if (e != cudaSuccess) return e;
     dim3 grid(a.nch, LG);
-    score_tc_kernel<DH, MODE><<<grid, kTcThreads, smem, s>>>(mk, mq, a, rm, rz, rzc, part, rtok, status);
+    score_tc_kernel<DH, MODE><<<grid, kTcThreads, smem, s>>>(mk, mq, a, rmneg, lg_scale, part, rtok, status);
     return cudaGetLastError();
 }
 
@@ -412,7 +399,6 @@ TcArgs base_args(const Ctx &c) {
     a.cs = c.p.ctx_start; a.cend = c.c_end; a.Nc = c.Nc;
     a.nrow_all = c.p.L * c.p.Hq * c.p.W;
     a.scale = (float)(1.4426950408889634 / sqrt((double)c.p.d));
-    a.eps = (float)c.p.eps;
     return a;
 }
 
@@ -440,8 +426,8 @@ cudaError_t launch_row_stats_tc(Ctx &c, const void *K, const void *Q, cudaStream
     const int LG = c.p.L * c.p.G;
     const int64_t krows = (int64_t)LG * c.p.T, qrows = (int64_t)a.nrow_all;
     cudaError_t e = c.p.d == 128
-        ? launch_tc<128, 0>(a, LG, K, Q, krows, qrows, nullptr, nullptr, nullptr, c.w.rowp, nullptr, c.w.dev_int + 1, s)
-        : launch_tc<64, 0>(a, LG, K, Q, krows, qrows, nullptr, nullptr, nullptr, c.w.rowp, nullptr, c.w.dev_int + 1, s);
+        ? launch_tc<128, 0>(a, LG, K, Q, krows, qrows, nullptr, nullptr, c.w.rowp, nullptr, c.w.dev_int + 1, s)
+        : launch_tc<64, 0>(a, LG, K, Q, krows, qrows, nullptr, nullptr, c.w.rowp, nullptr, c.w.dev_int + 1, s);
     if (e == cudaSuccess) c.launches += 1;
     return e;
 }
@@ -455,9 +441,9 @@ cudaError_t launch_token_values_tc(Ctx &c, const void *K, const void *Q, cudaStr
     const int LG = c.p.L * c.p.G;
     const int64_t krows = (int64_t)LG * c.p.T, qrows = (int64_t)a.nrow_all;
     cudaError_t e = c.p.d == 128
-        ? launch_tc<128, 1>(a, LG, K, Q, krows, qrows, c.w.row_m, c.w.row_Z, c.w.row_ZC, nullptr, c.w.rtok,
+        ? launch_tc<128, 1>(a, LG, K, Q, krows, qrows, c.w.row_mneg, c.w.lg_scale, nullptr, c.w.rtok,
                             c.w.dev_int + 1, s)
-        : launch_tc<64, 1>(a, LG, K, Q, krows, qrows, c.w.row_m, c.w.row_Z, c.w.row_ZC, nullptr, c.w.rtok,
+        : launch_tc<64, 1>(a, LG, K, Q, krows, qrows, c.w.row_mneg, c.w.lg_scale, nullptr, c.w.rtok,
                            c.w.dev_int + 1, s);
     if (e == cudaSuccess) c.launches += 1;
     return e;
