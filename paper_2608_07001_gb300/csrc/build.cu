@@ -258,15 +258,30 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     const float om = A.omega ? A.omega[lg] : 1.0f;
 
     // ---- load the slot ------------------------------------------------------
-    for (int e = tid * 8; e < n * DH; e += kNT * 8) {
-        Vec8<Tin> kx, vx;
-        kx.load(Kp + e);
-        vx.load(Vp + e);
-        int t = e / DH, i = e - t * DH;
+    // DH / 8 consecutive threads hold a token; they also form ||k_t||, which
+    // equals ||k_circ_t|| (a rotation keeps the norm).
+    {
+        constexpr int TPT = DH / 8;
+        const int iters = (n * DH + kNT * 8 - 1) / (kNT * 8);
+        for (int it = 0; it < iters; it++) {   // the same trip count for every thread
+            const int e = it * kNT * 8 + tid * 8;
+            const bool in = e < n * DH;
+            const int t = e / DH, i = e - t * DH;
+            float ss = 0.f;
+            if (in) {
+                Vec8<Tin> kx, vx;
+                kx.load(Kp + e);
+                vx.load(Vp + e);
 #pragma unroll
-        for (int q = 0; q < 8; q++) {
-            sm.kc[t][i + q] = kx.v[q];
-            sm.vv[t][i + q] = vx.v[q];
+                for (int q = 0; q < 8; q++) {
+                    sm.kc[t][i + q] = kx.v[q];
+                    sm.vv[t][i + q] = vx.v[q];
+                    ss = fmaf(kx.v[q], kx.v[q], ss);
+                }
+            }
+#pragma unroll
+            for (int o = 1; o < TPT; o <<= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+            if (in && i == 0) sm.kn[t] = sqrtf(ss);
         }
     }
     for (int t = tid; t < n; t += kNT) {
@@ -390,19 +405,30 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         }
     }
     // ---- k_circ = RoPE^-1(k, t) ----------------------------------------------
-    for (int e = tid; e < n * HALF; e += kNT) {
-        int t = e / HALF, i = e - t * HALF;
-        float2 cs = A.rope[(size_t)(sa + t) * HALF + i];
-        float x = sm.kc[t][i], y = sm.kc[t][i + HALF];
-        sm.kc[t][i] = x * cs.x + y * cs.y;
-        sm.kc[t][i + HALF] = y * cs.x - x * cs.y;
-    }
-    __syncthreads();
-    for (int t = warp; t < n; t += NWARPS) {
-        float s = 0.f;
-        for (int i = lane; i < DH; i += 32) s = fmaf(sm.kc[t][i], sm.kc[t][i], s);
-        s = warp_sum(s);
-        if (lane == 0) sm.kn[t] = sqrtf(s);
+    // batches of RB rotation-table loads are issued before any is used
+    {
+        constexpr int RB = 8;
+        for (int e0 = tid; e0 < n * HALF; e0 += kNT * RB) {
+            float2 cs[RB];
+#pragma unroll
+            for (int q = 0; q < RB; q++) {
+                const int e = e0 + q * kNT;
+                if (e < n * HALF) {
+                    const int t = e / HALF, i = e - t * HALF;
+                    cs[q] = A.rope[(size_t)(sa + t) * HALF + i];
+                }
+            }
+#pragma unroll
+            for (int q = 0; q < RB; q++) {
+                const int e = e0 + q * kNT;
+                if (e < n * HALF) {
+                    const int t = e / HALF, i = e - t * HALF;
+                    const float x = sm.kc[t][i], y = sm.kc[t][i + HALF];
+                    sm.kc[t][i] = x * cs[q].x + y * cs[q].y;
+                    sm.kc[t][i + HALF] = y * cs[q].x - x * cs[q].y;
+                }
+            }
+        }
     }
     // ---- tree state: a fresh root, or the unit's records so far --------------
     if (!A.resume) {
@@ -472,9 +498,13 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             const float wsum = rs + (float)nJ * beta;
             const float winv = 1.0f / (wsum + A.eps);
             const int p = round_half_even_mid(sa + ja, sa + jb);   // absolute positions
-            // lane owns the rotation pairs (i, i + d/2), i = PPL lane + j
+            // lane owns the rotation pairs (i, i + d/2), i = PPL lane + j; the
+            // rotation to p is loaded first so that its latency overlaps the sums
             constexpr int PPL = HALF / 32;
             const int i0 = lane * PPL;
+            float2 rot[PPL];
+#pragma unroll
+            for (int j = 0; j < PPL; j++) rot[j] = A.rope[(size_t)p * HALF + i0 + j];
             float m0[PPL], m1[PPL], v0[PPL], v1[PPL];
 #pragma unroll
             for (int j = 0; j < PPL; j++) m0[j] = m1[j] = v0[j] = v1[j] = 0.f;
@@ -499,7 +529,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             for (int j = 0; j < PPL; j++) {
                 const float a0 = m0[j] * ninv, a1 = m1[j] * ninv;
                 mu2 = fmaf(a0, a0, fmaf(a1, a1, mu2));
-                const float2 cs = A.rope[(size_t)p * HALF + i0 + j];
+                const float2 cs = rot[j];
                 sm.ktil[row][i0 + j] = a0 * cs.x - a1 * cs.y;
                 sm.ktil[row][i0 + j + HALF] = a0 * cs.y + a1 * cs.x;
                 sm.vtil[row][i0 + j] = v0[j] * winv;
