@@ -17,6 +17,8 @@
 //      order (U desc, unit asc, a asc, b desc) takes it.
 // Ties in U are therefore resolved exactly as the heap resolves them.
 //
+// The ops are the Add of every unit and the Split ops of the compact list the
+// unit kernel appends to as it evaluates nodes.
 // Kernels: alloc_hist (cost-weighted histogram of the 32-bit keys, three
 // passes of 11/11/10 bits), alloc_scan (pick the digit, one block), alloc_mark
 // (main set + units holding ties), alloc_ties (one block, units in order),
@@ -32,7 +34,9 @@ namespace {
 enum { ST_PREFIX = 0, ST_ABOVE, ST_ALL, ST_R, ST_ENDU, ST_ENDKEY, ST_TOTAL, ST_USED, ST_N };
 
 struct AllocArgs {
-    int64_t n_units, n_nodes;
+    int64_t n_units;
+    const uint2 *ops;        // Split ops built so far: (key bits, node index << 1 | cost - 1)
+    const unsigned int *n_ops;
     const float *u_U;        // Add keys (kappa = U)
     const float *nd_kappa;
     const int8_t *nd_cost;
@@ -49,22 +53,21 @@ struct AllocArgs {
     int *status;
 };
 
-__device__ __forceinline__ bool op_key(const AllocArgs &A, int64_t i, uint32_t &key, int &cost) {
+// Op i of the enumeration: the Add of unit i (i < n_units), else Split op
+// i - n_units of the compact list; v receives the node index (-1 for an Add).
+__device__ __forceinline__ void op_key(const AllocArgs &A, int64_t i, uint32_t &key, int &cost, int64_t &v) {
     if (i < A.n_units) {
-        float x = A.u_U[i];
-        key = __float_as_uint(x);
+        key = __float_as_uint(A.u_U[i]);
         cost = 1;
-        if (!(x >= 0.f) || isinf(x)) atomicOr(A.status, 8);
-        return true;
+        v = -1;
+    } else {
+        const uint2 o = A.ops[i - A.n_units];
+        key = o.x;
+        cost = (int)(o.y & 1u) + 1;
+        v = (int64_t)(o.y >> 1);
     }
-    int64_t v = i - A.n_units;
-    int c = A.nd_cost[v];
-    if (c <= 0) return false;
-    float x = A.nd_kappa[v];
+    const float x = __uint_as_float(key);
     if (!(x >= 0.f) || isinf(x)) atomicOr(A.status, 8);
-    key = __float_as_uint(x);
-    cost = c;
-    return true;
 }
 
 __global__ void alloc_hist_kernel(AllocArgs A, int shift, int nbits, uint32_t mask) {
@@ -93,30 +96,15 @@ __global__ void alloc_hist_kernel(AllocArgs A, int shift, int nbits, uint32_t ma
         if (in && (!(x >= 0.f) || isinf(x))) atomicOr(A.status, 8);
         consume(in, __float_as_uint(x), 1);
     }
-    // Split ops: 4 node slots per thread and step (one 32-bit load of their
-    // costs, one 16-byte load of their keys when any is an op)
-    const int64_t nq = A.n_nodes / 4;
-    for (int64_t q0 = w0; q0 < nq; q0 += stride) {
-        const int64_t q = q0 + lane;
-        const uint32_t cw = q < nq ? reinterpret_cast<const uint32_t *>(A.nd_cost)[q] : 0u;
-        float4 kv = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (cw) kv = reinterpret_cast<const float4 *>(A.nd_kappa)[q];
-        const float ks[4] = {kv.x, kv.y, kv.z, kv.w};
-#pragma unroll
-        for (int j = 0; j < 4; j++) {
-            const int c = (int)(int8_t)(cw >> (8 * j));
-            const bool op = c > 0;
-            if (op && (!(ks[j] >= 0.f) || isinf(ks[j]))) atomicOr(A.status, 8);
-            consume(op, __float_as_uint(ks[j]), c);
-        }
-    }
-    if (blockIdx.x == 0 && threadIdx.x < 32) {   // the last n_nodes % 4 slots
-        const int64_t v = 4 * nq + lane;
-        const bool in = v < A.n_nodes;
-        const int c = in ? (int)A.nd_cost[v] : 0;
-        const float x = c > 0 ? A.nd_kappa[v] : 0.f;
-        if (c > 0 && (!(x >= 0.f) || isinf(x))) atomicOr(A.status, 8);
-        consume(c > 0, __float_as_uint(x), c);
+    // Split ops of the compact list
+    const int64_t nops = *A.n_ops;
+    for (int64_t i0 = w0; i0 < nops; i0 += stride) {
+        const int64_t i = i0 + lane;
+        const bool in = i < nops;
+        const uint2 o = in ? A.ops[i] : make_uint2(0u, 0u);
+        const float x = __uint_as_float(o.x);
+        if (in && (!(x >= 0.f) || isinf(x))) atomicOr(A.status, 8);
+        consume(in, o.x, (int)(o.y & 1u) + 1);
     }
     __syncthreads();
     for (int b = threadIdx.x; b < nbin; b += blockDim.x)
@@ -180,18 +168,18 @@ __global__ void __launch_bounds__(1024) alloc_scan_kernel(AllocArgs A, int shift
 __global__ void alloc_mark_kernel(AllocArgs A) {
     const bool all = A.st[ST_ALL] != 0;
     const uint32_t tau = (uint32_t)A.st[ST_PREFIX];
-    const int64_t n = A.n_units + A.n_nodes;
+    const int64_t n = A.n_units + *A.n_ops;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
         uint32_t key;
         int cost;
-        if (!op_key(A, i, key, cost)) continue;
+        int64_t v;
+        op_key(A, i, key, cost, v);
         uint8_t s = (all || key > tau) ? 1 : 0;
-        if (i < A.n_units) {
+        if (v < 0) {
             A.u_sel[i] = s;
             if (!all && key == tau) A.u_flag[i] = 1;
         } else {
-            int64_t v = i - A.n_units;
             A.nd_sel[v] = s;
             if (!all && key == tau) A.u_flag[A.nd_unit[v]] = 1;
         }
@@ -295,7 +283,7 @@ __device__ __forceinline__ bool end_cand(const AllocArgs &A, int64_t i, float &U
         key = ((unsigned long long)i << 37) | ((unsigned long long)a << 17) | (0x1FFFFull - (unsigned)(b - a));
         return true;
     }
-    int64_t v = i - A.n_units;
+    const int64_t v = (int64_t)(A.ops[i - A.n_units].y >> 1);
     if (A.nd_cost[v] != 1 || A.nd_sel[v] != 0) return false;
     int32_t p = A.nd_parent[v];
     bool exposed = p < 0 ? A.u_sel[-2 - p] == 1 : A.nd_sel[p] == 1;
@@ -309,7 +297,7 @@ __device__ __forceinline__ bool end_cand(const AllocArgs &A, int64_t i, float &U
 
 __global__ void alloc_end_max_kernel(AllocArgs A) {
     if (A.st[ST_R] != 1) return;
-    const int64_t n = A.n_units + A.n_nodes;
+    const int64_t n = A.n_units + *A.n_ops;
     unsigned best = 0;
     bool any = false;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
@@ -327,7 +315,7 @@ __global__ void alloc_end_max_kernel(AllocArgs A) {
 __global__ void alloc_end_key_kernel(AllocArgs A) {
     if (A.st[ST_R] != 1 || A.st[ST_ENDU] == 0) return;
     const unsigned target = (unsigned)A.st[ST_ENDU] - 1u;
-    const int64_t n = A.n_units + A.n_nodes;
+    const int64_t n = A.n_units + *A.n_ops;
     unsigned long long best = ~0ull;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
@@ -341,7 +329,7 @@ __global__ void alloc_end_key_kernel(AllocArgs A) {
 }
 
 __global__ void alloc_end_pick_kernel(AllocArgs A) {
-    const int64_t n = A.n_units + A.n_nodes;
+    const int64_t n = A.n_units + *A.n_ops;
     const bool go = A.st[ST_R] == 1 && A.st[ST_ENDU] != 0;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
@@ -351,7 +339,7 @@ __global__ void alloc_end_pick_kernel(AllocArgs A) {
         if (!end_cand(A, i, U, k)) continue;
         if (k != A.st[ST_ENDKEY] || __float_as_uint(U) + 1u != (unsigned)A.st[ST_ENDU]) continue;
         if (i < A.n_units) A.u_sel[i] = 1;
-        else A.nd_sel[i - A.n_units] = 1;
+        else A.nd_sel[A.ops[i - A.n_units].y >> 1] = 1;
     }
 }
 
@@ -374,7 +362,7 @@ AllocArgs make_args(Ctx &c, int J) {
     Workspace &w = c.w;
     AllocArgs A;
     A.n_units = (int64_t)c.p.L * c.p.G * J;
-    A.n_nodes = c.node_cap;
+    A.ops = w.ops; A.n_ops = w.n_ops;
     A.u_U = w.u_Uadd; A.nd_kappa = w.nd_kappa; A.nd_cost = w.nd_cost; A.nd_U = w.nd_U;
     A.nd_a = w.nd_a; A.nd_b = w.nd_b; A.nd_parent = w.nd_parent; A.nd_unit = w.nd_unit;
     A.nd_child0 = w.nd_child0; A.nd_nchild = w.nd_nchild; A.u_nnodes = w.u_nnodes;
@@ -476,7 +464,7 @@ __global__ void slot_classes_kernel(const int32_t *slots, int J, int32_t *list, 
 cudaError_t launch_threshold(Ctx &c, int J, cudaStream_t s) {
     AllocArgs A = make_args(c, J);
     alloc_init_kernel<<<1, 256, 0, s>>>(c.w.alloc_state, c.w.hist);
-    const int blocks = grid_for(c, A.n_units + A.n_nodes);
+    const int blocks = grid_for(c, A.n_units + c.node_cap / 2);
     const int shifts[3] = {21, 10, 0};
     const int bits[3] = {11, 11, 10};
     uint32_t mask = 0;
@@ -528,7 +516,7 @@ cudaError_t launch_allocate(Ctx &c, int J, cudaStream_t s) {
     cudaMemsetAsync(w.u_count, 0, sizeof(int32_t) * A.n_units, s);
     cudaError_t e = launch_threshold(c, J, s);
     if (e != cudaSuccess) return e;
-    const int blocks = grid_for(c, A.n_units + A.n_nodes);
+    const int blocks = grid_for(c, A.n_units + c.node_cap / 2);
     alloc_mark_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_ties_kernel<<<1, 1024, 0, s>>>(A);
     alloc_end_max_kernel<<<blocks, 256, 0, s>>>(A);

@@ -203,6 +203,10 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
                                                              std::max(1, p.T / 256)));
     if (gkv::use_tc(c)) c.n_chunks = std::max(c.n_chunks, gkv::tc_row_chunks(c));
     c.node_cap = LG * 2 * Nc;
+    if (c.node_cap >= (1LL << 31)) {   // node records are addressed with int32
+        delete x;
+        return GKV_EINVAL;
+    }
     const int nb = p.n_max - p.n_min + 1;
     const int64_t nrow = (int64_t)p.L * p.Hq * p.W;
     gkv::Workspace &w = c.w;
@@ -227,6 +231,7 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
               dalloc(x, &w.nd_cost, (size_t)c.node_cap) && dalloc(x, &w.nd_D, (size_t)c.node_cap) &&
               dalloc(x, &w.nd_R, (size_t)c.node_cap) && dalloc(x, &w.nd_U, (size_t)c.node_cap) &&
               dalloc(x, &w.nd_kappa, (size_t)c.node_cap) && dalloc(x, &w.nd_sel, (size_t)c.node_cap) &&
+              dalloc(x, &w.ops, (size_t)c.node_cap / 2 + 1) && dalloc(x, &w.n_ops, 1) &&
               dalloc(x, &w.hist, 2048) && dalloc(x, &w.alloc_state, 16) && dalloc(x, &w.work, 4) &&
               dalloc(x, &w.pend_hist, 1 << 16) && dalloc(x, &w.pend_cut, 1) && dalloc(x, &w.pend_n, 1) &&
               dalloc(x, &w.pend_pot, 1);
@@ -365,6 +370,7 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
     if (e == cudaSuccess && !root_only)
         e = cudaMemcpyAsync(w.pend_cut, &kNoCut, sizeof(float), cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = cudaMemsetAsync(w.work, 0, 4 * sizeof(unsigned long long), s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(w.n_ops, 0, sizeof(unsigned int), s);
     if (e == cudaSuccess) {
         int cnt[2] = {0, 0};
         {

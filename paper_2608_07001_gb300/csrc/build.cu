@@ -74,6 +74,8 @@ struct BuildArgs {
     float *nd_D;
     float *nd_R, *nd_U, *nd_kappa;
     uint8_t *nd_sel;
+    uint2 *ops;                  // compact list of the Split ops (allocation input)
+    unsigned int *n_ops;
     int32_t *u_nnodes;
     float *u_Uadd, *u_Ddrop, *u_pend;
     uint8_t *u_sel;
@@ -983,6 +985,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     A.nd_child0[gv] = child0; A.nd_nchild[gv] = (int8_t)nch;
                     A.nd_cost[gv] = (int8_t)cost; A.nd_U[gv] = U; A.nd_kappa[gv] = kap;
                     A.nd_sel[gv] = 0;
+                    A.ops[atomicAdd(A.n_ops, 1u)] = make_uint2(__float_as_uint(kap), ((uint32_t)gv << 1) | (uint32_t)(cost - 1));
                 }
                 if (lane < nch) {   // lane q writes child q
                     const int q = lane, ci = child0 + q;
@@ -1083,6 +1086,7 @@ cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *
     A.nd_a = c.w.nd_a; A.nd_b = c.w.nd_b; A.nd_child0 = c.w.nd_child0;
     A.nd_parent = c.w.nd_parent; A.nd_unit = c.w.nd_unit;
     A.nd_nchild = c.w.nd_nchild; A.nd_cost = c.w.nd_cost;
+    A.ops = c.w.ops; A.n_ops = c.w.n_ops;
     A.nd_D = c.w.nd_D; A.nd_R = c.w.nd_R; A.nd_U = c.w.nd_U; A.nd_kappa = c.w.nd_kappa;
     A.nd_sel = c.w.nd_sel;
     A.u_nnodes = c.w.u_nnodes; A.u_Uadd = c.w.u_Uadd; A.u_Ddrop = c.w.u_Ddrop; A.u_sel = c.w.u_sel;

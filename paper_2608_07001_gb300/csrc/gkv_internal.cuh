@@ -54,6 +54,8 @@ struct Workspace {
                                    // exactly the value their parent computed)
     float *nd_R = nullptr, *nd_U = nullptr, *nd_kappa = nullptr;
     uint8_t *nd_sel = nullptr;     // split selected (1), discarded tie (2)
+    uint2 *ops = nullptr;          // [node_cap / 2] Split ops built so far: (key bits, node << 1 | cost - 1)
+    unsigned int *n_ops = nullptr; // [1] entries of ops
     // per-unit arrays (capacity units_cap), unit id = lg * J + j
     int64_t units_cap = 0;
     int32_t *u_nnodes = nullptr;
