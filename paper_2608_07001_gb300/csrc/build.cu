@@ -51,6 +51,9 @@ constexpr int kMaxCuts = 18;     // K + midpoint, K <= 16 (+1 spare)
 constexpr int kNT = 256;         // threads per CTA
 constexpr int kNPP = 32;         // probe pairs: thread handles probes p and p + 32 (W <= 64)
 constexpr int kNCL = 8;          // threads per probe pair (4-element groups, interleaved)
+constexpr int kPPW = 32 / kNCL;  // probe pairs per warp: lane = 4 c + (pair % 4), so that the
+                                 // 4 lanes reading one 16-byte chunk are adjacent (one shared-
+                                 // memory wavefront serves them; lanes 8 apart would not merge)
 constexpr int kNCD = 19;         // candidate intervals per direction and batch: 17 cuts + p* side + whole node
 
 struct BuildArgs {
@@ -291,8 +294,8 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         sm.Rt[t] = A.rtok[(size_t)lg * A.Nc + (sa - A.cs) + t];
     }
     // probe registers: thread (pp, c) owns probes pp and pp + 32, elements
-    // 4 c + 32 g + j, so that 8 consecutive threads read 128 contiguous bytes
-    const int pp = tid / kNCL, c = tid - pp * kNCL;
+    // 4 c + 32 g + j; the 8 chunk lanes of a pair read 128 contiguous bytes
+    const int c = lane / kPPW, pp = warp * kPPW + (lane & (kPPW - 1));
     float2 qa0[CH / 2], qa1[CH / 2];   // q of the two probes as element pairs
     float mu0 = 0.f, mu1 = 0.f, invZ0 = 0.f, invZ1 = 0.f;
 #pragma unroll
@@ -374,7 +377,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             }
             float y0 = x0.x + x0.y, y1 = x1.x + x1.y;
 #pragma unroll
-            for (int o = 1; o < kNCL; o <<= 1) {
+            for (int o = kPPW; o < 32; o <<= 1) {   // over the pair's chunk lanes
                 y0 += __shfl_xor_sync(0xffffffffu, y0, o);
                 y1 += __shfl_xor_sync(0xffffffffu, y1, o);
             }
@@ -566,7 +569,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         }
         float x0 = xa.x + xa.y, x1 = xb.x + xb.y;
 #pragma unroll
-        for (int o = 1; o < kNCL; o <<= 1) {
+        for (int o = kPPW; o < 32; o <<= 1) {   // over the pair's chunk lanes
             x0 += __shfl_xor_sync(0xffffffffu, x0, o);
             x1 += __shfl_xor_sync(0xffffffffu, x1, o);
         }
@@ -591,7 +594,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         }
         float res0 = r0.x + r0.y, res1 = r1.x + r1.y, mm0 = m0.x + m0.y, mm1 = m1.x + m1.y;
 #pragma unroll
-        for (int o = 1; o < kNCL; o <<= 1) {
+        for (int o = kPPW; o < 32; o <<= 1) {
             res0 += __shfl_xor_sync(0xffffffffu, res0, o);
             res1 += __shfl_xor_sync(0xffffffffu, res1, o);
             mm0 += __shfl_xor_sync(0xffffffffu, mm0, o);
@@ -606,7 +609,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         const float p0 = Z0 * invZ0, p1 = Z1 * invZ1;
         float pd = fmaf(p0, D0, p1 * D1), pw = p0 + p1;
 #pragma unroll
-        for (int o = kNCL; o < 32; o <<= 1) {
+        for (int o = 1; o < kPPW; o <<= 1) {   // over the warp's probe pairs
             pd += __shfl_xor_sync(0xffffffffu, pd, o);
             pw += __shfl_xor_sync(0xffffffffu, pw, o);
         }
