@@ -207,7 +207,8 @@ struct Smem {
     static constexpr int NWARPS = kNT / 32;
     static constexpr int NB = 16;            // nodes per batch
     static constexpr int MAXNODES = 2 * NMAX;
-    float kc[NMAX][DH];
+    float kc[NMAX][DH + 8];                  // rows padded by 32 B: the probe-weight MMA reads
+                                             // 8 rows at once, which then fall in distinct banks
     float vv[NMAX][DH];                      // values, converted once to fp32
     float2 E[NMAX][kNPP];                    // probe weights of probes (p, p + 32)
     float ktil[kNCD][DH];                    // prototypes of one direction at a time
