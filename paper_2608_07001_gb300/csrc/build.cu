@@ -135,6 +135,32 @@ __device__ __forceinline__ double okey_inv(unsigned long long k) {
     return __longlong_as_double((long long)u);
 }
 
+// 8 consecutive input elements held raw in registers (the load is issued
+// first, the conversion to fp32 happens at get).
+template <typename T> struct Raw8;
+template <> struct Raw8<float> {
+    float4 a, b;
+    __device__ __forceinline__ void load(const float *p) {
+        a = reinterpret_cast<const float4 *>(p)[0];
+        b = reinterpret_cast<const float4 *>(p)[1];
+    }
+    __device__ __forceinline__ void get(float v[8]) const {
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    }
+};
+template <> struct Raw8<__nv_bfloat16> {
+    uint4 u;
+    __device__ __forceinline__ void load(const __nv_bfloat16 *p) { u = *reinterpret_cast<const uint4 *>(p); }
+    __device__ __forceinline__ void get(float v[8]) const {
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int i = 0; i < 4; i++) {   // bf16 -> fp32 is exact: the bits move to the high half
+            v[2 * i] = __uint_as_float(w[i] << 16);
+            v[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+        }
+    }
+};
+
 __device__ __forceinline__ int round_half_even_mid(int a, int b) {
     int s = a + b - 1;
     if ((s & 1) == 0) return s >> 1;
@@ -264,35 +290,52 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     const float om = A.omega ? A.omega[lg] : 1.0f;
 
     // ---- load the slot ------------------------------------------------------
-    // DH / 8 consecutive threads hold a token; they also form ||k_t||, which
-    // equals ||k_circ_t|| (a rotation keeps the norm).
+    // Every global load of a group is issued before any is used.  DH / 8
+    // consecutive threads hold a token; they also form ||k_t||, which equals
+    // ||k_circ_t|| (a rotation keeps the norm).
     {
-        constexpr int TPT = DH / 8;
+        const bool own = tid < n;
+        const double kapv = own ? A.kappa[sa + tid] : 0.0;
+        const float rtv = own ? A.rtok[(size_t)lg * A.Nc + (sa - A.cs) + tid] : 0.f;
+        constexpr int TPT = DH / 8, GRP = 4;
         const int iters = (n * DH + kNT * 8 - 1) / (kNT * 8);
-        for (int it = 0; it < iters; it++) {   // the same trip count for every thread
-            const int e = it * kNT * 8 + tid * 8;
-            const bool in = e < n * DH;
-            const int t = e / DH, i = e - t * DH;
-            float ss = 0.f;
-            if (in) {
-                Vec8<Tin> kx, vx;
-                kx.load(Kp + e);
-                vx.load(Vp + e);
+        for (int i0 = 0; i0 < iters; i0 += GRP) {   // the same trip counts for every thread
+            Raw8<Tin> kr[GRP], vr[GRP];
 #pragma unroll
-                for (int q = 0; q < 8; q++) {
-                    sm.kc[t][i + q] = kx.v[q];
-                    sm.vv[t][i + q] = vx.v[q];
-                    ss = fmaf(kx.v[q], kx.v[q], ss);
+            for (int q = 0; q < GRP; q++) {
+                const int e = (i0 + q) * kNT * 8 + tid * 8;
+                if (i0 + q < iters && e < n * DH) {
+                    kr[q].load(Kp + e);
+                    vr[q].load(Vp + e);
                 }
             }
 #pragma unroll
-            for (int o = 1; o < TPT; o <<= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-            if (in && i == 0) sm.kn[t] = sqrtf(ss);
+            for (int q = 0; q < GRP; q++) {
+                if (i0 + q >= iters) break;
+                const int e = (i0 + q) * kNT * 8 + tid * 8;
+                const bool in = e < n * DH;
+                const int t = e / DH, i = e - t * DH;
+                float ss = 0.f;
+                if (in) {
+                    float kx[8], vx[8];
+                    kr[q].get(kx);
+                    vr[q].get(vx);
+#pragma unroll
+                    for (int u = 0; u < 8; u++) {
+                        sm.kc[t][i + u] = kx[u];
+                        sm.vv[t][i + u] = vx[u];
+                        ss = fmaf(kx[u], kx[u], ss);
+                    }
+                }
+#pragma unroll
+                for (int o = 1; o < TPT; o <<= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+                if (in && i == 0) sm.kn[t] = sqrtf(ss);
+            }
         }
-    }
-    for (int t = tid; t < n; t += kNT) {
-        sm.kap[t] = okey(A.kappa[sa + t]);
-        sm.Rt[t] = A.rtok[(size_t)lg * A.Nc + (sa - A.cs) + t];
+        for (int t = tid; t < n; t += kNT) {
+            sm.kap[t] = okey(t == tid ? kapv : A.kappa[sa + t]);
+            sm.Rt[t] = t == tid ? rtv : A.rtok[(size_t)lg * A.Nc + (sa - A.cs) + t];
+        }
     }
     // probe registers: thread (pp, c) owns probes pp and pp + 32, elements
     // 4 c + 32 g + j; the 8 chunk lanes of a pair read 128 contiguous bytes

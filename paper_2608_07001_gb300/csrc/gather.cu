@@ -13,9 +13,9 @@
 // Kernels: gather_count (frontier entries per unit), gather_scan (one block,
 // ordered exclusive scan -> per-unit and per-(l, g) offsets), gather_list
 // (warp per unit, depth-first in ascending position: entry descriptors by
-// output position), gather_emit (persistent warps, one entry at a time:
-// prototypes or single-token copies), gather_tokens (prefix / recent / suffix
-// copies).
+// output position), gather_emit (persistent warps, one entry at a time, rows
+// streamed through a per-warp cp.async ring: prototypes or single-token
+// copies), gather_tokens (prefix / recent / suffix copies).
 #include "gkv_internal.cuh"
 
 #include <algorithm>
@@ -100,6 +100,37 @@ __global__ void __launch_bounds__(1024) gather_scan_kernel(GatherArgs A) {
         for (int lg = 0; lg <= A.L * A.G; lg++) A.offsets[lg] = (long long)lg * extra;
 }
 
+// 8 consecutive elements held raw (loaded from shared memory, converted to
+// fp32 on get, or stored back bit for bit).
+template <typename T> struct Raw8;
+template <> struct Raw8<float> {
+    float4 a, b;
+    __device__ __forceinline__ void load_shared(const float *p) {
+        a = reinterpret_cast<const float4 *>(p)[0];
+        b = reinterpret_cast<const float4 *>(p)[1];
+    }
+    __device__ __forceinline__ void get(float v[8]) const {
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    }
+    __device__ __forceinline__ void store(float *p) const {
+        reinterpret_cast<float4 *>(p)[0] = a;
+        reinterpret_cast<float4 *>(p)[1] = b;
+    }
+};
+template <> struct Raw8<__nv_bfloat16> {
+    uint4 u;
+    __device__ __forceinline__ void load_shared(const __nv_bfloat16 *p) { u = *reinterpret_cast<const uint4 *>(p); }
+    __device__ __forceinline__ void get(float v[8]) const {
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int i = 0; i < 4; i++) {   // bf16 -> fp32 is exact: the bits move to the high half
+            v[2 * i] = __uint_as_float(w[i] << 16);
+            v[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+        }
+    }
+    __device__ __forceinline__ void store(__nv_bfloat16 *p) const { *reinterpret_cast<uint4 *>(p) = u; }
+};
+
 // 8 consecutive elements copied bit for bit.
 __device__ __forceinline__ void copy8(__nv_bfloat16 *dst, const __nv_bfloat16 *src) {
     *reinterpret_cast<uint4 *>(dst) = *reinterpret_cast<const uint4 *>(src);
@@ -118,127 +149,6 @@ __device__ __forceinline__ void store8(__nv_bfloat16 *dst, const float v[8]) {
 __device__ __forceinline__ void store8(float *dst, const float v[8]) {
     reinterpret_cast<float4 *>(dst)[0] = make_float4(v[0], v[1], v[2], v[3]);
     reinterpret_cast<float4 *>(dst)[1] = make_float4(v[4], v[5], v[6], v[7]);
-}
-
-// One frontier node [a, b) of head lg -> cache entry e (one warp).  Rows are
-// read as 8-element chunks, LPR = d / 8 lanes per row and 32 / LPR rows per
-// group, U groups in flight; the chunk holding elements i .. i+7 of the first
-// half and the one holding i + d/2 .. of the second half sit PX = LPR / 2
-// lanes apart, so the rotation partner comes from a shuffle.  The key
-// prototype RoPE(mean_t RoPE^-1(k_t, t), p) is formed as mean_t of k_t rotated
-// by p - t (rotations compose), from a table of the 2 n_max - 1 offsets; its
-// norm equals the norm of the mean inverse-rotated key.  The value prototype
-// uses sum_t (R_t + beta) v_t = sum R v + beta sum v.  All arithmetic is fp32.
-template <typename Tin, int DH>
-__device__ void emit_node(const GatherArgs &A, int lg, int a, int b, int64_t e, int lane) {
-    constexpr int HALF = DH / 2, LPR = DH / 8, RPW = 32 / LPR, PX = LPR / 2, U = 3;
-    const int r = lane / LPR, c = lane - r * LPR;
-    const bool hi = c >= PX;                   // chunk in the second half
-    const int i0 = 8 * (c - (hi ? PX : 0));    // pair index of the chunk's first element
-    const Tin *K = static_cast<const Tin *>(A.K) + (size_t)lg * A.T * DH;
-    const Tin *V = static_cast<const Tin *>(A.V) + (size_t)lg * A.T * DH;
-    Tin *Ko = static_cast<Tin *>(A.K_out) + (size_t)e * DH;
-    Tin *Vo = static_cast<Tin *>(A.V_out) + (size_t)e * DH;
-    const int n = b - a;
-    if (n == 1) {   // single token: original bits, p = t, log m = 0
-        if (lane < LPR) {
-            copy8(Ko + 8 * c, K + (size_t)a * DH + 8 * c);
-            copy8(Vo + 8 * c, V + (size_t)a * DH + 8 * c);
-        }
-        if (lane == 0) { A.pos[e] = a; A.log_m[e] = 0.f; A.src_lo[e] = a; A.src_hi[e] = b; }
-        return;
-    }
-    const float *R = A.rtok + (size_t)lg * A.Nc - A.cs;
-    const int p = round_half_even_mid(a, b);
-    float mk[8], sv[8], srv[8], kn = 0.f, rs = 0.f;
-#pragma unroll
-    for (int j = 0; j < 8; j++) mk[j] = sv[j] = srv[j] = 0.f;
-    for (int t0 = a; t0 < b; t0 += U * RPW) {
-        Vec8<Tin> kx[U], vx[U];
-        float rr[U];
-        int tt[U];
-#pragma unroll
-        for (int g = 0; g < U; g++) {   // issue every group's loads first
-            const int t = t0 + g * RPW + r;
-            const bool ok = t < b;
-            tt[g] = ok ? t : b - 1;
-            if (ok) {
-                kx[g].load(K + (size_t)t * DH + 8 * c);
-                vx[g].load(V + (size_t)t * DH + 8 * c);
-                rr[g] = R[t];
-            } else {
-#pragma unroll
-                for (int j = 0; j < 8; j++) kx[g].v[j] = vx[g].v[j] = 0.f;
-                rr[g] = 0.f;
-            }
-        }
-#pragma unroll
-        for (int g = 0; g < U; g++) {
-            float y[8], nn = 0.f;
-#pragma unroll
-            for (int j = 0; j < 8; j++) {
-                y[j] = __shfl_xor_sync(0xffffffffu, kx[g].v[j], PX);
-                nn = fmaf(kx[g].v[j], kx[g].v[j], nn);
-            }
-#pragma unroll
-            for (int o = 1; o < LPR; o <<= 1) nn += __shfl_xor_sync(0xffffffffu, nn, o);
-            if (c == 0) kn += sqrtf(nn);   // |k_t| (rows past b are zero)
-            rs += rr[g];
-            const float4 *cs4 = reinterpret_cast<const float4 *>(
-                A.rope_rel + (size_t)(p - tt[g] + kMaxUnit - 1) * HALF + i0);
-#pragma unroll
-            for (int j2 = 0; j2 < 4; j2++) {
-                const float4 q = cs4[j2];          // (cos, sin) of pairs i0 + 2 j2, i0 + 2 j2 + 1
-                const float cc[2] = {q.x, q.z}, sn[2] = {q.y, q.w};
-#pragma unroll
-                for (int h = 0; h < 2; h++) {
-                    const int j = 2 * j2 + h;
-                    // rotation by p - t: x' = x cos - y sin, y' = x sin + y cos
-                    mk[j] += hi ? fmaf(kx[g].v[j], cc[h], y[j] * sn[h]) : fmaf(kx[g].v[j], cc[h], -y[j] * sn[h]);
-                    sv[j] += vx[g].v[j];
-                    srv[j] = fmaf(rr[g], vx[g].v[j], srv[j]);
-                }
-            }
-        }
-    }
-    // combine the row groups
-#pragma unroll
-    for (int o = LPR; o < 32; o <<= 1) {
-#pragma unroll
-        for (int j = 0; j < 8; j++) {
-            mk[j] += __shfl_xor_sync(0xffffffffu, mk[j], o);
-            sv[j] += __shfl_xor_sync(0xffffffffu, sv[j], o);
-            srv[j] += __shfl_xor_sync(0xffffffffu, srv[j], o);
-        }
-        kn += __shfl_xor_sync(0xffffffffu, kn, o);
-        rs += __shfl_xor_sync(0xffffffffu, rs, o);
-    }
-    kn = __shfl_sync(0xffffffffu, kn, 0);
-    const float ninv = 1.0f / (float)n;
-    const float beta = (float)A.base_frac * (rs * ninv);
-    const float winv = 1.0f / (rs + (float)n * beta + (float)A.eps);
-    float ko[8], vo[8], mu2 = 0.f;
-#pragma unroll
-    for (int j = 0; j < 8; j++) {
-        ko[j] = mk[j] * ninv;
-        vo[j] = fmaf(beta, sv[j], srv[j]) * winv;
-        mu2 = fmaf(ko[j], ko[j], mu2);
-    }
-#pragma unroll
-    for (int o = 1; o < LPR; o <<= 1) mu2 += __shfl_xor_sync(0xffffffffu, mu2, o);
-    if (lane < LPR) {
-        store8(Ko + 8 * c, ko);
-        store8(Vo + 8 * c, vo);
-    }
-    if (lane == 0) {
-        const float coh = sqrtf(mu2) / (kn * ninv + (float)A.eps);
-        float me = (float)n * coh * coh;
-        me = me < 1.0f ? 1.0f : (me > (float)n ? (float)n : me);
-        A.pos[e] = p;
-        A.log_m[e] = logf(me);
-        A.src_lo[e] = a;
-        A.src_hi[e] = b;
-    }
 }
 
 // Frontier entries of every covered unit in ascending position (warp per
@@ -268,16 +178,193 @@ __global__ void gather_list_kernel(GatherArgs A) {
     }
 }
 
-// Prototypes of the listed entries: persistent warps, one entry at a time.
+// Prototypes of the listed entries (one warp per entry; rows read as
+// 8-element chunks, LPR = d / 8 lanes per row and RPW = 32 / LPR rows per step).
+// Each warp walks its entries (warp id, + number of warps, ...) as one stream of
+// steps; the K and V rows and token values of step s + D - 1 are copied into
+// the warp's ring of D steps (cp.async, zero-filled past an entry's end) while
+// step s is consumed, so D - 1 steps of loads stay in flight across entry
+// boundaries.  The chunk holding elements i .. i+7 of the first half of a key
+// and the one holding i + d/2 .. sit PX = LPR / 2 lanes apart, so the rotation
+// partner comes from a shuffle.  The key prototype RoPE(mean_t RoPE^-1(k_t, t),
+// p) is formed as mean_t of k_t rotated by p - t (rotations compose), from a
+// table of the 2 n_max - 1 offsets; its norm equals the norm of the mean
+// inverse-rotated key.  The value prototype uses sum_t (R_t + beta) v_t =
+// sum R v + beta sum v.  All arithmetic is fp32.
+constexpr int kRingSteps = 8;
+
+template <typename Tin, int DH>
+struct EmitGeom {
+    static constexpr int LPR = DH / 8, RPW = 32 / LPR, PX = LPR / 2;
+    static constexpr int KB = DH * (int)sizeof(Tin);      // bytes of a K (or V) row
+    static constexpr int RB = 2 * KB;                      // ring bytes of a row: K, then V
+    static constexpr int CPR = RB / 16;                    // 16-byte chunks of a ring row
+    static constexpr int WARP_BYTES = kRingSteps * RPW * (RB + 4);
+};
+
+__device__ __forceinline__ void cp_async4(void *smem, const void *gmem, bool pred) {
+    unsigned s = (unsigned)__cvta_generic_to_shared(smem);
+    int n = pred ? 4 : 0;
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(s), "l"(gmem), "r"(n));
+}
+
 template <typename Tin, int DH>
 __global__ void __launch_bounds__(256, 2) gather_emit_kernel(GatherArgs A, int64_t n_ent) {
-    const int lane = threadIdx.x & 31;
+    using Gm = EmitGeom<Tin, DH>;
+    constexpr int HALF = DH / 2, LPR = Gm::LPR, RPW = Gm::RPW, PX = Gm::PX, RB = Gm::RB, CPR = Gm::CPR;
+    constexpr int D = kRingSteps;
+    extern __shared__ __align__(16) unsigned char gsm[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    unsigned char *ring = gsm + (size_t)warp * Gm::WARP_BYTES;
+    float *rring = reinterpret_cast<float *>(ring + D * RPW * RB);
     const int64_t nw = (int64_t)gridDim.x * 8;
-    for (int64_t e = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5); e < n_ent; e += nw) {
-        const int4 en = A.ent[e];
-        if (en.w == 0) continue;   // prefix / recent / suffix token (gather_tokens)
-        emit_node<Tin, DH>(A, en.z, en.x, en.y, e, lane);
+    const int r = lane / LPR, c = lane - r * LPR;
+    const bool hi = c >= PX;                   // chunk in the second half
+    const int i0 = 8 * (c - (hi ? PX : 0));    // pair index of the chunk's first element
+
+    struct Cur { int64_t e; int s, nst, lg, a, b; };
+    // first compressible entry at or after e in this warp's sequence
+    auto seek = [&](Cur &cu, int64_t e) {
+        for (; e < n_ent; e += nw) {
+            const int4 en = A.ent[e];
+            if (en.w == 0) continue;   // prefix / recent / suffix token (gather_tokens)
+            cu.e = e; cu.s = 0; cu.lg = en.z; cu.a = en.x; cu.b = en.y;
+            cu.nst = (en.y - en.x + RPW - 1) / RPW;
+            return;
+        }
+        cu.e = n_ent;
+    };
+    Cur pf, cs;
+    seek(pf, (int64_t)blockIdx.x * 8 + warp);
+    cs = pf;
+    // copy the prefetch cursor's step into ring slot `slot` and advance it
+    auto issue = [&](int slot) {
+        if (pf.e < n_ent) {
+            const char *K = static_cast<const char *>(A.K) + (size_t)pf.lg * A.T * Gm::KB;
+            const char *V = static_cast<const char *>(A.V) + (size_t)pf.lg * A.T * Gm::KB;
+            const int t0 = pf.a + pf.s * RPW;
+#pragma unroll
+            for (int q = lane; q < RPW * CPR; q += 32) {
+                const int rr = q / CPR, ch = q - rr * CPR;
+                const int t = t0 + rr;
+                const bool ok = t < pf.b;
+                const size_t row = (size_t)(ok ? t : pf.a) * Gm::KB;
+                const char *src = ch < CPR / 2 ? K + row + ch * 16 : V + row + (ch - CPR / 2) * 16;
+                cp_async16(ring + ((size_t)slot * RPW + rr) * RB + ch * 16, src, ok);
+            }
+            if (lane < RPW) {
+                const int t = t0 + lane;
+                const bool ok = t < pf.b;
+                cp_async4(&rring[slot * RPW + lane], A.rtok + (size_t)pf.lg * A.Nc + ((ok ? t : pf.a) - A.cs), ok);
+            }
+            if (++pf.s == pf.nst) seek(pf, pf.e + nw);
+        }
+        cp_async_commit();
+    };
+    for (int q = 0; q < D - 1; q++) issue(q);
+    int slot = 0;
+    while (cs.e < n_ent) {
+        const int lg = cs.lg, a = cs.a, b = cs.b, n = b - a;
+        const int64_t e = cs.e;
+        Tin *Ko = static_cast<Tin *>(A.K_out) + (size_t)e * DH;
+        Tin *Vo = static_cast<Tin *>(A.V_out) + (size_t)e * DH;
+        const int p = round_half_even_mid(a, b);
+        float mk[8], sv[8], srv[8], kn = 0.f, rs = 0.f;
+#pragma unroll
+        for (int j = 0; j < 8; j++) mk[j] = sv[j] = srv[j] = 0.f;
+        for (int st = 0; st < cs.nst; st++) {
+            issue((slot + D - 1) % D);   // the slot consumed last
+            cp_async_wait<D - 1>();      // this step's group has landed
+            __syncwarp();
+            const unsigned char *row = ring + ((size_t)slot * RPW + r) * RB;
+            Raw8<Tin> kraw, vraw;
+            kraw.load_shared(reinterpret_cast<const Tin *>(row) + 8 * c);
+            vraw.load_shared(reinterpret_cast<const Tin *>(row + Gm::KB) + 8 * c);
+            const float rr = rring[slot * RPW + r];
+            const int t = a + st * RPW + r;
+            const int tt = t < b ? t : b - 1;   // rows past b are zero
+            if (n == 1) {   // single token: original bits, p = t, log m = 0
+                if (lane < LPR) {
+                    kraw.store(Ko + 8 * c);
+                    vraw.store(Vo + 8 * c);
+                }
+            } else {
+                float kx[8], vx[8], y[8], nn = 0.f;
+                kraw.get(kx);
+                vraw.get(vx);
+#pragma unroll
+                for (int j = 0; j < 8; j++) {
+                    y[j] = __shfl_xor_sync(0xffffffffu, kx[j], PX);
+                    nn = fmaf(kx[j], kx[j], nn);
+                }
+#pragma unroll
+                for (int o = 1; o < LPR; o <<= 1) nn += __shfl_xor_sync(0xffffffffu, nn, o);
+                if (c == 0) kn += sqrtf(nn);   // |k_t|
+                rs += rr;
+                const float4 *cs4 = reinterpret_cast<const float4 *>(
+                    A.rope_rel + (size_t)(p - tt + kMaxUnit - 1) * HALF + i0);
+#pragma unroll
+                for (int j2 = 0; j2 < 4; j2++) {
+                    const float4 q = cs4[j2];          // (cos, sin) of pairs i0 + 2 j2, i0 + 2 j2 + 1
+                    const float cc[2] = {q.x, q.z}, sn[2] = {q.y, q.w};
+#pragma unroll
+                    for (int h = 0; h < 2; h++) {
+                        const int j = 2 * j2 + h;
+                        // rotation by p - t: x' = x cos - y sin, y' = x sin + y cos
+                        mk[j] += hi ? fmaf(kx[j], cc[h], y[j] * sn[h]) : fmaf(kx[j], cc[h], -y[j] * sn[h]);
+                        sv[j] += vx[j];
+                        srv[j] = fmaf(rr, vx[j], srv[j]);
+                    }
+                }
+            }
+            __syncwarp();   // the slot may be refilled by the next issue
+            slot = slot + 1 == D ? 0 : slot + 1;
+        }
+        if (n == 1) {
+            if (lane == 0) { A.pos[e] = a; A.log_m[e] = 0.f; A.src_lo[e] = a; A.src_hi[e] = b; }
+        } else {
+            // combine the row groups
+#pragma unroll
+            for (int o = LPR; o < 32; o <<= 1) {
+#pragma unroll
+                for (int j = 0; j < 8; j++) {
+                    mk[j] += __shfl_xor_sync(0xffffffffu, mk[j], o);
+                    sv[j] += __shfl_xor_sync(0xffffffffu, sv[j], o);
+                    srv[j] += __shfl_xor_sync(0xffffffffu, srv[j], o);
+                }
+                kn += __shfl_xor_sync(0xffffffffu, kn, o);
+                rs += __shfl_xor_sync(0xffffffffu, rs, o);
+            }
+            kn = __shfl_sync(0xffffffffu, kn, 0);
+            const float ninv = 1.0f / (float)n;
+            const float beta = (float)A.base_frac * (rs * ninv);
+            const float winv = 1.0f / (rs + (float)n * beta + (float)A.eps);
+            float ko[8], vo[8], mu2 = 0.f;
+#pragma unroll
+            for (int j = 0; j < 8; j++) {
+                ko[j] = mk[j] * ninv;
+                vo[j] = fmaf(beta, sv[j], srv[j]) * winv;
+                mu2 = fmaf(ko[j], ko[j], mu2);
+            }
+#pragma unroll
+            for (int o = 1; o < LPR; o <<= 1) mu2 += __shfl_xor_sync(0xffffffffu, mu2, o);
+            if (lane < LPR) {
+                store8(Ko + 8 * c, ko);
+                store8(Vo + 8 * c, vo);
+            }
+            if (lane == 0) {
+                const float coh = sqrtf(mu2) / (kn * ninv + (float)A.eps);
+                float me = (float)n * coh * coh;
+                me = me < 1.0f ? 1.0f : (me > (float)n ? (float)n : me);
+                A.pos[e] = p;
+                A.log_m[e] = logf(me);
+                A.src_lo[e] = a;
+                A.src_hi[e] = b;
+            }
+        }
+        seek(cs, cs.e + nw);
     }
+    cp_async_wait<0>();
 }
 
 template <typename Tin>
@@ -297,6 +384,22 @@ __global__ void gather_tokens_kernel(GatherArgs A) {
     Tin *Vo = static_cast<Tin *>(A.V_out) + (size_t)e * A.d;
     for (int i = lane; i < A.d; i += 32) { Ko[i] = K[i]; Vo[i] = V[i]; }
     if (lane == 0) { A.pos[e] = t; A.log_m[e] = 0.f; A.src_lo[e] = t; A.src_hi[e] = t + 1; }
+}
+
+// Persistent grid: as many blocks as fit on the device at once.
+template <typename Tin, int DH>
+cudaError_t launch_emit(const Ctx &c, const GatherArgs &A, int64_t n_ent, cudaStream_t s) {
+    const size_t smem = 8 * (size_t)EmitGeom<Tin, DH>::WARP_BYTES;
+    cudaError_t e = cudaFuncSetAttribute(gather_emit_kernel<Tin, DH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, gather_emit_kernel<Tin, DH>, 256, smem);
+    if (e != cudaSuccess) return e;
+    const int64_t want = std::max<int64_t>(1, (int64_t)c.num_sms * std::max(per_sm, 1));
+    const unsigned ge = (unsigned)std::min<int64_t>((n_ent + 7) / 8, want);
+    gather_emit_kernel<Tin, DH><<<ge, 256, smem, s>>>(A, n_ent);
+    return cudaGetLastError();
 }
 
 }  // namespace
@@ -325,14 +428,15 @@ cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *s
     if (me != cudaSuccess) return me;
     if (gu) {
         gather_list_kernel<<<gu, 256, 0, s>>>(A);
-        const unsigned ge = (unsigned)std::min<int64_t>((n_ent + 7) / 8, (int64_t)c.num_sms * 2 * 8);
+        cudaError_t le;
         if (c.p.d == 128) {
-            if (bf) gather_emit_kernel<__nv_bfloat16, 128><<<ge, 256, 0, s>>>(A, n_ent);
-            else gather_emit_kernel<float, 128><<<ge, 256, 0, s>>>(A, n_ent);
+            if (bf) le = launch_emit<__nv_bfloat16, 128>(c, A, n_ent, s);
+            else le = launch_emit<float, 128>(c, A, n_ent, s);
         } else {
-            if (bf) gather_emit_kernel<__nv_bfloat16, 64><<<ge, 256, 0, s>>>(A, n_ent);
-            else gather_emit_kernel<float, 64><<<ge, 256, 0, s>>>(A, n_ent);
+            if (bf) le = launch_emit<__nv_bfloat16, 64>(c, A, n_ent, s);
+            else le = launch_emit<float, 64>(c, A, n_ent, s);
         }
+        if (le != cudaSuccess) return le;
     }
     int ntok = c.p.ctx_start + (c.p.T - c.c_end);
     c.launches += 2 + (gu ? 2 : 0) + (ntok > 0 ? 1 : 0);
