@@ -131,6 +131,34 @@ template <> struct Raw8<__nv_bfloat16> {
     __device__ __forceinline__ void store(__nv_bfloat16 *p) const { *reinterpret_cast<uint4 *>(p) = u; }
 };
 
+// 4 consecutive elements held raw.
+template <typename T> struct Raw4;
+template <> struct Raw4<float> {
+    float4 a;
+    __device__ __forceinline__ void load_shared(const float *p) { a = *reinterpret_cast<const float4 *>(p); }
+    __device__ __forceinline__ void get(float v[4]) const { v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; }
+    __device__ __forceinline__ void store(float *p) const { *reinterpret_cast<float4 *>(p) = a; }
+};
+template <> struct Raw4<__nv_bfloat16> {
+    uint2 u;
+    __device__ __forceinline__ void load_shared(const __nv_bfloat16 *p) { u = *reinterpret_cast<const uint2 *>(p); }
+    __device__ __forceinline__ void get(float v[4]) const {
+        v[0] = __uint_as_float(u.x << 16); v[1] = __uint_as_float(u.x & 0xFFFF0000u);
+        v[2] = __uint_as_float(u.y << 16); v[3] = __uint_as_float(u.y & 0xFFFF0000u);
+    }
+    __device__ __forceinline__ void store(__nv_bfloat16 *p) const { *reinterpret_cast<uint2 *>(p) = u; }
+};
+__device__ __forceinline__ void store4(__nv_bfloat16 *dst, const float v[4]) {
+    uint2 u;
+    __nv_bfloat162 *h = reinterpret_cast<__nv_bfloat162 *>(&u);
+    h[0] = __floats2bfloat162_rn(v[0], v[1]);
+    h[1] = __floats2bfloat162_rn(v[2], v[3]);
+    *reinterpret_cast<uint2 *>(dst) = u;
+}
+__device__ __forceinline__ void store4(float *dst, const float v[4]) {
+    *reinterpret_cast<float4 *>(dst) = make_float4(v[0], v[1], v[2], v[3]);
+}
+
 // 8 consecutive elements copied bit for bit.
 __device__ __forceinline__ void copy8(__nv_bfloat16 *dst, const __nv_bfloat16 *src) {
     *reinterpret_cast<uint4 *>(dst) = *reinterpret_cast<const uint4 *>(src);
@@ -184,9 +212,8 @@ __global__ void gather_list_kernel(GatherArgs A) {
 // steps; the K and V rows and token values of step s + D - 1 are copied into
 // the warp's ring of D steps (cp.async, zero-filled past an entry's end) while
 // step s is consumed, so D - 1 steps of loads stay in flight across entry
-// boundaries.  The chunk holding elements i .. i+7 of the first half of a key
-// and the one holding i + d/2 .. sit PX = LPR / 2 lanes apart, so the rotation
-// partner comes from a shuffle.  The key prototype RoPE(mean_t RoPE^-1(k_t, t),
+// boundaries.  Lane c of a row holds the key's rotation pairs (i, i + d/2) for
+// i = 4 c .. 4 c + 3 and the value elements 8 c .. 8 c + 7.  The key prototype RoPE(mean_t RoPE^-1(k_t, t),
 // p) is formed as mean_t of k_t rotated by p - t (rotations compose), from a
 // table of the 2 n_max - 1 offsets; its norm equals the norm of the mean
 // inverse-rotated key.  The value prototype uses sum_t (R_t + beta) v_t =
@@ -195,7 +222,7 @@ constexpr int kRingSteps = 8;
 
 template <typename Tin, int DH>
 struct EmitGeom {
-    static constexpr int LPR = DH / 8, RPW = 32 / LPR, PX = LPR / 2;
+    static constexpr int LPR = DH / 8, RPW = 32 / LPR;
     static constexpr int KB = DH * (int)sizeof(Tin);      // bytes of a K (or V) row
     static constexpr int RB = 2 * KB;                      // ring bytes of a row: K, then V
     static constexpr int CPR = RB / 16;                    // 16-byte chunks of a ring row
@@ -211,7 +238,8 @@ __device__ __forceinline__ void cp_async4(void *smem, const void *gmem, bool pre
 template <typename Tin, int DH>
 __global__ void __launch_bounds__(256, 2) gather_emit_kernel(GatherArgs A, int64_t n_ent) {
     using Gm = EmitGeom<Tin, DH>;
-    constexpr int HALF = DH / 2, LPR = Gm::LPR, RPW = Gm::RPW, PX = Gm::PX, RB = Gm::RB, CPR = Gm::CPR;
+    constexpr int HALF = DH / 2, LPR = Gm::LPR, RPW = Gm::RPW, RB = Gm::RB, CPR = Gm::CPR;
+    const float base_frac = (float)A.base_frac, eps = (float)A.eps;
     constexpr int D = kRingSteps;
     extern __shared__ __align__(16) unsigned char gsm[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -219,8 +247,7 @@ __global__ void __launch_bounds__(256, 2) gather_emit_kernel(GatherArgs A, int64
     float *rring = reinterpret_cast<float *>(ring + D * RPW * RB);
     const int64_t nw = (int64_t)gridDim.x * 8;
     const int r = lane / LPR, c = lane - r * LPR;
-    const bool hi = c >= PX;                   // chunk in the second half
-    const int i0 = 8 * (c - (hi ? PX : 0));    // pair index of the chunk's first element
+    const int i0 = 4 * c;                      // the lane's rotation pairs i0 .. i0 + 3 (both halves)
 
     struct Cur { int64_t e; int s, nst, lg, a, b; };
     // first compressible entry at or after e in this warp's sequence
@@ -269,7 +296,7 @@ __global__ void __launch_bounds__(256, 2) gather_emit_kernel(GatherArgs A, int64
         Tin *Ko = static_cast<Tin *>(A.K_out) + (size_t)e * DH;
         Tin *Vo = static_cast<Tin *>(A.V_out) + (size_t)e * DH;
         const int p = round_half_even_mid(a, b);
-        float mk[8], sv[8], srv[8], kn = 0.f, rs = 0.f;
+        float mk[8], sv[8], srv[8], kn = 0.f, rs = 0.f;   // mk: pairs i0 + j (j < 4) and their partners
 #pragma unroll
         for (int j = 0; j < 8; j++) mk[j] = sv[j] = srv[j] = 0.f;
         for (int st = 0; st < cs.nst; st++) {
@@ -277,26 +304,27 @@ __global__ void __launch_bounds__(256, 2) gather_emit_kernel(GatherArgs A, int64
             cp_async_wait<D - 1>();      // this step's group has landed
             __syncwarp();
             const unsigned char *row = ring + ((size_t)slot * RPW + r) * RB;
-            Raw8<Tin> kraw, vraw;
-            kraw.load_shared(reinterpret_cast<const Tin *>(row) + 8 * c);
+            Raw4<Tin> klo, khi;
+            Raw8<Tin> vraw;
+            klo.load_shared(reinterpret_cast<const Tin *>(row) + i0);
+            khi.load_shared(reinterpret_cast<const Tin *>(row) + HALF + i0);
             vraw.load_shared(reinterpret_cast<const Tin *>(row + Gm::KB) + 8 * c);
             const float rr = rring[slot * RPW + r];
             const int t = a + st * RPW + r;
             const int tt = t < b ? t : b - 1;   // rows past b are zero
             if (n == 1) {   // single token: original bits, p = t, log m = 0
                 if (lane < LPR) {
-                    kraw.store(Ko + 8 * c);
+                    klo.store(Ko + i0);
+                    khi.store(Ko + HALF + i0);
                     vraw.store(Vo + 8 * c);
                 }
             } else {
-                float kx[8], vx[8], y[8], nn = 0.f;
-                kraw.get(kx);
+                float x[4], y[4], vx[8], nn = 0.f;
+                klo.get(x);
+                khi.get(y);
                 vraw.get(vx);
 #pragma unroll
-                for (int j = 0; j < 8; j++) {
-                    y[j] = __shfl_xor_sync(0xffffffffu, kx[j], PX);
-                    nn = fmaf(kx[j], kx[j], nn);
-                }
+                for (int j = 0; j < 4; j++) nn = fmaf(x[j], x[j], fmaf(y[j], y[j], nn));
 #pragma unroll
                 for (int o = 1; o < LPR; o <<= 1) nn += __shfl_xor_sync(0xffffffffu, nn, o);
                 if (c == 0) kn += sqrtf(nn);   // |k_t|
@@ -304,17 +332,21 @@ __global__ void __launch_bounds__(256, 2) gather_emit_kernel(GatherArgs A, int64
                 const float4 *cs4 = reinterpret_cast<const float4 *>(
                     A.rope_rel + (size_t)(p - tt + kMaxUnit - 1) * HALF + i0);
 #pragma unroll
-                for (int j2 = 0; j2 < 4; j2++) {
+                for (int j2 = 0; j2 < 2; j2++) {
                     const float4 q = cs4[j2];          // (cos, sin) of pairs i0 + 2 j2, i0 + 2 j2 + 1
                     const float cc[2] = {q.x, q.z}, sn[2] = {q.y, q.w};
 #pragma unroll
                     for (int h = 0; h < 2; h++) {
                         const int j = 2 * j2 + h;
                         // rotation by p - t: x' = x cos - y sin, y' = x sin + y cos
-                        mk[j] += hi ? fmaf(kx[j], cc[h], y[j] * sn[h]) : fmaf(kx[j], cc[h], -y[j] * sn[h]);
-                        sv[j] += vx[j];
-                        srv[j] = fmaf(rr, vx[j], srv[j]);
+                        mk[j] = fmaf(x[j], cc[h], fmaf(-y[j], sn[h], mk[j]));
+                        mk[4 + j] = fmaf(x[j], sn[h], fmaf(y[j], cc[h], mk[4 + j]));
                     }
+                }
+#pragma unroll
+                for (int j = 0; j < 8; j++) {
+                    sv[j] += vx[j];
+                    srv[j] = fmaf(rr, vx[j], srv[j]);
                 }
             }
             __syncwarp();   // the slot may be refilled by the next issue
@@ -337,8 +369,8 @@ __global__ void __launch_bounds__(256, 2) gather_emit_kernel(GatherArgs A, int64
             }
             kn = __shfl_sync(0xffffffffu, kn, 0);
             const float ninv = 1.0f / (float)n;
-            const float beta = (float)A.base_frac * (rs * ninv);
-            const float winv = 1.0f / (rs + (float)n * beta + (float)A.eps);
+            const float beta = base_frac * (rs * ninv);
+            const float winv = 1.0f / (rs + (float)n * beta + eps);
             float ko[8], vo[8], mu2 = 0.f;
 #pragma unroll
             for (int j = 0; j < 8; j++) {
@@ -349,11 +381,12 @@ __global__ void __launch_bounds__(256, 2) gather_emit_kernel(GatherArgs A, int64
 #pragma unroll
             for (int o = 1; o < LPR; o <<= 1) mu2 += __shfl_xor_sync(0xffffffffu, mu2, o);
             if (lane < LPR) {
-                store8(Ko + 8 * c, ko);
+                store4(Ko + i0, ko);
+                store4(Ko + HALF + i0, ko + 4);
                 store8(Vo + 8 * c, vo);
             }
             if (lane == 0) {
-                const float coh = sqrtf(mu2) / (kn * ninv + (float)A.eps);
+                const float coh = sqrtf(mu2) / (kn * ninv + eps);
                 float me = (float)n * coh * coh;
                 me = me < 1.0f ? 1.0f : (me > (float)n ? (float)n : me);
                 A.pos[e] = p;
