@@ -217,7 +217,7 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
               dalloc(x, &w.nrm2, (size_t)c.nseg * p.T) &&
               dalloc(x, &w.klw, (size_t)c.nseg * c.nwin * p.T) &&
               dalloc(x, &w.kappa, (size_t)p.T) && dalloc(x, &w.bscore, (size_t)p.T) &&
-              dalloc(x, &w.zbuf, (size_t)p.T) && dalloc(x, &w.p2, (size_t)Nc + 1) &&
+              dalloc(x, &w.zbuf, (size_t)p.T) && dalloc(x, &w.zdev, (size_t)p.T) && dalloc(x, &w.p2, (size_t)Nc + 1) &&
               dalloc(x, &w.ew, (size_t)(Nc + 1) * ((nb + 3) & ~3)) && dalloc(x, &w.ewt, (size_t)p.n_max + 1) &&
               dalloc(x, &w.slots, (size_t)Nc + 2) &&
               dalloc(x, &w.dev_int, 16) &&
@@ -341,7 +341,8 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
         bool ok = dalloc(x, &w.u_nnodes, cap) && dalloc(x, &w.u_Uadd, cap) &&
                   dalloc(x, &w.u_Ddrop, cap) && dalloc(x, &w.u_sel, cap) &&
                   dalloc(x, &w.u_count, cap) && dalloc(x, &w.u_off, cap) &&
-                  dalloc(x, &w.u_pend, cap) && dalloc(x, &w.u_list, cap);
+                  dalloc(x, &w.u_pend, cap) && dalloc(x, &w.u_list, cap) &&
+                  dalloc(x, &w.u_bsum, cap / 1024 + 2);
         if (!ok) return fail(x, GKV_ENOMEM, "build_trees: unit arrays");
         w.units_cap = cap;
     }

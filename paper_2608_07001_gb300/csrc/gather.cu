@@ -10,8 +10,9 @@
 // Eqs. app_rope_prototype, app_value_prototype, app_effective_multiplicity,
 // recomputed here from K, V and the token values.
 //
-// Kernels: gather_count (frontier entries per unit), gather_scan (one block,
-// ordered exclusive scan -> per-unit and per-(l, g) offsets), gather_list
+// Kernels: gather_count (frontier entries per unit), gather_bsum /
+// gather_bscan / gather_offs (ordered exclusive scan -> per-unit and per-(l, g)
+// offsets), gather_list
 // (warp per unit, depth-first in ascending position: entry descriptors by
 // output position), gather_emit (persistent warps, one entry at a time, rows
 // streamed through a per-warp cp.async ring: prototypes or single-token
@@ -69,35 +70,88 @@ __global__ void gather_count_kernel(GatherArgs A) {
     A.u_count[uid] = cnt;
 }
 
-// Ordered exclusive scan of the per-unit counts; unit offsets include the
-// prefix tokens of its (l, g) and the prefix + tail tokens of earlier (l, g).
-__global__ void __launch_bounds__(1024) gather_scan_kernel(GatherArgs A) {
-    __shared__ long long part[1024];
-    const int64_t nu = (int64_t)A.L * A.G * A.J;
+// Ordered exclusive scan of the per-unit counts in three steps (block sums,
+// one block scanning the block sums, block-local scans); unit offsets include
+// the prefix tokens of its (l, g) and the prefix + tail tokens of earlier (l, g).
+constexpr int kScanB = 1024;
+
+__global__ void __launch_bounds__(kScanB) gather_bsum_kernel(const int32_t *cnt, int64_t nu, long long *bsum) {
+    __shared__ long long ws[kScanB / 32];
+    const int64_t i = (int64_t)blockIdx.x * kScanB + threadIdx.x;
+    long long v = i < nu ? cnt[i] : 0;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if ((threadIdx.x & 31) == 0) ws[threadIdx.x >> 5] = v;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        long long w = ws[threadIdx.x];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) w += __shfl_xor_sync(0xffffffffu, w, o);
+        if (threadIdx.x == 0) bsum[blockIdx.x] = w;
+    }
+}
+
+// In place: bsum[b] becomes the exclusive prefix of the block sums; bsum[nb]
+// the total.  One block; thread t scans a contiguous run of blocks.
+__global__ void __launch_bounds__(kScanB) gather_bscan_kernel(long long *bsum, int nb) {
+    __shared__ long long part[kScanB];
     const int tid = threadIdx.x;
-    const int64_t per = (nu + 1023) / 1024;
-    const int64_t b = tid * per, e = b + per < nu ? b + per : nu;
+    const int per = (nb + kScanB - 1) / kScanB;
+    const int b0 = tid * per, b1 = min(nb, b0 + per);
     long long s = 0;
-    for (int64_t i = b; i < e; i++) s += A.u_count[i];
+    for (int q = b0; q < b1; q++) s += bsum[q];
     part[tid] = s;
     __syncthreads();
     if (tid == 0) {
         long long acc = 0;
-        for (int k = 0; k < 1024; k++) { long long v = part[k]; part[k] = acc; acc += v; }
+        for (int k = 0; k < kScanB; k++) { const long long v = part[k]; part[k] = acc; acc += v; }
+        bsum[nb] = acc;
+    }
+    __syncthreads();
+    long long acc = part[tid];
+    for (int q = b0; q < b1; q++) { const long long v = bsum[q]; bsum[q] = acc; acc += v; }
+}
+
+__global__ void __launch_bounds__(kScanB) gather_offs_kernel(GatherArgs A, const long long *bsum, int nb) {
+    __shared__ long long ws[kScanB / 32];
+    const int64_t nu = (int64_t)A.L * A.G * A.J;
+    const int64_t i = (int64_t)blockIdx.x * kScanB + threadIdx.x;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const long long v = i < nu ? A.u_count[i] : 0;
+    long long incl = v;   // inclusive warp scan
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const long long y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) ws[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        const long long w = ws[lane];
+        long long wi = w;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const long long y = __shfl_up_sync(0xffffffffu, wi, o);
+            if (lane >= o) wi += y;
+        }
+        ws[lane] = wi - w;   // exclusive over the block's warps
     }
     __syncthreads();
     const long long extra = (long long)A.cs + (A.T - A.cend);   // uncompressed entries per (l, g)
-    long long acc = part[tid];
-    for (int64_t i = b; i < e; i++) {
-        int lg = (int)(i / A.J), j = (int)(i - (int64_t)lg * A.J);
-        long long off = acc + (long long)lg * extra + A.cs;
+    if (i < nu) {
+        const long long excl = bsum[blockIdx.x] + ws[warp] + incl - v;
+        const int lg = (int)(i / A.J), j = (int)(i - (int64_t)lg * A.J);
+        const long long off = excl + (long long)lg * extra + A.cs;
         A.u_off[i] = off;
         if (j == 0) A.offsets[lg] = off - A.cs;
-        acc += A.u_count[i];
     }
-    if (tid == 1023) A.offsets[A.L * A.G] = acc + (long long)A.L * A.G * extra;
-    if (nu == 0 && tid == 0)
-        for (int lg = 0; lg <= A.L * A.G; lg++) A.offsets[lg] = (long long)lg * extra;
+    if (blockIdx.x == 0 && threadIdx.x == 0) A.offsets[A.L * A.G] = bsum[nb] + (long long)A.L * A.G * extra;
+}
+
+// No covered unit at all: every (l, g) holds only its uncompressed tokens.
+__global__ void gather_offs_empty_kernel(GatherArgs A) {
+    const long long extra = (long long)A.cs + (A.T - A.cend);
+    for (int lg = threadIdx.x; lg <= A.L * A.G; lg += blockDim.x) A.offsets[lg] = (long long)lg * extra;
 }
 
 // 8 consecutive elements held raw (loaded from shared memory, converted to
@@ -451,8 +505,15 @@ cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *s
     A.K_out = K_out; A.V_out = V_out; A.pos = pos; A.log_m = log_m; A.src_lo = src_lo;
     A.src_hi = src_hi; A.offsets = offsets;
     const int64_t nu = (int64_t)c.p.L * c.p.G * J;
-    gather_count_kernel<<<(unsigned)((nu + 255) / 256), 256, 0, s>>>(A);
-    gather_scan_kernel<<<1, 1024, 0, s>>>(A);
+    const int nb = (int)((nu + kScanB - 1) / kScanB);
+    if (nu > 0) {
+        gather_count_kernel<<<(unsigned)((nu + 255) / 256), 256, 0, s>>>(A);
+        gather_bsum_kernel<<<nb, kScanB, 0, s>>>(c.w.u_count, nu, c.w.u_bsum);
+        gather_bscan_kernel<<<1, kScanB, 0, s>>>(c.w.u_bsum, nb);
+        gather_offs_kernel<<<nb, kScanB, 0, s>>>(A, c.w.u_bsum, nb);
+    } else {
+        gather_offs_empty_kernel<<<1, 256, 0, s>>>(A);
+    }
     const bool bf = c.p.dtype == GKV_BF16;
     unsigned gu = (unsigned)((nu + 7) / 8);
     // descriptors by output position; positions of uncompressed tokens stay 0
@@ -472,7 +533,7 @@ cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *s
         if (le != cudaSuccess) return le;
     }
     int ntok = c.p.ctx_start + (c.p.T - c.c_end);
-    c.launches += 2 + (gu ? 2 : 0) + (ntok > 0 ? 1 : 0);
+    c.launches += (nu > 0 ? 4 : 1) + (gu ? 2 : 0) + (ntok > 0 ? 1 : 0);
     if (ntok > 0) {
         dim3 g((ntok + 7) / 8, c.p.L * c.p.G);
         if (bf) gather_tokens_kernel<__nv_bfloat16><<<g, 256, 0, s>>>(A);

@@ -33,6 +33,7 @@ struct Workspace {
     double *kappa = nullptr;       // [T] stabilised curvature
     double *bscore = nullptr;      // [T] boundary score
     double *zbuf = nullptr;        // [T] scratch for robust z
+    unsigned long long *zdev = nullptr;   // [T] keys of the absolute deviations (robust z)
     double *p2 = nullptr;          // [N_c + 1] prefix of sum_l ||d_t||^2
     float *ew = nullptr;           // [(N_c + 1) * nbp] DP edge weights (len n_min..n_max), rows padded to 4
     float2 *ewt = nullptr;         // [n_max + 1] terminal edge weights (len 1..n_max) at i = N_c
@@ -65,8 +66,7 @@ struct Workspace {
     int32_t *u_count = nullptr;    // frontier entries per unit
     int64_t *u_off = nullptr;      // entry offset of each unit's frontier
     int32_t *u_list = nullptr;     // compacted unit ids (ties)
-    int32_t *u_blk = nullptr;      // per-block counts for compaction / scans
-    int64_t *u_blk64 = nullptr;
+    long long *u_bsum = nullptr;   // [units_cap / 1024 + 2] block sums of the gather's offset scan
     // allocation
     unsigned long long *hist = nullptr;        // [2048] cost-weighted histogram
     unsigned long long *alloc_state = nullptr; // see alloc.cu

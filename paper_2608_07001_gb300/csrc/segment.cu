@@ -253,7 +253,7 @@ __global__ void seg_combine_kernel(const double *klw, int nk, int T, double lamb
 }
 
 // ---------------------------------------------------------------------------
-// Robust z: exact lower median and MAD by 8-bit radix select over the ordered
+// Robust z: exact lower median and MAD by radix select over the ordered
 // 64-bit keys of doubles; one block of 1024 threads.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ unsigned long long dkey(double x) {
@@ -265,50 +265,90 @@ __device__ __forceinline__ double dkey_inv(unsigned long long k) {
     return __longlong_as_double((long long)u);
 }
 
-// Select the element of ascending rank `rank` of f(i) over i < n, where f is
-// x[i] (mode 0) or |x[i] - center| (mode 1).
-__device__ double block_select(const double *x, int n, int rank, int mode, double center,
-                               unsigned int *hist, unsigned long long *shared_prefix,
-                               int *shared_rank) {
+// Select the element of ascending rank `rank` of the keys key(i), i < n, by
+// radix select over 11-bit digits (6 passes).  Histogram updates are
+// aggregated per warp (one shared atomic per distinct bin), since the keys of
+// a pass crowd into few bins; the digit is found by a block-wide scan.
+constexpr int kSelBits = 11, kSelBins = 1 << kSelBits;
+
+template <typename KeyF>
+__device__ unsigned long long block_select(int n, int rank, KeyF key, unsigned int *hist,
+                                           unsigned long long *shared_prefix, int *shared_rank,
+                                           unsigned int *wsum) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     unsigned long long prefix = 0, mask = 0;
     int r = rank;
-    for (int shift = 56; shift >= 0; shift -= 8) {
-        for (int b = threadIdx.x; b < 256; b += blockDim.x) hist[b] = 0;
+    for (int top = 64; top > 0; top -= kSelBits) {
+        const int shift = top > kSelBits ? top - kSelBits : 0, bits = top - shift;
+        const unsigned int nbin = 1u << bits;
+        for (int b = tid; b < kSelBins; b += blockDim.x) hist[b] = 0;
         __syncthreads();
-        for (int i = threadIdx.x; i < n; i += blockDim.x) {
-            double v = mode ? fabs(x[i] - center) : x[i];
-            unsigned long long k = dkey(v);
-            if ((k & mask) == prefix) atomicAdd(&hist[(k >> shift) & 255], 1u);
+        for (int i0 = warp * 32; i0 < n; i0 += blockDim.x) {   // whole warps step together
+            const int i = i0 + lane;
+            int bin = -1;
+            if (i < n) {
+                const unsigned long long k = key(i);
+                if ((k & mask) == prefix) bin = (int)((k >> shift) & (nbin - 1));
+            }
+            const unsigned grp = __match_any_sync(0xffffffffu, bin);
+            if (bin >= 0 && lane == __ffs(grp) - 1) atomicAdd(&hist[bin], (unsigned)__popc(grp));
         }
         __syncthreads();
-        if (threadIdx.x == 0) {
-            int acc = 0, b = 0;
-            for (; b < 256; b++) {
-                if (acc + (int)hist[b] > r) break;
-                acc += hist[b];
+        // inclusive scan of the bins in ascending order: thread t owns bins 2t, 2t + 1
+        const unsigned int h0 = 2 * tid < (int)nbin ? hist[2 * tid] : 0u;
+        const unsigned int h1 = 2 * tid + 1 < (int)nbin ? hist[2 * tid + 1] : 0u;
+        unsigned int incl = h0 + h1;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const unsigned int y = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += y;
+        }
+        if (lane == 31) wsum[warp] = incl;
+        __syncthreads();
+        if (warp == 0) {
+            const unsigned int wv = lane < (int)(blockDim.x >> 5) ? wsum[lane] : 0u;
+            unsigned int wi = wv;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const unsigned int y = __shfl_up_sync(0xffffffffu, wi, o);
+                if (lane >= o) wi += y;
             }
-            *shared_prefix = prefix | ((unsigned long long)b << shift);
-            *shared_rank = r - acc;
+            wsum[lane] = wi - wv;
+        }
+        __syncthreads();
+        const unsigned int before = wsum[warp] + incl - (h0 + h1);   // keys in lower bins
+        // the bin holding rank r: before <= r < before + count
+        if ((unsigned)r >= before && (unsigned)r < before + h0) {
+            *shared_prefix = prefix | ((unsigned long long)(2 * tid) << shift);
+            *shared_rank = r - (int)before;
+        } else if ((unsigned)r >= before + h0 && (unsigned)r < before + h0 + h1) {
+            *shared_prefix = prefix | ((unsigned long long)(2 * tid + 1) << shift);
+            *shared_rank = r - (int)(before + h0);
         }
         __syncthreads();
         prefix = *shared_prefix;
         r = *shared_rank;
-        mask |= (255ull << shift);
+        mask |= (unsigned long long)(nbin - 1) << shift;
         __syncthreads();
     }
-    return dkey_inv(prefix);
+    return prefix;
 }
 
-// out[i] (+)= scale * (x[i] - median) / (1.4826 MAD + eps)
+// out[i] (+)= scale * (x[i] - median) / (1.4826 MAD + eps); the lower median
+// of the absolute deviations is selected over keys written once to `dev`.
 __global__ void __launch_bounds__(1024) seg_robust_z_kernel(const double *x, int n, double scale,
-                                                            int accumulate, double *out) {
-    __shared__ unsigned int hist[256];
+                                                            int accumulate, double *out,
+                                                            unsigned long long *dev) {
+    __shared__ unsigned int hist[kSelBins];
+    __shared__ unsigned int wsum[32];
     __shared__ unsigned long long sp;
     __shared__ int sr;
-    int rank = (n - 1) / 2;
-    double med = block_select(x, n, rank, 0, 0.0, hist, &sp, &sr);
-    double mad = block_select(x, n, rank, 1, med, hist, &sp, &sr);
-    double den = 1.4826 * mad + kEps;
+    const int rank = (n - 1) / 2;
+    const double med = dkey_inv(block_select(n, rank, [&](int i) { return dkey(x[i]); }, hist, &sp, &sr, wsum));
+    for (int i = threadIdx.x; i < n; i += blockDim.x) dev[i] = dkey(fabs(x[i] - med));
+    __syncthreads();
+    const double mad = dkey_inv(block_select(n, rank, [&](int i) { return dev[i]; }, hist, &sp, &sr, wsum));
+    const double den = 1.4826 * mad + kEps;
     for (int i = threadIdx.x; i < n; i += blockDim.x) {
         double z = scale * ((x[i] - med) / den);
         out[i] = accumulate ? out[i] + z : z;
@@ -859,10 +899,10 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
     seg_combine_kernel<<<(p.T + 255) / 256, 256, 0, s>>>(w.klw, c.nseg * c.nwin, p.T, p.lambda_stab,
                                                           w.kappa, kappa_out, w.dev_int + 1);
     // boundary score b = z(kappa) + lambda_s z(surprisal)
-    seg_robust_z_kernel<<<1, 1024, 0, s>>>(w.kappa, p.T, 1.0, 0, w.bscore);
+    seg_robust_z_kernel<<<1, 1024, 0, s>>>(w.kappa, p.T, 1.0, 0, w.bscore, w.zdev);
     if (surprisal) {
         f32_to_f64_kernel<<<(p.T + 255) / 256, 256, 0, s>>>(surprisal, p.T, w.zbuf);
-        seg_robust_z_kernel<<<1, 1024, 0, s>>>(w.zbuf, p.T, p.lambda_s, 1, w.bscore);
+        seg_robust_z_kernel<<<1, 1024, 0, s>>>(w.zbuf, p.T, p.lambda_s, 1, w.bscore, w.zdev);
     }
     // prefix of sum_l ||d_t||^2 over the compressible region
     int N = c.Nc;
