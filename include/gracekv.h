@@ -134,6 +134,24 @@ gkv_status gracekv_segment(gracekv_ctx *ctx, const void *V, const float *hidden,
                            int32_t *n_slots_host, float *kappa, void *stream);
 
 /*
+ * Stage 2a (optional) -- the observation-query score passes of stage 2: row
+ * statistics (max logit, partition over [0, T), partition over the
+ * compressible region) of every probe row (l, h, u), and the token values of
+ * the compressible region (App. A.3 max-logit shift; App. A.4 Eqs.
+ * app_attention_probability, app_direct_relevance, app_bottom_up_value).
+ * They read K and Q only, so they can overlap the segmentation: the passes
+ * are enqueued on `stream` (which should differ from the segmentation's) --
+ * right away when a segmentation has been done and its trees not yet built,
+ * otherwise by the next gracekv_segment, after an event recorded where its
+ * single-block dynamic program starts.  The next gracekv_build_trees with
+ * the same K and Q pointers uses these results instead of recomputing them,
+ * after making its own stream wait for them; K and Q must not change until
+ * then.  Asynchronous.
+ * Errors: GKV_EINVAL (null or misaligned pointer), GKV_ESTATE, GKV_ECUDA.
+ */
+gkv_status gracekv_score(gracekv_ctx *ctx, const void *K, const void *Q, void *stream);
+
+/*
  * Stage 2 -- prototype trees (App. A.3), token and node values (App. A.4),
  * gains (App. A.5 Eq. app_operation_gains).  Requires a prior
  * gracekv_segment (its curvature drives the split candidates).  If

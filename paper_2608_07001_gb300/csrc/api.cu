@@ -130,6 +130,8 @@ const char *gracekv_last_error(const gracekv_ctx *x) {
 void gracekv_destroy(gracekv_ctx *x) {
     if (!x) return;
     for (cudaEvent_t e : x->c.ev_pool) cudaEventDestroy(e);
+    if (x->c.score_ev) cudaEventDestroy(x->c.score_ev);
+    if (x->c.dp_ev) cudaEventDestroy(x->c.dp_ev);
     for (void *p : x->allocs) cudaFree(p);
     delete x;
 }
@@ -268,6 +270,8 @@ static bool al16(const void *p) { return p && (reinterpret_cast<uintptr_t>(p) & 
 static bool al4(const void *p) { return !p || (reinterpret_cast<uintptr_t>(p) & 3u) == 0; }
 static bool al8(const void *p) { return !p || (reinterpret_cast<uintptr_t>(p) & 7u) == 0; }
 
+static cudaError_t launch_score(Ctx &c, const void *K, const void *Q, cudaStream_t s);
+
 gkv_status gracekv_segment(gracekv_ctx *x, const void *V, const float *hidden, int32_t Dh,
                            const float *surprisal, int32_t *slot_starts, int32_t cap,
                            int32_t *n_slots_host, float *kappa, void *stream) {
@@ -280,10 +284,16 @@ gkv_status gracekv_segment(gracekv_ctx *x, const void *V, const float *hidden, i
     if (hidden && (Dh <= 0 || Dh > 2048 || Dh % 8))
         return fail(x, GKV_EINVAL, "segment: hidden dim must be a multiple of 8 in [8, 2048]");
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    cudaError_t e = cudaMemsetAsync(c.w.dev_int, 0, 16 * sizeof(int), s);
+    cudaError_t e = cudaSuccess;
+    if (c.score_pending && !c.dp_ev) e = cudaEventCreateWithFlags(&c.dp_ev, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaMemsetAsync(c.w.dev_int, 0, 16 * sizeof(int), s);
     if (e == cudaSuccess) {
         gkv::StageTimer tm(c, 0, s);
         e = gkv::launch_segment(c, V, hidden, hidden ? Dh : 0, surprisal, kappa, s);
+    }
+    if (e == cudaSuccess && c.score_pending) {   // requested score passes overlap the DP
+        e = cudaStreamWaitEvent(c.score_stream, c.dp_ev, 0);
+        if (e == cudaSuccess) e = launch_score(c, c.score_K, c.score_Q, c.score_stream);
     }
     if (e != cudaSuccess) return cuda_fail(x, e, "segment launch");
     int h[2];
@@ -300,6 +310,44 @@ gkv_status gracekv_segment(gracekv_ctx *x, const void *V, const float *hidden, i
     if (e != cudaSuccess) return cuda_fail(x, e, "segment copy");
     c.J = h[0];
     c.stage = 1;
+    return GKV_OK;
+}
+
+// The score passes on stream s, then the event the tree build waits for.
+static cudaError_t launch_score(Ctx &c, const void *K, const void *Q, cudaStream_t s) {
+    c.score_pending = false;
+    cudaError_t e = cudaMemsetAsync(c.w.dev_int + gkv::kScoreStatus, 0, sizeof(int), s);
+    if (e == cudaSuccess) {
+        gkv::StageTimer tm(c, 1, s);
+        e = gkv::launch_row_stats(c, K, Q, s);
+    }
+    if (e == cudaSuccess) {
+        gkv::StageTimer tm(c, 2, s);
+        e = gkv::launch_token_values(c, K, Q, s);
+    }
+    if (e == cudaSuccess && !c.score_ev) e = cudaEventCreateWithFlags(&c.score_ev, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventRecord(c.score_ev, s);
+    if (e == cudaSuccess) c.scored = true;
+    return e;
+}
+
+gkv_status gracekv_score(gracekv_ctx *x, const void *K, const void *Q, void *stream) {
+    if (!x) return GKV_EINVAL;
+    if (x->c.sticky != GKV_OK) return GKV_ESTATE;
+    Ctx &c = x->c;
+    if (!K || !Q) return fail(x, GKV_EINVAL, "score: null tensor");
+    if (!al16(K) || !al16(Q)) return fail(x, GKV_EINVAL, "score: misaligned pointer (K, Q need 16 bytes)");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    c.scored = false;
+    c.score_K = K;
+    c.score_Q = Q;
+    c.score_stream = s;
+    if (c.stage != 1) {   // the next segmentation enqueues them when its DP starts
+        c.score_pending = true;
+        return GKV_OK;
+    }
+    cudaError_t e = launch_score(c, K, Q, s);
+    if (e != cudaSuccess) return cuda_fail(x, e, "score");
     return GKV_OK;
 }
 
@@ -346,14 +394,25 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
         if (!ok) return fail(x, GKV_ENOMEM, "build_trees: unit arrays");
         w.units_cap = cap;
     }
-    {
-        gkv::StageTimer tm(c, 1, s);
-        e = gkv::launch_row_stats(c, K, Q, s);
+    if (c.score_pending && c.score_K == K && c.score_Q == Q) {
+        e = launch_score(c, K, Q, c.score_stream);
+        if (e != cudaSuccess) return cuda_fail(x, e, "score");
     }
-    if (e == cudaSuccess) {
-        gkv::StageTimer tm(c, 2, s);
-        e = gkv::launch_token_values(c, K, Q, s);
+    c.score_pending = false;
+    if (c.scored && c.score_K == K && c.score_Q == Q) {   // issued ahead by gracekv_score
+        e = cudaStreamWaitEvent(s, c.score_ev, 0);
+    } else {
+        e = cudaMemsetAsync(c.w.dev_int + gkv::kScoreStatus, 0, sizeof(int), s);
+        if (e == cudaSuccess) {
+            gkv::StageTimer tm(c, 1, s);
+            e = gkv::launch_row_stats(c, K, Q, s);
+        }
+        if (e == cudaSuccess) {
+            gkv::StageTimer tm(c, 2, s);
+            e = gkv::launch_token_values(c, K, Q, s);
+        }
     }
+    c.scored = false;
     // Trees (build.cu).  Every op's key is bounded before it is built: a pending
     // node's split key is at most min(creator key, omega R D).  Each pass derives
     // the threshold tau of the ops built so far (a lower bound of the final one)
@@ -445,10 +504,12 @@ gkv_status gracekv_allocate(gracekv_ctx *x, int64_t *n_entries_host, void *strea
     unsigned long long used = 0;
     int h = 0;
     e = cudaMemcpyAsync(&used, c.w.alloc_state + 7, sizeof used, cudaMemcpyDeviceToHost, s);
+    int hs = 0;
     if (e == cudaSuccess) e = cudaMemcpyAsync(&h, c.w.dev_int + 1, sizeof(int), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(&hs, c.w.dev_int + gkv::kScoreStatus, sizeof(int), cudaMemcpyDeviceToHost, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_fail(x, e, "allocate");
-    st = check_status(x, h);
+    st = check_status(x, h | hs);
     if (st) return st;
     const int64_t LG = (int64_t)c.p.L * c.p.G;
     c.used = (int64_t)used;

@@ -14,7 +14,8 @@
 namespace gkv {
 
 constexpr int kMaxUnit = 128;
-constexpr int kStPipeTimeout = 32;   // status bit: a bounded wait of a tensor-core pipeline gave up      // longest slot a unit kernel holds in shared memory
+constexpr int kStPipeTimeout = 32;   // status bit: a bounded wait of a tensor-core pipeline gave up
+constexpr int kScoreStatus = 8;      // dev_int word of the score passes' status bits      // longest slot a unit kernel holds in shared memory
 constexpr int kMaxSegLayers = 8;
 constexpr int kMaxWindows = 4;
 
@@ -96,6 +97,14 @@ struct Ctx {
     // measurement
     int64_t launches = 0;          // kernels launched (host count)
     int build_passes = 1;          // unit-kernel launches of the last build (pruning passes)
+    // score passes issued ahead by gracekv_score (consumed by the next build);
+    // requested before a segmentation, they are enqueued when its dynamic
+    // program (one block) starts, so that they overlap it
+    bool scored = false, score_pending = false;
+    const void *score_K = nullptr, *score_Q = nullptr;
+    cudaStream_t score_stream = nullptr;
+    cudaEvent_t score_ev = nullptr;
+    cudaEvent_t dp_ev = nullptr;   // recorded on the segmentation stream before the DP
     bool profile = false;
     std::vector<cudaEvent_t> ev_pool;          // recorded (begin, end) pairs
     std::vector<int> ev_stage;                 // stage of each pair

@@ -512,7 +512,7 @@ cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t 
         if (e != cudaSuccess) return e;
         int nrow = a.L * a.Hq * a.W;
         row_combine_kernel<<<(nrow + 255) / 256, 256, 0, s>>>(c.w.rowp, nrow, tc_row_chunks(c), c.w.row_m,
-                                                              c.w.row_Z, c.w.row_ZC, c.w.dev_int + 1, c.w.row_mneg);
+                                                              c.w.row_Z, c.w.row_ZC, c.w.dev_int + kScoreStatus, c.w.row_mneg);
         lg_scale_kernel<<<a.L * a.G, 32, 0, s>>>(c.w.row_Z, c.w.row_ZC, a.G, a.Hq, a.W, a.gq, (double)c.p.eps,
                                                   c.w.lg_scale);
         c.launches += 1;
@@ -526,7 +526,7 @@ cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t 
         else launch_mma_a<64>(c, a, K, Q, chunk, s);
         int nrow = a.L * a.Hq * a.W;
         row_combine_kernel<<<(nrow + 255) / 256, 256, 0, s>>>(c.w.rowp, nrow, c.n_chunks, c.w.row_m,
-                                                              c.w.row_Z, c.w.row_ZC, c.w.dev_int + 1, nullptr);
+                                                              c.w.row_Z, c.w.row_ZC, c.w.dev_int + kScoreStatus, nullptr);
         c.launches += 2;
         return cudaGetLastError();
     }
@@ -541,7 +541,7 @@ cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t 
                                               c.w.rowp);
     int nrow = a.L * a.Hq * a.W;
     row_combine_kernel<<<(nrow + 255) / 256, 256, 0, s>>>(c.w.rowp, nrow, c.n_chunks, c.w.row_m,
-                                                          c.w.row_Z, c.w.row_ZC, c.w.dev_int + 1, nullptr);
+                                                          c.w.row_Z, c.w.row_ZC, c.w.dev_int + kScoreStatus, nullptr);
     c.launches += 2;
     return cudaGetLastError();
 }

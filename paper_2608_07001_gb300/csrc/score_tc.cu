@@ -426,8 +426,8 @@ cudaError_t launch_row_stats_tc(Ctx &c, const void *K, const void *Q, cudaStream
     const int LG = c.p.L * c.p.G;
     const int64_t krows = (int64_t)LG * c.p.T, qrows = (int64_t)a.nrow_all;
     cudaError_t e = c.p.d == 128
-        ? launch_tc<128, 0>(a, LG, K, Q, krows, qrows, nullptr, nullptr, c.w.rowp, nullptr, c.w.dev_int + 1, s)
-        : launch_tc<64, 0>(a, LG, K, Q, krows, qrows, nullptr, nullptr, c.w.rowp, nullptr, c.w.dev_int + 1, s);
+        ? launch_tc<128, 0>(a, LG, K, Q, krows, qrows, nullptr, nullptr, c.w.rowp, nullptr, c.w.dev_int + kScoreStatus, s)
+        : launch_tc<64, 0>(a, LG, K, Q, krows, qrows, nullptr, nullptr, c.w.rowp, nullptr, c.w.dev_int + kScoreStatus, s);
     if (e == cudaSuccess) c.launches += 1;
     return e;
 }
@@ -442,9 +442,9 @@ cudaError_t launch_token_values_tc(Ctx &c, const void *K, const void *Q, cudaStr
     const int64_t krows = (int64_t)LG * c.p.T, qrows = (int64_t)a.nrow_all;
     cudaError_t e = c.p.d == 128
         ? launch_tc<128, 1>(a, LG, K, Q, krows, qrows, c.w.row_mneg, c.w.lg_scale, nullptr, c.w.rtok,
-                            c.w.dev_int + 1, s)
+                            c.w.dev_int + kScoreStatus, s)
         : launch_tc<64, 1>(a, LG, K, Q, krows, qrows, c.w.row_mneg, c.w.lg_scale, nullptr, c.w.rtok,
-                           c.w.dev_int + 1, s);
+                           c.w.dev_int + kScoreStatus, s);
     if (e == cudaSuccess) c.launches += 1;
     return e;
 }

@@ -938,6 +938,7 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
     const size_t smd = dp_smem(N, nb);
     if (smd > 227 * 1024 || nb > 32 * kDpLen) return cudaErrorInvalidConfiguration;
     cudaFuncSetAttribute(seg_dp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smd);
+    if (c.dp_ev) cudaEventRecord(c.dp_ev, s);   // work that overlaps the DP may start here
     seg_dp_kernel<<<1, kDpEp * 32, smd, s>>>(w.ew, w.ewt, N, p.n_min, p.n_max, p.ctx_start,
                                              w.slots, w.dev_int);
     c.launches += 8 + (surprisal ? 2 : 0) + (N > 1 ? 1 : 0);

@@ -50,7 +50,7 @@ _lib = None
 
 EXPORTED = ["gracekv_default_params", "gracekv_budget_for_ratio", "gracekv_create",
             "gracekv_destroy", "gracekv_last_error", "gracekv_status_string", "gracekv_query",
-            "gracekv_segment", "gracekv_build_trees", "gracekv_allocate", "gracekv_gather",
+            "gracekv_segment", "gracekv_score", "gracekv_build_trees", "gracekv_allocate", "gracekv_gather",
             "gracekv_export", "gracekv_profile", "gracekv_stats", "gracekv_row_stats_noalloc"]
 
 
@@ -76,6 +76,7 @@ def lib() -> C.CDLL:
     L.gracekv_query.argtypes = [vp, C.POINTER(i32), C.POINTER(i32), C.POINTER(i64), C.POINTER(i32)]
     L.gracekv_segment.argtypes = [vp, vp, vp, i32, vp, vp, i32, C.POINTER(i32), vp, vp]
     L.gracekv_build_trees.argtypes = [vp, vp, vp, vp, vp, vp, i32, vp]
+    L.gracekv_score.argtypes = [vp, vp, vp, vp]
     L.gracekv_allocate.argtypes = [vp, C.POINTER(i64), vp]
     L.gracekv_gather.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, i64, vp]
     L.gracekv_export.argtypes = [vp, i64, C.POINTER(i64)] + [vp] * 18 + [vp]
@@ -183,6 +184,9 @@ class Context:
                                           _ptr(kappa), _stream(stream)))
         return n.value
 
+    def gracekv_score(self, K, Q, stream=None):
+        self._check(lib().gracekv_score(self.h, _ptr(K), _ptr(Q), _stream(stream)))
+
     def gracekv_build_trees(self, K, V, Q, omega=None, slot_starts=None, n_slots=0, stream=None):
         self._check(lib().gracekv_build_trees(self.h, _ptr(K), _ptr(V), _ptr(Q), _ptr(omega),
                                               _ptr(slot_starts), n_slots, _stream(stream)))
@@ -281,11 +285,21 @@ class Compressor:
         self.cache = Cache.empty(cap, p.d, p.L * p.G, dt, device)
         self.n_slots = 0
         self.n_entries = 0
+        self._side = None
 
     def __call__(self, K, V, Q, omega=None, hidden=None, surprisal=None, slot_starts=None,
                  stream=None) -> "Cache":
         c = self.ctx
-        self.n_slots = c.gracekv_segment(V, self.slots, hidden, surprisal, self.kappa, stream)
+        # the score passes (K, Q only) run on a second stream while the
+        # segmentation runs; the tree build waits for them
+        main = stream if stream is not None else torch.cuda.current_stream()
+        if self._side is None:
+            self._side = torch.cuda.Stream(device=K.device)
+        self._side.wait_stream(main)
+        c.gracekv_score(K, Q, self._side)
+        K.record_stream(self._side)
+        Q.record_stream(self._side)
+        self.n_slots = c.gracekv_segment(V, self.slots, hidden, surprisal, self.kappa, main)
         if slot_starts is not None:
             c.gracekv_build_trees(K, V, Q, omega, slot_starts, slot_starts.numel() - 1, stream)
         else:

@@ -158,3 +158,27 @@ def test_errors_are_reported_not_trapped():
     with pytest.raises(gk.GraceKVError) as e:
         ctx3.gracekv_allocate()
     assert e.value.status == gk.GKV_ENONFINITE
+
+
+def test_score_ahead_matches_inline():
+    # The score passes issued ahead on a second stream (gracekv_score, as the
+    # Compressor does) give the same bits as the passes the tree build runs
+    # itself, and so the same trees and selection.
+    from paper_2608_07001_gb300 import gracekv as gk
+    w = synth.WORKLOADS["small"]
+    x = synth.make_inputs(w, layers=[0, 1], heads=[0, 1], T=1000)
+    L, G, T, d = x.K.shape
+    p = gk.make_params(L, G, x.Q.shape[1], T, d, x.Q.shape[2], dtype=x.K.dtype, budget=(L * G * T) // 8,
+                       rope_base=w.rope_base)
+    K, V, Q = (t.cuda() for t in (x.K, x.V, x.Q))
+    comp = gk.Compressor(p)
+    comp(K, V, Q)
+    a = comp.ctx.gracekv_export()
+    ctx = gk.Context(p)
+    slots = torch.empty(ctx.n_c + 2, dtype=torch.int32, device="cuda")
+    ctx.gracekv_segment(V, slots)
+    ctx.gracekv_build_trees(K, V, Q)
+    ctx.gracekv_allocate()
+    b = ctx.gracekv_export()
+    for k in ["row_m", "row_Z", "row_ZC", "rtok", "unit_Uadd", "add_sel", "a", "b", "D", "U", "split_sel"]:
+        assert np.array_equal(np.asarray(a[k]), np.asarray(b[k])), k
