@@ -557,7 +557,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             float m0[PPL], m1[PPL], v0[PPL], v1[PPL];
 #pragma unroll
             for (int j = 0; j < PPL; j++) m0[j] = m1[j] = v0[j] = v1[j] = 0.f;
-#pragma unroll 2
+#pragma unroll 8
             for (int t = ja; t < jb; t++) {
                 float k0[PPL], k1[PPL], x0[PPL], x1[PPL];
                 ld_pairs<PPL>(&sm.kc[t][i0], k0);
