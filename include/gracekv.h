@@ -195,6 +195,28 @@ gkv_status gracekv_gather(gracekv_ctx *ctx, const void *K, const void *V, void *
                           int32_t *src_hi, int64_t *offsets, int64_t cap, void *stream);
 
 /*
+ * The whole pass from host buffers: K, V [L][G][T][d] and Q [L][Hq][W][d]
+ * (dtype of the params; page-locked host memory gives the full copy rate),
+ * omega (host [L][G] fp32, nullable).  The inputs are copied to device
+ * buffers the context keeps (allocated on the first call), layer group by
+ * layer group on a copy stream of the context, and the work that needs only
+ * the layers already copied starts as they land: the segmentation after Q
+ * and its layers of V, the score passes and the first tree-building launch
+ * of each layer group after that group (tensor-core score path; otherwise
+ * after the last group); the pruning passes, the allocation and the packing
+ * follow on `stream`.  The cache is then copied to the host arrays (layouts
+ * of gracekv_gather; capacity `cap` entries, offsets [L G + 1]).
+ * Synchronous: returns when the host arrays hold the cache; *n_entries_host
+ * receives E.  No hidden states, surprisal or supplied slots (use the stage
+ * calls for those).  Errors: those of the stage calls, GKV_ECAPACITY (E >
+ * cap), GKV_ENOMEM (device copies of the inputs).
+ */
+gkv_status gracekv_compress_host(gracekv_ctx *ctx, const void *K, const void *V, const void *Q,
+                                 const float *omega, void *K_out, void *V_out, int32_t *pos, float *log_m,
+                                 int32_t *src_lo, int32_t *src_hi, int64_t *offsets, int64_t cap,
+                                 int64_t *n_entries_host, void *stream);
+
+/*
  * Introspection for tests and tools (not needed to compress).  Copies the
  * current trees and selection to caller-owned HOST arrays (synchronises
  * `stream`).  Node records of all units are packed unit after unit, unit

@@ -132,6 +132,8 @@ void gracekv_destroy(gracekv_ctx *x) {
     for (cudaEvent_t e : x->c.ev_pool) cudaEventDestroy(e);
     if (x->c.score_ev) cudaEventDestroy(x->c.score_ev);
     if (x->c.dp_ev) cudaEventDestroy(x->c.dp_ev);
+    for (cudaEvent_t e : x->c.copy_ev) cudaEventDestroy(e);
+    if (x->c.copy_stream) cudaStreamDestroy(x->c.copy_stream);
     for (void *p : x->allocs) cudaFree(p);
     delete x;
 }
@@ -351,16 +353,11 @@ gkv_status gracekv_score(gracekv_ctx *x, const void *K, const void *Q, void *str
     return GKV_OK;
 }
 
-gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, const void *Q,
-                               const float *omega, const int32_t *slot_starts, int32_t n_slots,
-                               void *stream) {
-    gkv_status st = ready(x, 1);
-    if (st) return st;
+// ---- tree building, in pieces (used by gracekv_build_trees and the host pipeline)
+
+// Supplied slots (validated) or the segmentation's; unit arrays sized for them.
+static gkv_status build_setup(gracekv_ctx *x, const int32_t *slot_starts, int32_t n_slots, cudaStream_t s) {
     Ctx &c = x->c;
-    if (!K || !V || !Q) return fail(x, GKV_EINVAL, "build_trees: null tensor");
-    if (!al16(K) || !al16(V) || !al16(Q) || !al4(omega) || !al4(slot_starts))
-        return fail(x, GKV_EINVAL, "build_trees: misaligned pointer (K, V, Q need 16 bytes)");
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t e;
     if (slot_starts) {
         if (n_slots < 1 || n_slots > c.Nc) return fail(x, GKV_EINVAL, "build_trees: bad n_slots");
@@ -377,12 +374,11 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
         if (e == cudaSuccess) e = cudaMemcpyAsync(&h, c.w.dev_int + 1, sizeof(int), cudaMemcpyDeviceToHost, s);
         if (e == cudaSuccess) e = cudaStreamSynchronize(s);
         if (e != cudaSuccess) return cuda_fail(x, e, "build_trees slots");
-        st = check_status(x, h);
+        gkv_status st = check_status(x, h);
         if (st) return st;
         c.J = n_slots;
     }
-    const int J = c.J;
-    const int64_t nu = (int64_t)c.p.L * c.p.G * J;
+    const int64_t nu = (int64_t)c.p.L * c.p.G * c.J;
     gkv::Workspace &w = c.w;
     if (nu > w.units_cap) {   // grows only when a partition has more slots than any before
         int64_t cap = std::max<int64_t>(nu, w.units_cap * 2);
@@ -394,57 +390,59 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
         if (!ok) return fail(x, GKV_ENOMEM, "build_trees: unit arrays");
         w.units_cap = cap;
     }
-    if (c.score_pending && c.score_K == K && c.score_Q == Q) {
-        e = launch_score(c, K, Q, c.score_stream);
-        if (e != cudaSuccess) return cuda_fail(x, e, "score");
-    }
-    c.score_pending = false;
-    if (c.scored && c.score_K == K && c.score_Q == Q) {   // issued ahead by gracekv_score
-        e = cudaStreamWaitEvent(s, c.score_ev, 0);
-    } else {
-        e = cudaMemsetAsync(c.w.dev_int + gkv::kScoreStatus, 0, sizeof(int), s);
-        if (e == cudaSuccess) {
-            gkv::StageTimer tm(c, 1, s);
-            e = gkv::launch_row_stats(c, K, Q, s);
-        }
-        if (e == cudaSuccess) {
-            gkv::StageTimer tm(c, 2, s);
-            e = gkv::launch_token_values(c, K, Q, s);
-        }
-    }
-    c.scored = false;
-    // Trees (build.cu).  Every op's key is bounded before it is built: a pending
-    // node's split key is at most min(creator key, omega R D).  Each pass derives
-    // the threshold tau of the ops built so far (a lower bound of the final one)
-    // and expands one level of the pending nodes whose bound reaches it, until
-    // none does; nodes left pending can never be selected.  When the budget is
-    // smaller than the number of units, the first launch evaluates only the
-    // roots' own distortion (their Add ops) and later passes expand the units
-    // with the largest bounds first, about 32768 at a time, so that tau rises
-    // before weaker units are considered; otherwise it evaluates every root's
-    // split at once.  When the budget left provably covers the complete
-    // expansion of every unit that reaches tau, those trees are built to the end.
-    const bool root_only = c.B_free < nu;
-    const int pass_units = 32768;
+    return GKV_OK;
+}
+
+// Work counters and the op list cleared; slots split into the short and long
+// classes of the unit kernel (cnt: their sizes, synchronises s).
+static cudaError_t build_classes(Ctx &c, int cnt[2], cudaStream_t s) {
+    gkv::Workspace &w = c.w;
+    const int64_t nu = (int64_t)c.p.L * c.p.G * c.J;
     static const float kNoCut = -INFINITY;
-    if (e == cudaSuccess && !root_only)
-        e = cudaMemcpyAsync(w.pend_cut, &kNoCut, sizeof(float), cudaMemcpyHostToDevice, s);
+    cudaError_t e = cudaSuccess;
+    if (!(c.B_free < nu)) e = cudaMemcpyAsync(w.pend_cut, &kNoCut, sizeof(float), cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = cudaMemsetAsync(w.work, 0, 4 * sizeof(unsigned long long), s);
     if (e == cudaSuccess) e = cudaMemsetAsync(w.n_ops, 0, sizeof(unsigned int), s);
+    cnt[0] = cnt[1] = 0;
     if (e == cudaSuccess) {
-        int cnt[2] = {0, 0};
-        {
-            gkv::StageTimer tm(c, 3, s);
-            e = gkv::launch_slot_classes(c, w.slots, J, w.u_list, w.dev_int + 2, s);
-        }
-        if (e == cudaSuccess) e = cudaMemcpyAsync(cnt, w.dev_int + 2, 2 * sizeof(int), cudaMemcpyDeviceToHost, s);
-        if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-        if (e == cudaSuccess) {
-            gkv::StageTimer tm(c, 3, s);
-            e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 0, root_only ? 1 : 0, 1, 0.f, w.u_list, cnt[0],
-                                       w.u_list + (J - cnt[1]), cnt[1], s);
-        }
+        gkv::StageTimer tm(c, 3, s);
+        e = gkv::launch_slot_classes(c, w.slots, c.J, w.u_list, w.dev_int + 2, s);
     }
+    if (e == cudaSuccess) e = cudaMemcpyAsync(cnt, w.dev_int + 2, 2 * sizeof(int), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    return e;
+}
+
+// The first tree-building launch of the units of (l, g) in [lg0, lg0 + nlg).
+static cudaError_t build_fresh(Ctx &c, const void *K, const void *V, const void *Q, const float *omega,
+                               const int cnt[2], int lg0, int nlg, cudaStream_t s) {
+    gkv::Workspace &w = c.w;
+    const int64_t nu = (int64_t)c.p.L * c.p.G * c.J;
+    const bool root_only = c.B_free < nu;
+    gkv::StageTimer tm(c, 3, s);
+    return gkv::launch_unit_build(c, K, V, Q, omega, w.slots, c.J, 0, root_only ? 1 : 0, 1, 0.f, w.u_list, cnt[0],
+                                  w.u_list + (c.J - cnt[1]), cnt[1], s, lg0, nlg);
+}
+
+// Trees (build.cu).  Every op's key is bounded before it is built: a pending
+// node's split key is at most min(creator key, omega R D).  Each pass derives
+// the threshold tau of the ops built so far (a lower bound of the final one)
+// and expands one level of the pending nodes whose bound reaches it, until
+// none does; nodes left pending can never be selected.  When the budget is
+// smaller than the number of units, the first launch evaluates only the
+// roots' own distortion (their Add ops) and later passes expand the units
+// with the largest bounds first, about 32768 at a time, so that tau rises
+// before weaker units are considered; otherwise it evaluates every root's
+// split at once.  When the budget left provably covers the complete
+// expansion of every unit that reaches tau, those trees are built to the end.
+static cudaError_t build_passes(Ctx &c, const void *K, const void *V, const void *Q, const float *omega,
+                                cudaStream_t s) {
+    gkv::Workspace &w = c.w;
+    const int J = c.J;
+    const int64_t nu = (int64_t)c.p.L * c.p.G * J;
+    const bool root_only = c.B_free < nu;
+    const int pass_units = 32768;
+    cudaError_t e = cudaSuccess;
     for (int it = 0; e == cudaSuccess; it++) {
         struct {
             int count[2];
@@ -484,8 +482,183 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
                                    h.count[0], w.u_list + (nu - h.count[1]), h.count[1], s);
         c.build_passes = it + 2;
     }
+    return e;
+}
+
+gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, const void *Q,
+                               const float *omega, const int32_t *slot_starts, int32_t n_slots,
+                               void *stream) {
+    gkv_status st = ready(x, 1);
+    if (st) return st;
+    Ctx &c = x->c;
+    if (!K || !V || !Q) return fail(x, GKV_EINVAL, "build_trees: null tensor");
+    if (!al16(K) || !al16(V) || !al16(Q) || !al4(omega) || !al4(slot_starts))
+        return fail(x, GKV_EINVAL, "build_trees: misaligned pointer (K, V, Q need 16 bytes)");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    st = build_setup(x, slot_starts, n_slots, s);
+    if (st) return st;
+    cudaError_t e = cudaSuccess;
+    if (c.score_pending && c.score_K == K && c.score_Q == Q) {
+        e = launch_score(c, K, Q, c.score_stream);
+        if (e != cudaSuccess) return cuda_fail(x, e, "score");
+    }
+    c.score_pending = false;
+    if (c.scored && c.score_K == K && c.score_Q == Q) {   // issued ahead by gracekv_score
+        e = cudaStreamWaitEvent(s, c.score_ev, 0);
+    } else {
+        e = cudaMemsetAsync(c.w.dev_int + gkv::kScoreStatus, 0, sizeof(int), s);
+        if (e == cudaSuccess) {
+            gkv::StageTimer tm(c, 1, s);
+            e = gkv::launch_row_stats(c, K, Q, s);
+        }
+        if (e == cudaSuccess) {
+            gkv::StageTimer tm(c, 2, s);
+            e = gkv::launch_token_values(c, K, Q, s);
+        }
+    }
+    c.scored = false;
+    int cnt[2];
+    if (e == cudaSuccess) e = build_classes(c, cnt, s);
+    if (e == cudaSuccess) e = build_fresh(c, K, V, Q, omega, cnt, 0, c.p.L * c.p.G, s);
+    if (e == cudaSuccess) e = build_passes(c, K, V, Q, omega, s);
     if (e != cudaSuccess) return cuda_fail(x, e, "build_trees launch");
     c.stage = 2;
+    return GKV_OK;
+}
+
+// ---- the whole pass from host buffers, copies overlapped with the work -------
+
+gkv_status gracekv_compress_host(gracekv_ctx *x, const void *K, const void *V, const void *Q,
+                                 const float *omega, void *K_out, void *V_out, int32_t *pos, float *log_m,
+                                 int32_t *src_lo, int32_t *src_hi, int64_t *offsets, int64_t cap,
+                                 int64_t *n_entries_host, void *stream) {
+    gkv_status st = ready(x, 0);
+    if (st) return st;
+    Ctx &c = x->c;
+    const gkv_params &p = c.p;
+    if (!K || !V || !Q || !K_out || !V_out || !pos || !log_m || !src_lo || !src_hi || !offsets || !n_entries_host)
+        return fail(x, GKV_EINVAL, "compress_host: null argument");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const size_t es = p.dtype == GKV_BF16 ? 2 : 4;
+    const int LG = p.L * p.G;
+    const size_t layer = (size_t)p.G * p.T * p.d * es;   // bytes of one layer of K (or V)
+    const size_t qbytes = (size_t)p.L * p.Hq * p.W * p.d * es;
+    const int ngrp = std::min(p.L, 4);
+    // device buffers, allocated on the first call
+    if (!c.hK) {
+        const int64_t ecap = p.budget + (int64_t)LG * (p.T - c.Nc) + 8;
+        bool ok = dalloc(x, reinterpret_cast<unsigned char **>(&c.hK), layer * p.L) &&
+                  dalloc(x, reinterpret_cast<unsigned char **>(&c.hV), layer * p.L) &&
+                  dalloc(x, reinterpret_cast<unsigned char **>(&c.hQ), qbytes) && dalloc(x, &c.hOm, (size_t)LG) &&
+                  dalloc(x, &c.hSlots, (size_t)c.Nc + 2) &&
+                  dalloc(x, reinterpret_cast<unsigned char **>(&c.oK), (size_t)ecap * p.d * es) &&
+                  dalloc(x, reinterpret_cast<unsigned char **>(&c.oV), (size_t)ecap * p.d * es) &&
+                  dalloc(x, &c.opos, (size_t)ecap) && dalloc(x, &c.olo, (size_t)ecap) &&
+                  dalloc(x, &c.ohi, (size_t)ecap) && dalloc(x, &c.ologm, (size_t)ecap) &&
+                  dalloc(x, &c.ooff, (size_t)LG + 1);
+        if (!ok) {
+            c.hK = nullptr;
+            return fail(x, GKV_ENOMEM, "compress_host: device copies of the inputs");
+        }
+        c.ocap = ecap;
+    }
+    cudaError_t e = cudaSuccess;
+    if (!c.copy_stream) e = cudaStreamCreateWithFlags(&c.copy_stream, cudaStreamNonBlocking);
+    while (e == cudaSuccess && (int)c.copy_ev.size() < 2 + ngrp) {
+        cudaEvent_t ev;
+        e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+        if (e == cudaSuccess) c.copy_ev.push_back(ev);
+    }
+    if (e != cudaSuccess) return cuda_fail(x, e, "compress_host setup");
+    cudaStream_t cs = c.copy_stream;
+    unsigned char *dK = static_cast<unsigned char *>(c.hK), *dV = static_cast<unsigned char *>(c.hV);
+    const unsigned char *Kh = static_cast<const unsigned char *>(K), *Vh = static_cast<const unsigned char *>(V);
+    auto is_seg = [&](int l) {
+        for (int i = 0; i < c.nseg; i++)
+            if (c.seg_layers[i] == l) return true;
+        return false;
+    };
+    // copies: Q and the segmentation layers of V first, then the layer groups
+    // (the copy stream starts after the work already on `stream`, which may
+    // still read these buffers)
+    e = cudaEventRecord(c.copy_ev[0], s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, c.copy_ev[0], 0);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(c.hQ, Q, qbytes, cudaMemcpyHostToDevice, cs);
+    if (e == cudaSuccess && omega) e = cudaMemcpyAsync(c.hOm, omega, (size_t)LG * sizeof(float), cudaMemcpyHostToDevice, cs);
+    for (int i = 0; e == cudaSuccess && i < c.nseg; i++) {
+        const size_t off = (size_t)c.seg_layers[i] * layer;
+        e = cudaMemcpyAsync(dV + off, Vh + off, layer, cudaMemcpyHostToDevice, cs);
+    }
+    if (e == cudaSuccess) e = cudaEventRecord(c.copy_ev[1], cs);
+    for (int gi = 0; e == cudaSuccess && gi < ngrp; gi++) {
+        const int l0 = gi * p.L / ngrp, l1 = (gi + 1) * p.L / ngrp;
+        e = cudaMemcpyAsync(dK + l0 * layer, Kh + l0 * layer, (l1 - l0) * layer, cudaMemcpyHostToDevice, cs);
+        for (int l = l0; e == cudaSuccess && l < l1; l++)
+            if (!is_seg(l)) e = cudaMemcpyAsync(dV + l * layer, Vh + l * layer, layer, cudaMemcpyHostToDevice, cs);
+        if (e == cudaSuccess) e = cudaEventRecord(c.copy_ev[2 + gi], cs);
+    }
+    if (e != cudaSuccess) return cuda_fail(x, e, "compress_host copies");
+    const float *om = omega ? c.hOm : nullptr;
+    // segmentation as soon as its layers are in
+    e = cudaStreamWaitEvent(s, c.copy_ev[1], 0);
+    if (e != cudaSuccess) return cuda_fail(x, e, "compress_host");
+    int32_t J = 0;
+    c.score_pending = false;
+    c.scored = false;
+    st = gracekv_segment(x, c.hV, nullptr, 0, nullptr, c.hSlots, c.Nc + 1, &J, nullptr, stream);
+    if (st) return st;
+    st = build_setup(x, nullptr, 0, s);
+    if (st) return st;
+    int cnt[2];
+    e = cudaMemsetAsync(c.w.dev_int + gkv::kScoreStatus, 0, sizeof(int), s);
+    if (e == cudaSuccess) e = build_classes(c, cnt, s);
+    // per layer group, once it is in: score passes and the first tree-building launch
+    const bool ranged = gkv::use_tc(c);
+    for (int gi = 0; e == cudaSuccess && gi < ngrp; gi++) {
+        const int l0 = gi * p.L / ngrp, l1 = (gi + 1) * p.L / ngrp;
+        e = cudaStreamWaitEvent(s, c.copy_ev[2 + gi], 0);
+        if (!ranged || e != cudaSuccess) continue;
+        {
+            gkv::StageTimer tm(c, 1, s);
+            e = gkv::launch_row_stats(c, c.hK, c.hQ, s, l0, l1);
+        }
+        if (e == cudaSuccess) {
+            gkv::StageTimer tm(c, 2, s);
+            e = gkv::launch_token_values(c, c.hK, c.hQ, s, l0, l1);
+        }
+        if (e == cudaSuccess) e = build_fresh(c, c.hK, c.hV, c.hQ, om, cnt, l0 * p.G, (l1 - l0) * p.G, s);
+    }
+    if (e == cudaSuccess && !ranged) {   // other score paths: whole layers range at once
+        {
+            gkv::StageTimer tm(c, 1, s);
+            e = gkv::launch_row_stats(c, c.hK, c.hQ, s);
+        }
+        if (e == cudaSuccess) {
+            gkv::StageTimer tm(c, 2, s);
+            e = gkv::launch_token_values(c, c.hK, c.hQ, s);
+        }
+        if (e == cudaSuccess) e = build_fresh(c, c.hK, c.hV, c.hQ, om, cnt, 0, LG, s);
+    }
+    if (e == cudaSuccess) e = build_passes(c, c.hK, c.hV, c.hQ, om, s);
+    if (e != cudaSuccess) return cuda_fail(x, e, "compress_host trees");
+    c.stage = 2;
+    int64_t E = 0;
+    st = gracekv_allocate(x, &E, stream);
+    if (st) return st;
+    *n_entries_host = E;
+    if (E > cap) return fail(x, GKV_ECAPACITY, "compress_host: more cache entries than cap");
+    st = gracekv_gather(x, c.hK, c.hV, c.oK, c.oV, c.opos, c.ologm, c.olo, c.ohi, c.ooff, c.ocap, stream);
+    if (st) return st;
+    const size_t row = (size_t)p.d * es;
+    e = cudaMemcpyAsync(K_out, c.oK, (size_t)E * row, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(V_out, c.oV, (size_t)E * row, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(pos, c.opos, (size_t)E * 4, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(log_m, c.ologm, (size_t)E * 4, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(src_lo, c.olo, (size_t)E * 4, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(src_hi, c.ohi, (size_t)E * 4, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(offsets, c.ooff, (size_t)(LG + 1) * 8, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(x, e, "compress_host results");
     return GKV_OK;
 }
 

@@ -71,6 +71,7 @@ struct BuildArgs {
     int max_levels;              // levels evaluated by this launch
     float tau;                   // resume: evaluate pending nodes whose key bound >= tau
     const int32_t *list;         // fresh: slot indices; resume: unit ids
+    int lg0, nlg;                // fresh: the (l, g) range [lg0, lg0 + nlg) of the launch
     // outputs
     int32_t *nd_a, *nd_b, *nd_child0, *nd_parent, *nd_unit;
     int8_t *nd_nchild, *nd_cost;
@@ -266,15 +267,14 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     extern __shared__ __align__(16) unsigned char smem_raw[];
     S &sm = *reinterpret_cast<S *>(smem_raw);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int LG = A.L * A.G;
     int j, lg;
     if (A.resume) {
         const int uidr = A.list[blockIdx.x];
         lg = uidr / A.J;
         j = uidr - lg * A.J;
     } else {
-        j = A.list[blockIdx.x / LG];   // slot-major: the units of a slot share its table rows
-        lg = blockIdx.x % LG;
+        j = A.list[blockIdx.x / A.nlg];   // slot-major: the units of a slot share its table rows
+        lg = A.lg0 + blockIdx.x % A.nlg;
     }
     const int l = lg / A.G, g = lg - l * A.G;
     const int sa = A.slots[j], sb = A.slots[j + 1];
@@ -1118,7 +1118,7 @@ cudaError_t launch_dt(Ctx &c, BuildArgs &A, unsigned grid, cudaStream_t s) {
 cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *Q,
                               const float *omega, const int32_t *slots, int J, int resume,
                               int root_only, int max_levels, float tau, const int32_t *list_short, int n_short,
-                              const int32_t *list_long, int n_long, cudaStream_t s) {
+                              const int32_t *list_long, int n_long, cudaStream_t s, int lg0, int nlg) {
     const gkv_params &p = c.p;
     BuildArgs A;
     A.K = K; A.V = V; A.Q = Q;
@@ -1140,7 +1140,10 @@ cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *
     A.u_pend = c.w.u_pend;
     A.status = c.w.dev_int + 1;
     A.work = c.w.work;
-    const unsigned LG = (unsigned)(p.L * p.G);
+    if (nlg < 0) nlg = p.L * p.G - lg0;
+    A.lg0 = lg0;
+    A.nlg = nlg;
+    const unsigned LG = (unsigned)nlg;
     const bool bf = p.dtype == GKV_BF16;
     // short slots (<= 64 tokens) on the two-CTA-per-SM instance, the rest on the 128-token one
     A.list = list_short;

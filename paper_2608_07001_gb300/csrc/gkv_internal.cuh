@@ -105,6 +105,18 @@ struct Ctx {
     cudaStream_t score_stream = nullptr;
     cudaEvent_t score_ev = nullptr;
     cudaEvent_t dp_ev = nullptr;   // recorded on the segmentation stream before the DP
+    // host pipeline (gracekv_compress_host): device copies of the inputs, the
+    // cache before its copy to the host, a copy stream and its events
+    void *hK = nullptr, *hV = nullptr, *hQ = nullptr;
+    float *hOm = nullptr;
+    int32_t *hSlots = nullptr;
+    void *oK = nullptr, *oV = nullptr;
+    int32_t *opos = nullptr, *olo = nullptr, *ohi = nullptr;
+    float *ologm = nullptr;
+    int64_t *ooff = nullptr;
+    int64_t ocap = 0;
+    cudaStream_t copy_stream = nullptr;
+    std::vector<cudaEvent_t> copy_ev;   // [0] start, [1] Q and the segmentation layers, [2 + g] layer group g
     bool profile = false;
     std::vector<cudaEvent_t> ev_pool;          // recorded (begin, end) pairs
     std::vector<int> ev_stage;                 // stage of each pair
@@ -234,14 +246,15 @@ cudaError_t launch_rope_table(Ctx &c, cudaStream_t s);
 cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
                            const float *surprisal, float *kappa_out, cudaStream_t s);
 
-cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t s);
+// layers [l0, l1) (l1 < 0: all); a partial range needs use_tc(c)
+cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t s, int l0 = 0, int l1 = -1);
 // tcgen05 score passes (score_tc.cu): applicable to bf16, d in {64, 128}, at
 // most 256 probe rows per KV head; row-statistics partials per row = tc_row_chunks.
 bool use_tc(const Ctx &c);
 int tc_row_chunks(const Ctx &c);
-cudaError_t launch_row_stats_tc(Ctx &c, const void *K, const void *Q, cudaStream_t s);
-cudaError_t launch_token_values_tc(Ctx &c, const void *K, const void *Q, cudaStream_t s);
-cudaError_t launch_token_values(Ctx &c, const void *K, const void *Q, cudaStream_t s);
+cudaError_t launch_row_stats_tc(Ctx &c, const void *K, const void *Q, cudaStream_t s, int lg0, int nlg);
+cudaError_t launch_token_values_tc(Ctx &c, const void *K, const void *Q, cudaStream_t s, int lg0, int nlg);
+cudaError_t launch_token_values(Ctx &c, const void *K, const void *Q, cudaStream_t s, int l0 = 0, int l1 = -1);
 // Slots of at most kShortUnit tokens run on the unit kernel instance that fits
 // two CTAs per SM; the work lists hold them (slot indices for a fresh build,
 // unit ids for a resumed one) separately from the longer ones.
@@ -249,7 +262,8 @@ constexpr int kShortUnit = 64;
 cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *Q,
                               const float *omega, const int32_t *slots, int J, int resume,
                               int root_only, int max_levels, float tau, const int32_t *list_short,
-                              int n_short, const int32_t *list_long, int n_long, cudaStream_t s);
+                              int n_short, const int32_t *list_long, int n_long, cudaStream_t s,
+                              int lg0 = 0, int nlg = -1);   // fresh launches: (l, g) in [lg0, lg0 + nlg);
 // Slot indices split by length class: short ones at list[0, count[0]), long
 // ones at list[J - count[1], J).
 cudaError_t launch_slot_classes(Ctx &c, const int32_t *slots, int J, int32_t *list, int *count,

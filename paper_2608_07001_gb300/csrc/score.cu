@@ -151,9 +151,9 @@ __global__ void __launch_bounds__(256) row_stats_kernel(const Tin *K, const Tin 
 // Combines the per-chunk partials of every row; rmneg (nullable) receives
 // -(m_r log2 e + log2 Z_r), the base-2 exponent offset of exp(x - m_r) / Z_r.
 __global__ void row_combine_kernel(const float *part, int nrow, int nchunks, float *rm, float *rz,
-                                   float *rzc, int *status, float *rmneg) {
-    int row = blockIdx.x * blockDim.x + threadIdx.x;
-    if (row >= nrow) return;
+                                   float *rzc, int *status, float *rmneg, int row0 = 0, int row1 = -1) {
+    const int row = row0 + blockIdx.x * blockDim.x + threadIdx.x;   // rows [row0, row1) of nrow
+    if (row >= (row1 < 0 ? nrow : row1)) return;
     const float *pm = part + (size_t)row * nchunks;
     const float *pz = part + ((size_t)nrow + row) * nchunks;
     const float *pc = part + ((size_t)2 * nrow + row) * nchunks;
@@ -175,8 +175,8 @@ __global__ void row_combine_kernel(const float *part, int nrow, int nchunks, flo
 
 // Pass-B normaliser of every KV head: 1 / (sum_r Z^C_r / Z_r + eps) over its rows.
 __global__ void lg_scale_kernel(const float *rz, const float *rzc, int G, int Hq, int W, int gq, double eps,
-                                double *out) {
-    const int lg = blockIdx.x, l = lg / G, g = lg - l * G;
+                                double *out, int lg0) {
+    const int lg = lg0 + blockIdx.x, l = lg / G, g = lg - l * G;
     const size_t rowbase = (size_t)(l * Hq + g * gq) * W;
     double s = 0.0;
     for (int r = threadIdx.x; r < gq * W; r += 32) s += (double)rzc[rowbase + r] / (double)rz[rowbase + r];
@@ -505,20 +505,23 @@ void launch_mma_b(const Ctx &c, const ScoreArgs &a, const void *K, const void *Q
         c.w.row_m, c.w.row_Z, c.w.row_ZC, eps, c.w.rtok);
 }
 
-cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t s) {
+cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t s, int l0, int l1) {
     ScoreArgs a = make_args(c);
-    if (use_tc(c)) {   // tcgen05 pass (score_tc.cu), then the same combine
-        cudaError_t e = launch_row_stats_tc(c, K, Q, s);
+    if (l1 < 0) l1 = a.L;
+    if (use_tc(c)) {   // tcgen05 pass (score_tc.cu) over layers [l0, l1), then the same combine
+        cudaError_t e = launch_row_stats_tc(c, K, Q, s, l0 * a.G, (l1 - l0) * a.G);
         if (e != cudaSuccess) return e;
-        int nrow = a.L * a.Hq * a.W;
-        row_combine_kernel<<<(nrow + 255) / 256, 256, 0, s>>>(c.w.rowp, nrow, tc_row_chunks(c), c.w.row_m,
-                                                              c.w.row_Z, c.w.row_ZC, c.w.dev_int + kScoreStatus, c.w.row_mneg);
-        lg_scale_kernel<<<a.L * a.G, 32, 0, s>>>(c.w.row_Z, c.w.row_ZC, a.G, a.Hq, a.W, a.gq, (double)c.p.eps,
-                                                  c.w.lg_scale);
+        const int nrow = a.L * a.Hq * a.W, r0 = l0 * a.Hq * a.W, r1 = l1 * a.Hq * a.W;
+        row_combine_kernel<<<(r1 - r0 + 255) / 256, 256, 0, s>>>(c.w.rowp, nrow, tc_row_chunks(c), c.w.row_m,
+                                                                 c.w.row_Z, c.w.row_ZC, c.w.dev_int + kScoreStatus,
+                                                                 c.w.row_mneg, r0, r1);
+        lg_scale_kernel<<<(l1 - l0) * a.G, 32, 0, s>>>(c.w.row_Z, c.w.row_ZC, a.G, a.Hq, a.W, a.gq, (double)c.p.eps,
+                                                        c.w.lg_scale, l0 * a.G);
         c.launches += 1;
         c.launches += 1;
         return cudaGetLastError();
     }
+    if (l0 != 0 || l1 != a.L) return cudaErrorInvalidValue;   // layer ranges: tensor-core path only
     int chunk = (c.p.T + c.n_chunks - 1) / c.n_chunks;
     chunk = (chunk + kTT - 1) / kTT * kTT;
     if (use_mma(c, a)) {
@@ -546,11 +549,13 @@ cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t 
     return cudaGetLastError();
 }
 
-cudaError_t launch_token_values(Ctx &c, const void *K, const void *Q, cudaStream_t s) {
+cudaError_t launch_token_values(Ctx &c, const void *K, const void *Q, cudaStream_t s, int l0, int l1) {
     ScoreArgs a = make_args(c);
     dim3 grid((c.Nc + kTT - 1) / kTT, a.L * a.G);
     float eps = (float)c.p.eps;
-    if (use_tc(c)) return launch_token_values_tc(c, K, Q, s);
+    if (l1 < 0) l1 = a.L;
+    if (use_tc(c)) return launch_token_values_tc(c, K, Q, s, l0 * a.G, (l1 - l0) * a.G);
+    if (l0 != 0 || l1 != a.L) return cudaErrorInvalidValue;   // layer ranges: tensor-core path only
     if (use_mma(c, a)) {
         // about 4 CTAs of 16 warps per SM-pass over the compressible region
         int64_t want = 4LL * c.num_sms;

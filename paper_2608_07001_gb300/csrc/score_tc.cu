@@ -55,6 +55,7 @@ struct TcArgs {
     int t_lo, t_hi;          // token range the pass covers for every (l, g)
     int chunk_tiles, nch;    // tiles per block, blocks per (l, g)
     int nq;                  // probe rows staged: 128 * halves (pass A) or the padded width N (pass B)
+    int lg0;                 // first (l, g) of the launch (grid.y covers the following ones)
     float scale;             // log2(e) / sqrt(d)
 };
 
@@ -91,7 +92,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
     __shared__ float scale_s;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int lg = blockIdx.y, l = lg / a.G, g = lg - l * a.G;
+    const int lg = a.lg0 + blockIdx.y, l = lg / a.G, g = lg - l * a.G;
     const int t_begin = a.t_lo + blockIdx.x * a.chunk_tiles * kTcTile;
     const int t_end = min(a.t_hi, t_begin + a.chunk_tiles * kTcTile);
     const int ntile = t_end > t_begin ? (t_end - t_begin + kTcTile - 1) / kTcTile : 0;
@@ -416,15 +417,16 @@ int tc_row_chunks(const Ctx &c) {
     return nch;
 }
 
-cudaError_t launch_row_stats_tc(Ctx &c, const void *K, const void *Q, cudaStream_t s) {
+cudaError_t launch_row_stats_tc(Ctx &c, const void *K, const void *Q, cudaStream_t s, int lg0, int nlg) {
     TcArgs a = base_args(c);
     a.t_lo = 0;
     a.t_hi = c.p.T;
     split((c.p.T + kTcTile - 1) / kTcTile, c.p.L * c.p.G, c.num_sms, &a.chunk_tiles, &a.nch);
     if (a.nch > c.n_chunks) return cudaErrorInvalidValue;   // the partial buffer holds n_chunks per row
     a.nq = a.Rg <= 128 ? 128 : 256;
-    const int LG = c.p.L * c.p.G;
-    const int64_t krows = (int64_t)LG * c.p.T, qrows = (int64_t)a.nrow_all;
+    a.lg0 = lg0;
+    const int LG = nlg;
+    const int64_t krows = (int64_t)c.p.L * c.p.G * c.p.T, qrows = (int64_t)a.nrow_all;
     cudaError_t e = c.p.d == 128
         ? launch_tc<128, 0>(a, LG, K, Q, krows, qrows, nullptr, nullptr, c.w.rowp, nullptr, c.w.dev_int + kScoreStatus, s)
         : launch_tc<64, 0>(a, LG, K, Q, krows, qrows, nullptr, nullptr, c.w.rowp, nullptr, c.w.dev_int + kScoreStatus, s);
@@ -432,14 +434,15 @@ cudaError_t launch_row_stats_tc(Ctx &c, const void *K, const void *Q, cudaStream
     return e;
 }
 
-cudaError_t launch_token_values_tc(Ctx &c, const void *K, const void *Q, cudaStream_t s) {
+cudaError_t launch_token_values_tc(Ctx &c, const void *K, const void *Q, cudaStream_t s, int lg0, int nlg) {
     TcArgs a = base_args(c);
     a.t_lo = c.p.ctx_start;
     a.t_hi = c.c_end;
     split((c.Nc + kTcTile - 1) / kTcTile, c.p.L * c.p.G, c.num_sms, &a.chunk_tiles, &a.nch);
     a.nq = (a.Rg + 63) / 64 * 64;
-    const int LG = c.p.L * c.p.G;
-    const int64_t krows = (int64_t)LG * c.p.T, qrows = (int64_t)a.nrow_all;
+    a.lg0 = lg0;
+    const int LG = nlg;
+    const int64_t krows = (int64_t)c.p.L * c.p.G * c.p.T, qrows = (int64_t)a.nrow_all;
     cudaError_t e = c.p.d == 128
         ? launch_tc<128, 1>(a, LG, K, Q, krows, qrows, c.w.row_mneg, c.w.lg_scale, nullptr, c.w.rtok,
                             c.w.dev_int + kScoreStatus, s)

@@ -51,7 +51,8 @@ _lib = None
 EXPORTED = ["gracekv_default_params", "gracekv_budget_for_ratio", "gracekv_create",
             "gracekv_destroy", "gracekv_last_error", "gracekv_status_string", "gracekv_query",
             "gracekv_segment", "gracekv_score", "gracekv_build_trees", "gracekv_allocate", "gracekv_gather",
-            "gracekv_export", "gracekv_profile", "gracekv_stats", "gracekv_row_stats_noalloc"]
+            "gracekv_export", "gracekv_profile", "gracekv_stats", "gracekv_row_stats_noalloc",
+            "gracekv_compress_host"]
 
 
 def lib() -> C.CDLL:
@@ -77,6 +78,7 @@ def lib() -> C.CDLL:
     L.gracekv_segment.argtypes = [vp, vp, vp, i32, vp, vp, i32, C.POINTER(i32), vp, vp]
     L.gracekv_build_trees.argtypes = [vp, vp, vp, vp, vp, vp, i32, vp]
     L.gracekv_score.argtypes = [vp, vp, vp, vp]
+    L.gracekv_compress_host.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, i64, C.POINTER(i64), vp]
     L.gracekv_allocate.argtypes = [vp, C.POINTER(i64), vp]
     L.gracekv_gather.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, i64, vp]
     L.gracekv_export.argtypes = [vp, i64, C.POINTER(i64)] + [vp] * 18 + [vp]
@@ -112,6 +114,14 @@ def gracekv_row_stats_noalloc(K, Q, c_lo: int, c_hi: int, row_m, row_Z, row_ZC, 
                                          _ptr(row_m), _ptr(row_Z), _ptr(row_ZC), _stream(stream))
     if st != GKV_OK:
         raise GraceKVError(st, lib().gracekv_status_string(st).decode())
+
+
+def _host_ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if t.is_cuda or not t.is_contiguous():
+        raise ValueError("tensors must be contiguous host tensors")
+    return C.c_void_p(t.data_ptr())
 
 
 def _ptr(t: Optional[torch.Tensor]):
@@ -182,6 +192,15 @@ class Context:
         self._check(lib().gracekv_segment(self.h, _ptr(V), _ptr(hidden), Dh, _ptr(surprisal),
                                           _ptr(slot_starts), slot_starts.numel() - 1, C.byref(n),
                                           _ptr(kappa), _stream(stream)))
+        return n.value
+
+    def gracekv_compress_host(self, K, V, Q, out: "Cache", omega=None, stream=None) -> int:
+        """The whole pass from host tensors (pinned for the full copy rate)
+        into the host cache `out`; returns the number of entries."""
+        n = C.c_int64()
+        hp = [_host_ptr(t) for t in (K, V, Q, omega, out.K, out.V, out.pos, out.log_m, out.src_lo,
+                                     out.src_hi, out.offsets)]
+        self._check(lib().gracekv_compress_host(self.h, *hp, out.K.shape[0], C.byref(n), _stream(stream)))
         return n.value
 
     def gracekv_score(self, K, Q, stream=None):
@@ -260,6 +279,12 @@ class Cache:
     src_lo: torch.Tensor
     src_hi: torch.Tensor
     offsets: torch.Tensor
+
+    @staticmethod
+    def empty_host(cap: int, d: int, LG: int, dtype) -> "Cache":
+        """Page-locked host arrays (the output of gracekv_compress_host)."""
+        c = Cache.empty(cap, d, LG, dtype, device="cpu")
+        return Cache(*(t.pin_memory() for t in (c.K, c.V, c.pos, c.log_m, c.src_lo, c.src_hi, c.offsets)))
 
     @staticmethod
     def empty(cap: int, d: int, LG: int, dtype, device="cuda") -> "Cache":

@@ -182,3 +182,30 @@ def test_score_ahead_matches_inline():
     b = ctx.gracekv_export()
     for k in ["row_m", "row_Z", "row_ZC", "rtok", "unit_Uadd", "add_sel", "a", "b", "D", "U", "split_sel"]:
         assert np.array_equal(np.asarray(a[k]), np.asarray(b[k])), k
+
+
+@pytest.mark.parametrize("wname,kw", [("small", dict(layers=[0, 1, 2, 3], heads=[0, 1], T=1000)),
+                                      ("pr1", dict(T=700))])
+def test_compress_host_matches_device(wname, kw):
+    # The host-buffer pipeline (layer-group copies overlapped with the score
+    # passes and the first tree launch) gives the device path's cache bits.
+    from paper_2608_07001_gb300 import gracekv as gk
+    w = synth.WORKLOADS[wname]
+    x = synth.make_inputs(w, **kw)
+    L, G, T, d = x.K.shape
+    p = gk.make_params(L, G, x.Q.shape[1], T, d, x.Q.shape[2], dtype=x.K.dtype, budget=(L * G * T) // 8,
+                       rope_base=w.rope_base)
+    comp = gk.Compressor(p)
+    dev = comp(x.K.cuda(), x.V.cuda(), x.Q.cuda())
+    E = comp.n_entries
+    hc = gk.Cache.empty_host(dev.K.shape[0], d, L * G, x.K.dtype)
+    ctx = gk.Context(p)
+    Kh, Vh, Qh = (t.contiguous().pin_memory() for t in (x.K, x.V, x.Q))
+    for _ in range(2):   # a second call reuses the context's device buffers
+        n = ctx.gracekv_compress_host(Kh, Vh, Qh, hc)
+        assert n == E
+        for name in ["K", "V", "pos", "log_m", "src_lo", "src_hi"]:
+            a, b = getattr(hc, name)[:n], getattr(dev, name)[:n].cpu()
+            assert torch.equal(a.view(torch.int32) if a.dtype == torch.float32 else a,
+                               b.view(torch.int32) if b.dtype == torch.float32 else b), name
+        assert torch.equal(hc.offsets, dev.offsets.cpu())
