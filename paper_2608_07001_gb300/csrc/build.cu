@@ -62,6 +62,7 @@ struct BuildArgs {
     const float2 *rope;
     const double *kappa;
     const float *rtok, *row_m, *row_Z, *omega;
+    const float *Eg;             // nullable: [L G][W][N_c] probe weights of every token (score pass B)
     int L, G, Hq, T, d, W, gq, cs, Nc, J, k_cand;
     float inv_sqrt_d, lamZ, lamM, eps;
     float lam_kappa, base_frac;
@@ -289,6 +290,21 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     const Tin *Vp = static_cast<const Tin *>(A.V) + ((size_t)lg * A.T + sa) * DH;
     const float om = A.omega ? A.omega[lg] : 1.0f;
 
+    // Probe weights E[t][u] (Eq. app_probe_distortion), stored at E[t][u % 32].x
+    // (u < 32) or .y (u >= 32).  When the score pass wrote them for every token
+    // they are copied in with the slot (cp.async, 4 bytes each); otherwise
+    // they are formed below from the raw keys.
+    float *Ef = reinterpret_cast<float *>(&sm.E[0][0]);
+    auto eidx = [](int t, int u) { return t * 2 * kNPP + 2 * (u & (kNPP - 1)) + (u >> 5); };
+    if (A.Eg) {
+        const float *Eu = A.Eg + (size_t)lg * A.W * A.Nc + (sa - A.cs);
+        for (int idx = tid; idx < 2 * kNPP * n; idx += kNT) {
+            const int u = idx / n, t = idx - u * n;
+            const bool ok = u < A.W;
+            cp_async4(&Ef[eidx(t, u)], Eu + (size_t)(ok ? u : 0) * A.Nc + t, ok);
+        }
+        cp_async_commit();
+    }
     // ---- load the slot ------------------------------------------------------
     // Every global load of a group is issued before any is used.  DH / 8
     // consecutive threads hold a token; they also form ||k_t||, which equals
@@ -365,10 +381,9 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     __syncthreads();
 
     // ---- E[t][u] from the raw (post-RoPE) keys -------------------------------
-    // Probe u is stored at E[t][u % 32].x (u < 32) or .y (u >= 32).
-    float *Ef = reinterpret_cast<float *>(&sm.E[0][0]);
-    auto eidx = [](int t, int u) { return t * 2 * kNPP + 2 * (u & (kNPP - 1)) + (u >> 5); };
-    if constexpr (std::is_same<Tin, __nv_bfloat16>::value) {
+    if (A.Eg) {
+        cp_async_wait<0>();   // the copies above have landed (each thread its own)
+    } else if constexpr (std::is_same<Tin, __nv_bfloat16>::value) {
         // Tensor cores: logits = Q_probes (64 x DH) . K_slot^T, one 16x8 tile
         // per (probe block, token block); warp w keeps probe block w % 4.
         constexpr int MT = 4, WSTEP = NWARPS / MT;
@@ -1124,6 +1139,7 @@ cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *
     A.K = K; A.V = V; A.Q = Q;
     A.slots = slots; A.rope = c.w.rope; A.kappa = c.w.kappa;
     A.rtok = c.w.rtok; A.row_m = c.w.row_m; A.row_Z = c.w.row_Z; A.omega = omega;
+    A.Eg = use_tc(c) ? c.w.Eg : nullptr;   // written by the tensor-core pass B
     A.L = p.L; A.G = p.G; A.Hq = p.Hq; A.T = p.T; A.d = p.d; A.W = p.W; A.gq = p.Hq / p.G;
     A.cs = p.ctx_start; A.Nc = c.Nc; A.J = J; A.k_cand = p.k_cand;
     A.inv_sqrt_d = (float)(1.0 / sqrt((double)p.d));

@@ -283,12 +283,6 @@ struct EmitGeom {
     static constexpr int WARP_BYTES = kRingSteps * RPW * (RB + 4);
 };
 
-__device__ __forceinline__ void cp_async4(void *smem, const void *gmem, bool pred) {
-    unsigned s = (unsigned)__cvta_generic_to_shared(smem);
-    int n = pred ? 4 : 0;
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(s), "l"(gmem), "r"(n));
-}
-
 template <typename Tin, int DH>
 __global__ void __launch_bounds__(256, 2) gather_emit_kernel(GatherArgs A, int64_t n_ent) {
     using Gm = EmitGeom<Tin, DH>;

@@ -45,6 +45,8 @@ struct Workspace {
     float *row_m = nullptr, *row_Z = nullptr, *row_ZC = nullptr;  // [L*Hq*W]
     float *rowp = nullptr;         // [3][L*Hq*W][n_chunks] pass-A partials
     float *row_mneg = nullptr;     // [L*Hq*W] -(m log2 e + log2 Z): pass-B exponent offset
+    float *Eg = nullptr;           // [L*G][W][N_c] probe weights exp(q_u.k_t / sqrt(d) - m_u) of every
+                                   // compressible token (written by the tensor-core pass B)
     double *lg_scale = nullptr;    // [L*G] pass-B normaliser 1 / (sum_r Z^C_r / Z_r + eps)
     float *rtok = nullptr;         // [L*G*N_c]
     // node records, indexed lg*2*N_c + 2*(slot start - c_s) + k
@@ -212,6 +214,11 @@ __device__ __forceinline__ void cp_async16(void *smem, const void *gmem, bool pr
     unsigned s = (unsigned)__cvta_generic_to_shared(smem);
     int n = pred ? 16 : 0;   // zero-fill past the end
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(s), "l"(gmem), "r"(n));
+}
+__device__ __forceinline__ void cp_async4(void *smem, const void *gmem, bool pred) {
+    unsigned s = (unsigned)__cvta_generic_to_shared(smem);
+    int n = pred ? 4 : 0;   // zero-fill when not pred
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(s), "l"(gmem), "r"(n));
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
 template <int N>

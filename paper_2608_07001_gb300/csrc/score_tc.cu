@@ -79,7 +79,8 @@ struct TcBars {
 template <int DH, int MODE>
 __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
         const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CUtensorMap mapQ, TcArgs a,
-        const float *rmneg, const double *lg_scale, float *part, float *rtok, int *status) {
+        const float *rmneg, const double *lg_scale, float *part, float *rtok, int *status,
+        const float *rm, float *Eg) {
     constexpr int NKB = DH / 64;
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     unsigned char *sbase = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -89,6 +90,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
     unsigned char *Ks = sbase + (size_t)NKB * QR * 128;     // [stage][NKB][128][128 B]
     __shared__ TcBars sb;
     __shared__ __align__(16) float mneg[256];   // pass B: -(m_r log2 e + log2 Z_r), -inf past the rows
+    __shared__ float eoff[256];                 // pass B: -m_r log2 e of the probe rows
+    __shared__ short eu[256];                   // pass B: probe u of row r = (u mod gq) W + u, else -1
+    __shared__ unsigned pmask[8];               // pass B: probe rows of each 32-column chunk
     __shared__ float scale_s;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -116,7 +120,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
         tc::fence_barrier_init();
     }
     if (MODE == 1) {
-        for (int r = threadIdx.x; r < 256; r += kTcThreads) mneg[r] = r < a.Rg ? rmneg[rowbase + r] : -INFINITY;
+        if (threadIdx.x < 8) pmask[threadIdx.x] = 0u;
+        __syncthreads();
+        for (int r = threadIdx.x; r < 256; r += kTcThreads) {
+            mneg[r] = r < a.Rg ? rmneg[rowbase + r] : -INFINITY;
+            const int h = r / a.W, u = r - h * a.W;
+            const bool probe = Eg && r < a.Rg && u % a.gq == h;
+            eu[r] = probe ? (short)u : (short)-1;
+            eoff[r] = probe ? (float)(-(double)rm[rowbase + r] * 1.4426950408889634) : 0.f;
+            if (probe) atomicOr(&pmask[r >> 5], 1u << (r & 31));
+        }
         if (threadIdx.x == 0) scale_s = (float)lg_scale[lg];
     }
     if (warp == kTcWarpMma) {
@@ -320,6 +333,18 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
                     acc0 = fadd2(acc0, make_float2(tc::ex2(y0.x), tc::ex2(y0.y)));
                     acc1 = fadd2(acc1, make_float2(tc::ex2(y1.x), tc::ex2(y1.y)));
                 }
+                // probe weights of the probe rows (Eq. app_probe_distortion's E, no 1 / Z):
+                // one coalesced store per probe row over the warp's 32 tokens
+                const unsigned pm = pmask[c >> 5];
+                const int t = t_begin + i * kTcTile + q * 32 + lane;
+                if (pm && t < t_end) {
+#pragma unroll
+                    for (int j = 0; j < 32; j++) {
+                        if (!((pm >> j) & 1u)) continue;
+                        const float e = tc::ex2(fmaf(v[j], a.scale, eoff[c + j]));
+                        Eg[((size_t)lg * a.W + eu[c + j]) * a.Nc + (t - a.cs)] = e;
+                    }
+                }
             }
             const float s = (acc0.x + acc0.y) + (acc1.x + acc1.y);
             const int t = t_begin + i * kTcTile + q * 32 + lane;
@@ -371,7 +396,7 @@ size_t tc_smem(int DH, int nq) {
 template <int DH, int MODE>
 cudaError_t launch_tc(const TcArgs &a, int LG, const void *K, const void *Q, int64_t krows, int64_t qrows,
                       const float *rmneg, const double *lg_scale, float *part, float *rtok, int *status,
-                      cudaStream_t s) {
+                      cudaStream_t s, const float *rm = nullptr, float *Eg = nullptr) {
     CUtensorMap mk, mq;
     if (!make_map(&mk, K, krows, DH) || !make_map(&mq, Q, qrows, DH)) return cudaErrorNotSupported;
     const size_t smem = tc_smem(DH, a.nq);
@@ -379,7 +404,7 @@ cudaError_t launch_tc(const TcArgs &a, int LG, const void *K, const void *Q, int
                                          (int)tc_smem(DH, 256));
     if (e != cudaSuccess) return e;
     dim3 grid(a.nch, LG);
-    score_tc_kernel<DH, MODE><<<grid, kTcThreads, smem, s>>>(mk, mq, a, rmneg, lg_scale, part, rtok, status);
+    score_tc_kernel<DH, MODE><<<grid, kTcThreads, smem, s>>>(mk, mq, a, rmneg, lg_scale, part, rtok, status, rm, Eg);
     return cudaGetLastError();
 }
 
@@ -445,9 +470,9 @@ cudaError_t launch_token_values_tc(Ctx &c, const void *K, const void *Q, cudaStr
     const int64_t krows = (int64_t)c.p.L * c.p.G * c.p.T, qrows = (int64_t)a.nrow_all;
     cudaError_t e = c.p.d == 128
         ? launch_tc<128, 1>(a, LG, K, Q, krows, qrows, c.w.row_mneg, c.w.lg_scale, nullptr, c.w.rtok,
-                            c.w.dev_int + kScoreStatus, s)
+                            c.w.dev_int + kScoreStatus, s, c.w.row_m, c.w.Eg)
         : launch_tc<64, 1>(a, LG, K, Q, krows, qrows, c.w.row_mneg, c.w.lg_scale, nullptr, c.w.rtok,
-                           c.w.dev_int + kScoreStatus, s);
+                           c.w.dev_int + kScoreStatus, s, c.w.row_m, c.w.Eg);
     if (e == cudaSuccess) c.launches += 1;
     return e;
 }
