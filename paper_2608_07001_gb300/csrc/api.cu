@@ -236,7 +236,7 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
               dalloc(x, &w.nd_R, (size_t)c.node_cap) && dalloc(x, &w.nd_U, (size_t)c.node_cap) &&
               dalloc(x, &w.nd_kappa, (size_t)c.node_cap) && dalloc(x, &w.nd_sel, (size_t)c.node_cap) &&
               dalloc(x, &w.ops, (size_t)c.node_cap / 2 + 1) && dalloc(x, &w.n_ops, 1) &&
-              (!gkv::use_tc(c) || dalloc(x, &w.Eg, (size_t)LG * p.W * Nc)) &&
+              (!gkv::use_tc(c) || (dalloc(x, &w.Eg, (size_t)LG * Nc * 64) && dalloc(x, &w.qperm, (size_t)256))) &&
               dalloc(x, &w.hist, 2048) && dalloc(x, &w.alloc_state, 16) && dalloc(x, &w.work, 4) &&
               dalloc(x, &w.pend_hist, 1 << 16) && dalloc(x, &w.pend_cut, 1) && dalloc(x, &w.pend_n, 1) &&
               dalloc(x, &w.pend_pot, 1);
@@ -245,6 +245,15 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
         return GKV_ENOMEM;
     }
     cudaError_t e = cudaMemset(w.nd_cost, 0, (size_t)c.node_cap);
+    if (e == cudaSuccess && w.qperm) {   // pass B's column order: probe u's row (u mod gq) W + u first
+        const int gq = p.Hq / p.G;
+        std::vector<short> perm;
+        for (int u = 0; u < p.W; u++) perm.push_back((short)((u % gq) * p.W + u));
+        for (int r = 0; r < gq * p.W; r++)
+            if ((r % p.W) % gq != r / p.W) perm.push_back((short)r);
+        perm.resize(256, 0);
+        e = cudaMemcpy(w.qperm, perm.data(), 256 * sizeof(short), cudaMemcpyHostToDevice);
+    }
     if (e == cudaSuccess) e = cudaMemset(w.dev_int, 0, 16 * sizeof(int));
     if (e == cudaSuccess) e = gkv::launch_rope_table(c, 0);
     if (e == cudaSuccess) e = cudaDeviceSynchronize();

@@ -62,7 +62,7 @@ struct BuildArgs {
     const float2 *rope;
     const double *kappa;
     const float *rtok, *row_m, *row_Z, *omega;
-    const float *Eg;             // nullable: [L G][W][N_c] probe weights of every token (score pass B)
+    const float *Eg;             // nullable: [L G][N_c][32][2] probe weights of every token (score pass B)
     int L, G, Hq, T, d, W, gq, cs, Nc, J, k_cand;
     float inv_sqrt_d, lamZ, lamM, eps;
     float lam_kappa, base_frac;
@@ -296,13 +296,9 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     // they are formed below from the raw keys.
     float *Ef = reinterpret_cast<float *>(&sm.E[0][0]);
     auto eidx = [](int t, int u) { return t * 2 * kNPP + 2 * (u & (kNPP - 1)) + (u >> 5); };
-    if (A.Eg) {
-        const float *Eu = A.Eg + (size_t)lg * A.W * A.Nc + (sa - A.cs);
-        for (int idx = tid; idx < 2 * kNPP * n; idx += kNT) {
-            const int u = idx / n, t = idx - u * n;
-            const bool ok = u < A.W;
-            cp_async4(&Ef[eidx(t, u)], Eu + (size_t)(ok ? u : 0) * A.Nc + t, ok);
-        }
+    if (A.Eg) {   // the same layout, n rows of 256 bytes: 16-byte copies
+        const float *Eu = A.Eg + ((size_t)lg * A.Nc + (sa - A.cs)) * (2 * kNPP);
+        for (int idx = tid; idx < n * (2 * kNPP / 4); idx += kNT) cp_async16(Ef + 4 * idx, Eu + 4 * idx, true);
         cp_async_commit();
     }
     // ---- load the slot ------------------------------------------------------

@@ -45,8 +45,9 @@ struct Workspace {
     float *row_m = nullptr, *row_Z = nullptr, *row_ZC = nullptr;  // [L*Hq*W]
     float *rowp = nullptr;         // [3][L*Hq*W][n_chunks] pass-A partials
     float *row_mneg = nullptr;     // [L*Hq*W] -(m log2 e + log2 Z): pass-B exponent offset
-    float *Eg = nullptr;           // [L*G][W][N_c] probe weights exp(q_u.k_t / sqrt(d) - m_u) of every
-                                   // compressible token (written by the tensor-core pass B)
+    float *Eg = nullptr;           // [L*G][N_c][32][2] probe weights exp(q_u.k_t / sqrt(d) - m_u) of every
+                                   // compressible token, (u, u + 32) pairs (written by the tensor-core pass B)
+    short *qperm = nullptr;        // [gq W] rows of a KV head in pass B's column order: probe rows first
     double *lg_scale = nullptr;    // [L*G] pass-B normaliser 1 / (sum_r Z^C_r / Z_r + eps)
     float *rtok = nullptr;         // [L*G*N_c]
     // node records, indexed lg*2*N_c + 2*(slot start - c_s) + k

@@ -78,7 +78,8 @@ struct TcBars {
 // MODE 0: pass A (row statistics); MODE 1: pass B (token values).
 template <int DH, int MODE>
 __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
-        const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CUtensorMap mapQ, TcArgs a,
+        const __grid_constant__ CUtensorMap mapK, const __grid_constant__ CUtensorMap mapQ,
+        const __grid_constant__ CUtensorMap mapQ1, const short *qperm, TcArgs a,
         const float *rmneg, const double *lg_scale, float *part, float *rtok, int *status,
         const float *rm, float *Eg) {
     constexpr int NKB = DH / 64;
@@ -90,9 +91,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
     unsigned char *Ks = sbase + (size_t)NKB * QR * 128;     // [stage][NKB][128][128 B]
     __shared__ TcBars sb;
     __shared__ __align__(16) float mneg[256];   // pass B: -(m_r log2 e + log2 Z_r), -inf past the rows
-    __shared__ float eoff[256];                 // pass B: -m_r log2 e of the probe rows
-    __shared__ short eu[256];                   // pass B: probe u of row r = (u mod gq) W + u, else -1
-    __shared__ unsigned pmask[8];               // pass B: probe rows of each 32-column chunk
+    __shared__ float eoff[64];                  // pass B: -m_r log2 e of probe u's row (columns 0 .. W-1)
     __shared__ float scale_s;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -120,15 +119,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
         tc::fence_barrier_init();
     }
     if (MODE == 1) {
-        if (threadIdx.x < 8) pmask[threadIdx.x] = 0u;
-        __syncthreads();
-        for (int r = threadIdx.x; r < 256; r += kTcThreads) {
-            mneg[r] = r < a.Rg ? rmneg[rowbase + r] : -INFINITY;
-            const int h = r / a.W, u = r - h * a.W;
-            const bool probe = Eg && r < a.Rg && u % a.gq == h;
-            eu[r] = probe ? (short)u : (short)-1;
-            eoff[r] = probe ? (float)(-(double)rm[rowbase + r] * 1.4426950408889634) : 0.f;
-            if (probe) atomicOr(&pmask[r >> 5], 1u << (r & 31));
+        // column n of pass B holds row qperm[n] of the KV head: the probe rows
+        // (u mod gq) W + u first (n = u < W), then the other rows
+        for (int n = threadIdx.x; n < 256; n += kTcThreads) {
+            const int r = n < a.Rg ? qperm[n] : -1;
+            mneg[n] = r >= 0 ? rmneg[rowbase + r] : -INFINITY;
+            if (n < 64) eoff[n] = n < a.W ? (float)(-(double)rm[rowbase + r] * 1.4426950408889634) : 0.f;
         }
         if (threadIdx.x == 0) scale_s = (float)lg_scale[lg];
     }
@@ -143,16 +139,29 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
 
     if (warp == kTcWarpTma) {
         // ---------------- producer ----------------
+        if (MODE == 1) {   // probe rows first: one-row boxes, placed by qperm, spread over the warp
+            const uint32_t qbar = tc::smem_u32(&sb.qfull);
+            if (lane == 0) tc::mbar_expect_tx(qbar, (uint32_t)(NKB * QR * 128));
+            __syncwarp();
+            for (int e = lane; e < NKB * QR; e += 32) {
+                const int kb = e / QR, n = e - kb * QR;
+                const int r = n < a.Rg ? qperm[n] : 0;   // rows past Rg: any row (their columns are masked)
+                tc::tma_load_2d(tc::smem_u32(Qs + ((size_t)kb * QR + n) * 128), &mapQ1, kb * 64, rowbase + r, qbar);
+            }
+        }
         if (lane == 0) {
             tc::tma_prefetch_desc(&mapK);
             tc::tma_prefetch_desc(&mapQ);
             const uint32_t qbar = tc::smem_u32(&sb.qfull);
-            tc::mbar_expect_tx(qbar, (uint32_t)(NKB * QR * 128));
-            for (int kb = 0; kb < NKB; kb++)
-                for (int j = 0; j < QR; j += 128)
-                    tc::tma_load_2d(tc::smem_u32(Qs + ((size_t)kb * QR + j) * 128), &mapQ, kb * 64, rowbase + j, qbar);
+            if (MODE == 0) {
+                tc::mbar_expect_tx(qbar, (uint32_t)(NKB * QR * 128));
+                for (int kb = 0; kb < NKB; kb++)
+                    for (int j = 0; j < QR; j += 128)
+                        tc::tma_load_2d(tc::smem_u32(Qs + ((size_t)kb * QR + j) * 128), &mapQ, kb * 64, rowbase + j, qbar);
+            }
             const int krow = lg * a.T + t_begin;
             int issued = 0;
+            (void)krow;
             for (int i = 0; i < ntile; i++) {
                 const int st = i % kTcStages, r = i / kTcStages;
                 if (*(volatile int *)&sb.abort) break;
@@ -315,15 +324,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
             tc::tc_fence_after();
             const uint32_t tcol = tb + ((uint32_t)(q * 32) << 16) + (uint32_t)b * acc_cols;
             float2 acc0 = make_float2(0.f, 0.f), acc1 = acc0;
-#pragma unroll 1
-            for (int c = 0; c < a.nq; c += 32) {
-                float v[32];
-                tc::tmem_ld32(tcol + c, v);
-                if (c + 32 >= a.nq) {   // the buffer is free for the MMA of tile i + 2
-                    tc::tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) tc::mbar_arrive(tc::smem_u32(&sb.accempty[b]));
-                }
+            const int t = t_begin + i * kTcTile + q * 32 + lane;
+            // 32 columns of the accumulator: their probabilities into acc0 / acc1
+            auto chunk = [&](const float v[32], int c) {
                 const float *mn = &mneg[c];
 #pragma unroll
                 for (int j = 0; j < 32; j += 4) {
@@ -333,21 +336,44 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
                     acc0 = fadd2(acc0, make_float2(tc::ex2(y0.x), tc::ex2(y0.y)));
                     acc1 = fadd2(acc1, make_float2(tc::ex2(y1.x), tc::ex2(y1.y)));
                 }
-                // probe weights of the probe rows (Eq. app_probe_distortion's E, no 1 / Z):
-                // one coalesced store per probe row over the warp's 32 tokens
-                const unsigned pm = pmask[c >> 5];
-                const int t = t_begin + i * kTcTile + q * 32 + lane;
-                if (pm && t < t_end) {
+            };
+            auto release = [&](int c) {   // after the last load: the buffer is free for tile i + 2
+                if (c + 32 >= a.nq) {
+                    tc::tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) tc::mbar_arrive(tc::smem_u32(&sb.accempty[b]));
+                }
+            };
+            {   // columns 0 .. 63 are the probes u: their weights E (no 1 / Z), stored
+                // token-major as the unit kernel keeps them, (E_u, E_{u+32}) pairs
+                float v0[32], v1[32];
+                tc::tmem_ld32(tcol, v0);
+                release(0);
+                tc::tmem_ld32(tcol + 32, v1);
+                release(32);
+                if (Eg && t < t_end) {
+                    float4 *dst = reinterpret_cast<float4 *>(Eg + ((size_t)lg * a.Nc + (t - a.cs)) * 64);
 #pragma unroll
-                    for (int j = 0; j < 32; j++) {
-                        if (!((pm >> j) & 1u)) continue;
-                        const float e = tc::ex2(fmaf(v[j], a.scale, eoff[c + j]));
-                        Eg[((size_t)lg * a.W + eu[c + j]) * a.Nc + (t - a.cs)] = e;
+                    for (int j = 0; j < 32; j += 2) {
+                        const float e0 = tc::ex2(fmaf(v0[j], a.scale, eoff[j]));
+                        const float e1 = tc::ex2(fmaf(v1[j], a.scale, eoff[32 + j]));
+                        const float e2 = tc::ex2(fmaf(v0[j + 1], a.scale, eoff[j + 1]));
+                        const float e3 = tc::ex2(fmaf(v1[j + 1], a.scale, eoff[33 + j]));
+                        dst[j >> 1] = make_float4(j < a.W ? e0 : 0.f, j + 32 < a.W ? e1 : 0.f,
+                                                  j + 1 < a.W ? e2 : 0.f, j + 33 < a.W ? e3 : 0.f);
                     }
                 }
+                chunk(v0, 0);
+                chunk(v1, 32);
+            }
+#pragma unroll 1
+            for (int c = 64; c < a.nq; c += 32) {
+                float v[32];
+                tc::tmem_ld32(tcol + c, v);
+                release(c);
+                chunk(v, c);
             }
             const float s = (acc0.x + acc0.y) + (acc1.x + acc1.y);
-            const int t = t_begin + i * kTcTile + q * 32 + lane;
             if (t < t_end) rtok[(size_t)lg * a.Nc + (t - a.cs)] = s * scale_s;
         }
     }
@@ -376,12 +402,12 @@ PFN_cuTensorMapEncodeTiled_v12000 encoder() {
 }
 
 // [rows][DH] row-major bf16, boxes of [128 rows][64 columns], 128-byte swizzle.
-bool make_map(CUtensorMap *m, const void *p, int64_t rows, int DH) {
+bool make_map(CUtensorMap *m, const void *p, int64_t rows, int DH, int box_rows = 128) {
     auto enc = encoder();
     if (!enc) return false;
     cuuint64_t gdim[2] = {(cuuint64_t)DH, (cuuint64_t)rows};
     cuuint64_t gstr[1] = {(cuuint64_t)DH * 2};
-    cuuint32_t box[2] = {64, 128};
+    cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
     cuuint32_t es[2] = {1, 1};
     return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(p), gdim, gstr, box, es,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -396,15 +422,17 @@ size_t tc_smem(int DH, int nq) {
 template <int DH, int MODE>
 cudaError_t launch_tc(const TcArgs &a, int LG, const void *K, const void *Q, int64_t krows, int64_t qrows,
                       const float *rmneg, const double *lg_scale, float *part, float *rtok, int *status,
-                      cudaStream_t s, const float *rm = nullptr, float *Eg = nullptr) {
-    CUtensorMap mk, mq;
-    if (!make_map(&mk, K, krows, DH) || !make_map(&mq, Q, qrows, DH)) return cudaErrorNotSupported;
+                      cudaStream_t s, const float *rm = nullptr, float *Eg = nullptr, const short *qperm = nullptr) {
+    CUtensorMap mk, mq, mq1;
+    if (!make_map(&mk, K, krows, DH) || !make_map(&mq, Q, qrows, DH) || !make_map(&mq1, Q, qrows, DH, 1))
+        return cudaErrorNotSupported;
     const size_t smem = tc_smem(DH, a.nq);
     cudaError_t e = cudaFuncSetAttribute(score_tc_kernel<DH, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)tc_smem(DH, 256));
     if (e != cudaSuccess) return e;
     dim3 grid(a.nch, LG);
-    score_tc_kernel<DH, MODE><<<grid, kTcThreads, smem, s>>>(mk, mq, a, rmneg, lg_scale, part, rtok, status, rm, Eg);
+    score_tc_kernel<DH, MODE><<<grid, kTcThreads, smem, s>>>(mk, mq, mq1, qperm, a, rmneg, lg_scale, part, rtok, status,
+                                                               rm, Eg);
     return cudaGetLastError();
 }
 
@@ -470,9 +498,9 @@ cudaError_t launch_token_values_tc(Ctx &c, const void *K, const void *Q, cudaStr
     const int64_t krows = (int64_t)c.p.L * c.p.G * c.p.T, qrows = (int64_t)a.nrow_all;
     cudaError_t e = c.p.d == 128
         ? launch_tc<128, 1>(a, LG, K, Q, krows, qrows, c.w.row_mneg, c.w.lg_scale, nullptr, c.w.rtok,
-                            c.w.dev_int + kScoreStatus, s, c.w.row_m, c.w.Eg)
+                            c.w.dev_int + kScoreStatus, s, c.w.row_m, c.w.Eg, c.w.qperm)
         : launch_tc<64, 1>(a, LG, K, Q, krows, qrows, c.w.row_mneg, c.w.lg_scale, nullptr, c.w.rtok,
-                           c.w.dev_int + kScoreStatus, s, c.w.row_m, c.w.Eg);
+                           c.w.dev_int + kScoreStatus, s, c.w.row_m, c.w.Eg, c.w.qperm);
     if (e == cudaSuccess) c.launches += 1;
     return e;
 }
