@@ -549,14 +549,6 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             const int row = k - kb;
             const int ja = sm.cand[k].a, jb = sm.cand[k].b, nJ = jb - ja;
             if (nJ <= 0) continue;
-            float rs = 0.f, ks = 0.f;
-            for (int t = ja + lane; t < jb; t += 32) { rs += sm.Rt[t]; ks += sm.kn[t]; }
-            rs = warp_sum(rs);
-            ks = warp_sum(ks);
-            const float ninv = 1.0f / (float)nJ;
-            const float beta = (float)A.base_frac * (rs * ninv);
-            const float wsum = rs + (float)nJ * beta;
-            const float winv = 1.0f / (wsum + A.eps);
             const int p = round_half_even_mid(sa + ja, sa + jb);   // absolute positions
             // lane owns the rotation pairs (i, i + d/2), i = PPL lane + j; the
             // rotation to p is loaded first so that its latency overlaps the sums
@@ -565,9 +557,13 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             float2 rot[PPL];
 #pragma unroll
             for (int j = 0; j < PPL; j++) rot[j] = A.rope[(size_t)p * HALF + i0 + j];
-            float m0[PPL], m1[PPL], v0[PPL], v1[PPL];
+            // one pass over the tokens: sum k_circ, sum R v and sum v (the weights
+            // R_t + beta need the mean R, so sum (R + beta) v = sum R v + beta sum v),
+            // and the scalars sum R, sum ||k_circ|| (the same in every lane)
+            float m0[PPL], m1[PPL], r0[PPL], r1[PPL], s0[PPL], s1[PPL];
+            float rs = 0.f, ks = 0.f;
 #pragma unroll
-            for (int j = 0; j < PPL; j++) m0[j] = m1[j] = v0[j] = v1[j] = 0.f;
+            for (int j = 0; j < PPL; j++) m0[j] = m1[j] = r0[j] = r1[j] = s0[j] = s1[j] = 0.f;
 #pragma unroll 8
             for (int t = ja; t < jb; t++) {
                 float k0[PPL], k1[PPL], x0[PPL], x1[PPL];
@@ -575,15 +571,22 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 ld_pairs<PPL>(&sm.kc[t][i0 + HALF], k1);
                 ld_pairs<PPL>(&sm.vv[t][i0], x0);
                 ld_pairs<PPL>(&sm.vv[t][i0 + HALF], x1);
-                const float wt = sm.Rt[t] + beta;
+                const float rt = sm.Rt[t];
+                rs += rt;
+                ks += sm.kn[t];
 #pragma unroll
                 for (int j = 0; j < PPL; j++) {
                     m0[j] += k0[j];
                     m1[j] += k1[j];
-                    v0[j] = fmaf(wt, x0[j], v0[j]);
-                    v1[j] = fmaf(wt, x1[j], v1[j]);
+                    r0[j] = fmaf(rt, x0[j], r0[j]);
+                    r1[j] = fmaf(rt, x1[j], r1[j]);
+                    s0[j] += x0[j];
+                    s1[j] += x1[j];
                 }
             }
+            const float ninv = 1.0f / (float)nJ;
+            const float beta = (float)A.base_frac * (rs * ninv);
+            const float winv = 1.0f / ((rs + (float)nJ * beta) + A.eps);
             float mu2 = 0.f;
 #pragma unroll
             for (int j = 0; j < PPL; j++) {
@@ -592,8 +595,8 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 const float2 cs = rot[j];
                 sm.ktil[row][i0 + j] = a0 * cs.x - a1 * cs.y;
                 sm.ktil[row][i0 + j + HALF] = a0 * cs.y + a1 * cs.x;
-                sm.vtil[row][i0 + j] = v0[j] * winv;
-                sm.vtil[row][i0 + j + HALF] = v1[j] * winv;
+                sm.vtil[row][i0 + j] = fmaf(beta, s0[j], r0[j]) * winv;
+                sm.vtil[row][i0 + j + HALF] = fmaf(beta, s1[j], r1[j]) * winv;
             }
             mu2 = warp_sum(mu2);
             if (lane == 0) {
