@@ -102,8 +102,9 @@ class ClockSampler:
                 "reasons": sorted(reasons)}
 
 
-def cpu_baseline(w, ratio: float, T_s: int = 1536):
-    """Oracle on one layer x one KV head x T_s tokens of the workload's recipe."""
+def cpu_baseline(w, ratio: float, T_s: int = 4608):
+    """Oracle on one layer x one KV head x T_s tokens of the workload's recipe
+    (about 10 s of one host core)."""
     import oracle as O
     from paper_2608_07001_gb300 import synth
     x = synth.make_inputs(w, layers=[0], heads=[0], T=T_s)
