@@ -303,6 +303,32 @@ def gather(p: Params, K, V, rtok, tr: Trees, add_sel, split_sel, cap: int):
                 offsets=off)
 
 
+def decode_attention(q, K, V, log_m, offsets, K_app=None, V_app=None, n_app: int = 0,
+                     *, L: int, G: int, l0: int = 0):
+    """Eq. (app_decode_logit) over the packed cache plus n_app appended rows.
+
+    q [nl, Hq, d]; K, V [E, d]; log_m [E]; offsets [L*G + 1];
+    K_app, V_app [L, G, app_cap, d] or None.  Returns out [nl, Hq, d]."""
+    q, K, V, log_m = map(_f64, (q, K, V, log_m))
+    nl, Hq, d = q.shape
+    off = np.ascontiguousarray(np.asarray(offsets, dtype=np.int64))
+    if K_app is None:
+        K_app = np.zeros((L, G, 1, d))
+        V_app = np.zeros((L, G, 1, d))
+    K_app, V_app = _f64(K_app), _f64(V_app)
+    app_cap = K_app.shape[2]
+    if K.size == 0:
+        K, V, log_m = np.zeros((1, d)), np.zeros((1, d)), np.zeros(1)
+    out = np.zeros((nl, Hq, d))
+    rc = lib().orc_decode_attention(*(C.c_int32(v) for v in (L, G, Hq, d, l0, nl)),
+                                    _p(q, C.c_double), _p(K, C.c_double), _p(V, C.c_double),
+                                    _p(log_m, C.c_double), _p(off, C.c_int64),
+                                    _p(K_app, C.c_double), _p(V_app, C.c_double),
+                                    C.c_int32(app_cap), C.c_int32(n_app), _p(out, C.c_double))
+    assert rc == 0, rc
+    return out
+
+
 def run(K, V, Q, B_total: int, rope_base: float, *, ctx_start=0, ctx_end=None, omega=None,
         surprisal=None, hidden=None, slot_starts=None, **overrides) -> dict:
     """Whole compression pass on the oracle; returns every intermediate."""

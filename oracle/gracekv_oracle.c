@@ -996,3 +996,56 @@ int orc_gather(const orc_params *p, const double *K, const double *V, const doub
     free(buf);
     return e <= cap ? ORC_OK : ORC_ECAP;
 }
+
+/* Decoding on the packed cache, App. A.3 Eq. (app_decode_logit) with the
+ * appends of App. A.5 ("Frontier updates and physical packing": a token
+ * generated after the compression joins its (l, g) cache with effective
+ * multiplicity 1, i.e. log m = 0).  For layer l = l0 + i and query head h of KV
+ * head g = h / (Hq / G), the entries of (l, g) are the packed ones
+ * [off[lg], off[lg + 1]) followed by the first n_app appended rows; each has
+ * the logit  x_e = q . k_e / sqrt(d) + log m_e  and the output is the
+ * softmax(x)-weighted sum of the values.  The largest logit is subtracted
+ * before exp (the weights are unchanged in exact arithmetic).  An (l, g) with
+ * no entry gives a zero output. */
+int orc_decode_attention(int32_t L, int32_t G, int32_t Hq, int32_t d, int32_t l0, int32_t nl,
+                         const double *q, const double *K, const double *V, const double *log_m,
+                         const int64_t *off, const double *K_app, const double *V_app,
+                         int32_t app_cap, int32_t n_app, double *out)
+{
+    if (G <= 0 || Hq % G || d <= 0 || l0 < 0 || nl < 0 || l0 + nl > L || n_app < 0 ||
+        n_app > app_cap)
+        return ORC_EINVAL;
+    int gq = Hq / G;
+    int64_t nmax = 0;
+    for (int lg = 0; lg < L * G; lg++)
+        if (off[lg + 1] - off[lg] > nmax) nmax = off[lg + 1] - off[lg];
+    double *x = (double *)malloc(sizeof(double) * (size_t)(nmax + n_app + 1));
+    if (!x) return ORC_ENOMEM;
+    for (int i = 0; i < nl; i++)
+        for (int h = 0; h < Hq; h++) {
+            int g = h / gq, lg = (l0 + i) * G + g;
+            const double *qh = q + ((size_t)i * Hq + h) * d;
+            double *o = out + ((size_t)i * Hq + h) * d;
+            int64_t n_pk = off[lg + 1] - off[lg], n = n_pk + n_app;
+            for (int c = 0; c < d; c++) o[c] = 0.0;
+            if (n == 0) continue;
+            double xmax = -DBL_MAX;
+            for (int64_t e = 0; e < n; e++) {
+                const double *k = e < n_pk ? K + (size_t)(off[lg] + e) * d
+                                           : K_app + ((size_t)lg * app_cap + (e - n_pk)) * d;
+                double lm = e < n_pk ? log_m[off[lg] + e] : 0.0;
+                x[e] = logit(qh, k, d) + lm;       /* logit() divides by sqrt(d) */
+                if (x[e] > xmax) xmax = x[e];
+            }
+            double z = 0.0;
+            for (int64_t e = 0; e < n; e++) z += exp(x[e] - xmax);
+            for (int64_t e = 0; e < n; e++) {
+                const double *v = e < n_pk ? V + (size_t)(off[lg] + e) * d
+                                           : V_app + ((size_t)lg * app_cap + (e - n_pk)) * d;
+                double w = exp(x[e] - xmax) / z;
+                for (int c = 0; c < d; c++) o[c] += w * v[c];
+            }
+        }
+    free(x);
+    return ORC_OK;
+}

@@ -28,6 +28,8 @@
  *   gains / costs     App. A.5 Eqs. (app_operation_gains) .. (app_unit_utility)
  *   greedy allocation App. A.5 Stage II, App. C.3 (max-priority queue)
  *   packing           App. A.5 "Frontier updates and physical packing"
+ *   decoding          App. A.3 Eq. (app_decode_logit) over the packed cache
+ *                     plus appended tokens at multiplicity 1 (App. A.5)
  *
  * Readings of silent or ambiguous passages:
  *   R1  trajectory h^(l)_t = concat_g v^(l,g)_t unless hidden states are given;
@@ -123,5 +125,13 @@ int orc_gather(const orc_params *p, const double *K, const double *V, const doub
                const uint8_t *add_sel, const uint8_t *split_sel, int64_t cap,
                double *K_out, double *V_out, int32_t *pos, double *log_m,
                int32_t *src_lo, int32_t *src_hi, int64_t *offsets, int64_t *n_entries);
+
+/* q [nl][Hq][d] for layers l0 .. l0 + nl - 1; packed cache K, V [E][d],
+ * log_m [E], off [L G + 1]; appended rows K_app, V_app [L][G][app_cap][d]
+ * (the first n_app of each (l, g) are valid); out [nl][Hq][d]. */
+int orc_decode_attention(int32_t L, int32_t G, int32_t Hq, int32_t d, int32_t l0, int32_t nl,
+                         const double *q, const double *K, const double *V, const double *log_m,
+                         const int64_t *off, const double *K_app, const double *V_app,
+                         int32_t app_cap, int32_t n_app, double *out);
 
 #endif

@@ -29,6 +29,17 @@ Recipe (one per workload, all seeded):
   the keys of its region.  Its slot boundaries are drawn, not segmented:
   length 1 with p = 0.01, U{4097..8192} with p = 0.01, else U{16..128}.
 
+Decoding inputs (make_decode_cache) stand in for a packed compressed cache
+at compression ratio x: L G T / x entries split over the (l, g) by
+lognormal(0, 0.35) shares (largest remainder, at least 32 each); within an
+(l, g) the last 32 entries are a recent window of single tokens, and every
+other entry is a single token with p = 0.3, else a prototype of n = 2^U(1, 7)
+tokens with coherence c ~ U(0.35, 1): log m = log clamp(n c, 1, n), key
+N(0, c) per channel, value N(0, 1) times U(0.3, 1).  Single tokens carry
+N(0, 1) keys and values and log m = 0.  Decode queries are N(0, 1) per
+channel, every other query head scaled by 3 (sharper softmax).  Appended
+rows are N(0, 1).  These are draws, not the compression's arithmetic.
+
 Every tensor is produced on the requested device with a torch.Generator
 seeded from numpy's SeedSequence(seed, spawn_key=(...)), so a slice (a subset
 of layers / heads) regenerates independently of the rest.  CPU and CUDA
@@ -45,7 +56,7 @@ import numpy as np
 import torch
 
 __all__ = ["Workload", "WORKLOADS", "Inputs", "make_inputs", "segment_lengths",
-           "supplied_slots"]
+           "supplied_slots", "DecodeCache", "make_decode_cache"]
 
 
 @dataclasses.dataclass(frozen=True)
@@ -234,3 +245,68 @@ def make_inputs(w: Workload, device="cpu", layers: Optional[Sequence[int]] = Non
         slots = supplied_slots(w, T - 32)
     return Inputs(K, V, Q, lens, slots, layers, heads)
 
+
+
+@dataclasses.dataclass
+class DecodeCache:
+    q: torch.Tensor           # [L, Hq, d] decode queries (one step)
+    K: torch.Tensor           # [E, d] packed keys
+    V: torch.Tensor           # [E, d] packed values
+    log_m: torch.Tensor       # [E] fp32
+    offsets: torch.Tensor     # [L*G + 1] int64
+    K_app: torch.Tensor       # [L, G, app_cap, d] appended keys
+    V_app: torch.Tensor       # [L, G, app_cap, d]
+    n_app: int
+
+
+def decode_counts(L: int, G: int, E: int, seed: int) -> np.ndarray:
+    """Entries per (l, g): lognormal(0, 0.35) shares of E, at least 32 each."""
+    rng = _np_stream(seed, 2_000_001)
+    w = rng.lognormal(0.0, 0.35, size=L * G)
+    spare = E - 32 * L * G
+    assert spare >= 0
+    exact = w * spare / w.sum()
+    base = np.floor(exact).astype(np.int64)
+    order = np.argsort(-(exact - base), kind="stable")
+    base[order[:spare - int(base.sum())]] += 1
+    return base + 32
+
+
+def make_decode_cache(w: Workload, ratio: int, n_app: int = 0, app_cap: Optional[int] = None,
+                      device="cpu", counts: Optional[np.ndarray] = None,
+                      seed: Optional[int] = None) -> DecodeCache:
+    """Seeded packed cache + appended rows + one step of decode queries."""
+    seed = w.seed if seed is None else seed
+    L, G, Hq, d = w.L, w.G, w.Hq, w.d
+    if counts is None:
+        counts = decode_counts(L, G, L * G * w.T // ratio, seed)
+    counts = np.asarray(counts, dtype=np.int64)
+    E = int(counts.sum())
+    off = np.zeros(L * G + 1, dtype=np.int64)
+    off[1:] = np.cumsum(counts)
+    rng = _np_stream(seed, 2_000_002)
+    single = rng.random(E) < 0.3
+    n = np.exp2(rng.uniform(1.0, 7.0, size=E))
+    coh = rng.uniform(0.35, 1.0, size=E)
+    vs = rng.uniform(0.3, 1.0, size=E)
+    for lg in range(L * G):                       # recent window: single tokens
+        single[max(off[lg + 1] - 32, off[lg]):off[lg + 1]] = True
+    logm = np.where(single, 0.0, np.log(np.clip(n * coh, 1.0, n)))
+    kscale = np.where(single, 1.0, np.sqrt(coh))
+    vscale = np.where(single, 1.0, vs)
+    tdt = torch.float32 if w.dtype == "f32" else torch.bfloat16
+    gen = _stream(seed, 2_000_003, device=device)
+    K = torch.randn(E, d, generator=gen, device=device)
+    K *= torch.as_tensor(kscale, dtype=torch.float32, device=device)[:, None]
+    V = torch.randn(E, d, generator=gen, device=device)
+    V *= torch.as_tensor(vscale, dtype=torch.float32, device=device)[:, None]
+    app_cap = max(n_app, 1) if app_cap is None else app_cap
+    gen = _stream(seed, 2_000_004, device=device)
+    Ka = torch.randn(L, G, app_cap, d, generator=gen, device=device)
+    Va = torch.randn(L, G, app_cap, d, generator=gen, device=device)
+    gen = _stream(seed, 2_000_005, device=device)
+    q = torch.randn(L, Hq, d, generator=gen, device=device)
+    q[:, 1::2] *= 3.0
+    return DecodeCache(q.to(tdt), K.to(tdt), V.to(tdt),
+                       torch.as_tensor(logm, dtype=torch.float32, device=device),
+                       torch.as_tensor(off, device=device), Ka.to(tdt), Va.to(tdt), n_app)
