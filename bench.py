@@ -152,6 +152,99 @@ def workload_config(w, ratio, L=None):
             "l2": "inputs larger than L2 (no flush needed)"}
 
 
+def decode_leg(args, w, comp, L, G, Hq, d, dev):
+    """Decoding on the cache the pass just wrote (Eq. app_decode_logit).
+
+    One decode step of one token: for every layer, the new token's K/V is
+    appended to its (l, g) (multiplicity 1) and the attention of the Hq query
+    heads runs over the packed entries plus the appended rows.  Timed two
+    ways, CUDA events on the launching stream, after warm-up:
+      * all_layers: one attention launch over the L layers (the bandwidth
+        figure of the kernel; it sets the roofline below),
+      * per_layer:  L x (append + attention) launches, replayed from a CUDA
+        graph (the per-token cost when the model runs layer by layer).
+    The packed cache is larger than L2, so repeated steps read it from HBM.
+    """
+    from paper_2608_07001_gb300 import gracekv as gk
+    c = comp.cache
+    E = comp.n_entries
+    n_app = args.decode_app
+    dec = gk.Decoder(c.K[:max(E, 1)], c.V[:max(E, 1)], c.log_m[:max(E, 1)], c.offsets,
+                     L=L, G=G, Hq=Hq, app_cap=n_app + 1)
+    gen = torch.Generator(device=dev).manual_seed(7)
+    dt = c.K.dtype
+    dec.K_app.copy_(torch.randn(dec.K_app.shape, generator=gen, device=dev).to(dt))
+    dec.V_app.copy_(torch.randn(dec.V_app.shape, generator=gen, device=dev).to(dt))
+    q = torch.randn(L, Hq, d, generator=gen, device=dev).to(dt)
+    k_new = torch.randn(L, G, d, generator=gen, device=dev).to(dt)
+    v_new = torch.randn(L, G, d, generator=gen, device=dev).to(dt)
+    out = torch.empty(L, Hq, d, device=dev, dtype=torch.float32)
+    qs = [q[l:l + 1] for l in range(L)]
+    ks = [k_new[l:l + 1] for l in range(L)]
+    vs = [v_new[l:l + 1] for l in range(L)]
+    outs = [out[l:l + 1] for l in range(L)]
+
+    def step_all():
+        dec.n_app = n_app
+        dec.append(k_new, v_new)                      # row n_app of every (l, g); n_app + 1 rows
+        dec.attention(q, out=out)
+
+    def step_layers():
+        for l in range(L):
+            dec.n_app = n_app
+            dec.append(ks[l], vs[l], l0=l)
+            dec.n_app = n_app + 1
+            dec.attention(qs[l], l0=l, out=outs[l])
+
+    s = torch.cuda.current_stream(dev)
+    for _ in range(max(args.warmup, 3)):
+        step_all()
+        step_layers()
+    torch.cuda.synchronize(dev)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        step_layers()
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize(dev)
+    reps = 50
+    e = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
+    e[0].record(s)
+    for _ in range(reps):
+        dec.attention(q, out=out)                    # the attention kernel alone
+    e[1].record(s)
+    for _ in range(reps):
+        step_all()
+    e[2].record(s)
+    for _ in range(reps):
+        g.replay()
+    e[3].record(s)
+    torch.cuda.synchronize(dev)
+    dec.status()
+    t_kern = e[0].elapsed_time(e[1]) / reps
+    t_all = e[1].elapsed_time(e[2]) / reps
+    t_layers = e[2].elapsed_time(e[3]) / reps
+    elem = c.K.element_size()
+    rows = E + L * G * (n_app + 1)
+    # algorithmic bytes of one attention launch over all layers: every packed
+    # entry (K row, V row, log m), every appended row (K, V), the offsets,
+    # the queries and the fp32 outputs
+    byt = (E * (2 * d * elem + 4) + L * G * (n_app + 1) * 2 * d * elem + (L * G + 1) * 8
+           + L * Hq * d * (elem + 4))
+    pk, pk_kind = peaks()
+    ach = byt / (t_kern / 1e3) / 1e9
+    return {"workload": f"decode step on the {w.name}@{int(args.ratio)}x packed cache "
+                        f"({E} entries) + {n_app + 1} appended rows per (l, g)",
+            "entries_read": rows, "bytes_per_launch": byt,
+            "us_attention_all_layers": t_kern * 1e3,
+            "us_per_token_all_layers": t_all * 1e3,
+            "us_per_token_per_layer_graph": t_layers * 1e3,
+            "tokens_per_s_per_layer_graph": 1e3 / t_layers,
+            "roofline": {"kernel": "decode_attention_kernel", "bound": "hbm", "achieved": ach,
+                         "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": ach / pk["hbm_gbs"],
+                         "peak_kind": pk_kind, "traffic": None}}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -166,6 +259,12 @@ def main():
     ap.add_argument("--ref-tokens", type=int, default=1024)
     ap.add_argument("--layers", type=int, default=0,
                     help="compress only the first N layers (small cases for profiler captures)")
+    ap.add_argument("--no-decode", action="store_true",
+                    help="skip the decoding-attention leg on the compressed cache")
+    ap.add_argument("--decode-only", action="store_true",
+                    help="compress once, then time only the decoding attention")
+    ap.add_argument("--decode-app", type=int, default=64,
+                    help="tokens already appended to every (l, g) when decoding is timed")
     args = ap.parse_args()
 
     from paper_2608_07001_gb300 import synth
@@ -199,6 +298,14 @@ def main():
         if dist is not None:
             dist.barrier()
         torch.cuda.synchronize(dev)
+
+    if args.decode_only:
+        comp(K, V, Q)
+        torch.cuda.synchronize(dev)
+        dec = decode_leg(args, w, comp, L, G, Q.shape[1], d, dev)
+        if rank == 0:
+            print(json.dumps({"decode": dec}))
+        return
 
     for _ in range(args.warmup):
         comp(K, V, Q)
@@ -297,6 +404,10 @@ def main():
         v, dt, sample = cpu_baseline(w, args.ratio)
         cpu = {"value": v, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": sample}
 
+    dec = None
+    if not args.no_decode:
+        dec = decode_leg(args, w, comp, L, G, Q.shape[1], d, dev)
+
     if rank == 0:
         out = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
                "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
@@ -306,7 +417,7 @@ def main():
                               slots=comp.n_slots, parallelism=f"replicas{world}"),
                "roofline": roof, "hbm_pass": hbm, "stages_ms": per_step, "tree_work": work,
                "cpu_baseline": cpu, "e2e": e2e,
-               "gpu_launches": launches1 - launches0, "clocks": clocks}
+               "gpu_launches": launches1 - launches0, "clocks": clocks, "decode": dec}
         print(json.dumps(out))
     if dist is not None:
         dist.destroy_process_group()

@@ -14,6 +14,9 @@
  *   gracekv_allocate     global greedy Add/Split allocation   (App. A.5, C.3)
  *   gracekv_gather       ragged compressed cache + index map  (App. A.5)
  *
+ * Decoding on the result (gracekv_decode_*, App. A.3 Eq. app_decode_logit)
+ * follows at the end of this header.
+ *
  * Conventions for every call:
  *   - Tensor arguments are DEVICE pointers to contiguous row-major arrays owned
  *     by the caller; the library never frees or retains them past the call.
@@ -38,6 +41,7 @@
 #ifndef GRACEKV_H
 #define GRACEKV_H
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -277,6 +281,68 @@ gkv_status gracekv_row_stats_noalloc(const void *K, const void *Q, int32_t L, in
                                      int32_t Hq, int32_t T, int32_t d, int32_t W, int32_t dtype,
                                      int32_t c_lo, int32_t c_hi, float *row_m, float *row_Z,
                                      float *row_ZC, void *stream);
+
+/*
+ * Decoding on the compressed cache (App. A.3, Eq. app_decode_logit, and the
+ * packing paragraph of App. A.5).  The packed cache of gracekv_gather stays
+ * read-only while decoding; every token generated afterwards is appended to
+ * its (l, g) with effective multiplicity 1 (log m = 0), in an append area the
+ * caller owns.  For layer l, query head h of KV head g = h / (Hq / G):
+ *     x_e = q_h . k_e / sqrt(d) + log m_e  over the entries e of (l, g),
+ *     out_h = sum_e softmax(x)_e v_e ;
+ * the entries of (l, g) are the packed ones [offsets[lg], offsets[lg + 1])
+ * followed by the first n_app appended rows.  An (l, g) with no entry gives a
+ * zero output.  These calls need no context and never allocate.
+ *
+ * gkv_decode_cache describes the cache (all pointers DEVICE memory, owned by
+ * the caller): L, G, Hq, d and dtype as at compression (d in {64, 128},
+ * Hq / G in {1, 2, 4, 8}, else GKV_EUNSUPPORTED); K, V [n_entries][d] dtype
+ * (16-byte aligned), log_m [n_entries] fp32 and offsets [L G + 1] int64 as
+ * written by gracekv_gather, n_entries = E its count (below 2^31; offsets past
+ * it make gracekv_decode_status report GKV_EINVAL and nothing is read);
+ * K_app, V_app [L][G][app_cap][d] dtype (16-byte aligned; nullable when
+ * app_cap = 0).
+ */
+typedef struct {
+    int32_t L, G, Hq, d, dtype;
+    const void *K, *V;
+    const float *log_m;
+    const int64_t *offsets;
+    int64_t n_entries;
+    void *K_app, *V_app;
+    int32_t app_cap;
+} gkv_decode_cache;
+
+/* Bytes of the device workspace gracekv_decode_attention needs for this
+ * cache geometry (the per-piece partials, a counter per (l, g) and a status
+ * word).  The caller allocates it 256-byte aligned and zeroes it once; every
+ * call leaves it zeroed again (the status word aside, see
+ * gracekv_decode_status).  One workspace serves one stream at a time. */
+gkv_status gracekv_decode_workspace_size(const gkv_decode_cache *c, size_t *bytes);
+
+/* Append the new token of layers [l0, l0 + n_layers): k_new, v_new
+ * [n_layers][G][d] dtype (device, 16-byte aligned) become row n_app of the
+ * append area of each (l, g).  The caller then counts n_app + 1 rows.
+ * Errors: GKV_EINVAL, GKV_ECAPACITY (n_app >= app_cap), GKV_ECUDA. */
+gkv_status gracekv_decode_append(const gkv_decode_cache *c, int32_t l0, int32_t n_layers,
+                                 int32_t n_app, const void *k_new, const void *v_new, void *stream);
+
+/* Decoding attention of layers [l0, l0 + n_layers) over the packed entries
+ * and the first n_app appended rows.  q [n_layers][Hq][d] dtype (device,
+ * already rotated for the current position, like the cached keys); out
+ * [n_layers][Hq][d] fp32 (device, 16-byte aligned).  Asynchronous on
+ * `stream`; a device-side failure sets the workspace's status word, which
+ * gracekv_decode_status reports.  Errors: GKV_EINVAL (shapes, pointers,
+ * n_app > app_cap), GKV_EUNSUPPORTED, GKV_ECUDA. */
+gkv_status gracekv_decode_attention(const gkv_decode_cache *c, int32_t l0, int32_t n_layers,
+                                    int32_t n_app, const void *q, float *out, void *workspace,
+                                    void *stream);
+
+/* Synchronises `stream` and reports (then clears) the workspace's status
+ * word: GKV_ETIMEOUT when a bounded device-side wait of an earlier
+ * gracekv_decode_attention on this workspace gave up, GKV_EINVAL when the
+ * offsets of a call pointed past n_entries, else GKV_OK. */
+gkv_status gracekv_decode_status(void *workspace, void *stream);
 
 #ifdef __cplusplus
 }

@@ -386,20 +386,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(
 }
 
 // ---- host side -------------------------------------------------------------
-PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
-std::once_flag g_encode_once;
-
-PFN_cuTensorMapEncodeTiled_v12000 encoder() {
-    std::call_once(g_encode_once, [] {
-        void *fn = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-    });
-    return g_encode;
-}
+PFN_cuTensorMapEncodeTiled_v12000 encoder() { return tc::tensor_map_encoder(); }
 
 // [rows][DH] row-major bf16, boxes of [128 rows][64 columns], 128-byte swizzle.
 bool make_map(CUtensorMap *m, const void *p, int64_t rows, int DH, int box_rows = 128) {

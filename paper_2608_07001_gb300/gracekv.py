@@ -40,6 +40,15 @@ class GkvParams(C.Structure):
     ]
 
 
+class GkvDecodeCache(C.Structure):
+    _fields_ = [
+        ("L", C.c_int32), ("G", C.c_int32), ("Hq", C.c_int32), ("d", C.c_int32),
+        ("dtype", C.c_int32), ("K", C.c_void_p), ("V", C.c_void_p), ("log_m", C.c_void_p),
+        ("offsets", C.c_void_p), ("n_entries", C.c_int64), ("K_app", C.c_void_p),
+        ("V_app", C.c_void_p), ("app_cap", C.c_int32),
+    ]
+
+
 class GraceKVError(RuntimeError):
     def __init__(self, status: int, msg: str):
         super().__init__(f"gracekv status {status}: {msg}")
@@ -52,7 +61,8 @@ EXPORTED = ["gracekv_default_params", "gracekv_budget_for_ratio", "gracekv_creat
             "gracekv_destroy", "gracekv_last_error", "gracekv_status_string", "gracekv_query",
             "gracekv_segment", "gracekv_score", "gracekv_build_trees", "gracekv_allocate", "gracekv_gather",
             "gracekv_export", "gracekv_profile", "gracekv_stats", "gracekv_row_stats_noalloc",
-            "gracekv_compress_host"]
+            "gracekv_compress_host", "gracekv_decode_workspace_size", "gracekv_decode_append",
+            "gracekv_decode_attention", "gracekv_decode_status"]
 
 
 def lib() -> C.CDLL:
@@ -85,6 +95,11 @@ def lib() -> C.CDLL:
     L.gracekv_profile.argtypes = [vp, i32]
     L.gracekv_stats.argtypes = [vp, vp, i32, C.POINTER(i64), vp, i32]
     L.gracekv_row_stats_noalloc.argtypes = [vp, vp] + [i32] * 9 + [vp, vp, vp, vp]
+    dcp = C.POINTER(GkvDecodeCache)
+    L.gracekv_decode_workspace_size.argtypes = [dcp, C.POINTER(C.c_size_t)]
+    L.gracekv_decode_append.argtypes = [dcp, i32, i32, i32, vp, vp, vp]
+    L.gracekv_decode_attention.argtypes = [dcp, i32, i32, i32, vp, vp, vp, vp]
+    L.gracekv_decode_status.argtypes = [vp, vp]
     _lib = L
     return L
 
@@ -332,3 +347,60 @@ class Compressor:
         self.n_entries = c.gracekv_allocate(stream)
         c.gracekv_gather(K, V, self.cache, stream)
         return self.cache
+
+
+def _raise(st: int):
+    if st != GKV_OK:
+        raise GraceKVError(st, lib().gracekv_status_string(st).decode())
+
+
+class Decoder:
+    """Decoding attention on a packed cache (gracekv_decode_* of the C ABI).
+
+    K, V [E, d], log_m [E] fp32 and offsets [L*G + 1] int64 are the device
+    outputs of gracekv_gather (or any cache in that layout); the append area
+    [L, G, app_cap, d] and the workspace are allocated here.  ``n_app`` counts
+    the appended rows; ``append`` adds one row to every (l, g) of the layers
+    it is given and ``attention`` reads the packed entries plus the first
+    ``n_app`` appended rows.
+    """
+
+    def __init__(self, K, V, log_m, offsets, *, L: int, G: int, Hq: int, app_cap: int = 0):
+        d = K.shape[1]
+        if K.numel() == 0:              # no packed entry at all: pass a valid address
+            K = V = torch.zeros(1, d, dtype=K.dtype, device=K.device)
+            log_m = torch.zeros(1, dtype=torch.float32, device=K.device)
+        self.dtype = K.dtype
+        dt = GKV_BF16 if K.dtype == torch.bfloat16 else GKV_F32
+        self.K_app = torch.empty(L, G, max(app_cap, 1), d, dtype=K.dtype, device=K.device)
+        self.V_app = torch.empty_like(self.K_app)
+        self._keep = (K, V, log_m, offsets)
+        ptr = lambda t: _ptr(t).value
+        self.desc = GkvDecodeCache(L, G, Hq, d, dt, ptr(K), ptr(V), ptr(log_m), ptr(offsets),
+                                   K.shape[0], ptr(self.K_app), ptr(self.V_app), app_cap)
+        n = C.c_size_t()
+        _raise(lib().gracekv_decode_workspace_size(C.byref(self.desc), C.byref(n)))
+        self.workspace = torch.zeros(n.value, dtype=torch.uint8, device=K.device)
+        self.L, self.G, self.Hq, self.d = L, G, Hq, d
+        self.n_app = 0
+
+    def append(self, k_new, v_new, l0: int = 0, stream=None):
+        """k_new, v_new [n_layers, G, d]: row n_app of layers l0.. (n_app is
+        advanced when the call covers the last layer)."""
+        nl = k_new.shape[0]
+        _raise(lib().gracekv_decode_append(C.byref(self.desc), l0, nl, self.n_app, _ptr(k_new),
+                                           _ptr(v_new), _stream(stream)))
+        if l0 + nl == self.L:
+            self.n_app += 1
+
+    def attention(self, q, l0: int = 0, out=None, stream=None):
+        """q [n_layers, Hq, d] -> out [n_layers, Hq, d] fp32."""
+        nl = q.shape[0]
+        if out is None:
+            out = torch.empty(nl, self.Hq, self.d, dtype=torch.float32, device=q.device)
+        _raise(lib().gracekv_decode_attention(C.byref(self.desc), l0, nl, self.n_app, _ptr(q),
+                                              _ptr(out), _ptr(self.workspace), _stream(stream)))
+        return out
+
+    def status(self, stream=None):
+        _raise(lib().gracekv_decode_status(_ptr(self.workspace), _stream(stream)))
