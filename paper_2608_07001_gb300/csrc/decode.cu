@@ -9,7 +9,7 @@
 //
 // The work is one read of the cache: 2 d elements per entry plus log m, with
 // O(gq d) arithmetic per entry (gq = Hq / G query heads share one KV head).
-// So the kernel is built for HBM bandwidth:
+// So the kernels are built for HBM bandwidth:
 //
 //   * The entries of the launch -- for every (l, g) its packed range
 //     [off[lg], off[lg+1]) followed by its first n_app appended rows -- form one
@@ -17,17 +17,20 @@
 //     whatever the per-head lengths (the global allocation makes them very
 //     uneven).  A chunk meets one or more (l, g); each meeting is a "piece".
 //   * One producer lane streams the rows of a piece through a ring of shared
-//     memory, completion on mbarriers: first the keys of a sub-chunk, then its
-//     values.  bf16 caches arrive as 2-D TMA tiles with the 128-byte swizzle;
-//     fp32 caches as 1-D bulk copies of whole rows.  Keys and values are read
-//     from HBM exactly once.
-//   * Eight consumer warps compute, per sub-chunk, the base-2 logits of all gq
-//     heads -- bf16: one m16n8k16 tensor-core MMA per 16 rows x 16 channels
-//     (exact products, fp32 sums; the gq queries are the 8-column operand);
-//     fp32: packed fp32x2 FMA and a butterfly across the lanes of a row --,
-//     the sub-chunk maximum, the weights p = 2^(x - M) in fp32 and the
-//     weighted value sums with packed fp32x2 FMA (the weights never leave
-//     fp32).
+//     memory, completion on mbarriers: the keys of a sub-chunk, then its
+//     values; packed rows and appended rows go to separate stages.  bf16
+//     caches arrive as 2-D TMA tiles with the 128-byte swizzle; fp32 caches as
+//     1-D bulk copies of whole rows.  Keys and values are read from HBM once.
+//   * bf16 (decode_tc_kernel): eight consumer warps run both products on the
+//     tensor cores (m16n8k16, exact bf16 products, fp32 sums).  Logits: the
+//     keys are the 16-row operand and the gq queries the 8-column one.  After
+//     the sub-chunk maximum, the fp32 weights p = 2^(x - M) are split exactly
+//     enough into three bf16 parts (hi + mid + lo, residual below 2^-26 p)
+//     that form the 8-column operand of the value product, whose 16-row
+//     operand is a 16-channel slice of the values (ldmatrix.trans); each warp
+//     owns one channel slice, so its accumulator is the piece's result.
+//   * fp32 (decode_cc_kernel): the same flow on CUDA cores -- packed fp32x2
+//     FMA, a butterfly across the lanes of a row for the logits.
 //   * A piece leaves (max, sum of weights, weighted value sum) per head.  The
 //     CTA that finishes the last piece of an (l, g) -- found with an atomic
 //     counter after a memory fence, nothing waits on anything -- merges the
@@ -76,34 +79,44 @@ struct DecArgs {
     float qscale;               // log2(e) / sqrt(d)
 };
 
+// Tensor maps of the bf16 path: [rows][d] with boxes of [RPS rows][64 columns]
+// and the 128-byte swizzle, for the packed and the appended keys and values.
+struct DecMaps {
+    CUtensorMap K, V, Ka, Va;
+};
+
 template <typename T, int D, int GQ>
 struct DecCfg {
-    static constexpr bool TC = sizeof(T) == 2;               // bf16: tensor-core logits, swizzled tiles
-    static constexpr int NB = D / 64;                        // 64-column boxes per row (bf16)
+    static constexpr bool TC = sizeof(T) == 2;               // bf16: tensor cores, swizzled tiles
     static constexpr int RB = D * (int)sizeof(T);            // bytes per row
+    static constexpr int RPS = kDecStageBytes / RB;          // rows per ring stage
+    static constexpr int SUB = TC ? 512 : 2048 / GQ;         // entries per sub-chunk
+    static constexpr int EPT = SUB / (kDecWarps * 32);       // sub-chunk entries per consumer thread
+    static constexpr int PART = GQ * (D + 2);                // floats per piece partial
+    // tensor-core path
+    static constexpr int NB = D / 64;                        // 64-column boxes per row
+    static constexpr int TPS = RPS / 16;                     // 16-row steps per stage
+    static constexpr int MAXST = SUB / RPS + 1;              // stages of one sub-chunk, at most
+    static constexpr int NMT = D / 16;                       // 16-channel slices of the values
+    static constexpr int WPM = kDecWarps / NMT;              // warps per slice
+    static constexpr int FRW = MAXST * TPS * 3 * 64;         // words of the weight operands
+    // CUDA-core path
     static constexpr int CPR = RB / 16;                      // 16-byte chunks per row
     static constexpr int LPR = CPR < 16 ? CPR : 16;          // lanes per row
     static constexpr int CPL = CPR / LPR;                    // chunks per lane
     static constexpr int EPC = 16 / (int)sizeof(T);          // elements per chunk
     static constexpr int EPL = CPL * EPC;                    // elements per lane
     static constexpr int RPW = 32 / LPR;                     // rows per warp step
-    static constexpr int RPS = kDecStageBytes / RB;          // rows per ring stage
-    static constexpr int SUB = 2048 / GQ;                    // entries per sub-chunk
-    static constexpr int EPT = SUB / (kDecWarps * 32);       // sub-chunk entries per consumer thread
-    static constexpr int RED = kDecWarps * GQ * D;           // floats of the cross-warp reduction
-    static constexpr int LGB = 2 * SUB * GQ;                 // floats of the two logit buffers
-    static constexpr int SCR = RED > LGB ? RED : LGB;
-    static constexpr int PART = GQ * (D + 2);                // floats per piece partial
-    static constexpr int TPS = RPS / 16;                     // 16-row MMA tiles per stage (bf16)
-    static_assert(GQ <= LPR && LPR * RPW == 32 && SUB % RPS == 0, "decode tiling");
-    static_assert(RPS % (kDecWarps * RPW) == 0, "decode stage rows");
-    static_assert(SUB % (kDecWarps * 32) == 0, "decode sub-chunk");
-};
-
-// Tensor maps of the bf16 path: [rows][d] with boxes of [RPS rows][64 columns]
-// and the 128-byte swizzle, for the packed and the appended keys and values.
-struct DecMaps {
-    CUtensorMap K, V, Ka, Va;
+    // shared memory after the head and the ring (floats)
+    static constexpr int LGF = TC ? SUB * GQ : 2 * SUB * GQ; // logits (two buffers on CUDA cores)
+    static constexpr int FRF = TC ? FRW : 0;
+    static constexpr int REDF = TC ? (WPM > 1 ? WPM * GQ * D : 0) : kDecWarps * GQ * D;
+    static constexpr int SUMF = GQ * D;
+    static constexpr size_t SMEM =
+        1024 + (size_t)kDecStages * kDecStageBytes + (size_t)(LGF + FRF + REDF + SUMF) * sizeof(float);
+    static_assert(SUB % RPS == 0 && SUB % (kDecWarps * 32) == 0, "decode sub-chunk");
+    static_assert(!TC || (RPS % 16 == 0 && kDecWarps % NMT == 0 && TPS % WPM == 0), "decode tensor tiles");
+    static_assert(TC || (GQ <= LPR && LPR * RPW == 32 && RPS % (kDecWarps * RPW) == 0), "decode lanes");
 };
 
 struct alignas(16) DecSmemHead {
@@ -111,6 +124,7 @@ struct alignas(16) DecSmemHead {
     uint64_t empty[kDecStages];
     float wmax[kDecWarps][8];
     float wsum[kDecWarps][8];
+    float hsum[8];
     int abort;
     int last;
 };
@@ -121,9 +135,13 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t
         "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar)
         : "memory");
 }
-
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t a[4]) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3])
+                 : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t a[4]) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
                  : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3])
                  : "r"(addr));
 }
@@ -134,18 +152,19 @@ __device__ __forceinline__ void mma16816(float c[4], const uint32_t a[4], uint32
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
+// Two floats rounded to bf16 (lo -> bits 0..15, hi -> bits 16..31).
+__device__ __forceinline__ uint32_t bf16x2_rn(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
 
-// Byte offset, inside a stage, of the 16-byte chunk `ch` (of 128-byte row
-// halves) of row r.  bf16 stages hold NB boxes of [RPS][128 B], each written
-// by TMA with the 128-byte swizzle (chunk ^ row % 8; the stage is 1024-byte
-// aligned); fp32 stages hold plain rows.
-template <typename T, int D, int GQ>
-__device__ __forceinline__ uint32_t chunk_off(int r, int ch) {
-    using C = DecCfg<T, D, GQ>;
-    if constexpr (C::TC)
-        return (uint32_t)((ch >> 3) * C::RPS * 128 + r * 128 + (((ch & 7) ^ (r & 7)) << 4));
-    else
-        return (uint32_t)(r * C::RB + ch * 16);
+// Byte offset, inside a bf16 stage, of the 16-byte chunk `ch` of row r: the
+// stage holds NB boxes of [RPS][128 B] written by TMA with the 128-byte
+// swizzle (chunk ^ row % 8; stages are 1024-byte aligned).
+template <int RPS>
+__device__ __forceinline__ uint32_t sw_off(int r, int ch) {
+    return (uint32_t)((ch >> 3) * RPS * 128 + r * 128 + (((ch & 7) ^ (r & 7)) << 4));
 }
 
 // Bounded wait that also gives up at once when another thread has given up.
@@ -180,61 +199,39 @@ __device__ __forceinline__ int chunk_of(int64_t i, int64_t total, int64_t nc) {
     return (int)(((i + 1) * nc + total - 1) / total - 1);
 }
 
-template <typename T>
-__device__ __forceinline__ void chunk_to_float(const uint4 &u, float *f);
-template <>
-__device__ __forceinline__ void chunk_to_float<__nv_bfloat16>(const uint4 &u, float *f) {
-    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-    for (int i = 0; i < 4; i++) {
-        f[2 * i] = __uint_as_float(w[i] << 16);
-        f[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
-    }
-}
-template <>
-__device__ __forceinline__ void chunk_to_float<float>(const uint4 &u, float *f) {
-    f[0] = __uint_as_float(u.x);
-    f[1] = __uint_as_float(u.y);
-    f[2] = __uint_as_float(u.z);
-    f[3] = __uint_as_float(u.w);
-}
-
-template <typename T, int D, int GQ>
-__global__ void __launch_bounds__(kDecThreads, 2)
-    decode_attention_kernel(const DecArgs a, const __grid_constant__ DecMaps maps) {
-    using C = DecCfg<T, D, GQ>;
-    extern __shared__ __align__(1024) unsigned char dsm[];
-    DecSmemHead &hd = *reinterpret_cast<DecSmemHead *>(dsm);
-    unsigned char *ring = dsm + 1024;          // 1024-byte aligned stages (swizzle atoms)
-    float *scr = reinterpret_cast<float *>(ring + kDecStages * kDecStageBytes);
-
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+// The CTA's share of the launch: chunk [lo, hi) of the virtual sequence, the
+// first head it meets, the number of chunks.  Block 0 also writes the zero
+// outputs of heads without any entry.  Returns false when the CTA has no
+// work (or the offsets do not fit the cache).
+template <int D, int GQ>
+__device__ __forceinline__ bool dec_setup(const DecArgs &a, int64_t &lo, int64_t &hi, int64_t &total, int64_t &nc, int &s_first) {
+    const int tid = threadIdx.x;
     if (a.off[a.s0 + a.nS] > a.n_entries) {      // the offsets do not fit the cache
-        if (blockIdx.x == 0 && threadIdx.x == 0) atomicOr(a.status, kDecStatusRange);
-        return;
+        if (blockIdx.x == 0 && tid == 0) atomicOr(a.status, kDecStatusRange);
+        return false;
     }
-    const int64_t total = vstart(a, a.s0 + a.nS);
-    const int64_t nc = total < (int64_t)gridDim.x ? total : (int64_t)gridDim.x;
-
-    // heads without any entry give zeros (the merging below never visits them)
+    total = vstart(a, a.s0 + a.nS);
+    nc = total < (int64_t)gridDim.x ? total : (int64_t)gridDim.x;
     if (blockIdx.x == 0)
         for (int s = a.s0 + tid; s < a.s0 + a.nS; s += kDecThreads)
             if (a.off[s + 1] == a.off[s] && a.n_app == 0) {
                 float *o = a.out + ((size_t)(s / a.G - a.s0 / a.G) * a.Hq + (size_t)(s % a.G) * GQ) * D;
                 for (int i = 0; i < GQ * D; i++) o[i] = 0.f;
             }
-    if ((int64_t)blockIdx.x >= nc) return;
-    const int64_t lo = (int64_t)blockIdx.x * total / nc, hi = ((int64_t)blockIdx.x + 1) * total / nc;
-
-    // first head of the chunk: the last s with vstart(s) <= lo
-    int sb = a.s0, se = a.s0 + a.nS;
+    if ((int64_t)blockIdx.x >= nc) return false;
+    lo = (int64_t)blockIdx.x * total / nc;
+    hi = ((int64_t)blockIdx.x + 1) * total / nc;
+    int sb = a.s0, se = a.s0 + a.nS;              // the last s with vstart(s) <= lo
     while (se - sb > 1) {
         const int mid = (sb + se) >> 1;
         if (vstart(a, mid) <= lo) sb = mid; else se = mid;
     }
-    const int s_first = sb;
+    s_first = sb;
+    return true;
+}
 
-    if (tid == 0) {
+__device__ __forceinline__ void dec_init_barriers(DecSmemHead &hd) {
+    if (threadIdx.x == 0) {
         for (int i = 0; i < kDecStages; i++) {
             tc::mbar_init(tc::smem_u32(&hd.full[i]), 1);
             tc::mbar_init(tc::smem_u32(&hd.empty[i]), kDecWarps);
@@ -243,63 +240,381 @@ __global__ void __launch_bounds__(kDecThreads, 2)
         tc::fence_barrier_init();
     }
     __syncthreads();
+}
 
-    if (warp == kDecWarps) {
-        // ---------------- producer: one lane issues every bulk copy ----------------
-        if (lane == 0) {
-            uint32_t it = 0;
-            bool ok = true;
-            for (int s = s_first; ok && s < a.s0 + a.nS; s++) {
-                const int64_t vs = vstart(a, s), ve = vstart(a, s + 1);
-                if (vs >= hi) break;
-                if (ve <= lo || ve == vs) continue;      // before the chunk, or no entry
-                const int64_t pa = (lo > vs ? lo : vs) - vs, pb = (hi < ve ? hi : ve) - vs;
-                const int64_t npk = a.off[s + 1] - a.off[s];
-                for (int64_t sa = pa; ok && sa < pb; sa += C::SUB) {
-                    const int64_t sbnd = sa + C::SUB < pb ? sa + C::SUB : pb;
-                    for (int kv = 0; ok && kv < 2; kv++) {
-                        // stages of the sub-chunk: its packed rows, then its appended rows
-                        for (int part = 0; ok && part < 2; part++) {
-                            const int64_t p0 = part ? (sa > npk ? sa : npk) : sa;
-                            const int64_t p1 = part ? sbnd : (sbnd < npk ? sbnd : npk);
-                            for (int64_t r0 = p0; r0 < p1; r0 += C::RPS, it++) {
-                                const int st = it % kDecStages;
-                                if (*(volatile int *)&hd.abort ||
-                                    !dec_wait(tc::smem_u32(&hd.empty[st]), ((it / kDecStages) & 1) ^ 1, hd,
-                                              a.status)) {
-                                    ok = false;
-                                    break;
-                                }
-                                const int64_t nr = p1 - r0 < C::RPS ? p1 - r0 : C::RPS;
-                                const int64_t row = part ? (int64_t)s * a.app_cap + (r0 - npk) : a.off[s] + r0;
-                                const uint32_t fb = tc::smem_u32(&hd.full[st]);
-                                const uint32_t dst = tc::smem_u32(ring + st * kDecStageBytes);
-                                if constexpr (C::TC) {
-                                    // whole boxes (rows past the tensor read as zeros)
-                                    const CUtensorMap *mp = part ? (kv ? &maps.Va : &maps.Ka) : (kv ? &maps.V : &maps.K);
-                                    tc::mbar_expect_tx(fb, (uint32_t)(C::NB * C::RPS * 128));
+// Producer lane: every stage of every piece of the chunk, in the order the
+// consumers take them -- per sub-chunk the key stages, then the value stages;
+// within each, the packed rows and then the appended rows, RPS rows a stage.
+template <typename T, int D, int GQ>
+__device__ void dec_produce(const DecArgs &a, const DecMaps &maps, DecSmemHead &hd, unsigned char *ring,
+                            int64_t lo, int64_t hi, int s_first) {
+    using C = DecCfg<T, D, GQ>;
+    uint32_t it = 0;
+    bool ok = true;
+    for (int s = s_first; ok && s < a.s0 + a.nS; s++) {
+        const int64_t vs = vstart(a, s), ve = vstart(a, s + 1);
+        if (vs >= hi) break;
+        if (ve <= lo || ve == vs) continue;      // before the chunk, or no entry
+        const int64_t pa = (lo > vs ? lo : vs) - vs, pb = (hi < ve ? hi : ve) - vs;
+        const int64_t npk = a.off[s + 1] - a.off[s];
+        for (int64_t sa = pa; ok && sa < pb; sa += C::SUB) {
+            const int64_t sbnd = sa + C::SUB < pb ? sa + C::SUB : pb;
+            for (int kv = 0; ok && kv < 2; kv++)
+                for (int part = 0; ok && part < 2; part++) {
+                    const int64_t p0 = part ? (sa > npk ? sa : npk) : sa;
+                    const int64_t p1 = part ? sbnd : (sbnd < npk ? sbnd : npk);
+                    for (int64_t r0 = p0; r0 < p1; r0 += C::RPS, it++) {
+                        const int st = it % kDecStages;
+                        if (*(volatile int *)&hd.abort ||
+                            !dec_wait(tc::smem_u32(&hd.empty[st]), ((it / kDecStages) & 1) ^ 1, hd, a.status)) {
+                            ok = false;
+                            break;
+                        }
+                        const int64_t nr = p1 - r0 < C::RPS ? p1 - r0 : C::RPS;
+                        const int64_t row = part ? (int64_t)s * a.app_cap + (r0 - npk) : a.off[s] + r0;
+                        const uint32_t fb = tc::smem_u32(&hd.full[st]);
+                        const uint32_t dst = tc::smem_u32(ring + st * kDecStageBytes);
+                        if constexpr (C::TC) {
+                            // whole boxes (rows past the tensor read as zeros)
+                            const CUtensorMap *mp = part ? (kv ? &maps.Va : &maps.Ka) : (kv ? &maps.V : &maps.K);
+                            tc::mbar_expect_tx(fb, (uint32_t)(C::NB * C::RPS * 128));
 #pragma unroll
-                                    for (int b = 0; b < C::NB; b++)
-                                        tc::tma_load_2d(dst + (uint32_t)(b * C::RPS * 128), mp, b * 64, (int)row, fb);
-                                } else {
-                                    const char *src = part ? (kv ? a.Va : a.Ka) : (kv ? a.V : a.K);
-                                    tc::mbar_expect_tx(fb, (uint32_t)(nr * C::RB));
-                                    bulk_g2s(dst, src + row * C::RB, (uint32_t)(nr * C::RB), fb);
-                                }
-                            }
+                            for (int b = 0; b < C::NB; b++)
+                                tc::tma_load_2d(dst + (uint32_t)(b * C::RPS * 128), mp, b * 64, (int)row, fb);
+                        } else {
+                            const char *src = part ? (kv ? a.Va : a.Ka) : (kv ? a.V : a.K);
+                            tc::mbar_expect_tx(fb, (uint32_t)(nr * C::RB));
+                            bulk_g2s(dst, src + row * C::RB, (uint32_t)(nr * C::RB), fb);
                         }
                     }
                 }
-            }
-            // the copies still in flight land before the block exits
-            const uint32_t n_issued = it;
-            for (uint32_t i = n_issued > kDecStages ? n_issued - kDecStages : 0; i < n_issued; i++)
-                tc::mbar_wait(tc::smem_u32(&hd.full[i % kDecStages]), (i / kDecStages) & 1, kDecWaitNs);
         }
+    }
+    // the copies still in flight land before the block exits
+    for (uint32_t i = it > kDecStages ? it - kDecStages : 0; i < it; i++)
+        tc::mbar_wait(tc::smem_u32(&hd.full[i % kDecStages]), (i / kDecStages) & 1, kDecWaitNs);
+}
+
+// End of a piece: sums [GQ][D] (weighted value sums) and hd.hsum (sums of the
+// weights) in shared memory, mrun the running maxima (base 2).  Writes the
+// output when the piece is the whole head, else the piece's partial; the CTA
+// finishing the head's last piece merges all of them.
+template <int D, int GQ>
+__device__ __forceinline__ void dec_finish(const DecArgs &a, DecSmemHead &hd, const float *sums, const float (&mrun)[GQ], int s,
+                           int64_t vs, int64_t ve, int64_t total, int64_t nc) {
+    constexpr int PART = GQ * (D + 2);
+    const int tid = threadIdx.x;
+    const int l_rel = s / a.G - a.s0 / a.G, g = s % a.G;
+    const int c_lo = chunk_of(vs, total, nc), c_hi = chunk_of(ve - 1, total, nc);
+    float *o_base = a.out + ((size_t)l_rel * a.Hq + (size_t)g * GQ) * D;
+    if (c_lo == c_hi) {
+        for (int i = tid; i < GQ * D; i += kDecWarps * 32) o_base[i] = sums[i] / hd.hsum[i / D];
+    } else {
+        float *pp = a.part + (size_t)((s - a.s0) + (int)blockIdx.x) * PART;
+        for (int i = tid; i < GQ * D; i += kDecWarps * 32) pp[i] = sums[i];
+#pragma unroll
+        for (int h = 0; h < GQ; h++)
+            if (tid == h) {
+                pp[GQ * D + h] = mrun[h];
+                pp[GQ * D + GQ + h] = hd.hsum[h];
+            }
+        __threadfence();
+        consumer_sync();
+        if (tid == 0) hd.last = (atomicAdd(a.cnt + s, 1) == c_hi - c_lo);
+        consumer_sync();
+        if (hd.last) {
+            __threadfence();
+            for (int i = tid; i < GQ * D; i += kDecWarps * 32) {
+                const int h = i / D;
+                float M = -INFINITY;
+                for (int c = c_lo; c <= c_hi; c++)
+                    M = fmaxf(M, __ldcg(a.part + (size_t)((s - a.s0) + c) * PART + GQ * D + h));
+                float num = 0.f, den = 0.f;
+                for (int c = c_lo; c <= c_hi; c++) {
+                    const float *q = a.part + (size_t)((s - a.s0) + c) * PART;
+                    const float w = tc::ex2(__ldcg(q + GQ * D + h) - M);
+                    num += w * __ldcg(q + i);
+                    den += w * __ldcg(q + GQ * D + GQ + h);
+                }
+                o_base[i] = num / den;
+            }
+            if (tid == 0) a.cnt[s] = 0;
+        }
+    }
+    consumer_sync();                 // the sums and the head words are reused by the next piece
+}
+
+// Sub-chunk maximum of the base-2 logits (log m added into lg in place) and
+// the rescaling factors of the running sums; returns via mrun / alpha.
+template <int GQ, int EPT>
+__device__ __forceinline__ void dec_subchunk_max(DecSmemHead &hd, float *lg, const float (&lmv)[EPT], int nsub,
+                                                 float (&mrun)[GQ], float (&alpha)[GQ]) {
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    float mx[GQ];
+#pragma unroll
+    for (int h = 0; h < GQ; h++) mx[h] = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < EPT; i++) {
+        const int e = tid + i * (kDecWarps * 32);
+        if (e < nsub) {
+#pragma unroll
+            for (int h = 0; h < GQ; h++) {
+                const float x = lg[e * GQ + h] + lmv[i];
+                lg[e * GQ + h] = x;
+                mx[h] = fmaxf(mx[h], x);
+            }
+        }
+    }
+#pragma unroll
+    for (int h = 0; h < GQ; h++) {
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], o));
+        if (lane == 0) hd.wmax[warp][h] = mx[h];
+    }
+    consumer_sync();
+#pragma unroll
+    for (int h = 0; h < GQ; h++) {
+        float m = hd.wmax[0][h];
+#pragma unroll
+        for (int w = 1; w < kDecWarps; w++) m = fmaxf(m, hd.wmax[w][h]);
+        const float mn = fmaxf(mrun[h], m);
+        alpha[h] = tc::ex2(mrun[h] - mn);          // 0 on the first sub-chunk
+        mrun[h] = mn;
+    }
+}
+
+// ============================ bf16: tensor cores ============================
+template <int D, int GQ>
+__global__ void __launch_bounds__(kDecThreads, 2)
+    decode_tc_kernel(const DecArgs a, const __grid_constant__ DecMaps maps) {
+    using C = DecCfg<__nv_bfloat16, D, GQ>;
+    extern __shared__ __align__(1024) unsigned char dsm[];
+    DecSmemHead &hd = *reinterpret_cast<DecSmemHead *>(dsm);
+    unsigned char *ring = dsm + 1024;          // 1024-byte aligned stages (swizzle atoms)
+    float *lg = reinterpret_cast<float *>(ring + kDecStages * kDecStageBytes);
+    uint32_t *fr = reinterpret_cast<uint32_t *>(lg + C::LGF);
+    float *red = reinterpret_cast<float *>(fr + C::FRF);
+    float *sums = red + C::REDF;
+
+    int64_t lo, hi, total, nc;
+    int s_first;
+    if (!dec_setup<D, GQ>(a, lo, hi, total, nc, s_first)) return;
+    dec_init_barriers(hd);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    if (warp == kDecWarps) {
+        if (lane == 0) dec_produce<__nv_bfloat16, D, GQ>(a, maps, hd, ring, lo, hi, s_first);
         return;
     }
 
-    // ---------------- consumers ----------------
+    const int hq = lane >> 2, tq = lane & 3;               // MMA fragment row group / column pair
+    const int mt = warp % C::NMT, kg = warp / C::NMT;      // this warp's value channels / row steps
+    const int fl = (tid >> 1) % (4 * GQ);                  // lane of the weight operand this thread fills
+    const int hs = fl >> 2;                                // ... and its head
+    uint32_t it = 0;
+
+    for (int s = s_first; s < a.s0 + a.nS; s++) {
+        const int64_t vs = vstart(a, s), ve = vstart(a, s + 1);
+        if (vs >= hi) break;
+        if (ve <= lo || ve == vs) continue;
+        const int64_t pa = (lo > vs ? lo : vs) - vs, pb = (hi < ve ? hi : ve) - vs;
+        const int64_t npk = a.off[s + 1] - a.off[s];
+        const int l_rel = s / a.G - a.s0 / a.G, g = s % a.G;
+
+        // the queries as the logit MMA's 16 x 8 column operand: column n = head
+        // n (zero past GQ), k = channel, per 16-channel step
+        uint32_t qb[D / 16][2];
+        {
+            const uint32_t *qh = reinterpret_cast<const uint32_t *>(
+                static_cast<const __nv_bfloat16 *>(a.q) + ((size_t)l_rel * a.Hq + (size_t)g * GQ + (hq < GQ ? hq : 0)) * D);
+#pragma unroll
+            for (int kk = 0; kk < D / 16; kk++) {
+                qb[kk][0] = hq < GQ ? __ldg(qh + kk * 8 + tq) : 0u;
+                qb[kk][1] = hq < GQ ? __ldg(qh + kk * 8 + 4 + tq) : 0u;
+            }
+        }
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};   // channels 16 mt + hq (+8) x heads 2 tq, 2 tq + 1
+        float mrun[GQ], lsum = 0.f;            // lsum: head hs
+#pragma unroll
+        for (int h = 0; h < GQ; h++) mrun[h] = -INFINITY;
+
+        for (int64_t sa = pa; sa < pb; sa += C::SUB) {
+            const int64_t sbnd = sa + C::SUB < pb ? sa + C::SUB : pb;
+            const int nsub = (int)(sbnd - sa);
+            const int pk_rel = (int)(npk - sa < 0 ? 0 : (npk - sa < nsub ? npk - sa : nsub));
+            const int n_pk_st = (pk_rel + C::RPS - 1) / C::RPS;
+            const int n_st = n_pk_st + (nsub - pk_rel + C::RPS - 1) / C::RPS;
+            float lmv[C::EPT];
+#pragma unroll
+            for (int i = 0; i < C::EPT; i++) {
+                const int64_t k = sa + tid + i * (kDecWarps * 32);
+                lmv[i] = (k < sbnd && k < npk) ? __ldg(a.log_m + a.off[s] + k) * kLog2e : 0.f;
+            }
+            // ---- keys: lg[row][head] = q . k log2(e) / sqrt(d)
+            for (int st = 0; st < n_st; st++, it++) {
+                const int slot = it % kDecStages;
+                dec_wait(tc::smem_u32(&hd.full[slot]), (it / kDecStages) & 1, hd, a.status);
+                const int r0 = st < n_pk_st ? st * C::RPS : pk_rel + (st - n_pk_st) * C::RPS;
+                const int nr = min(C::RPS, (st < n_pk_st ? pk_rel : nsub) - r0);
+                const uint32_t sbase = tc::smem_u32(ring + slot * kDecStageBytes);
+                const int mi = lane >> 3, ri = lane & 7;
+#pragma unroll
+                for (int t = 0; t < C::TPS; t++) {
+                    if ((int)((it * C::TPS + t) % kDecWarps) != warp || t * 16 >= nr) continue;
+                    float c[4] = {0.f, 0.f, 0.f, 0.f};
+                    const int ar = t * 16 + ri + (mi & 1) * 8;     // row this lane addresses
+#pragma unroll
+                    for (int kk = 0; kk < D / 16; kk++) {
+                        uint32_t af[4];
+                        ldsm_x4(sbase + sw_off<C::RPS>(ar, kk * 2 + (mi >> 1)), af);
+                        mma16816(c, af, qb[kk][0], qb[kk][1]);
+                    }
+                    // c[0], c[1]: row hq, heads 2 tq, 2 tq + 1; c[2], c[3]: row hq + 8
+                    const int h0 = 2 * tq, ra = t * 16 + hq, rb = ra + 8;
+                    if (h0 < GQ) {
+                        if (ra < nr) lg[(r0 + ra) * GQ + h0] = c[0] * a.qscale;
+                        if (rb < nr) lg[(r0 + rb) * GQ + h0] = c[2] * a.qscale;
+                    }
+                    if (h0 + 1 < GQ) {
+                        if (ra < nr) lg[(r0 + ra) * GQ + h0 + 1] = c[1] * a.qscale;
+                        if (rb < nr) lg[(r0 + rb) * GQ + h0 + 1] = c[3] * a.qscale;
+                    }
+                }
+                __syncwarp();
+                if (lane == 0) tc::mbar_arrive(tc::smem_u32(&hd.empty[slot]));
+            }
+            consumer_sync();
+            float alpha[GQ];
+            dec_subchunk_max<GQ, C::EPT>(hd, lg, lmv, nsub, mrun, alpha);
+            float ahs = alpha[0], Mh = mrun[0];            // this thread's head (no dynamic indexing)
+#pragma unroll
+            for (int h = 1; h < GQ; h++)
+                if (h == hs) { ahs = alpha[h]; Mh = mrun[h]; }
+            lsum *= ahs;
+            {
+                float a0 = 0.f, a1 = 0.f;                  // heads 2 tq, 2 tq + 1 (0 past GQ)
+#pragma unroll
+                for (int h = 0; h < GQ; h++) {
+                    if (h == 2 * tq) a0 = alpha[h];
+                    if (h == 2 * tq + 1) a1 = alpha[h];
+                }
+                acc[0] *= a0; acc[1] *= a1; acc[2] *= a0; acc[3] *= a1;
+            }
+            // ---- weights as the value MMA's column operand: for each stage and
+            // 16-row step, lane (head h, tq) holds rows 2 tq, 2 tq + 1 (word 0)
+            // and 2 tq + 8, 2 tq + 9 (word 1); p = hi + mid + lo in bf16
+            {
+                const int reg = tid & 1, t4 = fl & 3;
+                const int nw = n_st * C::TPS * 8 * GQ;          // words of this sub-chunk
+                for (int w = tid; w < nw; w += kDecWarps * 32) {
+                    const int ksst = (w >> 1) / (4 * GQ);
+                    const int ks = ksst % C::TPS, st = ksst / C::TPS;
+                    const int r0 = st < n_pk_st ? st * C::RPS : pk_rel + (st - n_pk_st) * C::RPS;
+                    const int nr = min(C::RPS, (st < n_pk_st ? pk_rel : nsub) - r0);
+                    const int rr = ks * 16 + reg * 8 + 2 * t4;
+                    const float p0 = rr < nr ? tc::ex2(lg[(r0 + rr) * GQ + hs] - Mh) : 0.f;
+                    const float p1 = rr + 1 < nr ? tc::ex2(lg[(r0 + rr + 1) * GQ + hs] - Mh) : 0.f;
+                    lsum += p0 + p1;
+                    const uint32_t w_hi = bf16x2_rn(p0, p1);
+                    const float r10 = p0 - __uint_as_float(w_hi << 16), r11 = p1 - __uint_as_float(w_hi & 0xffff0000u);
+                    const uint32_t w_mid = bf16x2_rn(r10, r11);
+                    const float r20 = r10 - __uint_as_float(w_mid << 16), r21 = r11 - __uint_as_float(w_mid & 0xffff0000u);
+                    const uint32_t w_lo = bf16x2_rn(r20, r21);
+                    uint32_t *dst = fr + (size_t)(st * C::TPS + ks) * 3 * 64 + fl * 2 + reg;
+                    dst[0] = w_hi;
+                    dst[64] = w_mid;
+                    dst[128] = w_lo;
+                }
+            }
+            consumer_sync();
+            // ---- values: acc[channels][heads] += V^T P over this warp's row steps
+            for (int st = 0; st < n_st; st++, it++) {
+                const int slot = it % kDecStages;
+                dec_wait(tc::smem_u32(&hd.full[slot]), (it / kDecStages) & 1, hd, a.status);
+                const uint32_t sbase = tc::smem_u32(ring + slot * kDecStageBytes);
+                const int mi = lane >> 3;
+#pragma unroll
+                for (int ks = 0; ks < C::TPS; ks++) {
+                    if (ks % C::WPM != kg) continue;
+                    uint32_t af[4];
+                    // rows 16 ks + (lane & 7) + 8 (mi >> 1), channels 16 mt + 8 (mi & 1) .. + 7
+                    ldsm_x4_t(sbase + sw_off<C::RPS>(ks * 16 + (lane & 7) + (mi >> 1) * 8, mt * 2 + (mi & 1)), af);
+                    const uint32_t *b = fr + (size_t)(st * C::TPS + ks) * 3 * 64 + lane * 2;
+#pragma unroll
+                    for (int part = 0; part < 3; part++) {
+                        const uint2 bw = *reinterpret_cast<const uint2 *>(b + part * 64);
+                        mma16816(acc, af, bw.x, bw.y);
+                    }
+                }
+                __syncwarp();
+                if (lane == 0) tc::mbar_arrive(tc::smem_u32(&hd.empty[slot]));
+            }
+        }
+
+        // ---- piece result: weight sums per head, value sums per (head, channel)
+        // lanes 8k .. 8k + 7 of warp w share the head (4 w + k) % GQ
+#pragma unroll
+        for (int o = 1; o < 8; o <<= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
+        if ((lane & 7) == 0) hd.wsum[warp][lane >> 3] = lsum;
+        {
+            const int d0 = mt * 16 + hq, h0 = 2 * tq;
+            float *dst = C::WPM > 1 ? red + (size_t)kg * GQ * D : sums;
+            if (h0 < GQ) { dst[h0 * D + d0] = acc[0]; dst[h0 * D + d0 + 8] = acc[2]; }
+            if (h0 + 1 < GQ) { dst[(h0 + 1) * D + d0] = acc[1]; dst[(h0 + 1) * D + d0 + 8] = acc[3]; }
+        }
+        consumer_sync();
+        if (tid < GQ) {                  // fixed order: results do not depend on timing
+            float v = 0.f;
+#pragma unroll
+            for (int w = 0; w < kDecWarps; w++)
+#pragma unroll
+                for (int k = 0; k < 4; k++)
+                    if ((4 * w + k) % GQ == tid) v += hd.wsum[w][k];
+            hd.hsum[tid] = v;
+        }
+        if constexpr (C::WPM > 1) {
+            for (int i = tid; i < GQ * D; i += kDecWarps * 32) {
+                float v = 0.f;
+#pragma unroll
+                for (int k = 0; k < C::WPM; k++) v += red[(size_t)k * GQ * D + i];
+                sums[i] = v;
+            }
+        }
+        consumer_sync();
+        dec_finish<D, GQ>(a, hd, sums, mrun, s, vs, ve, total, nc);
+    }
+}
+
+// ============================ fp32: CUDA cores ==============================
+template <typename T>
+__device__ __forceinline__ void chunk_to_float(const uint4 &u, float *f) {
+    f[0] = __uint_as_float(u.x);
+    f[1] = __uint_as_float(u.y);
+    f[2] = __uint_as_float(u.z);
+    f[3] = __uint_as_float(u.w);
+}
+
+template <int D, int GQ>
+__global__ void __launch_bounds__(kDecThreads, 2)
+    decode_cc_kernel(const DecArgs a, const __grid_constant__ DecMaps maps) {
+    using T = float;
+    using C = DecCfg<T, D, GQ>;
+    extern __shared__ __align__(1024) unsigned char dsm[];
+    DecSmemHead &hd = *reinterpret_cast<DecSmemHead *>(dsm);
+    unsigned char *ring = dsm + 1024;
+    float *lgb = reinterpret_cast<float *>(ring + kDecStages * kDecStageBytes);
+    float *red = lgb + C::LGF;
+    float *sums = red + C::REDF;
+
+    int64_t lo, hi, total, nc;
+    int s_first;
+    if (!dec_setup<D, GQ>(a, lo, hi, total, nc, s_first)) return;
+    dec_init_barriers(hd);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    if (warp == kDecWarps) {
+        if (lane == 0) dec_produce<T, D, GQ>(a, maps, hd, ring, lo, hi, s_first);
+        return;
+    }
+
     const int rg = lane / C::LPR, j = lane % C::LPR;
     const int hsel = j / (C::LPR / GQ);                 // head whose logit this lane ends with
     const bool writer = (j % (C::LPR / GQ)) == 0;
@@ -314,32 +629,18 @@ __global__ void __launch_bounds__(kDecThreads, 2)
         const int64_t npk = a.off[s + 1] - a.off[s];
         const int l_rel = s / a.G - a.s0 / a.G, g = s % a.G;
 
-        // queries: fp32 -- this lane's elements of the GQ heads, pre-scaled to
-        // base 2; bf16 -- the MMA's 16 x 8 column operand (column n = head n,
-        // zero past GQ), k = channel, per 16-channel step
-        float2 q2[C::TC ? 1 : GQ][C::TC ? 1 : C::EPL / 2];
-        uint32_t qb[C::TC ? D / 16 : 1][2];
-        if constexpr (C::TC) {
-            const int hq = lane >> 2, tq = lane & 3;
-            const uint32_t *qh = reinterpret_cast<const uint32_t *>(
-                static_cast<const T *>(a.q) + ((size_t)l_rel * a.Hq + (size_t)g * GQ + (hq < GQ ? hq : 0)) * D);
+        // this lane's elements of the GQ queries, pre-scaled to base 2
+        float2 q2[GQ][C::EPL / 2];
 #pragma unroll
-            for (int kk = 0; kk < D / 16; kk++) {
-                qb[kk][0] = hq < GQ ? __ldg(qh + kk * 8 + tq) : 0u;
-                qb[kk][1] = hq < GQ ? __ldg(qh + kk * 8 + 4 + tq) : 0u;
-            }
-        } else {
+        for (int h = 0; h < GQ; h++) {
+            const T *qh = static_cast<const T *>(a.q) + ((size_t)l_rel * a.Hq + (size_t)g * GQ + h) * D;
 #pragma unroll
-            for (int h = 0; h < GQ; h++) {
-                const T *qh = static_cast<const T *>(a.q) + ((size_t)l_rel * a.Hq + (size_t)g * GQ + h) * D;
+            for (int c = 0; c < C::CPL; c++) {
+                float f[C::EPC];
+                chunk_to_float<T>(__ldg(reinterpret_cast<const uint4 *>(qh) + j + C::LPR * c), f);
 #pragma unroll
-                for (int c = 0; c < C::CPL; c++) {
-                    float f[C::EPC];
-                    chunk_to_float<T>(__ldg(reinterpret_cast<const uint4 *>(qh) + j + C::LPR * c), f);
-#pragma unroll
-                    for (int e = 0; e < C::EPC; e += 2)
-                        q2[h][(c * C::EPC + e) / 2] = make_float2(f[e] * a.qscale, f[e + 1] * a.qscale);
-                }
+                for (int e = 0; e < C::EPC; e += 2)
+                    q2[h][(c * C::EPC + e) / 2] = make_float2(f[e] * a.qscale, f[e + 1] * a.qscale);
             }
         }
         float2 acc[GQ][C::EPL / 2];
@@ -354,130 +655,74 @@ __global__ void __launch_bounds__(kDecThreads, 2)
         for (int64_t sa = pa; sa < pb; sa += C::SUB) {
             const int64_t sbnd = sa + C::SUB < pb ? sa + C::SUB : pb;
             const int nsub = (int)(sbnd - sa);
-            float *lg = scr + buf * (C::SUB * GQ);
+            float *lg = lgb + buf * (C::SUB * GQ);
             buf ^= 1;
-            // log m of this thread's entries of the sub-chunk, used after the keys
             float lmv[C::EPT];
 #pragma unroll
             for (int i = 0; i < C::EPT; i++) {
                 const int64_t k = sa + tid + i * (kDecWarps * 32);
                 lmv[i] = (k < sbnd && k < npk) ? __ldg(a.log_m + a.off[s] + k) * kLog2e : 0.f;
             }
-            // ---- keys: base-2 logits q . k log2(e) / sqrt(d) into lg[row][head]
+            // ---- keys: base-2 logits into lg[row][head]
             for (int part = 0; part < 2; part++) {
                 const int64_t p0 = part ? (sa > npk ? sa : npk) : sa;
                 const int64_t p1 = part ? sbnd : (sbnd < npk ? sbnd : npk);
                 for (int64_t r0l = p0; r0l < p1; r0l += C::RPS, it++) {
-                    const int st = it % kDecStages;
-                    dec_wait(tc::smem_u32(&hd.full[st]), (it / kDecStages) & 1, hd, a.status);
+                    const int slot = it % kDecStages;
+                    dec_wait(tc::smem_u32(&hd.full[slot]), (it / kDecStages) & 1, hd, a.status);
                     const int nr = (int)(p1 - r0l < C::RPS ? p1 - r0l : C::RPS);
-                    const int r0 = (int)(r0l - sa);              // first row's place in the sub-chunk
-                    const unsigned char *stage = ring + st * kDecStageBytes;
-                    if constexpr (C::TC) {
-                        const uint32_t sbase = tc::smem_u32(stage);
-                        const int mi = lane >> 3, ri = lane & 7, hq = lane >> 2, tq = lane & 3;
+                    const int r0 = (int)(r0l - sa);
+                    const unsigned char *stage = ring + slot * kDecStageBytes;
 #pragma unroll
-                        for (int t = 0; t < C::TPS; t++) {
-                            if ((int)((it * C::TPS + t) % kDecWarps) != warp || t * 16 >= nr) continue;
-                            float c[4] = {0.f, 0.f, 0.f, 0.f};
-                            const int ar = t * 16 + ri + (mi & 1) * 8;   // row this lane addresses
+                    for (int k = 0; k < C::RPS / (kDecWarps * C::RPW); k++) {
+                        const int r = (k * kDecWarps + warp) * C::RPW + rg;
+                        if ((k * kDecWarps + warp) * C::RPW >= nr) break;
+                        float v[GQ];
 #pragma unroll
-                            for (int kk = 0; kk < D / 16; kk++) {
-                                uint32_t af[4];
-                                ldsm_x4(sbase + chunk_off<T, D, GQ>(ar, kk * 2 + (mi >> 1)), af);
-                                mma16816(c, af, qb[kk][0], qb[kk][1]);
-                            }
-                            // c[0], c[1]: row hq, heads 2 tq, 2 tq + 1; c[2], c[3]: row hq + 8
-                            const int h0 = 2 * tq;
-                            const int ra = t * 16 + hq, rb = ra + 8;
-                            if (h0 < GQ) {
-                                if (ra < nr) lg[(r0 + ra) * GQ + h0] = c[0] * a.qscale;
-                                if (rb < nr) lg[(r0 + rb) * GQ + h0] = c[2] * a.qscale;
-                            }
-                            if (h0 + 1 < GQ) {
-                                if (ra < nr) lg[(r0 + ra) * GQ + h0 + 1] = c[1] * a.qscale;
-                                if (rb < nr) lg[(r0 + rb) * GQ + h0 + 1] = c[3] * a.qscale;
+                        for (int h = 0; h < GQ; h++) v[h] = 0.f;
+#pragma unroll
+                        for (int c = 0; c < C::CPL; c++) {
+                            const uint4 u = *reinterpret_cast<const uint4 *>(stage + r * C::RB + (j + C::LPR * c) * 16);
+                            float f[C::EPC];
+                            chunk_to_float<T>(u, f);
+#pragma unroll
+                            for (int h = 0; h < GQ; h++) {
+                                float2 p2 = make_float2(0.f, 0.f);
+#pragma unroll
+                                for (int e = 0; e < C::EPC; e += 2)
+                                    p2 = __ffma2_rn(q2[h][(c * C::EPC + e) / 2], make_float2(f[e], f[e + 1]), p2);
+                                v[h] += p2.x + p2.y;
                             }
                         }
-                    } else {
+                        // butterfly over the lanes of the row: each step halves the
+                        // heads a lane keeps until every lane holds one full sum
 #pragma unroll
-                        for (int k = 0; k < C::RPS / (kDecWarps * C::RPW); k++) {
-                            const int r = (k * kDecWarps + warp) * C::RPW + rg;
-                            if ((k * kDecWarps + warp) * C::RPW >= nr) break;
-                            float v[GQ];
+                        for (int step = 0; (C::LPR >> (step + 1)) >= 1; step++) {
+                            const int o = C::LPR >> (step + 1);
+                            const int nv = (GQ >> step) > 1 ? (GQ >> step) : 1;
+                            if (nv > 1) {
+                                const bool up = (lane & o) != 0;
 #pragma unroll
-                            for (int h = 0; h < GQ; h++) v[h] = 0.f;
-#pragma unroll
-                            for (int c = 0; c < C::CPL; c++) {
-                                const uint4 u = *reinterpret_cast<const uint4 *>(stage + chunk_off<T, D, GQ>(r, j + C::LPR * c));
-                                float f[C::EPC];
-                                chunk_to_float<T>(u, f);
-#pragma unroll
-                                for (int h = 0; h < GQ; h++) {
-                                    float2 p2 = make_float2(0.f, 0.f);
-#pragma unroll
-                                    for (int e = 0; e < C::EPC; e += 2)
-                                        p2 = __ffma2_rn(q2[h][(c * C::EPC + e) / 2], make_float2(f[e], f[e + 1]), p2);
-                                    v[h] += p2.x + p2.y;
+                                for (int i = 0; i < nv / 2; i++) {
+                                    const float send = up ? v[i] : v[i + nv / 2];
+                                    const float keep = up ? v[i + nv / 2] : v[i];
+                                    v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
                                 }
+                            } else {
+                                v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
                             }
-                            // butterfly over the lanes of the row: each step halves the
-                            // heads a lane keeps until every lane holds one full sum
-#pragma unroll
-                            for (int step = 0; (C::LPR >> (step + 1)) >= 1; step++) {
-                                const int o = C::LPR >> (step + 1);
-                                const int nv = (GQ >> step) > 1 ? (GQ >> step) : 1;
-                                if (nv > 1) {
-                                    const bool up = (lane & o) != 0;
-#pragma unroll
-                                    for (int i = 0; i < nv / 2; i++) {
-                                        const float send = up ? v[i] : v[i + nv / 2];
-                                        const float keep = up ? v[i + nv / 2] : v[i];
-                                        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
-                                    }
-                                } else {
-                                    v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
-                                }
-                            }
-                            if (writer && r < nr) lg[(r0 + r) * GQ + hsel] = v[0];
                         }
+                        if (writer && r < nr) lg[(r0 + r) * GQ + hsel] = v[0];
                     }
                     __syncwarp();
-                    if (lane == 0) tc::mbar_arrive(tc::smem_u32(&hd.empty[st]));
+                    if (lane == 0) tc::mbar_arrive(tc::smem_u32(&hd.empty[slot]));
                 }
-            }
-            consumer_sync();
-            // ---- add log m, sub-chunk maximum per head
-            float x[C::EPT][GQ], mx[GQ];
-#pragma unroll
-            for (int h = 0; h < GQ; h++) mx[h] = -INFINITY;
-#pragma unroll
-            for (int i = 0; i < C::EPT; i++) {
-                const int e = tid + i * (kDecWarps * 32);
-#pragma unroll
-                for (int h = 0; h < GQ; h++) {
-                    x[i][h] = e < nsub ? lg[e * GQ + h] + lmv[i] : -INFINITY;
-                    mx[h] = fmaxf(mx[h], x[i][h]);
-                }
-            }
-#pragma unroll
-            for (int h = 0; h < GQ; h++) {
-#pragma unroll
-                for (int o = 16; o >= 1; o >>= 1) mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], o));
-                if (lane == 0) hd.wmax[warp][h] = mx[h];
             }
             consumer_sync();
             float alpha[GQ];
+            dec_subchunk_max<GQ, C::EPT>(hd, lg, lmv, nsub, mrun, alpha);
 #pragma unroll
-            for (int h = 0; h < GQ; h++) {
-                float m = hd.wmax[0][h];
-#pragma unroll
-                for (int w = 1; w < kDecWarps; w++) m = fmaxf(m, hd.wmax[w][h]);
-                const float mn = fmaxf(mrun[h], m);
-                alpha[h] = tc::ex2(mrun[h] - mn);          // 0 on the first sub-chunk
-                mrun[h] = mn;
-                lsum[h] *= alpha[h];
-            }
+            for (int h = 0; h < GQ; h++) lsum[h] *= alpha[h];
             // ---- weights p = 2^(x - M) in place of the logits
 #pragma unroll
             for (int i = 0; i < C::EPT; i++) {
@@ -485,7 +730,7 @@ __global__ void __launch_bounds__(kDecThreads, 2)
                 if (e < nsub) {
 #pragma unroll
                     for (int h = 0; h < GQ; h++) {
-                        const float p = tc::ex2(x[i][h] - mrun[h]);
+                        const float p = tc::ex2(lg[e * GQ + h] - mrun[h]);
                         lsum[h] += p;
                         lg[e * GQ + h] = p;
                     }
@@ -504,11 +749,11 @@ __global__ void __launch_bounds__(kDecThreads, 2)
                 const int64_t p0 = part ? (sa > npk ? sa : npk) : sa;
                 const int64_t p1 = part ? sbnd : (sbnd < npk ? sbnd : npk);
                 for (int64_t r0l = p0; r0l < p1; r0l += C::RPS, it++) {
-                    const int st = it % kDecStages;
-                    dec_wait(tc::smem_u32(&hd.full[st]), (it / kDecStages) & 1, hd, a.status);
+                    const int slot = it % kDecStages;
+                    dec_wait(tc::smem_u32(&hd.full[slot]), (it / kDecStages) & 1, hd, a.status);
                     const int nr = (int)(p1 - r0l < C::RPS ? p1 - r0l : C::RPS);
                     const int r0 = (int)(r0l - sa);
-                    const unsigned char *stage = ring + st * kDecStageBytes;
+                    const unsigned char *stage = ring + slot * kDecStageBytes;
 #pragma unroll
                     for (int k = 0; k < C::RPS / (kDecWarps * C::RPW); k++) {
                         const int r = (k * kDecWarps + warp) * C::RPW + rg;
@@ -519,7 +764,7 @@ __global__ void __launch_bounds__(kDecThreads, 2)
                             for (int h = 0; h < GQ; h++) p[h] = lg[(r0 + r) * GQ + h];
 #pragma unroll
                             for (int c = 0; c < C::CPL; c++) {
-                                const uint4 u = *reinterpret_cast<const uint4 *>(stage + chunk_off<T, D, GQ>(r, j + C::LPR * c));
+                                const uint4 u = *reinterpret_cast<const uint4 *>(stage + r * C::RB + (j + C::LPR * c) * 16);
                                 float f[C::EPC];
                                 chunk_to_float<T>(u, f);
 #pragma unroll
@@ -533,7 +778,7 @@ __global__ void __launch_bounds__(kDecThreads, 2)
                         }
                     }
                     __syncwarp();
-                    if (lane == 0) tc::mbar_arrive(tc::smem_u32(&hd.empty[st]));
+                    if (lane == 0) tc::mbar_arrive(tc::smem_u32(&hd.empty[slot]));
                 }
             }
         }
@@ -562,65 +807,24 @@ __global__ void __launch_bounds__(kDecThreads, 2)
                 for (int c = 0; c < C::CPL; c++)
 #pragma unroll
                     for (int e = 0; e < C::EPC; e += 2)
-                        *reinterpret_cast<float2 *>(scr + ((size_t)warp * GQ + h) * D + (j + C::LPR * c) * C::EPC + e) =
+                        *reinterpret_cast<float2 *>(red + ((size_t)warp * GQ + h) * D + (j + C::LPR * c) * C::EPC + e) =
                             acc[h][(c * C::EPC + e) / 2];
         }
         consumer_sync();
-        const int c_lo = chunk_of(vs, total, nc), c_hi = chunk_of(ve - 1, total, nc);
-        const int npieces = c_hi - c_lo + 1;
-        float *o_base = a.out + ((size_t)l_rel * a.Hq + (size_t)g * GQ) * D;
-        if (npieces == 1) {
-            for (int i = tid; i < GQ * D; i += kDecWarps * 32) {
-                const int h = i / D;
-                float sacc = 0.f, sl = 0.f;
+        for (int i = tid; i < GQ * D; i += kDecWarps * 32) {
+            float v = 0.f;
 #pragma unroll
-                for (int w = 0; w < kDecWarps; w++) {
-                    sacc += scr[(size_t)w * GQ * D + i];
-                    sl += hd.wsum[w][h];
-                }
-                o_base[i] = sacc / sl;
-            }
-        } else {
-            float *pp = a.part + (size_t)((s - a.s0) + (int)blockIdx.x) * C::PART;
-            for (int i = tid; i < GQ * D; i += kDecWarps * 32) {
-                float sacc = 0.f;
-#pragma unroll
-                for (int w = 0; w < kDecWarps; w++) sacc += scr[(size_t)w * GQ * D + i];
-                pp[i] = sacc;
-            }
-#pragma unroll
-            for (int h = 0; h < GQ; h++)
-                if (tid == h) {
-                    float sl = 0.f;
-#pragma unroll
-                    for (int w = 0; w < kDecWarps; w++) sl += hd.wsum[w][h];
-                    pp[GQ * D + h] = mrun[h];
-                    pp[GQ * D + GQ + h] = sl;
-                }
-            __threadfence();
-            consumer_sync();
-            if (tid == 0) hd.last = (atomicAdd(a.cnt + s, 1) == npieces - 1);
-            consumer_sync();
-            if (hd.last) {
-                __threadfence();
-                for (int i = tid; i < GQ * D; i += kDecWarps * 32) {
-                    const int h = i / D;
-                    float M = -INFINITY;
-                    for (int c = c_lo; c <= c_hi; c++)
-                        M = fmaxf(M, __ldcg(a.part + (size_t)((s - a.s0) + c) * C::PART + GQ * D + h));
-                    float num = 0.f, den = 0.f;
-                    for (int c = c_lo; c <= c_hi; c++) {
-                        const float *q = a.part + (size_t)((s - a.s0) + c) * C::PART;
-                        const float w = tc::ex2(__ldcg(q + GQ * D + h) - M);
-                        num += w * __ldcg(q + i);
-                        den += w * __ldcg(q + GQ * D + GQ + h);
-                    }
-                    o_base[i] = num / den;
-                }
-                if (tid == 0) a.cnt[s] = 0;
-            }
+            for (int w = 0; w < kDecWarps; w++) v += red[(size_t)w * GQ * D + i];
+            sums[i] = v;
         }
-        consumer_sync();                 // scr and the head words are reused by the next piece
+        if (tid < GQ) {
+            float v = 0.f;
+#pragma unroll
+            for (int w = 0; w < kDecWarps; w++) v += hd.wsum[w][tid];
+            hd.hsum[tid] = v;
+        }
+        consumer_sync();
+        dec_finish<D, GQ>(a, hd, sums, mrun, s, vs, ve, total, nc);
     }
 }
 
@@ -642,9 +846,9 @@ template <typename T, int D, int GQ>
 cudaError_t launch_decode(const DecArgs &a, const DecMaps &m, int dev, cudaStream_t s) {
     using C = DecCfg<T, D, GQ>;
     static std::atomic<int> grid_of[kDecMaxDevices];
-    const size_t smem = 1024 + (size_t)kDecStages * kDecStageBytes + (size_t)C::SCR * sizeof(float);
+    const size_t smem = C::SMEM;
     static_assert(sizeof(DecSmemHead) <= 1024, "decode shared-memory head");
-    auto kern = decode_attention_kernel<T, D, GQ>;
+    auto kern = C::TC ? decode_tc_kernel<D, GQ> : decode_cc_kernel<D, GQ>;
     if (dev < 0 || dev >= kDecMaxDevices) return cudaErrorInvalidDevice;
     int grid = grid_of[dev].load(std::memory_order_relaxed);
     if (grid == 0) {
