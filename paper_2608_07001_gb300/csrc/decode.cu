@@ -59,10 +59,16 @@ constexpr int kDecThreads = (kDecWarps + 1) * 32;    // + one producer warp
 constexpr int kDecStages = 8;                        // ring depth
 constexpr int kDecStageBytes = 8192;                 // bytes per ring stage
 constexpr int kDecMaxGrid = 1024;                    // partial slots beyond the heads
+constexpr int kDecMaxHeads = 1023;                   // (l, g) heads of one launch (offsets in shared memory)
 constexpr int kDecStatusTimeout = 1;
 constexpr int kDecStatusRange = 2;                   // offsets point past n_entries
 constexpr uint64_t kDecWaitNs = 2000000000ull;
 constexpr float kLog2e = 1.4426950408889634f;
+
+// Floats of one piece's partial: the weighted value sums [gq][d], then the
+// maxima [gq] and the weight sums [gq], padded so that every partial starts
+// on a 64-byte boundary (the merge reads the sums as float4).
+__host__ __device__ constexpr int dec_part_floats(int gq, int d) { return gq * d + 16; }
 
 struct DecArgs {
     const char *K, *V;          // packed rows [E][d]
@@ -90,9 +96,8 @@ struct DecCfg {
     static constexpr bool TC = sizeof(T) == 2;               // bf16: tensor cores, swizzled tiles
     static constexpr int RB = D * (int)sizeof(T);            // bytes per row
     static constexpr int RPS = kDecStageBytes / RB;          // rows per ring stage
-    static constexpr int SUB = TC ? 512 : 2048 / GQ;         // entries per sub-chunk
+    static constexpr int SUB = TC ? (GQ < 8 ? 512 : 256) : 2048 / GQ;   // entries per sub-chunk
     static constexpr int EPT = SUB / (kDecWarps * 32);       // sub-chunk entries per consumer thread
-    static constexpr int PART = GQ * (D + 2);                // floats per piece partial
     // tensor-core path
     static constexpr int NB = D / 64;                        // 64-column boxes per row
     static constexpr int TPS = RPS / 16;                     // 16-row steps per stage
@@ -112,8 +117,9 @@ struct DecCfg {
     static constexpr int FRF = TC ? FRW : 0;
     static constexpr int REDF = TC ? (WPM > 1 ? WPM * GQ * D : 0) : kDecWarps * GQ * D;
     static constexpr int SUMF = GQ * D;
+    static constexpr int VOFF = kDecMaxHeads + 1;            // the launch's offsets (int32, relative)
     static constexpr size_t SMEM =
-        1024 + (size_t)kDecStages * kDecStageBytes + (size_t)(LGF + FRF + REDF + SUMF) * sizeof(float);
+        1024 + (size_t)kDecStages * kDecStageBytes + (size_t)(LGF + FRF + REDF + SUMF + VOFF) * sizeof(float);
     static_assert(SUB % RPS == 0 && SUB % (kDecWarps * 32) == 0, "decode sub-chunk");
     static_assert(!TC || (RPS % 16 == 0 && kDecWarps % NMT == 0 && TPS % WPM == 0), "decode tensor tiles");
     static_assert(TC || (GQ <= LPR && LPR * RPW == 32 && RPS % (kDecWarps * RPW) == 0), "decode lanes");
@@ -188,11 +194,19 @@ __device__ __forceinline__ void consumer_sync() {
     asm volatile("bar.sync 1, %0;" ::"r"(kDecWarps * 32) : "memory");
 }
 
-// Virtual start of head s of the launch: its packed entries come first, then
-// its appended rows.
-__device__ __forceinline__ int64_t vstart(const DecArgs &a, int s) {
-    return (a.off[s] - a.off[a.s0]) + (int64_t)(s - a.s0) * a.n_app;
-}
+// The launch's heads as the CTA sees them: voff (shared memory) holds
+// off[s] - off[s0] for s in [s0, s0 + nS].
+struct DecView {
+    const int *voff;
+    int64_t base;               // off[s0]
+    int s0, n_app;
+    // virtual start of head s: its packed entries come first, then its appended rows
+    __device__ __forceinline__ int64_t vstart(int s) const {
+        return (int64_t)voff[s - s0] + (int64_t)(s - s0) * n_app;
+    }
+    __device__ __forceinline__ int64_t packed(int s) const { return voff[s + 1 - s0] - voff[s - s0]; }
+    __device__ __forceinline__ int64_t first_row(int s) const { return base + voff[s - s0]; }
+};
 // Chunk (CTA) holding virtual index i when `total` entries are cut into
 // `nc` chunks [floor(c total / nc), floor((c + 1) total / nc)).
 __device__ __forceinline__ int chunk_of(int64_t i, int64_t total, int64_t nc) {
@@ -200,21 +214,30 @@ __device__ __forceinline__ int chunk_of(int64_t i, int64_t total, int64_t nc) {
 }
 
 // The CTA's share of the launch: chunk [lo, hi) of the virtual sequence, the
-// first head it meets, the number of chunks.  Block 0 also writes the zero
-// outputs of heads without any entry.  Returns false when the CTA has no
-// work (or the offsets do not fit the cache).
+// first head it meets, the number of chunks.  Loads the launch's offsets into
+// shared memory first (one coalesced pass instead of a chain of dependent
+// loads); block 0 also writes the zero outputs of heads without any entry.
+// Returns false when the CTA has no work (or the offsets do not fit the cache).
 template <int D, int GQ>
-__device__ __forceinline__ bool dec_setup(const DecArgs &a, int64_t &lo, int64_t &hi, int64_t &total, int64_t &nc, int &s_first) {
+__device__ __forceinline__ bool dec_setup(const DecArgs &a, int *voff, DecView &v, int64_t &lo, int64_t &hi,
+                                          int64_t &total, int64_t &nc, int &s_first) {
     const int tid = threadIdx.x;
-    if (a.off[a.s0 + a.nS] > a.n_entries) {      // the offsets do not fit the cache
+    const int64_t base = a.off[a.s0];
+    for (int i = tid; i <= a.nS; i += kDecThreads) voff[i] = (int)(a.off[a.s0 + i] - base);
+    __syncthreads();
+    v.voff = voff;
+    v.base = base;
+    v.s0 = a.s0;
+    v.n_app = a.n_app;
+    if (base + voff[a.nS] > a.n_entries) {      // the offsets do not fit the cache
         if (blockIdx.x == 0 && tid == 0) atomicOr(a.status, kDecStatusRange);
         return false;
     }
-    total = vstart(a, a.s0 + a.nS);
+    total = v.vstart(a.s0 + a.nS);
     nc = total < (int64_t)gridDim.x ? total : (int64_t)gridDim.x;
-    if (blockIdx.x == 0)
+    if (blockIdx.x == 0 && a.n_app == 0)
         for (int s = a.s0 + tid; s < a.s0 + a.nS; s += kDecThreads)
-            if (a.off[s + 1] == a.off[s] && a.n_app == 0) {
+            if (v.packed(s) == 0) {
                 float *o = a.out + ((size_t)(s / a.G - a.s0 / a.G) * a.Hq + (size_t)(s % a.G) * GQ) * D;
                 for (int i = 0; i < GQ * D; i++) o[i] = 0.f;
             }
@@ -224,7 +247,7 @@ __device__ __forceinline__ bool dec_setup(const DecArgs &a, int64_t &lo, int64_t
     int sb = a.s0, se = a.s0 + a.nS;              // the last s with vstart(s) <= lo
     while (se - sb > 1) {
         const int mid = (sb + se) >> 1;
-        if (vstart(a, mid) <= lo) sb = mid; else se = mid;
+        if (v.vstart(mid) <= lo) sb = mid; else se = mid;
     }
     s_first = sb;
     return true;
@@ -246,17 +269,23 @@ __device__ __forceinline__ void dec_init_barriers(DecSmemHead &hd) {
 // consumers take them -- per sub-chunk the key stages, then the value stages;
 // within each, the packed rows and then the appended rows, RPS rows a stage.
 template <typename T, int D, int GQ>
-__device__ void dec_produce(const DecArgs &a, const DecMaps &maps, DecSmemHead &hd, unsigned char *ring,
-                            int64_t lo, int64_t hi, int s_first) {
+__device__ void dec_produce(const DecArgs &a, const DecMaps &maps, const DecView &v, DecSmemHead &hd,
+                            unsigned char *ring, int64_t lo, int64_t hi, int s_first) {
     using C = DecCfg<T, D, GQ>;
+    if constexpr (C::TC) {
+        tc::tma_prefetch_desc(&maps.K);
+        tc::tma_prefetch_desc(&maps.V);
+        tc::tma_prefetch_desc(&maps.Ka);
+        tc::tma_prefetch_desc(&maps.Va);
+    }
     uint32_t it = 0;
     bool ok = true;
     for (int s = s_first; ok && s < a.s0 + a.nS; s++) {
-        const int64_t vs = vstart(a, s), ve = vstart(a, s + 1);
+        const int64_t vs = v.vstart(s), ve = v.vstart(s + 1);
         if (vs >= hi) break;
         if (ve <= lo || ve == vs) continue;      // before the chunk, or no entry
         const int64_t pa = (lo > vs ? lo : vs) - vs, pb = (hi < ve ? hi : ve) - vs;
-        const int64_t npk = a.off[s + 1] - a.off[s];
+        const int64_t npk = v.packed(s);
         for (int64_t sa = pa; ok && sa < pb; sa += C::SUB) {
             const int64_t sbnd = sa + C::SUB < pb ? sa + C::SUB : pb;
             for (int kv = 0; ok && kv < 2; kv++)
@@ -271,7 +300,7 @@ __device__ void dec_produce(const DecArgs &a, const DecMaps &maps, DecSmemHead &
                             break;
                         }
                         const int64_t nr = p1 - r0 < C::RPS ? p1 - r0 : C::RPS;
-                        const int64_t row = part ? (int64_t)s * a.app_cap + (r0 - npk) : a.off[s] + r0;
+                        const int64_t row = part ? (int64_t)s * a.app_cap + (r0 - npk) : v.first_row(s) + r0;
                         const uint32_t fb = tc::smem_u32(&hd.full[st]);
                         const uint32_t dst = tc::smem_u32(ring + st * kDecStageBytes);
                         if constexpr (C::TC) {
@@ -298,20 +327,27 @@ __device__ void dec_produce(const DecArgs &a, const DecMaps &maps, DecSmemHead &
 // End of a piece: sums [GQ][D] (weighted value sums) and hd.hsum (sums of the
 // weights) in shared memory, mrun the running maxima (base 2).  Writes the
 // output when the piece is the whole head, else the piece's partial; the CTA
-// finishing the head's last piece merges all of them.
+// finishing the head's last piece merges all of them, in parallel over the
+// pieces and the outputs (scratch: at least 1024 floats of shared memory).
 template <int D, int GQ>
-__device__ __forceinline__ void dec_finish(const DecArgs &a, DecSmemHead &hd, const float *sums, const float (&mrun)[GQ], int s,
-                           int64_t vs, int64_t ve, int64_t total, int64_t nc) {
-    constexpr int PART = GQ * (D + 2);
-    const int tid = threadIdx.x;
+__device__ __forceinline__ void dec_finish(const DecArgs &a, DecSmemHead &hd, const float *sums,
+                                           const float (&mrun)[GQ], int s, int64_t vs, int64_t ve, int64_t total,
+                                           int64_t nc, float *scratch) {
+    constexpr int PART = dec_part_floats(GQ, D);
+    static_assert(PART % 16 == 0 && 2 * GQ <= 16, "decode partial layout");
+    constexpr int NT = kDecWarps * 32;
+    constexpr int NQ = GQ * D / 4;                   // float4 groups of one partial's sums
+    constexpr int NG = NT / NQ > 0 ? NT / NQ : 1;    // pieces taken at once
+    static_assert(NG * GQ * D <= 1024 && (NQ <= NT ? NT % NQ == 0 : NQ % NT == 0), "decode merge tiling");
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int l_rel = s / a.G - a.s0 / a.G, g = s % a.G;
     const int c_lo = chunk_of(vs, total, nc), c_hi = chunk_of(ve - 1, total, nc);
     float *o_base = a.out + ((size_t)l_rel * a.Hq + (size_t)g * GQ) * D;
     if (c_lo == c_hi) {
-        for (int i = tid; i < GQ * D; i += kDecWarps * 32) o_base[i] = sums[i] / hd.hsum[i / D];
+        for (int i = tid; i < GQ * D; i += NT) o_base[i] = sums[i] / hd.hsum[i / D];
     } else {
         float *pp = a.part + (size_t)((s - a.s0) + (int)blockIdx.x) * PART;
-        for (int i = tid; i < GQ * D; i += kDecWarps * 32) pp[i] = sums[i];
+        for (int i = tid; i < GQ * D; i += NT) pp[i] = sums[i];
 #pragma unroll
         for (int h = 0; h < GQ; h++)
             if (tid == h) {
@@ -324,24 +360,70 @@ __device__ __forceinline__ void dec_finish(const DecArgs &a, DecSmemHead &hd, co
         consumer_sync();
         if (hd.last) {
             __threadfence();
-            for (int i = tid; i < GQ * D; i += kDecWarps * 32) {
-                const int h = i / D;
-                float M = -INFINITY;
-                for (int c = c_lo; c <= c_hi; c++)
-                    M = fmaxf(M, __ldcg(a.part + (size_t)((s - a.s0) + c) * PART + GQ * D + h));
-                float num = 0.f, den = 0.f;
-                for (int c = c_lo; c <= c_hi; c++) {
-                    const float *q = a.part + (size_t)((s - a.s0) + c) * PART;
-                    const float w = tc::ex2(__ldcg(q + GQ * D + h) - M);
-                    num += w * __ldcg(q + i);
-                    den += w * __ldcg(q + GQ * D + GQ + h);
+            const int np = c_hi - c_lo + 1;
+            const float *p0 = a.part + (size_t)((s - a.s0) + c_lo) * PART;   // the head's pieces, consecutive
+            // overall maximum per head
+            float mx[GQ];
+#pragma unroll
+            for (int h = 0; h < GQ; h++) mx[h] = -INFINITY;
+            for (int p = tid; p < np; p += NT)
+#pragma unroll
+                for (int h = 0; h < GQ; h++) mx[h] = fmaxf(mx[h], __ldcg(p0 + (size_t)p * PART + GQ * D + h));
+#pragma unroll
+            for (int h = 0; h < GQ; h++) {
+#pragma unroll
+                for (int o = 16; o >= 1; o >>= 1) mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], o));
+                if (lane == 0) hd.wmax[warp][h] = mx[h];
+            }
+            consumer_sync();
+            float M[GQ], den[GQ];
+#pragma unroll
+            for (int h = 0; h < GQ; h++) {
+                M[h] = hd.wmax[0][h];
+#pragma unroll
+                for (int w = 1; w < kDecWarps; w++) M[h] = fmaxf(M[h], hd.wmax[w][h]);
+                den[h] = 0.f;
+            }
+            // weight sums: pieces spread over the threads
+            for (int p = tid; p < np; p += NT)
+#pragma unroll
+                for (int h = 0; h < GQ; h++) {
+                    const float *q = p0 + (size_t)p * PART + GQ * D;
+                    den[h] += tc::ex2(__ldcg(q + h) - M[h]) * __ldcg(q + GQ + h);
                 }
-                o_base[i] = num / den;
+            // value sums: thread = (group of NG pieces, float4 of the sums)
+            for (int qd = tid % NQ; qd < NQ; qd += NT) {
+                const int h = qd * 4 / D;
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+                for (int p = tid / NQ; p < np; p += NG) {
+                    const float *q = p0 + (size_t)p * PART;
+                    const float w = tc::ex2(__ldcg(q + GQ * D + h) - M[h]);
+                    const float4 x = __ldcg(reinterpret_cast<const float4 *>(q) + qd);
+                    acc.x += w * x.x; acc.y += w * x.y; acc.z += w * x.z; acc.w += w * x.w;
+                }
+                if (tid / NQ < NG) reinterpret_cast<float4 *>(scratch)[(tid / NQ) * NQ + qd] = acc;
+            }
+#pragma unroll
+            for (int h = 0; h < GQ; h++) {
+#pragma unroll
+                for (int o = 16; o >= 1; o >>= 1) den[h] += __shfl_xor_sync(0xffffffffu, den[h], o);
+                if (lane == 0) hd.wsum[warp][h] = den[h];
+            }
+            consumer_sync();
+            for (int i = tid; i < GQ * D; i += NT) {
+                const int h = i / D;
+                float num = 0.f, dd = 0.f;
+#pragma unroll
+                for (int k = 0; k < NG; k++) num += scratch[k * GQ * D + i];
+#pragma unroll
+                for (int w = 0; w < kDecWarps; w++) dd += hd.wsum[w][h];
+                o_base[i] = num / dd;
             }
             if (tid == 0) a.cnt[s] = 0;
         }
     }
-    consumer_sync();                 // the sums and the head words are reused by the next piece
+    consumer_sync();                 // the sums, the scratch and the head words are reused next
 }
 
 // Sub-chunk maximum of the base-2 logits (log m added into lg in place) and
@@ -395,14 +477,16 @@ __global__ void __launch_bounds__(kDecThreads, 2)
     uint32_t *fr = reinterpret_cast<uint32_t *>(lg + C::LGF);
     float *red = reinterpret_cast<float *>(fr + C::FRF);
     float *sums = red + C::REDF;
+    int *voff = reinterpret_cast<int *>(sums + C::SUMF);
 
     int64_t lo, hi, total, nc;
     int s_first;
-    if (!dec_setup<D, GQ>(a, lo, hi, total, nc, s_first)) return;
+    DecView v;
+    if (!dec_setup<D, GQ>(a, voff, v, lo, hi, total, nc, s_first)) return;
     dec_init_barriers(hd);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     if (warp == kDecWarps) {
-        if (lane == 0) dec_produce<__nv_bfloat16, D, GQ>(a, maps, hd, ring, lo, hi, s_first);
+        if (lane == 0) dec_produce<__nv_bfloat16, D, GQ>(a, maps, v, hd, ring, lo, hi, s_first);
         return;
     }
 
@@ -413,11 +497,11 @@ __global__ void __launch_bounds__(kDecThreads, 2)
     uint32_t it = 0;
 
     for (int s = s_first; s < a.s0 + a.nS; s++) {
-        const int64_t vs = vstart(a, s), ve = vstart(a, s + 1);
+        const int64_t vs = v.vstart(s), ve = v.vstart(s + 1);
         if (vs >= hi) break;
         if (ve <= lo || ve == vs) continue;
         const int64_t pa = (lo > vs ? lo : vs) - vs, pb = (hi < ve ? hi : ve) - vs;
-        const int64_t npk = a.off[s + 1] - a.off[s];
+        const int64_t npk = v.packed(s);
         const int l_rel = s / a.G - a.s0 / a.G, g = s % a.G;
 
         // the queries as the logit MMA's 16 x 8 column operand: column n = head
@@ -447,7 +531,7 @@ __global__ void __launch_bounds__(kDecThreads, 2)
 #pragma unroll
             for (int i = 0; i < C::EPT; i++) {
                 const int64_t k = sa + tid + i * (kDecWarps * 32);
-                lmv[i] = (k < sbnd && k < npk) ? __ldg(a.log_m + a.off[s] + k) * kLog2e : 0.f;
+                lmv[i] = (k < sbnd && k < npk) ? __ldg(a.log_m + v.first_row(s) + k) * kLog2e : 0.f;
             }
             // ---- keys: lg[row][head] = q . k log2(e) / sqrt(d)
             for (int st = 0; st < n_st; st++, it++) {
@@ -580,7 +664,7 @@ __global__ void __launch_bounds__(kDecThreads, 2)
             }
         }
         consumer_sync();
-        dec_finish<D, GQ>(a, hd, sums, mrun, s, vs, ve, total, nc);
+        dec_finish<D, GQ>(a, hd, sums, mrun, s, vs, ve, total, nc, reinterpret_cast<float *>(fr));
     }
 }
 
@@ -604,14 +688,16 @@ __global__ void __launch_bounds__(kDecThreads, 2)
     float *lgb = reinterpret_cast<float *>(ring + kDecStages * kDecStageBytes);
     float *red = lgb + C::LGF;
     float *sums = red + C::REDF;
+    int *voff = reinterpret_cast<int *>(sums + C::SUMF);
 
     int64_t lo, hi, total, nc;
     int s_first;
-    if (!dec_setup<D, GQ>(a, lo, hi, total, nc, s_first)) return;
+    DecView v;
+    if (!dec_setup<D, GQ>(a, voff, v, lo, hi, total, nc, s_first)) return;
     dec_init_barriers(hd);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     if (warp == kDecWarps) {
-        if (lane == 0) dec_produce<T, D, GQ>(a, maps, hd, ring, lo, hi, s_first);
+        if (lane == 0) dec_produce<T, D, GQ>(a, maps, v, hd, ring, lo, hi, s_first);
         return;
     }
 
@@ -622,11 +708,11 @@ __global__ void __launch_bounds__(kDecThreads, 2)
     int buf = 0;
 
     for (int s = s_first; s < a.s0 + a.nS; s++) {
-        const int64_t vs = vstart(a, s), ve = vstart(a, s + 1);
+        const int64_t vs = v.vstart(s), ve = v.vstart(s + 1);
         if (vs >= hi) break;
         if (ve <= lo || ve == vs) continue;
         const int64_t pa = (lo > vs ? lo : vs) - vs, pb = (hi < ve ? hi : ve) - vs;
-        const int64_t npk = a.off[s + 1] - a.off[s];
+        const int64_t npk = v.packed(s);
         const int l_rel = s / a.G - a.s0 / a.G, g = s % a.G;
 
         // this lane's elements of the GQ queries, pre-scaled to base 2
@@ -661,7 +747,7 @@ __global__ void __launch_bounds__(kDecThreads, 2)
 #pragma unroll
             for (int i = 0; i < C::EPT; i++) {
                 const int64_t k = sa + tid + i * (kDecWarps * 32);
-                lmv[i] = (k < sbnd && k < npk) ? __ldg(a.log_m + a.off[s] + k) * kLog2e : 0.f;
+                lmv[i] = (k < sbnd && k < npk) ? __ldg(a.log_m + v.first_row(s) + k) * kLog2e : 0.f;
             }
             // ---- keys: base-2 logits into lg[row][head]
             for (int part = 0; part < 2; part++) {
@@ -824,7 +910,7 @@ __global__ void __launch_bounds__(kDecThreads, 2)
             hd.hsum[tid] = v;
         }
         consumer_sync();
-        dec_finish<D, GQ>(a, hd, sums, mrun, s, vs, ve, total, nc);
+        dec_finish<D, GQ>(a, hd, sums, mrun, s, vs, ve, total, nc, lgb);
     }
 }
 
@@ -906,7 +992,7 @@ gkv_status check_cache(const gkv_decode_cache *c) {
 }
 
 size_t part_floats(const gkv_decode_cache *c) {
-    return (size_t)((int64_t)c->L * c->G + kDecMaxGrid) * (c->Hq / c->G) * (c->d + 2);
+    return (size_t)((int64_t)c->L * c->G + kDecMaxGrid) * dec_part_floats(c->Hq / c->G, c->d);
 }
 constexpr size_t kWsHeadBytes = 256;    // status word + padding
 size_t cnt_bytes(const gkv_decode_cache *c) { return (((size_t)c->L * c->G * sizeof(int)) + 255) / 256 * 256; }
@@ -970,10 +1056,11 @@ extern "C" gkv_status gracekv_decode_attention(const gkv_decode_cache *c, int32_
     a.nS = n_layers * c->G;
     a.qscale = (float)(1.4426950408889634 / sqrt((double)c->d));
     const int gq = c->Hq / c->G;
+    if (c->G > kDecMaxHeads) return GKV_EUNSUPPORTED;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     DecMaps m;
     memset(&m, 0, sizeof(m));
-    cudaError_t e;
+    cudaError_t e = cudaSuccess;
     if (c->dtype == GKV_BF16) {
         const int box_rows = kDecStageBytes / (c->d * 2);
         const int64_t app_rows = (int64_t)c->L * c->G * c->app_cap;
@@ -982,13 +1069,27 @@ extern "C" gkv_status gracekv_decode_attention(const gkv_decode_cache *c, int32_
             !dec_map(&m.Ka, ka, c->app_cap > 0 ? app_rows : 1, c->d, box_rows) ||
             !dec_map(&m.Va, va, c->app_cap > 0 ? app_rows : 1, c->d, box_rows))
             return GKV_ECUDA;
-        e = c->d == 128 ? launch_decode_gq<__nv_bfloat16, 128>(a, m, gq, dev, s)
-                        : launch_decode_gq<__nv_bfloat16, 64>(a, m, gq, dev, s);
-    } else {
-        e = c->d == 128 ? launch_decode_gq<float, 128>(a, m, gq, dev, s)
-                        : launch_decode_gq<float, 64>(a, m, gq, dev, s);
     }
-    return e == cudaSuccess ? GKV_OK : GKV_ECUDA;
+    // one launch covers at most kDecMaxHeads heads (its offsets sit in shared
+    // memory): longer layer ranges run as consecutive launches
+    const int lpl = kDecMaxHeads / c->G;
+    const size_t esz = c->dtype == GKV_BF16 ? 2 : 4;
+    for (int lb = 0; lb < n_layers; lb += lpl) {
+        const int nl = std::min(lpl, n_layers - lb);
+        DecArgs b = a;
+        b.s0 = (l0 + lb) * c->G;
+        b.nS = nl * c->G;
+        b.q = static_cast<const char *>(q) + (size_t)lb * c->Hq * c->d * esz;
+        b.out = out + (size_t)lb * c->Hq * c->d;
+        if (c->dtype == GKV_BF16)
+            e = c->d == 128 ? launch_decode_gq<__nv_bfloat16, 128>(b, m, gq, dev, s)
+                            : launch_decode_gq<__nv_bfloat16, 64>(b, m, gq, dev, s);
+        else
+            e = c->d == 128 ? launch_decode_gq<float, 128>(b, m, gq, dev, s)
+                            : launch_decode_gq<float, 64>(b, m, gq, dev, s);
+        if (e != cudaSuccess) return GKV_ECUDA;
+    }
+    return GKV_OK;
 }
 
 extern "C" gkv_status gracekv_decode_status(void *workspace, void *stream) {

@@ -174,6 +174,19 @@ def test_decode_layer_slices_and_repeats_are_identical():
     assert not torch.any(dec.workspace[256:256 + 4 * w.L * w.G])
 
 
+def test_decode_more_heads_than_one_launch_holds():
+    # 160 layers x 8 KV heads = 1280 heads: the call runs as consecutive
+    # launches over layer groups
+    w = synth.Workload("m", 160, 8, 16, 64, 320, 8, "bf16", "lognormal", 0, 1.0, 1e4, (8,), 41)
+    dc = synth.make_decode_cache(w, 8, n_app=1, app_cap=1)
+    c = _as_dict(dc, w.L, w.G)
+    out, dec = _run(c, w.Hq, app_cap=1)
+    _check(c, out)
+    part = dec.attention(c["q"][100:].cuda().contiguous(), l0=100)
+    torch.cuda.synchronize()
+    _check(c, part, 100, 60)
+
+
 def test_decode_append_through_the_api():
     # tokens appended with gracekv_decode_append join with log m = 0
     w = synth.Workload("a", 4, 2, 8, 128, 2048, 8, "bf16", "lognormal", 0, 1.0, 1e4, (8,), 31)
