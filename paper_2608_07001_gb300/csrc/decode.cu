@@ -60,6 +60,7 @@ constexpr int kDecStages = 8;                        // ring depth
 constexpr int kDecStageBytes = 8192;                 // bytes per ring stage
 constexpr int kDecMaxGrid = 1024;                    // partial slots beyond the heads
 constexpr int kDecMaxHeads = 1023;                   // (l, g) heads of one launch (offsets in shared memory)
+constexpr int kDecMinRows = 128;                     // rows a CTA takes at least (small launches)
 constexpr int kDecStatusTimeout = 1;
 constexpr int kDecStatusRange = 2;                   // offsets point past n_entries
 constexpr uint64_t kDecWaitNs = 2000000000ull;
@@ -928,8 +929,13 @@ constexpr int kDecMaxDevices = 64;
 
 // Grid of one launch: as many CTAs as fit on the device at once (set up once
 // per device and instantiation; the shared-memory opt-in is per device).
+// Grid of one launch: as many CTAs as fit on the device at once (set up once
+// per device and instantiation; the shared-memory opt-in is per device), fewer
+// when the launch holds fewer than kDecMinRows rows per CTA (estimated from
+// the average head length): small launches then split each head into fewer
+// pieces, which shortens the merge.
 template <typename T, int D, int GQ>
-cudaError_t launch_decode(const DecArgs &a, const DecMaps &m, int dev, cudaStream_t s) {
+cudaError_t launch_decode(const DecArgs &a, const DecMaps &m, int64_t rows_est, int dev, cudaStream_t s) {
     using C = DecCfg<T, D, GQ>;
     static std::atomic<int> grid_of[kDecMaxDevices];
     const size_t smem = C::SMEM;
@@ -948,17 +954,18 @@ cudaError_t launch_decode(const DecArgs &a, const DecMaps &m, int dev, cudaStrea
         grid = std::min(kDecMaxGrid, std::max(1, per_sm) * sms);
         grid_of[dev].store(grid, std::memory_order_relaxed);
     }
+    grid = (int)std::max<int64_t>(1, std::min<int64_t>(grid, (rows_est + kDecMinRows - 1) / kDecMinRows));
     kern<<<grid, kDecThreads, smem, s>>>(a, m);
     return cudaGetLastError();
 }
 
 template <typename T, int D>
-cudaError_t launch_decode_gq(const DecArgs &a, const DecMaps &m, int gq, int dev, cudaStream_t s) {
+cudaError_t launch_decode_gq(const DecArgs &a, const DecMaps &m, int gq, int64_t rows, int dev, cudaStream_t s) {
     switch (gq) {
-        case 1: return launch_decode<T, D, 1>(a, m, dev, s);
-        case 2: return launch_decode<T, D, 2>(a, m, dev, s);
-        case 4: return launch_decode<T, D, 4>(a, m, dev, s);
-        case 8: return launch_decode<T, D, 8>(a, m, dev, s);
+        case 1: return launch_decode<T, D, 1>(a, m, rows, dev, s);
+        case 2: return launch_decode<T, D, 2>(a, m, rows, dev, s);
+        case 4: return launch_decode<T, D, 4>(a, m, rows, dev, s);
+        case 8: return launch_decode<T, D, 8>(a, m, rows, dev, s);
         default: return cudaErrorInvalidValue;
     }
 }
@@ -1081,12 +1088,13 @@ extern "C" gkv_status gracekv_decode_attention(const gkv_decode_cache *c, int32_
         b.nS = nl * c->G;
         b.q = static_cast<const char *>(q) + (size_t)lb * c->Hq * c->d * esz;
         b.out = out + (size_t)lb * c->Hq * c->d;
+        const int64_t rows = c->n_entries * b.nS / ((int64_t)c->L * c->G) + (int64_t)b.nS * n_app;
         if (c->dtype == GKV_BF16)
-            e = c->d == 128 ? launch_decode_gq<__nv_bfloat16, 128>(b, m, gq, dev, s)
-                            : launch_decode_gq<__nv_bfloat16, 64>(b, m, gq, dev, s);
+            e = c->d == 128 ? launch_decode_gq<__nv_bfloat16, 128>(b, m, gq, rows, dev, s)
+                            : launch_decode_gq<__nv_bfloat16, 64>(b, m, gq, rows, dev, s);
         else
-            e = c->d == 128 ? launch_decode_gq<float, 128>(b, m, gq, dev, s)
-                            : launch_decode_gq<float, 64>(b, m, gq, dev, s);
+            e = c->d == 128 ? launch_decode_gq<float, 128>(b, m, gq, rows, dev, s)
+                            : launch_decode_gq<float, 64>(b, m, gq, rows, dev, s);
         if (e != cudaSuccess) return GKV_ECUDA;
     }
     return GKV_OK;
