@@ -240,7 +240,7 @@ def decode_leg(args, w, comp, L, G, Hq, d, dev):
             "us_per_token_all_layers": t_all * 1e3,
             "us_per_token_per_layer_graph": t_layers * 1e3,
             "tokens_per_s_per_layer_graph": 1e3 / t_layers,
-            "roofline": {"kernel": "decode_attention_kernel", "bound": "hbm", "achieved": ach,
+            "roofline": {"kernel": "decode_tc_kernel", "bound": "hbm", "achieved": ach,
                          "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": ach / pk["hbm_gbs"],
                          "peak_kind": pk_kind, "traffic": None}}
 
