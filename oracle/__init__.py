@@ -46,7 +46,7 @@ class Params(C.Structure):
         ("k_cand", C.c_int32),
         ("lambda_kappa", C.c_double), ("lambda_Z", C.c_double), ("lambda_M", C.c_double),
         ("eps", C.c_double), ("base_frac", C.c_double),
-        ("disp_mode", C.c_int32),
+        ("disp_mode", C.c_int32), ("seg_mode", C.c_int32), ("quota_alloc", C.c_int32),
     ]
 
 
@@ -84,7 +84,7 @@ PAPER_DEFAULTS = dict(
     recent=32, n_min=16, n_max=128, n0=64, lambda_stab=0.25, lambda_s=0.15,
     lambda_d=0.25, lambda_n=0.10, c_cut=1.0, windows=(4, 8, 16), k_cand=16,
     lambda_kappa=0.05, lambda_Z=0.25, lambda_M=0.75, eps=1e-6, base_frac=0.1,
-    seg_layers=(), disp_mode=0)
+    seg_layers=(), disp_mode=0, seg_mode=0, quota_alloc=0)
 
 
 def make_params(L, G, Hq, T, d, W, rope_base, ctx_start=0, ctx_end=None, **kw) -> Params:
@@ -110,6 +110,8 @@ def make_params(L, G, Hq, T, d, W, rope_base, ctx_start=0, ctx_end=None, **kw) -
     p.lambda_kappa, p.lambda_Z, p.lambda_M = o["lambda_kappa"], o["lambda_Z"], o["lambda_M"]
     p.eps, p.base_frac = o["eps"], o["base_frac"]
     p.disp_mode = o["disp_mode"]
+    p.seg_mode = o["seg_mode"]
+    p.quota_alloc = o["quota_alloc"]
     return p
 
 
@@ -142,6 +144,16 @@ def robust_z(a):
     rc = lib().orc_robust_z(_p(a, C.c_double), C.c_int32(a.size), _p(z, C.c_double))
     assert rc == 0
     return z
+
+
+def uniform_slots(p: Params):
+    """Slot starts of the "w/o CS" ablation (uniform slots of target n0)."""
+    N = p.ctx_end - p.recent - p.ctx_start
+    starts = np.zeros(N + 2, dtype=np.int32)
+    J = C.c_int32()
+    rc = lib().orc_uniform_slots(C.byref(p), _p(starts, C.c_int32), C.c_int32(N + 1), C.byref(J))
+    assert rc == 0, rc
+    return starts[:J.value + 1].copy()
 
 
 def segment(p: Params, V, hidden=None, surprisal=None):
@@ -338,7 +350,10 @@ def run(K, V, Q, B_total: int, rope_base: float, *, ctx_start=0, ctx_end=None, o
     r_eff, B_free = budget(p, B_total)
     p.recent = r_eff
     K64, V64, Q64 = _f64(K), _f64(V), _f64(Q)
-    if slot_starts is None:
+    if slot_starts is None and p.seg_mode == 1:
+        seg = dict(kappa=np.zeros(p.T), b=None, slot_starts=uniform_slots(p), dp_best=None,
+                   dp_second=None)
+    elif slot_starts is None:
         seg = segment(p, V64, hidden, surprisal)
     else:
         kap, _ = curvature(p, V64, hidden)

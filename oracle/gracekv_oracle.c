@@ -364,6 +364,22 @@ int orc_segment(const orc_params *p, const double *V, const double *hidden, int3
 /* to check the optimality of a partition locally at sizes where the full DP  */
 /* is too slow.                                                               */
 /* ------------------------------------------------------------------------ */
+/* "w/o CS" ablation, App. B.4 (last paragraph): the curvature-guided
+ * segmentation is replaced by uniform slots of target length n0 (64) over the
+ * compressible context [c_s, c_e - r) (reading R13). */
+int orc_uniform_slots(const orc_params *p, int32_t *slot_starts, int32_t cap, int32_t *n_slots)
+{
+    int cs = p->ctx_start;
+    int N = p->ctx_end - p->recent - cs;
+    if (N < 1 || p->n0 < 1) return ORC_EINVAL;
+    int J = (N + p->n0 / 2) / p->n0;
+    if (J < 1) J = 1;
+    *n_slots = J;
+    if (J > cap) return ORC_ECAP;
+    for (int j = 0; j <= J; j++) slot_starts[j] = cs + (int32_t)(((int64_t)j * N) / J);
+    return ORC_OK;
+}
+
 int orc_dp_weights(const orc_params *p, const double *V, const double *hidden, int32_t Dh,
                    const double *b, int32_t n, const int32_t *a_rel, const int32_t *i_rel,
                    double *w_out)
@@ -732,7 +748,7 @@ int orc_build_trees(const orc_params *p, const double *K, const double *V, const
                     for (int t = a; t <= b - 2; t++) { kv[t - a].v = kappa[t]; kv[t - a].t = t; }
                     qsort(kv, np, sizeof(kv_t), cmp_kv_desc);
                     int K_ = p->k_cand < np ? p->k_cand : np;
-                    if (np > K_) nd->m_topk[v] = rel_gap(kv[K_ - 1].v, kv[K_].v, 0.0);
+                    if (K_ > 0 && np > K_) nd->m_topk[v] = rel_gap(kv[K_ - 1].v, kv[K_].v, 0.0);
                     int nc = 0;
                     for (int k = 0; k < K_; k++) cand[nc++] = kv[k].t + 1;
                     int mid = a + n / 2;
@@ -891,12 +907,19 @@ int orc_allocate(const orc_params *p, int64_t B_free, int32_t n_slots,
         hitem it = {unit_Uadd[u], u, nd->a[r], nd->b[r], r, 1};
         hpush(h, &n, it);
     }
+    /* remaining capacity: one shared budget, or one per (l, g) (reading R14) */
+    int64_t LG = (int64_t)p->L * p->G, nq = p->quota_alloc ? LG : 1;
+    int64_t *Rq = (int64_t *)malloc(sizeof(int64_t) * (size_t)nq);
+    if (!Rq) { free(h); return ORC_ENOMEM; }
+    for (int64_t q = 0; q < nq; q++) Rq[q] = B_free / nq + (q < B_free % nq ? 1 : 0);
     int64_t R = B_free;
     while (R > 0 && n > 0) {
         hitem it = hpop(h, &n);
         int64_t v = it.node;
         int cost = it.is_add ? 1 : nd->cost[v];
-        if (cost > R) continue;                         /* discard */
+        int64_t q = p->quota_alloc ? it.unit / n_slots : 0;
+        if (cost > Rq[q]) continue;                     /* discard */
+        Rq[q] -= cost;
         R -= cost;
         int64_t first, cnt;
         if (it.is_add) {
@@ -913,7 +936,12 @@ int orc_allocate(const orc_params *p, int64_t B_free, int32_t n_slots,
             hpush(h, &n, c);
         }
     }
+    if (p->quota_alloc) {                               /* unused capacity is lost */
+        R = 0;
+        for (int64_t q = 0; q < nq; q++) R += Rq[q];
+    }
     *used = B_free - R;
+    free(Rq);
     free(h);
     return ORC_OK;
 }

@@ -53,6 +53,13 @@
  *       RoPE^-1(k, t) = RoPE(k, -t); base 0 means keys carry no rotation.
  *   R12 gains are clamped at 0; heap order (U desc, unit asc, a asc, b desc);
  *       an unaffordable pop is discarded for good.
+ *   R13 "w/o CS": J = max(1, round-half-up(N_c / n0)) slots, slot j starting at
+ *       c_s + floor(j N_c / J) (lengths differ by at most one); curvature is
+ *       taken as 0 everywhere; the split candidates and the curvature reward
+ *       are removed with k_cand = 0 and lambda_kappa = 0 (midpoint only).
+ *   R14 "w/o GA": (l, g) number lg gets the capacity floor(B_free / LG), plus
+ *       one for lg < B_free mod LG; the heap pops as before and discards an op
+ *       its (l, g) cannot afford; a pair's unused capacity is lost.
  *
  * Parity is pinned for every function here (see tests/test_oracle_*.py);
  * no function is "parity unpinned".
@@ -75,6 +82,10 @@ typedef struct {
     int32_t k_cand;
     double lambda_kappa, lambda_Z, lambda_M, eps, base_frac;
     int32_t disp_mode;            /* 0: definition, 1: paper's prefix form */
+    int32_t seg_mode;             /* 0: curvature DP; 1: uniform slots of target length n0
+                                     and curvature 0 (the "w/o CS" ablation, App. B.4 end) */
+    int32_t quota_alloc;          /* 0: one shared budget; 1: fixed per-(l, g) capacity
+                                     B_free / LG (the "w/o GA" ablation, App. C.1) */
 } orc_params;
 
 /* Per-node records of all trees (flat, capacity = L*G*2*N_c). */
@@ -95,6 +106,8 @@ int orc_segment(const orc_params *p, const double *V, const double *hidden, int3
                 const double *surprisal, double *kappa_out, double *b_out,
                 int32_t *slot_starts, int32_t cap, int32_t *n_slots,
                 double *dp_best, double *dp_second);
+
+int orc_uniform_slots(const orc_params *p, int32_t *slot_starts, int32_t cap, int32_t *n_slots);
 
 int orc_dp_weights(const orc_params *p, const double *V, const double *hidden, int32_t Dh,
                    const double *b, int32_t n, const int32_t *a_rel, const int32_t *i_rel,
