@@ -48,7 +48,7 @@
 extern "C" {
 #endif
 
-#define GRACEKV_ABI_VERSION 1
+#define GRACEKV_ABI_VERSION 2
 
 typedef enum {
     GKV_OK = 0,
@@ -88,10 +88,21 @@ typedef struct {
     int32_t n_seg_layers;          /*   for the relative-depth rule of App. B.2 */
     int32_t windows[4];            /* curvature window scales (App. B.2) */
     int32_t n_windows;
-    int32_t k_cand;                /* top-K curvature split candidates (App. B.4) */
+    int32_t k_cand;                /* top-K curvature split candidates (App. B.4); 0..16 */
     double lambda_kappa, lambda_Z, lambda_M, eps, base_frac;
     double lambda_graph;           /* multi-hop weight: only 0 is built (GKV_EUNSUPPORTED) */
     double alpha_floor;            /* singleton-floor cap: only 0 is built (GKV_EUNSUPPORTED) */
+    /* The paper's ablations (App. B.4 last paragraph, App. C.1); 0 = the method.
+     * seg_mode 1 ("w/o CS" with k_cand = 0 and lambda_kappa = 0): uniform slots
+     *   of target length n0 over the compressible context -- J = max(1,
+     *   round-half-up(N_c / n0)) slots, slot j starting at c_s + floor(j N_c / J)
+     *   -- and curvature 0 everywhere (k_cand = 0 leaves the midpoint as the
+     *   only binary cut, lambda_kappa = 0 drops the curvature reward).
+     * quota_alloc 1 ("w/o GA"): each (l, g) gets the fixed capacity
+     *   floor(B_free / LG) (+1 for the first B_free mod LG pairs) and cannot use
+     *   capacity another pair leaves; trees are then built completely. */
+    int32_t seg_mode;
+    int32_t quota_alloc;
 } gkv_params;
 
 /* Fill *p with the paper's defaults; shapes and budget are left zero.  Host only. */

@@ -17,6 +17,12 @@
 //      order (U desc, unit asc, a asc, b desc) takes it.
 // Ties in U are therefore resolved exactly as the heap resolves them.
 //
+// With fixed per-(l, g) capacities (the "w/o GA" ablation, App. C.1) the heap
+// decomposes into one independent heap per (l, g) with budget
+// floor(B_free / LG) (+1 for the first B_free mod LG pairs): every step above
+// then runs per (l, g) "segment", each with its own state words and histogram
+// (nseg = LG; nseg = 1 is the shared budget).
+//
 // The ops are the Add of every unit and the Split ops of the compact list the
 // unit kernel appends to as it evaluates nodes.
 // Kernels: alloc_hist (cost-weighted histogram of the 32-bit keys, three
@@ -51,7 +57,27 @@ struct AllocArgs {
     unsigned long long *hist, *st;
     int64_t B_free;
     int *status;
+    int nseg;                // 1: one shared budget; L G: a fixed capacity per (l, g)
 };
+
+// State words, histogram and budget of segment seg.  With one segment the
+// state sits at st[0 .. ST_N); with per-(l, g) capacities st[0 .. ST_N) holds
+// the totals and segment seg uses st[ST_N (1 + seg) ..].
+__device__ __forceinline__ unsigned long long *seg_st(const AllocArgs &A, int seg) {
+    return A.nseg > 1 ? A.st + ST_N * (1 + seg) : A.st;
+}
+__device__ __forceinline__ unsigned long long *seg_hist(const AllocArgs &A, int seg) {
+    return A.hist + (size_t)2048 * seg;
+}
+__device__ __forceinline__ long long seg_budget(const AllocArgs &A, int seg) {
+    if (A.nseg == 1) return A.B_free;
+    return A.B_free / A.nseg + (seg < A.B_free % A.nseg ? 1 : 0);
+}
+// Segment of op i (unit i for an Add, the unit of node v for a Split).
+__device__ __forceinline__ int op_seg(const AllocArgs &A, int64_t i, int64_t v) {
+    if (A.nseg == 1) return 0;
+    return (int)((v < 0 ? i : (int64_t)A.nd_unit[v]) / A.J);
+}
 
 // Op i of the enumeration: the Add of unit i (i < n_units), else Split op
 // i - n_units of the compact list; v receives the node index (-1 for an Add).
@@ -115,17 +141,54 @@ __global__ void alloc_hist_kernel(AllocArgs A, int shift, int nbits, uint32_t ma
     }
 }
 
+// The same histogram per segment (per-(l, g) capacities): global atomics,
+// combined per warp over equal (segment, bin) pairs.
+__global__ void alloc_hist_seg_kernel(AllocArgs A, int shift, int nbits, uint32_t mask) {
+    const int nbin = 1 << nbits;
+    const int lane = threadIdx.x & 31;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t w0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31);
+    const int64_t n = A.n_units + *A.n_ops;
+    for (int64_t i0 = w0; i0 < n; i0 += stride) {
+        const int64_t i = i0 + lane;
+        const bool in = i < n;
+        uint32_t key = 0;
+        int cost = 0;
+        int64_t v = -1;
+        int seg = 0;
+        if (in) {
+            op_key(A, i, key, cost, v);
+            seg = op_seg(A, i, v);
+        }
+        unsigned long long *st = seg_st(A, seg);
+        const uint32_t prefix = in ? (uint32_t)st[ST_PREFIX] : 0u;
+        const int bin = in && (key & mask) == prefix ? (int)((key >> shift) & (nbin - 1)) : -1;
+        const long long tag = bin >= 0 ? ((long long)seg << 11) | bin : -1;
+        const unsigned grp = __match_any_sync(0xffffffffu, tag);
+        const unsigned sum = __reduce_add_sync(grp, (unsigned)(bin >= 0 ? cost : 0));
+        if (bin >= 0 && lane == __ffs(grp) - 1) atomicAdd(seg_hist(A, seg) + bin, (unsigned long long)sum);
+        if (shift == 21) {   // first pass: total cost per segment
+            const int stag = in ? seg : -1;
+            const unsigned g2 = __match_any_sync(0xffffffffu, stag);
+            const unsigned tot = __reduce_add_sync(g2, (unsigned)(in ? cost : 0));
+            if (in && lane == __ffs(g2) - 1) atomicAdd(&st[ST_TOTAL], (unsigned long long)tot);
+        }
+    }
+}
+
 // Pick the digit of this pass: scanning bins from the top, the bin where the
-// cost of higher keys first exceeds B_free.  One block of 1024 threads; thread
-// t owns bins nbin-1-2t and nbin-2-2t.
+// cost of higher keys first exceeds the budget.  One block of 1024 threads
+// per segment; thread t owns bins nbin-1-2t and nbin-2-2t.
 __global__ void __launch_bounds__(1024) alloc_scan_kernel(AllocArgs A, int shift, int nbits) {
     __shared__ unsigned long long wsum[32];
     const int nbin = 1 << nbits;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const unsigned long long B = (unsigned long long)A.B_free;
-    const bool all = (shift == 21) ? (A.st[ST_TOTAL] <= B) : (A.st[ST_ALL] != 0);
+    const int seg = blockIdx.x;
+    unsigned long long *st = seg_st(A, seg), *hist = seg_hist(A, seg);
+    const unsigned long long B = (unsigned long long)seg_budget(A, seg);
+    const bool all = (shift == 21) ? (st[ST_TOTAL] <= B) : (st[ST_ALL] != 0);
     const int b0 = nbin - 1 - 2 * tid, b1 = b0 - 1;
-    unsigned long long h0 = b0 >= 0 ? A.hist[b0] : 0ull, h1 = b1 >= 0 ? A.hist[b1] : 0ull;
+    unsigned long long h0 = b0 >= 0 ? hist[b0] : 0ull, h1 = b1 >= 0 ? hist[b1] : 0ull;
     // exclusive scan of (h0 + h1) over threads, in descending bin order
     unsigned long long x = h0 + h1, incl = x;
 #pragma unroll
@@ -145,29 +208,27 @@ __global__ void __launch_bounds__(1024) alloc_scan_kernel(AllocArgs A, int shift
         wsum[lane] = iv - v;   // exclusive prefix of warp totals
     }
     __syncthreads();
-    const unsigned long long above = A.st[ST_ABOVE];
+    const unsigned long long above = st[ST_ABOVE];
     const unsigned long long before = above + wsum[warp] + (incl - x);
     __syncthreads();
     if (all) {
-        if (tid == 0 && shift == 21) A.st[ST_ALL] = 1;
+        if (tid == 0 && shift == 21) st[ST_ALL] = 1;
     } else {
         // the crossing bin is unique: above + cost(higher bins) <= B < ... + h
         if (b0 >= 0 && before <= B && before + h0 > B) {
-            A.st[ST_PREFIX] |= ((unsigned long long)b0 << shift);
-            A.st[ST_ABOVE] = before;
+            st[ST_PREFIX] |= ((unsigned long long)b0 << shift);
+            st[ST_ABOVE] = before;
         } else if (b1 >= 0 && before + h0 <= B && before + h0 + h1 > B) {
-            A.st[ST_PREFIX] |= ((unsigned long long)b1 << shift);
-            A.st[ST_ABOVE] = before + h0;
+            st[ST_PREFIX] |= ((unsigned long long)b1 << shift);
+            st[ST_ABOVE] = before + h0;
         }
     }
-    if (b0 >= 0) A.hist[b0] = 0;
-    if (b1 >= 0) A.hist[b1] = 0;
+    if (b0 >= 0) hist[b0] = 0;
+    if (b1 >= 0) hist[b1] = 0;
 }
 
 // Main set (kappa > tau, or everything when it fits) and units holding ties.
 __global__ void alloc_mark_kernel(AllocArgs A) {
-    const bool all = A.st[ST_ALL] != 0;
-    const uint32_t tau = (uint32_t)A.st[ST_PREFIX];
     const int64_t n = A.n_units + *A.n_ops;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
@@ -175,6 +236,9 @@ __global__ void alloc_mark_kernel(AllocArgs A) {
         int cost;
         int64_t v;
         op_key(A, i, key, cost, v);
+        const unsigned long long *st = seg_st(A, op_seg(A, i, v));
+        const bool all = st[ST_ALL] != 0;
+        const uint32_t tau = (uint32_t)st[ST_PREFIX];
         uint8_t s = (all || key > tau) ? 1 : 0;
         if (v < 0) {
             A.u_sel[i] = s;
@@ -192,28 +256,33 @@ __device__ __forceinline__ int64_t unit_base(const AllocArgs &A, int64_t uid) {
     return node_base(lg, A.slots[j], A.cs, A.Nc);
 }
 
-// One block: walk the units in ascending order; thread 0 replays every unit
-// that holds tie ops with the unit's own queue.
+// One block per segment: walk its units in ascending order; thread 0 replays
+// every unit that holds tie ops with the unit's own queue.
 __global__ void __launch_bounds__(1024) alloc_ties_kernel(AllocArgs A) {
     __shared__ int list[1024];
     __shared__ int nlist;
     __shared__ long long Rs;
     __shared__ short parent[2 * kMaxUnit];
+    const int seg = blockIdx.x;
+    unsigned long long *st = seg_st(A, seg);
+    const long long Bseg = seg_budget(A, seg);
+    const int64_t u_lo = A.nseg > 1 ? (int64_t)seg * A.J : 0;
+    const int64_t u_hi = A.nseg > 1 ? u_lo + A.J : A.n_units;
     if (threadIdx.x == 0) {
-        const bool all = A.st[ST_ALL] != 0;
-        long long above = (long long)A.st[ST_ABOVE];
-        Rs = all ? (long long)A.B_free - (long long)A.st[ST_TOTAL] : (long long)A.B_free - above;
+        const bool all = st[ST_ALL] != 0;
+        long long above = (long long)st[ST_ABOVE];
+        Rs = all ? Bseg - (long long)st[ST_TOTAL] : Bseg - above;
     }
     __syncthreads();
-    if (A.st[ST_ALL]) {
-        if (threadIdx.x == 0) A.st[ST_R] = 0, A.st[ST_USED] = A.st[ST_TOTAL];
+    if (st[ST_ALL]) {
+        if (threadIdx.x == 0) st[ST_R] = 0, st[ST_USED] = st[ST_TOTAL];
         return;
     }
-    const uint32_t tau = (uint32_t)A.st[ST_PREFIX];
-    for (int64_t base = 0; base < A.n_units && Rs > 0; base += 1024) {
+    const uint32_t tau = (uint32_t)st[ST_PREFIX];
+    for (int64_t base = u_lo; base < u_hi && Rs > 0; base += 1024) {
         // ordered compaction of flagged units in [base, base + 1024)
         int64_t uid = base + threadIdx.x;
-        bool f = uid < A.n_units && A.u_flag[uid];
+        bool f = uid < u_hi && A.u_flag[uid];
         if (threadIdx.x == 0) nlist = 0;
         __syncthreads();
         unsigned bal = __ballot_sync(0xffffffffu, f);
@@ -269,7 +338,7 @@ __global__ void __launch_bounds__(1024) alloc_ties_kernel(AllocArgs A) {
         }
         __syncthreads();
     }
-    if (threadIdx.x == 0) A.st[ST_R] = (unsigned long long)Rs;
+    if (threadIdx.x == 0) st[ST_R] = (unsigned long long)Rs;
 }
 
 // Endgame: when exactly one budget unit is left, the best exposed cost-1 op.
@@ -295,66 +364,77 @@ __device__ __forceinline__ bool end_cand(const AllocArgs &A, int64_t i, float &U
     return true;
 }
 
+// Segment of endgame candidate i (its unit's (l, g) with per-pair capacities).
+__device__ __forceinline__ int end_seg(const AllocArgs &A, int64_t i) {
+    if (A.nseg == 1) return 0;
+    return op_seg(A, i, i < A.n_units ? -1 : (int64_t)(A.ops[i - A.n_units].y >> 1));
+}
+
 __global__ void alloc_end_max_kernel(AllocArgs A) {
-    if (A.st[ST_R] != 1) return;
     const int64_t n = A.n_units + *A.n_ops;
-    unsigned best = 0;
-    bool any = false;
+    if (A.nseg == 1 && A.st[ST_R] != 1) return;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
+        unsigned long long *st = seg_st(A, end_seg(A, i));
+        if (st[ST_R] != 1) continue;
         float U;
         unsigned long long k;
         if (!end_cand(A, i, U, k)) continue;
-        unsigned b = __float_as_uint(U) + 1u;     // +1: distinguish "no candidate" (0)
-        if (!any || b > best) best = b;
-        any = true;
+        const unsigned b = __float_as_uint(U) + 1u;     // +1: distinguish "no candidate" (0)
+        if (b > (unsigned)st[ST_ENDU]) atomicMax(&st[ST_ENDU], (unsigned long long)b);
     }
-    if (any) atomicMax(reinterpret_cast<unsigned long long *>(&A.st[ST_ENDU]), (unsigned long long)best);
 }
 
 __global__ void alloc_end_key_kernel(AllocArgs A) {
-    if (A.st[ST_R] != 1 || A.st[ST_ENDU] == 0) return;
-    const unsigned target = (unsigned)A.st[ST_ENDU] - 1u;
     const int64_t n = A.n_units + *A.n_ops;
-    unsigned long long best = ~0ull;
+    if (A.nseg == 1 && (A.st[ST_R] != 1 || A.st[ST_ENDU] == 0)) return;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
+        unsigned long long *st = seg_st(A, end_seg(A, i));
+        if (st[ST_R] != 1 || st[ST_ENDU] == 0) continue;
         float U;
         unsigned long long k;
         if (!end_cand(A, i, U, k)) continue;
-        if (__float_as_uint(U) != target) continue;
-        if (k < best) best = k;
+        if (__float_as_uint(U) != (unsigned)st[ST_ENDU] - 1u) continue;
+        if (k < st[ST_ENDKEY]) atomicMin(&st[ST_ENDKEY], k);
     }
-    if (best != ~0ull) atomicMin(&A.st[ST_ENDKEY], best);
 }
 
 __global__ void alloc_end_pick_kernel(AllocArgs A) {
     const int64_t n = A.n_units + *A.n_ops;
-    const bool go = A.st[ST_R] == 1 && A.st[ST_ENDU] != 0;
+    if (A.nseg == 1 && (A.st[ST_R] != 1 || A.st[ST_ENDU] == 0)) return;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
-        if (!go) break;
+        const unsigned long long *st = seg_st(A, end_seg(A, i));
+        if (st[ST_R] != 1 || st[ST_ENDU] == 0) continue;
         float U;
         unsigned long long k;
         if (!end_cand(A, i, U, k)) continue;
-        if (k != A.st[ST_ENDKEY] || __float_as_uint(U) + 1u != (unsigned)A.st[ST_ENDU]) continue;
+        if (k != st[ST_ENDKEY] || __float_as_uint(U) + 1u != (unsigned)st[ST_ENDU]) continue;
         if (i < A.n_units) A.u_sel[i] = 1;
         else A.nd_sel[A.ops[i - A.n_units].y >> 1] = 1;
     }
 }
 
+// Budget left and used per segment; with per-pair capacities the totals add
+// up into st[ST_USED].
 __global__ void alloc_final_kernel(AllocArgs A) {
-    if (threadIdx.x) return;
-    long long R = (long long)A.st[ST_R];
-    if (!A.st[ST_ALL] && R == 1 && A.st[ST_ENDU] != 0) R = 0;
-    A.st[ST_R] = (unsigned long long)R;
-    if (!A.st[ST_ALL]) A.st[ST_USED] = (unsigned long long)(A.B_free - R);
+    for (int seg = blockIdx.x * blockDim.x + threadIdx.x; seg < A.nseg; seg += gridDim.x * blockDim.x) {
+        unsigned long long *st = seg_st(A, seg);
+        long long R = (long long)st[ST_R];
+        if (!st[ST_ALL] && R == 1 && st[ST_ENDU] != 0) R = 0;
+        st[ST_R] = (unsigned long long)R;
+        if (!st[ST_ALL]) st[ST_USED] = (unsigned long long)(seg_budget(A, seg) - R);
+        if (A.nseg > 1) atomicAdd(&A.st[ST_USED], st[ST_USED]);
+    }
 }
 
-__global__ void alloc_init_kernel(unsigned long long *st, unsigned long long *hist) {
-    int i = threadIdx.x;
-    if (i < ST_N) st[i] = (i == ST_ENDKEY) ? ~0ull : 0ull;
-    for (int b = i; b < 2048; b += blockDim.x) hist[b] = 0;
+__global__ void alloc_init_kernel(unsigned long long *st, unsigned long long *hist, int nseg) {
+    const int nst = ST_N * (nseg > 1 ? nseg + 1 : 1);
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < nst; i += gridDim.x * blockDim.x)
+        st[i] = (i % ST_N == ST_ENDKEY) ? ~0ull : 0ull;
+    for (int64_t b = blockIdx.x * blockDim.x + threadIdx.x; b < (int64_t)2048 * nseg; b += gridDim.x * blockDim.x)
+        hist[b] = 0;
 }
 
 
@@ -370,6 +450,7 @@ AllocArgs make_args(Ctx &c, int J) {
     A.J = J; A.LG = c.p.L * c.p.G; A.cs = c.p.ctx_start; A.Nc = c.Nc;
     A.u_sel = w.u_sel; A.nd_sel = w.nd_sel; A.u_flag = w.u_count;
     A.hist = w.hist; A.st = w.alloc_state; A.B_free = c.B_free; A.status = w.dev_int + 1;
+    A.nseg = c.p.quota_alloc ? c.p.L * c.p.G : 1;
     return A;
 }
 
@@ -463,14 +544,17 @@ __global__ void slot_classes_kernel(const int32_t *slots, int J, int32_t *list, 
 
 cudaError_t launch_threshold(Ctx &c, int J, cudaStream_t s) {
     AllocArgs A = make_args(c, J);
-    alloc_init_kernel<<<1, 256, 0, s>>>(c.w.alloc_state, c.w.hist);
+    alloc_init_kernel<<<A.nseg > 1 ? 256 : 1, 256, 0, s>>>(c.w.alloc_state, c.w.hist, A.nseg);
     const int blocks = grid_for(c, A.n_units + c.node_cap / 2);
     const int shifts[3] = {21, 10, 0};
     const int bits[3] = {11, 11, 10};
     uint32_t mask = 0;
     for (int ps = 0; ps < 3; ps++) {
-        alloc_hist_kernel<<<blocks, 256, 0, s>>>(A, shifts[ps], bits[ps], mask);
-        alloc_scan_kernel<<<1, 1024, 0, s>>>(A, shifts[ps], bits[ps]);
+        if (A.nseg > 1)
+            alloc_hist_seg_kernel<<<blocks, 256, 0, s>>>(A, shifts[ps], bits[ps], mask);
+        else
+            alloc_hist_kernel<<<blocks, 256, 0, s>>>(A, shifts[ps], bits[ps], mask);
+        alloc_scan_kernel<<<A.nseg, 1024, 0, s>>>(A, shifts[ps], bits[ps]);
         mask |= ((1u << bits[ps]) - 1u) << shifts[ps];
     }
     c.launches += 7;
@@ -518,11 +602,11 @@ cudaError_t launch_allocate(Ctx &c, int J, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     const int blocks = grid_for(c, A.n_units + c.node_cap / 2);
     alloc_mark_kernel<<<blocks, 256, 0, s>>>(A);
-    alloc_ties_kernel<<<1, 1024, 0, s>>>(A);
+    alloc_ties_kernel<<<A.nseg, 1024, 0, s>>>(A);
     alloc_end_max_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_end_key_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_end_pick_kernel<<<blocks, 256, 0, s>>>(A);
-    alloc_final_kernel<<<1, 32, 0, s>>>(A);
+    alloc_final_kernel<<<(A.nseg + 255) / 256, 256, 0, s>>>(A);
     c.launches += 6;
     return cudaGetLastError();
 }

@@ -154,7 +154,8 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
     if (p.n_seg_layers < 0 || p.n_seg_layers > gkv::kMaxSegLayers) return GKV_EINVAL;
     for (int i = 0; i < p.n_seg_layers; i++)
         if (p.seg_layers[i] < 0 || p.seg_layers[i] >= p.L) return GKV_EINVAL;
-    if (p.k_cand < 1 || p.k_cand > 16) return GKV_EINVAL;
+    if (p.k_cand < 0 || p.k_cand > 16) return GKV_EINVAL;
+    if ((p.seg_mode != 0 && p.seg_mode != 1) || (p.quota_alloc != 0 && p.quota_alloc != 1)) return GKV_EINVAL;
     if (!(p.eps > 0) || !(p.base_frac >= 0)) return GKV_EINVAL;
     if (p.lambda_graph != 0.0 || p.alpha_floor != 0.0) return GKV_EUNSUPPORTED;
     if ((p.d != 64 && p.d != 128) || p.W > 64 || p.n_max > gkv::kMaxUnit ||
@@ -237,7 +238,8 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
               dalloc(x, &w.nd_kappa, (size_t)c.node_cap) && dalloc(x, &w.nd_sel, (size_t)c.node_cap) &&
               dalloc(x, &w.ops, (size_t)c.node_cap / 2 + 1) && dalloc(x, &w.n_ops, 1) &&
               (!gkv::use_tc(c) || (dalloc(x, &w.Eg, (size_t)LG * Nc * 64) && dalloc(x, &w.qperm, (size_t)256))) &&
-              dalloc(x, &w.hist, 2048) && dalloc(x, &w.alloc_state, 16) && dalloc(x, &w.work, 4) &&
+              dalloc(x, &w.hist, (size_t)2048 * (p.quota_alloc ? LG : 1)) &&
+              dalloc(x, &w.alloc_state, (size_t)16 + (p.quota_alloc ? (size_t)8 * LG : 0)) && dalloc(x, &w.work, 4) &&
               dalloc(x, &w.pend_hist, 1 << 16) && dalloc(x, &w.pend_cut, 1) && dalloc(x, &w.pend_n, 1) &&
               dalloc(x, &w.pend_pot, 1);
     if (!ok) {
@@ -299,7 +301,21 @@ gkv_status gracekv_segment(gracekv_ctx *x, const void *V, const float *hidden, i
     cudaError_t e = cudaSuccess;
     if (c.score_pending && !c.dp_ev) e = cudaEventCreateWithFlags(&c.dp_ev, cudaEventDisableTiming);
     if (e == cudaSuccess) e = cudaMemsetAsync(c.w.dev_int, 0, 16 * sizeof(int), s);
-    if (e == cudaSuccess) {
+    if (c.p.seg_mode == 1) {
+        // "w/o CS" ablation: uniform slots of target length n0, curvature 0
+        const int N = c.Nc, J = std::max(1, (N + c.p.n0 / 2) / c.p.n0);
+        std::vector<int32_t> hs(J + 1);
+        for (int j = 0; j <= J; j++) hs[j] = c.p.ctx_start + (int32_t)(((int64_t)j * N) / J);
+        if (e == cudaSuccess) {
+            gkv::StageTimer tm(c, 0, s);
+            e = cudaMemcpyAsync(c.w.slots, hs.data(), (size_t)(J + 1) * sizeof(int32_t), cudaMemcpyHostToDevice, s);
+            if (e == cudaSuccess) e = cudaMemsetAsync(c.w.kappa, 0, (size_t)c.p.T * sizeof(double), s);
+            if (e == cudaSuccess && kappa) e = cudaMemsetAsync(kappa, 0, (size_t)c.p.T * sizeof(float), s);
+            if (e == cudaSuccess) e = cudaMemcpyAsync(c.w.dev_int, &J, sizeof(int), cudaMemcpyHostToDevice, s);
+            if (e == cudaSuccess) e = cudaStreamSynchronize(s);   // hs and J leave scope
+            if (e == cudaSuccess && c.dp_ev) e = cudaEventRecord(c.dp_ev, s);
+        }
+    } else if (e == cudaSuccess) {
         gkv::StageTimer tm(c, 0, s);
         e = gkv::launch_segment(c, V, hidden, hidden ? Dh : 0, surprisal, kappa, s);
     }
@@ -428,10 +444,13 @@ static cudaError_t build_fresh(Ctx &c, const void *K, const void *V, const void 
                                const int cnt[2], int lg0, int nlg, cudaStream_t s) {
     gkv::Workspace &w = c.w;
     const int64_t nu = (int64_t)c.p.L * c.p.G * c.J;
-    const bool root_only = c.B_free < nu;
+    // with per-(l, g) capacities ("w/o GA") the global threshold cannot prune:
+    // the trees are built completely in this launch
+    const bool full = c.p.quota_alloc != 0;
+    const bool root_only = !full && c.B_free < nu;
     gkv::StageTimer tm(c, 3, s);
-    return gkv::launch_unit_build(c, K, V, Q, omega, w.slots, c.J, 0, root_only ? 1 : 0, 1, 0.f, w.u_list, cnt[0],
-                                  w.u_list + (c.J - cnt[1]), cnt[1], s, lg0, nlg);
+    return gkv::launch_unit_build(c, K, V, Q, omega, w.slots, c.J, 0, root_only ? 1 : 0, full ? 4 * gkv::kMaxUnit : 1,
+                                  0.f, w.u_list, cnt[0], w.u_list + (c.J - cnt[1]), cnt[1], s, lg0, nlg);
 }
 
 // Trees (build.cu).  Every op's key is bounded before it is built: a pending
@@ -447,6 +466,7 @@ static cudaError_t build_fresh(Ctx &c, const void *K, const void *V, const void 
 // expansion of every unit that reaches tau, those trees are built to the end.
 static cudaError_t build_passes(Ctx &c, const void *K, const void *V, const void *Q, const float *omega,
                                 cudaStream_t s) {
+    if (c.p.quota_alloc) return cudaSuccess;     // complete trees: nothing is pending
     gkv::Workspace &w = c.w;
     const int J = c.J;
     const int64_t nu = (int64_t)c.p.L * c.p.G * J;

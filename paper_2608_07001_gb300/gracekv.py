@@ -37,6 +37,7 @@ class GkvParams(C.Structure):
         ("lambda_kappa", C.c_double), ("lambda_Z", C.c_double), ("lambda_M", C.c_double),
         ("eps", C.c_double), ("base_frac", C.c_double),
         ("lambda_graph", C.c_double), ("alpha_floor", C.c_double),
+        ("seg_mode", C.c_int32), ("quota_alloc", C.c_int32),
     ]
 
 

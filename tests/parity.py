@@ -75,16 +75,25 @@ def run_oracle(K, V, Q, B, rope_base, *, ctx_start=0, ctx_end=None, omega=None, 
                  hidden=hidden, surprisal=surprisal, slot_starts=slot_starts, **ov)
 
 
-def oracle_tau(o):
-    """Cost-weighted threshold of the oracle's bottleneck keys (fp64)."""
+def oracle_tau(o, lg=None):
+    """Cost-weighted threshold of the oracle's bottleneck keys (fp64); with
+    per-(l, g) capacities, the threshold of pair lg against its capacity."""
     tr = o["trees"]
     nd = tr.nodes
-    keys = np.concatenate([tr.unit_Uadd, nd["kappa"][nd["cost"] > 0]])
-    cost = np.concatenate([np.ones(len(tr.unit_Uadd)), nd["cost"][nd["cost"] > 0]])
+    ua = tr.unit_Uadd
+    nm = nd["cost"] > 0
+    B = o["B_free"]
+    if lg is not None:
+        p = o["params"]
+        LG, J = p.L * p.G, tr.n_slots
+        ua = ua[lg * J:(lg + 1) * J]
+        nm = nm & (nd["lg"] == lg)
+        B = B // LG + (1 if lg < B % LG else 0)
+    keys = np.concatenate([ua, nd["kappa"][nm]])
+    cost = np.concatenate([np.ones(len(ua)), nd["cost"][nm]])
     order = np.argsort(-keys, kind="stable")
     cum = np.cumsum(cost[order])
-    B = o["B_free"]
-    if cum[-1] <= B:
+    if len(cum) == 0 or cum[-1] <= B:
         return -np.inf
     k = np.searchsorted(cum, B, side="right")
     return keys[order][k]
@@ -129,9 +138,18 @@ def compare(g, o, dtype, report=None, require_exact_selection=True):
     assert len(uf) == nu + 1
     excluded = set()
     worst_D = worst_U = 0.0
-    tau = oracle_tau(o)
+    quota = bool(getattr(o["params"], "quota_alloc", 0))
+    tau_g = None if quota else oracle_tau(o)
+    taus = {}
     mism = exempt = pruned = pending = 0
     for u in range(nu):
+        if quota:
+            lgu = u // tr.n_slots
+            if lgu not in taus:
+                taus[lgu] = oracle_tau(o, lgu)
+            tau = taus[lgu]
+        else:
+            tau = tau_g
         gs, ge = uf[u], uf[u + 1]
         os_, oe = roots[u], roots[u + 1]
         okey = {(int(ond["a"][v]), int(ond["b"][v])): v for v in range(os_, oe)}

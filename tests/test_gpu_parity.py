@@ -59,6 +59,44 @@ def test_budget_sweep_bf16(x_ratio):
     print(f"x={x_ratio}", json.dumps(rep))
 
 
+@pytest.mark.parametrize("ablation", ["wo_cs", "wo_ga", "both"])
+def test_ablations_match_the_oracle(ablation):
+    # the paper's "w/o CS" (uniform slots of target 64, midpoint-only cuts, no
+    # curvature reward) and "w/o GA" (fixed per-(l, g) capacity; trees built
+    # completely) variants, on a 2-layer x 2-head bf16 slice and on PR1 fp32
+    kw = {}
+    if ablation in ("wo_cs", "both"):
+        kw.update(seg_mode=1, k_cand=0, lambda_kappa=0.0)
+    if ablation in ("wo_ga", "both"):
+        kw.update(quota_alloc=1)
+    w = synth.WORKLOADS["small"]
+    x = synth.make_inputs(w, layers=[0, 1], heads=[0, 1], T=1000)
+    L, G, T, d = x.K.shape
+    B = (L * G * T) // 8
+    P, g, o = _run(x.K, x.V, x.Q, B, w.rope_base, **kw)
+    rep = P.compare(g, o, torch.bfloat16)
+    print(ablation, json.dumps(rep))
+    if "seg_mode" in kw:
+        np.testing.assert_array_equal(g["slots"], o["seg"]["slot_starts"])
+    if "quota_alloc" in kw:
+        # every (l, g) stays within its capacity
+        LG, J = L * G, g["J"]
+        Bf = o["B_free"]
+        ex = g["export"]
+        first = ex["unit_first"]
+        for lg in range(LG):
+            q = Bf // LG + (1 if lg < Bf % LG else 0)
+            u0, u1 = lg * J, (lg + 1) * J
+            used = int((ex["add_sel"][u0:u1] == 1).sum())
+            sl = slice(int(first[u0]), int(first[u1]))
+            used += int(((ex["split_sel"][sl] == 1) * ex["cost"][sl]).sum())
+            assert used <= q, (lg, used, q)
+    wp = synth.WORKLOADS["pr1"]
+    xp = synth.make_inputs(wp)
+    P, g, o = _run(xp.K, xp.V, xp.Q, 256, wp.rope_base, **kw)
+    P.compare(g, o, torch.float32)
+
+
 def test_fullkv_identity_is_bit_exact():
     # x = 1: every tree expands to its leaves; the cache is the input (App. C.5)
     w = synth.WORKLOADS["pr1"]

@@ -4,8 +4,6 @@
 curvature split candidates and no curvature reward (midpoint only).
 "w/o GA": fixed per-(l, g) capacity instead of one shared budget.
 """
-import dataclasses
-
 import numpy as np
 import pytest
 
