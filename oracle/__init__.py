@@ -46,11 +46,14 @@ class Params(C.Structure):
         ("k_cand", C.c_int32),
         ("lambda_kappa", C.c_double), ("lambda_Z", C.c_double), ("lambda_M", C.c_double),
         ("eps", C.c_double), ("base_frac", C.c_double),
-        ("disp_mode", C.c_int32), ("seg_mode", C.c_int32), ("quota_alloc", C.c_int32),
+        ("disp_mode", C.c_int32),
+        ("alpha_floor", C.c_double), ("floor_c", C.c_double), ("floor_gamma", C.c_double),
+        ("floor_eta", C.c_double), ("floor_half", C.c_int32),
+        ("seg_mode", C.c_int32), ("quota_alloc", C.c_int32),
     ]
 
 
-_NODE_I32 = ["lg", "slot", "a", "b", "parent", "child0", "nchild", "form", "cost"]
+_NODE_I32 = ["lg", "slot", "a", "b", "parent", "child0", "nchild", "form", "cost", "floor_op"]
 _NODE_F64 = ["D", "Ddrop", "R", "U", "kappa", "kscale", "m_cut", "m_form", "m_topk", "m_ext"]
 
 
@@ -84,7 +87,8 @@ PAPER_DEFAULTS = dict(
     recent=32, n_min=16, n_max=128, n0=64, lambda_stab=0.25, lambda_s=0.15,
     lambda_d=0.25, lambda_n=0.10, c_cut=1.0, windows=(4, 8, 16), k_cand=16,
     lambda_kappa=0.05, lambda_Z=0.25, lambda_M=0.75, eps=1e-6, base_frac=0.1,
-    seg_layers=(), disp_mode=0, seg_mode=0, quota_alloc=0)
+    seg_layers=(), disp_mode=0, seg_mode=0, quota_alloc=0,
+    alpha_floor=0.0, floor_c=0.5, floor_gamma=1.2, floor_eta=0.95, floor_half=3)
 
 
 def make_params(L, G, Hq, T, d, W, rope_base, ctx_start=0, ctx_end=None, **kw) -> Params:
@@ -112,6 +116,8 @@ def make_params(L, G, Hq, T, d, W, rope_base, ctx_start=0, ctx_end=None, **kw) -
     p.disp_mode = o["disp_mode"]
     p.seg_mode = o["seg_mode"]
     p.quota_alloc = o["quota_alloc"]
+    p.alpha_floor, p.floor_c = o["alpha_floor"], o["floor_c"]
+    p.floor_gamma, p.floor_eta, p.floor_half = o["floor_gamma"], o["floor_eta"], o["floor_half"]
     return p
 
 
@@ -253,8 +259,35 @@ class Trees:
         return ns
 
 
-def build_trees(p: Params, K, V, Q, kappa, slot_starts, m, Z, rtok, omega=None) -> Trees:
+def floor(p: Params, rtok, slot_starts, B_base: int):
+    """Singleton floor (App. A.5 Stage I, App. C.2): scores f, accepted
+    positions [L*G, N_c] (uint8), B_floor, number of initial candidates."""
+    rtok = _f64(rtok)
+    LG, Nc = p.L * p.G, p.ctx_end - p.recent - p.ctx_start
+    ss = np.ascontiguousarray(np.asarray(slot_starts, dtype=np.int32))
+    f = np.zeros((LG, Nc))
+    acc = np.zeros((LG, Nc), dtype=np.uint8)
+    bf, nc = C.c_int64(), C.c_int64()
+    rc = lib().orc_floor(C.byref(p), _p(rtok, C.c_double), _p(ss, C.c_int32), C.c_int32(len(ss) - 1),
+                         C.c_int64(B_base), _p(f, C.c_double), _p(acc, C.c_uint8), C.byref(bf),
+                         C.byref(nc))
+    assert rc == 0, rc
+    return f, acc, bf.value, nc.value
+
+
+def unit_floor(p: Params, acc, slot_starts):
+    """1 for every slot (unit lg * J + j) holding an accepted floor position."""
+    ss = np.asarray(slot_starts) - p.ctx_start
+    J = len(ss) - 1
+    acc = np.asarray(acc).reshape(p.L * p.G, -1)
+    return np.stack([acc[:, ss[j]:ss[j + 1]].any(axis=1) for j in range(J)], axis=1).reshape(-1).astype(np.uint8)
+
+
+def build_trees(p: Params, K, V, Q, kappa, slot_starts, m, Z, rtok, omega=None,
+                floor_acc=None, floor_f=None) -> Trees:
     K, V, Q, kappa, m, Z, rtok, om = map(_f64, (K, V, Q, kappa, m, Z, rtok, omega))
+    fa = None if floor_acc is None else np.ascontiguousarray(floor_acc, dtype=np.uint8)
+    ff = None if floor_f is None else _f64(floor_f)
     ss = np.ascontiguousarray(np.asarray(slot_starts, dtype=np.int32))
     J = len(ss) - 1
     Nc = p.ctx_end - p.recent - p.ctx_start
@@ -273,20 +306,24 @@ def build_trees(p: Params, K, V, Q, kappa, slot_starts, m, Z, rtok, omega=None) 
                                _p(Q, C.c_double), None if om is None else _p(om, C.c_double),
                                _p(kappa, C.c_double), _p(ss, C.c_int32), C.c_int32(J),
                                _p(m, C.c_double), _p(Z, C.c_double), _p(rtok, C.c_double),
+                               None if fa is None else _p(fa, C.c_uint8),
+                               None if ff is None else _p(ff, C.c_double),
                                C.byref(ns), _p(uadd, C.c_double), _p(uroot, C.c_int64))
     assert rc == 0, rc
     n = ns.count
     return Trees({f: arr[f][:n].copy() for f in arr}, uadd, uroot, J)
 
 
-def allocate(p: Params, B_free: int, tr: Trees):
+def allocate(p: Params, B_free: int, tr: Trees, unit_fl=None):
     ns = tr.struct()
     nu = len(tr.unit_Uadd)
     add_sel = np.zeros(nu, dtype=np.uint8)
     split_sel = np.zeros(len(tr.nodes["a"]), dtype=np.uint8)
     used = C.c_int64()
+    uf = None if unit_fl is None else np.ascontiguousarray(unit_fl, dtype=np.uint8)
     rc = lib().orc_allocate(C.byref(p), C.c_int64(B_free), C.c_int32(tr.n_slots), C.byref(ns),
                             _p(tr.unit_Uadd, C.c_double), _p(tr.unit_root, C.c_int64),
+                            None if uf is None else _p(uf, C.c_uint8),
                             _p(add_sel, C.c_uint8), _p(split_sel, C.c_uint8), C.byref(used))
     assert rc == 0
     return add_sel, split_sel, used.value
@@ -361,9 +398,15 @@ def run(K, V, Q, B_total: int, rope_base: float, *, ctx_start=0, ctx_end=None, o
                    dp_best=None, dp_second=None)
     m, Z, ZC = row_stats(p, Q64, K64)
     rtok = token_values(p, Q64, K64, m, Z)
-    tr = build_trees(p, K64, V64, Q64, seg["kappa"], seg["slot_starts"], m, Z, rtok, omega)
-    add_sel, split_sel, used = allocate(p, B_free, tr)
+    fl = None
+    if p.alpha_floor > 0:
+        f, acc, B_floor, n_cand = floor(p, rtok, seg["slot_starts"], B_free)
+        fl = dict(f=f, accepted=acc, B_floor=B_floor, n_cand=n_cand,
+                  unit_floor=unit_floor(p, acc, seg["slot_starts"]))
+    tr = build_trees(p, K64, V64, Q64, seg["kappa"], seg["slot_starts"], m, Z, rtok, omega,
+                     None if fl is None else fl["accepted"], None if fl is None else fl["f"])
+    add_sel, split_sel, used = allocate(p, B_free, tr, None if fl is None else fl["unit_floor"])
     cap = B_total + L * G * (T - (p.ctx_end - p.ctx_start)) + 16
     cache = gather(p, K64, V64, rtok, tr, add_sel, split_sel, cap)
     return dict(params=p, r_eff=r_eff, B_free=B_free, seg=seg, m=m, Z=Z, ZC=ZC, rtok=rtok,
-                trees=tr, add_sel=add_sel, split_sel=split_sel, used=used, cache=cache)
+                trees=tr, add_sel=add_sel, split_sel=split_sel, used=used, cache=cache, floor=fl)

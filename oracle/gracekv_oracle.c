@@ -697,9 +697,124 @@ static int cmp_kv_desc(const void *x, const void *y)
     return (a->t > b->t) - (a->t < b->t);
 }
 
+/* ------------------------------------------------------------------------ */
+/* Stage I singleton floor, App. A.5 (Eqs. app_floor_score, app_floor_gate,   */
+/* app_floor_cap) and App. C.2 (candidates, path charging, the cap), in the   */
+/* reading R15 of the header.                                                  */
+/* ------------------------------------------------------------------------ */
+static int slot_of(const int32_t *slot_starts, int32_t n_slots, int t)
+{
+    int lo = 0, hi = n_slots;            /* the last j with slot_starts[j] <= t */
+    while (hi - lo > 1) {
+        int mid = (lo + hi) / 2;
+        if (slot_starts[mid] <= t) lo = mid; else hi = mid;
+    }
+    return lo;
+}
+
+int orc_floor(const orc_params *p, const double *rtok, const int32_t *slot_starts, int32_t n_slots,
+              int64_t B_base, double *f, uint8_t *accepted, int64_t *B_floor, int64_t *n_cand)
+{
+    int LG = p->L * p->G, c0 = p->ctx_start, Nc = p->ctx_end - p->recent - c0;
+    int h = p->floor_half;
+    memset(accepted, 0, (size_t)LG * Nc);
+    *B_floor = 0;
+    *n_cand = 0;
+    double *Rbar = (double *)calloc((size_t)Nc, sizeof(double));
+    double *mix = (double *)malloc(sizeof(double) * (size_t)Nc);
+    kv_t *ord = (kv_t *)malloc(sizeof(kv_t) * (size_t)Nc);
+    int32_t *cand = (int32_t *)malloc(sizeof(int32_t) * (size_t)LG * Nc);
+    int32_t *ncand = (int32_t *)calloc((size_t)LG, sizeof(int32_t));
+    uint8_t *inS = (uint8_t *)malloc((size_t)Nc);
+    uint8_t *covered = (uint8_t *)malloc((size_t)n_slots);
+    if (!Rbar || !mix || !ord || !cand || !ncand || !inS || !covered) {
+        free(Rbar); free(mix); free(ord); free(cand); free(ncand); free(inS); free(covered);
+        return ORC_ENOMEM;
+    }
+    /* consensus value and floor score (Eq. app_floor_score) */
+    for (int lg = 0; lg < LG; lg++)
+        for (int t = 0; t < Nc; t++) Rbar[t] += rtok[(size_t)lg * Nc + t];
+    for (int t = 0; t < Nc; t++) Rbar[t] /= LG;
+    for (int lg = 0; lg < LG; lg++) {
+        const double *R = rtok + (size_t)lg * Nc;
+        double *fl = f + (size_t)lg * Nc;
+        for (int t = 0; t < Nc; t++) mix[t] = (1.0 - p->floor_c) * R[t] + p->floor_c * Rbar[t];
+        for (int t = 0; t < Nc; t++) {
+            double mx = -INFINITY;
+            for (int u = t - h; u <= t + h; u++)
+                if (u >= 0 && u < Nc && mix[u] > mx) mx = mix[u];
+            fl[t] = mx;
+        }
+        /* candidates: f descending, the gate (Eq. app_floor_gate), the value mass eta */
+        for (int t = 0; t < Nc; t++) { ord[t].v = fl[t]; ord[t].t = t; }
+        qsort(ord, (size_t)Nc, sizeof(kv_t), cmp_kv_desc);
+        double cum = 0.0;
+        int n = 0;
+        for (int k = 0; k < Nc; k++) {
+            if (ord[k].v < p->floor_gamma / Nc) break;
+            if (cum + R[ord[k].t] > p->floor_eta) break;
+            cum += R[ord[k].t];
+            cand[(size_t)lg * Nc + n++] = ord[k].t;
+        }
+        ncand[lg] = n;
+        *n_cand += n;
+    }
+    /* joint cost of all candidates: per slot |S| + maximal runs outside S */
+    int64_t C0 = 0;
+    for (int lg = 0; lg < LG; lg++) {
+        if (!ncand[lg]) continue;
+        memset(inS, 0, (size_t)Nc);
+        for (int k = 0; k < ncand[lg]; k++) inS[cand[(size_t)lg * Nc + k]] = 1;
+        for (int j = 0; j < n_slots; j++) {
+            int a = slot_starts[j] - c0, b = slot_starts[j + 1] - c0, k = 0, runs = 0;
+            for (int t = a; t < b; t++) {
+                k += inS[t];
+                if (!inS[t] && (t == a || inS[t - 1])) runs++;
+            }
+            if (k) C0 += k + runs;
+        }
+    }
+    int64_t cap = (int64_t)floor(p->alpha_floor * (double)B_base);
+    int H = 0;
+    for (int lg = 0; lg < LG; lg++) {
+        if (ncand[lg] && C0 > cap) {
+            int64_t keep = (int64_t)floor((double)ncand[lg] * (double)cap / (double)C0);
+            ncand[lg] = (int32_t)(keep < 1 ? 1 : keep);
+        }
+        H += ncand[lg] > 0;
+    }
+    int64_t cap_h = H ? 2 * ((cap + H - 1) / H) : 0;
+    /* acceptance with path charging */
+    int64_t used = 0;
+    for (int lg = 0; lg < LG; lg++) {
+        if (!ncand[lg]) continue;
+        uint8_t *acc = accepted + (size_t)lg * Nc;
+        memset(covered, 0, (size_t)n_slots);
+        int64_t used_h = 0;
+        for (int k = 0; k < ncand[lg]; k++) {
+            int t = cand[(size_t)lg * Nc + k];
+            int j = slot_of(slot_starts, n_slots, t + c0);
+            int a = slot_starts[j] - c0, b = slot_starts[j + 1] - c0;
+            int lo = t, hi = t;                  /* frontier interval [lo, hi] holding t */
+            while (lo > a && !acc[lo - 1]) lo--;
+            while (hi < b - 1 && !acc[hi + 1]) hi++;
+            int64_t cost = (covered[j] ? 0 : 1) + (lo < t) + (t < hi);
+            if (used_h + cost > cap_h || used + cost > cap) continue;
+            acc[t] = 1;
+            covered[j] = 1;
+            used += cost;
+            used_h += cost;
+        }
+    }
+    *B_floor = used;
+    free(Rbar); free(mix); free(ord); free(cand); free(ncand); free(inS); free(covered);
+    return ORC_OK;
+}
+
 int orc_build_trees(const orc_params *p, const double *K, const double *V, const double *Q,
                     const double *omega, const double *kappa, const int32_t *slot_starts,
                     int32_t n_slots, const double *m, const double *Z, const double *rtok,
+                    const uint8_t *floor_acc, const double *floor_f,
                     orc_nodes *nd, double *unit_Uadd, int64_t *unit_root)
 {
     int L = p->L, G = p->G, d = p->d;
@@ -732,17 +847,36 @@ int orc_build_trees(const orc_params *p, const double *K, const double *V, const
                 if (dadd < 0.0) dadd = 0.0;
                 unit_Uadd[(size_t)lg * n_slots + j] = dadd;
                 double add_scale = fabs(om * Rr) * fmax(fabs(Ddr), fabs(Dr));
+                /* a slot holding an accepted floor position: its Add is a floor op,
+                   executed before the auction (it sets no bound on its children) */
+                int unit_fl = 0;
+                if (floor_acc)
+                    for (int t = sa; t < sb; t++) unit_fl |= floor_acc[(size_t)lg * Nc + (t - c0)];
                 /* breadth-first expansion of the unit's tree */
                 for (int64_t v = root; v < cnt; v++) {
                     int a = nd->a[v], b = nd->b[v], n = b - a;
                     nd->m_cut[v] = INFINITY; nd->m_form[v] = INFINITY;
                     nd->m_topk[v] = INFINITY; nd->m_ext[v] = INFINITY;
+                    nd->floor_op[v] = 0;
                     if (n == 1) {
                         nd->child0[v] = -1; nd->nchild[v] = 0; nd->form[v] = -1; nd->cost[v] = 0;
                         nd->U[v] = 0.0; nd->kappa[v] = 0.0; nd->kscale[v] = 0.0;
                         continue;
                     }
                     double DI = nd->D[v];
+                    /* forced extraction at the accepted floor position of largest f */
+                    int fp = -1;
+                    if (floor_acc) {
+                        double fb = -INFINITY;
+                        for (int t = a; t < b; t++) {
+                            size_t q = (size_t)lg * Nc + (t - c0);
+                            if (floor_acc[q] && floor_f[q] > fb) { fb = floor_f[q]; fp = t; }
+                        }
+                    }
+                    double best = -INFINITY, second = -INFINITY;
+                    int bxi = -1;
+                    double bDL = 0, bDR = 0;
+                    if (fp < 0) {
                     /* binary candidates: top-K positions in [a, b-2] by kappa, + midpoint */
                     int np = n - 1;
                     for (int t = a; t <= b - 2; t++) { kv[t - a].v = kappa[t]; kv[t - a].t = t; }
@@ -758,9 +892,6 @@ int orc_build_trees(const orc_params *p, const double *K, const double *V, const
                     /* kappa-hat: min-max of kappa over [a, b-2] */
                     double kmin = INFINITY, kmax = -INFINITY;
                     for (int t = a; t <= b - 2; t++) { kmin = fmin(kmin, kappa[t]); kmax = fmax(kmax, kappa[t]); }
-                    double best = -INFINITY, second = -INFINITY;
-                    int bxi = -1;
-                    double bDL = 0, bDR = 0;
                     /* candidates in ascending xi so that ties keep the smallest xi */
                     for (int x1 = 0; x1 < nc; x1++)
                         for (int x2 = x1 + 1; x2 < nc; x2++)
@@ -776,15 +907,20 @@ int orc_build_trees(const orc_params *p, const double *K, const double *V, const
                         else if (gb > second) second = gb;
                     }
                     if (nc > 1) nd->m_cut[v] = rel_gap(best, second, DI);
-                    /* salient-token extraction at argmax R_tok */
-                    int ps = a;
-                    double r1 = -INFINITY, r2 = -INFINITY;
-                    for (int t = a; t < b; t++) {
-                        double r = R[t - c0];
-                        if (r > r1) { r2 = r1; r1 = r; ps = t; }
-                        else if (r > r2) r2 = r;
                     }
-                    nd->m_ext[v] = rel_gap(r1, r2, 0.0);
+                    /* salient-token extraction at argmax R_tok (or the floor position) */
+                    int ps = a;
+                    if (fp >= 0) {
+                        ps = fp;
+                    } else {
+                        double r1 = -INFINITY, r2 = -INFINITY;
+                        for (int t = a; t < b; t++) {
+                            double r = R[t - c0];
+                            if (r > r1) { r2 = r1; r1 = r; ps = t; }
+                            else if (r > r2) r2 = r;
+                        }
+                        nd->m_ext[v] = rel_gap(r1, r2, 0.0);
+                    }
                     int ea[3], eb[3], ne = 0;
                     if (ps > a) { ea[ne] = a; eb[ne] = ps; ne++; }
                     ea[ne] = ps; eb[ne] = ps + 1; ne++;
@@ -797,8 +933,9 @@ int orc_build_trees(const orc_params *p, const double *K, const double *V, const
                     }
                     double rho_ext = gext / (ne - 1);
                     double rho_bin = best;
-                    nd->m_form[v] = rel_gap(rho_ext, rho_bin, DI);
-                    int use_ext = rho_ext > rho_bin;
+                    if (fp < 0) nd->m_form[v] = rel_gap(rho_ext, rho_bin, DI);
+                    int use_ext = fp >= 0 ? 1 : rho_ext > rho_bin;
+                    nd->floor_op[v] = fp >= 0;
                     int ca[3], cb[3], ncl;
                     double cD[3];
                     if (use_ext) {
@@ -830,9 +967,10 @@ int orc_build_trees(const orc_params *p, const double *K, const double *V, const
                     double own_scale = fabs(om * nd->R[v]) * fmax(fabs(DI), fabs(dsum)) / (ncl - 1);
                     /* bottleneck key: min over the path (creator = parent's split or Add) */
                     double ck, cs_;
-                    if (v == root) { ck = dadd; cs_ = add_scale; }
+                    if (v == root) { ck = unit_fl ? DBL_MAX : dadd; cs_ = add_scale; }
                     else { int64_t pv = root + nd->parent[v]; ck = nd->kappa[pv]; cs_ = nd->kscale[pv]; }
-                    if (nd->U[v] < ck) { nd->kappa[v] = nd->U[v]; nd->kscale[v] = own_scale; }
+                    if (fp >= 0) { nd->kappa[v] = DBL_MAX; nd->kscale[v] = 0.0; }   /* a floor op */
+                    else if (nd->U[v] < ck) { nd->kappa[v] = nd->U[v]; nd->kscale[v] = own_scale; }
                     else { nd->kappa[v] = ck; nd->kscale[v] = cs_; }
                 }
                 for (int64_t v = root; v < cnt; v++) {
@@ -894,7 +1032,7 @@ static hitem hpop(hitem *h, int64_t *n)
 
 int orc_allocate(const orc_params *p, int64_t B_free, int32_t n_slots,
                  const orc_nodes *nd, const double *unit_Uadd, const int64_t *unit_root,
-                 uint8_t *add_sel, uint8_t *split_sel, int64_t *used)
+                 const uint8_t *unit_floor, uint8_t *add_sel, uint8_t *split_sel, int64_t *used)
 {
     int64_t nu = (int64_t)p->L * p->G * n_slots;
     hitem *h = (hitem *)malloc(sizeof(hitem) * (size_t)(nu + nd->count + 1));
@@ -902,17 +1040,40 @@ int orc_allocate(const orc_params *p, int64_t B_free, int32_t n_slots,
     int64_t n = 0;
     memset(add_sel, 0, (size_t)nu);
     memset(split_sel, 0, (size_t)nd->count);
-    for (int64_t u = 0; u < nu; u++) {
-        int64_t r = unit_root[u];
-        hitem it = {unit_Uadd[u], u, nd->a[r], nd->b[r], r, 1};
-        hpush(h, &n, it);
-    }
     /* remaining capacity: one shared budget, or one per (l, g) (reading R14) */
     int64_t LG = (int64_t)p->L * p->G, nq = p->quota_alloc ? LG : 1;
     int64_t *Rq = (int64_t *)malloc(sizeof(int64_t) * (size_t)nq);
     if (!Rq) { free(h); return ORC_ENOMEM; }
     for (int64_t q = 0; q < nq; q++) Rq[q] = B_free / nq + (q < B_free % nq ? 1 : 0);
     int64_t R = B_free;
+    /* the singleton floor's ops execute first (App. A.5 Stage I, reading R15):
+       the Add of every floor slot and the forced extractions inside it */
+    if (unit_floor)
+        for (int64_t u = 0; u < nu; u++) {
+            if (!unit_floor[u]) continue;
+            int64_t r = unit_root[u], e = u + 1 < nu ? unit_root[u + 1] : nd->count;
+            int64_t q = p->quota_alloc ? u / n_slots : 0;
+            add_sel[u] = 1;
+            Rq[q] -= 1; R -= 1;
+            for (int64_t v = r; v < e; v++)
+                if (nd->floor_op[v]) { split_sel[v] = 1; Rq[q] -= nd->cost[v]; R -= nd->cost[v]; }
+        }
+    for (int64_t u = 0; u < nu; u++) {
+        int64_t r = unit_root[u];
+        if (!add_sel[u]) {
+            hitem it = {unit_Uadd[u], u, nd->a[r], nd->b[r], r, 1};
+            hpush(h, &n, it);
+            continue;
+        }
+        /* a floor slot: the Split of every frontier node the floor exposed */
+        int64_t e = u + 1 < nu ? unit_root[u + 1] : nd->count;
+        for (int64_t v = r; v < e; v++) {
+            if (split_sel[v] || nd->b[v] - nd->a[v] < 2) continue;
+            if (v != r && !split_sel[nd->parent[v]]) continue;
+            hitem c = {nd->U[v], u, nd->a[v], nd->b[v], v, 0};
+            hpush(h, &n, c);
+        }
+    }
     while (R > 0 && n > 0) {
         hitem it = hpop(h, &n);
         int64_t v = it.node;
@@ -938,7 +1099,7 @@ int orc_allocate(const orc_params *p, int64_t B_free, int32_t n_slots,
     }
     if (p->quota_alloc) {                               /* unused capacity is lost */
         R = 0;
-        for (int64_t q = 0; q < nq; q++) R += Rq[q];
+        for (int64_t q = 0; q < nq; q++) R += Rq[q] > 0 ? Rq[q] : 0;
     }
     *used = B_free - R;
     free(Rq);

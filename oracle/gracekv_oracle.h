@@ -60,6 +60,26 @@
  *   R14 "w/o GA": (l, g) number lg gets the capacity floor(B_free / LG), plus
  *       one for lg < B_free mod LG; the heap pops as before and discards an op
  *       its (l, g) cannot afford; a pair's unused capacity is lost.
+ *   R15 singleton floor (App. A.5 Stage I, App. C.2): R = the token values
+ *       (lambda_graph = 0); the consensus is the mean over all (l, g); the
+ *       max-pool window is clipped to the compressible context.  Candidates
+ *       of an (l, g): f descending (ties: lower t), while f >= gamma / N_c,
+ *       stopping before the running sum of R would exceed eta.  Joint cost
+ *       of a set S in a slot = the slot's frontier size after isolating S =
+ *       |S| + number of maximal runs of slot positions outside S.  When the
+ *       joint cost C0 of all candidates exceeds cap = floor(alpha B_base)
+ *       (B_base = the auction budget without a floor), every (l, g) with
+ *       n >= 1 candidates keeps its first max(1, floor(n cap / C0)).  Per-head
+ *       safeguard: an (l, g) may use at most 2 ceil(cap / H) entries, H = the
+ *       number of (l, g) with a candidate.  Acceptance in (l, g) order, then
+ *       candidate order: a candidate's incremental cost is 1 for its slot's
+ *       Add if the slot is still uncovered plus the new entries of extracting
+ *       it from its current frontier interval ([lo, t) and (t, hi] when
+ *       non-empty); it is accepted when both caps still hold, else skipped.
+ *       A node whose interval holds accepted positions is extracted at the one
+ *       with the largest f (ties: lower t); the floor ops (the Adds of slots
+ *       with an accepted position and these extractions) execute before the
+ *       auction, which gets B_base - B_floor.
  *
  * Parity is pinned for every function here (see tests/test_oracle_*.py);
  * no function is "parity unpinned".
@@ -82,6 +102,9 @@ typedef struct {
     int32_t k_cand;
     double lambda_kappa, lambda_Z, lambda_M, eps, base_frac;
     int32_t disp_mode;            /* 0: definition, 1: paper's prefix form */
+    double alpha_floor;           /* singleton-floor cap alpha (0: no floor, "w/o SF") */
+    double floor_c, floor_gamma, floor_eta;   /* consensus weight, gate, cumulative value */
+    int32_t floor_half;           /* max-pool half width (7 = 2 * 3 + 1) */
     int32_t seg_mode;             /* 0: curvature DP; 1: uniform slots of target length n0
                                      and curvature 0 (the "w/o CS" ablation, App. B.4 end) */
     int32_t quota_alloc;          /* 0: one shared budget; 1: fixed per-(l, g) capacity
@@ -93,6 +116,7 @@ typedef struct {
     int64_t cap;
     int64_t count;      /* out */
     int32_t *lg, *slot, *a, *b, *parent, *child0, *nchild, *form, *cost;
+    int32_t *floor_op;  /* 1: a forced extraction of the singleton floor */
     double *D, *Ddrop, *R, *U, *kappa, *kscale;
     double *m_cut, *m_form, *m_topk, *m_ext;
 } orc_nodes;
@@ -124,14 +148,25 @@ int orc_eval_interval(const orc_params *p, const double *K, const double *V,
                       double *D, double *Ddrop, double *ktil, double *vtil,
                       int32_t *pos, double *logm);
 
+/* Singleton floor (reading R15).  rtok [L G][N_c]; outputs f [L G][N_c],
+ * accepted [L G][N_c] (1 = an accepted floor position), *B_floor (its
+ * entries) and *n_cand (initial candidates before the cap). */
+int orc_floor(const orc_params *p, const double *rtok, const int32_t *slot_starts, int32_t n_slots,
+              int64_t B_base, double *f, uint8_t *accepted, int64_t *B_floor, int64_t *n_cand);
+
+/* floor_acc / floor_f (nullable): the accepted floor positions and their
+ * scores; nodes holding one are extracted there (floor_op = 1). */
 int orc_build_trees(const orc_params *p, const double *K, const double *V, const double *Q,
                     const double *omega, const double *kappa, const int32_t *slot_starts,
                     int32_t n_slots, const double *m, const double *Z, const double *rtok,
+                    const uint8_t *floor_acc, const double *floor_f,
                     orc_nodes *nodes, double *unit_Uadd, int64_t *unit_root);
 
+/* unit_floor (nullable): 1 for a slot whose Add is a floor op.  The floor ops
+ * execute first; *used counts them and the auction's entries. */
 int orc_allocate(const orc_params *p, int64_t B_free, int32_t n_slots,
                  const orc_nodes *nodes, const double *unit_Uadd, const int64_t *unit_root,
-                 uint8_t *add_sel, uint8_t *split_sel, int64_t *used);
+                 const uint8_t *unit_floor, uint8_t *add_sel, uint8_t *split_sel, int64_t *used);
 
 int orc_gather(const orc_params *p, const double *K, const double *V, const double *rtok,
                int32_t n_slots, const orc_nodes *nodes, const int64_t *unit_root,

@@ -15,7 +15,7 @@ import oracle as O
 
 
 def random_forest(rng, n_units, max_n, uvals=None, ext_p=0.35, lg_of_unit=None):
-    keys = ["lg", "slot", "a", "b", "parent", "child0", "nchild", "form", "cost"]
+    keys = ["lg", "slot", "a", "b", "parent", "child0", "nchild", "form", "cost", "floor_op"]
     fkeys = ["D", "Ddrop", "R", "U", "kappa", "kscale", "m_cut", "m_form", "m_topk", "m_ext"]
     nd = {k: [] for k in keys + fkeys}
     roots, uadd = [], []
@@ -27,7 +27,7 @@ def random_forest(rng, n_units, max_n, uvals=None, ext_p=0.35, lg_of_unit=None):
 
     def add(lg, j, a, b, parent):
         i = len(nd["a"])
-        for k, v in zip(keys, [lg, j, a, b, parent, -1, 0, -1, 0]):
+        for k, v in zip(keys, [lg, j, a, b, parent, -1, 0, -1, 0, 0]):
             nd[k].append(v)
         for k in fkeys:
             nd[k].append(0.0)
