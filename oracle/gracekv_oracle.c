@@ -775,19 +775,19 @@ int orc_floor(const orc_params *p, const double *rtok, const int32_t *slot_start
         }
     }
     int64_t cap = (int64_t)floor(p->alpha_floor * (double)B_base);
-    int H = 0;
+    int64_t nkept = 0;
     for (int lg = 0; lg < LG; lg++) {
         if (ncand[lg] && C0 > cap) {
-            int64_t keep = (int64_t)floor((double)ncand[lg] * (double)cap / (double)C0);
+            int64_t keep = (int64_t)ncand[lg] * cap / C0;        /* exact integer floor */
             ncand[lg] = (int32_t)(keep < 1 ? 1 : keep);
         }
-        H += ncand[lg] > 0;
+        nkept += ncand[lg];
     }
-    int64_t cap_h = H ? 2 * ((cap + H - 1) / H) : 0;
-    /* acceptance with path charging */
+    /* acceptance with path charging: the longest prefix within the head's share */
     int64_t used = 0;
     for (int lg = 0; lg < LG; lg++) {
         if (!ncand[lg]) continue;
+        int64_t cap_h = cap * ncand[lg] / nkept;               /* exact integer floor */
         uint8_t *acc = accepted + (size_t)lg * Nc;
         memset(covered, 0, (size_t)n_slots);
         int64_t used_h = 0;
@@ -799,7 +799,7 @@ int orc_floor(const orc_params *p, const double *rtok, const int32_t *slot_start
             while (lo > a && !acc[lo - 1]) lo--;
             while (hi < b - 1 && !acc[hi + 1]) hi++;
             int64_t cost = (covered[j] ? 0 : 1) + (lo < t) + (t < hi);
-            if (used_h + cost > cap_h || used + cost > cap) continue;
+            if (used_h + cost > cap_h) break;
             acc[t] = 1;
             covered[j] = 1;
             used += cost;

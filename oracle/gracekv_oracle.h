@@ -69,13 +69,15 @@
  *       |S| + number of maximal runs of slot positions outside S.  When the
  *       joint cost C0 of all candidates exceeds cap = floor(alpha B_base)
  *       (B_base = the auction budget without a floor), every (l, g) with
- *       n >= 1 candidates keeps its first max(1, floor(n cap / C0)).  Per-head
- *       safeguard: an (l, g) may use at most 2 ceil(cap / H) entries, H = the
- *       number of (l, g) with a candidate.  Acceptance in (l, g) order, then
- *       candidate order: a candidate's incremental cost is 1 for its slot's
- *       Add if the slot is still uncovered plus the new entries of extracting
- *       it from its current frontier interval ([lo, t) and (t, hi] when
- *       non-empty); it is accepted when both caps still hold, else skipped.
+ *       n >= 1 candidates keeps its first n' = max(1, floor(n cap / C0)).
+ *       Per-head safeguard: an (l, g) may use cap_h = floor(cap n' / sum n')
+ *       entries (its share of the cap by kept candidates; the shares sum to at
+ *       most cap, so the global cap holds).  An (l, g) accepts the longest
+ *       prefix of its kept candidates whose joint cost fits cap_h (the joint
+ *       cost never decreases along the prefix: a candidate adds 1 for its
+ *       slot's Add if the slot is still uncovered plus the new entries of
+ *       extracting it from its current frontier interval, [lo, t) and
+ *       (t, hi] when non-empty).
  *       A node whose interval holds accepted positions is extracted at the one
  *       with the largest f (ties: lower t); the floor ops (the Adds of slots
  *       with an accepted position and these extractions) execute before the
