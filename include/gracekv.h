@@ -48,7 +48,7 @@
 extern "C" {
 #endif
 
-#define GRACEKV_ABI_VERSION 2
+#define GRACEKV_ABI_VERSION 3
 
 typedef enum {
     GKV_OK = 0,
@@ -91,7 +91,8 @@ typedef struct {
     int32_t k_cand;                /* top-K curvature split candidates (App. B.4); 0..16 */
     double lambda_kappa, lambda_Z, lambda_M, eps, base_frac;
     double lambda_graph;           /* multi-hop weight: only 0 is built (GKV_EUNSUPPORTED) */
-    double alpha_floor;            /* singleton-floor cap: only 0 is built (GKV_EUNSUPPORTED) */
+    double alpha_floor;            /* singleton-floor cap alpha (App. A.5 Stage I, Eq. app_floor_cap);
+                                      0: no floor (the paper's "w/o SF"); the paper's value is 0.6 */
     /* The paper's ablations (App. B.4 last paragraph, App. C.1); 0 = the method.
      * seg_mode 1 ("w/o CS" with k_cand = 0 and lambda_kappa = 0): uniform slots
      *   of target length n0 over the compressible context -- J = max(1,
@@ -103,6 +104,19 @@ typedef struct {
      *   capacity another pair leaves; trees are then built completely. */
     int32_t seg_mode;
     int32_t quota_alloc;
+    /* Singleton floor (used when alpha_floor > 0; App. A.5 Stage I, App. C.2):
+     * consensus weight c (0.5), gate gamma (1.2, f >= gamma / N_c), value mass
+     * eta (0.95), max-pool half width (3: width 7).  Candidates of an (l, g):
+     * f descending (ties: lower t) up to the longest prefix whose token values
+     * sum to at most eta.  When their joint cost C0 (per slot: the frontier
+     * size after isolating them) exceeds cap = floor(alpha B_free), each (l, g)
+     * keeps its first max(1, floor(n cap / C0)); each then accepts the longest
+     * prefix of those whose joint cost fits floor(cap n' / sum n').  Accepted
+     * positions become singleton leaves by forced extraction, and the floor's
+     * Adds and extractions are executed before the auction.  Not combined with
+     * quota_alloc (GKV_EUNSUPPORTED). */
+    double floor_c, floor_gamma, floor_eta;
+    int32_t floor_half;
 } gkv_params;
 
 /* Fill *p with the paper's defaults; shapes and budget are left zero.  Host only. */
@@ -250,6 +264,15 @@ gkv_status gracekv_export(gracekv_ctx *ctx, int64_t node_cap, int64_t *n_nodes_h
                           int32_t *nchild, int32_t *cost, float *D, float *R, float *U,
                           float *kappa, uint8_t *split_sel, float *row_m, float *row_Z,
                           float *row_ZC, float *rtok, void *stream);
+
+/*
+ * The singleton floor of the last gracekv_build_trees (alpha_floor > 0), to
+ * caller-owned HOST arrays (synchronises `stream`): accepted [L G][N_c] uint8
+ * (1 = a floor singleton), f [L G][N_c] fp32 floor scores (nullable),
+ * *B_floor_host the entries the floor's ops take.  GKV_ESTATE without a floor.
+ */
+gkv_status gracekv_export_floor(gracekv_ctx *ctx, uint8_t *accepted, float *f, int64_t *B_floor_host,
+                                void *stream);
 
 /*
  * Measurement support (not needed to compress).  gracekv_profile(ctx, 1)

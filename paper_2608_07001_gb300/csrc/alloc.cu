@@ -32,6 +32,7 @@
 #include "gkv_internal.cuh"
 
 #include <algorithm>
+#include <cfloat>
 
 namespace gkv {
 namespace {
@@ -58,6 +59,7 @@ struct AllocArgs {
     int64_t B_free;
     int *status;
     int nseg;                // 1: one shared budget; L G: a fixed capacity per (l, g)
+    const uint8_t *u_floor;  // nullable: slots whose Add is a singleton-floor op (largest key)
 };
 
 // State words, histogram and budget of segment seg.  With one segment the
@@ -83,7 +85,7 @@ __device__ __forceinline__ int op_seg(const AllocArgs &A, int64_t i, int64_t v) 
 // i - n_units of the compact list; v receives the node index (-1 for an Add).
 __device__ __forceinline__ void op_key(const AllocArgs &A, int64_t i, uint32_t &key, int &cost, int64_t &v) {
     if (i < A.n_units) {
-        key = __float_as_uint(A.u_U[i]);
+        key = (A.u_floor && A.u_floor[i]) ? __float_as_uint(FLT_MAX) : __float_as_uint(A.u_U[i]);
         cost = 1;
         v = -1;
     } else {
@@ -118,7 +120,7 @@ __global__ void alloc_hist_kernel(AllocArgs A, int shift, int nbits, uint32_t ma
     for (int64_t i0 = w0; i0 < A.n_units; i0 += stride) {   // Add ops, cost 1
         const int64_t i = i0 + lane;
         const bool in = i < A.n_units;
-        const float x = in ? A.u_U[i] : 0.f;
+        const float x = in ? ((A.u_floor && A.u_floor[i]) ? FLT_MAX : A.u_U[i]) : 0.f;
         if (in && (!(x >= 0.f) || isinf(x))) atomicOr(A.status, 8);
         consume(in, __float_as_uint(x), 1);
     }
@@ -451,6 +453,7 @@ AllocArgs make_args(Ctx &c, int J) {
     A.u_sel = w.u_sel; A.nd_sel = w.nd_sel; A.u_flag = w.u_count;
     A.hist = w.hist; A.st = w.alloc_state; A.B_free = c.B_free; A.status = w.dev_int + 1;
     A.nseg = c.p.quota_alloc ? c.p.L * c.p.G : 1;
+    A.u_floor = c.p.alpha_floor > 0.0 ? w.u_floor : nullptr;
     return A;
 }
 

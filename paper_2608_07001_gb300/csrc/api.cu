@@ -95,6 +95,7 @@ gkv_status gracekv_default_params(gkv_params *p) {
     p->lambda_Z = 0.25; p->lambda_M = 0.75;
     p->eps = 1e-6; p->base_frac = 0.1;
     p->lambda_graph = 0.0; p->alpha_floor = 0.0;
+    p->floor_c = 0.5; p->floor_gamma = 1.2; p->floor_eta = 0.95; p->floor_half = 3;   // App. A.5 Stage I
     p->ctx_start = 0; p->ctx_end = -1;                 // -1: T
     return GKV_OK;
 }
@@ -157,7 +158,14 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
     if (p.k_cand < 0 || p.k_cand > 16) return GKV_EINVAL;
     if ((p.seg_mode != 0 && p.seg_mode != 1) || (p.quota_alloc != 0 && p.quota_alloc != 1)) return GKV_EINVAL;
     if (!(p.eps > 0) || !(p.base_frac >= 0)) return GKV_EINVAL;
-    if (p.lambda_graph != 0.0 || p.alpha_floor != 0.0) return GKV_EUNSUPPORTED;
+    if (p.lambda_graph != 0.0) return GKV_EUNSUPPORTED;
+    if (!(p.alpha_floor >= 0.0 && p.alpha_floor <= 1.0)) return GKV_EINVAL;
+    if (p.alpha_floor > 0.0) {
+        if (!(p.floor_c >= 0.0 && p.floor_c <= 1.0) || !(p.floor_gamma >= 0.0) ||
+            !(p.floor_eta >= 0.0 && p.floor_eta <= 1.0) || p.floor_half < 0 || p.floor_half > 64)
+            return GKV_EINVAL;
+        if (p.quota_alloc) return GKV_EUNSUPPORTED;
+    }
     if ((p.d != 64 && p.d != 128) || p.W > 64 || p.n_max > gkv::kMaxUnit ||
         (int64_t)p.G * p.d > 2048)
         return GKV_EUNSUPPORTED;
@@ -238,6 +246,10 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
               dalloc(x, &w.nd_kappa, (size_t)c.node_cap) && dalloc(x, &w.nd_sel, (size_t)c.node_cap) &&
               dalloc(x, &w.ops, (size_t)c.node_cap / 2 + 1) && dalloc(x, &w.n_ops, 1) &&
               (!gkv::use_tc(c) || (dalloc(x, &w.Eg, (size_t)LG * Nc * 64) && dalloc(x, &w.qperm, (size_t)256))) &&
+              (p.alpha_floor <= 0.0 || (dalloc(x, &w.fl_rbar, (size_t)Nc) && dalloc(x, &w.fl_f, (size_t)LG * Nc) &&
+                                          dalloc(x, &w.fl_acc, (size_t)LG * Nc) &&
+                                          dalloc(x, &w.fl_head, (size_t)LG * gkv::floor_head_words()) &&
+                                          dalloc(x, &w.fl_glob, (size_t)4))) &&
               dalloc(x, &w.hist, (size_t)2048 * (p.quota_alloc ? LG : 1)) &&
               dalloc(x, &w.alloc_state, (size_t)16 + (p.quota_alloc ? (size_t)8 * LG : 0)) && dalloc(x, &w.work, 4) &&
               dalloc(x, &w.pend_hist, 1 << 16) && dalloc(x, &w.pend_cut, 1) && dalloc(x, &w.pend_n, 1) &&
@@ -412,6 +424,7 @@ static gkv_status build_setup(gracekv_ctx *x, const int32_t *slot_starts, int32_
                   dalloc(x, &w.u_Ddrop, cap) && dalloc(x, &w.u_sel, cap) &&
                   dalloc(x, &w.u_count, cap) && dalloc(x, &w.u_off, cap) &&
                   dalloc(x, &w.u_pend, cap) && dalloc(x, &w.u_list, cap) &&
+                  (c.p.alpha_floor <= 0.0 || dalloc(x, &w.u_floor, cap)) &&
                   dalloc(x, &w.u_bsum, cap / 1024 + 2);
         if (!ok) return fail(x, GKV_ENOMEM, "build_trees: unit arrays");
         w.units_cap = cap;
@@ -548,6 +561,10 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
     }
     c.scored = false;
     int cnt[2];
+    if (e == cudaSuccess && c.p.alpha_floor > 0.0) {   // Stage I: needs every (l, g)'s token values
+        gkv::StageTimer tm(c, 3, s);
+        e = gkv::launch_floor(c, c.J, s);
+    }
     if (e == cudaSuccess) e = build_classes(c, cnt, s);
     if (e == cudaSuccess) e = build_fresh(c, K, V, Q, omega, cnt, 0, c.p.L * c.p.G, s);
     if (e == cudaSuccess) e = build_passes(c, K, V, Q, omega, s);
@@ -644,6 +661,7 @@ gkv_status gracekv_compress_host(gracekv_ctx *x, const void *K, const void *V, c
     if (e == cudaSuccess) e = build_classes(c, cnt, s);
     // per layer group, once it is in: score passes and the first tree-building launch
     const bool ranged = gkv::use_tc(c);
+    const bool fl = p.alpha_floor > 0.0;   // the floor needs every (l, g)'s token values first
     for (int gi = 0; e == cudaSuccess && gi < ngrp; gi++) {
         const int l0 = gi * p.L / ngrp, l1 = (gi + 1) * p.L / ngrp;
         e = cudaStreamWaitEvent(s, c.copy_ev[2 + gi], 0);
@@ -656,7 +674,14 @@ gkv_status gracekv_compress_host(gracekv_ctx *x, const void *K, const void *V, c
             gkv::StageTimer tm(c, 2, s);
             e = gkv::launch_token_values(c, c.hK, c.hQ, s, l0, l1);
         }
-        if (e == cudaSuccess) e = build_fresh(c, c.hK, c.hV, c.hQ, om, cnt, l0 * p.G, (l1 - l0) * p.G, s);
+        if (e == cudaSuccess && !fl) e = build_fresh(c, c.hK, c.hV, c.hQ, om, cnt, l0 * p.G, (l1 - l0) * p.G, s);
+    }
+    if (e == cudaSuccess && fl) {
+        if (ranged) {
+            gkv::StageTimer tm(c, 3, s);
+            e = gkv::launch_floor(c, c.J, s);
+            if (e == cudaSuccess) e = build_fresh(c, c.hK, c.hV, c.hQ, om, cnt, 0, LG, s);
+        }
     }
     if (e == cudaSuccess && !ranged) {   // other score paths: whole layers range at once
         {
@@ -666,6 +691,10 @@ gkv_status gracekv_compress_host(gracekv_ctx *x, const void *K, const void *V, c
         if (e == cudaSuccess) {
             gkv::StageTimer tm(c, 2, s);
             e = gkv::launch_token_values(c, c.hK, c.hQ, s);
+        }
+        if (e == cudaSuccess && fl) {
+            gkv::StageTimer tm(c, 3, s);
+            e = gkv::launch_floor(c, c.J, s);
         }
         if (e == cudaSuccess) e = build_fresh(c, c.hK, c.hV, c.hQ, om, cnt, 0, LG, s);
     }
@@ -718,6 +747,25 @@ gkv_status gracekv_allocate(gracekv_ctx *x, int64_t *n_entries_host, void *strea
     c.used = (int64_t)used;
     *n_entries_host = LG * (c.p.T - c.Nc) + c.used;
     c.stage = 3;
+    return GKV_OK;
+}
+
+gkv_status gracekv_export_floor(gracekv_ctx *x, uint8_t *accepted, float *f, int64_t *B_floor_host,
+                                void *stream) {
+    gkv_status st = ready(x, 2);
+    if (st) return st;
+    Ctx &c = x->c;
+    if (c.p.alpha_floor <= 0.0) return fail(x, GKV_ESTATE, "export_floor: no floor was built");
+    if (!accepted || !B_floor_host) return fail(x, GKV_EINVAL, "export_floor: null argument");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const size_t n = (size_t)c.p.L * c.p.G * c.Nc;
+    unsigned long long g[4] = {0, 0, 0, 0};
+    cudaError_t e = cudaMemcpyAsync(accepted, c.w.fl_acc, n, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess && f) e = cudaMemcpyAsync(f, c.w.fl_f, n * sizeof(float), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(g, c.w.fl_glob, sizeof g, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(x, e, "export_floor");
+    *B_floor_host = (int64_t)g[2];
     return GKV_OK;
 }
 

@@ -42,6 +42,8 @@
 // CTAs per SM; longer slots use the 128-token instance.
 #include "gkv_internal.cuh"
 
+#include <cfloat>
+
 #include <type_traits>
 
 namespace gkv {
@@ -63,6 +65,8 @@ struct BuildArgs {
     const double *kappa;
     const float *rtok, *row_m, *row_Z, *omega;
     const float *Eg;             // nullable: [L G][N_c][32][2] probe weights of every token (score pass B)
+    const uint8_t *fl_acc;       // nullable: [L G][N_c] accepted singleton-floor positions
+    const float *fl_f;           //           and their floor scores
     int L, G, Hq, T, d, W, gq, cs, Nc, J, k_cand;
     float inv_sqrt_d, lamZ, lamM, eps;
     float lam_kappa, base_frac;
@@ -102,6 +106,7 @@ struct BatchNode {
     int8_t pidx[kMaxCuts];   // candidate index of [a, xi) (-1: single token)
     int8_t sidx[kMaxCuts];   // candidate index of [xi, b) (-1: single token)
     int pstar, eL, eR, whole;
+    int forced;              // extraction at a singleton-floor position (a floor op)
     int pre_b, pre_e, suf_b, suf_e;   // prefixes (ascending end) in [0, NCD),
                                       // suffixes (descending start) in [NCD, 2 NCD)
     int pre_r, suf_r;                 // ends of the reserved ranges (unused entries empty)
@@ -242,6 +247,7 @@ struct Smem {
     float ktil[kNCD][DH];                    // prototypes of one direction at a time
     float vtil[kNCD][DH];
     float Rt[NMAX];
+    float Ff[NMAX];                          // floor score of an accepted floor position, -inf elsewhere
     float kn[NMAX];
     unsigned long long kap[NMAX];            // order-preserving keys of the curvature
     float redD[2 * kNCD][NWARPS];
@@ -464,6 +470,20 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             return;
         }
     }
+    // Singleton floor (App. A.5 Stage I): the accepted positions of this slot
+    // and their scores; a node holding one is extracted at the one of largest
+    // score, and the floor's ops carry the largest key (they execute first).
+    bool ufl = false;
+    if (A.fl_acc) {
+        bool any = false;
+        for (int t = tid; t < n; t += kNT) {
+            const size_t q = (size_t)lg * A.Nc + (sa - A.cs) + t;
+            const bool ac = A.fl_acc[q] != 0;
+            sm.Ff[t] = ac ? A.fl_f[q] : -INFINITY;
+            any |= ac;
+        }
+        ufl = __syncthreads_or(any);
+    }
     // ---- k_circ = RoPE^-1(k, t) ----------------------------------------------
     // batches of RB rotation-table loads are issued before any is used
     {
@@ -524,7 +544,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             nd.child0 = (short)A.nd_child0[v];
             nd.nchild = A.nd_nchild[v];
             nd.D = A.nd_D[v];
-            nd.kin = pg < 0 ? A.u_Uadd[uid] : A.nd_kappa[pg];
+            nd.kin = pg < 0 ? (ufl ? FLT_MAX : A.u_Uadd[uid]) : A.nd_kappa[pg];
             bnd_stage[k] = nd.nchild == -1 ? A.nd_U[v] : -1.f;   // key bound of a pending node
         }
         if (tid == 0) { sm.nnodes = nn; sm.nlvl[0] = 0; sm.pend = -1.f; }
@@ -809,6 +829,24 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     if (r2 > rb || (r2 == rb && p2 < pb)) { rb = r2; pb = p2; }
                 }
                 if (pb < a || pb >= b) pb = a;   // only reachable with non-finite values
+                // a node holding an accepted floor position is extracted at the one
+                // of largest floor score (ties: lower t)
+                int forced = 0;
+                if (ufl) {
+                    float fb = -INFINITY;
+                    int fpos = 0x7fffffff;
+                    for (int t = a + lane; t < b; t += 32) {
+                        const float fv = sm.Ff[t];
+                        if (fv > fb) { fb = fv; fpos = t; }
+                    }
+#pragma unroll
+                    for (int o = 16; o > 0; o >>= 1) {
+                        const float f2 = __shfl_xor_sync(0xffffffffu, fb, o);
+                        const int p2 = __shfl_xor_sync(0xffffffffu, fpos, o);
+                        if (f2 > fb || (f2 == fb && p2 < fpos)) { fb = f2; fpos = p2; }
+                    }
+                    if (fb > -INFINITY) { pb = fpos; forced = 1; }
+                }
                 // Candidate lists, lane-parallel (ranks from ballots): cuts xi in
                 // ascending order; prefixes [a, xi) (xi - a >= 2) and the
                 // extraction's left side [a, p*) in ascending end, then the whole
@@ -868,6 +906,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     B.kmin = kmn;
                     B.krange = kmx > kmn ? 1.0f / (float)(kmx - kmn) : 0.f;
                     B.pstar = pb;
+                    B.forced = forced;
                     B.ncut = ncut;
                     B.eL = el_sep ? eL_sep : (el_cand ? eL_cut : -1);
                     if (el_sep) sm.cand[eL_sep] = {a, pb, 0.f};
@@ -923,7 +962,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     nd.D = D;
                     float gain = om * sm.rootR * (Pd - D);
                     if (gain < 0.f) gain = 0.f;
-                    nd.kin = gain;
+                    nd.kin = ufl ? FLT_MAX : gain;   // a floor slot's Add is a floor op
                     A.u_Uadd[uid] = gain;
                     A.u_Ddrop[uid] = Pd;
                     A.nd_D[nbase] = D;
@@ -987,7 +1026,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     bR = B.sidx[0] >= 0 ? sm.candD[B.sidx[0]] : 0.f;
                 }
                 const float rho_ext = ne == 3 ? 0.5f * gext : gext;   // G_ext / (|children| - 1), exact
-                if (rho_ext > best) {
+                if (B.forced || rho_ext > best) {
                     B.nchild = ne;
                     for (int q = 0; q < ne; q++) { B.ca[q] = ea[q]; B.cb[q] = eb[q]; B.cD[q] = eD[q]; }
                 } else {
@@ -1010,7 +1049,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 const int nch = B.nchild;
                 if (nch < 0) {   // pending root: its split key is at most min(U_add, omega R D)
                     if (lane == 0) {
-                        const float bnd = fminf(nd.kin, key_bound(om * sm.rootR * nd.D));
+                        const float bnd = B.forced ? FLT_MAX : fminf(nd.kin, key_bound(om * sm.rootR * nd.D));
                         nd.nchild = -1; nd.child0 = -1;
                         A.nd_child0[gv] = -1; A.nd_nchild[gv] = -1; A.nd_cost[gv] = 0;
                         A.nd_U[gv] = bnd; A.nd_kappa[gv] = 0.f; A.nd_sel[gv] = 0;
@@ -1039,7 +1078,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 float gain = om * rnode * (nd.D - dsum);
                 if (gain < 0.f) gain = 0.f;
                 const float U = cost == 2 ? 0.5f * gain : gain;
-                const float kap = fminf(U, nd.kin);
+                const float kap = B.forced ? FLT_MAX : fminf(U, nd.kin);
                 if (lane == 0) {
                     nd.nchild = (signed char)nch;
                     nd.child0 = (short)child0;
@@ -1060,7 +1099,11 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     A.nd_D[gc] = B.cD[q]; A.nd_R[gc] = (float)rq;
                     A.nd_child0[gc] = -1; A.nd_nchild[gc] = 0; A.nd_cost[gc] = 0;
                     // until the child is evaluated, nd_U holds the bound of its split key
-                    A.nd_U[gc] = B.cb[q] - B.ca[q] >= 2 ? fminf(kap, key_bound(om * rq * B.cD[q])) : 0.f;
+                    // (the largest key when it holds a floor position: a floor op)
+                    bool chf = false;
+                    if (ufl)
+                        for (int t = B.ca[q]; t < B.cb[q] && !chf; t++) chf = sm.Ff[t] > -INFINITY;
+                    A.nd_U[gc] = B.cb[q] - B.ca[q] >= 2 ? (chf ? FLT_MAX : fminf(kap, key_bound(om * rq * B.cD[q]))) : 0.f;
                     A.nd_kappa[gc] = 0.f; A.nd_sel[gc] = 0;
                     if (B.cb[q] - B.ca[q] >= 2) {
                         const int pos = atomicAdd(&sm.nlvl[cur ^ 1], 1);
@@ -1138,7 +1181,9 @@ cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *
     A.K = K; A.V = V; A.Q = Q;
     A.slots = slots; A.rope = c.w.rope; A.kappa = c.w.kappa;
     A.rtok = c.w.rtok; A.row_m = c.w.row_m; A.row_Z = c.w.row_Z; A.omega = omega;
-    A.Eg = use_tc(c) ? c.w.Eg : nullptr;   // written by the tensor-core pass B
+    A.Eg = use_tc(c) ? c.w.Eg : nullptr;
+    A.fl_acc = c.p.alpha_floor > 0.0 ? c.w.fl_acc : nullptr;
+    A.fl_f = c.w.fl_f;   // written by the tensor-core pass B
     A.L = p.L; A.G = p.G; A.Hq = p.Hq; A.T = p.T; A.d = p.d; A.W = p.W; A.gq = p.Hq / p.G;
     A.cs = p.ctx_start; A.Nc = c.Nc; A.J = J; A.k_cand = p.k_cand;
     A.inv_sqrt_d = (float)(1.0 / sqrt((double)p.d));

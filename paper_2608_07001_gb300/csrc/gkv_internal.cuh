@@ -59,6 +59,13 @@ struct Workspace {
                                    // exactly the value their parent computed)
     float *nd_R = nullptr, *nd_U = nullptr, *nd_kappa = nullptr;
     uint8_t *nd_sel = nullptr;     // split selected (1), discarded tie (2)
+    // singleton floor (alpha_floor > 0)
+    float *fl_rbar = nullptr;      // [N_c] consensus token value
+    float *fl_f = nullptr;         // [L G][N_c] floor scores
+    uint8_t *fl_acc = nullptr;     // [L G][N_c] accepted floor positions
+    unsigned long long *fl_head = nullptr;   // [L G][8] per (l, g) selection state
+    unsigned long long *fl_glob = nullptr;   // [4] joint cost, kept candidates, floor entries
+    uint8_t *u_floor = nullptr;    // [units_cap] slots whose Add is a floor op
     uint2 *ops = nullptr;          // [node_cap / 2] Split ops built so far: (key bits, node << 1 | cost - 1)
     unsigned int *n_ops = nullptr; // [1] entries of ops
     // per-unit arrays (capacity units_cap), unit id = lg * J + j
@@ -292,6 +299,9 @@ cudaError_t launch_prune_list(Ctx &c, const int32_t *slots, int J, int32_t *list
 cudaError_t launch_pend_cut(Ctx &c, int J, int m, float *cut, unsigned int *n_qual, cudaStream_t s);
 
 cudaError_t launch_allocate(Ctx &c, int J, cudaStream_t s);
+// singleton floor (floor.cu): candidates, cap and accepted positions of every (l, g)
+cudaError_t launch_floor(Ctx &c, int J, cudaStream_t s);
+int floor_head_words();
 cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *slots, int J,
                           void *K_out, void *V_out, int32_t *pos, float *log_m,
                           int32_t *src_lo, int32_t *src_hi, int64_t *offsets, cudaStream_t s);

@@ -38,6 +38,8 @@ class GkvParams(C.Structure):
         ("eps", C.c_double), ("base_frac", C.c_double),
         ("lambda_graph", C.c_double), ("alpha_floor", C.c_double),
         ("seg_mode", C.c_int32), ("quota_alloc", C.c_int32),
+        ("floor_c", C.c_double), ("floor_gamma", C.c_double), ("floor_eta", C.c_double),
+        ("floor_half", C.c_int32),
     ]
 
 
@@ -62,7 +64,7 @@ EXPORTED = ["gracekv_default_params", "gracekv_budget_for_ratio", "gracekv_creat
             "gracekv_destroy", "gracekv_last_error", "gracekv_status_string", "gracekv_query",
             "gracekv_segment", "gracekv_score", "gracekv_build_trees", "gracekv_allocate", "gracekv_gather",
             "gracekv_export", "gracekv_profile", "gracekv_stats", "gracekv_row_stats_noalloc",
-            "gracekv_compress_host", "gracekv_decode_workspace_size", "gracekv_decode_append",
+            "gracekv_compress_host", "gracekv_export_floor", "gracekv_decode_workspace_size", "gracekv_decode_append",
             "gracekv_decode_attention", "gracekv_decode_status"]
 
 
@@ -93,6 +95,7 @@ def lib() -> C.CDLL:
     L.gracekv_allocate.argtypes = [vp, C.POINTER(i64), vp]
     L.gracekv_gather.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, i64, vp]
     L.gracekv_export.argtypes = [vp, i64, C.POINTER(i64)] + [vp] * 18 + [vp]
+    L.gracekv_export_floor.argtypes = [vp, vp, vp, C.POINTER(i64), vp]
     L.gracekv_profile.argtypes = [vp, i32]
     L.gracekv_stats.argtypes = [vp, vp, i32, C.POINTER(i64), vp, i32]
     L.gracekv_row_stats_noalloc.argtypes = [vp, vp] + [i32] * 9 + [vp, vp, vp, vp]
@@ -238,6 +241,18 @@ class Context:
                                          _stream(stream)))
 
     STAGES = ("segment", "row_stats", "token_values", "unit_trees", "allocate", "gather")
+
+    def gracekv_export_floor(self, stream=None) -> dict:
+        """The singleton floor of the last tree build (host arrays)."""
+        import numpy as np
+        p = self.params
+        LG = p.L * p.G
+        acc = np.zeros((LG, self.n_c), np.uint8)
+        f = np.zeros((LG, self.n_c), np.float32)
+        bf = C.c_int64()
+        self._check(lib().gracekv_export_floor(self.h, C.c_void_p(acc.ctypes.data), C.c_void_p(f.ctypes.data),
+                                               C.byref(bf), _stream(stream)))
+        return dict(accepted=acc, f=f, B_floor=bf.value)
 
     def gracekv_profile(self, enable: bool = True):
         self._check(lib().gracekv_profile(self.h, int(enable)))

@@ -81,6 +81,8 @@ def oracle_tau(o, lg=None):
     tr = o["trees"]
     nd = tr.nodes
     ua = tr.unit_Uadd
+    if o.get("floor") is not None:      # the floor's Adds execute first: infinite keys
+        ua = np.where(o["floor"]["unit_floor"] == 1, np.inf, ua)
     nm = nd["cost"] > 0
     B = o["B_free"]
     if lg is not None:

@@ -69,7 +69,9 @@ def _create(gk, **kw):
     (dict(windows=(4, 32)), 1),             # window scale above 16
     (dict(seg_layers=(3,)), 1),             # layer out of range
     (dict(lambda_graph=0.3), 8),            # multi-hop relevance not built
-    (dict(alpha_floor=0.6), 8),             # singleton floor not built
+    (dict(alpha_floor=1.5), 1),             # floor cap above the budget
+    (dict(alpha_floor=0.6, floor_eta=1.5), 1),
+    (dict(alpha_floor=0.6, quota_alloc=1), 8),   # floor with fixed per-pair capacity
     (dict(d=96), 8),
     (dict(W=128), 8),
     (dict(budget=7), 2),                    # floor(7 / 2) = 3 < 4 recent tokens

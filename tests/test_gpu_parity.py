@@ -97,6 +97,35 @@ def test_ablations_match_the_oracle(ablation):
     P.compare(g, o, torch.float32)
 
 
+@pytest.mark.parametrize("wname", ["small", "pr1"])
+def test_singleton_floor_matches_the_oracle(wname):
+    # Stage I singleton floor at the paper's alpha = 0.6: the accepted floor
+    # positions, then the trees (forced extraction), the selection (floor ops
+    # first) and the cache against the oracle
+    if wname == "small":
+        w = synth.WORKLOADS["small"]
+        x = synth.make_inputs(w, layers=[0, 1], heads=[0, 1], T=1000)
+        dt = torch.bfloat16
+    else:
+        w = synth.WORKLOADS["pr1"]
+        x = synth.make_inputs(w)
+        dt = torch.float32
+    L, G, T, d = x.K.shape
+    B = (L * G * T) // 8
+    P, g, o = _run(x.K, x.V, x.Q, B, w.rope_base, alpha_floor=0.6)
+    fl = g["comp"].ctx.gracekv_export_floor()
+    ofl = o["floor"]
+    assert ofl["accepted"].sum() > 0
+    diff = np.argwhere(fl["accepted"] != ofl["accepted"])
+    print(wname, "floor", int(ofl["accepted"].sum()), "B_floor", ofl["B_floor"], fl["B_floor"],
+          "differing positions", len(diff))
+    assert len(diff) == 0, diff[:10]
+    assert fl["B_floor"] == ofl["B_floor"]
+    np.testing.assert_allclose(fl["f"], ofl["f"], rtol=2e-5, atol=1e-9)
+    rep = P.compare(g, o, dt)
+    print(wname, json.dumps(rep))
+
+
 def test_fullkv_identity_is_bit_exact():
     # x = 1: every tree expands to its leaves; the cache is the input (App. C.5)
     w = synth.WORKLOADS["pr1"]
