@@ -265,6 +265,8 @@ def main():
                     help="compress once, then time only the decoding attention")
     ap.add_argument("--decode-app", type=int, default=64,
                     help="tokens already appended to every (l, g) when decoding is timed")
+    ap.add_argument("--alpha-floor", type=float, default=None,
+                    help="singleton-floor cap alpha (the library default when omitted)")
     ap.add_argument("--ablation", default="none", choices=["none", "wo_cs", "wo_ga"],
                     help="the paper's w/o CS (uniform slots, midpoint cuts) or w/o GA "
                          "(fixed per-(l, g) capacity) variant")
@@ -294,6 +296,8 @@ def main():
     B = gk.gracekv_budget_for_ratio(L, G, T, args.ratio)
     abl = {"none": {}, "wo_cs": dict(seg_mode=1, k_cand=0, lambda_kappa=0.0),
            "wo_ga": dict(quota_alloc=1)}[args.ablation]
+    if args.alpha_floor is not None:
+        abl = dict(abl, alpha_floor=args.alpha_floor)
     p = gk.make_params(L, G, Q.shape[1], T, d, Q.shape[2], dtype=K.dtype, budget=B,
                        rope_base=w.rope_base, **abl)
     comp = gk.Compressor(p, device=dev)
@@ -420,6 +424,7 @@ def main():
                "dtype": "bf16" if K.dtype == torch.bfloat16 else "f32", "data": "synthetic",
                "config": dict(workload_config(w, args.ratio, L), B_total=B, entries=E,
                               slots=comp.n_slots, parallelism=f"replicas{world}",
+                              alpha_floor=p.alpha_floor,
                               **({"ablation": args.ablation} if args.ablation != "none" else {})),
                "roofline": roof, "hbm_pass": hbm, "stages_ms": per_step, "tree_work": work,
                "cpu_baseline": cpu, "e2e": e2e,

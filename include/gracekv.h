@@ -278,7 +278,7 @@ gkv_status gracekv_export_floor(gracekv_ctx *ctx, uint8_t *accepted, float *f, i
  * Measurement support (not needed to compress).  gracekv_profile(ctx, 1)
  * makes every later stage call record CUDA events on its stream around each
  * kernel group: 0 segmentation, 1 row statistics, 2 token values, 3 unit
- * trees, 4 allocation, 5 gather.  gracekv_stats synchronises the events of
+ * trees, 4 allocation, 5 gather, 6 singleton floor.  gracekv_stats synchronises the events of
  * the calls made since the last gracekv_stats / gracekv_profile and returns
  * the summed milliseconds per group in stage_ms[0 .. n_stages-1] (nullable);
  * *launches (nullable) receives the number of kernels this context has
@@ -287,7 +287,7 @@ gkv_status gracekv_export_floor(gracekv_ctx *ctx, uint8_t *accepted, float *f, i
  * steps, [1] candidate intervals evaluated, [2] sum of candidate lengths,
  * [3] units built.
  */
-#define GRACEKV_N_STAGES 6
+#define GRACEKV_N_STAGES 7
 gkv_status gracekv_profile(gracekv_ctx *ctx, int32_t enable);
 gkv_status gracekv_stats(gracekv_ctx *ctx, float *stage_ms, int32_t n_stages, int64_t *launches,
                          uint64_t *work, int32_t n_work);

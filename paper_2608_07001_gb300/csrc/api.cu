@@ -562,7 +562,7 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
     c.scored = false;
     int cnt[2];
     if (e == cudaSuccess && c.p.alpha_floor > 0.0) {   // Stage I: needs every (l, g)'s token values
-        gkv::StageTimer tm(c, 3, s);
+        gkv::StageTimer tm(c, 6, s);
         e = gkv::launch_floor(c, c.J, s);
     }
     if (e == cudaSuccess) e = build_classes(c, cnt, s);
@@ -678,7 +678,7 @@ gkv_status gracekv_compress_host(gracekv_ctx *x, const void *K, const void *V, c
     }
     if (e == cudaSuccess && fl) {
         if (ranged) {
-            gkv::StageTimer tm(c, 3, s);
+            gkv::StageTimer tm(c, 6, s);
             e = gkv::launch_floor(c, c.J, s);
             if (e == cudaSuccess) e = build_fresh(c, c.hK, c.hV, c.hQ, om, cnt, 0, LG, s);
         }
@@ -693,7 +693,7 @@ gkv_status gracekv_compress_host(gracekv_ctx *x, const void *K, const void *V, c
             e = gkv::launch_token_values(c, c.hK, c.hQ, s);
         }
         if (e == cudaSuccess && fl) {
-            gkv::StageTimer tm(c, 3, s);
+            gkv::StageTimer tm(c, 6, s);
             e = gkv::launch_floor(c, c.J, s);
         }
         if (e == cudaSuccess) e = build_fresh(c, c.hK, c.hV, c.hQ, om, cnt, 0, LG, s);

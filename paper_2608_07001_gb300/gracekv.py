@@ -240,7 +240,7 @@ class Context:
                                          _ptr(out.src_hi), _ptr(out.offsets), out.K.shape[0],
                                          _stream(stream)))
 
-    STAGES = ("segment", "row_stats", "token_values", "unit_trees", "allocate", "gather")
+    STAGES = ("segment", "row_stats", "token_values", "unit_trees", "allocate", "gather", "floor")
 
     def gracekv_export_floor(self, stream=None) -> dict:
         """The singleton floor of the last tree build (host arrays)."""

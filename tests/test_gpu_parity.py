@@ -97,8 +97,8 @@ def test_ablations_match_the_oracle(ablation):
     P.compare(g, o, torch.float32)
 
 
-@pytest.mark.parametrize("wname", ["small", "pr1"])
-def test_singleton_floor_matches_the_oracle(wname):
+@pytest.mark.parametrize("wname,alpha", [("small", 0.6), ("pr1", 0.6), ("small", 0.05), ("pr1", 0.1)])
+def test_singleton_floor_matches_the_oracle(wname, alpha):
     # Stage I singleton floor at the paper's alpha = 0.6: the accepted floor
     # positions, then the trees (forced extraction), the selection (floor ops
     # first) and the cache against the oracle
@@ -112,7 +112,7 @@ def test_singleton_floor_matches_the_oracle(wname):
         dt = torch.float32
     L, G, T, d = x.K.shape
     B = (L * G * T) // 8
-    P, g, o = _run(x.K, x.V, x.Q, B, w.rope_base, alpha_floor=0.6)
+    P, g, o = _run(x.K, x.V, x.Q, B, w.rope_base, alpha_floor=alpha)
     fl = g["comp"].ctx.gracekv_export_floor()
     ofl = o["floor"]
     assert ofl["accepted"].sum() > 0
@@ -251,17 +251,19 @@ def test_score_ahead_matches_inline():
         assert np.array_equal(np.asarray(a[k]), np.asarray(b[k])), k
 
 
-@pytest.mark.parametrize("wname,kw", [("small", dict(layers=[0, 1, 2, 3], heads=[0, 1], T=1000)),
-                                      ("pr1", dict(T=700))])
-def test_compress_host_matches_device(wname, kw):
+@pytest.mark.parametrize("wname,kw,alpha", [("small", dict(layers=[0, 1, 2, 3], heads=[0, 1], T=1000), 0.0),
+                                            ("pr1", dict(T=700), 0.0),
+                                            ("small", dict(layers=[0, 1, 2, 3], heads=[0, 1], T=1000), 0.6)])
+def test_compress_host_matches_device(wname, kw, alpha):
     # The host-buffer pipeline (layer-group copies overlapped with the score
-    # passes and the first tree launch) gives the device path's cache bits.
+    # passes and the first tree launch; with a singleton floor the tree build
+    # waits for every group) gives the device path's cache bits.
     from paper_2608_07001_gb300 import gracekv as gk
     w = synth.WORKLOADS[wname]
     x = synth.make_inputs(w, **kw)
     L, G, T, d = x.K.shape
     p = gk.make_params(L, G, x.Q.shape[1], T, d, x.Q.shape[2], dtype=x.K.dtype, budget=(L * G * T) // 8,
-                       rope_base=w.rope_base)
+                       rope_base=w.rope_base, alpha_floor=alpha)
     comp = gk.Compressor(p)
     dev = comp(x.K.cuda(), x.V.cuda(), x.Q.cuda())
     E = comp.n_entries
