@@ -352,6 +352,19 @@ def gather(p: Params, K, V, rtok, tr: Trees, add_sel, split_sel, cap: int):
                 offsets=off)
 
 
+def head_sensitivity(W_O, o, G: int, eps: float = 1e-6):
+    """omega [L, G] from W_O [L, D, Hq*d] and o [L, Hq, U, d] (Eq. app_head_sensitivity)."""
+    W_O, o = _f64(W_O), _f64(o)
+    L, Hq, U, d = o.shape
+    D = W_O.shape[1]
+    om = np.zeros((L, G))
+    rc = lib().orc_head_sensitivity(*(C.c_int32(v) for v in (L, G, Hq, d, D, U)),
+                                    _p(W_O, C.c_double), _p(o, C.c_double), C.c_double(eps),
+                                    _p(om, C.c_double))
+    assert rc == 0, rc
+    return om
+
+
 def decode_attention(q, K, V, log_m, offsets, K_app=None, V_app=None, n_app: int = 0,
                      *, L: int, G: int, l0: int = 0):
     """Eq. (app_decode_logit) over the packed cache plus n_app appended rows.

@@ -1238,3 +1238,53 @@ int orc_decode_attention(int32_t L, int32_t G, int32_t Hq, int32_t d, int32_t l0
     free(x);
     return ORC_OK;
 }
+
+/* Layer-KV-head sensitivity, App. A.4 Eqs. (app_head_sensitivity_raw),
+ * (app_head_sensitivity):
+ *   static_{l,g} = ( sum_{h in H(g)} ||W_O^{l,h}||_F^2 )^{1/2}
+ *   input_{l,g}  = Mean_u || sum_{h in H(g)} W_O^{l,h} o_u^{l,h} ||_2
+ *   raw = sqrt(static input),  omega = raw / (Mean_{l,g} raw + eps). */
+int orc_head_sensitivity(int32_t L, int32_t G, int32_t Hq, int32_t d, int32_t D, int32_t U,
+                         const double *W_O, const double *o, double eps, double *omega)
+{
+    if (L <= 0 || G <= 0 || Hq % G || d <= 0 || D <= 0 || U <= 0) return ORC_EINVAL;
+    int gq = Hq / G;
+    size_t row = (size_t)Hq * d;                 /* a row of W_O: all heads' columns */
+    double *y = (double *)malloc(sizeof(double) * (size_t)D);
+    if (!y) return ORC_ENOMEM;
+    double mean = 0.0;
+    for (int l = 0; l < L; l++)
+        for (int g = 0; g < G; g++) {
+            const double *W = W_O + (size_t)l * D * row;
+            double st = 0.0;
+            for (int r = 0; r < D; r++)
+                for (int hh = 0; hh < gq; hh++)
+                    for (int i = 0; i < d; i++) {
+                        double w = W[(size_t)r * row + (size_t)(g * gq + hh) * d + i];
+                        st += w * w;
+                    }
+            st = sqrt(st);
+            double in = 0.0;
+            for (int u = 0; u < U; u++) {
+                for (int r = 0; r < D; r++) {
+                    double acc = 0.0;
+                    for (int hh = 0; hh < gq; hh++) {
+                        int h = g * gq + hh;
+                        const double *ou = o + (((size_t)l * Hq + h) * U + u) * d;
+                        for (int i = 0; i < d; i++) acc += W[(size_t)r * row + (size_t)h * d + i] * ou[i];
+                    }
+                    y[r] = acc;
+                }
+                double nn = 0.0;
+                for (int r = 0; r < D; r++) nn += y[r] * y[r];
+                in += sqrt(nn);
+            }
+            in /= U;
+            omega[l * G + g] = sqrt(st * in);
+            mean += omega[l * G + g];
+        }
+    mean /= (double)L * G;
+    for (int k = 0; k < L * G; k++) omega[k] /= mean + eps;
+    free(y);
+    return ORC_OK;
+}

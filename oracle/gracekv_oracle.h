@@ -28,6 +28,7 @@
  *   gains / costs     App. A.5 Eqs. (app_operation_gains) .. (app_unit_utility)
  *   greedy allocation App. A.5 Stage II, App. C.3 (max-priority queue)
  *   packing           App. A.5 "Frontier updates and physical packing"
+ *   head sensitivity  App. A.4 Eqs. (app_head_sensitivity_raw), (app_head_sensitivity)
  *   decoding          App. A.3 Eq. (app_decode_logit) over the packed cache
  *                     plus appended tokens at multiplicity 1 (App. A.5)
  *
@@ -175,6 +176,13 @@ int orc_gather(const orc_params *p, const double *K, const double *V, const doub
                const uint8_t *add_sel, const uint8_t *split_sel, int64_t cap,
                double *K_out, double *V_out, int32_t *pos, double *log_m,
                int32_t *src_lo, int32_t *src_hi, int64_t *offsets, int64_t *n_entries);
+
+/* Layer-KV-head sensitivity, App. A.4 Eqs. (app_head_sensitivity_raw),
+ * (app_head_sensitivity).  W_O [L][D][Hq d] (the output projection of each
+ * layer, row-major: column block h is W_O^{l,h}); o [L][Hq][U][d] (attention
+ * outputs of the U question probes before the projection); omega [L][G]. */
+int orc_head_sensitivity(int32_t L, int32_t G, int32_t Hq, int32_t d, int32_t D, int32_t U,
+                         const double *W_O, const double *o, double eps, double *omega);
 
 /* q [nl][Hq][d] for layers l0 .. l0 + nl - 1; packed cache K, V [E][d],
  * log_m [E], off [L G + 1]; appended rows K_app, V_app [L][G][app_cap][d]
