@@ -266,6 +266,25 @@ gkv_status gracekv_export(gracekv_ctx *ctx, int64_t node_cap, int64_t *n_nodes_h
                           float *row_ZC, float *rtok, void *stream);
 
 /*
+ * Layer-KV-head sensitivity omega (App. A.4, Eqs. app_head_sensitivity_raw,
+ * app_head_sensitivity), the per-(l, g) multiplier the pass takes as its
+ * omega input.  No context, no allocation.
+ *   W_O [L][D][Hq d] bf16: each layer's attention output projection, row-major
+ *     (out_features x in_features); column block h (d columns) is W_O^{l,h}.
+ *   o [L][Hq][U][d] bf16: the heads' attention outputs at the U question
+ *     probes, before the projection (U <= 64).
+ *   omega [L][G] fp32 (device, output); scratch: L G 65 fp32 (device).
+ * static = (sum_{h in H(g)} ||W_O^{l,h}||_F^2)^{1/2}, input = mean_u
+ * ||sum_{h in H(g)} W_O^{l,h} o_u^{l,h}||_2, raw = sqrt(static input),
+ * omega = raw / (mean raw + 1e-6).  Products on the tensor cores (exact bf16
+ * products, fp32 sums).  Errors: GKV_EINVAL, GKV_EUNSUPPORTED (dtype other
+ * than bf16, d not in {64, 128}, U > 64, D not a multiple of 8), GKV_ECUDA.
+ */
+gkv_status gracekv_head_sensitivity(const void *W_O, const void *o, int32_t L, int32_t G, int32_t Hq,
+                                    int32_t d, int32_t D, int32_t U, int32_t dtype, float *omega,
+                                    float *scratch, void *stream);
+
+/*
  * The singleton floor of the last gracekv_build_trees (alpha_floor > 0), to
  * caller-owned HOST arrays (synchronises `stream`): accepted [L G][N_c] uint8
  * (1 = a floor singleton), f [L G][N_c] fp32 floor scores (nullable),

@@ -64,7 +64,7 @@ EXPORTED = ["gracekv_default_params", "gracekv_budget_for_ratio", "gracekv_creat
             "gracekv_destroy", "gracekv_last_error", "gracekv_status_string", "gracekv_query",
             "gracekv_segment", "gracekv_score", "gracekv_build_trees", "gracekv_allocate", "gracekv_gather",
             "gracekv_export", "gracekv_profile", "gracekv_stats", "gracekv_row_stats_noalloc",
-            "gracekv_compress_host", "gracekv_export_floor", "gracekv_decode_workspace_size", "gracekv_decode_append",
+            "gracekv_compress_host", "gracekv_export_floor", "gracekv_head_sensitivity", "gracekv_decode_workspace_size", "gracekv_decode_append",
             "gracekv_decode_attention", "gracekv_decode_status"]
 
 
@@ -96,6 +96,7 @@ def lib() -> C.CDLL:
     L.gracekv_gather.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, i64, vp]
     L.gracekv_export.argtypes = [vp, i64, C.POINTER(i64)] + [vp] * 18 + [vp]
     L.gracekv_export_floor.argtypes = [vp, vp, vp, C.POINTER(i64), vp]
+    L.gracekv_head_sensitivity.argtypes = [vp, vp] + [i32] * 7 + [vp, vp, vp]
     L.gracekv_profile.argtypes = [vp, i32]
     L.gracekv_stats.argtypes = [vp, vp, i32, C.POINTER(i64), vp, i32]
     L.gracekv_row_stats_noalloc.argtypes = [vp, vp] + [i32] * 9 + [vp, vp, vp, vp]
@@ -133,6 +134,19 @@ def gracekv_row_stats_noalloc(K, Q, c_lo: int, c_hi: int, row_m, row_Z, row_ZC, 
                                          _ptr(row_m), _ptr(row_Z), _ptr(row_ZC), _stream(stream))
     if st != GKV_OK:
         raise GraceKVError(st, lib().gracekv_status_string(st).decode())
+
+
+def gracekv_head_sensitivity(W_O, o, G: int, stream=None):
+    """omega [L, G] (fp32, device) from W_O [L, D, Hq*d] and o [L, Hq, U, d] (bf16)."""
+    L, D, _ = W_O.shape
+    _, Hq, U, d = o.shape
+    om = torch.empty(L, G, dtype=torch.float32, device=W_O.device)
+    scratch = torch.empty(L * G * 65, dtype=torch.float32, device=W_O.device)
+    st = lib().gracekv_head_sensitivity(_ptr(W_O), _ptr(o), L, G, Hq, d, D, U, GKV_BF16, _ptr(om),
+                                        _ptr(scratch), _stream(stream))
+    if st != GKV_OK:
+        raise GraceKVError(st, lib().gracekv_status_string(st).decode())
+    return om
 
 
 def _host_ptr(t: Optional[torch.Tensor]):

@@ -126,6 +126,25 @@ def test_singleton_floor_matches_the_oracle(wname, alpha):
     print(wname, json.dumps(rep))
 
 
+@pytest.mark.parametrize("L,G,gq,d,D,U", [(3, 2, 4, 128, 1024, 32), (2, 8, 4, 128, 4096, 64),
+                                          (4, 4, 1, 64, 520, 5)])
+def test_head_sensitivity_matches_the_oracle(L, G, gq, d, D, U):
+    # omega of App. A.4 (Eq. app_head_sensitivity) on the tensor cores vs the
+    # oracle; the per-(l, g) output of the one call feeds the pass's omega
+    import oracle as O
+    from paper_2608_07001_gb300 import gracekv as gk
+    g = torch.Generator().manual_seed(L * 100 + D)
+    Hq = G * gq
+    W = (torch.randn(L, D, Hq * d, generator=g) / d ** 0.5)
+    W[:, :, :gq * d] *= 3.0                       # one group stands out
+    W = W.to(torch.bfloat16)
+    o = torch.randn(L, Hq, U, d, generator=g).to(torch.bfloat16)
+    om = gk.gracekv_head_sensitivity(W.cuda(), o.cuda(), G).cpu().double().numpy()
+    ref = O.head_sensitivity(W, o, G)
+    # fp32 sums of exact products: a few ulp of the sums per term, well below 1e-4
+    np.testing.assert_allclose(om, ref, rtol=1e-4, atol=1e-6)
+
+
 def test_fullkv_identity_is_bit_exact():
     # x = 1: every tree expands to its leaves; the cache is the input (App. C.5)
     w = synth.WORKLOADS["pr1"]
