@@ -245,6 +245,35 @@ def decode_leg(args, w, comp, L, G, Hq, d, dev):
                          "peak_kind": pk_kind, "traffic": None}}
 
 
+def sensitivity_leg(args, w, D=4096, U=32):
+    """omega (Eq. app_head_sensitivity) from a synthetic output projection
+    W_O [L, D, Hq d] and head outputs o [L, Hq, U, d] of the workload's shape;
+    the pass reads W_O once, so its bytes set the roofline."""
+    from paper_2608_07001_gb300 import gracekv as gk
+    dev = torch.device("cuda")
+    gen = torch.Generator(device=dev).manual_seed(11)
+    W = (torch.randn(w.L, D, w.Hq * w.d, generator=gen, device=dev) / w.d ** 0.5).to(torch.bfloat16)
+    o = torch.randn(w.L, w.Hq, U, w.d, generator=gen, device=dev).to(torch.bfloat16)
+    for _ in range(3):
+        gk.gracekv_head_sensitivity(W, o, w.G)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = 20
+    e0.record()
+    for _ in range(reps):
+        gk.gracekv_head_sensitivity(W, o, w.G)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    byt = W.numel() * 2 + o.numel() * 2
+    pk, pk_kind = peaks()
+    ach = byt / (ms / 1e3) / 1e9
+    return {"shape": f"L {w.L}, Hq {w.Hq}, d {w.d}, D {D}, U {U}", "ms": ms, "bytes": byt,
+            "roofline": {"kernel": "sens_tile_kernel", "bound": "hbm", "achieved": ach,
+                         "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": ach / pk["hbm_gbs"],
+                         "peak_kind": pk_kind, "traffic": None}}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -265,6 +294,8 @@ def main():
                     help="compress once, then time only the decoding attention")
     ap.add_argument("--decode-app", type=int, default=64,
                     help="tokens already appended to every (l, g) when decoding is timed")
+    ap.add_argument("--sensitivity-only", action="store_true",
+                    help="time only the layer-KV-head sensitivity on the workload's shape")
     ap.add_argument("--alpha-floor", type=float, default=None,
                     help="singleton-floor cap alpha (the library default when omitted)")
     ap.add_argument("--ablation", default="none", choices=["none", "wo_cs", "wo_ga"],
@@ -274,6 +305,9 @@ def main():
 
     from paper_2608_07001_gb300 import synth
     w = synth.WORKLOADS[args.workload]
+    if args.sensitivity_only:
+        print(json.dumps({"head_sensitivity": sensitivity_leg(args, w)}))
+        return
     if args.impl == "reference":
         run_reference(args, w)
         return

@@ -31,15 +31,26 @@ __device__ __forceinline__ void se_ldsm_x4(uint32_t addr, uint32_t a[4]) {
                  : "r"(addr));
 }
 
+// Two stages: the copies of chunk k + 1 fly while chunk k is multiplied.
+template <int NT8>
+struct SeSmem {
+    __nv_bfloat16 Ws[2][kSeRows][kSeK + kSePad];
+    __nv_bfloat16 Xs[2][NT8 * 8][kSeK + kSePad];
+    float red[8][NT8 * 8];
+    float fred[8];
+};
+
 // grid (D / 128, G, L), 256 threads: warp w owns rows 16 w .. 16 w + 15 of the tile.
 template <int NT8>
 __global__ void __launch_bounds__(256) sens_tile_kernel(const __nv_bfloat16 *__restrict__ W,
                                                         const __nv_bfloat16 *__restrict__ o, int G, int Hq,
                                                         int d, int D, int U, float *sumsq, float *fro) {
-    __shared__ __align__(16) __nv_bfloat16 Ws[kSeRows][kSeK + kSePad];
-    __shared__ __align__(16) __nv_bfloat16 Xs[NT8 * 8][kSeK + kSePad];
-    __shared__ float red[8][NT8 * 8];
-    __shared__ float fred[8];
+    extern __shared__ __align__(16) unsigned char se_raw[];
+    SeSmem<NT8> &sm = *reinterpret_cast<SeSmem<NT8> *>(se_raw);
+    auto &Ws = sm.Ws;
+    auto &Xs = sm.Xs;
+    auto &red = sm.red;
+    auto &fred = sm.fred;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int r0 = blockIdx.x * kSeRows, g = blockIdx.y, l = blockIdx.z;
     const int gq = Hq / G, Kg = gq * d;
@@ -50,13 +61,34 @@ __global__ void __launch_bounds__(256) sens_tile_kernel(const __nv_bfloat16 *__r
     for (int n = 0; n < NT8; n++) acc[n][0] = acc[n][1] = acc[n][2] = acc[n][3] = 0.f;
     float fsq = 0.f;
     const int hq = lane >> 2, tq = lane & 3, mi = lane >> 3, ri = lane & 7;
-    for (int k0 = 0; k0 < Kg; k0 += kSeK) {
-        // W tile [128][64]: 16-byte loads, their squares for the Frobenius norm
+    auto issue = [&](int k0, int st) {
+        for (int e = tid; e < kSeRows * kSeK / 8; e += 256) {      // W tile [128][64]
+            const int r = e / (kSeK / 8), c = e % (kSeK / 8);
+            const bool in = r0 + r < D;
+            cp_async16(&Ws[st][r][8 * c], in ? Wl + (size_t)(r0 + r) * row + k0 + 8 * c : Wl, in);
+        }
+        const int hh = k0 / d, i0 = k0 % d;                         // inside one head (d >= 64)
+        for (int e = tid; e < NT8 * 8 * kSeK / 8; e += 256) {      // X chunk [probes][64]
+            const int u = e / (kSeK / 8), c = e % (kSeK / 8);
+            const bool in = u < U;
+            cp_async16(&Xs[st][u][8 * c],
+                       in ? o + (((size_t)l * Hq + g * gq + hh) * U + u) * d + i0 + 8 * c : o, in);
+        }
+        cp_async_commit();
+    };
+    issue(0, 0);
+    for (int k0 = 0, st = 0; k0 < Kg; k0 += kSeK, st ^= 1) {
+        if (k0 + kSeK < Kg) {
+            issue(k0 + kSeK, st ^ 1);
+            cp_async_wait<1>();
+        } else {
+            cp_async_wait<0>();
+        }
+        __syncthreads();
+        // squares of the W values this thread copied, for the Frobenius norm
         for (int e = tid; e < kSeRows * kSeK / 8; e += 256) {
             const int r = e / (kSeK / 8), c = e % (kSeK / 8);
-            uint4 v = make_uint4(0u, 0u, 0u, 0u);
-            if (r0 + r < D) v = *reinterpret_cast<const uint4 *>(Wl + (size_t)(r0 + r) * row + k0 + 8 * c);
-            *reinterpret_cast<uint4 *>(&Ws[r][8 * c]) = v;
+            const uint4 v = *reinterpret_cast<const uint4 *>(&Ws[st][r][8 * c]);
             const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
             for (int q = 0; q < 4; q++) {
@@ -65,30 +97,20 @@ __global__ void __launch_bounds__(256) sens_tile_kernel(const __nv_bfloat16 *__r
                 fsq = fmaf(hi, hi, fsq);
             }
         }
-        // X chunk: probe u's outputs at k0 .. k0 + 63 (inside one head, d >= 64)
-        const int hh = k0 / d, i0 = k0 % d;
-        for (int e = tid; e < NT8 * 8 * kSeK / 8; e += 256) {
-            const int u = e / (kSeK / 8), c = e % (kSeK / 8);
-            uint4 v = make_uint4(0u, 0u, 0u, 0u);
-            if (u < U)
-                v = *reinterpret_cast<const uint4 *>(o + (((size_t)l * Hq + g * gq + hh) * U + u) * d + i0 + 8 * c);
-            *reinterpret_cast<uint4 *>(&Xs[u][8 * c]) = v;
-        }
-        __syncthreads();
 #pragma unroll
         for (int ks = 0; ks < kSeK / 16; ks++) {
             uint32_t a[4];
             se_ldsm_x4(static_cast<uint32_t>(__cvta_generic_to_shared(
-                           &Ws[warp * 16 + ri + (mi & 1) * 8][ks * 16 + (mi >> 1) * 8])),
+                           &Ws[st][warp * 16 + ri + (mi & 1) * 8][ks * 16 + (mi >> 1) * 8])),
                        a);
 #pragma unroll
             for (int n = 0; n < NT8; n++) {
-                const uint32_t b0 = *reinterpret_cast<const uint32_t *>(&Xs[n * 8 + hq][ks * 16 + 2 * tq]);
-                const uint32_t b1 = *reinterpret_cast<const uint32_t *>(&Xs[n * 8 + hq][ks * 16 + 8 + 2 * tq]);
+                const uint32_t b0 = *reinterpret_cast<const uint32_t *>(&Xs[st][n * 8 + hq][ks * 16 + 2 * tq]);
+                const uint32_t b1 = *reinterpret_cast<const uint32_t *>(&Xs[st][n * 8 + hq][ks * 16 + 8 + 2 * tq]);
                 mma_bf16(acc[n], a, b0, b1);
             }
         }
-        __syncthreads();
+        __syncthreads();    // the stage is refilled by the next issue
     }
     // squared 2-norm pieces per probe: rows hq and hq + 8 of the warp's 16
 #pragma unroll
@@ -152,6 +174,21 @@ __global__ void __launch_bounds__(1024) sens_final_kernel(const float *sumsq, co
     for (int k = tid; k < LG; k += 1024) omega[k] = omega[k] / (mean + eps);
 }
 
+template <int NT8>
+cudaError_t launch_sens_tile(dim3 grid, cudaStream_t s, const __nv_bfloat16 *W, const __nv_bfloat16 *o, int G,
+                             int Hq, int d, int D, int U, float *sumsq, float *fro) {
+    constexpr size_t smem = sizeof(SeSmem<NT8>);
+    static bool attr = false;     // the opt-in above 48 KB, once per instantiation
+    if (!attr) {
+        cudaError_t e = cudaFuncSetAttribute(sens_tile_kernel<NT8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)smem);
+        if (e != cudaSuccess) return e;
+        attr = true;
+    }
+    sens_tile_kernel<NT8><<<grid, 256, smem, s>>>(W, o, G, Hq, d, D, U, sumsq, fro);
+    return cudaGetLastError();
+}
+
 }  // namespace
 }  // namespace gkv
 
@@ -172,12 +209,14 @@ extern "C" gkv_status gracekv_head_sensitivity(const void *W_O, const void *o, i
     const dim3 grid((D + gkv::kSeRows - 1) / gkv::kSeRows, G, L);
     const auto *Wb = static_cast<const __nv_bfloat16 *>(W_O);
     const auto *ob = static_cast<const __nv_bfloat16 *>(o);
+    cudaError_t e;
     if (U <= 16)
-        gkv::sens_tile_kernel<2><<<grid, 256, 0, s>>>(Wb, ob, G, Hq, d, D, U, sumsq, fro);
+        e = gkv::launch_sens_tile<2>(grid, s, Wb, ob, G, Hq, d, D, U, sumsq, fro);
     else if (U <= 32)
-        gkv::sens_tile_kernel<4><<<grid, 256, 0, s>>>(Wb, ob, G, Hq, d, D, U, sumsq, fro);
+        e = gkv::launch_sens_tile<4>(grid, s, Wb, ob, G, Hq, d, D, U, sumsq, fro);
     else
-        gkv::sens_tile_kernel<8><<<grid, 256, 0, s>>>(Wb, ob, G, Hq, d, D, U, sumsq, fro);
+        e = gkv::launch_sens_tile<8>(grid, s, Wb, ob, G, Hq, d, D, U, sumsq, fro);
+    if (e != cudaSuccess) return GKV_ECUDA;
     gkv::sens_final_kernel<<<1, 1024, 0, s>>>(sumsq, fro, LG, U, 1e-6f, omega);
     return cudaGetLastError() == cudaSuccess ? GKV_OK : GKV_ECUDA;
 }
