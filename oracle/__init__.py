@@ -49,6 +49,8 @@ class Params(C.Structure):
         ("disp_mode", C.c_int32),
         ("alpha_floor", C.c_double), ("floor_c", C.c_double), ("floor_gamma", C.c_double),
         ("floor_eta", C.c_double), ("floor_half", C.c_int32),
+        ("lambda_graph", C.c_double), ("eta_seed", C.c_double), ("rho_hop", C.c_double),
+        ("m_seed", C.c_int32), ("r_hop", C.c_int32),
         ("seg_mode", C.c_int32), ("quota_alloc", C.c_int32),
     ]
 
@@ -88,7 +90,8 @@ PAPER_DEFAULTS = dict(
     lambda_d=0.25, lambda_n=0.10, c_cut=1.0, windows=(4, 8, 16), k_cand=16,
     lambda_kappa=0.05, lambda_Z=0.25, lambda_M=0.75, eps=1e-6, base_frac=0.1,
     seg_layers=(), disp_mode=0, seg_mode=0, quota_alloc=0,
-    alpha_floor=0.0, floor_c=0.5, floor_gamma=1.2, floor_eta=0.95, floor_half=3)
+    alpha_floor=0.0, floor_c=0.5, floor_gamma=1.2, floor_eta=0.95, floor_half=3,
+    lambda_graph=0.0, eta_seed=0.9, rho_hop=0.5, m_seed=64, r_hop=2)
 
 
 def make_params(L, G, Hq, T, d, W, rope_base, ctx_start=0, ctx_end=None, **kw) -> Params:
@@ -118,6 +121,8 @@ def make_params(L, G, Hq, T, d, W, rope_base, ctx_start=0, ctx_end=None, **kw) -
     p.quota_alloc = o["quota_alloc"]
     p.alpha_floor, p.floor_c = o["alpha_floor"], o["floor_c"]
     p.floor_gamma, p.floor_eta, p.floor_half = o["floor_gamma"], o["floor_eta"], o["floor_half"]
+    p.lambda_graph, p.eta_seed, p.rho_hop = o["lambda_graph"], o["eta_seed"], o["rho_hop"]
+    p.m_seed, p.r_hop = o["m_seed"], o["r_hop"]
     return p
 
 
@@ -352,6 +357,28 @@ def gather(p: Params, K, V, rtok, tr: Trees, add_sel, split_sel, cap: int):
                 offsets=off)
 
 
+def graph_layers(p: Params):
+    out = np.zeros(4, dtype=np.int32)
+    n = lib().orc_graph_layers(C.byref(p), _p(out, C.c_int32))
+    return out[:n].copy()
+
+
+def multihop(p: Params, shat, Qg, K, graph_l=None):
+    """d-hat [N_c] and the seeds [r_hop, m_seed] / weights of every hop (App. A.4)."""
+    shat, Qg, K = _f64(shat), _f64(Qg), _f64(K)
+    gl = graph_layers(p) if graph_l is None else np.asarray(graph_l, dtype=np.int32)
+    gl = np.ascontiguousarray(gl, dtype=np.int32)
+    Nc = p.ctx_end - p.recent - p.ctx_start
+    dh = np.zeros(Nc)
+    sd = np.zeros((p.r_hop, p.m_seed), dtype=np.int32)
+    sw = np.zeros((p.r_hop, p.m_seed))
+    rc = lib().orc_multihop(C.byref(p), _p(shat, C.c_double), _p(Qg, C.c_double), _p(gl, C.c_int32),
+                            C.c_int32(len(gl)), _p(K, C.c_double), _p(dh, C.c_double), _p(sd, C.c_int32),
+                            _p(sw, C.c_double))
+    assert rc == 0, rc
+    return dh, sd, sw
+
+
 def head_sensitivity(W_O, o, G: int, eps: float = 1e-6):
     """omega [L, G] from W_O [L, D, Hq*d] and o [L, Hq, U, d] (Eq. app_head_sensitivity)."""
     W_O, o = _f64(W_O), _f64(o)
@@ -392,7 +419,7 @@ def decode_attention(q, K, V, log_m, offsets, K_app=None, V_app=None, n_app: int
 
 
 def run(K, V, Q, B_total: int, rope_base: float, *, ctx_start=0, ctx_end=None, omega=None,
-        surprisal=None, hidden=None, slot_starts=None, **overrides) -> dict:
+        surprisal=None, hidden=None, slot_starts=None, Qg=None, **overrides) -> dict:
     """Whole compression pass on the oracle; returns every intermediate."""
     L, G, T, d = K.shape
     Hq, W = Q.shape[1], Q.shape[2]
@@ -411,6 +438,13 @@ def run(K, V, Q, B_total: int, rope_base: float, *, ctx_start=0, ctx_end=None, o
                    dp_best=None, dp_second=None)
     m, Z, ZC = row_stats(p, Q64, K64)
     rtok = token_values(p, Q64, K64, m, Z)
+    mh = None
+    if p.lambda_graph > 0:
+        # App. A.4 Eq. (app_bottom_up_value): R = (1 - lambda) s-hat + lambda d-hat
+        assert Qg is not None, "multi-hop relevance needs the graph layers' queries"
+        dh, sd, sw = multihop(p, rtok, Qg, K64)
+        mh = dict(dhat=dh, seeds=sd, weights=sw, shat=rtok.copy())
+        rtok = (1.0 - p.lambda_graph) * rtok + p.lambda_graph * dh[None, None, :]
     fl = None
     if p.alpha_floor > 0:
         f, acc, B_floor, n_cand = floor(p, rtok, seg["slot_starts"], B_free)
@@ -422,4 +456,5 @@ def run(K, V, Q, B_total: int, rope_base: float, *, ctx_start=0, ctx_end=None, o
     cap = B_total + L * G * (T - (p.ctx_end - p.ctx_start)) + 16
     cache = gather(p, K64, V64, rtok, tr, add_sel, split_sel, cap)
     return dict(params=p, r_eff=r_eff, B_free=B_free, seg=seg, m=m, Z=Z, ZC=ZC, rtok=rtok,
-                trees=tr, add_sel=add_sel, split_sel=split_sel, used=used, cache=cache, floor=fl)
+                trees=tr, add_sel=add_sel, split_sel=split_sel, used=used, cache=cache, floor=fl,
+                multihop=mh)

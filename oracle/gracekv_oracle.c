@@ -1288,3 +1288,107 @@ int orc_head_sensitivity(int32_t L, int32_t G, int32_t Hq, int32_t d, int32_t D,
     free(y);
     return ORC_OK;
 }
+
+/* Graph layers: relative depths 0.50 and 0.75 (reading R16). */
+int orc_graph_layers(const orc_params *p, int32_t *out)
+{
+    static const double rho[2] = {0.50, 0.75};
+    int n = 0;
+    for (int k = 0; k < 2; k++) {
+        int l = (int)floor(rho[k] * p->L);
+        if (l > p->L - 1) l = p->L - 1;
+        int dup = 0;
+        for (int j = 0; j < n; j++) dup |= (out[j] == l);
+        if (!dup) out[n++] = l;
+    }
+    return n;
+}
+
+/* Seeds of a hop (reading R16): score sc[Nc] over C, descending (ties lower
+ * t), while fewer than m_seed are taken and the running mass is below eta. */
+static int pick_seeds(const orc_params *p, const double *sc, int Nc, kv_t *ord, int32_t *sd, double *w)
+{
+    double tot = 0.0;
+    for (int t = 0; t < Nc; t++) { ord[t].v = sc[t]; ord[t].t = t; tot += sc[t]; }
+    qsort(ord, (size_t)Nc, sizeof(kv_t), cmp_kv_desc);
+    int n = 0;
+    double cum = 0.0, ws = 0.0;
+    while (n < p->m_seed && n < Nc && cum < p->eta_seed) {
+        sd[n] = ord[n].t;
+        w[n] = ord[n].v;
+        cum += ord[n].v;
+        ws += ord[n].v;
+        n++;
+    }
+    for (int k = 0; k < n; k++) w[k] = ws > 0.0 ? w[k] / ws : 1.0 / n;
+    (void)tot;
+    return n;
+}
+
+int orc_multihop(const orc_params *p, const double *shat, const double *Qg, const int32_t *graph_l,
+                 int32_t n_graph, const double *K, double *dhat, int32_t *seeds, double *seed_w)
+{
+    int L = p->L, G = p->G, Hq = p->Hq, T = p->T, d = p->d, gq = Hq / G;
+    int c0 = p->ctx_start, Nc = p->ctx_end - p->recent - c0, LG = L * G;
+    double *S = (double *)calloc((size_t)Nc, sizeof(double));
+    double *sc = (double *)malloc(sizeof(double) * (size_t)Nc);
+    double *dk = (double *)malloc(sizeof(double) * (size_t)Nc);
+    double *acc = (double *)calloc((size_t)Nc, sizeof(double));
+    double *x = (double *)malloc(sizeof(double) * (size_t)T);
+    kv_t *ord = (kv_t *)malloc(sizeof(kv_t) * (size_t)Nc);
+    int32_t *sd = (int32_t *)malloc(sizeof(int32_t) * (size_t)(p->m_seed + 1));
+    double *w = (double *)malloc(sizeof(double) * (size_t)(p->m_seed + 1));
+    uint8_t *was = (uint8_t *)calloc((size_t)Nc, 1);
+    if (!S || !sc || !dk || !acc || !x || !ord || !sd || !w || !was) {
+        free(S); free(sc); free(dk); free(acc); free(x); free(ord); free(sd); free(w); free(was);
+        return ORC_ENOMEM;
+    }
+    if (seeds)
+        for (int k = 0; k < p->r_hop * p->m_seed; k++) seeds[k] = -1;
+    /* global seed score, Eq. (app_global_seed_score) */
+    for (int lg = 0; lg < LG; lg++)
+        for (int t = 0; t < Nc; t++) S[t] += shat[(size_t)lg * Nc + t];
+    double tot = 0.0;
+    for (int t = 0; t < Nc; t++) { S[t] /= LG; tot += S[t]; }
+    for (int t = 0; t < Nc; t++) sc[t] = S[t] / (tot + p->eps);
+    double decay = 1.0;
+    for (int k = 0; k < p->r_hop; k++) {
+        int ns = pick_seeds(p, sc, Nc, ord, sd, w);
+        if (seeds)
+            for (int q = 0; q < ns; q++) { seeds[k * p->m_seed + q] = sd[q] + c0; seed_w[k * p->m_seed + q] = w[q]; }
+        for (int q = 0; q < ns; q++) was[sd[q]] = 1;
+        /* propagation, Eq. (app_hop_propagation) */
+        for (int t = 0; t < Nc; t++) dk[t] = 0.0;
+        for (int gi = 0; gi < n_graph; gi++) {
+            int l = graph_l[gi];
+            for (int h = 0; h < Hq; h++) {
+                int g = h / gq;
+                const double *Kg = K + (((size_t)l * G + g) * T) * d;
+                for (int q = 0; q < ns; q++) {
+                    int u = sd[q] + c0;                      /* absolute position of the seed */
+                    const double *qu = Qg + (((size_t)gi * Hq + h) * T + u) * d;
+                    double mx = -INFINITY;
+                    for (int tau = 0; tau <= u; tau++) {     /* visible range [0, u] */
+                        x[tau] = logit(qu, Kg + (size_t)tau * d, d);
+                        if (x[tau] > mx) mx = x[tau];
+                    }
+                    double Z = 0.0;
+                    for (int tau = 0; tau <= u; tau++) Z += exp(x[tau] - mx);
+                    for (int t = c0; t < c0 + Nc && t <= u; t++) dk[t - c0] += w[q] * exp(x[t] - mx) / Z;
+                }
+            }
+        }
+        for (int t = 0; t < Nc; t++) if (was[t]) dk[t] = 0.0;
+        for (int t = 0; t < Nc; t++) acc[t] += decay * dk[t];
+        decay *= p->rho_hop;
+        double sk = 0.0;
+        for (int t = 0; t < Nc; t++) sk += dk[t];
+        for (int t = 0; t < Nc; t++) sc[t] = sk > 0.0 ? dk[t] / sk : 0.0;
+    }
+    /* Eq. (app_diffused_relevance) */
+    double sa = 0.0;
+    for (int t = 0; t < Nc; t++) sa += acc[t];
+    for (int t = 0; t < Nc; t++) dhat[t] = acc[t] / (sa + p->eps);
+    free(S); free(sc); free(dk); free(acc); free(x); free(ord); free(sd); free(w); free(was);
+    return ORC_OK;
+}

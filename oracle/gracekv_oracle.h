@@ -61,6 +61,16 @@
  *   R14 "w/o GA": (l, g) number lg gets the capacity floor(B_free / LG), plus
  *       one for lg < B_free mod LG; the heap pops as before and discards an op
  *       its (l, g) cannot afford; a pair's unused capacity is lost.
+ *   R16 multi-hop relevance (App. A.4): graph layers at relative depths 0.50
+ *       and 0.75 (floor(rho L), duplicates dropped); seeds of a hop = tokens
+ *       of C in order of their score descending (ties: lower t), taken while
+ *       fewer than m_seed are taken and their running mass is below eta_seed
+ *       (the seed that reaches eta is included); hop 1 scores = S-hat (Eq.
+ *       app_global_seed_score), later hops = the previous hop's propagation
+ *       score normalised over C; a hop's seed weights are its scores over
+ *       the seed set, normalised to sum 1 (uniform when they sum to 0); seed u
+ *       attends to [0, u] (its causal visible range); the propagation score
+ *       of a hop is zeroed at that hop's and all earlier seeds.
  *   R15 singleton floor (App. A.5 Stage I, App. C.2): R = the token values
  *       (lambda_graph = 0); the consensus is the mean over all (l, g); the
  *       max-pool window is clipped to the compressible context.  Candidates
@@ -108,6 +118,9 @@ typedef struct {
     double alpha_floor;           /* singleton-floor cap alpha (0: no floor, "w/o SF") */
     double floor_c, floor_gamma, floor_eta;   /* consensus weight, gate, cumulative value */
     int32_t floor_half;           /* max-pool half width (7 = 2 * 3 + 1) */
+    double lambda_graph;          /* multi-hop weight (0: direct relevance only) */
+    double eta_seed, rho_hop;     /* seed mass, inter-hop decay */
+    int32_t m_seed, r_hop;        /* at most m_seed seeds per hop, r_hop hops */
     int32_t seg_mode;             /* 0: curvature DP; 1: uniform slots of target length n0
                                      and curvature 0 (the "w/o CS" ablation, App. B.4 end) */
     int32_t quota_alloc;          /* 0: one shared budget; 1: fixed per-(l, g) capacity
@@ -176,6 +189,16 @@ int orc_gather(const orc_params *p, const double *K, const double *V, const doub
                const uint8_t *add_sel, const uint8_t *split_sel, int64_t cap,
                double *K_out, double *V_out, int32_t *pos, double *log_m,
                int32_t *src_lo, int32_t *src_hi, int64_t *offsets, int64_t *n_entries);
+
+/* Multi-hop relevance, App. A.4 Eqs. (app_global_seed_score),
+ * (app_hop_propagation), (app_diffused_relevance), reading R16.  shat
+ * [L G][N_c] the direct relevance (Eq. app_direct_relevance); Qg
+ * [n_graph][Hq][T][d] the queries of every position at the graph layers
+ * graph_l[]; K [L][G][T][d].  Output dhat [N_c]; seeds [r_hop][m_seed]
+ * (absolute positions, -1 padded) and their weights (nullable). */
+int orc_multihop(const orc_params *p, const double *shat, const double *Qg, const int32_t *graph_l,
+                 int32_t n_graph, const double *K, double *dhat, int32_t *seeds, double *seed_w);
+int orc_graph_layers(const orc_params *p, int32_t *out);
 
 /* Layer-KV-head sensitivity, App. A.4 Eqs. (app_head_sensitivity_raw),
  * (app_head_sensitivity).  W_O [L][D][Hq d] (the output projection of each
