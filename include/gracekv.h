@@ -48,7 +48,7 @@
 extern "C" {
 #endif
 
-#define GRACEKV_ABI_VERSION 3
+#define GRACEKV_ABI_VERSION 4
 
 typedef enum {
     GKV_OK = 0,
@@ -90,7 +90,8 @@ typedef struct {
     int32_t n_windows;
     int32_t k_cand;                /* top-K curvature split candidates (App. B.4); 0..16 */
     double lambda_kappa, lambda_Z, lambda_M, eps, base_frac;
-    double lambda_graph;           /* multi-hop weight: only 0 is built (GKV_EUNSUPPORTED) */
+    double lambda_graph;           /* multi-hop weight (App. A.4; the paper's value 0.3, 0: direct
+                                      relevance only); > 0 needs gracekv_set_graph_queries */
     double alpha_floor;            /* singleton-floor cap alpha (App. A.5 Stage I, Eq. app_floor_cap);
                                       0: no floor (the paper's "w/o SF"); the paper's value is 0.6 */
     /* The paper's ablations (App. B.4 last paragraph, App. C.1); 0 = the method.
@@ -117,6 +118,12 @@ typedef struct {
      * quota_alloc (GKV_EUNSUPPORTED). */
     double floor_c, floor_gamma, floor_eta;
     int32_t floor_half;
+    /* Multi-hop relevance (lambda_graph > 0; App. A.4): seed mass eta_seed
+     * (0.9), at most m_seed seeds per hop (64, at most 64), r_hop hops (2),
+     * inter-hop decay rho_hop (0.5).  Graph layers at relative depths 0.50 and
+     * 0.75.  Needs bf16, d in {64, 128} and N_c <= 131072 (GKV_EUNSUPPORTED). */
+    double eta_seed, rho_hop;
+    int32_t m_seed, r_hop;
 } gkv_params;
 
 /* Fill *p with the paper's defaults; shapes and budget are left zero.  Host only. */
@@ -264,6 +271,19 @@ gkv_status gracekv_export(gracekv_ctx *ctx, int64_t node_cap, int64_t *n_nodes_h
                           int32_t *nchild, int32_t *cost, float *D, float *R, float *U,
                           float *kappa, uint8_t *split_sel, float *row_m, float *row_Z,
                           float *row_ZC, float *rtok, void *stream);
+
+/*
+ * The queries of every position at the graph layers, for the multi-hop
+ * relevance of the next gracekv_build_trees (App. A.4, Eqs.
+ * app_global_seed_score, app_hop_propagation, app_diffused_relevance):
+ * Qg [n_graph][Hq][T][d] bf16 (device; the caller keeps it alive until the
+ * build returns), n_graph = the number of graph layers (the distinct layers
+ * floor(0.50 L) and floor(0.75 L)), in ascending layer order.  The seeds'
+ * rows attend to their causal range [0, u]; the token values become
+ * R = (1 - lambda_graph) s-hat + lambda_graph d-hat.  Errors: GKV_EINVAL,
+ * GKV_ESTATE (lambda_graph = 0).
+ */
+gkv_status gracekv_set_graph_queries(gracekv_ctx *ctx, const void *Qg, int32_t n_graph);
 
 /*
  * Layer-KV-head sensitivity omega (App. A.4, Eqs. app_head_sensitivity_raw,

@@ -96,6 +96,7 @@ gkv_status gracekv_default_params(gkv_params *p) {
     p->eps = 1e-6; p->base_frac = 0.1;
     p->lambda_graph = 0.0; p->alpha_floor = 0.0;
     p->floor_c = 0.5; p->floor_gamma = 1.2; p->floor_eta = 0.95; p->floor_half = 3;   // App. A.5 Stage I
+    p->eta_seed = 0.9; p->rho_hop = 0.5; p->m_seed = 64; p->r_hop = 2;               // App. A.4
     p->ctx_start = 0; p->ctx_end = -1;                 // -1: T
     return GKV_OK;
 }
@@ -158,7 +159,13 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
     if (p.k_cand < 0 || p.k_cand > 16) return GKV_EINVAL;
     if ((p.seg_mode != 0 && p.seg_mode != 1) || (p.quota_alloc != 0 && p.quota_alloc != 1)) return GKV_EINVAL;
     if (!(p.eps > 0) || !(p.base_frac >= 0)) return GKV_EINVAL;
-    if (p.lambda_graph != 0.0) return GKV_EUNSUPPORTED;
+    if (!(p.lambda_graph >= 0.0 && p.lambda_graph <= 1.0)) return GKV_EINVAL;
+    if (p.lambda_graph > 0.0) {
+        if (!(p.eta_seed > 0.0 && p.eta_seed <= 1.0) || p.m_seed < 1 || p.m_seed > 64 || p.r_hop < 1 ||
+            p.r_hop > 8 || !(p.rho_hop >= 0.0))
+            return GKV_EINVAL;
+        if (p.dtype != GKV_BF16 || (p.d != 64 && p.d != 128)) return GKV_EUNSUPPORTED;
+    }
     if (!(p.alpha_floor >= 0.0 && p.alpha_floor <= 1.0)) return GKV_EINVAL;
     if (p.alpha_floor > 0.0) {
         if (!(p.floor_c >= 0.0 && p.floor_c <= 1.0) || !(p.floor_gamma >= 0.0) ||
@@ -181,6 +188,7 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
     int64_t Nc = (int64_t)p.ctx_end - r - p.ctx_start;
     if (Nc < 1) return GKV_EBUDGET;
     if (Nc + 1 + 4096 > 227 * 1024) return GKV_EUNSUPPORTED;   // DP keeps lengths in shared memory
+    if (p.lambda_graph > 0.0 && Nc > gkv::multihop_max_context()) return GKV_EUNSUPPORTED;
 
     gracekv_ctx *x = new (std::nothrow) gracekv_ctx();
     if (!x) return GKV_ENOMEM;
@@ -250,6 +258,14 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
                                           dalloc(x, &w.fl_acc, (size_t)LG * Nc) &&
                                           dalloc(x, &w.fl_head, (size_t)LG * gkv::floor_head_words()) &&
                                           dalloc(x, &w.fl_glob, (size_t)4))) &&
+              (p.lambda_graph <= 0.0 ||
+               (dalloc(x, &w.mh_sc, (size_t)Nc) && dalloc(x, &w.mh_acc, (size_t)Nc) &&
+                dalloc(x, &w.mh_dpart, (size_t)2 * p.Hq * Nc) &&
+                dalloc(x, &w.mh_stat, (size_t)2 * p.Hq * gkv::multihop_chunks(p.T) * 64 * 2) &&
+                dalloc(x, &w.mh_rowmz, (size_t)2 * p.Hq * 64 * 2) && dalloc(x, &w.mh_was, (size_t)Nc) &&
+                dalloc(x, &w.mh_seeds, (size_t)64) && dalloc(x, &w.mh_nseed, (size_t)1) &&
+                dalloc(x, &w.mh_graph_l, (size_t)2) && dalloc(x, &w.mh_w, (size_t)64) &&
+                dalloc(x, &w.mh_red, (size_t)2))) &&
               dalloc(x, &w.hist, (size_t)2048 * (p.quota_alloc ? LG : 1)) &&
               dalloc(x, &w.alloc_state, (size_t)16 + (p.quota_alloc ? (size_t)8 * LG : 0)) && dalloc(x, &w.work, 4) &&
               dalloc(x, &w.pend_hist, 1 << 16) && dalloc(x, &w.pend_cut, 1) && dalloc(x, &w.pend_n, 1) &&
@@ -269,6 +285,16 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
         e = cudaMemcpy(w.qperm, perm.data(), 256 * sizeof(short), cudaMemcpyHostToDevice);
     }
     if (e == cudaSuccess) e = cudaMemset(w.dev_int, 0, 16 * sizeof(int));
+    if (e == cudaSuccess && w.mh_graph_l) {   // graph layers: relative depths 0.50 and 0.75
+        int32_t gl[2];
+        int n = 0;
+        for (double rho : {0.50, 0.75}) {
+            int l = std::min((int)std::floor(rho * p.L), p.L - 1);
+            if (n == 0 || gl[n - 1] != l) gl[n++] = l;
+        }
+        c.mh_ngraph = n;
+        e = cudaMemcpy(w.mh_graph_l, gl, n * sizeof(int32_t), cudaMemcpyHostToDevice);
+    }
     if (e == cudaSuccess) e = gkv::launch_rope_table(c, 0);
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
@@ -561,6 +587,12 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
     }
     c.scored = false;
     int cnt[2];
+    if (e == cudaSuccess && c.p.lambda_graph > 0.0) {   // R = (1 - lambda) s-hat + lambda d-hat
+        if (!c.mh_Qg) return fail(x, GKV_EINVAL, "build_trees: multi-hop relevance needs gracekv_set_graph_queries");
+        c.mh_K = K;
+        gkv::StageTimer tm(c, 2, s);
+        e = gkv::launch_multihop(c, s);
+    }
     if (e == cudaSuccess && c.p.alpha_floor > 0.0) {   // Stage I: needs every (l, g)'s token values
         gkv::StageTimer tm(c, 6, s);
         e = gkv::launch_floor(c, c.J, s);
@@ -579,6 +611,8 @@ gkv_status gracekv_compress_host(gracekv_ctx *x, const void *K, const void *V, c
                                  const float *omega, void *K_out, void *V_out, int32_t *pos, float *log_m,
                                  int32_t *src_lo, int32_t *src_hi, int64_t *offsets, int64_t cap,
                                  int64_t *n_entries_host, void *stream) {
+    if (x && x->c.p.lambda_graph > 0.0)
+        return fail(x, GKV_EUNSUPPORTED, "compress_host: multi-hop relevance needs the device path");
     gkv_status st = ready(x, 0);
     if (st) return st;
     Ctx &c = x->c;
@@ -747,6 +781,17 @@ gkv_status gracekv_allocate(gracekv_ctx *x, int64_t *n_entries_host, void *strea
     c.used = (int64_t)used;
     *n_entries_host = LG * (c.p.T - c.Nc) + c.used;
     c.stage = 3;
+    return GKV_OK;
+}
+
+gkv_status gracekv_set_graph_queries(gracekv_ctx *x, const void *Qg, int32_t n_graph) {
+    if (!x) return GKV_EINVAL;
+    if (x->c.sticky != GKV_OK) return GKV_ESTATE;
+    Ctx &c = x->c;
+    if (c.p.lambda_graph <= 0.0) return fail(x, GKV_ESTATE, "set_graph_queries: lambda_graph is 0");
+    if (!Qg || !al16(Qg)) return fail(x, GKV_EINVAL, "set_graph_queries: null or misaligned Qg");
+    if (n_graph != c.mh_ngraph) return fail(x, GKV_EINVAL, "set_graph_queries: wrong number of graph layers");
+    c.mh_Qg = Qg;
     return GKV_OK;
 }
 

@@ -66,6 +66,14 @@ struct Workspace {
     unsigned long long *fl_head = nullptr;   // [L G][8] per (l, g) selection state
     unsigned long long *fl_glob = nullptr;   // [4] joint cost, kept candidates, floor entries
     uint8_t *u_floor = nullptr;    // [units_cap] slots whose Add is a floor op
+    // multi-hop relevance (lambda_graph > 0)
+    float *mh_sc = nullptr, *mh_acc = nullptr;   // [N_c] seed scores, accumulated propagation
+    float *mh_dpart = nullptr;     // [n_graph Hq][N_c] propagation per (graph layer, head)
+    float *mh_stat = nullptr;      // [n_graph Hq][chunks][64][2] row statistics per chunk
+    float *mh_rowmz = nullptr;     // [n_graph Hq][64][2]
+    uint8_t *mh_was = nullptr;     // [N_c]
+    int32_t *mh_seeds = nullptr, *mh_nseed = nullptr, *mh_graph_l = nullptr;
+    float *mh_w = nullptr, *mh_red = nullptr;
     uint2 *ops = nullptr;          // [node_cap / 2] Split ops built so far: (key bits, node << 1 | cost - 1)
     unsigned int *n_ops = nullptr; // [1] entries of ops
     // per-unit arrays (capacity units_cap), unit id = lg * J + j
@@ -106,6 +114,9 @@ struct Ctx {
     int n_chunks = 0;              // pass-A chunks per row
     // measurement
     int64_t launches = 0;          // kernels launched (host count)
+    const void *mh_Qg = nullptr;   // graph layers' queries of the next build (multi-hop relevance)
+    const void *mh_K = nullptr;    // the keys of the build in progress
+    int mh_ngraph = 0;
     int build_passes = 1;          // unit-kernel launches of the last build (pruning passes)
     // score passes issued ahead by gracekv_score (consumed by the next build);
     // requested before a segmentation, they are enqueued when its dynamic
@@ -301,6 +312,10 @@ cudaError_t launch_pend_cut(Ctx &c, int J, int m, float *cut, unsigned int *n_qu
 cudaError_t launch_allocate(Ctx &c, int J, cudaStream_t s);
 // singleton floor (floor.cu): candidates, cap and accepted positions of every (l, g)
 cudaError_t launch_floor(Ctx &c, int J, cudaStream_t s);
+// multi-hop relevance (relevance.cu): d-hat mixed into the token values
+cudaError_t launch_multihop(Ctx &c, cudaStream_t s);
+int multihop_chunks(int T);
+int multihop_max_context();
 int floor_head_words();
 cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *slots, int J,
                           void *K_out, void *V_out, int32_t *pos, float *log_m,

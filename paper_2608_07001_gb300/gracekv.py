@@ -40,6 +40,7 @@ class GkvParams(C.Structure):
         ("seg_mode", C.c_int32), ("quota_alloc", C.c_int32),
         ("floor_c", C.c_double), ("floor_gamma", C.c_double), ("floor_eta", C.c_double),
         ("floor_half", C.c_int32),
+        ("eta_seed", C.c_double), ("rho_hop", C.c_double), ("m_seed", C.c_int32), ("r_hop", C.c_int32),
     ]
 
 
@@ -64,7 +65,8 @@ EXPORTED = ["gracekv_default_params", "gracekv_budget_for_ratio", "gracekv_creat
             "gracekv_destroy", "gracekv_last_error", "gracekv_status_string", "gracekv_query",
             "gracekv_segment", "gracekv_score", "gracekv_build_trees", "gracekv_allocate", "gracekv_gather",
             "gracekv_export", "gracekv_profile", "gracekv_stats", "gracekv_row_stats_noalloc",
-            "gracekv_compress_host", "gracekv_export_floor", "gracekv_head_sensitivity", "gracekv_decode_workspace_size", "gracekv_decode_append",
+            "gracekv_compress_host", "gracekv_export_floor", "gracekv_head_sensitivity",
+            "gracekv_set_graph_queries", "gracekv_decode_workspace_size", "gracekv_decode_append",
             "gracekv_decode_attention", "gracekv_decode_status"]
 
 
@@ -96,6 +98,7 @@ def lib() -> C.CDLL:
     L.gracekv_gather.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, i64, vp]
     L.gracekv_export.argtypes = [vp, i64, C.POINTER(i64)] + [vp] * 18 + [vp]
     L.gracekv_export_floor.argtypes = [vp, vp, vp, C.POINTER(i64), vp]
+    L.gracekv_set_graph_queries.argtypes = [vp, vp, i32]
     L.gracekv_head_sensitivity.argtypes = [vp, vp] + [i32] * 7 + [vp, vp, vp]
     L.gracekv_profile.argtypes = [vp, i32]
     L.gracekv_stats.argtypes = [vp, vp, i32, C.POINTER(i64), vp, i32]
@@ -256,6 +259,11 @@ class Context:
 
     STAGES = ("segment", "row_stats", "token_values", "unit_trees", "allocate", "gather", "floor")
 
+    def gracekv_set_graph_queries(self, Qg):
+        """Qg [n_graph, Hq, T, d] bf16: queries of every position at the graph layers."""
+        self._check(lib().gracekv_set_graph_queries(self.h, _ptr(Qg), Qg.shape[0]))
+        self._Qg = Qg
+
     def gracekv_export_floor(self, stream=None) -> dict:
         """The singleton floor of the last tree build (host arrays)."""
         import numpy as np
@@ -358,8 +366,10 @@ class Compressor:
         self._side = None
 
     def __call__(self, K, V, Q, omega=None, hidden=None, surprisal=None, slot_starts=None,
-                 stream=None) -> "Cache":
+                 stream=None, Qg=None) -> "Cache":
         c = self.ctx
+        if Qg is not None:          # multi-hop relevance: the graph layers' queries
+            c.gracekv_set_graph_queries(Qg)
         # the score passes (K, Q only) run on a second stream while the
         # segmentation runs; the tree build waits for them
         main = stream if stream is not None else torch.cuda.current_stream()

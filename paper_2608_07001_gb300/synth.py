@@ -56,7 +56,7 @@ import numpy as np
 import torch
 
 __all__ = ["Workload", "WORKLOADS", "Inputs", "make_inputs", "segment_lengths",
-           "supplied_slots", "DecodeCache", "make_decode_cache"]
+           "supplied_slots", "DecodeCache", "make_decode_cache", "make_graph_queries"]
 
 
 @dataclasses.dataclass(frozen=True)
@@ -310,3 +310,20 @@ def make_decode_cache(w: Workload, ratio: int, n_app: int = 0, app_cap: Optional
     return DecodeCache(q.to(tdt), K.to(tdt), V.to(tdt),
                        torch.as_tensor(logm, dtype=torch.float32, device=device),
                        torch.as_tensor(off, device=device), Ka.to(tdt), Va.to(tdt), n_app)
+
+
+def make_graph_queries(w: Workload, graph_layers: Sequence[int], T: Optional[int] = None,
+                       device="cpu", heads: Optional[Sequence[int]] = None) -> torch.Tensor:
+    """Queries of every position at the graph layers, [n_graph, Hq', T, d]:
+    N(0, 1) per channel, rotated like the keys (the position's RoPE angle), so
+    that a seed's attention over its past carries the keys' structure."""
+    T = w.T if T is None else int(T)
+    heads = tuple(range(w.Hq)) if heads is None else tuple(int(h) for h in heads)
+    tdt = torch.float32 if w.dtype == "f32" else torch.bfloat16
+    out = torch.empty(len(graph_layers), len(heads), T, w.d, dtype=tdt, device=device)
+    for gi, l in enumerate(graph_layers):
+        for hi, h in enumerate(heads):
+            gen = _stream(w.seed, 3_000_001, l, h, device=device)
+            q = torch.randn(T, w.d, generator=gen, device=device, dtype=torch.float64)
+            out[gi, hi] = _rotate_like_rope_model(q, w.rope_base).to(tdt)
+    return out

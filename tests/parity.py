@@ -42,7 +42,7 @@ LOGM_ATOL = 1e-4
 
 
 def run_gpu(K, V, Q, B, rope_base, *, ctx_start=0, ctx_end=None, omega=None, hidden=None,
-            surprisal=None, slot_starts=None, **ov):
+            surprisal=None, slot_starts=None, Qg=None, **ov):
     L, G, T, d = K.shape
     Hq, W = Q.shape[1], Q.shape[2]
     p = gk.make_params(L, G, Hq, T, d, W, dtype=K.dtype, budget=B, rope_base=rope_base,
@@ -56,7 +56,8 @@ def run_gpu(K, V, Q, B, rope_base, *, ctx_start=0, ctx_end=None, omega=None, hid
     ss = None
     if slot_starts is not None:
         ss = dev(torch.as_tensor(np.asarray(slot_starts) + ctx_start, dtype=torch.int32))
-    cache = comp(Kc, Vc, Qc, omega=om, hidden=hid, surprisal=sur, slot_starts=ss)
+    cache = comp(Kc, Vc, Qc, omega=om, hidden=hid, surprisal=sur, slot_starts=ss,
+                 Qg=None if Qg is None else dev(Qg))
     torch.cuda.synchronize()
     ex = comp.ctx.gracekv_export()
     E = comp.n_entries
@@ -70,9 +71,9 @@ def run_gpu(K, V, Q, B, rope_base, *, ctx_start=0, ctx_end=None, omega=None, hid
 
 
 def run_oracle(K, V, Q, B, rope_base, *, ctx_start=0, ctx_end=None, omega=None, hidden=None,
-               surprisal=None, slot_starts=None, **ov):
+               surprisal=None, slot_starts=None, Qg=None, **ov):
     return O.run(K, V, Q, B, rope_base, ctx_start=ctx_start, ctx_end=ctx_end, omega=omega,
-                 hidden=hidden, surprisal=surprisal, slot_starts=slot_starts, **ov)
+                 hidden=hidden, surprisal=surprisal, slot_starts=slot_starts, Qg=Qg, **ov)
 
 
 def oracle_tau(o, lg=None):

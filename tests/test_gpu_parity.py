@@ -145,6 +145,30 @@ def test_head_sensitivity_matches_the_oracle(L, G, gq, d, D, U):
     np.testing.assert_allclose(om, ref, rtol=1e-4, atol=1e-6)
 
 
+@pytest.mark.parametrize("m_seed", [64, 8])
+def test_multihop_relevance_matches_the_oracle(m_seed):
+    # App. A.4: seeds from the global seed score, two hops of causal seed
+    # attention at the graph layers, R = 0.7 s-hat + 0.3 d-hat; then the trees,
+    # selection and cache of the pass against the oracle
+    import oracle as O
+    w = synth.WORKLOADS["small"]
+    x = synth.make_inputs(w, layers=[0, 1, 2, 3], heads=[0, 1], T=1000)
+    L, G, T, d = x.K.shape
+    p = O.make_params(L, G, x.Q.shape[1], T, d, x.Q.shape[2], w.rope_base, recent=32)
+    gl = O.graph_layers(p)
+    Qg = synth.make_graph_queries(w, [int(l) for l in gl], T=T, heads=range(x.Q.shape[1]))
+    B = (L * G * T) // 8
+    P, g, o = _run(x.K, x.V, x.Q, B, w.rope_base, Qg=Qg, lambda_graph=0.3, m_seed=m_seed)
+    ex = g["export"]
+    mh = o["multihop"]
+    rt = np.asarray(ex["rtok"]).reshape(o["rtok"].shape)
+    err = np.abs(rt - o["rtok"]).max() / np.abs(o["rtok"]).max()
+    print("multihop seeds", [int(v) for v in mh["seeds"][0][:8]], "rtok rel err", err)
+    assert err < 1e-4
+    rep = P.compare(g, o, torch.bfloat16)
+    print("multihop", json.dumps(rep))
+
+
 def test_fullkv_identity_is_bit_exact():
     # x = 1: every tree expands to its leaves; the cache is the input (App. C.5)
     w = synth.WORKLOADS["pr1"]
