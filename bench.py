@@ -298,6 +298,10 @@ def main():
                     help="time only the layer-KV-head sensitivity on the workload's shape")
     ap.add_argument("--alpha-floor", type=float, default=None,
                     help="singleton-floor cap alpha (the library default when omitted)")
+    ap.add_argument("--lambda-graph", type=float, default=0.0,
+                    help="multi-hop relevance weight lambda (0: the four-stage pass alone); "
+                         "graph-layer queries are synthesised on the device, and the "
+                         "host-buffer pass, which takes no graph queries, is not timed")
     ap.add_argument("--ablation", default="none", choices=["none", "wo_cs", "wo_ga"],
                     help="the paper's w/o CS (uniform slots, midpoint cuts) or w/o GA "
                          "(fixed per-(l, g) capacity) variant")
@@ -332,6 +336,11 @@ def main():
            "wo_ga": dict(quota_alloc=1)}[args.ablation]
     if args.alpha_floor is not None:
         abl = dict(abl, alpha_floor=args.alpha_floor)
+    Qg = None
+    if args.lambda_graph > 0:
+        abl = dict(abl, lambda_graph=args.lambda_graph)
+        args.no_e2e = True
+        Qg = synth.make_graph_queries(w, gk.graph_layers(K.shape[0]), device=dev)
     p = gk.make_params(L, G, Q.shape[1], T, d, Q.shape[2], dtype=K.dtype, budget=B,
                        rope_base=w.rope_base, **abl)
     comp = gk.Compressor(p, device=dev)
@@ -343,7 +352,7 @@ def main():
         torch.cuda.synchronize(dev)
 
     if args.decode_only:
-        comp(K, V, Q)
+        comp(K, V, Q, Qg=Qg)
         torch.cuda.synchronize(dev)
         dec = decode_leg(args, w, comp, L, G, Q.shape[1], d, dev)
         if rank == 0:
@@ -351,7 +360,7 @@ def main():
         return
 
     for _ in range(args.warmup):
-        comp(K, V, Q)
+        comp(K, V, Q, Qg=Qg)
     comp.ctx.gracekv_profile(True)
     comp.ctx.gracekv_stats()
     _, launches0, _ = comp.ctx.gracekv_stats()
@@ -363,7 +372,7 @@ def main():
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for _ in range(args.steps):
-        comp(K, V, Q)
+        comp(K, V, Q, Qg=Qg)
     e1.record(stream)
     barrier()
     clocks = clk.stop()
@@ -458,7 +467,7 @@ def main():
                "dtype": "bf16" if K.dtype == torch.bfloat16 else "f32", "data": "synthetic",
                "config": dict(workload_config(w, args.ratio, L), B_total=B, entries=E,
                               slots=comp.n_slots, parallelism=f"replicas{world}",
-                              alpha_floor=p.alpha_floor,
+                              alpha_floor=p.alpha_floor, lambda_graph=p.lambda_graph,
                               **({"ablation": args.ablation} if args.ablation != "none" else {})),
                "roofline": roof, "hbm_pass": hbm, "stages_ms": per_step, "tree_work": work,
                "cpu_baseline": cpu, "e2e": e2e,

@@ -133,6 +133,12 @@ gkv_status gracekv_default_params(gkv_params *p);
  * (App. A.1 Eq. app_total_budget).  Returns -1 for invalid arguments.  Host only. */
 int64_t gracekv_budget_for_ratio(int32_t L, int32_t G, int32_t n_ctx, double x);
 
+/* The graph layers of the multi-hop relevance (App. A.4): the distinct
+ * layers floor(0.50 L) and floor(0.75 L) (each at most L - 1), ascending,
+ * written to out[0 .. n-1] (nullable; room for 2).  Returns n (1 or 2), or -1
+ * for L <= 0.  Host only. */
+int32_t gracekv_graph_layers(int32_t L, int32_t *out);
+
 /* Validate *p, resolve the recent window against the budget (r = 32, shrunk to
  * floor(B_total / (L G)) when L G r > B_total, never below 4: App. A.1) and
  * allocate the device workspace on the current device.  On success *out owns
@@ -317,8 +323,9 @@ gkv_status gracekv_export_floor(gracekv_ctx *ctx, uint8_t *accepted, float *f, i
  * Measurement support (not needed to compress).  gracekv_profile(ctx, 1)
  * makes every later stage call record CUDA events on its stream around each
  * kernel group: 0 segmentation, 1 row statistics, 2 token values, 3 unit
- * trees, 4 allocation, 5 gather, 6 singleton floor.  gracekv_stats synchronises the events of
- * the calls made since the last gracekv_stats / gracekv_profile and returns
+ * trees, 4 allocation, 5 gather, 6 singleton floor, 7 multi-hop relevance.
+ * gracekv_stats synchronises the events of the calls made since the last
+ * gracekv_stats / gracekv_profile and returns
  * the summed milliseconds per group in stage_ms[0 .. n_stages-1] (nullable);
  * *launches (nullable) receives the number of kernels this context has
  * launched since it was created; work[0 .. n_work-1] (nullable) receives the
@@ -326,7 +333,7 @@ gkv_status gracekv_export_floor(gracekv_ctx *ctx, uint8_t *accepted, float *f, i
  * steps, [1] candidate intervals evaluated, [2] sum of candidate lengths,
  * [3] units built.
  */
-#define GRACEKV_N_STAGES 7
+#define GRACEKV_N_STAGES 8
 gkv_status gracekv_profile(gracekv_ctx *ctx, int32_t enable);
 gkv_status gracekv_stats(gracekv_ctx *ctx, float *stage_ms, int32_t n_stages, int64_t *launches,
                          uint64_t *work, int32_t n_work);

@@ -108,6 +108,19 @@ int64_t gracekv_budget_for_ratio(int32_t L, int32_t G, int32_t n_ctx, double x) 
     return (int64_t)std::floor(n / x);
 }
 
+int32_t gracekv_graph_layers(int32_t L, int32_t *out) {
+    if (L <= 0) return -1;
+    int32_t gl[2];
+    int32_t n = 0;
+    for (double rho : {0.50, 0.75}) {   // relative depths of the graph layers (App. A.4)
+        int32_t l = std::min((int32_t)std::floor(rho * L), L - 1);
+        if (n == 0 || gl[n - 1] != l) gl[n++] = l;
+    }
+    if (out)
+        for (int32_t k = 0; k < n; k++) out[k] = gl[k];
+    return n;
+}
+
 const char *gracekv_status_string(gkv_status s) {
     switch (s) {
         case GKV_OK: return "ok";
@@ -265,7 +278,8 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
                 dalloc(x, &w.mh_rowmz, (size_t)2 * p.Hq * 64 * 2) && dalloc(x, &w.mh_was, (size_t)Nc) &&
                 dalloc(x, &w.mh_seeds, (size_t)64) && dalloc(x, &w.mh_nseed, (size_t)1) &&
                 dalloc(x, &w.mh_graph_l, (size_t)2) && dalloc(x, &w.mh_w, (size_t)64) &&
-                dalloc(x, &w.mh_red, (size_t)2))) &&
+                dalloc(x, &w.mh_red, (size_t)2) && dalloc(x, &w.mh_pkeys, (size_t)64 * 64) &&
+                dalloc(x, &w.mh_psum, (size_t)64))) &&
               dalloc(x, &w.hist, (size_t)2048 * (p.quota_alloc ? LG : 1)) &&
               dalloc(x, &w.alloc_state, (size_t)16 + (p.quota_alloc ? (size_t)8 * LG : 0)) && dalloc(x, &w.work, 4) &&
               dalloc(x, &w.pend_hist, 1 << 16) && dalloc(x, &w.pend_cut, 1) && dalloc(x, &w.pend_n, 1) &&
@@ -285,13 +299,9 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
         e = cudaMemcpy(w.qperm, perm.data(), 256 * sizeof(short), cudaMemcpyHostToDevice);
     }
     if (e == cudaSuccess) e = cudaMemset(w.dev_int, 0, 16 * sizeof(int));
-    if (e == cudaSuccess && w.mh_graph_l) {   // graph layers: relative depths 0.50 and 0.75
+    if (e == cudaSuccess && w.mh_graph_l) {
         int32_t gl[2];
-        int n = 0;
-        for (double rho : {0.50, 0.75}) {
-            int l = std::min((int)std::floor(rho * p.L), p.L - 1);
-            if (n == 0 || gl[n - 1] != l) gl[n++] = l;
-        }
+        int n = gracekv_graph_layers(p.L, gl);
         c.mh_ngraph = n;
         e = cudaMemcpy(w.mh_graph_l, gl, n * sizeof(int32_t), cudaMemcpyHostToDevice);
     }
@@ -590,7 +600,7 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
     if (e == cudaSuccess && c.p.lambda_graph > 0.0) {   // R = (1 - lambda) s-hat + lambda d-hat
         if (!c.mh_Qg) return fail(x, GKV_EINVAL, "build_trees: multi-hop relevance needs gracekv_set_graph_queries");
         c.mh_K = K;
-        gkv::StageTimer tm(c, 2, s);
+        gkv::StageTimer tm(c, 7, s);
         e = gkv::launch_multihop(c, s);
     }
     if (e == cudaSuccess && c.p.alpha_floor > 0.0) {   // Stage I: needs every (l, g)'s token values

@@ -74,6 +74,8 @@ struct Workspace {
     uint8_t *mh_was = nullptr;     // [N_c]
     int32_t *mh_seeds = nullptr, *mh_nseed = nullptr, *mh_graph_l = nullptr;
     float *mh_w = nullptr, *mh_red = nullptr;
+    uint64_t *mh_pkeys = nullptr;  // [N_c / 2048][64] seed candidates of every part
+    float *mh_psum = nullptr;      // [N_c / 2048] score sums of every part
     uint2 *ops = nullptr;          // [node_cap / 2] Split ops built so far: (key bits, node << 1 | cost - 1)
     unsigned int *n_ops = nullptr; // [1] entries of ops
     // per-unit arrays (capacity units_cap), unit id = lg * J + j

@@ -47,6 +47,8 @@ struct MhArgs {
     float *rowmz;                   // [n_graph Hq][64][2]
     uint8_t *was;                   // [N_c] seeds of this or an earlier hop
     int32_t *seeds;                 // [64] C-relative positions
+    uint64_t *pkeys;                // [parts][64] the best keys of every part
+    float *psum;                    // [parts] score sums
     float *w;                       // [64]
     int *nseed;
     float *red;                     // [2] scratch sums
@@ -76,71 +78,114 @@ __global__ void mh_mean_kernel(MhArgs a) {
     a.was[t] = 0;
 }
 
-// One CTA: the hop's seeds (iterative block argmax; ties: lower t).  hop1:
-// the scores are S (normalised with eps, Eq. app_global_seed_score), else a
-// propagation score (normalised by its sum).
-constexpr int kMhMaxNc = 4096 * 32;       // context tokens the seed bitmap holds
-__global__ void __launch_bounds__(1024) mh_seeds_kernel(MhArgs a, int hop1) {
-    __shared__ float wv[32];
-    __shared__ int wt[32];
-    __shared__ float tot_s;
-    __shared__ int pick;
-    __shared__ uint32_t taken[kMhMaxNc / 32];
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    for (int k = tid; k < (a.Nc + 31) / 32; k += 1024) taken[k] = 0u;
-    float part = 0.f;
-    for (int t = tid; t < a.Nc; t += 1024) part += a.sc[t];
-    part = warp_sum(part);
-    if (lane == 0) wv[warp] = part;
+// The seeds come from a top-64 selection: the order "score descending, ties
+// lower t" is the descending order of the 64-bit key (order-preserving bits
+// of the score) << 32 | ~t, so the first m_seed keys of the sorted context
+// are the seeds that m_seed successive argmax picks would give.  A part
+// kernel sorts 2048-token chunks in shared memory (bitonic) and keeps each
+// chunk's best 64 and its score sum; one CTA sorts the survivors and applies
+// the mass rule to the head of the list.
+constexpr int kMhMaxNc = 4096 * 32;       // context tokens (N_c) the selection supports
+constexpr int kMhPart = 2048;             // tokens per part CTA
+constexpr int kMhMaxParts = kMhMaxNc / kMhPart;
+constexpr int kMhTop = 64;                // survivors per part (>= m_seed)
+static_assert(kMhMaxParts * kMhTop == 64 * 64, "workspace sizes of the seed candidates");
+
+__device__ __forceinline__ uint64_t mh_key(float v, int t) {
+    uint32_t b = __float_as_uint(v);
+    b = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+    return ((uint64_t)b << 32) | (uint32_t)(~(uint32_t)t);
+}
+__device__ __forceinline__ float mh_key_value(uint64_t k) {
+    uint32_t b = (uint32_t)(k >> 32);
+    b = (b & 0x80000000u) ? (b & 0x7fffffffu) : ~b;
+    return __uint_as_float(b);
+}
+
+// Descending bitonic sort of n (a power of two) keys in shared memory by the
+// whole block; ends with a barrier.
+__device__ void mh_bitonic_desc(uint64_t *x, int n) {
+    for (int k = 2; k <= n; k <<= 1)
+        for (int j = k >> 1; j > 0; j >>= 1) {
+            for (int i = threadIdx.x; i < n / 2; i += blockDim.x) {
+                const int lo = 2 * i - (i & (j - 1)), hi = lo + j;
+                const uint64_t p = x[lo], q = x[hi];
+                if ((p < q) == ((lo & k) == 0)) { x[lo] = q; x[hi] = p; }
+            }
+            __syncthreads();
+        }
+}
+
+// Block sum in a fixed order (warp shuffles, then the warps in order).
+__device__ float mh_block_sum(float v, float *wv) {
+    v = warp_sum(v);
+    if ((threadIdx.x & 31) == 0) wv[threadIdx.x >> 5] = v;
     __syncthreads();
-    if (tid == 0) {
+    float s = 0.f;
+    for (int k = 0; k < (int)(blockDim.x >> 5); k++) s += wv[k];
+    __syncthreads();
+    return s;
+}
+
+__global__ void __launch_bounds__(1024) mh_top_part_kernel(MhArgs a) {
+    __shared__ uint64_t key[kMhPart];
+    __shared__ float wv[32];
+    const int t0 = blockIdx.x * kMhPart;
+    float part = 0.f;
+    for (int i = threadIdx.x; i < kMhPart; i += 1024) {
+        const int t = t0 + i;
+        uint64_t k = 0;                               // below every token's key
+        if (t < a.Nc) {
+            const float v = a.sc[t];
+            part += v;
+            k = mh_key(v, t);
+        }
+        key[i] = k;
+    }
+    const float tot = mh_block_sum(part, wv);
+    mh_bitonic_desc(key, kMhPart);
+    if (threadIdx.x < kMhTop) a.pkeys[(size_t)blockIdx.x * kMhTop + threadIdx.x] = key[threadIdx.x];
+    if (threadIdx.x == 0) a.psum[blockIdx.x] = tot;
+}
+
+// One CTA: the hop's seeds.  hop1: the scores are S (normalised with eps,
+// Eq. app_global_seed_score), else a propagation score (normalised by its
+// sum).  Seeds are taken while fewer than m_seed are taken and the running
+// mass is below eta_seed.
+__global__ void __launch_bounds__(1024) mh_seeds_kernel(MhArgs a, int n_parts, int hop1) {
+    __shared__ uint64_t key[kMhMaxParts * kMhTop];
+    __shared__ float tot_s;
+    __shared__ int n_s;
+    int n = kMhTop;
+    while (n < n_parts * kMhTop) n <<= 1;
+    for (int i = threadIdx.x; i < n; i += 1024) key[i] = i < n_parts * kMhTop ? a.pkeys[i] : 0ull;
+    if (threadIdx.x == 0) {
         float s = 0.f;
-        for (int k = 0; k < 32; k++) s += wv[k];
+        for (int p = 0; p < n_parts; p++) s += a.psum[p];
         tot_s = s;
     }
     __syncthreads();
-    const float tot = tot_s;
-    const float inv = hop1 ? 1.f / (tot + a.eps) : (tot > 0.f ? 1.f / tot : 0.f);
-    float cum = 0.f, wsum = 0.f;
-    int n = 0;
-    while (n < a.m_seed && n < a.Nc && cum < a.eta) {
-        float bv = -INFINITY;
-        int bt = 0x7fffffff;
-        for (int t = tid; t < a.Nc; t += 1024) {
-            if ((taken[t >> 5] >> (t & 31)) & 1u) continue;
-            const float v = a.sc[t];
-            if (v > bv || (v == bv && t < bt)) { bv = v; bt = t; }
+    mh_bitonic_desc(key, n);
+    if (threadIdx.x == 0) {
+        const float tot = tot_s;
+        const float inv = hop1 ? 1.f / (tot + a.eps) : (tot > 0.f ? 1.f / tot : 0.f);
+        float cum = 0.f, wsum = 0.f;
+        int m = 0;
+        while (m < a.m_seed && m < a.Nc && cum < a.eta) {
+            const uint64_t k = key[m];
+            const float v = mh_key_value(k);
+            a.seeds[m] = (int)(~(uint32_t)k);
+            a.w[m] = v;
+            cum += v * inv;
+            wsum += v;
+            m++;
         }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const float v2 = __shfl_xor_sync(0xffffffffu, bv, o);
-            const int t2 = __shfl_xor_sync(0xffffffffu, bt, o);
-            if (v2 > bv || (v2 == bv && t2 < bt)) { bv = v2; bt = t2; }
-        }
-        if (lane == 0) { wv[warp] = bv; wt[warp] = bt; }
-        __syncthreads();
-        if (tid == 0) {
-            float v = wv[0];
-            int t = wt[0];
-            for (int k = 1; k < 32; k++)
-                if (wv[k] > v || (wv[k] == v && wt[k] < t)) { v = wv[k]; t = wt[k]; }
-            pick = t;
-            taken[t >> 5] |= 1u << (t & 31);
-            a.seeds[n] = t;
-            a.w[n] = v;
-        }
-        __syncthreads();
-        const float v = a.sc[pick];
-        cum += v * inv;
-        wsum += v;
-        n++;
+        for (int k = 0; k < m; k++) a.w[k] = wsum > 0.f ? a.w[k] / wsum : 1.f / m;
+        *a.nseed = m;
+        n_s = m;
     }
     __syncthreads();
-    if (tid < n) {
-        a.w[tid] = wsum > 0.f ? a.w[tid] / wsum : 1.f / n;
-        a.was[a.seeds[tid]] = 1;
-    }
-    if (tid == 0) *a.nseed = n;
+    if (threadIdx.x < n_s) a.was[a.seeds[threadIdx.x]] = 1;
 }
 
 // Logit tiles of the seed rows of (graph layer gi, query head h) against the
@@ -385,14 +430,17 @@ cudaError_t launch_multihop(Ctx &c, cudaStream_t s) {
     a.eps = (float)p.eps;
     a.rtok = w.rtok; a.sc = w.mh_sc; a.acc = w.mh_acc; a.dpart = w.mh_dpart; a.stat = w.mh_stat;
     a.rowmz = w.mh_rowmz; a.was = w.mh_was; a.seeds = w.mh_seeds; a.w = w.mh_w; a.nseed = w.mh_nseed;
+    a.pkeys = w.mh_pkeys; a.psum = w.mh_psum;
     a.red = w.mh_red;
     mh_mean_kernel<<<(a.Nc + 255) / 256, 256, 0, s>>>(a);
     c.launches += 1;
     float decay = 1.f;
     const int GH = a.n_graph * a.Hq;
     const int nc_ctx = (a.Nc + kMhChunk - 1) / kMhChunk;
+    const int n_parts = (a.Nc + kMhPart - 1) / kMhPart;
     for (int k = 0; k < p.r_hop; k++) {
-        mh_seeds_kernel<<<1, 1024, 0, s>>>(a, k == 0);
+        mh_top_part_kernel<<<n_parts, 1024, 0, s>>>(a);
+        mh_seeds_kernel<<<1, 1024, 0, s>>>(a, n_parts, k == 0);
         cudaError_t e = p.d == 128 ? launch_mh_tile<128, 0>(a, dim3(a.n_chunks, GH), s)
                                    : launch_mh_tile<64, 0>(a, dim3(a.n_chunks, GH), s);
         if (e != cudaSuccess) return e;
@@ -401,7 +449,7 @@ cudaError_t launch_multihop(Ctx &c, cudaStream_t s) {
         if (e != cudaSuccess) return e;
         mh_reduce_kernel<<<(a.Nc + 255) / 256, 256, 0, s>>>(a, decay);
         decay *= (float)p.rho_hop;
-        c.launches += 5;
+        c.launches += 6;
     }
     mh_total_kernel<<<1, 1024, 0, s>>>(a);
     const size_t n = (size_t)p.L * p.G * a.Nc;

@@ -61,7 +61,8 @@ class GraceKVError(RuntimeError):
 
 _lib = None
 
-EXPORTED = ["gracekv_default_params", "gracekv_budget_for_ratio", "gracekv_create",
+EXPORTED = ["gracekv_default_params", "gracekv_budget_for_ratio", "gracekv_graph_layers",
+            "gracekv_create",
             "gracekv_destroy", "gracekv_last_error", "gracekv_status_string", "gracekv_query",
             "gracekv_segment", "gracekv_score", "gracekv_build_trees", "gracekv_allocate", "gracekv_gather",
             "gracekv_export", "gracekv_profile", "gracekv_stats", "gracekv_row_stats_noalloc",
@@ -82,6 +83,8 @@ def lib() -> C.CDLL:
     L.gracekv_default_params.argtypes = [C.POINTER(GkvParams)]
     L.gracekv_budget_for_ratio.argtypes = [i32, i32, i32, C.c_double]
     L.gracekv_budget_for_ratio.restype = i64
+    L.gracekv_graph_layers.argtypes = [i32, C.POINTER(i32)]
+    L.gracekv_graph_layers.restype = i32
     L.gracekv_create.argtypes = [C.POINTER(GkvParams), C.POINTER(vp)]
     L.gracekv_destroy.argtypes = [vp]
     L.gracekv_destroy.restype = None
@@ -120,6 +123,18 @@ def gracekv_default_params() -> GkvParams:
 
 def gracekv_budget_for_ratio(L: int, G: int, n_ctx: int, x: float) -> int:
     return int(lib().gracekv_budget_for_ratio(L, G, n_ctx, float(x)))
+
+
+def gracekv_graph_layers(L: int) -> list:
+    """The multi-hop relevance's graph layers for an L-layer model."""
+    out = (C.c_int32 * 2)()
+    n = int(lib().gracekv_graph_layers(int(L), out))
+    if n < 0:
+        _raise(GKV_EINVAL)
+    return [int(out[k]) for k in range(n)]
+
+
+graph_layers = gracekv_graph_layers
 
 
 def gracekv_row_stats_noalloc(K, Q, c_lo: int, c_hi: int, row_m, row_Z, row_ZC, stream=None):
@@ -257,7 +272,8 @@ class Context:
                                          _ptr(out.src_hi), _ptr(out.offsets), out.K.shape[0],
                                          _stream(stream)))
 
-    STAGES = ("segment", "row_stats", "token_values", "unit_trees", "allocate", "gather", "floor")
+    STAGES = ("segment", "row_stats", "token_values", "unit_trees", "allocate", "gather", "floor",
+              "multihop")
 
     def gracekv_set_graph_queries(self, Qg):
         """Qg [n_graph, Hq, T, d] bf16: queries of every position at the graph layers."""

@@ -52,6 +52,15 @@ def test_budget_for_ratio(gk):
     assert gk.gracekv_budget_for_ratio(1, 2, 1024, 0.5) == -1
 
 
+def test_graph_layers_match_the_oracle(gk, oracle_lib):
+    # the library's host rule for the multi-hop graph layers against the oracle's
+    import oracle as O
+    for L in range(1, 65):
+        p = O.make_params(L, 1, 1, 64, 8, 2, 0.0, recent=8)
+        assert gk.gracekv_graph_layers(L) == [int(v) for v in O.graph_layers(p)]
+    assert gk.lib().gracekv_graph_layers(0, None) == -1
+
+
 def _create(gk, **kw):
     base = dict(L=1, G=2, Hq=2, T=1024, d=128, W=32)
     base.update({k: kw.pop(k) for k in list(kw) if k in base})
