@@ -72,7 +72,8 @@
  *       attends to [0, u] (its causal visible range); the propagation score
  *       of a hop is zeroed at that hop's and all earlier seeds.
  *   R15 singleton floor (App. A.5 Stage I, App. C.2): R = the token values
- *       (lambda_graph = 0); the consensus is the mean over all (l, g); the
+ *       after the multi-hop mix (the direct ones when lambda_graph = 0); the
+ *       consensus is the mean over all (l, g); the
  *       max-pool window is clipped to the compressible context.  Candidates
  *       of an (l, g): f descending (ties: lower t), while f >= gamma / N_c,
  *       stopping before the running sum of R would exceed eta.  Joint cost

@@ -21,6 +21,11 @@ outputs the oracle computes one by one, and by properties that hold at any size:
                  op, tree consistency of the selected splits, entry count
   gather         the group's entries partition its covered slots; 256 sampled
                  entries equal the oracle's prototype of the same interval
+  multi-hop      a second compression with lambda = 0.3 (App. A.4): the
+                 implied d-hat is the same for every (l, g), non-negative, sums
+                 to 1 and is exactly zero at the first hop's seeds, chosen on
+                 the host in fp64 from the direct token values (64 merged
+                 selection parts, the last one ragged)
 """
 from __future__ import annotations
 
@@ -288,3 +293,50 @@ def test_gather_of_one_group(run):
     print(f"prototypes K {worst_k:.3e} V {worst_v:.3e} log m {worst_m:.3e}")
     assert worst_k <= P.PROTO_RTOL[torch.bfloat16] and worst_v <= P.PROTO_RTOL[torch.bfloat16]
     assert worst_m <= P.LOGM_ATOL
+
+
+def test_multihop_full_size_properties(run):
+    from paper_2608_07001_gb300 import gracekv as gk
+    w = run["w"]
+    L, G, T, d, Hq, W, Nc = (run[k] for k in ("L", "G", "T", "d", "Hq", "W", "Nc"))
+    lam = 0.3
+    x = synth.make_inputs(w, device="cuda")
+    Qg = synth.make_graph_queries(w, gk.graph_layers(L), device="cuda")
+    p = gk.make_params(L, G, Hq, T, d, W, dtype=x.K.dtype, budget=run["B"], rope_base=w.rope_base,
+                       lambda_graph=lam)
+    comp = gk.Compressor(p)
+    comp(x.K, x.V, x.Q, Qg=Qg)
+    torch.cuda.synchronize()
+    R = comp.ctx.gracekv_export()["rtok"].reshape(L * G, Nc)
+    comp.ctx.close()
+    del x, Qg
+    torch.cuda.empty_cache()
+    shat = run["ex"]["rtok"].reshape(L * G, Nc)       # the direct values, same inputs
+    one_m = np.float32(np.float32(1.0) - np.float32(lam))
+    prod = one_m * shat                               # fp32, as the device rounds it
+    dh = (R.astype(np.float64) - prod.astype(np.float64)) / lam
+    mean = dh.mean(0)
+    # the same d-hat in every row, up to the rounding of the mix's last add
+    tol = 4 * 2.0 ** -24 * (np.abs(R) + np.abs(prod)).max(0).astype(np.float64) / lam
+    assert np.all(np.abs(dh - mean[None]) <= tol[None] + 1e-15)
+    assert mean.min() >= -tol.max() and abs(mean.sum() - 1.0) < 1e-4
+    # the first hop's seeds: S descending (ties lower t) while fewer than 64
+    # and the mass is below 0.9 (Eq. app_global_seed_score); there d-hat is 0
+    # and R is exactly the rounded (1 - lambda) s-hat
+    S = shat.astype(np.float64).mean(0)
+    S = S / (S.sum() + 1e-6)
+    order = np.lexsort((np.arange(Nc), -S))
+    cum, seeds, before = 0.0, [], []
+    while len(seeds) < 64 and cum < 0.9:
+        seeds.append(int(order[len(seeds)]))
+        before.append(cum)
+        cum += S[seeds[-1]]
+    # skip seeds whose rank or membership fp32 sums could change
+    gap = np.abs(np.diff(S[order[:len(seeds) + 1]])) / S[order[0]]
+    sure = [t for k, t in enumerate(seeds) if gap[k] > 1e-4 and (k == 0 or gap[k - 1] > 1e-4)]
+    if len(seeds) < 64 or 0.9 - before[-1] < 1e-4:
+        sure = [t for t in sure if t != seeds[-1] or 0.9 - before[-1] >= 1e-4]
+    print("multihop full size: seeds", len(seeds), "checked", len(sure), "d-hat max", mean.max())
+    assert len(sure) >= len(seeds) // 2
+    for t in sure:
+        assert np.all(R[:, t] == prod[:, t]), t

@@ -169,6 +169,62 @@ def test_multihop_relevance_matches_the_oracle(m_seed):
     print("multihop", json.dumps(rep))
 
 
+@pytest.mark.parametrize("T,cs", [(6000, 0), (4500, 7)])
+def test_multihop_over_several_selection_parts(T, cs):
+    # N_c > 2048: the seed selection merges several sorted 2048-token parts,
+    # the last one ragged; a sink prefix (cs > 0) lies inside every seed's
+    # causal range but outside C.  The mixed token values against the
+    # oracle's token values (App. A.2) and multi-hop relevance (App. A.4)
+    import oracle as O
+    from tests import parity as P
+    w = synth.WORKLOADS["small"]
+    x = synth.make_inputs(w, layers=[0, 1, 2, 3], heads=[0, 1], T=T)
+    L, G, T, d = x.K.shape
+    Hq, W = x.Q.shape[1], x.Q.shape[2]
+    p = O.make_params(L, G, Hq, T, d, W, w.rope_base, cs, lambda_graph=0.3)
+    B = (L * G * (T - cs)) // 8
+    r_eff, _ = O.budget(p, B)
+    p.recent = r_eff
+    Nc = T - cs - r_eff
+    assert Nc > 2 * 2048 and Nc % 2048 != 0
+    gl = O.graph_layers(p)
+    Qg = synth.make_graph_queries(w, [int(l) for l in gl], T=T, heads=range(Hq))
+    g = P.run_gpu(x.K, x.V, x.Q, B, w.rope_base, ctx_start=cs, Qg=Qg, lambda_graph=0.3)
+    rt = np.asarray(g["export"]["rtok"]).reshape(L, G, Nc)
+    K64, Q64 = x.K.double().numpy(), x.Q.double().numpy()
+    m, Z, _ = O.row_stats(p, Q64, K64)
+    shat = O.token_values(p, Q64, K64, m, Z)
+    dh, sd, _ = O.multihop(p, shat, Qg, K64)
+    ref = 0.7 * shat + 0.3 * dh[None, None, :]
+    err = np.abs(rt - ref).max() / np.abs(ref).max()
+    print("multihop parts", -(-Nc // 2048), "seeds", int((sd[0] >= 0).sum()), int((sd[1] >= 0).sum()),
+          "rel err", err)
+    assert err < 1e-4
+
+
+def test_floor_reads_the_multihop_mixed_values():
+    # both NEXT stages at the paper's values (alpha 0.6, lambda 0.3): the floor
+    # (App. A.5 Stage I) takes R after the multi-hop mix (Eq.
+    # app_bottom_up_value); accepted positions, trees, selection and cache
+    import oracle as O
+    w = synth.WORKLOADS["small"]
+    x = synth.make_inputs(w, layers=[0, 1, 2, 3], heads=[0, 1], T=1000)
+    L, G, T, d = x.K.shape
+    p = O.make_params(L, G, x.Q.shape[1], T, d, x.Q.shape[2], w.rope_base, recent=32)
+    gl = O.graph_layers(p)
+    Qg = synth.make_graph_queries(w, [int(l) for l in gl], T=T, heads=range(x.Q.shape[1]))
+    B = (L * G * T) // 8
+    P, g, o = _run(x.K, x.V, x.Q, B, w.rope_base, Qg=Qg, lambda_graph=0.3, alpha_floor=0.6)
+    fl = g["comp"].ctx.gracekv_export_floor()
+    ofl = o["floor"]
+    assert ofl["accepted"].sum() > 0
+    assert np.array_equal(fl["accepted"], ofl["accepted"])
+    assert fl["B_floor"] == ofl["B_floor"]
+    np.testing.assert_allclose(fl["f"], ofl["f"], rtol=2e-5, atol=1e-9)
+    rep = P.compare(g, o, torch.bfloat16)
+    print("floor+multihop", int(ofl["accepted"].sum()), json.dumps(rep))
+
+
 def test_fullkv_identity_is_bit_exact():
     # x = 1: every tree expands to its leaves; the cache is the input (App. C.5)
     w = synth.WORKLOADS["pr1"]
