@@ -21,6 +21,12 @@ outputs the oracle computes one by one, and by properties that hold at any size:
                  op, tree consistency of the selected splits, entry count
   gather         the group's entries partition its covered slots; 256 sampled
                  entries equal the oracle's prototype of the same interval
+  floor          a compression with the singleton floor at alpha 0.6 (App.
+                 A.5 Stage I): B_floor within floor(alpha B_free); per (l, g)
+                 the accepted tokens pass the gate gamma / N_c and are an
+                 f-descending prefix; each is its own entry (m = 1) in the
+                 final cache, with the input's K/V bits in the (l, g) that
+                 holds the most of them
   multi-hop      a second compression with lambda = 0.3 (App. A.4): the
                  implied d-hat is the same for every (l, g), non-negative, sums
                  to 1 and is exactly zero at the first hop's seeds, chosen on
@@ -340,3 +346,51 @@ def test_multihop_full_size_properties(run):
     assert len(sure) >= len(seeds) // 2
     for t in sure:
         assert np.all(R[:, t] == prod[:, t]), t
+
+
+def test_singleton_floor_full_size_properties(run):
+    from paper_2608_07001_gb300 import gracekv as gk
+    w = run["w"]
+    L, G, T, d, Hq, W, Nc = (run[k] for k in ("L", "G", "T", "d", "Hq", "W", "Nc"))
+    alpha = 0.6
+    x = synth.make_inputs(w, device="cuda")
+    p = gk.make_params(L, G, Hq, T, d, W, dtype=x.K.dtype, budget=run["B"], rope_base=w.rope_base,
+                       alpha_floor=alpha)
+    comp = gk.Compressor(p)
+    cache = comp(x.K, x.V, x.Q)
+    torch.cuda.synchronize()
+    fl = comp.ctx.gracekv_export_floor()
+    E = comp.n_entries
+    off = cache.offsets.cpu().numpy()
+    pos, lo, hi = (getattr(cache, k)[:E].cpu().numpy() for k in ("pos", "src_lo", "src_hi"))
+    logm = cache.log_m[:E].cpu().numpy()
+    acc, f = fl["accepted"].astype(bool), fl["f"]
+    lg_b = int(acc.sum(1).argmax())                       # the (l, g) with the most floor tokens
+    Ks, Vs = x.K[lg_b // G, lg_b % G].cpu(), x.V[lg_b // G, lg_b % G].cpu()
+    cK, cV = cache.K[:E].cpu(), cache.V[:E].cpu()
+    comp.ctx.close()
+    del x, cache
+    torch.cuda.empty_cache()
+    cap = int(math.floor(alpha * run["b_free"]))
+    assert 0 < fl["B_floor"] <= cap and E <= run["B"]
+    gate = np.float32(1.2 / Nc)
+    n_acc = 0
+    for lg in range(L * G):
+        a_idx = np.nonzero(acc[lg])[0]
+        if len(a_idx) == 0:
+            continue
+        n_acc += len(a_idx)
+        fmin = f[lg, a_idx].min()
+        assert fmin >= gate * np.float32(1 - 1e-6), lg
+        assert np.all(f[lg, ~acc[lg]] <= fmin), lg        # a prefix in f-descending order
+        e0, e1 = int(off[lg]), int(off[lg + 1])
+        single = (hi[e0:e1] - lo[e0:e1]) == 1
+        where = {int(t): e0 + k for k, t in enumerate(pos[e0:e1]) if single[k]}
+        for t in a_idx:
+            e = where.get(int(t))                         # context starts at 0 here
+            assert e is not None and logm[e] == 0.0, (lg, int(t))
+            if lg == lg_b:
+                assert torch.equal(cK[e], Ks[t]) and torch.equal(cV[e], Vs[t])
+    print("floor full size: accepted", n_acc, "B_floor", fl["B_floor"], "cap", cap,
+          "bit-checked (l, g)", lg_b, int(acc[lg_b].sum()))
+    assert n_acc > 0
