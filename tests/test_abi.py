@@ -65,7 +65,7 @@ def _create(gk, **kw):
     base = dict(L=1, G=2, Hq=2, T=1024, d=128, W=32)
     base.update({k: kw.pop(k) for k in list(kw) if k in base})
     p = gk.make_params(base["L"], base["G"], base["Hq"], base["T"], base["d"], base["W"],
-                       dtype="f32", budget=kw.pop("budget", 256), rope_base=1e4, **kw)
+                       dtype=kw.pop("dtype", "f32"), budget=kw.pop("budget", 256), rope_base=1e4, **kw)
     h = C.c_void_p()
     return gk.lib().gracekv_create(C.byref(p), C.byref(h)), h
 
@@ -77,7 +77,14 @@ def _create(gk, **kw):
     (dict(k_cand=17), 1),
     (dict(windows=(4, 32)), 1),             # window scale above 16
     (dict(seg_layers=(3,)), 1),             # layer out of range
-    (dict(lambda_graph=0.3), 8),            # multi-hop relevance not built
+    (dict(lambda_graph=0.3), 8),            # multi-hop relevance needs bf16
+    (dict(lambda_graph=1.5, dtype="bf16"), 1),
+    (dict(lambda_graph=0.3, dtype="bf16", m_seed=65), 1),     # one 64-row seed tile
+    (dict(lambda_graph=0.3, dtype="bf16", m_seed=0), 1),
+    (dict(lambda_graph=0.3, dtype="bf16", eta_seed=0.0), 1),
+    (dict(lambda_graph=0.3, dtype="bf16", r_hop=0), 1),
+    (dict(lambda_graph=0.3, dtype="bf16", rho_hop=-0.5), 1),
+    (dict(lambda_graph=0.3, dtype="bf16", T=131072 + 64), 8),  # N_c above the seed selection's
     (dict(alpha_floor=1.5), 1),             # floor cap above the budget
     (dict(alpha_floor=0.6, floor_eta=1.5), 1),
     (dict(alpha_floor=0.6, quota_alloc=1), 8),   # floor with fixed per-pair capacity

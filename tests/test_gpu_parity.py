@@ -326,6 +326,45 @@ def test_errors_are_reported_not_trapped():
     assert e.value.status == gk.GKV_ENONFINITE
 
 
+def test_multihop_errors_are_reported():
+    # the graph queries' contract (App. A.4 inputs): statuses, not faults
+    from paper_2608_07001_gb300 import gracekv as gk
+    w = synth.WORKLOADS["small"]
+    x = synth.make_inputs(w, layers=[0, 1, 2, 3], heads=[0, 1], T=300)
+    L, G, T, d = x.K.shape
+    Hq, W = x.Q.shape[1], x.Q.shape[2]
+    K, V, Q = x.K.cuda(), x.V.cuda(), x.Q.cuda()
+    gl = gk.graph_layers(L)
+    Qg = synth.make_graph_queries(w, gl, T=T, heads=range(Hq), device="cuda")
+    mk = lambda lam: gk.make_params(L, G, Hq, T, d, W, dtype=torch.bfloat16, budget=L * G * T // 8,
+                                    rope_base=w.rope_base, lambda_graph=lam)
+    ctx0 = gk.Context(mk(0.0))
+    with pytest.raises(gk.GraceKVError) as e:           # no multi-hop stage to feed
+        ctx0.gracekv_set_graph_queries(Qg)
+    assert e.value.status == gk.GKV_ESTATE
+    ctx = gk.Context(mk(0.3))
+    slots = torch.empty(T, dtype=torch.int32, device="cuda")
+    ctx.gracekv_segment(V, slots)
+    with pytest.raises(gk.GraceKVError) as e:           # build without the queries
+        ctx.gracekv_build_trees(K, V, Q)
+    assert e.value.status == gk.GKV_EINVAL
+    buf = torch.empty(Qg.numel() + 8, dtype=Qg.dtype, device="cuda")
+    with pytest.raises(gk.GraceKVError) as e:           # one element past a 16-byte boundary
+        ctx.gracekv_set_graph_queries(buf[1:1 + Qg.numel()].view(Qg.shape))
+    assert e.value.status == gk.GKV_EINVAL
+    with pytest.raises(gk.GraceKVError) as e:           # one graph layer instead of two
+        ctx.gracekv_set_graph_queries(Qg[:1])
+    assert e.value.status == gk.GKV_EINVAL
+    hc = gk.Cache.empty_host(L * G * T, d, L * G, K.dtype)
+    with pytest.raises(gk.GraceKVError) as e:           # the host-buffer pass takes no queries
+        ctx.gracekv_compress_host(x.K.contiguous(), x.V.contiguous(), x.Q.contiguous(), hc)
+    assert e.value.status == gk.GKV_EUNSUPPORTED
+    # the context still works: the same build with the queries set
+    ctx.gracekv_set_graph_queries(Qg)
+    ctx.gracekv_build_trees(K, V, Q)
+    assert ctx.gracekv_allocate() > 0
+
+
 def test_score_ahead_matches_inline():
     # The score passes issued ahead on a second stream (gracekv_score, as the
     # Compressor does) give the same bits as the passes the tree build runs
