@@ -103,3 +103,45 @@ def test_hops_zero_their_seeds_and_mix_into_the_token_values(oracle_lib):
     np.testing.assert_allclose(res["rtok"], 0.7 * mh["shat"] + 0.3 * mh["dhat"][None, None, :], rtol=1e-13)
     res0 = O.run(K, V, Q, 120, 0.0, recent=8)
     np.testing.assert_allclose(mh["shat"], res0["rtok"], rtol=1e-13)
+
+
+def test_decay_weights_only_the_later_hops(oracle_lib):
+    # d = d1 + rho d2: rho = 0 gives the one-hop result, and d-hat at rho = 1/2
+    # lies on the segment from d-hat(0) to d-hat(1), strictly past its middle
+    # when the second hop carries mass (the weights are (A + eps) / 2 and
+    # (A + B + eps) / 2 over A + B / 2 + eps, A and B the hops' sums)
+    p, K, Qg, shat, gl = setup(5)
+    p.r_hop = 1
+    d_one, _, _ = O.multihop(p, shat, Qg, K)
+    p.r_hop = 2
+    res = {}
+    for rho in (0.0, 0.5, 1.0):
+        p.rho_hop = rho
+        res[rho], _, _ = O.multihop(p, shat, Qg, K)
+    np.testing.assert_allclose(res[0.0], d_one, rtol=1e-12, atol=1e-15)
+    a, diff = res[0.0], res[1.0] - res[0.0]
+    theta = np.dot(res[0.5] - a, diff) / np.dot(diff, diff)
+    np.testing.assert_allclose(res[0.5], a + theta * diff, rtol=1e-9, atol=1e-14)
+    assert 0.5 < theta < 1.0
+
+
+def test_second_hop_seeds_follow_the_first_hops_propagation(oracle_lib):
+    # hop 2 chooses its seeds by the same rule from hop 1's propagation score
+    # normalised over C (the one-hop d-hat up to its eps), and weights them by
+    # that score over the seed set
+    p, K, Qg, shat, gl = setup(6)
+    p.r_hop = 1
+    d1, sd1, _ = O.multihop(p, shat, Qg, K)
+    p.r_hop = 2
+    dh, sd, sw = O.multihop(p, shat, Qg, K)
+    np.testing.assert_array_equal(sd[0], sd1[0])
+    score = d1 / d1.sum()
+    order = np.lexsort((np.arange(len(score)), -score))
+    cum, want = 0.0, []
+    while len(want) < p.m_seed and cum < p.eta_seed:
+        want.append(int(order[len(want)]))
+        cum += score[want[-1]]
+    n = len(want)
+    assert 1 < n < p.m_seed
+    assert list(sd[1][:n]) == want and np.all(sd[1][n:] == -1)
+    np.testing.assert_allclose(sw[1][:n], score[want] / score[want].sum(), rtol=1e-12)
