@@ -144,3 +144,30 @@ def test_alpha_zero_and_fullkv_are_unchanged(oracle_lib):
     c = O.run(K, V, Q, 2 * T, 1e4, recent=16, alpha_floor=0.6)
     np.testing.assert_array_equal(c["cache"]["K"], K.reshape(-1, K.shape[-1]))
     assert np.all(c["cache"]["log_m"] == 0)
+
+
+@pytest.mark.parametrize("alpha,acc0,acc1,b_floor", [
+    (0.6, {5, 15, 25}, {10}, 10),    # cap 12: n' = 3, 1; shares 9, 3
+    (0.5, {5, 15, 25}, set(), 7),    # cap 10: n' = 3, 1; shares 7, 2 < head 1's cost 3
+    (0.35, {5}, set(), 3),           # cap 7: n' = 2, 1; shares 4, 2; {5, 15} costs 5 > 4
+])
+def test_proportional_reduction_and_per_head_shares(oracle_lib, alpha, acc0, acc1, b_floor):
+    # Worked by hand (Eq. app_floor_cap and its per-head safeguard).  f = R
+    # (no consensus, no pooling).  Head 0: six spikes of 0.15, three interior,
+    # non-adjacent ones per slot: joint cost 3 + 4 = 7 per slot.  Head 1: two
+    # spikes of 0.45, one per slot: 1 + 2 = 3 per slot.  C0 = 14 + 6 = 20 over
+    # the cap floor(alpha 20): each head keeps max(1, floor(n cap / C0)) of
+    # its candidates (ties: lower t), may spend floor(cap n' / sum n'), and
+    # accepts the longest prefix that fits.
+    Nc = 80
+    R = np.zeros((2, Nc))
+    R[0] = 0.1 / 74
+    R[0, [5, 15, 25, 45, 55, 65]] = 0.15
+    R[1] = 0.1 / 78
+    R[1, [10, 50]] = 0.45
+    p = O.make_params(1, 2, 2, Nc + 8, 8, 2, 0.0, recent=8, alpha_floor=alpha, floor_c=0.0,
+                      floor_half=0)
+    f, acc, bf, nc = O.floor(p, R, [0, 40, 80], 20)
+    assert nc == 8
+    assert set(np.nonzero(acc[0])[0]) == acc0 and set(np.nonzero(acc[1])[0]) == acc1
+    assert bf == b_floor <= int(alpha * 20)
