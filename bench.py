@@ -120,6 +120,22 @@ def cpu_baseline(w, ratio: float, T_s: int = 4608):
     return value, dt, sample
 
 
+def max_over_ranks(x: float, dist, device) -> float:
+    """The largest x over the ranks of the process group (x itself when dist
+    is None): the job's time is its slowest rank's."""
+    if dist is None:
+        return float(x)
+    t = torch.tensor([float(x)], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world: int, tokens: int, steps: int, seconds: float) -> float:
+    """Context tokens/s of the whole job: every rank compresses its own
+    request of `tokens` tokens per step."""
+    return world * tokens * steps / seconds
+
+
 def run_reference(args, w):
     """Reference arm: the CPU oracle, timed on the host cores."""
     rank = int(os.environ.get("RANK", "0"))
@@ -379,12 +395,9 @@ def main():
     ms_total = e0.elapsed_time(e1)
     stage_ms, launches1, work = comp.ctx.gracekv_stats()
     comp.ctx.gracekv_profile(False)
-    t = torch.tensor([ms_total], device=dev, dtype=torch.float64)
-    if dist is not None:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    ms_total = float(t.item())
+    ms_total = max_over_ranks(ms_total, dist, dev)
     ms_step = ms_total / args.steps
-    value = world * T * args.steps / (ms_total / 1e3)
+    value = whole_job_rate(world, T, args.steps, ms_total / 1e3)
     E = comp.n_entries
 
     # ---- roofline ----------------------------------------------------------------
@@ -442,13 +455,10 @@ def main():
             n = e2e_step()
         barrier()
         dt = time.perf_counter() - t0
-        tt = torch.tensor([dt], device=dev, dtype=torch.float64)
-        if dist is not None:
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        dt = float(tt.item())
+        dt = max_over_ranks(dt, dist, dev)
         h2d = sum(t_.numel() * t_.element_size() for t_ in (K, V, Q))
         d2h = n * (2 * d * elem + 16) + hc.offsets.numel() * 8
-        e2e = {"value": world * T * args.e2e_steps / dt, "unit": "tokens/s",
+        e2e = {"value": whole_job_rate(world, T, args.e2e_steps, dt), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
     cpu = None
