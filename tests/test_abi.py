@@ -108,3 +108,12 @@ def test_null_context_is_rejected(gk):
     n = C.c_int64()
     assert lib.gracekv_allocate(None, C.byref(n), None) == gk.GKV_EINVAL
     assert lib.gracekv_last_error(None) == b"null context"
+
+
+def test_stage_names_match_the_header(gk):
+    # gracekv_stats fills GRACEKV_N_STAGES timers; the binding names each one
+    hdr = open(os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))),
+                            "include", "gracekv.h")).read()
+    n = int(re.search(r"#define GRACEKV_N_STAGES (\d+)", hdr).group(1))
+    assert len(gk.Context.STAGES) == n
+    assert gk.Context.STAGES[6:] == ("floor", "multihop")
