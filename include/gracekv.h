@@ -202,7 +202,12 @@ gkv_status gracekv_score(gracekv_ctx *ctx, const void *K, const void *Q, void *s
  * omega (device [L][G] fp32, nullable = all ones) is the head sensitivity.
  * Row statistics (max logit, partition over [0, T), partition over the
  * compressible region) are computed for every probe row (l, h, u); the trees
- * stay in the context's workspace.  Errors: GKV_EINVAL, GKV_ESTATE,
+ * stay in the context's workspace.  In order, after the token values: with
+ * lambda_graph > 0 the multi-hop relevance (App. A.4) mixes into them, from
+ * the queries of the last gracekv_set_graph_queries; with alpha_floor > 0
+ * the singleton floor (App. A.5 Stage I) is chosen from the (mixed) values;
+ * then the trees are built, floor positions extracted first.  Errors:
+ * GKV_EINVAL (also: lambda_graph > 0 without graph queries), GKV_ESTATE,
  * GKV_EUNSUPPORTED (a slot longer than 128 tokens), GKV_ECUDA.
  */
 gkv_status gracekv_build_trees(gracekv_ctx *ctx, const void *K, const void *V, const void *Q,
