@@ -254,9 +254,10 @@ gkv_status gracekv_gather(gracekv_ctx *ctx, const void *K, const void *V, void *
  * follow on `stream`.  The cache is then copied to the host arrays (layouts
  * of gracekv_gather; capacity `cap` entries, offsets [L G + 1]).
  * Synchronous: returns when the host arrays hold the cache; *n_entries_host
- * receives E.  No hidden states, surprisal or supplied slots (use the stage
- * calls for those).  Errors: those of the stage calls, GKV_ECAPACITY (E >
- * cap), GKV_ENOMEM (device copies of the inputs).
+ * receives E.  No hidden states, surprisal, supplied slots or graph queries
+ * (use the stage calls for those).  Errors: those of the stage calls,
+ * GKV_ECAPACITY (E > cap), GKV_ENOMEM (device copies of the inputs),
+ * GKV_EUNSUPPORTED (lambda_graph > 0).
  */
 gkv_status gracekv_compress_host(gracekv_ctx *ctx, const void *K, const void *V, const void *Q,
                                  const float *omega, void *K_out, void *V_out, int32_t *pos, float *log_m,
