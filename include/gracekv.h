@@ -105,7 +105,7 @@ typedef struct {
      *   capacity another pair leaves; trees are then built completely. */
     int32_t seg_mode;
     int32_t quota_alloc;
-    /* Singleton floor (used when alpha_floor > 0; App. A.5 Stage I, App. C.2):
+    /* Singleton floor (used when alpha_floor > 0; App. A.5 Stage I, App. C.4):
      * consensus weight c (0.5), gate gamma (1.2, f >= gamma / N_c), value mass
      * eta (0.95), max-pool half width (3: width 7).  Candidates of an (l, g):
      * f descending (ties: lower t) up to the longest prefix whose token values
@@ -133,10 +133,10 @@ gkv_status gracekv_default_params(gkv_params *p);
  * (App. A.1 Eq. app_total_budget).  Returns -1 for invalid arguments.  Host only. */
 int64_t gracekv_budget_for_ratio(int32_t L, int32_t G, int32_t n_ctx, double x);
 
-/* The graph layers of the multi-hop relevance (App. A.4): the distinct
- * layers floor(0.50 L) and floor(0.75 L) (each at most L - 1), ascending,
- * written to out[0 .. n-1] (nullable; room for 2).  Returns n (1 or 2), or -1
- * for L <= 0.  Host only. */
+/* The graph layers of the multi-hop relevance (App. A.4; their depths are
+ * stated in App. A.1): the distinct layers floor(0.50 L) and floor(0.75 L)
+ * (each at most L - 1), ascending, written to out[0 .. n-1] (nullable; room
+ * for 2).  Returns n (1 or 2), or -1 for L <= 0.  Host only. */
 int32_t gracekv_graph_layers(int32_t L, int32_t *out);
 
 /* Validate *p, resolve the recent window against the budget (r = 32, shrunk to

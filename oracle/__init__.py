@@ -265,7 +265,7 @@ class Trees:
 
 
 def floor(p: Params, rtok, slot_starts, B_base: int):
-    """Singleton floor (App. A.5 Stage I, App. C.2): scores f, accepted
+    """Singleton floor (App. A.5 Stage I, App. C.4): scores f, accepted
     positions [L*G, N_c] (uint8), B_floor, number of initial candidates."""
     rtok = _f64(rtok)
     LG, Nc = p.L * p.G, p.ctx_end - p.recent - p.ctx_start

@@ -699,7 +699,7 @@ static int cmp_kv_desc(const void *x, const void *y)
 
 /* ------------------------------------------------------------------------ */
 /* Stage I singleton floor, App. A.5 (Eqs. app_floor_score, app_floor_gate,   */
-/* app_floor_cap) and App. C.2 (candidates, path charging, the cap), in the   */
+/* app_floor_cap) and App. C.4 (candidates, path charging, the cap), in the   */
 /* reading R15 of the header.                                                  */
 /* ------------------------------------------------------------------------ */
 static int slot_of(const int32_t *slot_starts, int32_t n_slots, int t)

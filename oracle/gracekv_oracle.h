@@ -61,8 +61,9 @@
  *   R14 "w/o GA": (l, g) number lg gets the capacity floor(B_free / LG), plus
  *       one for lg < B_free mod LG; the heap pops as before and discards an op
  *       its (l, g) cannot afford; a pair's unused capacity is lost.
- *   R16 multi-hop relevance (App. A.4): graph layers at relative depths 0.50
- *       and 0.75 (floor(rho L), duplicates dropped); seeds of a hop = tokens
+ *   R16 multi-hop relevance (App. A.4): graph layers at the relative depths
+ *       0.50 and 0.75 that App. A.1 states, read as floor(rho L) with
+ *       duplicates dropped; seeds of a hop = tokens
  *       of C in order of their score descending (ties: lower t), taken while
  *       fewer than m_seed are taken and their running mass is below eta_seed
  *       (the seed that reaches eta is included); hop 1 scores = S-hat (Eq.
@@ -71,7 +72,7 @@
  *       the seed set, normalised to sum 1 (uniform when they sum to 0); seed u
  *       attends to [0, u] (its causal visible range); the propagation score
  *       of a hop is zeroed at that hop's and all earlier seeds.
- *   R15 singleton floor (App. A.5 Stage I, App. C.2): R = the token values
+ *   R15 singleton floor (App. A.5 Stage I, App. C.4): R = the token values
  *       after the multi-hop mix (the direct ones when lambda_graph = 0); the
  *       consensus is the mean over all (l, g); the
  *       max-pool window is clipped to the compressible context.  Candidates

@@ -112,7 +112,7 @@ int32_t gracekv_graph_layers(int32_t L, int32_t *out) {
     if (L <= 0) return -1;
     int32_t gl[2];
     int32_t n = 0;
-    for (double rho : {0.50, 0.75}) {   // relative depths of the graph layers (App. A.4)
+    for (double rho : {0.50, 0.75}) {   // relative depths of the graph layers (App. A.1)
         int32_t l = std::min((int32_t)std::floor(rho * L), L - 1);
         if (n == 0 || gl[n - 1] != l) gl[n++] = l;
     }

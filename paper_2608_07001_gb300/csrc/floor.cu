@@ -1,5 +1,5 @@
 // floor.cu -- the Stage I singleton floor (App. A.5 Stage I, Eqs.
-// app_floor_score, app_floor_gate, app_floor_cap; App. C.2), between the
+// app_floor_score, app_floor_gate, app_floor_cap; App. C.4), between the
 // token values and the tree build.
 //
 //   f_{l,g,t} = max_{|tau - t| <= 3, tau in C} [(1 - c) R_{l,g,tau} + c mean_{l,g} R_{l,g,tau}]

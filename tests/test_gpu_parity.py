@@ -174,7 +174,7 @@ def test_multihop_over_several_selection_parts(T, cs):
     # N_c > 2048: the seed selection merges several sorted 2048-token parts,
     # the last one ragged; a sink prefix (cs > 0) lies inside every seed's
     # causal range but outside C.  The mixed token values against the
-    # oracle's token values (App. A.2) and multi-hop relevance (App. A.4)
+    # oracle's token values and multi-hop relevance (App. A.4)
     import oracle as O
     from tests import parity as P
     w = synth.WORKLOADS["small"]
@@ -226,7 +226,7 @@ def test_floor_reads_the_multihop_mixed_values():
 
 
 def test_fullkv_identity_is_bit_exact():
-    # x = 1: every tree expands to its leaves; the cache is the input (App. C.5)
+    # x = 1: every tree expands to its leaves; the cache is the input (App. C.6)
     w = synth.WORKLOADS["pr1"]
     x = synth.make_inputs(w, T=640)
     L, G, T, d = x.K.shape

@@ -1,4 +1,4 @@
-"""End-to-end pins of the oracle pipeline (App. A.5 packing, App. C.5)."""
+"""End-to-end pins of the oracle pipeline (App. A.5 packing, App. C.6)."""
 import numpy as np
 import pytest
 
@@ -18,7 +18,7 @@ SMALL = dict(n_min=8, n_max=32, n0=16, recent=8, windows=(2, 4, 8))
 
 @pytest.mark.parametrize("ctx", [(0, None), (5, 140)])
 def test_full_budget_recovers_fullkv_exactly(oracle_lib, ctx):
-    # App. C.5 "FullKV recovery": x = 1 -> every tree expands to its leaves and
+    # App. C.6 "FullKV recovery": x = 1 -> every tree expands to its leaves and
     # the cache equals the input entry by entry, positions 0..T-1, log m = 0.
     K, V, Q = inputs(0)
     L, G, T, d = K.shape

@@ -1,4 +1,4 @@
-"""Pins of the oracle's singleton floor (App. A.5 Stage I, App. C.2).
+"""Pins of the oracle's singleton floor (App. A.5 Stage I, App. C.4).
 
 f = width-7 max-pool of (1 - c) R + c mean_{l,g} R (Eq. app_floor_score); the
 gate f >= gamma / N_c (Eq. app_floor_gate); candidates up to value mass eta;

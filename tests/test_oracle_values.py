@@ -159,7 +159,7 @@ def test_distortion_drop_is_mean_attention_mass(oracle_lib):
     assert res["Ddrop"] == pytest.approx(exp, rel=1e-12)
 
 
-# --- trees: App. A.3 refinement, App. A.4 conservation, App. C.5 telescoping ------------
+# --- trees: App. A.3 refinement, App. A.4 conservation, App. C.6 telescoping ------------
 
 @pytest.fixture(scope="module")
 def small_run(oracle_lib):
@@ -199,7 +199,7 @@ def test_tree_structure_and_value_conservation(small_run):
 
 
 def test_telescoping_cost_identity(small_run):
-    # App. C.5: 1 + sum over expanded nodes (|child| - 1) = n per tree.
+    # App. C.6: 1 + sum over expanded nodes (|child| - 1) = n per tree.
     K, V, Q, res = small_run
     nd, tr = res["trees"].nodes, res["trees"]
     for u, root in enumerate(tr.unit_root):
