@@ -72,8 +72,9 @@ typedef struct gracekv_ctx gracekv_ctx;
  * paper's: App. A.1 (recent window 32), App. B.2 (windows {4,8,16},
  * lambda_stab 0.25, lambda_s 0.15, segmentation layers at relative depths
  * 0.33/0.50/0.67), App. B.3 (n_min 16, n_max 128, n0 64, lambda_d 0.25,
- * lambda_n 0.10, c_cut 1.0), App. A.3 (K = 16 split candidates, lambda_kappa
- * 0.05, lambda_Z 0.25, lambda_M 0.75, value base 0.1), epsilon 1e-6.
+ * lambda_n 0.10, c_cut 1.0), App. B.4 (K = 16 split candidates), App. A.3
+ * (lambda_kappa 0.05, lambda_Z 0.25, lambda_M 0.75, value base 0.1), App. B.2
+ * (epsilon 1e-6).
  */
 typedef struct {
     int32_t L, G, Hq, T, d, W;     /* layers, KV heads, query heads, tokens, head dim, probes */
