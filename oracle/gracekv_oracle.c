@@ -783,7 +783,8 @@ int orc_floor(const orc_params *p, const double *rtok, const int32_t *slot_start
         }
         nkept += ncand[lg];
     }
-    /* acceptance with path charging: the longest prefix within the head's share */
+    /* acceptance with path charging: every kept candidate, in order, whose
+       complete path fits the head's share; one that does not fit is skipped */
     int64_t used = 0;
     for (int lg = 0; lg < LG; lg++) {
         if (!ncand[lg]) continue;
@@ -799,7 +800,7 @@ int orc_floor(const orc_params *p, const double *rtok, const int32_t *slot_start
             while (lo > a && !acc[lo - 1]) lo--;
             while (hi < b - 1 && !acc[hi + 1]) hi++;
             int64_t cost = (covered[j] ? 0 : 1) + (lo < t) + (t < hi);
-            if (used_h + cost > cap_h) break;
+            if (used_h + cost > cap_h) continue;
             acc[t] = 1;
             covered[j] = 1;
             used += cost;

@@ -85,12 +85,15 @@
  *       n >= 1 candidates keeps its first n' = max(1, floor(n cap / C0)).
  *       Per-head safeguard: an (l, g) may use cap_h = floor(cap n' / sum n')
  *       entries (its share of the cap by kept candidates; the shares sum to at
- *       most cap, so the global cap holds).  An (l, g) accepts the longest
- *       prefix of its kept candidates whose joint cost fits cap_h (the joint
- *       cost never decreases along the prefix: a candidate adds 1 for its
- *       slot's Add if the slot is still uncovered plus the new entries of
- *       extracting it from its current frontier interval, [lo, t) and
- *       (t, hi] when non-empty).
+ *       most cap, so the global cap holds).  An (l, g) walks its kept
+ *       candidates in order and accepts each one whose complete path still
+ *       fits cap_h; one that does not fit is skipped and the walk goes on,
+ *       so a later, cheaper candidate can still be accepted (App. A.5: a
+ *       candidate is accepted only when its path remains feasible, and the
+ *       floor is not switched off for a head when the budget is tight).  A
+ *       candidate's path costs 1 for its slot's Add if the slot is still
+ *       uncovered, plus the new entries of extracting it from its current
+ *       frontier interval [lo, hi]: [lo, t) and (t, hi] when non-empty.
  *       A node whose interval holds accepted positions is extracted at the one
  *       with the largest f (ties: lower t); the floor ops (the Adds of slots
  *       with an accepted position and these extractions) execute before the

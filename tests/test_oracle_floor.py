@@ -158,7 +158,7 @@ def test_proportional_reduction_and_per_head_shares(oracle_lib, alpha, acc0, acc
     # spikes of 0.45, one per slot: 1 + 2 = 3 per slot.  C0 = 14 + 6 = 20 over
     # the cap floor(alpha 20): each head keeps max(1, floor(n cap / C0)) of
     # its candidates (ties: lower t), may spend floor(cap n' / sum n'), and
-    # accepts the longest prefix that fits.
+    # accepts, in order, each candidate whose path still fits.
     Nc = 80
     R = np.zeros((2, Nc))
     R[0] = 0.1 / 74
@@ -171,3 +171,44 @@ def test_proportional_reduction_and_per_head_shares(oracle_lib, alpha, acc0, acc
     assert nc == 8
     assert set(np.nonzero(acc[0])[0]) == acc0 and set(np.nonzero(acc[1])[0]) == acc1
     assert bf == b_floor <= int(alpha * 20)
+
+
+@pytest.mark.parametrize("R0,share,acc0,used0", [
+    # share 5; head 0 in f order: 10 (slot [0, 40) uncovered: Add + two sides = 3),
+    # 50 (slot [40, 80) uncovered: 3; 3 + 3 = 6 > share 5, skipped),
+    # 11 (its interval is now [11, 39]: one new side, 1; 3 + 1 = 4 <= 5)
+    ({10: 0.4, 50: 0.3, 11: 0.2}, 5, {10, 11}, 4),
+    # share 6: 10 (3), 12 (interval [11, 39]: two sides, 2; total 5), 50 (3;
+    # 5 + 3 = 8 > 6: skipped),
+    # 11 (interval [11, 11] is already {11}: free, 0)
+    ({10: 0.3, 12: 0.25, 50: 0.2, 11: 0.15}, 6, {10, 11, 12}, 5),
+])
+def test_an_unaffordable_candidate_is_skipped_and_later_ones_still_accepted(oracle_lib, R0, share, acc0,
+                                                                             used0):
+    # Worked by hand (App. A.5 Stage I, the paragraph after Eq. app_floor_cap:
+    # a candidate is accepted only when its complete path remains feasible,
+    # and the floor is not disabled for a whole head when the budget is
+    # tight).  f = R (no consensus, no pooling), slots [0, 40) and [40, 80).
+    # Head 1: candidates 0, 1, 2 at the start of slot [0, 40): joint cost
+    # 3 + one run = 4.  No proportional reduction (C0 <= cap), n' = 3 and
+    # len(R0), cap = C0, and each head's share is floor(cap n' / sum n').
+    Nc = 80
+    R = np.zeros((2, Nc))
+    R[0] = (1.0 - sum(R0.values())) / (Nc - len(R0)) / 4      # below the gate 1.2 / N_c
+    for t, v in R0.items():
+        R[0, t] = v
+    R[1] = 0.01 / (Nc - 3) / 4
+    R[1, [0, 1, 2]] = [0.4, 0.3, 0.2]
+    starts = [0, 40, 80]
+    c0 = _frontier_cost(np.isin(np.arange(Nc), list(R0)).astype(np.uint8), starts)
+    cap = c0 + 4
+    assert cap * len(R0) // (len(R0) + 3) == share   # the share the cases are worked against
+    p = O.make_params(1, 2, 2, Nc + 8, 8, 2, 0.0, recent=8, alpha_floor=1.0, floor_c=0.0,
+                      floor_half=0)
+    f, acc, bf, nc = O.floor(p, R, starts, cap)
+    assert nc == len(R0) + 3
+    assert set(np.nonzero(acc[0])[0]) == acc0
+    assert set(np.nonzero(acc[1])[0]) == {0, 1, 2}
+    assert bf == used0 + 4
+    # the accepted set's closed-form frontier count is what was charged
+    assert _frontier_cost(acc[0], starts) == used0
