@@ -112,8 +112,9 @@ typedef struct {
      * f descending (ties: lower t) up to the longest prefix whose token values
      * sum to at most eta.  When their joint cost C0 (per slot: the frontier
      * size after isolating them) exceeds cap = floor(alpha B_free), each (l, g)
-     * keeps its first max(1, floor(n cap / C0)); each then accepts the longest
-     * prefix of those whose joint cost fits floor(cap n' / sum n').  Accepted
+     * keeps its first max(1, floor(n cap / C0)); each then walks those in
+     * order and accepts every one whose path still fits what is left of its
+     * share floor(cap n' / sum n'), skipping those that do not.  Accepted
      * positions become singleton leaves by forced extraction, and the floor's
      * Adds and extractions are executed before the auction.  Not combined with
      * quota_alloc (GKV_EUNSUPPORTED). */
@@ -144,8 +145,10 @@ int32_t gracekv_graph_layers(int32_t L, int32_t *out);
  * floor(B_total / (L G)) when L G r > B_total, never below 4: App. A.1) and
  * allocate the device workspace on the current device.  On success *out owns
  * it; release with gracekv_destroy.  Errors: GKV_EINVAL, GKV_EBUDGET,
- * GKV_EUNSUPPORTED (lambda_graph != 0, alpha_floor != 0, d not in {64, 128},
- * W > 64, ...), GKV_ENOMEM, GKV_ECUDA. */
+ * GKV_EUNSUPPORTED (d not in {64, 128}, W > 64, n_max above 128, G d above
+ * 2048, N_c above 228,351 tokens; lambda_graph > 0 with fp32 inputs or
+ * N_c above 131072; alpha_floor > 0 together with quota_alloc), GKV_ENOMEM,
+ * GKV_ECUDA. */
 gkv_status gracekv_create(const gkv_params *p, gracekv_ctx **out);
 void gracekv_destroy(gracekv_ctx *ctx);
 const char *gracekv_last_error(const gracekv_ctx *ctx);
@@ -362,7 +365,12 @@ gkv_status gracekv_stats(gracekv_ctx *ctx, float *stage_ms, int32_t n_stages, in
  *   device address; make that first call before any stream capture.
  *   Calls share the array: calls that overlap on the GPU (other streams,
  *   other threads) race and must be serialised by the caller.
- *   Errors: GKV_EINVAL (shapes, pointers), GKV_ECAPACITY, GKV_ECUDA.
+ *   Non-finite inputs are not detected: a NaN or Inf in K or Q gives NaN or
+ *   Inf rows and the call still returns GKV_OK (it never synchronises, so it
+ *   has no point at which to report a device-side check); a caller whose
+ *   inputs may be non-finite checks the outputs.
+ *   Errors: GKV_EINVAL (shapes, pointers, L * G above 65535), GKV_ECAPACITY,
+ *   GKV_ECUDA.
  */
 gkv_status gracekv_row_stats_noalloc(const void *K, const void *Q, int32_t L, int32_t G,
                                      int32_t Hq, int32_t T, int32_t d, int32_t W, int32_t dtype,

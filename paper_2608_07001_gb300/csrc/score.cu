@@ -628,6 +628,7 @@ extern "C" gkv_status gracekv_row_stats_noalloc(const void *K, const void *Q, in
         (reinterpret_cast<uintptr_t>(row_ZC) & 3u))
         return GKV_EINVAL;
     if (L <= 0 || G <= 0 || Hq <= 0 || T <= 0 || d <= 0 || W <= 0 || Hq % G || d % 8) return GKV_EINVAL;
+    if ((int64_t)L * G > 65535) return GKV_EINVAL;     // one grid z-slice per (l, g)
     if (dtype != GKV_F32 && dtype != GKV_BF16) return GKV_EINVAL;
     if (c_lo < 0 || c_hi > T || c_lo > c_hi) return GKV_EINVAL;
     const int64_t nrow = (int64_t)L * Hq * W;
@@ -655,7 +656,9 @@ extern "C" gkv_status gracekv_row_stats_noalloc(const void *K, const void *Q, in
     int *status = reinterpret_cast<int *>(scratch + 3 * nrow * nchunks);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     // every (row, chunk) partial is overwritten by the pass; only the status
-    // word has to start at zero
+    // word has to start at zero.  The combine kernel flags non-finite rows in
+    // it, but this entry point does not read it back: such rows come out
+    // NaN / Inf with GKV_OK (documented at the declaration).
     if (cudaMemsetAsync(status, 0, sizeof(int), s) != cudaSuccess) return GKV_ECUDA;
     dim3 grid(nchunks, (a.Rg + gkv::kTR - 1) / gkv::kTR, L * G);
     if (dtype == GKV_BF16)

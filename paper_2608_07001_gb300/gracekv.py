@@ -144,9 +144,30 @@ def gracekv_row_stats_noalloc(K, Q, c_lo: int, c_hi: int, row_m, row_Z, row_ZC, 
     memory pool, or a loop that cannot afford an allocation's synchronisation):
     the scratch is a fixed 4 MiB array inside the library.  Outputs are
     caller-provided [L, Hq, W] fp32 CUDA tensors.  Overlapping calls race.
+    Every argument is checked here before the library is called (a wrong
+    element size or a short output would otherwise become an out-of-bounds
+    device access); a mismatch raises GraceKVError(GKV_EINVAL).
     """
+    def bad(why):
+        return GraceKVError(GKV_EINVAL, "row_stats_noalloc: " + why)
+
+    if K.dim() != 4 or Q.dim() != 4:
+        raise bad("K is [L, G, T, d] and Q is [L, Hq, W, d]")
     L, G, T, d = K.shape
     Hq, W = Q.shape[1], Q.shape[2]
+    if K.dtype not in (torch.bfloat16, torch.float32):
+        raise bad(f"K must be bf16 or fp32, not {K.dtype}")
+    if Q.dtype != K.dtype:
+        raise bad(f"Q must have K's dtype {K.dtype}, not {Q.dtype}")
+    if Q.shape[0] != L or Q.shape[3] != d:
+        raise bad(f"Q {tuple(Q.shape)} does not match K {tuple(K.shape)} in L or d")
+    for name, o in (("row_m", row_m), ("row_Z", row_Z), ("row_ZC", row_ZC)):
+        if o.dtype != torch.float32 or o.numel() < L * Hq * W:
+            raise bad(f"{name} must be fp32 with at least L*Hq*W = {L * Hq * W} elements")
+        if o.device != K.device:
+            raise bad(f"{name} is on {o.device}, K on {K.device}")
+    if Q.device != K.device:
+        raise bad(f"Q is on {Q.device}, K on {K.device}")
     dt = GKV_BF16 if K.dtype == torch.bfloat16 else GKV_F32
     st = lib().gracekv_row_stats_noalloc(_ptr(K), _ptr(Q), L, G, Hq, T, d, W, dt, c_lo, c_hi,
                                          _ptr(row_m), _ptr(row_Z), _ptr(row_ZC), _stream(stream))

@@ -48,3 +48,25 @@ def test_host_buffer_pass_rejects_device_or_strided_tensors(gk):
     with pytest.raises(ValueError, match="contiguous host"):
         gk._host_ptr(x.t())
     assert gk._host_ptr(None) is None and gk._host_ptr(x).value == x.data_ptr()
+
+
+def test_noalloc_refuses_mismatched_arguments_before_any_launch(gk):
+    # a wrong dtype, a Q of another dtype or shape, or a short or non-fp32
+    # output is refused in the binding: none of them reaches the library
+    bf = torch.bfloat16
+    K = torch.zeros(1, 2, 64, 64, dtype=bf)
+    Q = torch.zeros(1, 2, 4, 64, dtype=bf)
+    ok = torch.zeros(1, 2, 4)
+    cases = [
+        (K.half(), Q.half(), ok, "bf16 or fp32"),
+        (K, Q.float(), ok, "K's dtype"),
+        (K, torch.zeros(2, 2, 4, 64, dtype=bf), ok, "L or d"),
+        (K, torch.zeros(1, 2, 4, 32, dtype=bf), ok, "L or d"),
+        (K, Q, torch.zeros(7), "at least"),
+        (K, Q, torch.zeros(1, 2, 4, dtype=torch.float64), "fp32"),
+        (K[0], Q, ok, r"\[L, G, T, d\]"),
+    ]
+    for k, q, out, why in cases:
+        with pytest.raises(gk.GraceKVError, match=why) as e:
+            gk.gracekv_row_stats_noalloc(k, q, 0, 64, out, ok, ok)
+        assert e.value.status == gk.GKV_EINVAL
