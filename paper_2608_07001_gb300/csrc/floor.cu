@@ -10,16 +10,20 @@
 // cost C0 of all candidates -- per slot, the frontier size after isolating
 // them: |S| + maximal runs outside S -- exceeds it, each (l, g) keeps its first
 // max(1, floor(n cap / C0)) candidates; each (l, g) then has the share
-// floor(cap n' / sum n') and accepts the longest prefix of its kept
-// candidates whose joint cost fits the share (the joint cost never decreases
-// along the prefix).  The tree build then extracts every accepted position as
-// a singleton (forced extraction); the floor's ops carry the largest key.
+// floor(cap n' / sum n') and walks its kept candidates in order, accepting
+// each one whose complete path still fits the share and skipping the others
+// (App. A.5 Stage I: a candidate is accepted only when its path remains
+// feasible).  The tree build then extracts every accepted position as a
+// singleton (forced extraction); the floor's ops carry the largest key.
 //
-// One CTA per (l, g) finds every prefix with a block-wide weighted radix
-// select on the key (~bits(f) << 32 | t): three 11/11/10-bit passes over the
-// f part, then an ordered scan over t among the tokens of the crossing f.
-// Token values enter the select as fixed-point integers (2^-40 units), so the
-// sums are exact and independent of the order of accumulation.
+// One CTA per (l, g) finds the candidate and kept prefixes with a block-wide
+// weighted radix select on the key (~bits(f) << 32 | t): three 11/11/10-bit
+// passes over the f part, then an ordered scan over t among the tokens of the
+// crossing f.  Token values enter the select as fixed-point integers (2^-40
+// units), so the sums are exact and independent of the order of
+// accumulation.  The acceptance walk takes the kept candidates 1024 at a time
+// in key order (the same select, by count), sorts each chunk in shared
+// memory, and one warp walks it against a bitmap of the accepted positions.
 #include "gkv_internal.cuh"
 
 #include <cfloat>
@@ -44,7 +48,7 @@ struct FloorArgs {
     unsigned long long eta_fx;
     long long cap;
 };
-enum { FH_CUT = 0, FH_N, FH_COST0, FH_KEEP, FH_CUTK, FH_FINAL, FH_USED, kFlHead };
+enum { FH_CUT = 0, FH_N, FH_COST0, FH_KEEP, FH_CUTK, FH_USED, kFlHead };
 enum { FG_C0 = 0, FG_NKEEP, FG_USED };
 
 __device__ __forceinline__ uint64_t fl_key(float f, int t) {
@@ -260,45 +264,123 @@ __global__ void __launch_bounds__(kFlThreads) floor_keep_kernel(FloorArgs a) {
     }
 }
 
-// Acceptance: the longest prefix of the kept candidates within the head's share.
-__global__ void __launch_bounds__(kFlThreads) floor_accept_kernel(FloorArgs a) {
-    __shared__ unsigned long long hist[2048], wsum[32], bc[4];
-    const int lg = blockIdx.x;
-    unsigned long long *h = a.head + (size_t)lg * kFlHead;
-    const float *f = a.f + (size_t)lg * a.Nc;
-    const unsigned long long keep = h[FH_KEEP], nkeep = a.glob[FG_NKEEP];
-    uint64_t cut = 0;          // nothing accepted
-    unsigned long long used = 0;
-    if (keep) {
-        const unsigned long long share = (unsigned long long)a.cap * keep / nkeep;
-        const uint64_t kcut = h[FH_CUTK];
-        const unsigned long long ck = block_joint_cost(a, f, kcut, wsum);
-        if (ck <= share) {
-            cut = kcut;
-            used = ck;
-        } else {
-            // largest m in [0, keep) whose m-token prefix fits (cost never decreases with m)
-            unsigned long long lo = 0, hi = keep;   // prefix lo fits, prefix hi does not
-            while (hi - lo > 1) {
-                const unsigned long long mid = (lo + hi) / 2;
-                const uint64_t c = block_wselect(f, a.Nc, kcut, mid, [](int) { return 1ull; }, hist, wsum, bc);
-                const unsigned long long cm = block_joint_cost(a, f, c, wsum);
-                if (cm <= share) lo = mid; else hi = mid;
-            }
-            cut = lo ? block_wselect(f, a.Nc, kcut, lo, [](int) { return 1ull; }, hist, wsum, bc) : 0;
-            used = lo ? block_joint_cost(a, f, cut, wsum) : 0;
+// Nearest accepted position of [lo, hi] (context-relative, lo <= hi) in the
+// bitmap: the largest one when from_top, else the smallest; -1 when none.
+// Called by a whole warp; every lane returns the same value.
+__device__ __forceinline__ int fl_nearest(const uint32_t *bits, int lo, int hi, bool from_top) {
+    const int lane = threadIdx.x & 31, wlo = lo >> 5, whi = hi >> 5;
+    const uint32_t mlo = ~0u << (lo & 31), mhi = (2u << (hi & 31)) - 1u;   // bits >= lo, <= hi
+    for (int w0 = from_top ? whi : wlo; from_top ? w0 >= wlo : w0 <= whi; w0 += from_top ? -32 : 32) {
+        const int w = from_top ? w0 - lane : w0 + lane;
+        uint32_t x = 0;
+        if (w >= wlo && w <= whi) {
+            x = bits[w];
+            if (w == wlo) x &= mlo;
+            if (w == whi) x &= mhi;
+        }
+        const unsigned bal = __ballot_sync(0xffffffffu, x != 0);
+        if (bal) {
+            const int src = __ffs(bal) - 1;          // the lane nearest the start
+            const uint32_t xs = __shfl_sync(0xffffffffu, x, src);
+            const int ws = from_top ? w0 - src : w0 + src;
+            return from_top ? ws * 32 + 31 - __clz(xs) : ws * 32 + __ffs(xs) - 1;
         }
     }
-    uint8_t *acc = a.acc + (size_t)lg * a.Nc;
-    for (int t = threadIdx.x; t < a.Nc; t += kFlThreads) acc[t] = fl_key(f[t], t) < cut ? 1 : 0;
+    return -1;
+}
+
+// Acceptance: walk the kept candidates in order (f descending, ties lower t);
+// accept each one whose path fits what is left of the head's share, skip the
+// others.  A candidate's path costs 1 for its slot's Add when no accepted
+// position is in the slot yet, plus one entry for each non-empty side of it
+// inside its current frontier interval (bounded by the nearest accepted
+// positions of the slot, else by the slot's ends).  Dynamic shared memory: the
+// accepted positions as a bitmap of ceil(N_c / 32) words.
+__global__ void __launch_bounds__(kFlThreads) floor_accept_kernel(FloorArgs a) {
+    __shared__ unsigned long long hist[2048], wsum[32], bc[4];
+    __shared__ int cnt;
+    extern __shared__ uint32_t acc_bits[];
+    const int lg = blockIdx.x, tid = threadIdx.x;
+    unsigned long long *h = a.head + (size_t)lg * kFlHead;
+    const float *f = a.f + (size_t)lg * a.Nc;
+    const int nw = (a.Nc + 31) >> 5;
+    for (int w = tid; w < nw; w += kFlThreads) acc_bits[w] = 0u;
+    const unsigned long long keep = h[FH_KEEP], nkeep = a.glob[FG_NKEEP];
+    const unsigned long long share = keep ? (unsigned long long)a.cap * keep / nkeep : 0ull;
+    const uint64_t kcut = h[FH_CUTK];
+    // the chunk lives in hist between two selects: keys, then slot bounds
+    uint64_t *ck = reinterpret_cast<uint64_t *>(hist);
+    int *ca = reinterpret_cast<int *>(hist + kFlThreads);
+    int *cb = ca + kFlThreads;
+    unsigned long long used = 0, done = 0;      // used: meaningful in warp 0
+    uint64_t lo_cut = 0;
     __syncthreads();
-    for (int j = threadIdx.x; j < a.J; j += kFlThreads) {
+    while (done < keep) {
+        const unsigned long long m = keep - done < (unsigned long long)kFlThreads ? keep - done
+                                                                                 : (unsigned long long)kFlThreads;
+        const uint64_t hi_cut = done + m >= keep
+            ? kcut : block_wselect(f, a.Nc, kcut, done + m, [](int) { return 1ull; }, hist, wsum, bc);
+        ck[tid] = ~0ull;
+        if (tid == 0) cnt = 0;
+        __syncthreads();
+        for (int t = tid; t < a.Nc; t += kFlThreads) {
+            const uint64_t k = fl_key(f[t], t);
+            if (k >= lo_cut && k < hi_cut) {
+                const int i = atomicAdd(&cnt, 1);
+                if (i < kFlThreads) ck[i] = k;
+            }
+        }
+        __syncthreads();
+        // bitonic sort of the chunk's keys, ascending (unused entries are ~0)
+        for (int k2 = 2; k2 <= kFlThreads; k2 <<= 1)
+            for (int j2 = k2 >> 1; j2 > 0; j2 >>= 1) {
+                const int ix = tid ^ j2;
+                if (ix > tid) {
+                    const uint64_t x = ck[tid], y = ck[ix];
+                    if ((x > y) == ((tid & k2) == 0)) { ck[tid] = y; ck[ix] = x; }
+                }
+                __syncthreads();
+            }
+        const int mc = min((int)m, min(cnt, kFlThreads));   // keys collected (m when the select is exact)
+        if (tid < mc) {
+            const int t = (int)(uint32_t)ck[tid];
+            int lo = 0, hi = a.J;                  // the last j with slots[j] - cs <= t
+            while (hi - lo > 1) {
+                const int mid = (lo + hi) >> 1;
+                if (a.slots[mid] - a.cs <= t) lo = mid; else hi = mid;
+            }
+            ca[tid] = a.slots[lo] - a.cs;
+            cb[tid] = a.slots[lo + 1] - a.cs;
+        }
+        __syncthreads();
+        if (tid < 32) {
+            for (int i = 0; i < mc; i++) {
+                const int t = (int)(uint32_t)ck[i], sa = ca[i], sb = cb[i];
+                const int left = t > sa ? fl_nearest(acc_bits, sa, t - 1, true) : -1;
+                const int right = t < sb - 1 ? fl_nearest(acc_bits, t + 1, sb - 1, false) : -1;
+                const int lo = left >= 0 ? left + 1 : sa, hi = right >= 0 ? right - 1 : sb - 1;
+                const unsigned long long cost =
+                    (left < 0 && right < 0 ? 1ull : 0ull) + (lo < t ? 1ull : 0ull) + (t < hi ? 1ull : 0ull);
+                if (used + cost <= share) {
+                    used += cost;
+                    if (tid == 0) acc_bits[t >> 5] |= 1u << (t & 31);
+                }
+                __syncwarp();
+            }
+        }
+        __syncthreads();
+        lo_cut = hi_cut;
+        done += m;
+    }
+    uint8_t *acc = a.acc + (size_t)lg * a.Nc;
+    for (int t = tid; t < a.Nc; t += kFlThreads) acc[t] = (uint8_t)((acc_bits[t >> 5] >> (t & 31)) & 1u);
+    for (int j = tid; j < a.J; j += kFlThreads) {
         uint8_t any = 0;
-        for (int t = a.slots[j] - a.cs; t < a.slots[j + 1] - a.cs && !any; t++) any = acc[t];
+        for (int t = a.slots[j] - a.cs; t < a.slots[j + 1] - a.cs && !any; t++)
+            any = (uint8_t)((acc_bits[t >> 5] >> (t & 31)) & 1u);
         a.u_floor[(size_t)lg * a.J + j] = any;
     }
-    if (threadIdx.x == 0) {
-        h[FH_FINAL] = cut;
+    if (tid == 0) {
         h[FH_USED] = used;
         if (used) atomicAdd(&a.glob[FG_USED], used);
     }
@@ -334,7 +416,10 @@ cudaError_t launch_floor(Ctx &c, int J, cudaStream_t s) {
     floor_score_kernel<<<dim3((a.Nc + 255) / 256, a.LG), 256, 0, s>>>(a);
     floor_cand_kernel<<<a.LG, kFlThreads, 0, s>>>(a);
     floor_keep_kernel<<<a.LG, kFlThreads, 0, s>>>(a);
-    floor_accept_kernel<<<a.LG, kFlThreads, 0, s>>>(a);
+    const size_t bits_bytes = sizeof(uint32_t) * (size_t)((a.Nc + 31) / 32);
+    e = cudaFuncSetAttribute(floor_accept_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bits_bytes);
+    if (e != cudaSuccess) return e;
+    floor_accept_kernel<<<a.LG, kFlThreads, bits_bytes, s>>>(a);
     c.launches += 5;
     return cudaGetLastError();
 }

@@ -126,6 +126,46 @@ def test_singleton_floor_matches_the_oracle(wname, alpha):
     print(wname, json.dumps(rep))
 
 
+def _floor_skip_case(seed=11):
+    # Token values by construction: keys lie along e_0 with logit c_t (plus
+    # small noise), every query is sqrt(d) e_0, no RoPE; so R_t is about
+    # exp(c_t) / sum exp(c) over the context.  Head 0's candidates in f order:
+    # 100 (uncovered slot [64, 128): 3 entries), 300 (uncovered slot [256,
+    # 320): 3), 101 (next to 100: 1).  Head 1's: 0, 1, 2 at the start of slot
+    # [0, 64): 2 + 1 + 1.  Joint cost 7 + 4 = 11 = cap = floor(0.115 B_free),
+    # B_free = 100, so no reduction; shares floor(11 * 3 / 6) = 5 each.
+    L, G, Hq, T, d, W = 1, 2, 2, 544, 64, 4
+    rng = np.random.default_rng(seed)
+    K = 0.05 * rng.normal(size=(L, G, T, d))
+    V = rng.normal(size=(L, G, T, d))
+    c = np.zeros((G, T))
+    c[0, [100, 300, 101]] = np.log([400.0, 300.0, 200.0])
+    c[1, [0, 1, 2]] = np.log([400.0, 300.0, 200.0])
+    K[0, :, :, 0] += c
+    Q = np.zeros((L, Hq, W, d))
+    Q[..., 0] = np.sqrt(d)
+    f32 = lambda a: torch.as_tensor(a, dtype=torch.float32)
+    return f32(K), f32(V), f32(Q), np.arange(0, 513, 64)
+
+
+def test_floor_skips_an_unaffordable_candidate_on_the_device():
+    # App. A.5 Stage I: a candidate is accepted only when its complete path
+    # still fits; head 0 skips 300 (3 + 3 > 5) and then accepts 101 (3 + 1)
+    K, V, Q, slots = _floor_skip_case()
+    kw = dict(slot_starts=slots, alpha_floor=0.115, floor_c=0.0, floor_half=0)
+    P, g, o = _run(K, V, Q, 164, 0.0, **kw)
+    ofl = o["floor"]
+    assert o["B_free"] == 100
+    assert set(np.nonzero(ofl["accepted"][0])[0]) == {100, 101}
+    assert set(np.nonzero(ofl["accepted"][1])[0]) == {0, 1, 2}
+    assert ofl["B_floor"] == 8
+    fl = g["comp"].ctx.gracekv_export_floor()
+    np.testing.assert_array_equal(fl["accepted"], ofl["accepted"])
+    assert fl["B_floor"] == ofl["B_floor"]
+    rep = P.compare(g, o, torch.float32)
+    print("floor skip", json.dumps(rep))
+
+
 @pytest.mark.parametrize("L,G,gq,d,D,U", [(3, 2, 4, 128, 1024, 32), (2, 8, 4, 128, 4096, 64),
                                           (4, 4, 1, 64, 520, 5)])
 def test_head_sensitivity_matches_the_oracle(L, G, gq, d, D, U):
