@@ -9,10 +9,12 @@ outputs the oracle computes one by one, and by properties that hold at any size:
   curvature      kappa at 256 sampled interior positions: the oracle on a
                  33-row slice around each position (the slice holds every
                  window, so the value equals the full-sequence one)
-  segmentation   the partition is valid and locally optimal: moving any of 160
-                 sampled boundaries by up to 8 tokens does not raise the DP
-                 objective beyond the near-tie margin (oracle edge weights; the
-                 boundary score is the oracle's robust z of the GPU curvature)
+  segmentation   every slot start equals the oracle's segmentation of the
+                 whole context (its three segmentation layers, the paper's
+                 prefix form of the dispersion), and curvature matches at all
+                 positions; also the partition is locally optimal: moving any
+                 of 160 sampled boundaries by up to 8 tokens does not raise the
+                 DP objective beyond the near-tie margin
   row stats      all 256 rows of one KV-head group over all 131072 keys
   token values   every compressible token of that group
   trees          24 sampled units of that group: topology (near-tie aware),
@@ -152,6 +154,44 @@ def test_segmentation_valid_and_locally_optimal(run):
         worst = max(worst, gap)
         assert gap < P.NEAR_TIE, (j, s0, s1, s2, obj)
     print("largest relative improvement found", worst)
+
+
+def test_segmentation_bit_exact_over_the_full_context(run):
+    # The oracle's segmentation of the whole 131072-token context from the
+    # three segmentation layers (the partition depends on nothing else), in
+    # the paper's prefix form of the dispersion (App. B.3 Eq.
+    # app_prefix_dispersion, pinned equal to the sample-variance definition
+    # on CPU).  Every slot start must match; a differing DP decision is
+    # allowed only at an endpoint where the oracle's best and second-best
+    # predecessor values are within the near-tie margin.
+    import time
+    t0 = time.time()
+    V = run["Vseg"].double().cpu().numpy()
+    p = O.make_params(3, run["G"], run["Hq"], run["T"], run["d"], run["W"], run["w"].rope_base,
+                      seg_layers=(0, 1, 2), recent=run["r"], disp_mode=1)
+    seg = O.segment(p, V)
+    del V
+    kerr = float(np.abs(seg["kappa"] - run["kappa"]).max())
+    og, gs = seg["slot_starts"].astype(np.int64), run["slots"]
+    print(f"full-context segmentation: oracle {time.time() - t0:.0f} s, {len(og) - 1} slots, "
+          f"kappa max abs err {kerr:.2e} over all {run['T']} positions")
+    assert kerr <= P.KAPPA_ATOL
+    if np.array_equal(og, gs):
+        return
+    # the decision that differs: the last endpoint both paths reach, going
+    # back from N, whose predecessors differ
+    so, sg = set(og.tolist()), set(gs.tolist())
+    common = sorted(so & sg)
+    for i in reversed(common[1:]):
+        po = og[np.searchsorted(og, i) - 1]
+        pg = gs[np.searchsorted(gs, i) - 1]
+        if po != pg:
+            best, second = seg["dp_best"][i], seg["dp_second"][i]
+            margin = abs(best - second) / max(abs(best), 1e-300)
+            print("slot starts differ at endpoint", i, "oracle margin", margin)
+            assert margin < P.NEAR_TIE, (i, po, pg, margin)
+            return
+    raise AssertionError("slot starts differ")
 
 
 def _group_rows(run, key):
