@@ -210,9 +210,12 @@ gkv_status gracekv_score(gracekv_ctx *ctx, const void *K, const void *Q, void *s
  * lambda_graph > 0 the multi-hop relevance (App. A.4) mixes into them, from
  * the queries of the last gracekv_set_graph_queries; with alpha_floor > 0
  * the singleton floor (App. A.5 Stage I) is chosen from the (mixed) values;
- * then the trees are built, floor positions extracted first.  Errors:
- * GKV_EINVAL (also: lambda_graph > 0 without graph queries), GKV_ESTATE,
- * GKV_EUNSUPPORTED (a slot longer than 128 tokens), GKV_ECUDA.
+ * then the trees are built, floor positions extracted first.  A supplied
+ * slot may hold 1 to 16384 tokens (the segmentation's hold n_min..n_max);
+ * every tree recurses to single-token leaves whatever its slot's length.
+ * Errors: GKV_EINVAL (also: lambda_graph > 0 without graph queries, supplied
+ * slots that do not partition the region), GKV_ESTATE, GKV_EUNSUPPORTED (a
+ * supplied slot longer than 16384 tokens), GKV_ENOMEM, GKV_ECUDA.
  */
 gkv_status gracekv_build_trees(gracekv_ctx *ctx, const void *K, const void *V, const void *Q,
                                const float *omega, const int32_t *slot_starts, int32_t n_slots,

@@ -264,7 +264,6 @@ __global__ void __launch_bounds__(1024) alloc_ties_kernel(AllocArgs A) {
     __shared__ int list[1024];
     __shared__ int nlist;
     __shared__ long long Rs;
-    __shared__ short parent[2 * kMaxUnit];
     const int seg = blockIdx.x;
     unsigned long long *st = seg_st(A, seg);
     const long long Bseg = seg_budget(A, seg);
@@ -304,11 +303,11 @@ __global__ void __launch_bounds__(1024) alloc_ties_kernel(AllocArgs A) {
                 int64_t u = base + list[q];
                 int64_t nb = unit_base(A, u);
                 int nn = A.u_nnodes[u];
-                for (int k = 0; k < nn; k++) parent[k] = -1;
-                for (int k = 0; k < nn; k++) {
-                    int c0 = A.nd_child0[nb + k], nc = A.nd_nchild[nb + k];
-                    for (int x = 0; x < nc; x++) parent[c0 + x] = (short)k;
-                }
+                // the parent of local node k: -1 for the root (parent index -2 - unit)
+                auto parent_of = [&](int k) {
+                    const int32_t pg = A.nd_parent[nb + k];
+                    return pg < 0 ? -1 : (int)(pg - nb);
+                };
                 // the unit's queue restricted to tie ops; -1 stands for the Add
                 for (;;) {
                     int best = -2;
@@ -322,7 +321,8 @@ __global__ void __launch_bounds__(1024) alloc_ties_kernel(AllocArgs A) {
                         int64_t v = nb + k;
                         if (A.nd_cost[v] <= 0 || A.nd_sel[v] != 0) continue;
                         if (__float_as_uint(A.nd_kappa[v]) != tau) continue;
-                        bool exposed = parent[k] < 0 ? A.u_sel[u] == 1 : A.nd_sel[nb + parent[k]] == 1;
+                        const int pk = parent_of(k);
+                        bool exposed = pk < 0 ? A.u_sel[u] == 1 : A.nd_sel[nb + pk] == 1;
                         if (!exposed) continue;
                         float uu = A.nd_U[v];
                         int aa = A.nd_a[v], bbb = A.nd_b[v];
@@ -466,7 +466,7 @@ int grid_for(const Ctx &c, int64_t n) {
 // every op built so far fits the budget).
 __global__ void prune_list_kernel(const float *u_pend, const int32_t *slots, int J, int64_t n_units,
                                   const unsigned long long *st, const float *cut, int32_t *list,
-                                  int *count, unsigned long long *potential) {
+                                  int *count, int32_t *long_list, unsigned long long *potential) {
     int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= n_units) return;
     float p = u_pend[i];
@@ -479,8 +479,10 @@ __global__ void prune_list_kernel(const float *u_pend, const int32_t *slots, int
     }
     if (above && p >= *cut) {
         const int j = (int)(i % J);
-        if (slots[j + 1] - slots[j] <= kShortUnit) list[atomicAdd(count, 1)] = (int32_t)i;
-        else list[n_units - 1 - atomicAdd(count + 1, 1)] = (int32_t)i;
+        const int n = slots[j + 1] - slots[j];
+        if (n <= kShortUnit) list[atomicAdd(count, 1)] = (int32_t)i;
+        else if (n <= kMaxUnit) list[n_units - 1 - atomicAdd(count + 1, 1)] = (int32_t)i;
+        else long_list[atomicAdd(count + 2, 1)] = (int32_t)i;
     }
 }
 
@@ -536,11 +538,17 @@ __global__ void __launch_bounds__(1024) pend_cut_kernel(const unsigned int *hist
     if (tid == 1023 && before + own < (unsigned)m) *cut = -INFINITY;   // fewer than m qualify: no cut
 }
 
-__global__ void slot_classes_kernel(const int32_t *slots, int J, int32_t *list, int *count) {
+__global__ void slot_classes_kernel(const int32_t *slots, int J, int32_t *list, int *count,
+                                    int32_t *long_slots) {
     int j = blockIdx.x * blockDim.x + threadIdx.x;
     if (j >= J) return;
-    if (slots[j + 1] - slots[j] <= kShortUnit) list[atomicAdd(count, 1)] = j;
-    else list[J - 1 - atomicAdd(count + 1, 1)] = j;
+    const int n = slots[j + 1] - slots[j];
+    if (n <= kShortUnit) list[atomicAdd(count, 1)] = j;
+    else if (n <= kMaxUnit) list[J - 1 - atomicAdd(count + 1, 1)] = j;
+    else {
+        long_slots[atomicAdd(count + 2, 1)] = j;
+        atomicAdd(count + 3, n);
+    }
 }
 
 }  // namespace
@@ -565,14 +573,14 @@ cudaError_t launch_threshold(Ctx &c, int J, cudaStream_t s) {
 }
 
 cudaError_t launch_prune_list(Ctx &c, const int32_t *slots, int J, int32_t *list, int *count,
-                              cudaStream_t s) {
+                              int32_t *long_list, cudaStream_t s) {
     const int64_t nu = (int64_t)c.p.L * c.p.G * J;
-    cudaError_t e = cudaMemsetAsync(count, 0, 2 * sizeof(int), s);
+    cudaError_t e = cudaMemsetAsync(count, 0, 3 * sizeof(int), s);
     if (e == cudaSuccess) e = cudaMemsetAsync(c.w.pend_pot, 0, sizeof(unsigned long long), s);
     if (e != cudaSuccess) return e;
     prune_list_kernel<<<(unsigned)((nu + 255) / 256), 256, 0, s>>>(c.w.u_pend, slots, J, nu,
                                                                     c.w.alloc_state, c.w.pend_cut, list,
-                                                                    count, c.w.pend_pot);
+                                                                    count, long_list, c.w.pend_pot);
     c.launches += 1;
     return cudaGetLastError();
 }
@@ -589,10 +597,10 @@ cudaError_t launch_pend_cut(Ctx &c, int J, int m, float *cut, unsigned int *n_qu
 }
 
 cudaError_t launch_slot_classes(Ctx &c, const int32_t *slots, int J, int32_t *list, int *count,
-                                cudaStream_t s) {
-    cudaError_t e = cudaMemsetAsync(count, 0, 2 * sizeof(int), s);
+                                int32_t *long_slots, cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(count, 0, 4 * sizeof(int), s);
     if (e != cudaSuccess) return e;
-    slot_classes_kernel<<<(J + 255) / 256, 256, 0, s>>>(slots, J, list, count);
+    slot_classes_kernel<<<(J + 255) / 256, 256, 0, s>>>(slots, J, list, count, long_slots);
     c.launches += 1;
     return cudaGetLastError();
 }

@@ -20,7 +20,7 @@ namespace {
 
 // Device status bits (dev_int[1]).
 enum : int { ST_NONFINITE_KAPPA = 1, ST_NONFINITE_ROWS = 2, ST_LONG_SLOT = 4, ST_NONFINITE_GAIN = 8,
-             ST_BAD_SLOTS = 16, ST_PIPE_TIMEOUT = gkv::kStPipeTimeout };
+             ST_BAD_SLOTS = 16, ST_PIPE_TIMEOUT = gkv::kStPipeTimeout, ST_LONG_CAP = gkv::kStLongCap };
 
 gkv_status fail(gracekv_ctx *x, gkv_status s, const char *msg) {
     if (x) {
@@ -53,8 +53,9 @@ bool dalloc(gracekv_ctx *x, T **p, size_t n) {
 
 gkv_status check_status(gracekv_ctx *x, int st) {
     if (st & ST_PIPE_TIMEOUT) return fail(x, GKV_ECUDA, "a tensor-core pipeline wait timed out");
-    if (st & ST_BAD_SLOTS) return fail(x, GKV_EINVAL, "supplied slot starts are not a partition of [c_s, c_e - r) into slots of 1..128 tokens");
-    if (st & ST_LONG_SLOT) return fail(x, GKV_EUNSUPPORTED, "a slot is longer than 128 tokens (unit kernel limit)");
+    if (st & ST_BAD_SLOTS) return fail(x, GKV_EINVAL, "supplied slot starts are not a partition of [c_s, c_e - r) into non-empty slots");
+    if (st & ST_LONG_SLOT) return fail(x, GKV_EUNSUPPORTED, "a slot is longer than 16384 tokens");
+    if (st & ST_LONG_CAP) return fail(x, GKV_ENOMEM, "long-unit work items exceeded their capacity");
     if (st & ST_NONFINITE_KAPPA) return fail(x, GKV_ENONFINITE, "non-finite curvature (NaN/Inf in the trajectory)");
     if (st & ST_NONFINITE_ROWS) return fail(x, GKV_ENONFINITE, "non-finite attention row statistics (NaN/Inf in K or Q)");
     if (st & ST_NONFINITE_GAIN) return fail(x, GKV_ENONFINITE, "non-finite gain (NaN/Inf in K, V, Q or omega)");
@@ -74,7 +75,7 @@ __global__ void validate_slots_kernel(const int32_t *s, int J, int cs, int cend,
     int a = s[j], b = s[j + 1];
     bool bad = b - a < 1 || (j == 0 && a != cs) || (j == J - 1 && b != cend);
     if (bad) atomicOr(status, ST_BAD_SLOTS);
-    else if (b - a > gkv::kMaxUnit) atomicOr(status, ST_LONG_SLOT);
+    else if (b - a > gkv::kMaxSlot) atomicOr(status, ST_LONG_SLOT);
 }
 
 }  // namespace
@@ -245,7 +246,8 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
     const int64_t nrow = (int64_t)p.L * p.Hq * p.W;
     gkv::Workspace &w = c.w;
     bool ok = dalloc(x, &w.rope, (size_t)p.T * (p.d / 2)) &&
-              dalloc(x, &w.rope_rel, (size_t)(2 * gkv::kMaxUnit - 1) * (p.d / 2)) &&
+              dalloc(x, &w.rope_rel, (size_t)(2 * gkv::kMaxSlot - 1) * (p.d / 2)) &&
+              dalloc(x, &w.long_slots, (size_t)Nc + 2) && dalloc(x, &w.long_n, 1) &&
               dalloc(x, &w.ent, (size_t)p.budget + (size_t)p.L * p.G * (p.T - Nc)) &&
               dalloc(x, &w.inv_norm, (size_t)c.nseg * p.T) &&
               dalloc(x, &w.nrm2, (size_t)c.nseg * p.T) &&
@@ -461,6 +463,7 @@ static gkv_status build_setup(gracekv_ctx *x, const int32_t *slot_starts, int32_
                   dalloc(x, &w.u_count, cap) && dalloc(x, &w.u_off, cap) &&
                   dalloc(x, &w.u_pend, cap) && dalloc(x, &w.u_list, cap) &&
                   (c.p.alpha_floor <= 0.0 || dalloc(x, &w.u_floor, cap)) &&
+                  dalloc(x, &w.long_list, cap) &&
                   dalloc(x, &w.u_bsum, cap / 1024 + 2);
         if (!ok) return fail(x, GKV_ENOMEM, "build_trees: unit arrays");
         w.units_cap = cap;
@@ -469,8 +472,9 @@ static gkv_status build_setup(gracekv_ctx *x, const int32_t *slot_starts, int32_
 }
 
 // Work counters and the op list cleared; slots split into the short and long
-// classes of the unit kernel (cnt: their sizes, synchronises s).
-static cudaError_t build_classes(Ctx &c, int cnt[2], cudaStream_t s) {
+// classes of the unit kernel and the long units (cnt: their sizes and the
+// long units' tokens; synchronises s).
+static cudaError_t build_classes(Ctx &c, int cnt[4], cudaStream_t s) {
     gkv::Workspace &w = c.w;
     const int64_t nu = (int64_t)c.p.L * c.p.G * c.J;
     static const float kNoCut = -INFINITY;
@@ -478,19 +482,57 @@ static cudaError_t build_classes(Ctx &c, int cnt[2], cudaStream_t s) {
     if (!(c.B_free < nu)) e = cudaMemcpyAsync(w.pend_cut, &kNoCut, sizeof(float), cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = cudaMemsetAsync(w.work, 0, 4 * sizeof(unsigned long long), s);
     if (e == cudaSuccess) e = cudaMemsetAsync(w.n_ops, 0, sizeof(unsigned int), s);
-    cnt[0] = cnt[1] = 0;
+    cnt[0] = cnt[1] = cnt[2] = cnt[3] = 0;
     if (e == cudaSuccess) {
         gkv::StageTimer tm(c, 3, s);
-        e = gkv::launch_slot_classes(c, w.slots, c.J, w.u_list, w.dev_int + 2, s);
+        e = gkv::launch_slot_classes(c, w.slots, c.J, w.u_list, w.dev_int + 2, w.long_slots, s);
     }
-    if (e == cudaSuccess) e = cudaMemcpyAsync(cnt, w.dev_int + 2, 2 * sizeof(int), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(cnt, w.dev_int + 2, 4 * sizeof(int), cudaMemcpyDeviceToHost, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    return e;
+}
+
+// The classes, and the work-item arrays of the long units sized for them: a
+// level's items of one unit are disjoint intervals of >= 2 tokens, so at most
+// n / 2 of them (or its root).
+static gkv_status classes(gracekv_ctx *x, int cnt[4], cudaStream_t s) {
+    Ctx &c = x->c;
+    gkv::Workspace &w = c.w;
+    cudaError_t e = build_classes(c, cnt, s);
+    if (e != cudaSuccess) return cuda_fail(x, e, "build_trees classes");
+    c.n_long = cnt[2];
+    if (cnt[2] == 0) return GKV_OK;
+    const int64_t LG = (int64_t)c.p.L * c.p.G;
+    const int64_t items = LG * ((int64_t)cnt[3] / 2 + cnt[2]) + 16, units = LG * cnt[2];
+    if (items > w.long_cap) {
+        bool ok = dalloc(x, &w.long_gv, items) && dalloc(x, &w.long_uid, items) &&
+                  dalloc(x, &w.long_kin, items) && dalloc(x, &w.long_ufl, items) &&
+                  dalloc(x, reinterpret_cast<unsigned char **>(&w.long_res), items * gkv::long_res_bytes());
+        if (!ok) return fail(x, GKV_ENOMEM, "build_trees: long-unit work items");
+        w.long_cap = items;
+    }
+    if (units > w.long_units_cap) {
+        if (!(dalloc(x, &w.long_start, units) && dalloc(x, &w.long_cnt, units)))
+            return fail(x, GKV_ENOMEM, "build_trees: long-unit lists");
+        w.long_units_cap = units;
+    }
+    return GKV_OK;
+}
+
+// Long units (build_long.cu): further levels of the listed units, every
+// pending node at once, until none is left.
+static cudaError_t long_to_leaves(Ctx &c, const void *K, const void *V, const void *Q, const float *omega,
+                                  const int32_t *units, int n_units, cudaStream_t s) {
+    cudaError_t e = cudaSuccess;
+    for (unsigned int items = 1; e == cudaSuccess && items > 0;)
+        e = gkv::launch_long_level(c, K, V, Q, omega, c.w.slots, c.J, 0, 0, -INFINITY, units, n_units, 0, -1, s,
+                                   &items);
     return e;
 }
 
 // The first tree-building launch of the units of (l, g) in [lg0, lg0 + nlg).
 static cudaError_t build_fresh(Ctx &c, const void *K, const void *V, const void *Q, const float *omega,
-                               const int cnt[2], int lg0, int nlg, cudaStream_t s) {
+                               const int cnt[4], int lg0, int nlg, cudaStream_t s) {
     gkv::Workspace &w = c.w;
     const int64_t nu = (int64_t)c.p.L * c.p.G * c.J;
     // with per-(l, g) capacities ("w/o GA") the global threshold cannot prune:
@@ -498,8 +540,16 @@ static cudaError_t build_fresh(Ctx &c, const void *K, const void *V, const void 
     const bool full = c.p.quota_alloc != 0;
     const bool root_only = !full && c.B_free < nu;
     gkv::StageTimer tm(c, 3, s);
-    return gkv::launch_unit_build(c, K, V, Q, omega, w.slots, c.J, 0, root_only ? 1 : 0, full ? 4 * gkv::kMaxUnit : 1,
-                                  0.f, w.u_list, cnt[0], w.u_list + (c.J - cnt[1]), cnt[1], s, lg0, nlg);
+    cudaError_t e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, c.J, 0, root_only ? 1 : 0,
+                                           full ? 4 * gkv::kMaxUnit : 1, 0.f, w.u_list, cnt[0],
+                                           w.u_list + (c.J - cnt[1]), cnt[1], s, lg0, nlg);
+    if (e != cudaSuccess || cnt[2] == 0) return e;
+    e = gkv::launch_long_level(c, K, V, Q, omega, w.slots, c.J, 1, root_only ? 1 : 0, 0.f, w.long_slots, cnt[2],
+                               lg0, nlg, s, nullptr);
+    if (e != cudaSuccess || !full) return e;
+    e = gkv::launch_long_units(c, w.long_slots, cnt[2], lg0, nlg, c.J, w.long_list, s);
+    if (e != cudaSuccess) return e;
+    return long_to_leaves(c, K, V, Q, omega, w.long_list, cnt[2] * nlg, s);
 }
 
 // Trees (build.cu).  Every op's key is bounded before it is built: a pending
@@ -524,18 +574,18 @@ static cudaError_t build_passes(Ctx &c, const void *K, const void *V, const void
     cudaError_t e = cudaSuccess;
     for (int it = 0; e == cudaSuccess; it++) {
         struct {
-            int count[2];
+            int count[3];
             unsigned long long prefix, all, total, pot;
             float cut;
             unsigned int nqual;
-        } h = {{0, 0}, 0, 0, 0, 0, 0.f, 0};
+        } h = {{0, 0, 0}, 0, 0, 0, 0, 0.f, 0};
         {
             gkv::StageTimer tm(c, 3, s);
             e = gkv::launch_threshold(c, J, s);
             if (e == cudaSuccess && root_only) e = gkv::launch_pend_cut(c, J, pass_units, w.pend_cut, w.pend_n, s);
-            if (e == cudaSuccess) e = gkv::launch_prune_list(c, w.slots, J, w.u_list, w.dev_int + 2, s);
+            if (e == cudaSuccess) e = gkv::launch_prune_list(c, w.slots, J, w.u_list, w.dev_int + 2, w.long_list, s);
         }
-        if (e == cudaSuccess) e = cudaMemcpyAsync(h.count, w.dev_int + 2, 2 * sizeof(int), cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(h.count, w.dev_int + 2, 3 * sizeof(int), cudaMemcpyDeviceToHost, s);
         if (e == cudaSuccess) e = cudaMemcpyAsync(&h.prefix, w.alloc_state, 2 * sizeof(unsigned long long),
                                                   cudaMemcpyDeviceToHost, s);
         if (e == cudaSuccess) e = cudaMemcpyAsync(&h.all, w.alloc_state + 2, sizeof(unsigned long long),
@@ -547,7 +597,7 @@ static cudaError_t build_passes(Ctx &c, const void *K, const void *V, const void
         if (e == cudaSuccess) e = cudaMemcpyAsync(&h.pot, w.pend_pot, sizeof(unsigned long long),
                                                   cudaMemcpyDeviceToHost, s);
         if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-        if (e != cudaSuccess || h.count[0] + h.count[1] == 0) break;
+        if (e != cudaSuccess || h.count[0] + h.count[1] + h.count[2] == 0) break;
         uint32_t bits = (uint32_t)h.prefix;
         float tau;
         memcpy(&tau, &bits, sizeof tau);
@@ -559,6 +609,11 @@ static cudaError_t build_passes(Ctx &c, const void *K, const void *V, const void
         gkv::StageTimer tm(c, 3, s);
         e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 1, 0, levels, tau_eff, w.u_list,
                                    h.count[0], w.u_list + (nu - h.count[1]), h.count[1], s);
+        if (e == cudaSuccess && h.count[2] > 0) {   // long units: one level, or all of them when they fit
+            e = gkv::launch_long_level(c, K, V, Q, omega, w.slots, J, 0, 0, tau_eff, w.long_list, h.count[2], 0, -1,
+                                       s, nullptr);
+            if (e == cudaSuccess && fits) e = long_to_leaves(c, K, V, Q, omega, w.long_list, h.count[2], s);
+        }
         c.build_passes = it + 2;
     }
     return e;
@@ -596,7 +651,7 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
         }
     }
     c.scored = false;
-    int cnt[2];
+    int cnt[4];
     if (e == cudaSuccess && c.p.lambda_graph > 0.0) {   // R = (1 - lambda) s-hat + lambda d-hat
         if (!c.mh_Qg) return fail(x, GKV_EINVAL, "build_trees: multi-hop relevance needs gracekv_set_graph_queries");
         c.mh_K = K;
@@ -607,8 +662,10 @@ gkv_status gracekv_build_trees(gracekv_ctx *x, const void *K, const void *V, con
         gkv::StageTimer tm(c, 6, s);
         e = gkv::launch_floor(c, c.J, s);
     }
-    if (e == cudaSuccess) e = build_classes(c, cnt, s);
-    if (e == cudaSuccess) e = build_fresh(c, K, V, Q, omega, cnt, 0, c.p.L * c.p.G, s);
+    if (e != cudaSuccess) return cuda_fail(x, e, "build_trees launch");
+    st = classes(x, cnt, s);
+    if (st) return st;
+    e = build_fresh(c, K, V, Q, omega, cnt, 0, c.p.L * c.p.G, s);
     if (e == cudaSuccess) e = build_passes(c, K, V, Q, omega, s);
     if (e != cudaSuccess) return cuda_fail(x, e, "build_trees launch");
     c.stage = 2;
@@ -700,9 +757,11 @@ gkv_status gracekv_compress_host(gracekv_ctx *x, const void *K, const void *V, c
     if (st) return st;
     st = build_setup(x, nullptr, 0, s);
     if (st) return st;
-    int cnt[2];
+    int cnt[4];
     e = cudaMemsetAsync(c.w.dev_int + gkv::kScoreStatus, 0, sizeof(int), s);
-    if (e == cudaSuccess) e = build_classes(c, cnt, s);
+    if (e != cudaSuccess) return cuda_fail(x, e, "compress_host");
+    st = classes(x, cnt, s);
+    if (st) return st;
     // per layer group, once it is in: score passes and the first tree-building launch
     const bool ranged = gkv::use_tc(c);
     const bool fl = p.alpha_floor > 0.0;   // the floor needs every (l, g)'s token values first

@@ -28,10 +28,10 @@ struct GatherArgs {
     const void *K, *V;
     const float *rtok;
     const float2 *rope;
-    const float2 *rope_rel;    // [2 kMaxUnit - 1][d/2]: rotation by the offset p - t
+    const float2 *rope_rel;    // [2 kMaxSlot - 1][d/2]: rotation by the offset p - t
     int4 *ent;                 // [entries]: (a, b, lg, 1) of every frontier entry, by output position
     const int32_t *slots;
-    const int32_t *nd_a, *nd_b, *nd_child0;
+    const int32_t *nd_a, *nd_b, *nd_child0, *nd_parent;
     const int8_t *nd_nchild;
     const uint8_t *nd_sel, *u_sel;
     const int32_t *u_nnodes;
@@ -243,6 +243,7 @@ __global__ void gather_list_kernel(GatherArgs A) {
     const int64_t uid = (int64_t)blockIdx.x * 8 + warp;
     if (uid >= nu || A.u_sel[uid] != 1 || lane != 0) return;
     const int lg = (int)(uid / A.J), j = (int)(uid - (int64_t)lg * A.J);
+    if (A.slots[j + 1] - A.slots[j] > kMaxUnit) return;   // a long unit: gather_list_long
     const int64_t nb = node_base(lg, A.slots[j], A.cs, A.Nc);
     int64_t e = A.u_off[uid];
     short *st = stack[warp];
@@ -260,6 +261,65 @@ __global__ void gather_list_kernel(GatherArgs A) {
     }
 }
 
+// The same for the units of slots longer than kMaxUnit (CTA per unit): a node
+// is a frontier entry when it is reached (the root with its Add selected, or a
+// child of a selected split) and its own split is not selected; the entries of
+// a unit are disjoint intervals, so an entry's output rank is the number of
+// entry starts before its own, counted over a bitmap of the slot's positions.
+__global__ void __launch_bounds__(256) gather_list_long_kernel(GatherArgs A, const int32_t *long_slots) {
+    __shared__ uint32_t bits[kMaxSlot / 32];
+    __shared__ int wpre[kMaxSlot / 32];
+    __shared__ int warp_tot[8];
+    const int LG = A.L * A.G;
+    const int lg = blockIdx.x % LG, j = long_slots[blockIdx.x / LG];
+    const int64_t uid = (int64_t)lg * A.J + j;
+    if (A.u_sel[uid] != 1) return;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int sa = A.slots[j], n = A.slots[j + 1] - sa;
+    const int nw = (n + 31) / 32;
+    const int64_t nb = node_base(lg, sa, A.cs, A.Nc);
+    const int nn = A.u_nnodes[uid];
+    for (int w = tid; w < nw; w += 256) bits[w] = 0u;
+    __syncthreads();
+    auto frontier = [&](int k) {
+        const int64_t v = nb + k;
+        if (A.nd_sel[v] == 1) return false;
+        const int32_t pg = A.nd_parent[v];
+        return pg < 0 ? true : A.nd_sel[pg] == 1;   // the root is reached: its Add is selected
+    };
+    for (int k = tid; k < nn; k += 256)
+        if (frontier(k)) {
+            const int off = A.nd_a[nb + k] - sa;
+            atomicOr(&bits[off >> 5], 1u << (off & 31));
+        }
+    __syncthreads();
+    // exclusive prefix of the set bits in word order (thread t: words 2 t, 2 t + 1)
+    const int w0 = 2 * tid;
+    const int c0 = w0 < nw ? __popc(bits[w0]) : 0, c1 = w0 + 1 < nw ? __popc(bits[w0 + 1]) : 0;
+    const int x = c0 + c1;
+    int incl = x;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) warp_tot[warp] = incl;
+    __syncthreads();
+    int before = 0;
+    for (int w = 0; w < warp; w++) before += warp_tot[w];
+    const int ex = before + incl - x;
+    if (w0 < nw) wpre[w0] = ex;
+    if (w0 + 1 < nw) wpre[w0 + 1] = ex + c0;
+    __syncthreads();
+    const int64_t e0 = A.u_off[uid];
+    for (int k = tid; k < nn; k += 256)
+        if (frontier(k)) {
+            const int off = A.nd_a[nb + k] - sa;
+            const int rank = wpre[off >> 5] + __popc(bits[off >> 5] & ((1u << (off & 31)) - 1u));
+            A.ent[e0 + rank] = make_int4(A.nd_a[nb + k], A.nd_b[nb + k], lg, 1);
+        }
+}
+
 // Prototypes of the listed entries (one warp per entry; rows read as
 // 8-element chunks, LPR = d / 8 lanes per row and RPW = 32 / LPR rows per step).
 // Each warp walks its entries (warp id, + number of warps, ...) as one stream of
@@ -269,7 +329,7 @@ __global__ void gather_list_kernel(GatherArgs A) {
 // boundaries.  Lane c of a row holds the key's rotation pairs (i, i + d/2) for
 // i = 4 c .. 4 c + 3 and the value elements 8 c .. 8 c + 7.  The key prototype RoPE(mean_t RoPE^-1(k_t, t),
 // p) is formed as mean_t of k_t rotated by p - t (rotations compose), from a
-// table of the 2 n_max - 1 offsets; its norm equals the norm of the mean
+// table of the offsets -(kMaxSlot - 1) .. kMaxSlot - 1; its norm equals the norm of the mean
 // inverse-rotated key.  The value prototype uses sum_t (R_t + beta) v_t =
 // sum R v + beta sum v.  All arithmetic is fp32.
 constexpr int kRingSteps = 8;
@@ -378,7 +438,7 @@ __global__ void __launch_bounds__(256, 2) gather_emit_kernel(GatherArgs A, int64
                 if (c == 0) kn += sqrtf(nn);   // |k_t|
                 rs += rr;
                 const float4 *cs4 = reinterpret_cast<const float4 *>(
-                    A.rope_rel + (size_t)(p - tt + kMaxUnit - 1) * HALF + i0);
+                    A.rope_rel + (size_t)(p - tt + kMaxSlot - 1) * HALF + i0);
 #pragma unroll
                 for (int j2 = 0; j2 < 2; j2++) {
                     const float4 q = cs4[j2];          // (cos, sin) of pairs i0 + 2 j2, i0 + 2 j2 + 1
@@ -491,7 +551,8 @@ cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *s
     GatherArgs A;
     A.K = K; A.V = V; A.rtok = c.w.rtok; A.rope = c.w.rope; A.rope_rel = c.w.rope_rel; A.ent = c.w.ent;
     A.slots = slots;
-    A.nd_a = c.w.nd_a; A.nd_b = c.w.nd_b; A.nd_child0 = c.w.nd_child0; A.nd_nchild = c.w.nd_nchild;
+    A.nd_a = c.w.nd_a; A.nd_b = c.w.nd_b; A.nd_child0 = c.w.nd_child0; A.nd_parent = c.w.nd_parent;
+    A.nd_nchild = c.w.nd_nchild;
     A.nd_sel = c.w.nd_sel; A.u_sel = c.w.u_sel; A.u_nnodes = c.w.u_nnodes;
     A.u_count = c.w.u_count; A.u_off = c.w.u_off;
     A.L = c.p.L; A.G = c.p.G; A.T = c.p.T; A.d = c.p.d; A.J = J; A.cs = c.p.ctx_start;
@@ -516,6 +577,10 @@ cudaError_t launch_gather(Ctx &c, const void *K, const void *V, const int32_t *s
     if (me != cudaSuccess) return me;
     if (gu) {
         gather_list_kernel<<<gu, 256, 0, s>>>(A);
+        if (c.n_long > 0) {
+            gather_list_long_kernel<<<(unsigned)(c.n_long * c.p.L * c.p.G), 256, 0, s>>>(A, c.w.long_slots);
+            c.launches += 1;
+        }
         cudaError_t le;
         if (c.p.d == 128) {
             if (bf) le = launch_emit<__nv_bfloat16, 128>(c, A, n_ent, s);

@@ -13,9 +13,11 @@
 
 namespace gkv {
 
-constexpr int kMaxUnit = 128;
+constexpr int kMaxUnit = 128;       // longest slot a unit kernel holds in shared memory
+constexpr int kMaxSlot = 16384;     // longest slot of a supplied partition (longer ones: long units, build_long.cu)
 constexpr int kStPipeTimeout = 32;   // status bit: a bounded wait of a tensor-core pipeline gave up
-constexpr int kScoreStatus = 8;      // dev_int word of the score passes' status bits      // longest slot a unit kernel holds in shared memory
+constexpr int kStLongCap = 64;       // status bit: the long-unit work items exceeded their capacity
+constexpr int kScoreStatus = 8;      // dev_int word of the score passes' status bits
 constexpr int kMaxSegLayers = 8;
 constexpr int kMaxWindows = 4;
 
@@ -25,7 +27,7 @@ constexpr int kMaxWindows = 4;
 struct Workspace {
     // RoPE rotation table: (cos, sin)(t * theta_i) for t in [0, T), i < d/2.
     float2 *rope = nullptr;
-    float2 *rope_rel = nullptr;    // [2 kMaxUnit - 1][d/2] rotations by the offsets -(kMaxUnit-1)..kMaxUnit-1
+    float2 *rope_rel = nullptr;    // [2 kMaxSlot - 1][d/2] rotations by the offsets -(kMaxSlot-1)..kMaxSlot-1
     int4 *ent = nullptr;           // [B_total + L G (T - N_c)] frontier entry descriptors of the gather
     // segmentation
     float *inv_norm = nullptr;     // [n_seg][T] 1 / max(||h_t||, eps)
@@ -97,6 +99,18 @@ struct Workspace {
     float *pend_cut = nullptr;                 // [1] lower bound of the next pass
     unsigned int *pend_n = nullptr;            // [1] units that reach the threshold
     unsigned long long *pend_pot = nullptr;    // [1] entries a full expansion of those units could take
+    // trees of long units (slots above kMaxUnit tokens, build_long.cu): one
+    // level's work items, per listed unit its block of them, the unit lists
+    int64_t long_cap = 0;          // work items
+    int64_t long_units_cap = 0;    // listed units
+    int64_t *long_gv = nullptr, *long_uid = nullptr;
+    float *long_kin = nullptr;
+    uint8_t *long_ufl = nullptr;
+    void *long_res = nullptr;      // [long_cap] results (long_res_bytes() each)
+    int32_t *long_start = nullptr, *long_cnt = nullptr;   // [long_units_cap]
+    unsigned int *long_n = nullptr;                       // [1] work items of the level
+    int32_t *long_slots = nullptr;  // [N_c + 1] slot indices of the long slots
+    int32_t *long_list = nullptr;   // [units_cap] long units to resume
 };
 
 struct Ctx {
@@ -120,6 +134,7 @@ struct Ctx {
     const void *mh_K = nullptr;    // the keys of the build in progress
     int mh_ngraph = 0;
     int build_passes = 1;          // unit-kernel launches of the last build (pruning passes)
+    int n_long = 0;                // slots of the last build longer than kMaxUnit (w.long_slots)
     // score passes issued ahead by gracekv_score (consumed by the next build);
     // requested before a segmentation, they are enqueued when its dynamic
     // program (one block) starts, so that they overlap it
@@ -292,18 +307,34 @@ cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *
                               int root_only, int max_levels, float tau, const int32_t *list_short,
                               int n_short, const int32_t *list_long, int n_long, cudaStream_t s,
                               int lg0 = 0, int nlg = -1);   // fresh launches: (l, g) in [lg0, lg0 + nlg);
-// Slot indices split by length class: short ones at list[0, count[0]), long
-// ones at list[J - count[1], J).
+// Slot indices split by length class: short ones at list[0, count[0]), those
+// of kShortUnit + 1 .. kMaxUnit tokens at list[J - count[1], J), longer ones
+// at long_slots[0, count[2]); count[3] receives the tokens of the longer ones.
 cudaError_t launch_slot_classes(Ctx &c, const int32_t *slots, int J, int32_t *list, int *count,
-                                cudaStream_t s);
+                                int32_t *long_slots, cudaStream_t s);
+// One level of the trees of long units (build_long.cu): with fresh = 1 the
+// roots of the listed slots for (l, g) in [lg0, lg0 + nlg) (root_only: their
+// own distortion and Add gain, the split left pending), else the pending
+// nodes of the listed units whose key bound reaches tau.  With n_items_host
+// the level's work-item count is read back (synchronises s) and a level
+// without work launches nothing more.
+cudaError_t launch_long_level(Ctx &c, const void *K, const void *V, const void *Q, const float *omega,
+                              const int32_t *slots, int J, int fresh, int root_only, float tau,
+                              const int32_t *list, int n_list, int lg0, int nlg, cudaStream_t s,
+                              unsigned int *n_items_host);
+size_t long_res_bytes();
+// out[q nlg + i] = the unit id of long slot long_slots[q] for (l, g) = lg0 + i.
+cudaError_t launch_long_units(Ctx &c, const int32_t *long_slots, int n_long, int lg0, int nlg, int J,
+                              int32_t *out, cudaStream_t s);
 // Allocation threshold tau over the ops built so far (alloc_state prefix /
 // all-fit flag), and the units whose largest pending key bound reaches
 // max(tau, cut), split by slot length class: short units at list[0, count[0]),
-// long units at list[n_units - count[1], n_units); *pend_pot receives the
-// entries a complete expansion of every unit reaching tau could take.
+// those of up to kMaxUnit tokens at list[n_units - count[1], n_units), longer
+// ones at long_list[0, count[2]); *pend_pot receives the entries a complete
+// expansion of every unit reaching tau could take.
 cudaError_t launch_threshold(Ctx &c, int J, cudaStream_t s);
 cudaError_t launch_prune_list(Ctx &c, const int32_t *slots, int J, int32_t *list, int *count,
-                              cudaStream_t s);
+                              int32_t *long_list, cudaStream_t s);
 // Bound-ordered expansion: among the units whose largest pending key bound
 // reaches the threshold, the cut that keeps about `m` of them (the lower edge
 // of the bin of the m-th largest bound; -inf when fewer qualify), written to

@@ -474,10 +474,10 @@ ScoreArgs make_args(const Ctx &c) {
 cudaError_t launch_rope_table(Ctx &c, cudaStream_t s) {
     int64_t n = (int64_t)c.p.T * (c.p.d / 2);
     rope_table_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(c.p.T, c.p.d, c.p.rope_base, c.w.rope, 0);
-    // rotations by the offsets -(kMaxUnit - 1) .. kMaxUnit - 1 (prototype position minus token position)
-    int64_t nr = (int64_t)(2 * kMaxUnit - 1) * (c.p.d / 2);
-    rope_table_kernel<<<(unsigned)((nr + 255) / 256), 256, 0, s>>>(2 * kMaxUnit - 1, c.p.d, c.p.rope_base,
-                                                                   c.w.rope_rel, -(kMaxUnit - 1));
+    // rotations by the offsets -(kMaxSlot - 1) .. kMaxSlot - 1 (prototype position minus token position)
+    int64_t nr = (int64_t)(2 * kMaxSlot - 1) * (c.p.d / 2);
+    rope_table_kernel<<<(unsigned)((nr + 255) / 256), 256, 0, s>>>(2 * kMaxSlot - 1, c.p.d, c.p.rope_base,
+                                                                   c.w.rope_rel, -(kMaxSlot - 1));
     return cudaGetLastError();
 }
 

@@ -64,3 +64,44 @@ def build_trees_pooled(kw: dict, K, V, Q, kappa, slot_starts, m, Z, rtok, worker
         base += n
     return O.Trees({k: np.concatenate(v) for k, v in nodes.items()}, np.concatenate(uadd),
                    np.concatenate(uroot), J)
+
+
+def run_pooled(K, V, Q, budgets, rope_base, slot_starts=None, **overrides):
+    """The oracle pass of O.run for one layer and one KV head at several
+    budgets, with the tree build pooled.  The trees do not depend on the
+    budget (only the recent window does, and it is the same for every budget
+    here), so segmentation, statistics and trees are computed once; each
+    budget gets its own allocation and gather.  Without slot_starts the
+    segmentation runs with the dispersion in the paper's prefix form (App.
+    B.3 Eq. app_prefix_dispersion, pinned equal to the definition); with them
+    the curvature is still computed (the refinement rule reads it)."""
+    K64, V64, Q64 = (np.asarray(t.double().numpy() if hasattr(t, "double") else t, np.float64)
+                     for t in (K, V, Q))
+    L, G, T, d = K64.shape
+    Hq, W = Q64.shape[1], Q64.shape[2]
+    kw = dict(L=L, G=G, Hq=Hq, T=T, d=d, W=W, rope_base=rope_base, disp_mode=1, **overrides)
+    p = O.make_params(**kw)
+    r_eff, _ = O.budget(p, budgets[0])
+    p.recent = r_eff
+    kw["recent"] = r_eff
+    if slot_starts is None:
+        seg = O.segment(p, V64)
+    else:
+        kap, _ = O.curvature(p, V64)
+        seg = dict(kappa=kap, b=None, slot_starts=np.asarray(slot_starts, np.int32) + p.ctx_start,
+                   dp_best=None, dp_second=None)
+    m, Z, ZC = O.row_stats(p, Q64, K64)
+    rtok = O.token_values(p, Q64, K64, m, Z)
+    tr = build_trees_pooled(kw, K64, V64, Q64, seg["kappa"], seg["slot_starts"], m, Z, rtok)
+    out = []
+    for B in budgets:
+        pb = O.make_params(**kw)
+        r_b, B_free = O.budget(pb, B)
+        assert r_b == r_eff, "the budgets must share the recent window"
+        pb.recent = r_eff
+        add_sel, split_sel, used = O.allocate(pb, B_free, tr)
+        cap = B + L * G * (T - (pb.ctx_end - pb.ctx_start)) + 16
+        cache = O.gather(pb, K64, V64, rtok, tr, add_sel, split_sel, cap)
+        out.append(dict(params=pb, r_eff=r_eff, B_free=B_free, seg=seg, m=m, Z=Z, ZC=ZC, rtok=rtok,
+                        trees=tr, add_sel=add_sel, split_sel=split_sel, used=used, cache=cache, floor=None))
+    return out

@@ -342,14 +342,26 @@ def test_errors_are_reported_not_trapped():
         ctx.gracekv_segment(Vm, slots)
     assert e.value.status == gk.GKV_EINVAL
     ctx.gracekv_segment(V, slots)
-    bad = torch.tensor([0, 200, T - 32], dtype=torch.int32, device="cuda")   # slot of 200 tokens
-    with pytest.raises(gk.GraceKVError) as e:
-        ctx.gracekv_build_trees(K, V, Q, None, bad, 2)
-    assert e.value.status == gk.GKV_EUNSUPPORTED
+    long = torch.tensor([0, 200, T - 32], dtype=torch.int32, device="cuda")   # a slot of 200 tokens builds
+    ctx.gracekv_build_trees(K, V, Q, None, long, 2)
+    assert ctx.gracekv_allocate() > 0
+    ctx = gk.Context(p)
+    ctx.gracekv_segment(V, slots)
     bad = torch.tensor([0, 50, 40, T - 32], dtype=torch.int32, device="cuda")
     with pytest.raises(gk.GraceKVError) as e:
         ctx.gracekv_build_trees(K, V, Q, None, bad, 3)
     assert e.value.status == gk.GKV_EINVAL
+    # a supplied slot longer than 16384 tokens is refused before any tree work
+    xl = synth.make_inputs(w, T=16500)
+    pl = gk.make_params(L, G, 2, 16500, d, 32, dtype=torch.float32, budget=2000, rope_base=w.rope_base)
+    ctxl = gk.Context(pl)
+    Kl, Vl, Ql = xl.K.cuda(), xl.V.cuda(), xl.Q.cuda()
+    ctxl.gracekv_segment(Vl, torch.empty(16500, dtype=torch.int32, device="cuda"))
+    over = torch.tensor([0, 16400, 16500 - 32], dtype=torch.int32, device="cuda")
+    with pytest.raises(gk.GraceKVError) as e:
+        ctxl.gracekv_build_trees(Kl, Vl, Ql, None, over, 2)
+    assert e.value.status == gk.GKV_EUNSUPPORTED
+    del ctxl, Kl, Vl, Ql
     Vn = V.clone()
     Vn[0, 0, 17, 3] = float("nan")
     ctx2 = gk.Context(p)

@@ -17,37 +17,14 @@ import numpy as np
 import pytest
 import torch
 
-import oracle as O
 from paper_2608_07001_gb300 import synth
 from tests import parity as P
-from tests.oracle_pool import build_trees_pooled
+from tests.oracle_pool import run_pooled
 
 pytestmark = pytest.mark.gpu
 
 L_S, G_S = 13, 5          # the sliced (layer, KV head) of the 32 x 8 workload
 RATIO = 32
-
-
-def oracle_slice(K, V, Q, B, base):
-    """The oracle pass of O.run for L = G = 1, with the tree build pooled."""
-    L, G, T, d = K.shape
-    Hq, W = Q.shape[1], Q.shape[2]
-    # the dispersion in the paper's prefix form (App. B.3 Eq.
-    # app_prefix_dispersion), pinned equal to the sample-variance definition
-    kw = dict(L=L, G=G, Hq=Hq, T=T, d=d, W=W, rope_base=base, disp_mode=1)
-    p = O.make_params(**kw)
-    r_eff, B_free = O.budget(p, B)
-    p.recent = r_eff
-    kw["recent"] = r_eff
-    K64, V64, Q64 = (t.double().numpy() for t in (K, V, Q))
-    seg = O.segment(p, V64)
-    m, Z, ZC = O.row_stats(p, Q64, K64)
-    rtok = O.token_values(p, Q64, K64, m, Z)
-    tr = build_trees_pooled(kw, K64, V64, Q64, seg["kappa"], seg["slot_starts"], m, Z, rtok)
-    add_sel, split_sel, used = O.allocate(p, B_free, tr)
-    cache = O.gather(p, K64, V64, rtok, tr, add_sel, split_sel, B + 16)
-    return dict(params=p, r_eff=r_eff, B_free=B_free, seg=seg, m=m, Z=Z, ZC=ZC, rtok=rtok,
-                trees=tr, add_sel=add_sel, split_sel=split_sel, used=used, cache=cache, floor=None)
 
 
 def test_full_context_slice_matches_the_oracle():
@@ -59,7 +36,7 @@ def test_full_context_slice_matches_the_oracle():
     assert (L, G, T, d) == (1, 1, 131072, 128) and x.K.dtype == torch.bfloat16
     B = (L * G * T) // RATIO
     t0 = time.time()
-    o = oracle_slice(x.K, x.V, x.Q, B, w.rope_base)
+    o = run_pooled(x.K, x.V, x.Q, [B], w.rope_base)[0]
     t1 = time.time()
     gr = P.run_gpu(x.K, x.V, x.Q, B, w.rope_base)
     rep = P.compare(gr, o, torch.bfloat16)
