@@ -36,7 +36,6 @@ import torch
 METRIC = "context tokens compressed/sec per GB300 and % of HBM roofline (vs CPU oracle)"
 PEAK_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
                  "sm_max_mhz": 2070.0}
-N_SMS = 152
 FP32_LANES = 128
 
 
@@ -102,22 +101,68 @@ class ClockSampler:
                 "reasons": sorted(reasons)}
 
 
-def cpu_baseline(w, ratio: float, T_s: int = 4608):
-    """Oracle on one layer x one KV head x T_s tokens of the workload's recipe
-    (about 10 s of one host core)."""
+def _oracle_sample(args):
+    """Child process: the oracle pass on the bounded sample, pinned to one
+    host core when the platform allows it; returns (seconds, cores, cpu)."""
+    wname, ratio, T_s = args
+    cores = None
+    try:
+        allowed = sorted(os.sched_getaffinity(0))
+        os.sched_setaffinity(0, {allowed[0]})
+        cores = len(os.sched_getaffinity(0))
+    except (AttributeError, OSError):
+        pass
     import oracle as O
     from paper_2608_07001_gb300 import synth
+    w = synth.WORKLOADS[wname]
     x = synth.make_inputs(w, layers=[0], heads=[0], T=T_s)
     L1, G1, T1, d = x.K.shape
     B = max(int(L1 * G1 * T1 // ratio), 4 * L1 * G1 + 1)
+    slots = None if x.slots is None else x.slots
     t0 = time.perf_counter()
-    O.run(x.K, x.V, x.Q, B, w.rope_base)
-    dt = time.perf_counter() - t0
-    # linear extrapolation in L*G*T: tokens/s = T / (dt * L * G * T / T_s)
+    O.run(x.K, x.V, x.Q, B, w.rope_base, slot_starts=slots)
+    return time.perf_counter() - t0, cores
+
+
+def host_info():
+    """nproc and the CPU model of the host the oracle runs on."""
+    model = None
+    try:
+        for ln in open("/proc/cpuinfo"):
+            k = ln.split(":")[0].strip().lower()
+            if k in ("model name", "cpu model", "hardware"):
+                model = ln.split(":", 1)[1].strip()
+                break
+    except OSError:
+        pass
+    if model is None:
+        try:
+            out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+            for ln in out.splitlines():
+                if ln.lower().startswith("model name"):
+                    model = ln.split(":", 1)[1].strip()
+                    break
+        except (OSError, subprocess.SubprocessError):
+            pass
+    return {"nproc": os.cpu_count(), "cpu_model": model}
+
+
+REF_TOKENS = 4096
+
+
+def cpu_baseline(w, ratio: float, T_s: int = REF_TOKENS):
+    """The oracle as it stands on one layer x one KV head x T_s tokens of the
+    workload's recipe (for a workload with supplied slots, the recipe's slots
+    of that length), in a spawned child pinned to one host core: about 10 s
+    of CPU work.  Its tokens/s is extrapolated linearly in L G T."""
+    import multiprocessing as mp
+    with mp.get_context("spawn").Pool(1) as pool:
+        dt, cores = pool.apply(_oracle_sample, ((w.name, ratio, T_s),))
     value = T_s / (dt * w.L * w.G)
-    sample = (f"oracle pipeline on 1 layer x 1 KV head x {T_s} tokens "
-              f"({dt:.1f} s), extrapolated linearly to {w.L} x {w.G} x {w.T}")
-    return value, dt, sample
+    sample = (f"oracle pipeline (segmentation, row statistics, token values, trees, heap "
+              f"allocation, gather) on 1 layer x 1 KV head x {T_s} tokens ({dt:.1f} s on one "
+              f"host core), extrapolated linearly to {w.L} x {w.G} x {w.T}")
+    return value, dt, sample, (cores or 1)
 
 
 def max_over_ranks(x: float, dist, device) -> float:
@@ -143,7 +188,7 @@ def run_reference(args, w):
         return
     vals = []
     for i in range(args.warmup + args.steps):
-        v, dt, sample = cpu_baseline(w, args.ratio, T_s=args.ref_tokens)
+        v, dt, sample, cores = cpu_baseline(w, args.ratio, T_s=args.ref_tokens)
         if i >= args.warmup:
             vals.append((v, dt))
     value = statistics.median(v for v, _ in vals)
@@ -153,8 +198,8 @@ def run_reference(args, w):
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
            "data": "synthetic", "impl": "reference",
            "config": workload_config(w, args.ratio),
-           "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
-                            "sample": sample},
+           "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                            "sample": sample, **host_info()},
            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                    "d2h_bytes_per_step": 0}}
     print(json.dumps(out))
@@ -301,7 +346,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
-    ap.add_argument("--ref-tokens", type=int, default=1024)
+    ap.add_argument("--ref-tokens", type=int, default=REF_TOKENS,
+                    help="tokens of the oracle's bounded sample (cpu_baseline and --impl reference)")
     ap.add_argument("--layers", type=int, default=0,
                     help="compress only the first N layers (small cases for profiler captures)")
     ap.add_argument("--no-decode", action="store_true",
@@ -347,6 +393,9 @@ def main():
     x = synth.make_inputs(w, device=dev, layers=layers)
     K, V, Q = x.K, x.V, x.Q
     L, G, T, d = K.shape
+    n_sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    # a workload with a supplied partition (the skewed one) passes its slots
+    slots = None if x.slots is None else torch.as_tensor(x.slots, dtype=torch.int32, device=dev)
     B = gk.gracekv_budget_for_ratio(L, G, T, args.ratio)
     abl = {"none": {}, "wo_cs": dict(seg_mode=1, k_cand=0, lambda_kappa=0.0),
            "wo_ga": dict(quota_alloc=1)}[args.ablation]
@@ -368,7 +417,7 @@ def main():
         torch.cuda.synchronize(dev)
 
     if args.decode_only:
-        comp(K, V, Q, Qg=Qg)
+        comp(K, V, Q, Qg=Qg, slot_starts=slots)
         torch.cuda.synchronize(dev)
         dec = decode_leg(args, w, comp, L, G, Q.shape[1], d, dev)
         if rank == 0:
@@ -376,7 +425,7 @@ def main():
         return
 
     for _ in range(args.warmup):
-        comp(K, V, Q, Qg=Qg)
+        comp(K, V, Q, Qg=Qg, slot_starts=slots)
     comp.ctx.gracekv_profile(True)
     comp.ctx.gracekv_stats()
     _, launches0, _ = comp.ctx.gracekv_stats()
@@ -388,7 +437,7 @@ def main():
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for _ in range(args.steps):
-        comp(K, V, Q, Qg=Qg)
+        comp(K, V, Q, Qg=Qg, slot_starts=slots)
     e1.record(stream)
     barrier()
     clocks = clk.stop()
@@ -416,14 +465,14 @@ def main():
         # probe weights of every token (W d FMA)
         flops = (2 * Wp * d * work["scan_steps"] + 8 * Wp * d * work["cand_evals"]
                  + 6 * d * work["cand_len_sum"] + 2 * Wp * d * L * G * comp.ctx.n_c)
-        peak = N_SMS * FP32_LANES * 2 * pk.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+        peak = n_sms * FP32_LANES * 2 * pk.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
         ach = flops / (per_step[dom] / 1e3) / 1e12
         roof = {"kernel": "unit_build_kernel", "bound": "alu", "achieved": ach, "peak": peak,
                 "unit": "TFLOP/s", "frac": ach / peak, "traffic": None,
-                "peak_basis": f"{N_SMS} SMs x {FP32_LANES} fp32 lanes x 2 x max SM clock"}
+                "peak_basis": f"{n_sms} SMs x {FP32_LANES} fp32 lanes x 2 x max SM clock"}
     elif dom in ("row_stats", "token_values"):
         flops = 2 * L * Q.shape[1] * Wp * d * (T if dom == "row_stats" else comp.ctx.n_c)
-        peak = N_SMS * FP32_LANES * 2 * pk.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+        peak = n_sms * FP32_LANES * 2 * pk.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
         ach = flops / (per_step[dom] / 1e3) / 1e12
         roof = {"kernel": dom, "bound": "alu", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
                 "frac": ach / peak, "traffic": None}
@@ -443,10 +492,29 @@ def main():
         c = comp.cache
         hc = gk.Cache.empty_host(c.K.shape[0], d, L * G, K.dtype)
 
-        def e2e_step():
-            # the library copies the inputs layer group by layer group on a
-            # copy stream and starts each group's work as it lands
-            return comp.ctx.gracekv_compress_host(Kh, Vh, Qh, hc)
+        if slots is None:
+            def e2e_step():
+                # the library copies the inputs layer group by layer group on a
+                # copy stream and starts each group's work as it lands
+                return comp.ctx.gracekv_compress_host(Kh, Vh, Qh, hc)
+        else:
+            # a supplied partition: the device API with the copies in the
+            # step (the host-buffer call segments the context itself)
+            Kd, Vd, Qd = torch.empty_like(K), torch.empty_like(V), torch.empty_like(Q)
+            sh = x.slots.astype(np.int32)
+
+            def e2e_step():
+                Kd.copy_(Kh, non_blocking=True)
+                Vd.copy_(Vh, non_blocking=True)
+                Qd.copy_(Qh, non_blocking=True)
+                sd = torch.from_numpy(sh).to(dev, non_blocking=False)
+                cache = comp(Kd, Vd, Qd, slot_starts=sd)
+                n = comp.n_entries
+                for k_ in ("K", "V", "pos", "log_m", "src_lo", "src_hi"):
+                    getattr(hc, k_)[:n].copy_(getattr(cache, k_)[:n], non_blocking=True)
+                hc.offsets.copy_(cache.offsets, non_blocking=True)
+                torch.cuda.synchronize(dev)
+                return n
 
         e2e_step()
         barrier()
@@ -456,15 +524,16 @@ def main():
         barrier()
         dt = time.perf_counter() - t0
         dt = max_over_ranks(dt, dist, dev)
-        h2d = sum(t_.numel() * t_.element_size() for t_ in (K, V, Q))
+        h2d = sum(t_.numel() * t_.element_size() for t_ in (K, V, Q)) + (0 if slots is None else slots.numel() * 4)
         d2h = n * (2 * d * elem + 16) + hc.offsets.numel() * 8
         e2e = {"value": whole_job_rate(world, T, args.e2e_steps, dt), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
-        v, dt, sample = cpu_baseline(w, args.ratio)
-        cpu = {"value": v, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": sample}
+        v, dt, sample, cores = cpu_baseline(w, args.ratio, T_s=args.ref_tokens)
+        cpu = {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": sample,
+               **host_info()}
 
     dec = None
     if not args.no_decode:
