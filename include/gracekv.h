@@ -275,11 +275,14 @@ gkv_status gracekv_compress_host(gracekv_ctx *ctx, const void *K, const void *V,
  * Introspection for tests and tools (not needed to compress).  Copies the
  * current trees and selection to caller-owned HOST arrays (synchronises
  * `stream`).  Node records of all units are packed unit after unit, unit
- * order (l, g, j); within a unit in creation (breadth-first) order.
+ * order (l, g, j); within a unit in creation order (breadth-first for slots
+ * of at most 128 tokens; a longer slot's tree is created level by level,
+ * each node of at most 128 tokens getting slots reserved for its subtree).
  *   unit_first [L G J + 1] int64: node range of each unit
  *   unit_Uadd, unit_Ddrop [L G J] fp32; add_sel [L G J] uint8
  *   per node (capacity node_cap): a, b, child0 (index within the unit, -1 for
- *   leaves), nchild, cost int32; D, R, U, kappa fp32; split_sel uint8
+ *   leaves), nchild (-1: pending, not evaluated; -2: an unused reserved
+ *   slot, to be skipped), cost int32; D, R, U, kappa fp32; split_sel uint8
  *   row stats (nullable) [L][Hq][W] fp32: max logit, Z over [0,T), Z over C
  *   rtok (nullable) [L][G][N_c] fp32 token values
  * *n_nodes_host receives the node count (GKV_ECAPACITY if > node_cap).

@@ -38,7 +38,8 @@ namespace gkv {
 namespace {
 
 // alloc_state layout (unsigned long long)
-enum { ST_PREFIX = 0, ST_ABOVE, ST_ALL, ST_R, ST_ENDU, ST_ENDKEY, ST_TOTAL, ST_USED, ST_N };
+enum { ST_PREFIX = 0, ST_ABOVE, ST_ALL, ST_R, ST_ENDU, ST_ENDKEY, ST_TOTAL, ST_USED, ST_CROSS, ST_N };
+static_assert(ST_N <= 16, "alloc_state holds 16 words per segment");
 
 struct AllocArgs {
     int64_t n_units;
@@ -54,7 +55,8 @@ struct AllocArgs {
     const int32_t *slots;
     int J, LG, cs, Nc;
     uint8_t *u_sel, *nd_sel;
-    int32_t *u_flag;
+    int32_t *u_flag;         // units holding ties (alloc_mark), then their tie state (alloc_tie_scan)
+    int64_t *u_tcost;        // cost of each unit's tie closure
     unsigned long long *hist, *st;
     int64_t B_free;
     int *status;
@@ -252,95 +254,187 @@ __global__ void alloc_mark_kernel(AllocArgs A) {
     }
 }
 
+// ---------------------------------------------------------------------------
+// Ties (ops whose key equals tau).  The heap takes them unit by unit in
+// ascending unit order, each unit's in its own heap order, while budget is
+// left.  A unit whose tie ops all fit executes every tie op reachable from
+// the main set (its tie closure), so:
+//   alloc_tie_cost   every unit's closure and its cost, in parallel (a
+//                    closure op is marked 3; parents precede children in a
+//                    unit's node order, so one pass in that order suffices)
+//   alloc_tie_scan   per segment, the ordered prefix of the costs: units
+//                    whose closure fits select it whole, the first that does
+//                    not is the crossing unit, with the budget left for it
+//   alloc_tie_apply  the closures of the units before it selected (3 -> 1),
+//                    the others cleared (3 -> 0)
+//   alloc_ties       the crossing unit and the ones after it, while budget is
+//                    left, replayed op by op (block-wide argmax per pop).
+// ---------------------------------------------------------------------------
+__global__ void alloc_tie_cost_kernel(AllocArgs A) {
+    const int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (u >= A.n_units) return;
+    int64_t cost = 0;
+    if (A.u_flag[u]) {
+        const unsigned long long *st = seg_st(A, A.nseg > 1 ? (int)(u / A.J) : 0);
+        const uint32_t tau = (uint32_t)st[ST_PREFIX];
+        const int lg = (int)(u / A.J), j = (int)(u - (int64_t)lg * A.J);
+        const int64_t nb = node_base(lg, A.slots[j], A.cs, A.Nc);
+        const bool addtie = A.u_sel[u] == 0 && !(A.u_floor && A.u_floor[u]) && __float_as_uint(A.u_U[u]) == tau;
+        if (addtie) { A.u_sel[u] = 3; cost += 1; }
+        const bool root_open = A.u_sel[u] == 1 || A.u_sel[u] == 3;
+        const int nn = A.u_nnodes[u];
+        for (int k = 0; k < nn; k++) {
+            const int64_t v = nb + k;
+            if (A.nd_cost[v] <= 0 || A.nd_sel[v] != 0 || __float_as_uint(A.nd_kappa[v]) != tau) continue;
+            const int32_t pg = A.nd_parent[v];
+            const bool open = pg < 0 ? root_open : (A.nd_sel[pg] == 1 || A.nd_sel[pg] == 3);
+            if (!open) continue;
+            A.nd_sel[v] = 3;
+            cost += A.nd_cost[v];
+        }
+    }
+    A.u_tcost[u] = cost;
+}
+
+// One block per segment: ordered inclusive scan of the closure costs.
+__global__ void __launch_bounds__(1024) alloc_tie_scan_kernel(AllocArgs A) {
+    __shared__ long long wsum[32];
+    __shared__ long long carry_s;
+    const int seg = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    unsigned long long *st = seg_st(A, seg);
+    if (st[ST_ALL]) return;
+    const long long R = seg_budget(A, seg) - (long long)st[ST_ABOVE];
+    const int64_t u_lo = A.nseg > 1 ? (int64_t)seg * A.J : 0;
+    const int64_t u_hi = A.nseg > 1 ? u_lo + A.J : A.n_units;
+    if (tid == 0) carry_s = 0;
+    __syncthreads();
+    for (int64_t base = u_lo; base < u_hi; base += 1024) {
+        const int64_t u = base + tid;
+        const long long c = u < u_hi ? (long long)A.u_tcost[u] : 0;
+        long long incl = c;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const long long y = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += y;
+        }
+        if (lane == 31) wsum[warp] = incl;
+        __syncthreads();
+        long long before = carry_s;
+        for (int w = 0; w < warp; w++) before += wsum[w];
+        const long long hi = before + incl, lo = hi - c;   // prefix after / before this unit
+        if (u < u_hi) {
+            int state = 0;
+            if (c > 0 && hi <= R) state = 1;                 // its whole closure fits
+            else if (c > 0 && lo <= R && hi > R) {           // the crossing unit
+                state = 2;
+                st[ST_CROSS] = (unsigned long long)u;
+                st[ST_R] = (unsigned long long)(R - lo);
+            }
+            A.u_flag[u] = state;
+        }
+        __syncthreads();
+        if (tid == 1023) carry_s = hi;
+        __syncthreads();
+    }
+    if (tid == 0 && st[ST_CROSS] == ~0ull) st[ST_R] = (unsigned long long)(R - carry_s);
+}
+
+__global__ void alloc_tie_apply_kernel(AllocArgs A) {
+    const int64_t n = A.n_units + *A.n_ops;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        if (i < A.n_units) {
+            if (A.u_sel[i] == 3) A.u_sel[i] = A.u_flag[i] == 1 ? 1 : 0;
+        } else {
+            const int64_t v = (int64_t)(A.ops[i - A.n_units].y >> 1);
+            if (A.nd_sel[v] == 3) A.nd_sel[v] = A.u_flag[A.nd_unit[v]] == 1 ? 1 : 0;
+        }
+    }
+}
+
 // Node index base of unit uid.
 __device__ __forceinline__ int64_t unit_base(const AllocArgs &A, int64_t uid) {
     int lg = (int)(uid / A.J), j = (int)(uid - (int64_t)lg * A.J);
     return node_base(lg, A.slots[j], A.cs, A.Nc);
 }
 
-// One block per segment: walk its units in ascending order; thread 0 replays
-// every unit that holds tie ops with the unit's own queue.
+// One block per segment: from its crossing unit on, while budget is left,
+// each unit holding ties is replayed with its own queue restricted to tie ops
+// (U descending, then the node's position ascending and length descending);
+// each pop is a block-wide argmax over the unit's nodes.  An op costing more
+// than the budget left is discarded (2): its subtree is never exposed.
 __global__ void __launch_bounds__(1024) alloc_ties_kernel(AllocArgs A) {
-    __shared__ int list[1024];
-    __shared__ int nlist;
+    __shared__ unsigned long long wk[32];
+    __shared__ int wi[32];
     __shared__ long long Rs;
-    const int seg = blockIdx.x;
+    __shared__ unsigned long long bkey;
+    __shared__ int bidx;
+    const int seg = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     unsigned long long *st = seg_st(A, seg);
-    const long long Bseg = seg_budget(A, seg);
-    const int64_t u_lo = A.nseg > 1 ? (int64_t)seg * A.J : 0;
-    const int64_t u_hi = A.nseg > 1 ? u_lo + A.J : A.n_units;
-    if (threadIdx.x == 0) {
-        const bool all = st[ST_ALL] != 0;
-        long long above = (long long)st[ST_ABOVE];
-        Rs = all ? Bseg - (long long)st[ST_TOTAL] : Bseg - above;
-    }
-    __syncthreads();
     if (st[ST_ALL]) {
-        if (threadIdx.x == 0) st[ST_R] = 0, st[ST_USED] = st[ST_TOTAL];
+        if (tid == 0) st[ST_R] = 0, st[ST_USED] = st[ST_TOTAL];
         return;
     }
+    if (st[ST_CROSS] == ~0ull) return;   // every tie closure fit (alloc_tie_scan set ST_R)
     const uint32_t tau = (uint32_t)st[ST_PREFIX];
-    for (int64_t base = u_lo; base < u_hi && Rs > 0; base += 1024) {
-        // ordered compaction of flagged units in [base, base + 1024)
-        int64_t uid = base + threadIdx.x;
-        bool f = uid < u_hi && A.u_flag[uid];
-        if (threadIdx.x == 0) nlist = 0;
-        __syncthreads();
-        unsigned bal = __ballot_sync(0xffffffffu, f);
-        __shared__ int wcnt[32];
-        if ((threadIdx.x & 31) == 0) wcnt[threadIdx.x >> 5] = __popc(bal);
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            int acc = 0;
-            for (int w = 0; w < 32; w++) { int c = wcnt[w]; wcnt[w] = acc; acc += c; }
-            nlist = acc;
-        }
-        __syncthreads();
-        if (f) list[wcnt[threadIdx.x >> 5] + __popc(bal & ((1u << (threadIdx.x & 31)) - 1))] = (int)(uid - base);
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            for (int q = 0; q < nlist && Rs > 0; q++) {
-                int64_t u = base + list[q];
-                int64_t nb = unit_base(A, u);
-                int nn = A.u_nnodes[u];
-                // the parent of local node k: -1 for the root (parent index -2 - unit)
-                auto parent_of = [&](int k) {
-                    const int32_t pg = A.nd_parent[nb + k];
-                    return pg < 0 ? -1 : (int)(pg - nb);
-                };
-                // the unit's queue restricted to tie ops; -1 stands for the Add
-                for (;;) {
-                    int best = -2;
-                    float bu = 0.f;
-                    int ba = 0, bb = 0;
-                    // Add
-                    if (A.u_sel[u] == 0 && __float_as_uint(A.u_U[u]) == tau) {
-                        best = -1; bu = A.u_U[u]; ba = A.nd_a[nb]; bb = A.nd_b[nb];
-                    }
-                    for (int k = 0; k < nn; k++) {
-                        int64_t v = nb + k;
-                        if (A.nd_cost[v] <= 0 || A.nd_sel[v] != 0) continue;
-                        if (__float_as_uint(A.nd_kappa[v]) != tau) continue;
-                        const int pk = parent_of(k);
-                        bool exposed = pk < 0 ? A.u_sel[u] == 1 : A.nd_sel[nb + pk] == 1;
-                        if (!exposed) continue;
-                        float uu = A.nd_U[v];
-                        int aa = A.nd_a[v], bbb = A.nd_b[v];
-                        bool better = best == -2 || uu > bu || (uu == bu && (aa < ba || (aa == ba && bbb > bb)));
-                        if (better) { best = k; bu = uu; ba = aa; bb = bbb; }
-                    }
-                    if (best == -2 || Rs <= 0) break;
-                    int cost = best == -1 ? 1 : A.nd_cost[nb + best];
-                    uint8_t s = cost > Rs ? 2 : 1;     // 2 = discarded (subtree never exposed)
-                    if (s == 1) Rs -= cost;
-                    if (best == -1) A.u_sel[u] = s;
-                    else A.nd_sel[nb + best] = s;
+    const int64_t u_hi = A.nseg > 1 ? (int64_t)seg * A.J + A.J : A.n_units;
+    if (tid == 0) Rs = (long long)st[ST_R];
+    __syncthreads();
+    for (int64_t u = (int64_t)st[ST_CROSS]; u < u_hi && Rs > 0; u++) {
+        if (A.u_tcost[u] <= 0) continue;            // no tie op exposed in this unit
+        const int lg = (int)(u / A.J), j = (int)(u - (int64_t)lg * A.J);
+        const int sa = A.slots[j];
+        const int64_t nb = node_base(lg, sa, A.cs, A.Nc);
+        const int nn = A.u_nnodes[u];
+        for (;;) {
+            // key: U bits (32) | 2^15 - 1 - (a - sa) (15) | b - a (15); -1 node: the Add
+            unsigned long long best = 0ull;
+            int bi = -2;
+            if (tid == 0 && A.u_sel[u] == 0 && !(A.u_floor && A.u_floor[u]) &&
+                __float_as_uint(A.u_U[u]) == tau) {
+                best = ((unsigned long long)__float_as_uint(A.u_U[u]) << 32) |
+                       ((unsigned long long)(32767u) << 15) | (unsigned long long)(A.nd_b[nb] - A.nd_a[nb]);
+                bi = -1;
+            }
+            for (int k = tid; k < nn; k += 1024) {
+                const int64_t v = nb + k;
+                if (A.nd_cost[v] <= 0 || A.nd_sel[v] != 0 || __float_as_uint(A.nd_kappa[v]) != tau) continue;
+                const int32_t pg = A.nd_parent[v];
+                const bool exposed = pg < 0 ? A.u_sel[u] == 1 : A.nd_sel[pg] == 1;
+                if (!exposed) continue;
+                const unsigned long long key = ((unsigned long long)__float_as_uint(A.nd_U[v]) << 32) |
+                                               ((unsigned long long)(32767u - (uint32_t)(A.nd_a[v] - sa)) << 15) |
+                                               (unsigned long long)(A.nd_b[v] - A.nd_a[v]);
+                if (bi == -2 || key > best) { best = key; bi = k; }
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                const unsigned long long k2 = __shfl_xor_sync(0xffffffffu, best, o);
+                const int i2 = __shfl_xor_sync(0xffffffffu, bi, o);
+                if (i2 != -2 && (bi == -2 || k2 > best)) { best = k2; bi = i2; }
+            }
+            if (lane == 0) { wk[warp] = best; wi[warp] = bi; }
+            __syncthreads();
+            if (tid == 0) {
+                unsigned long long b = 0ull;
+                int ix = -2;
+                for (int w = 0; w < 32; w++)
+                    if (wi[w] != -2 && (ix == -2 || wk[w] > b)) { b = wk[w]; ix = wi[w]; }
+                bkey = b;
+                bidx = ix;
+                if (ix != -2) {
+                    const int cost = ix == -1 ? 1 : A.nd_cost[nb + ix];
+                    const uint8_t sv = cost > Rs ? 2 : 1;   // 2 = discarded (subtree never exposed)
+                    if (sv == 1) Rs -= cost;
+                    if (ix == -1) A.u_sel[u] = sv;
+                    else A.nd_sel[nb + ix] = sv;
                 }
             }
+            __syncthreads();
+            if (bidx == -2 || Rs <= 0) break;
         }
-        __syncthreads();
     }
-    if (threadIdx.x == 0) st[ST_R] = (unsigned long long)Rs;
+    if (tid == 0) st[ST_R] = (unsigned long long)Rs;
 }
 
 // Endgame: when exactly one budget unit is left, the best exposed cost-1 op.
@@ -434,7 +528,7 @@ __global__ void alloc_final_kernel(AllocArgs A) {
 __global__ void alloc_init_kernel(unsigned long long *st, unsigned long long *hist, int nseg) {
     const int nst = ST_N * (nseg > 1 ? nseg + 1 : 1);
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < nst; i += gridDim.x * blockDim.x)
-        st[i] = (i % ST_N == ST_ENDKEY) ? ~0ull : 0ull;
+        st[i] = (i % ST_N == ST_ENDKEY || i % ST_N == ST_CROSS) ? ~0ull : 0ull;
     for (int64_t b = blockIdx.x * blockDim.x + threadIdx.x; b < (int64_t)2048 * nseg; b += gridDim.x * blockDim.x)
         hist[b] = 0;
 }
@@ -451,6 +545,7 @@ AllocArgs make_args(Ctx &c, int J) {
     A.slots = w.slots;
     A.J = J; A.LG = c.p.L * c.p.G; A.cs = c.p.ctx_start; A.Nc = c.Nc;
     A.u_sel = w.u_sel; A.nd_sel = w.nd_sel; A.u_flag = w.u_count;
+    A.u_tcost = w.u_off;     // scratch until the gather writes the entry offsets
     A.hist = w.hist; A.st = w.alloc_state; A.B_free = c.B_free; A.status = w.dev_int + 1;
     A.nseg = c.p.quota_alloc ? c.p.L * c.p.G : 1;
     A.u_floor = c.p.alpha_floor > 0.0 ? w.u_floor : nullptr;
@@ -613,12 +708,15 @@ cudaError_t launch_allocate(Ctx &c, int J, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     const int blocks = grid_for(c, A.n_units + c.node_cap / 2);
     alloc_mark_kernel<<<blocks, 256, 0, s>>>(A);
+    alloc_tie_cost_kernel<<<(unsigned)((A.n_units + 255) / 256), 256, 0, s>>>(A);
+    alloc_tie_scan_kernel<<<A.nseg, 1024, 0, s>>>(A);
+    alloc_tie_apply_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_ties_kernel<<<A.nseg, 1024, 0, s>>>(A);
     alloc_end_max_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_end_key_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_end_pick_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_final_kernel<<<(A.nseg + 255) / 256, 256, 0, s>>>(A);
-    c.launches += 6;
+    c.launches += 9;
     return cudaGetLastError();
 }
 

@@ -247,7 +247,7 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
     gkv::Workspace &w = c.w;
     bool ok = dalloc(x, &w.rope, (size_t)p.T * (p.d / 2)) &&
               dalloc(x, &w.rope_rel, (size_t)(2 * gkv::kMaxSlot - 1) * (p.d / 2)) &&
-              dalloc(x, &w.long_slots, (size_t)Nc + 2) && dalloc(x, &w.long_n, 1) &&
+              dalloc(x, &w.long_slots, (size_t)Nc + 2) && dalloc(x, &w.long_n, 3) &&
               dalloc(x, &w.ent, (size_t)p.budget + (size_t)p.L * p.G * (p.T - Nc)) &&
               dalloc(x, &w.inv_norm, (size_t)c.nseg * p.T) &&
               dalloc(x, &w.nrm2, (size_t)c.nseg * p.T) &&
@@ -283,7 +283,7 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
                 dalloc(x, &w.mh_red, (size_t)2) && dalloc(x, &w.mh_pkeys, (size_t)64 * 64) &&
                 dalloc(x, &w.mh_psum, (size_t)64))) &&
               dalloc(x, &w.hist, (size_t)2048 * (p.quota_alloc ? LG : 1)) &&
-              dalloc(x, &w.alloc_state, (size_t)16 + (p.quota_alloc ? (size_t)8 * LG : 0)) && dalloc(x, &w.work, 4) &&
+              dalloc(x, &w.alloc_state, (size_t)16 * (p.quota_alloc ? (size_t)LG + 1 : 1)) && dalloc(x, &w.work, 4) &&
               dalloc(x, &w.pend_hist, 1 << 16) && dalloc(x, &w.pend_cut, 1) && dalloc(x, &w.pend_n, 1) &&
               dalloc(x, &w.pend_pot, 1);
     if (!ok) {
@@ -507,6 +507,7 @@ static gkv_status classes(gracekv_ctx *x, int cnt[4], cudaStream_t s) {
     if (items > w.long_cap) {
         bool ok = dalloc(x, &w.long_gv, items) && dalloc(x, &w.long_uid, items) &&
                   dalloc(x, &w.long_kin, items) && dalloc(x, &w.long_ufl, items) &&
+                  dalloc(x, &w.long_sub, 2 * items) &&
                   dalloc(x, reinterpret_cast<unsigned char **>(&w.long_res), items * gkv::long_res_bytes());
         if (!ok) return fail(x, GKV_ENOMEM, "build_trees: long-unit work items");
         w.long_cap = items;

@@ -72,6 +72,10 @@ struct BuildArgs {
     float lam_kappa, base_frac;
     // work list: fresh launches index (slot list entry, lg), resume launches units
     int resume;                  // 0: build from the root, 1: resume pending nodes
+    int subtree;                 // 1: the list holds pending nodes of at most NMAX tokens inside
+                                 //    long units (build_long.cu), as global node indices; each CTA
+                                 //    builds its node's subtree to the leaves into the node slots
+                                 //    reserved for it (the unit-relative index in its child0)
     int root_only;               // fresh: evaluate only the root's own distortion (split stays pending)
     int max_levels;              // levels evaluated by this launch
     float tau;                   // resume: evaluate pending nodes whose key bound >= tau
@@ -275,7 +279,13 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     S &sm = *reinterpret_cast<S *>(smem_raw);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     int j, lg;
-    if (A.resume) {
+    int64_t gv_sub = -1;         // subtree mode: the pending node whose subtree this CTA builds
+    if (A.subtree) {
+        gv_sub = A.list[blockIdx.x];
+        const int uidr = A.nd_unit[gv_sub];
+        lg = uidr / A.J;
+        j = uidr - lg * A.J;
+    } else if (A.resume) {
         const int uidr = A.list[blockIdx.x];
         lg = uidr / A.J;
         j = uidr - lg * A.J;
@@ -283,11 +293,20 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         j = A.list[blockIdx.x / A.nlg];   // slot-major: the units of a slot share its table rows
         lg = A.lg0 + blockIdx.x % A.nlg;
     }
+    const bool fresh = !A.resume && !A.subtree;
     const int l = lg / A.G, g = lg - l * A.G;
-    const int sa = A.slots[j], sb = A.slots[j + 1];
-    const int n = sb - sa;
     const int64_t uid = (int64_t)lg * A.J + j;
-    const int64_t nbase = node_base(lg, sa, A.cs, A.Nc);
+    const int64_t nbase = node_base(lg, A.slots[j], A.cs, A.Nc);   // the unit's node slots
+    // the tokens held: the slot, or in subtree mode the node's interval
+    const int sa = A.subtree ? A.nd_a[gv_sub] : A.slots[j];
+    const int sb = A.subtree ? A.nd_b[gv_sub] : A.slots[j + 1];
+    const int n = sb - sa;
+    // global node index of local node k, and its index inside the unit: the
+    // local nodes of a subtree are its root and then its reserved slots
+    const int64_t sub_res = A.subtree ? (int64_t)A.nd_child0[gv_sub] : 0;
+    auto gidx = [&](int k) -> int64_t {
+        return A.subtree ? (k == 0 ? gv_sub : nbase + sub_res + (k - 1)) : nbase + k;
+    };
     if (n < 1 || n > NMAX) {
         if (tid == 0) atomicOr(A.status, 4);
         return;
@@ -457,6 +476,14 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         for (int e = tid; e < n * 2 * kNPP; e += kNT) bad |= !isfinite(Ef[e]);
         for (int t = tid; t < n; t += kNT) bad |= !isfinite(sm.Rt[t]);
         if (__syncthreads_or(bad)) {
+            if (A.subtree) {   // the node stays a leaf; the unit is reported
+                if (tid == 0) {
+                    atomicOr(A.status, 8);
+                    A.nd_nchild[gv_sub] = 0; A.nd_child0[gv_sub] = -1; A.nd_cost[gv_sub] = 0;
+                    A.nd_U[gv_sub] = 0.f; A.nd_kappa[gv_sub] = 0.f;
+                }
+                return;
+            }
             if (tid == 0) {
                 atomicOr(A.status, 8);
                 A.nd_a[nbase] = sa; A.nd_b[nbase] = sb; A.nd_R[nbase] = 0.f; A.nd_D[nbase] = 0.f;
@@ -510,8 +537,20 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             }
         }
     }
-    // ---- tree state: a fresh root, or the unit's records so far --------------
-    if (!A.resume) {
+    // ---- tree state: a fresh root, a subtree's root, or the unit's records so far
+    if (A.subtree) {
+        if (tid == 0) {
+            NodeS &nd = sm.nodes[0];
+            nd.a = 0; nd.b = (short)n; nd.parent = -1; nd.child0 = -1; nd.nchild = -1;
+            nd.D = A.nd_D[gv_sub];
+            const int32_t pg = A.nd_parent[gv_sub];   // a node of the long unit, already evaluated
+            nd.kin = pg < 0 ? FLT_MAX : A.nd_kappa[pg];
+            sm.nnodes = 1;
+            sm.lvl[0][0] = 0;
+            sm.nlvl[0] = 1;
+            sm.pend = -1.f;
+        }
+    } else if (!A.resume) {
         if (warp == 0) {
             float r = 0.f;
             for (int t = lane; t < n; t += 32) r += sm.Rt[t];
@@ -745,8 +784,8 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 float pm = sm.pend;
                 for (int k = 0; k < nl; k++) {
                     const int v = sm.lvl[cur][k];
-                    A.nd_nchild[nbase + v] = -1;
-                    pm = fmaxf(pm, A.nd_U[nbase + v]);   // the key bound written at its creation
+                    A.nd_nchild[gidx(v)] = -1;
+                    pm = fmaxf(pm, A.nd_U[gidx(v)]);   // the key bound written at its creation
                 }
                 sm.pend = pm;
             }
@@ -762,7 +801,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 while (k < nl && nb < S::NB) {
                     const int v = sm.lvl[cur][k];
                     const int nv = sm.nodes[v].b - sm.nodes[v].a;
-                    const bool root = v == 0 && !A.resume;
+                    const bool root = v == 0 && fresh;
                     const int nc = (nv >= 3 && !(root && A.root_only)) ? min(A.k_cand + 1, nv - 1) + 1 : 0;
                     const int bp = nc + (root ? 1 : 0), bs = nc;
                     if (upre + bp > kNCD || usuf + bs > kNCD) break;
@@ -788,7 +827,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 BatchNode &B = sm.bn[bi];
                 const int v = B.node;
                 const int a = sm.nodes[v].a, b = sm.nodes[v].b, nv = b - a;
-                const bool ronly = v == 0 && !A.resume && A.root_only;   // only the node's own distortion
+                const bool ronly = v == 0 && fresh && A.root_only;   // only the node's own distortion
                 // top-K by curvature over positions [a, b-2] (ties: lower t)
                 unsigned sel[NMAX / 32];
                 unsigned long long kmin = ~0ull, kmax = 0ull;
@@ -911,7 +950,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     B.eL = el_sep ? eL_sep : (el_cand ? eL_cut : -1);
                     if (el_sep) sm.cand[eL_sep] = {a, pb, 0.f};
                     int k = B.pre_b + __popc(pm) + (el_sep ? 1 : 0);
-                    const bool whole = v == 0 && !A.resume;
+                    const bool whole = v == 0 && fresh;
                     B.whole = -1;
                     if (whole) { sm.cand[k] = {a, b, 0.f}; B.whole = k++; }
                     B.pre_e = k;
@@ -965,7 +1004,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     nd.kin = ufl ? FLT_MAX : gain;   // a floor slot's Add is a floor op
                     A.u_Uadd[uid] = gain;
                     A.u_Ddrop[uid] = Pd;
-                    A.nd_D[nbase] = D;
+                    A.nd_D[gidx(0)] = D;
                 }
                 __syncwarp();
                 if (A.root_only && B.whole >= 0 && nv >= 2) {   // its split is decided later
@@ -1042,7 +1081,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
             for (int bi = warp; bi < nb; bi += NWARPS) {
                 const BatchNode &B = sm.bn[bi];
                 NodeS &nd = sm.nodes[B.node];
-                const int64_t gv = nbase + B.node;
+                const int64_t gv = gidx(B.node);
                 int before = lane < bi ? max(sm.bn[lane].nchild, 0) : 0;
 #pragma unroll
                 for (int o = 16; o > 0; o >>= 1) before += __shfl_xor_sync(0xffffffffu, before, o);
@@ -1082,7 +1121,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                 if (lane == 0) {
                     nd.nchild = (signed char)nch;
                     nd.child0 = (short)child0;
-                    A.nd_child0[gv] = child0; A.nd_nchild[gv] = (int8_t)nch;
+                    A.nd_child0[gv] = (int32_t)(gidx(child0) - nbase); A.nd_nchild[gv] = (int8_t)nch;
                     A.nd_cost[gv] = (int8_t)cost; A.nd_U[gv] = U; A.nd_kappa[gv] = kap;
                     A.nd_sel[gv] = 0;
                     A.ops[atomicAdd(A.n_ops, 1u)] = make_uint2(__float_as_uint(kap), ((uint32_t)gv << 1) | (uint32_t)(cost - 1));
@@ -1093,7 +1132,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     NodeS &ch = sm.nodes[ci];
                     ch.a = (short)B.ca[q]; ch.b = (short)B.cb[q]; ch.parent = (short)B.node;
                     ch.child0 = -1; ch.nchild = 0; ch.D = B.cD[q]; ch.kin = kap;
-                    const int64_t gc = nbase + ci;
+                    const int64_t gc = gidx(ci);
                     A.nd_a[gc] = sa + B.ca[q]; A.nd_b[gc] = sa + B.cb[q];
                     A.nd_parent[gc] = (int32_t)gv; A.nd_unit[gc] = (int32_t)uid;
                     A.nd_D[gc] = B.cD[q]; A.nd_R[gc] = (float)rq;
@@ -1135,9 +1174,11 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     if (lane == 0) { sm.wcnt[warp][0] = w_scan; sm.wcnt[warp][1] = w_eval; sm.wcnt[warp][2] = w_len; }
     __syncthreads();
     if (tid == 0) {
-        A.u_nnodes[uid] = sm.nnodes;
-        A.u_pend[uid] = sm.pend;
-        if (!A.resume) A.u_sel[uid] = 0;
+        if (!A.subtree) {   // a subtree is built completely inside its reserved slots
+            A.u_nnodes[uid] = sm.nnodes;
+            A.u_pend[uid] = sm.pend;
+        }
+        if (fresh) A.u_sel[uid] = 0;
         unsigned long long tot[3] = {0, 0, 0};
         for (int w = 0; w < NWARPS; w++)
             for (int q = 0; q < 3; q++) tot[q] += sm.wcnt[w][q];
@@ -1147,7 +1188,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         atomicAdd(&A.work[3], 1ull);
     }
     // unused node slots of the unit carry cost 0 (no op)
-    if (!A.resume)
+    if (fresh)
         for (int k = sm.nnodes + tid; k < 2 * n; k += kNT) A.nd_cost[nbase + k] = 0;
 }
 
@@ -1189,7 +1230,7 @@ cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *
     A.inv_sqrt_d = (float)(1.0 / sqrt((double)p.d));
     A.lamZ = (float)p.lambda_Z; A.lamM = (float)p.lambda_M; A.eps = (float)p.eps;
     A.lam_kappa = p.lambda_kappa; A.base_frac = p.base_frac;
-    A.resume = resume; A.root_only = root_only; A.max_levels = max_levels; A.tau = tau;
+    A.resume = resume; A.subtree = 0; A.root_only = root_only; A.max_levels = max_levels; A.tau = tau;
     A.nd_a = c.w.nd_a; A.nd_b = c.w.nd_b; A.nd_child0 = c.w.nd_child0;
     A.nd_parent = c.w.nd_parent; A.nd_unit = c.w.nd_unit;
     A.nd_nchild = c.w.nd_nchild; A.nd_cost = c.w.nd_cost;
@@ -1213,6 +1254,46 @@ cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *
     A.list = list_long;
     unsigned g2 = resume ? (unsigned)n_long : (unsigned)n_long * LG;
     return bf ? launch_dt<__nv_bfloat16, kMaxUnit>(c, A, g2, s) : launch_dt<float, kMaxUnit>(c, A, g2, s);
+}
+
+cudaError_t launch_unit_subtrees(Ctx &c, const void *K, const void *V, const void *Q, const float *omega,
+                                 const int32_t *slots, int J, const int32_t *list_short, int n_short,
+                                 const int32_t *list_long, int n_long, cudaStream_t s) {
+    if (n_short + n_long == 0) return cudaSuccess;
+    cudaError_t e;
+    const gkv_params &p = c.p;
+    BuildArgs A;
+    A.K = K; A.V = V; A.Q = Q;
+    A.slots = slots; A.rope = c.w.rope; A.kappa = c.w.kappa;
+    A.rtok = c.w.rtok; A.row_m = c.w.row_m; A.row_Z = c.w.row_Z; A.omega = omega;
+    A.Eg = use_tc(c) ? c.w.Eg : nullptr;
+    A.fl_acc = p.alpha_floor > 0.0 ? c.w.fl_acc : nullptr;
+    A.fl_f = c.w.fl_f;
+    A.L = p.L; A.G = p.G; A.Hq = p.Hq; A.T = p.T; A.d = p.d; A.W = p.W; A.gq = p.Hq / p.G;
+    A.cs = p.ctx_start; A.Nc = c.Nc; A.J = J; A.k_cand = p.k_cand;
+    A.inv_sqrt_d = (float)(1.0 / sqrt((double)p.d));
+    A.lamZ = (float)p.lambda_Z; A.lamM = (float)p.lambda_M; A.eps = (float)p.eps;
+    A.lam_kappa = p.lambda_kappa; A.base_frac = p.base_frac;
+    A.resume = 0; A.subtree = 1; A.root_only = 0; A.max_levels = 4 * kMaxUnit; A.tau = -INFINITY;
+    A.nd_a = c.w.nd_a; A.nd_b = c.w.nd_b; A.nd_child0 = c.w.nd_child0;
+    A.nd_parent = c.w.nd_parent; A.nd_unit = c.w.nd_unit;
+    A.nd_nchild = c.w.nd_nchild; A.nd_cost = c.w.nd_cost;
+    A.ops = c.w.ops; A.n_ops = c.w.n_ops;
+    A.nd_D = c.w.nd_D; A.nd_R = c.w.nd_R; A.nd_U = c.w.nd_U; A.nd_kappa = c.w.nd_kappa;
+    A.nd_sel = c.w.nd_sel;
+    A.u_nnodes = c.w.u_nnodes; A.u_Uadd = c.w.u_Uadd; A.u_Ddrop = c.w.u_Ddrop; A.u_sel = c.w.u_sel;
+    A.u_pend = c.w.u_pend;
+    A.status = c.w.dev_int + 1;
+    A.work = c.w.work;
+    A.lg0 = 0;
+    A.nlg = p.L * p.G;
+    const bool bf = p.dtype == GKV_BF16;
+    A.list = list_short;
+    e = bf ? launch_dt<__nv_bfloat16, 64>(c, A, (unsigned)n_short, s) : launch_dt<float, 64>(c, A, (unsigned)n_short, s);
+    if (e != cudaSuccess) return e;
+    A.list = list_long;
+    return bf ? launch_dt<__nv_bfloat16, kMaxUnit>(c, A, (unsigned)n_long, s)
+              : launch_dt<float, kMaxUnit>(c, A, (unsigned)n_long, s);
 }
 
 }  // namespace gkv

@@ -87,7 +87,8 @@ struct LongArgs {
     uint8_t *it_ufl;               // the node's unit holds a singleton-floor position
     LongRes *res;
     int32_t *u_start, *u_cnt;      // per listed unit: its block of work items
-    unsigned int *n_items;
+    unsigned int *n_items;         // [3]: work items, small subtrees (<= kShortUnit, <= kMaxUnit tokens)
+    int32_t *sub;                  // [2][cap_items] small subtrees' roots (global node indices)
     int64_t cap_items;
     // node records and unit arrays (build.cu's layout)
     int32_t *nd_a, *nd_b, *nd_child0, *nd_parent, *nd_unit;
@@ -213,7 +214,7 @@ __global__ void __launch_bounds__(kLT) long_collect_kernel(LongArgs A) {
         const float rootR = block_sum(r, sf);
         for (int k = tid; k < 2 * n; k += kLT) A.nd_cost[nbase + k] = 0;   // unused slots carry no op
         if (tid == 0) {
-            const unsigned int pos = atomicAdd(A.n_items, 1u);
+            const unsigned int pos = atomicAdd(&A.n_items[0], 1u);
             if ((int64_t)pos < A.cap_items) {
                 A.it_gv[pos] = nbase;
                 A.it_uid[pos] = uid;
@@ -241,10 +242,17 @@ __global__ void __launch_bounds__(kLT) long_collect_kernel(LongArgs A) {
     int cnt = 0;
     float pend = -1.f;
     for (int k = tid; k < nn; k += kLT) {
-        if (A.nd_nchild[nbase + k] != -1) continue;
-        const float bnd = A.nd_U[nbase + k];
-        if (bnd >= A.tau) cnt++;
-        else pend = fmaxf(pend, bnd);
+        const int64_t v = nbase + k;
+        if (A.nd_nchild[v] != -1) continue;
+        const float bnd = A.nd_U[v];
+        if (bnd < A.tau) { pend = fmaxf(pend, bnd); continue; }
+        const int len = A.nd_b[v] - A.nd_a[v];
+        if (len > kMaxUnit) { cnt++; continue; }
+        // a small node: its subtree goes to the unit kernel (subtree mode)
+        const int cls = len <= kShortUnit ? 0 : 1;
+        const unsigned int pos = atomicAdd(&A.n_items[1 + cls], 1u);
+        if ((int64_t)pos < A.cap_items) A.sub[(size_t)cls * A.cap_items + pos] = (int32_t)v;
+        else atomicOr(A.status, 64);
     }
     pend = warp_max(pend);
     if (lane == 0) sf[warp] = pend;
@@ -255,7 +263,7 @@ __global__ void __launch_bounds__(kLT) long_collect_kernel(LongArgs A) {
         A.u_pend[uid] = pm;
         int b0 = 0;
         if (cnt > 0) {
-            const unsigned int pos = atomicAdd(A.n_items, (unsigned)cnt);
+            const unsigned int pos = atomicAdd(&A.n_items[0], (unsigned)cnt);
             if ((int64_t)pos + cnt <= A.cap_items) {
                 b0 = (int)pos;
             } else {
@@ -274,7 +282,8 @@ __global__ void __launch_bounds__(kLT) long_collect_kernel(LongArgs A) {
     for (int k0 = 0; k0 < nn; k0 += kLT) {
         const int k = k0 + tid;
         bool q = false;
-        if (k < nn && A.nd_nchild[nbase + k] == -1) q = A.nd_U[nbase + k] >= A.tau;
+        if (k < nn && A.nd_nchild[nbase + k] == -1)
+            q = A.nd_U[nbase + k] >= A.tau && A.nd_b[nbase + k] - A.nd_a[nbase + k] > kMaxUnit;
         const unsigned bal = __ballot_sync(0xffffffffu, q);
         if (lane == 0) wcnt[warp] = __popc(bal);
         __syncthreads();
@@ -960,13 +969,20 @@ __global__ void long_commit_kernel(LongArgs A) {
         const bool in = k < cnt;
         LongRes rs;
         int64_t gv = 0;
-        int nch = 0;
+        int nch = 0, used = 0;
         if (in) {
             rs = A.res[start + k];
             gv = A.it_gv[start + k];
             nch = rs.nch > 0 ? rs.nch : 0;
+            // the children's slots, then for each child of 2 .. kMaxUnit tokens the
+            // 2 len - 2 slots its subtree can need (the unit kernel fills them)
+            used = nch;
+            for (int q = 0; q < nch; q++) {
+                const int len = rs.cb[q] - rs.ca[q];
+                if (len >= 2 && len <= kMaxUnit) used += 2 * len - 2;
+            }
         }
-        int incl = nch;
+        int incl = used;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
             const int y = __shfl_up_sync(0xffffffffu, incl, o);
@@ -982,19 +998,31 @@ __global__ void long_commit_kernel(LongArgs A) {
                 A.nd_child0[gv] = -1; A.nd_nchild[gv] = 0; A.nd_cost[gv] = 0;
                 A.nd_U[gv] = 0.f; A.nd_kappa[gv] = 0.f; A.nd_sel[gv] = 0;
             } else {
-                const int child0 = base + incl - nch;   // local index
+                const int child0 = base + incl - used;   // unit-relative index
                 const int cost = nch - 1;
                 A.nd_child0[gv] = child0; A.nd_nchild[gv] = (int8_t)nch; A.nd_cost[gv] = (int8_t)cost;
                 A.nd_U[gv] = rs.U; A.nd_kappa[gv] = rs.kap; A.nd_sel[gv] = 0;
                 A.ops[atomicAdd(A.n_ops, 1u)] =
                     make_uint2(__float_as_uint(rs.kap), ((uint32_t)gv << 1) | (uint32_t)(cost - 1));
+                int res = child0 + nch;
                 for (int q = 0; q < nch; q++) {
                     const int64_t gc = nbase + child0 + q;
-                    const bool pending = rs.cb[q] - rs.ca[q] >= 2;
+                    const int len = rs.cb[q] - rs.ca[q];
+                    const bool pending = len >= 2;
                     A.nd_a[gc] = rs.ca[q]; A.nd_b[gc] = rs.cb[q];
                     A.nd_parent[gc] = (int32_t)gv; A.nd_unit[gc] = (int32_t)uid;
                     A.nd_D[gc] = rs.cD[q]; A.nd_R[gc] = rs.rch[q];
-                    A.nd_child0[gc] = -1; A.nd_nchild[gc] = pending ? -1 : 0; A.nd_cost[gc] = 0;
+                    // a pending child of at most kMaxUnit tokens keeps its reservation in
+                    // child0; the reserved slots are marked unused (child count -2) until
+                    // the unit kernel fills them
+                    A.nd_child0[gc] = (pending && len <= kMaxUnit) ? res : -1;
+                    if (pending && len <= kMaxUnit) {
+                        for (int r = res; r < res + 2 * len - 2; r++) {
+                            A.nd_nchild[nbase + r] = -2; A.nd_cost[nbase + r] = 0; A.nd_sel[nbase + r] = 0;
+                        }
+                        res += 2 * len - 2;
+                    }
+                    A.nd_nchild[gc] = pending ? -1 : 0; A.nd_cost[gc] = 0;
                     A.nd_U[gc] = pending ? rs.bnd[q] : 0.f;   // a pending node's key bound
                     A.nd_kappa[gc] = 0.f; A.nd_sel[gc] = 0;
                     if (pending) pend = fmaxf(pend, rs.bnd[q]);
@@ -1079,27 +1107,34 @@ cudaError_t launch_long_level(Ctx &c, const void *K, const void *V, const void *
     A.u_sel = w.u_sel;
     A.status = w.dev_int + 1;
     A.work = w.work;
-    cudaError_t e = cudaMemsetAsync(w.long_n, 0, sizeof(unsigned int), s);
+    A.sub = w.long_sub;
+    cudaError_t e = cudaMemsetAsync(w.long_n, 0, 3 * sizeof(unsigned int), s);
     if (e != cudaSuccess) return e;
     long_collect_kernel<<<(unsigned)n_units, kLT, 0, s>>>(A);
     c.launches += 1;
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    unsigned grid = (unsigned)c.num_sms * 2;
-    if (n_items_host) {
-        e = cudaMemcpyAsync(n_items_host, w.long_n, sizeof(unsigned int), cudaMemcpyDeviceToHost, s);
-        if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-        if (e != cudaSuccess) return e;
-        if (*n_items_host == 0) return cudaSuccess;
-        grid = (unsigned)std::min<int64_t>((int64_t)grid, (int64_t)*n_items_host);
-    }
-    e = p.dtype == GKV_BF16
-            ? (p.d == 128 ? launch_eval<128, __nv_bfloat16>(c, A, grid, s) : launch_eval<64, __nv_bfloat16>(c, A, grid, s))
-            : (p.d == 128 ? launch_eval<128, float>(c, A, grid, s) : launch_eval<64, float>(c, A, grid, s));
+    // the level's counts: long work items, small subtrees of each class
+    unsigned int cnt[3] = {0, 0, 0};
+    e = cudaMemcpyAsync(cnt, w.long_n, sizeof cnt, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return e;
-    long_commit_kernel<<<(unsigned)n_units, 32, 0, s>>>(A);
-    c.launches += 1;
-    return cudaGetLastError();
+    for (int q = 0; q < 3; q++) cnt[q] = (unsigned)std::min<int64_t>((int64_t)cnt[q], w.long_cap);
+    if (n_items_host) *n_items_host = cnt[0] + cnt[1] + cnt[2];
+    if (cnt[0] > 0) {
+        const unsigned grid = (unsigned)std::min<int64_t>((int64_t)c.num_sms * 2, (int64_t)cnt[0]);
+        e = p.dtype == GKV_BF16
+                ? (p.d == 128 ? launch_eval<128, __nv_bfloat16>(c, A, grid, s) : launch_eval<64, __nv_bfloat16>(c, A, grid, s))
+                : (p.d == 128 ? launch_eval<128, float>(c, A, grid, s) : launch_eval<64, float>(c, A, grid, s));
+        if (e != cudaSuccess) return e;
+        long_commit_kernel<<<(unsigned)n_units, 32, 0, s>>>(A);
+        c.launches += 1;
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    // nodes of at most kMaxUnit tokens: their subtrees on the unit kernel
+    return launch_unit_subtrees(c, K, V, Q, omega, slots, J, w.long_sub, (int)cnt[1], w.long_sub + w.long_cap,
+                                (int)cnt[2], s);
 }
 
 }  // namespace gkv

@@ -283,7 +283,7 @@ __global__ void __launch_bounds__(256) gather_list_long_kernel(GatherArgs A, con
     __syncthreads();
     auto frontier = [&](int k) {
         const int64_t v = nb + k;
-        if (A.nd_sel[v] == 1) return false;
+        if (A.nd_sel[v] == 1 || A.nd_nchild[v] == -2) return false;   // selected, or an unused slot
         const int32_t pg = A.nd_parent[v];
         return pg < 0 ? true : A.nd_sel[pg] == 1;   // the root is reached: its Add is selected
     };

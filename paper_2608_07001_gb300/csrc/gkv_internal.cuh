@@ -108,7 +108,9 @@ struct Workspace {
     uint8_t *long_ufl = nullptr;
     void *long_res = nullptr;      // [long_cap] results (long_res_bytes() each)
     int32_t *long_start = nullptr, *long_cnt = nullptr;   // [long_units_cap]
-    unsigned int *long_n = nullptr;                       // [1] work items of the level
+    unsigned int *long_n = nullptr;                       // [3] the level's work items, small subtrees
+                                                          //     of <= kShortUnit and <= kMaxUnit tokens
+    int32_t *long_sub = nullptr;    // [2][long_cap] the small subtrees' root nodes (global indices)
     int32_t *long_slots = nullptr;  // [N_c + 1] slot indices of the long slots
     int32_t *long_list = nullptr;   // [units_cap] long units to resume
 };
@@ -307,6 +309,13 @@ cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *
                               int root_only, int max_levels, float tau, const int32_t *list_short,
                               int n_short, const int32_t *list_long, int n_long, cudaStream_t s,
                               int lg0 = 0, int nlg = -1);   // fresh launches: (l, g) in [lg0, lg0 + nlg);
+// Subtree mode of the unit kernel (build.cu): the listed pending nodes of
+// long units (global node indices; at most kShortUnit tokens in list_short,
+// at most kMaxUnit in list_long) each get their subtree built to the leaves
+// into the node slots reserved for it (its child0, unit-relative).
+cudaError_t launch_unit_subtrees(Ctx &c, const void *K, const void *V, const void *Q, const float *omega,
+                                 const int32_t *slots, int J, const int32_t *list_short, int n_short,
+                                 const int32_t *list_long, int n_long, cudaStream_t s);
 // Slot indices split by length class: short ones at list[0, count[0]), those
 // of kShortUnit + 1 .. kMaxUnit tokens at list[J - count[1], J), longer ones
 // at long_slots[0, count[2]); count[3] receives the tokens of the longer ones.
