@@ -55,6 +55,7 @@ constexpr int kLNCD = 20;         // candidate rows per direction (17 cuts + p* 
 constexpr int kLMaxCut = 18;      // K + midpoint, K <= 16 (+1 spare)
 constexpr int kLMaxSeg = 24;      // segments between the boundaries a, b, the cuts, p*, p* + 1
 constexpr int kLFold = 32;        // tokens per fp32 partial sum of a scan
+constexpr int kLChunk = 32;       // tokens per staged chunk of a scan
 
 struct LongRes {
     int nch;               // -1: pending (root only), 0: leaf (non-finite inputs), 2 or 3
@@ -320,6 +321,9 @@ struct LongSmem {
     float ktil[2 * kLNCD][DH], vtil[2 * kLNCD][DH];
     float redD[2 * kLNCD][kLNW], redP[2 * kLNCD][kLNW];
     float candD[2 * kLNCD], candP[2 * kLNCD], meff[2 * kLNCD];
+    // the probe scans' staging ring: per buffer kLChunk value rows, then as
+    // many probe-weight rows (32 float2) or key rows
+    __align__(16) unsigned char ring[2][kLChunk * DH * 4 * 2];
     int ca[2 * kLNCD], cb[2 * kLNCD];   // prefixes at [0, npre) by ascending end, suffixes at
                                         // [kLNCD, kLNCD + nsuf) by descending start (absolute)
     int segb[kLMaxSeg + 1];
@@ -748,10 +752,19 @@ __global__ void __launch_bounds__(kLT, 1) long_eval_kernel(LongArgs A) {
             if (lane == 0) { sm.redD[k][warp] = pd; sm.redP[k][warp] = pw; }
         };
         // one direction: the running sums over the node's tokens, folded every
-        // kLFold tokens and at every candidate end, evaluated at each end
+        // kLFold tokens and at every candidate end, evaluated at each end.  The
+        // tokens are staged kLChunk at a time in a two-buffer cp.async ring:
+        // their value rows and their probe weights (pass B) or key rows.
         auto scan = [&](bool suffix) {
             const int nk = suffix ? nsuf : npre;
             if (nk == 0) return;
+            // tokens of the scan: forward a, a + 1, ..; backward b - 1, b - 2, ..
+            int last = suffix ? b : a;     // the farthest candidate end
+            for (int k = 0; k < nk; k++) {
+                const int kr = suffix ? kLNCD + k : k;
+                last = suffix ? min(last, sm.ca[kr]) : max(last, sm.cb[kr]);
+            }
+            const int ntok = suffix ? b - last : last - a;
             float2 Mt0[CH / 2], Mt1[CH / 2], Mc0[CH / 2], Mc1[CH / 2];
             float Zt0 = 0.f, Zt1 = 0.f, Zc0 = 0.f, Zc1 = 0.f;
 #pragma unroll
@@ -764,23 +777,55 @@ __global__ void __launch_bounds__(kLT, 1) long_eval_kernel(LongArgs A) {
                 }
                 Zt0 += Zc0; Zt1 += Zc1; Zc0 = Zc1 = 0.f;
             };
-            int t = suffix ? b - 1 : a, fold = 0;
+            // chunk c holds the scan's tokens [c kLChunk, (c + 1) kLChunk): rows
+            // tlo .. tlo + m - 1 of the input, tlo the smallest position
+            auto chunk_rows = [&](int c0, int &tlo, int &m) {
+                m = min(kLChunk, ntok - c0);
+                tlo = suffix ? b - c0 - m : a + c0;
+            };
+            auto issue = [&](int c0, int buf) {
+                if (c0 < ntok) {
+                    int tlo, m;
+                    chunk_rows(c0, tlo, m);
+                    unsigned char *dst = sm.ring[buf];
+                    constexpr int RB = DH * (int)sizeof(Tin);             // bytes of a K or V row
+                    const char *vsrc = reinterpret_cast<const char *>(Vl + (size_t)tlo * DH);
+                    for (int q = tid; q < m * RB / 16; q += kLT) cp_async16(dst + 16 * q, vsrc + 16 * q, true);
+                    unsigned char *dst2 = dst + kLChunk * RB;
+                    if (A.Eg) {
+                        const char *esrc = reinterpret_cast<const char *>(A.Eg + ((size_t)lg * A.Nc + (tlo - A.cs)) * kLPP);
+                        for (int q = tid; q < m * kLPP * 8 / 16; q += kLT) cp_async16(dst2 + 16 * q, esrc + 16 * q, true);
+                    } else {
+                        const char *ksrc = reinterpret_cast<const char *>(Kl + (size_t)tlo * DH);
+                        for (int q = tid; q < m * RB / 16; q += kLT) cp_async16(dst2 + 16 * q, ksrc + 16 * q, true);
+                    }
+                }
+                cp_async_commit();
+            };
+            int kk = 0, fold = 0;
             bool badt = false;
-            for (int kk = 0; kk < nk; kk++) {
-                const int k = suffix ? kLNCD + kk : kk;
-                const int stop = suffix ? sm.ca[k] : sm.cb[k];
-#pragma unroll 1
-                for (; suffix ? t >= stop : t < stop; t += suffix ? -1 : 1) {
+            issue(0, 0);
+            for (int c0 = 0, buf = 0; c0 < ntok; c0 += kLChunk, buf ^= 1) {
+                issue(c0 + kLChunk, buf ^ 1);
+                cp_async_wait<1>();   // this chunk's copies have landed (each thread its own)
+                __syncthreads();
+                int tlo, m;
+                chunk_rows(c0, tlo, m);
+                const Tin *vrow0 = reinterpret_cast<const Tin *>(sm.ring[buf]);
+                const unsigned char *aux = sm.ring[buf] + kLChunk * DH * (int)sizeof(Tin);
+                for (int i = 0; i < m; i++) {
+                    const int r = suffix ? m - 1 - i : i;   // row of the scan's token c0 + i
                     float e0, e1;
                     if (A.Eg) {
-                        const float2 e = A.Eg[((size_t)lg * A.Nc + (t - A.cs)) * kLPP + pp];
+                        const float2 e = reinterpret_cast<const float2 *>(aux)[r * kLPP + pp];
                         e0 = has0 ? e.x : 0.f;
                         e1 = has1 ? e.y : 0.f;
                     } else {
+                        const Tin *krow = reinterpret_cast<const Tin *>(aux) + (size_t)r * DH;
                         float2 ya = make_float2(0.f, 0.f), yb = ya;
 #pragma unroll
                         for (int gi = 0; gi < NG; gi++) {
-                            const float4 kv = lld4(Kl + (size_t)t * DH + 4 * c + 32 * gi);
+                            const float4 kv = lld4(krow + 4 * c + 32 * gi);
                             const float2 ka = make_float2(kv.x, kv.y), kb = make_float2(kv.z, kv.w);
                             ya = ffma2(qa0[2 * gi], ka, ya); ya = ffma2(qa0[2 * gi + 1], kb, ya);
                             yb = ffma2(qa1[2 * gi], ka, yb); yb = ffma2(qa1[2 * gi + 1], kb, yb);
@@ -798,9 +843,10 @@ __global__ void __launch_bounds__(kLT, 1) long_eval_kernel(LongArgs A) {
                     const float2 ee0 = make_float2(e0, e0), ee1 = make_float2(e1, e1);
                     Zc0 += e0;
                     Zc1 += e1;
+                    const Tin *vrow = vrow0 + (size_t)r * DH;
 #pragma unroll
                     for (int gi = 0; gi < NG; gi++) {
-                        const float4 x = lld4(Vl + (size_t)t * DH + 4 * c + 32 * gi);
+                        const float4 x = lld4(vrow + 4 * c + 32 * gi);
                         const float2 va = make_float2(x.x, x.y), vb = make_float2(x.z, x.w);
                         Mc0[2 * gi] = ffma2(ee0, va, Mc0[2 * gi]);
                         Mc0[2 * gi + 1] = ffma2(ee0, vb, Mc0[2 * gi + 1]);
@@ -808,11 +854,20 @@ __global__ void __launch_bounds__(kLT, 1) long_eval_kernel(LongArgs A) {
                         Mc1[2 * gi + 1] = ffma2(ee1, vb, Mc1[2 * gi + 1]);
                     }
                     if (++fold == kLFold) { fold_in(); fold = 0; }
+                    // candidates whose far end is this token
+                    const int t = suffix ? b - 1 - (c0 + i) : a + c0 + i;
+                    while (kk < nk) {
+                        const int kr = suffix ? kLNCD + kk : kk;
+                        if ((suffix ? sm.ca[kr] : sm.cb[kr] - 1) != t) break;
+                        fold_in();
+                        fold = 0;
+                        evaluate(kr, Zt0, Zt1, Mt0, Mt1);
+                        kk++;
+                    }
                 }
-                fold_in();
-                fold = 0;
-                evaluate(k, Zt0, Zt1, Mt0, Mt1);
+                __syncthreads();   // the buffer is refilled by the next issue
             }
+            cp_async_wait<0>();
             if (badt) sm.bad = 1;
         };
         scan(false);
