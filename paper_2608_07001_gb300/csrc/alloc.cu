@@ -38,7 +38,7 @@ namespace gkv {
 namespace {
 
 // alloc_state layout (unsigned long long)
-enum { ST_PREFIX = 0, ST_ABOVE, ST_ALL, ST_R, ST_ENDU, ST_ENDKEY, ST_TOTAL, ST_USED, ST_CROSS, ST_N };
+enum { ST_PREFIX = 0, ST_ABOVE, ST_ALL, ST_R, ST_ENDU, ST_ENDKEY, ST_TOTAL, ST_USED, ST_CROSS, ST_NTIE, ST_N };
 static_assert(ST_N <= 16, "alloc_state holds 16 words per segment");
 
 struct AllocArgs {
@@ -294,49 +294,104 @@ __global__ void alloc_tie_cost_kernel(AllocArgs A) {
         }
     }
     A.u_tcost[u] = cost;
+    if (cost > 0) atomicAdd(&seg_st(A, A.nseg > 1 ? (int)(u / A.J) : 0)[ST_NTIE], 1ull);
 }
 
-// One block per segment: ordered inclusive scan of the closure costs.
-__global__ void __launch_bounds__(1024) alloc_tie_scan_kernel(AllocArgs A) {
+// Ordered scan of the closure costs per segment, in three steps over chunks
+// of 1024 units (chunk c of segment seg covers units u_lo + 1024 c ..):
+// chunk sums, an exclusive scan of a segment's chunk sums, then each unit's
+// state -- 1: its whole closure fits, 2: the crossing unit (ST_CROSS, with the
+// budget left for it in ST_R), 0: otherwise.
+constexpr int kTieChunk = 1024;
+__device__ __forceinline__ void seg_units(const AllocArgs &A, int seg, int64_t &u_lo, int64_t &u_hi) {
+    u_lo = A.nseg > 1 ? (int64_t)seg * A.J : 0;
+    u_hi = A.nseg > 1 ? u_lo + A.J : A.n_units;
+}
+__device__ __forceinline__ long long block_incl_scan(long long c, long long *wsum, long long &total) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    long long incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const long long y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    long long before = 0;
+    total = 0;
+    for (int w = 0; w < 32; w++) {
+        if (w < warp) before += wsum[w];
+        total += wsum[w];
+    }
+    __syncthreads();
+    return before + incl;
+}
+
+// grid (chunks per segment, segments)
+__global__ void __launch_bounds__(kTieChunk) alloc_tie_bsum_kernel(AllocArgs A, long long *bsum, int nch) {
     __shared__ long long wsum[32];
-    __shared__ long long carry_s;
-    const int seg = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int seg = blockIdx.y, c = blockIdx.x;
+    const unsigned long long *st = seg_st(A, seg);
+    if (st[ST_ALL] || st[ST_NTIE] == 0) return;
+    int64_t u_lo, u_hi;
+    seg_units(A, seg, u_lo, u_hi);
+    const int64_t u = u_lo + (int64_t)c * kTieChunk + threadIdx.x;
+    long long tot;
+    block_incl_scan(u < u_hi ? (long long)A.u_tcost[u] : 0, wsum, tot);
+    if (threadIdx.x == 0) bsum[(size_t)seg * nch + c] = tot;
+}
+
+// one block per segment: exclusive prefix of its chunk sums
+__global__ void __launch_bounds__(kTieChunk) alloc_tie_bscan_kernel(AllocArgs A, long long *bsum, int nch) {
+    __shared__ long long wsum[32];
+    __shared__ long long carry;
+    const int seg = blockIdx.x;
     unsigned long long *st = seg_st(A, seg);
     if (st[ST_ALL]) return;
     const long long R = seg_budget(A, seg) - (long long)st[ST_ABOVE];
-    const int64_t u_lo = A.nseg > 1 ? (int64_t)seg * A.J : 0;
-    const int64_t u_hi = A.nseg > 1 ? u_lo + A.J : A.n_units;
-    if (tid == 0) carry_s = 0;
+    if (st[ST_NTIE] == 0) {   // no tie op is exposed: nothing to order
+        if (threadIdx.x == 0) st[ST_R] = (unsigned long long)R;
+        return;
+    }
+    if (threadIdx.x == 0) carry = 0;
     __syncthreads();
-    for (int64_t base = u_lo; base < u_hi; base += 1024) {
-        const int64_t u = base + tid;
-        const long long c = u < u_hi ? (long long)A.u_tcost[u] : 0;
-        long long incl = c;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const long long y = __shfl_up_sync(0xffffffffu, incl, o);
-            if (lane >= o) incl += y;
-        }
-        if (lane == 31) wsum[warp] = incl;
+    long long *b = bsum + (size_t)seg * nch;
+    for (int c0 = 0; c0 < nch; c0 += kTieChunk) {
+        const int c = c0 + threadIdx.x;
+        const long long x = c < nch ? b[c] : 0;
+        long long tot;
+        const long long incl = block_incl_scan(x, wsum, tot);
+        if (c < nch) b[c] = carry + incl - x;
         __syncthreads();
-        long long before = carry_s;
-        for (int w = 0; w < warp; w++) before += wsum[w];
-        const long long hi = before + incl, lo = hi - c;   // prefix after / before this unit
-        if (u < u_hi) {
-            int state = 0;
-            if (c > 0 && hi <= R) state = 1;                 // its whole closure fits
-            else if (c > 0 && lo <= R && hi > R) {           // the crossing unit
-                state = 2;
-                st[ST_CROSS] = (unsigned long long)u;
-                st[ST_R] = (unsigned long long)(R - lo);
-            }
-            A.u_flag[u] = state;
-        }
-        __syncthreads();
-        if (tid == 1023) carry_s = hi;
+        if (threadIdx.x == 0) carry += tot;
         __syncthreads();
     }
-    if (tid == 0 && st[ST_CROSS] == ~0ull) st[ST_R] = (unsigned long long)(R - carry_s);
+    if (threadIdx.x == 0 && carry <= R) st[ST_R] = (unsigned long long)(R - carry);   // every closure fits
+}
+
+// grid (chunks per segment, segments): each unit's state and the crossing unit
+__global__ void __launch_bounds__(kTieChunk) alloc_tie_scan_kernel(AllocArgs A, const long long *bsum, int nch) {
+    __shared__ long long wsum[32];
+    const int seg = blockIdx.y, c = blockIdx.x;
+    unsigned long long *st = seg_st(A, seg);
+    if (st[ST_ALL] || st[ST_NTIE] == 0) return;
+    const long long R = seg_budget(A, seg) - (long long)st[ST_ABOVE];
+    int64_t u_lo, u_hi;
+    seg_units(A, seg, u_lo, u_hi);
+    const int64_t u = u_lo + (int64_t)c * kTieChunk + threadIdx.x;
+    const long long cost = u < u_hi ? (long long)A.u_tcost[u] : 0;
+    long long tot;
+    const long long hi = bsum[(size_t)seg * nch + c] + block_incl_scan(cost, wsum, tot), lo = hi - cost;
+    if (u < u_hi) {
+        int state = 0;
+        if (cost > 0 && hi <= R) state = 1;                 // its whole closure fits
+        else if (cost > 0 && lo <= R && hi > R) {           // the crossing unit (at most one)
+            state = 2;
+            st[ST_CROSS] = (unsigned long long)u;
+            st[ST_R] = (unsigned long long)(R - lo);
+        }
+        A.u_flag[u] = state;
+    }
 }
 
 __global__ void alloc_tie_apply_kernel(AllocArgs A) {
@@ -709,14 +764,21 @@ cudaError_t launch_allocate(Ctx &c, int J, cudaStream_t s) {
     const int blocks = grid_for(c, A.n_units + c.node_cap / 2);
     alloc_mark_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_tie_cost_kernel<<<(unsigned)((A.n_units + 255) / 256), 256, 0, s>>>(A);
-    alloc_tie_scan_kernel<<<A.nseg, 1024, 0, s>>>(A);
+    {
+        const int64_t seg_len = A.nseg > 1 ? (int64_t)J : A.n_units;
+        const int nch = (int)((seg_len + kTieChunk - 1) / kTieChunk);
+        const dim3 g((unsigned)std::max(nch, 1), (unsigned)A.nseg);
+        alloc_tie_bsum_kernel<<<g, kTieChunk, 0, s>>>(A, w.tie_bsum, nch);
+        alloc_tie_bscan_kernel<<<A.nseg, kTieChunk, 0, s>>>(A, w.tie_bsum, nch);
+        alloc_tie_scan_kernel<<<g, kTieChunk, 0, s>>>(A, w.tie_bsum, nch);
+    }
     alloc_tie_apply_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_ties_kernel<<<A.nseg, 1024, 0, s>>>(A);
     alloc_end_max_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_end_key_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_end_pick_kernel<<<blocks, 256, 0, s>>>(A);
     alloc_final_kernel<<<(A.nseg + 255) / 256, 256, 0, s>>>(A);
-    c.launches += 9;
+    c.launches += 11;
     return cudaGetLastError();
 }
 

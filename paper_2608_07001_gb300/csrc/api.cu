@@ -464,7 +464,8 @@ static gkv_status build_setup(gracekv_ctx *x, const int32_t *slot_starts, int32_
                   dalloc(x, &w.u_pend, cap) && dalloc(x, &w.u_list, cap) &&
                   (c.p.alpha_floor <= 0.0 || dalloc(x, &w.u_floor, cap)) &&
                   dalloc(x, &w.long_list, cap) &&
-                  dalloc(x, &w.u_bsum, cap / 1024 + 2);
+                  dalloc(x, &w.u_bsum, cap / 1024 + 2) &&
+                  dalloc(x, &w.tie_bsum, cap / 1024 + (int64_t)c.p.L * c.p.G + 2);
         if (!ok) return fail(x, GKV_ENOMEM, "build_trees: unit arrays");
         w.units_cap = cap;
     }

@@ -269,7 +269,9 @@ struct Smem {
     float rootR;                             // R of a fresh root
 };
 
-template <int DH, typename Tin, int NMAX>
+// SUB: the subtree mode (BuildArgs::subtree) as a compile-time flag, so that
+// the other instances carry none of its index mapping
+template <int DH, typename Tin, int NMAX, bool SUB>
 __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(BuildArgs A) {
     using S = Smem<DH, Tin, NMAX>;
     // thread (p, c): probes p and p + 32, elements 4 c + 32 g + j (g < NG, j < 4)
@@ -280,7 +282,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     int j, lg;
     int64_t gv_sub = -1;         // subtree mode: the pending node whose subtree this CTA builds
-    if (A.subtree) {
+    if constexpr (SUB) {
         gv_sub = A.list[blockIdx.x];
         const int uidr = A.nd_unit[gv_sub];
         lg = uidr / A.J;
@@ -293,19 +295,20 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         j = A.list[blockIdx.x / A.nlg];   // slot-major: the units of a slot share its table rows
         lg = A.lg0 + blockIdx.x % A.nlg;
     }
-    const bool fresh = !A.resume && !A.subtree;
+    const bool fresh = !A.resume && !SUB;
     const int l = lg / A.G, g = lg - l * A.G;
     const int64_t uid = (int64_t)lg * A.J + j;
     const int64_t nbase = node_base(lg, A.slots[j], A.cs, A.Nc);   // the unit's node slots
     // the tokens held: the slot, or in subtree mode the node's interval
-    const int sa = A.subtree ? A.nd_a[gv_sub] : A.slots[j];
-    const int sb = A.subtree ? A.nd_b[gv_sub] : A.slots[j + 1];
+    const int sa = SUB ? A.nd_a[gv_sub] : A.slots[j];
+    const int sb = SUB ? A.nd_b[gv_sub] : A.slots[j + 1];
     const int n = sb - sa;
     // global node index of local node k, and its index inside the unit: the
     // local nodes of a subtree are its root and then its reserved slots
-    const int64_t sub_res = A.subtree ? (int64_t)A.nd_child0[gv_sub] : 0;
+    const int64_t sub_res = SUB ? (int64_t)A.nd_child0[gv_sub] : 0;
     auto gidx = [&](int k) -> int64_t {
-        return A.subtree ? (k == 0 ? gv_sub : nbase + sub_res + (k - 1)) : nbase + k;
+        if constexpr (SUB) return k == 0 ? gv_sub : nbase + sub_res + (k - 1);
+        else return nbase + k;
     };
     if (n < 1 || n > NMAX) {
         if (tid == 0) atomicOr(A.status, 4);
@@ -476,7 +479,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         for (int e = tid; e < n * 2 * kNPP; e += kNT) bad |= !isfinite(Ef[e]);
         for (int t = tid; t < n; t += kNT) bad |= !isfinite(sm.Rt[t]);
         if (__syncthreads_or(bad)) {
-            if (A.subtree) {   // the node stays a leaf; the unit is reported
+            if constexpr (SUB) {   // the node stays a leaf; the unit is reported
                 if (tid == 0) {
                     atomicOr(A.status, 8);
                     A.nd_nchild[gv_sub] = 0; A.nd_child0[gv_sub] = -1; A.nd_cost[gv_sub] = 0;
@@ -538,7 +541,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         }
     }
     // ---- tree state: a fresh root, a subtree's root, or the unit's records so far
-    if (A.subtree) {
+    if constexpr (SUB) {
         if (tid == 0) {
             NodeS &nd = sm.nodes[0];
             nd.a = 0; nd.b = (short)n; nd.parent = -1; nd.child0 = -1; nd.nchild = -1;
@@ -1174,7 +1177,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     if (lane == 0) { sm.wcnt[warp][0] = w_scan; sm.wcnt[warp][1] = w_eval; sm.wcnt[warp][2] = w_len; }
     __syncthreads();
     if (tid == 0) {
-        if (!A.subtree) {   // a subtree is built completely inside its reserved slots
+        if constexpr (!SUB) {   // a subtree is built completely inside its reserved slots
             A.u_nnodes[uid] = sm.nnodes;
             A.u_pend[uid] = sm.pend;
         }
@@ -1192,23 +1195,23 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
         for (int k = sm.nnodes + tid; k < 2 * n; k += kNT) A.nd_cost[nbase + k] = 0;
 }
 
-template <int DH, typename Tin, int NMAX>
+template <int DH, typename Tin, int NMAX, bool SUB = false>
 cudaError_t launch_t(Ctx &c, BuildArgs &A, unsigned grid, cudaStream_t s) {
     using S = Smem<DH, Tin, NMAX>;
     static_assert(sizeof(S) <= 227 * 1024, "unit kernel shared memory above the per-CTA limit");
     if (grid == 0) return cudaSuccess;
     size_t sm = sizeof(S);
-    cudaError_t e = cudaFuncSetAttribute(unit_build_kernel<DH, Tin, NMAX>,
+    cudaError_t e = cudaFuncSetAttribute(unit_build_kernel<DH, Tin, NMAX, SUB>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
-    unit_build_kernel<DH, Tin, NMAX><<<grid, kNT, sm, s>>>(A);
+    unit_build_kernel<DH, Tin, NMAX, SUB><<<grid, kNT, sm, s>>>(A);
     c.launches += 1;
     return cudaGetLastError();
 }
 
-template <typename Tin, int NMAX>
+template <typename Tin, int NMAX, bool SUB = false>
 cudaError_t launch_dt(Ctx &c, BuildArgs &A, unsigned grid, cudaStream_t s) {
-    return c.p.d == 128 ? launch_t<128, Tin, NMAX>(c, A, grid, s) : launch_t<64, Tin, NMAX>(c, A, grid, s);
+    return c.p.d == 128 ? launch_t<128, Tin, NMAX, SUB>(c, A, grid, s) : launch_t<64, Tin, NMAX, SUB>(c, A, grid, s);
 }
 
 }  // namespace
@@ -1289,11 +1292,12 @@ cudaError_t launch_unit_subtrees(Ctx &c, const void *K, const void *V, const voi
     A.nlg = p.L * p.G;
     const bool bf = p.dtype == GKV_BF16;
     A.list = list_short;
-    e = bf ? launch_dt<__nv_bfloat16, 64>(c, A, (unsigned)n_short, s) : launch_dt<float, 64>(c, A, (unsigned)n_short, s);
+    e = bf ? launch_dt<__nv_bfloat16, 64, true>(c, A, (unsigned)n_short, s)
+           : launch_dt<float, 64, true>(c, A, (unsigned)n_short, s);
     if (e != cudaSuccess) return e;
     A.list = list_long;
-    return bf ? launch_dt<__nv_bfloat16, kMaxUnit>(c, A, (unsigned)n_long, s)
-              : launch_dt<float, kMaxUnit>(c, A, (unsigned)n_long, s);
+    return bf ? launch_dt<__nv_bfloat16, kMaxUnit, true>(c, A, (unsigned)n_long, s)
+              : launch_dt<float, kMaxUnit, true>(c, A, (unsigned)n_long, s);
 }
 
 }  // namespace gkv

@@ -90,6 +90,7 @@ struct Workspace {
     int64_t *u_off = nullptr;      // entry offset of each unit's frontier
     int32_t *u_list = nullptr;     // compacted unit ids (ties)
     long long *u_bsum = nullptr;   // [units_cap / 1024 + 2] block sums of the gather's offset scan
+    long long *tie_bsum = nullptr; // [units_cap / 1024 + L G + 2] chunk sums of the allocation's tie scan
     // allocation
     unsigned long long *hist = nullptr;        // [2048] cost-weighted histogram
     unsigned long long *alloc_state = nullptr; // see alloc.cu
