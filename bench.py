@@ -37,6 +37,11 @@ METRIC = "context tokens compressed/sec per GB300 and % of HBM roofline (vs CPU 
 PEAK_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
                  "sm_max_mhz": 2070.0}
 FP32_LANES = 128
+# DRAM bytes of one compression in the dominant stage, from an ncu capture
+# (profiles/unit_build_llama128k_2layers_32x.md: the 2-layer slice's 2.31 GB
+# scaled by 16 to 32 layers); reported only for the workload it was taken on
+STAGE_TRAFFIC = {("unit_trees", "llama128k@32x"): (36.994e9, "ncu dram bytes of every unit_build launch "
+                                                           "of one compression on the 2-layer slice x 16")}
 
 
 def peaks():
@@ -467,9 +472,12 @@ def main():
                  + 6 * d * work["cand_len_sum"] + 2 * Wp * d * L * G * comp.ctx.n_c)
         peak = n_sms * FP32_LANES * 2 * pk.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
         ach = flops / (per_step[dom] / 1e3) / 1e12
+        tr = STAGE_TRAFFIC.get((dom, workload_config(w, args.ratio, L)["workload"]))
         roof = {"kernel": "unit_build_kernel", "bound": "alu", "achieved": ach, "peak": peak,
-                "unit": "TFLOP/s", "frac": ach / peak, "traffic": None,
+                "unit": "TFLOP/s", "frac": ach / peak, "traffic": None if tr is None else tr[0],
                 "peak_basis": f"{n_sms} SMs x {FP32_LANES} fp32 lanes x 2 x max SM clock"}
+        if tr is not None:
+            roof["traffic_basis"] = tr[1]
     elif dom in ("row_stats", "token_values"):
         flops = 2 * L * Q.shape[1] * Wp * d * (T if dom == "row_stats" else comp.ctx.n_c)
         peak = n_sms * FP32_LANES * 2 * pk.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
