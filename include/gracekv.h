@@ -126,6 +126,14 @@ typedef struct {
      * 0.75.  Needs bf16, d in {64, 128} and N_c <= 131072 (GKV_EUNSUPPORTED). */
     double eta_seed, rho_hop;
     int32_t m_seed, r_hop;
+    /* Execution of the segmentation DP (App. B.3 Eq. app_dp_recurrence); the
+     * slots do not depend on it.  The recurrence runs in chunks of 32 steps of
+     * min(n_min, 16) endpoints on separate CTAs, each started dp_warmup tokens
+     * early from a flat state; a chunk whose state at its start is not the
+     * previous chunk's up to a constant is run again, in order, from the
+     * previous chunk's exact state.  0: 512 tokens (rounded up to whole steps);
+     * negative: one chunk, the plain sequential recurrence on one CTA. */
+    int32_t dp_warmup;
 } gkv_params;
 
 /* Fill *p with the paper's defaults; shapes and budget are left zero.  Host only. */
@@ -347,7 +355,9 @@ gkv_status gracekv_export_floor(gracekv_ctx *ctx, uint8_t *accepted, float *f, i
  * launched since it was created; work[0 .. n_work-1] (nullable) receives the
  * tree-building work of the last gracekv_build_trees: [0] probe-scan token
  * steps, [1] candidate intervals evaluated, [2] sum of candidate lengths,
- * [3] units built.
+ * [3] units built, [4] chunks of the last segmentation DP, [5] of those, the
+ * chunks that were run again from the exact state (their warm-up had not
+ * reached the true state up to a constant).
  */
 #define GRACEKV_N_STAGES 8
 gkv_status gracekv_profile(gracekv_ctx *ctx, int32_t enable);

@@ -99,6 +99,7 @@ gkv_status gracekv_default_params(gkv_params *p) {
     p->floor_c = 0.5; p->floor_gamma = 1.2; p->floor_eta = 0.95; p->floor_half = 3;   // App. A.5 Stage I
     p->eta_seed = 0.9; p->rho_hop = 0.5; p->m_seed = 64; p->r_hop = 2;               // App. A.4
     p->ctx_start = 0; p->ctx_end = -1;                 // -1: T
+    p->dp_warmup = 0;                                  // 512 tokens
     return GKV_OK;
 }
 
@@ -201,7 +202,8 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
     }
     int64_t Nc = (int64_t)p.ctx_end - r - p.ctx_start;
     if (Nc < 1) return GKV_EBUDGET;
-    if (Nc + 1 + 4096 > 227 * 1024) return GKV_EUNSUPPORTED;   // DP keeps lengths in shared memory
+    if (gkv::dp_smem_bytes(p, (int)std::min<int64_t>(Nc, 1 << 30)) > 227 * 1024 - 64)
+        return GKV_EUNSUPPORTED;   // the DP's backtracking keeps every endpoint's length in shared memory
     if (p.lambda_graph > 0.0 && Nc > gkv::multihop_max_context()) return GKV_EUNSUPPORTED;
 
     gracekv_ctx *x = new (std::nothrow) gracekv_ctx();
@@ -244,6 +246,8 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
     }
     const int nb = p.n_max - p.n_min + 1;
     const int64_t nrow = (int64_t)p.L * p.Hq * p.W;
+    int dp_S, dp_Wu, dp_nch;
+    gkv::dp_chunking(p, (int)Nc, &dp_S, &dp_Wu, &dp_nch);
     gkv::Workspace &w = c.w;
     bool ok = dalloc(x, &w.rope, (size_t)p.T * (p.d / 2)) &&
               dalloc(x, &w.rope_rel, (size_t)(2 * gkv::kMaxSlot - 1) * (p.d / 2)) &&
@@ -255,7 +259,9 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
               dalloc(x, &w.kappa, (size_t)p.T) && dalloc(x, &w.bscore, (size_t)p.T) &&
               dalloc(x, &w.zbuf, (size_t)p.T) && dalloc(x, &w.zdev, (size_t)p.T) && dalloc(x, &w.p2, (size_t)Nc + 1) &&
               dalloc(x, &w.ew, (size_t)(Nc + 1) * ((nb + 3) & ~3)) && dalloc(x, &w.ewt, (size_t)p.n_max + 1) &&
-              dalloc(x, &w.slots, (size_t)Nc + 2) &&
+              dalloc(x, &w.slots, (size_t)Nc + 2) && dalloc(x, &w.dp_len, (size_t)Nc + 16) &&
+              dalloc(x, &w.dp_head, (size_t)dp_nch * 128) && dalloc(x, &w.dp_tail, (size_t)dp_nch * 256) &&
+              dalloc(x, &w.dp_rev, (size_t)Nc + 1) &&
               dalloc(x, &w.dev_int, 16) &&
               dalloc(x, &w.row_m, (size_t)nrow) && dalloc(x, &w.row_Z, (size_t)nrow) &&
               dalloc(x, &w.row_ZC, (size_t)nrow) && dalloc(x, &w.rowp, (size_t)3 * nrow * c.n_chunks) &&
@@ -374,10 +380,17 @@ gkv_status gracekv_segment(gracekv_ctx *x, const void *V, const float *hidden, i
         if (e == cudaSuccess) e = launch_score(c, c.score_K, c.score_Q, c.score_stream);
     }
     if (e != cudaSuccess) return cuda_fail(x, e, "segment launch");
-    int h[2];
-    e = cudaMemcpyAsync(h, c.w.dev_int, 2 * sizeof(int), cudaMemcpyDeviceToHost, s);
+    int h[gkv::kDpRerun + 1];
+    e = cudaMemcpyAsync(h, c.w.dev_int, sizeof h, cudaMemcpyDeviceToHost, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_fail(x, e, "segment");
+    if (c.p.seg_mode == 0) {
+        int S, Wu;
+        gkv::dp_chunking(c.p, c.Nc, &S, &Wu, &c.dp_chunks);
+        c.dp_rerun = h[gkv::kDpRerun];
+    } else {
+        c.dp_chunks = c.dp_rerun = 0;
+    }
     st = check_status(x, h[1]);
     if (st) return st;
     if (h[0] <= 0) return fail(x, GKV_EINVAL, "segmentation found no partition");
@@ -987,7 +1000,8 @@ gkv_status gracekv_stats(gracekv_ctx *x, float *stage_ms, int32_t n_stages, int6
         unsigned long long h[4] = {0, 0, 0, 0};
         cudaError_t e = cudaMemcpy(h, c.w.work, sizeof h, cudaMemcpyDeviceToHost);
         if (e != cudaSuccess) return cuda_fail(x, e, "stats");
-        for (int i = 0; i < n_work; i++) work[i] = i < 4 ? h[i] : 0;
+        for (int i = 0; i < n_work; i++)
+            work[i] = i < 4 ? h[i] : i == 4 ? (uint64_t)c.dp_chunks : i == 5 ? (uint64_t)c.dp_rerun : 0;
     }
     if (stage_ms) {
         for (int i = 0; i < n_stages; i++) stage_ms[i] = 0.f;

@@ -18,6 +18,7 @@ constexpr int kMaxSlot = 16384;     // longest slot of a supplied partition (lon
 constexpr int kStPipeTimeout = 32;   // status bit: a bounded wait of a tensor-core pipeline gave up
 constexpr int kStLongCap = 64;       // status bit: the long-unit work items exceeded their capacity
 constexpr int kScoreStatus = 8;      // dev_int word of the score passes' status bits
+constexpr int kDpRerun = 9;          // dev_int word: segmentation DP chunks re-run from the exact state
 constexpr int kMaxSegLayers = 8;
 constexpr int kMaxWindows = 4;
 
@@ -41,7 +42,11 @@ struct Workspace {
     float *ew = nullptr;           // [(N_c + 1) * nbp] DP edge weights (len n_min..n_max), rows padded to 4
     float2 *ewt = nullptr;         // [n_max + 1] terminal edge weights (len 1..n_max) at i = N_c
     int32_t *slots = nullptr;      // [N_c + 2] slot starts (absolute)
-    int32_t *dev_int = nullptr;    // [8] small device scalars (J, status, ...)
+    uint8_t *dp_len = nullptr;     // [N_c + 16] DP: chosen slot length of every endpoint
+    float2 *dp_head = nullptr;     // [chunks][128] DP state (double-float) on the window ending at a chunk's start
+    float2 *dp_tail = nullptr;     // [chunks][256] DP state on the window ending at a chunk's end
+    int32_t *dp_rev = nullptr;     // [N_c + 1] DP: the path's endpoints from N down (backtracking)
+    int32_t *dev_int = nullptr;    // [16] small device scalars (J, status, counts, ...)
     unsigned long long *sel_state = nullptr;   // radix-select state for the median
     // row statistics and token values
     float *row_m = nullptr, *row_Z = nullptr, *row_ZC = nullptr;  // [L*Hq*W]
@@ -138,6 +143,7 @@ struct Ctx {
     int mh_ngraph = 0;
     int build_passes = 1;          // unit-kernel launches of the last build (pruning passes)
     int n_long = 0;                // slots of the last build longer than kMaxUnit (w.long_slots)
+    int dp_chunks = 0, dp_rerun = 0;   // last segmentation: DP chunks, chunks re-run from the exact state
     // score passes issued ahead by gracekv_score (consumed by the next build);
     // requested before a segmentation, they are enqueued when its dynamic
     // program (one block) starts, so that they overlap it
@@ -291,6 +297,10 @@ cudaError_t launch_rope_table(Ctx &c, cudaStream_t s);
 
 cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
                            const float *surprisal, float *kappa_out, cudaStream_t s);
+// chunks of the segmentation DP over N endpoints: endpoints per chunk, warm-up tokens, count
+void dp_chunking(const gkv_params &p, int N, int *S, int *Wu, int *nch);
+// shared memory of the DP's finish kernel (bytes) for N endpoints
+size_t dp_smem_bytes(const gkv_params &p, int N);
 
 // layers [l0, l1) (l1 < 0: all); a partial range needs use_tc(c)
 cudaError_t launch_row_stats(Ctx &c, const void *K, const void *Q, cudaStream_t s, int l0 = 0, int l1 = -1);

@@ -718,60 +718,89 @@ __global__ void seg_band_terminal_kernel(const Tin *V, const float *hidden, Band
 }
 
 // ---------------------------------------------------------------------------
-// DP: one block, one warp per endpoint.  Endpoints are processed 16 (or n_min,
-// if smaller) at a time: F[i..i+15] only read F[< i] because i - a >= n_min,
+// DP (App. B.3 Eq. app_dp_recurrence): F[i] = max over lengths of
+// F[i - len] + w(i - len, i), lengths in [n_min, n_max], ties to the lower
+// predecessor.  The chain is cut into chunks that run on separate CTAs.
+//
+// Inside a CTA, one warp per endpoint: endpoints are processed 16 (or n_min,
+// if smaller) at a time -- F[i..i+15] only read F[< i] because i - a >= n_min,
 // so one barrier per step suffices.  Lane handles the lengths n_min + lane +
 // 32 j; the warp reduces its candidates (value desc, a asc) with shuffles.
 // The edge weights do not depend on F: each warp streams its own endpoint
 // rows kDpPD steps ahead into a private shared-memory ring with cp.async.
-// The chosen slot length of every endpoint is kept in shared memory (uint8)
-// so the backtracking runs without global round trips.  The state F is a
-// double-float; the edge weights are fp32 (their rounding, ~1e-7 of a weight,
-// is far below the DP's near-tie margin).
+// The state F is a double-float; the edge weights are fp32 (their rounding,
+// ~1e-7 of a weight, is far below the DP's near-tie margin).
+//
+// Across CTAs: chunk c owns the endpoints (e_c, e_c+1], e_c = c S.  Its run
+// starts Wu tokens before e_c from F = 0 on a window of n_max positions
+// instead of the true state.  The decisions read only differences of F inside
+// the window, and once the optimal paths from the window have coalesced, the
+// run's F is the true F plus a constant: products of max-plus transition
+// matrices converge to rank one (Maleki, Musuvathi and Mytkowicz, PPoPP 2014,
+// "Parallelizing dynamic programming through rank convergence").  Each chunk
+// records its state on the kDpWin positions ending at e_c (its head) and its
+// ring at the end of the run (its tail).  Chunk c's decisions are the true ones
+// when chunk c - 1's are and the previous tail minus this head is constant over
+// the window: checked in fp64 to kDpTol relative, nine orders below any
+// decision margin the tests accept as distinct (a run that has not converged
+// differs by whole edge weights).  Chunk 0, and every chunk whose warm-up
+// would reach back to the context start, runs from the true state F[0] = 0.
+// The finish kernel checks every boundary, re-runs in order each chunk whose
+// check fails from the previous tail (then exact), and backtracks.
 // ---------------------------------------------------------------------------
 constexpr int kDpRing = 256;
-constexpr int kDpEp = 16;    // endpoints per step (warps)
-constexpr int kDpPD = 8;     // steps of edge weights in flight per warp
-constexpr int kDpLen = 4;    // lengths per lane: n_max - n_min + 1 <= 128
+constexpr int kDpEp = 16;         // endpoints per step (warps)
+constexpr int kDpPD = 8;          // steps of edge weights in flight per warp
+constexpr int kDpLen = 4;         // lengths per lane: n_max - n_min + 1 <= 128
+constexpr int kDpWin = 128;       // state window compared at a boundary (>= n_max)
+constexpr int kDpChunkSteps = 32; // steps per chunk
+constexpr double kDpTol = 1e-9;   // boundary check: relative spread of tail - head
 
-__host__ __device__ constexpr size_t dp_smem(int N, int nb) {
-    return (size_t)kDpRing * 8 + (size_t)kDpEp * kDpPD * dp_row(nb) * 4 + (((size_t)N + 1 + 15) & ~(size_t)15);
+__host__ __device__ constexpr size_t dp_smem_base(int nb) {
+    return (size_t)kDpRing * 8 + (size_t)kDpEp * kDpPD * dp_row(nb) * 4;
+}
+__host__ __device__ constexpr size_t dp_smem(int N, int nb, int nch) {
+    return dp_smem_base(nb) + (((size_t)N + 1 + 15) & ~(size_t)15) + (size_t)nch;
 }
 
 __device__ __forceinline__ bool better(df2 v, int a, df2 bv, int ba) {
     return df_gt(v, bv) || (df_eq(v, bv) && a < ba);
 }
 
-__global__ void __launch_bounds__(kDpEp * 32) seg_dp_kernel(const float *ew, const float2 *ewt, int N,
-                                                            int n_min, int n_max, int cs,
-                                                            int32_t *slots, int *dev_int) {
-    extern __shared__ __align__(16) unsigned char smem_raw[];
+// A chunk's run starts from the true state when its warm-up would begin
+// within kDpWin tokens of the context start.
+__host__ __device__ __forceinline__ bool dp_exact(int c, int S, int Wu) {
+    return c == 0 || (long long)c * S - Wu < kDpWin;
+}
+
+// Runs the recurrence for the endpoints i_lo + 1 .. i_hi, step at a time.  On
+// entry the ring holds F of the positions i_lo - n_max .. i_lo; on exit the
+// positions i_hi - kDpRing + 1 .. i_hi.  The chosen length of endpoint i is
+// stored to len_out[i] for i > len_from.  With head non-null, the kDpWin
+// ring entries ending at head_at are copied there once endpoint head_at is
+// done (head_at - i_lo a multiple of step).  All threads of the block call it.
+__device__ void dp_run(const float *ew, int N, int n_min, int n_max, int i_lo, int i_hi,
+                       df2 *ring, float *wbuf, uint8_t *len_out, int len_from,
+                       int head_at, df2 *head) {
     const int nb = n_max - n_min + 1, nbp = dp_row(nb);
-    df2 *ring = reinterpret_cast<df2 *>(smem_raw);                                   // [kDpRing]
-    float *wbuf = reinterpret_cast<float *>(ring + kDpRing);                         // [kDpEp][kDpPD][nbp]
-    uint8_t *lenarr = reinterpret_cast<uint8_t *>(wbuf + (size_t)kDpEp * kDpPD * nbp);   // [N + 1]
     const int tid = threadIdx.x, lane = tid & 31, k = tid >> 5;
     const int step = min(n_min, kDpEp);
     const df2 NEG = df2{-INFINITY, 0.f};
-    if (tid == 0) {
-        ring[0] = df2{0.f, 0.f};
-        lenarr[0] = 0;
-    }
     float *mybuf = wbuf + (size_t)k * kDpPD * nbp;
     // row of endpoint i into stage q of this warp's ring (16-byte chunks)
     auto fetch = [&](int i, int q) {
-        const bool ok = k < step && i <= N;
+        const bool ok = k < step && i <= i_hi;
         for (int c4 = lane; c4 < nbp / 4; c4 += 32)
             cp_async16(mybuf + (size_t)q * nbp + 4 * c4, ew + (size_t)(ok ? i : 0) * nbp + 4 * c4, ok);
         cp_async_commit();
     };
 #pragma unroll
-    for (int q = 0; q < kDpPD; q++) fetch(1 + q * step + k, q);
+    for (int q = 0; q < kDpPD; q++) fetch(i_lo + 1 + q * step + k, q);
     __syncthreads();
     int q = 0;
-    for (int i0 = 1; i0 <= N; i0 += step) {
+    for (int i0 = i_lo + 1; i0 <= i_hi; i0 += step) {
         const int i = i0 + k;
-        const bool act = k < step && i <= N;
+        const bool act = k < step && i <= i_hi;
         cp_async_wait<kDpPD - 1>();   // this step's row (the oldest group) has landed
         __syncwarp();
         const float *wr = mybuf + (size_t)q * nbp;
@@ -806,50 +835,200 @@ __global__ void __launch_bounds__(kDpEp * 32) seg_dp_kernel(const float *ew, con
             if (better(ov, oa, best, ba)) { best = ov; ba = oa; }
         }
         if (lane == 0 && act) {
-            ring[i % kDpRing] = best;
-            lenarr[i] = best.hi == -INFINITY ? 0 : (uint8_t)(i - ba);
+            ring[i & (kDpRing - 1)] = best;
+            if (i > len_from) len_out[i] = best.hi == -INFINITY ? 0 : (uint8_t)(i - ba);
         }
         __syncthreads();
+        if (head && i0 + step - 1 == head_at && tid < kDpWin) {
+            const int x = head_at - kDpWin + 1 + tid;
+            head[tid] = x < 0 ? NEG : ring[x & (kDpRing - 1)];
+        }
     }
     cp_async_wait<0>();
-    if (tid == 0 && ring[N % kDpRing].hi == -INFINITY) {
-        // terminal relaxation (Eq. app_terminal_predecessor): 1 <= N - a <= n_max,
-        // read after every F[< N] has been written
-        df2 best = NEG;
-        int ba = 0x7fffffff;
-        for (int len = 1; len <= n_max; len++) {
-            int a = N - len;
-            if (a < 0) break;
-            df2 fa = ring[a % kDpRing];
-            if (fa.hi == -INFINITY || ewt[len].x == -INFINITY) continue;
-            df2 v = df_add(fa, ewt[len]);
-            if (better(v, a, best, ba)) { best = v; ba = a; }
-        }
-        lenarr[N] = best.hi == -INFINITY ? 0 : (uint8_t)(N - ba);
-    }
-    if (tid == 0) {
-        int J = 0, ok = 1;
-        for (int i = N; i > 0;) {
-            int len = lenarr[i];
-            if (len == 0) { ok = 0; break; }
-            i -= len;
-            J++;
-        }
-        if (!ok) {
-            dev_int[0] = -1;
-            return;
-        }
-        dev_int[0] = J;
-        slots[J] = cs + N;
-        int j = J;
-        for (int i = N; i > 0;) {
-            i -= lenarr[i];
-            slots[--j] = cs + i;
-        }
+    __syncthreads();
+}
+
+// The ring, in position order, ending at position e (entries before the
+// context start read as unreachable).
+__device__ __forceinline__ void dp_save_ring(const df2 *ring, int e, df2 *out) {
+    for (int t = threadIdx.x; t < kDpRing; t += blockDim.x) {
+        const int x = e - kDpRing + 1 + t;
+        out[t] = x < 0 ? df2{-INFINITY, 0.f} : ring[x & (kDpRing - 1)];
     }
 }
 
+__global__ void __launch_bounds__(kDpEp * 32) seg_dp_chunk_kernel(const float *ew, int N, int n_min, int n_max,
+                                                                int S, int Wu, uint8_t *len_g, df2 *head,
+                                                                df2 *tail) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    df2 *ring = reinterpret_cast<df2 *>(smem_raw);          // [kDpRing]
+    float *wbuf = reinterpret_cast<float *>(ring + kDpRing); // [kDpEp][kDpPD][nbp]
+    const int c = blockIdx.x;
+    const int e0 = c * S, e1 = min(N, e0 + S);
+    const bool exact = dp_exact(c, S, Wu);
+    const int s0 = exact ? 0 : e0 - Wu;
+    for (int t = threadIdx.x; t < kDpRing; t += blockDim.x)
+        ring[t] = exact ? df2{t == 0 ? 0.f : -INFINITY, 0.f} : df2{0.f, 0.f};
+    __syncthreads();
+    dp_run(ew, N, n_min, n_max, s0, e1, ring, wbuf, len_g, e0, exact ? -1 : e0,
+           exact ? nullptr : head + (size_t)c * kDpWin);
+    dp_save_ring(ring, e1, tail + (size_t)c * kDpRing);
+}
+
+// Difference of two double-float numbers in double-float (two-sum of the
+// high parts, then the low parts added).
+__device__ __forceinline__ df2 df_sub(df2 a, df2 b) {
+    const float s = a.hi - b.hi;
+    const float bb = s - a.hi;
+    float e = (a.hi - (s - bb)) + (-b.hi - bb);
+    e += a.lo - b.lo;
+    const float hi = s + e;
+    return df2{hi, e - (hi - s)};
+}
+
+// Whether the state window `b` (a chunk's head) equals `a` (the previous
+// tail's last kDpWin entries) up to a constant on its last n_max positions,
+// the only ones the endpoints after the boundary read.  The differences are
+// formed in double-float (fp64 is slow on this part).  One warp; the result
+// is returned to every lane.
+__device__ bool dp_match(const df2 *a, const df2 *b, int n_max, int lane) {
+    df2 dmin = df2{INFINITY, 0.f}, dmax = df2{-INFINITY, 0.f};
+    float scale = 0.f;
+    bool bad = false;
+    for (int t = kDpWin - n_max + lane; t < kDpWin; t += 32) {   // the positions later endpoints read
+        const df2 x = a[t], y = b[t];
+        const bool xi = x.hi == -INFINITY, yi = y.hi == -INFINITY;
+        if (xi && yi) continue;
+        const df2 dv = df_sub(x, y);
+        if (xi != yi || !(fabsf(dv.hi) <= FLT_MAX)) { bad = true; continue; }   // also NaN / Inf
+        if (df_gt(dmin, dv)) dmin = dv;
+        if (df_gt(dv, dmax)) dmax = dv;
+        scale = fmaxf(scale, fmaxf(fabsf(x.hi), fabsf(y.hi)));
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        df2 v;
+        v.hi = __shfl_xor_sync(0xffffffffu, dmin.hi, o);
+        v.lo = __shfl_xor_sync(0xffffffffu, dmin.lo, o);
+        if (df_gt(dmin, v)) dmin = v;
+        v.hi = __shfl_xor_sync(0xffffffffu, dmax.hi, o);
+        v.lo = __shfl_xor_sync(0xffffffffu, dmax.lo, o);
+        if (df_gt(v, dmax)) dmax = v;
+        scale = fmaxf(scale, __shfl_xor_sync(0xffffffffu, scale, o));
+    }
+    if (__any_sync(0xffffffffu, bad)) return false;
+    if (dmax.hi == -INFINITY) return true;   // nothing reachable on either side
+    return df_sub(dmax, dmin).hi <= (float)kDpTol * (1.f + scale);
+}
+
+__global__ void __launch_bounds__(kDpEp * 32) seg_dp_finish_kernel(const float *ew, const float2 *ewt, int N,
+                                                                 int n_min, int n_max, int S, int Wu, int nch,
+                                                                 const uint8_t *len_g, const df2 *head,
+                                                                 df2 *tail, int cs, int32_t *rev,
+                                                                 int32_t *slots, int *dev_int) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int nb = n_max - n_min + 1;
+    df2 *ring = reinterpret_cast<df2 *>(smem_raw);
+    float *wbuf = reinterpret_cast<float *>(ring + kDpRing);
+    uint8_t *lenarr = smem_raw + dp_smem_base(nb);                          // [N + 1]
+    uint8_t *ok = lenarr + (((size_t)N + 1 + 15) & ~(size_t)15);            // [nch]
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
+    for (int v = tid; v < (N + 1 + 15) / 16; v += blockDim.x)
+        reinterpret_cast<uint4 *>(lenarr)[v] = reinterpret_cast<const uint4 *>(len_g)[v];
+    for (int c = warp; c < nch; c += nw) {
+        const bool m = dp_exact(c, S, Wu) ||
+                       dp_match(tail + (size_t)(c - 1) * kDpRing + (kDpRing - kDpWin), head + (size_t)c * kDpWin, n_max, lane);
+        if (lane == 0) ok[c] = m;
+    }
+    __syncthreads();
+    // chunks in order: a chunk re-run changes its tail, so the next boundary is checked again
+    int rerun = 0;
+    bool prev = false;
+    for (int c = 1; c < nch; c++) {
+        if (prev) {
+            if (warp == 0) {
+                const bool m = dp_exact(c, S, Wu) ||
+                               dp_match(tail + (size_t)(c - 1) * kDpRing + (kDpRing - kDpWin),
+                                        head + (size_t)c * kDpWin, n_max, lane);
+                if (lane == 0) ok[c] = m;
+            }
+            __syncthreads();
+        }
+        prev = !ok[c];
+        if (!prev) continue;
+        const int e0 = c * S, e1 = min(N, e0 + S);
+        for (int t = tid; t < kDpRing; t += blockDim.x)
+            ring[(e0 - kDpRing + 1 + t) & (kDpRing - 1)] = tail[(size_t)(c - 1) * kDpRing + t];
+        __syncthreads();
+        dp_run(ew, N, n_min, n_max, e0, e1, ring, wbuf, lenarr, e0, -1, nullptr);
+        dp_save_ring(ring, e1, tail + (size_t)c * kDpRing);
+        __threadfence_block();
+        __syncthreads();
+        rerun++;
+    }
+    __shared__ int sJ;
+    if (tid == 0) {
+        dev_int[kDpRerun] = rerun;
+        const df2 *F = tail + (size_t)(nch - 1) * kDpRing;   // F(N - kDpRing + 1 + t) = F[t]
+        if (F[kDpRing - 1].hi == -INFINITY) {
+            // terminal relaxation (Eq. app_terminal_predecessor): 1 <= N - a <= n_max,
+            // read after every F[< N] has been written
+            df2 best = df2{-INFINITY, 0.f};
+            int ba = 0x7fffffff;
+            for (int len = 1; len <= n_max; len++) {
+                int a = N - len;
+                if (a < 0) break;
+                df2 fa = F[kDpRing - 1 - len];
+                if (fa.hi == -INFINITY || ewt[len].x == -INFINITY) continue;
+                df2 v = df_add(fa, ewt[len]);
+                if (better(v, a, best, ba)) { best = v; ba = a; }
+            }
+            lenarr[N] = best.hi == -INFINITY ? 0 : (uint8_t)(N - ba);
+        }
+        // backtracking in one pass: the path's endpoints from N down, into rev
+        int J = 0;
+        for (int i = N; i > 0;) {
+            const int len = lenarr[i];
+            if (len == 0) { J = -1; break; }
+            rev[J++] = i;
+            i -= len;
+        }
+        sJ = J;
+    }
+    __syncthreads();
+    const int J = sJ;
+    if (J < 0) {
+        if (tid == 0) dev_int[0] = -1;
+        return;
+    }
+    for (int j = tid; j <= J; j += blockDim.x) slots[j] = cs + (j == 0 ? 0 : rev[J - j]);
+    if (tid == 0) dev_int[0] = J;
+}
+
 }  // namespace
+
+// Chunks of the segmentation DP: S endpoints per chunk (kDpChunkSteps steps),
+// a warm-up of Wu tokens (p.dp_warmup rounded up to whole steps, default 512;
+// negative: one chunk, the plain sequential recurrence).
+void dp_chunking(const gkv_params &p, int N, int *S, int *Wu, int *nch) {
+    const int step = std::min(p.n_min, kDpEp);
+    if (p.dp_warmup < 0) {
+        *S = std::max(step, (N + step - 1) / step * step);
+        *Wu = step;
+        *nch = 1;
+        return;
+    }
+    const int w = p.dp_warmup == 0 ? 512 : std::min(p.dp_warmup, std::max(N, 1));
+    *S = kDpChunkSteps * step;
+    *Wu = std::max(step, (w + step - 1) / step * step);
+    *nch = std::max(1, (N + *S - 1) / *S);
+}
+
+size_t dp_smem_bytes(const gkv_params &p, int N) {
+    int S, Wu, nch;
+    dp_chunking(p, N, &S, &Wu, &nch);
+    return dp_smem(N, p.n_max - p.n_min + 1, nch);
+}
 
 // ---------------------------------------------------------------------------
 cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
@@ -935,13 +1114,18 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
         seg_band_kernel<<<gb, 256, smb, s>>>(Vf, hidden, b, w.inv_norm, w.nrm2, w.p2, w.bscore, w.ew);
         seg_band_terminal_kernel<<<(p.n_max + 7) / 8, 256, 0, s>>>(Vf, hidden, b, w.inv_norm, w.nrm2, w.p2, w.bscore, w.ewt);
     }
-    const size_t smd = dp_smem(N, nb);
-    if (smd > 227 * 1024 || nb > 32 * kDpLen) return cudaErrorInvalidConfiguration;
-    cudaFuncSetAttribute(seg_dp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smd);
+    int S, Wu, nch;
+    dp_chunking(p, N, &S, &Wu, &nch);
+    const size_t smc = dp_smem_base(nb), smd = dp_smem(N, nb, nch);
+    if (smd > 227 * 1024 - 64 || nb > 32 * kDpLen) return cudaErrorInvalidConfiguration;   // 64: static shared
+    cudaFuncSetAttribute(seg_dp_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smc);
+    cudaFuncSetAttribute(seg_dp_finish_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smd);
     if (c.dp_ev) cudaEventRecord(c.dp_ev, s);   // work that overlaps the DP may start here
-    seg_dp_kernel<<<1, kDpEp * 32, smd, s>>>(w.ew, w.ewt, N, p.n_min, p.n_max, p.ctx_start,
-                                             w.slots, w.dev_int);
-    c.launches += 8 + (surprisal ? 2 : 0) + (N > 1 ? 1 : 0);
+    df2 *head = reinterpret_cast<df2 *>(w.dp_head), *tail = reinterpret_cast<df2 *>(w.dp_tail);
+    seg_dp_chunk_kernel<<<nch, kDpEp * 32, smc, s>>>(w.ew, N, p.n_min, p.n_max, S, Wu, w.dp_len, head, tail);
+    seg_dp_finish_kernel<<<1, kDpEp * 32, smd, s>>>(w.ew, w.ewt, N, p.n_min, p.n_max, S, Wu, nch, w.dp_len,
+                                                    head, tail, p.ctx_start, w.dp_rev, w.slots, w.dev_int);
+    c.launches += 9 + (surprisal ? 2 : 0) + (N > 1 ? 1 : 0);
     return cudaGetLastError();
 }
 

@@ -41,6 +41,7 @@ class GkvParams(C.Structure):
         ("floor_c", C.c_double), ("floor_gamma", C.c_double), ("floor_eta", C.c_double),
         ("floor_half", C.c_int32),
         ("eta_seed", C.c_double), ("rho_hop", C.c_double), ("m_seed", C.c_int32), ("r_hop", C.c_int32),
+        ("dp_warmup", C.c_int32),
     ]
 
 
@@ -320,11 +321,11 @@ class Context:
         """(per-stage ms since the last call, kernels launched so far, tree work counters)."""
         import numpy as np
         ms = np.zeros(len(self.STAGES), np.float32)
-        work = np.zeros(4, np.uint64)
+        work = np.zeros(6, np.uint64)
         n = C.c_int64()
         self._check(lib().gracekv_stats(self.h, C.c_void_p(ms.ctypes.data), len(ms), C.byref(n),
-                                        C.c_void_p(work.ctypes.data), 4))
-        names = ("scan_steps", "cand_evals", "cand_len_sum", "units")
+                                        C.c_void_p(work.ctypes.data), len(work)))
+        names = ("scan_steps", "cand_evals", "cand_len_sum", "units", "dp_chunks", "dp_rerun")
         return dict(zip(self.STAGES, ms.tolist())), n.value, dict(zip(names, map(int, work)))
 
     def gracekv_export(self, node_cap: Optional[int] = None, stream=None) -> dict:
