@@ -196,8 +196,8 @@ gkv_status gracekv_segment(gracekv_ctx *ctx, const void *V, const float *hidden,
  * They read K and Q only, so they can overlap the segmentation: the passes
  * are enqueued on `stream` (which should differ from the segmentation's) --
  * right away when a segmentation has been done and its trees not yet built,
- * otherwise by the next gracekv_segment, after an event recorded where its
- * single-block dynamic program starts.  The next gracekv_build_trees with
+ * otherwise by the next gracekv_segment, after an event recorded on its
+ * stream before its first kernel.  The next gracekv_build_trees with
  * the same K and Q pointers uses these results instead of recomputing them,
  * after making its own stream wait for them; K and Q must not change until
  * then.  Asynchronous.

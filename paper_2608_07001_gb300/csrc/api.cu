@@ -357,6 +357,13 @@ gkv_status gracekv_segment(gracekv_ctx *x, const void *V, const float *hidden, i
     cudaError_t e = cudaSuccess;
     if (c.score_pending && !c.dp_ev) e = cudaEventCreateWithFlags(&c.dp_ev, cudaEventDisableTiming);
     if (e == cudaSuccess) e = cudaMemsetAsync(c.w.dev_int, 0, 16 * sizeof(int), s);
+    if (e == cudaSuccess && c.score_pending) {
+        // requested score passes: they read no output of the segmentation, so
+        // they run beside it, on the SMs its single-block kernels leave idle
+        e = cudaEventRecord(c.dp_ev, s);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(c.score_stream, c.dp_ev, 0);
+        if (e == cudaSuccess) e = launch_score(c, c.score_K, c.score_Q, c.score_stream);
+    }
     if (c.p.seg_mode == 1) {
         // "w/o CS" ablation: uniform slots of target length n0, curvature 0
         const int N = c.Nc, J = std::max(1, (N + c.p.n0 / 2) / c.p.n0);
@@ -369,15 +376,10 @@ gkv_status gracekv_segment(gracekv_ctx *x, const void *V, const float *hidden, i
             if (e == cudaSuccess && kappa) e = cudaMemsetAsync(kappa, 0, (size_t)c.p.T * sizeof(float), s);
             if (e == cudaSuccess) e = cudaMemcpyAsync(c.w.dev_int, &J, sizeof(int), cudaMemcpyHostToDevice, s);
             if (e == cudaSuccess) e = cudaStreamSynchronize(s);   // hs and J leave scope
-            if (e == cudaSuccess && c.dp_ev) e = cudaEventRecord(c.dp_ev, s);
         }
     } else if (e == cudaSuccess) {
         gkv::StageTimer tm(c, 0, s);
         e = gkv::launch_segment(c, V, hidden, hidden ? Dh : 0, surprisal, kappa, s);
-    }
-    if (e == cudaSuccess && c.score_pending) {   // requested score passes overlap the DP
-        e = cudaStreamWaitEvent(c.score_stream, c.dp_ev, 0);
-        if (e == cudaSuccess) e = launch_score(c, c.score_K, c.score_Q, c.score_stream);
     }
     if (e != cudaSuccess) return cuda_fail(x, e, "segment launch");
     int h[gkv::kDpRerun + 1];
@@ -433,7 +435,7 @@ gkv_status gracekv_score(gracekv_ctx *x, const void *K, const void *Q, void *str
     c.score_K = K;
     c.score_Q = Q;
     c.score_stream = s;
-    if (c.stage != 1) {   // the next segmentation enqueues them when its DP starts
+    if (c.stage != 1) {   // the next segmentation enqueues them when it starts
         c.score_pending = true;
         return GKV_OK;
     }

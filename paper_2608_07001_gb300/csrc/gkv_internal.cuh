@@ -151,7 +151,7 @@ struct Ctx {
     const void *score_K = nullptr, *score_Q = nullptr;
     cudaStream_t score_stream = nullptr;
     cudaEvent_t score_ev = nullptr;
-    cudaEvent_t dp_ev = nullptr;   // recorded on the segmentation stream before the DP
+    cudaEvent_t dp_ev = nullptr;   // recorded on the segmentation stream where it starts
     // host pipeline (gracekv_compress_host): device copies of the inputs, the
     // cache before its copy to the host, a copy stream and its events
     void *hK = nullptr, *hV = nullptr, *hQ = nullptr;

@@ -268,8 +268,9 @@ __device__ __forceinline__ double dkey_inv(unsigned long long k) {
 // Select the element of ascending rank `rank` of the keys key(i), i < n, by
 // radix select over 11-bit digits (6 passes).  Histogram updates are
 // aggregated per warp (one shared atomic per distinct bin), since the keys of
-// a pass crowd into few bins; the digit is found by a block-wide scan.
-constexpr int kSelBits = 11, kSelBins = 1 << kSelBits;
+// a pass crowd into few bins; the digit is found by a block-wide scan.  Each
+// thread issues the loads of kSelU keys before using any.
+constexpr int kSelBits = 11, kSelBins = 1 << kSelBits, kSelU = 8;
 
 template <typename KeyF>
 __device__ unsigned long long block_select(int n, int rank, KeyF key, unsigned int *hist,
@@ -283,15 +284,21 @@ __device__ unsigned long long block_select(int n, int rank, KeyF key, unsigned i
         const unsigned int nbin = 1u << bits;
         for (int b = tid; b < kSelBins; b += blockDim.x) hist[b] = 0;
         __syncthreads();
-        for (int i0 = warp * 32; i0 < n; i0 += blockDim.x) {   // whole warps step together
-            const int i = i0 + lane;
-            int bin = -1;
-            if (i < n) {
-                const unsigned long long k = key(i);
-                if ((k & mask) == prefix) bin = (int)((k >> shift) & (nbin - 1));
+        for (int i0 = warp * 32 * kSelU; i0 < n; i0 += blockDim.x * kSelU) {   // whole warps step together
+            unsigned long long kk[kSelU];
+#pragma unroll
+            for (int u = 0; u < kSelU; u++) {
+                const int i = i0 + 32 * u + lane;
+                kk[u] = i < n ? key(i) : 0ull;
             }
-            const unsigned grp = __match_any_sync(0xffffffffu, bin);
-            if (bin >= 0 && lane == __ffs(grp) - 1) atomicAdd(&hist[bin], (unsigned)__popc(grp));
+#pragma unroll
+            for (int u = 0; u < kSelU; u++) {
+                const int i = i0 + 32 * u + lane;
+                int bin = -1;
+                if (i < n && (kk[u] & mask) == prefix) bin = (int)((kk[u] >> shift) & (nbin - 1));
+                const unsigned grp = __match_any_sync(0xffffffffu, bin);
+                if (bin >= 0 && lane == __ffs(grp) - 1) atomicAdd(&hist[bin], (unsigned)__popc(grp));
+            }
         }
         __syncthreads();
         // inclusive scan of the bins in ascending order: thread t owns bins 2t, 2t + 1
@@ -345,13 +352,38 @@ __global__ void __launch_bounds__(1024) seg_robust_z_kernel(const double *x, int
     __shared__ int sr;
     const int rank = (n - 1) / 2;
     const double med = dkey_inv(block_select(n, rank, [&](int i) { return dkey(x[i]); }, hist, &sp, &sr, wsum));
-    for (int i = threadIdx.x; i < n; i += blockDim.x) dev[i] = dkey(fabs(x[i] - med));
+    for (int i0 = threadIdx.x; i0 < n; i0 += blockDim.x * kSelU) {
+        double xv[kSelU];
+#pragma unroll
+        for (int u = 0; u < kSelU; u++) {
+            const int i = i0 + u * blockDim.x;
+            xv[u] = i < n ? x[i] : 0.0;
+        }
+#pragma unroll
+        for (int u = 0; u < kSelU; u++) {
+            const int i = i0 + u * blockDim.x;
+            if (i < n) dev[i] = dkey(fabs(xv[u] - med));
+        }
+    }
     __syncthreads();
     const double mad = dkey_inv(block_select(n, rank, [&](int i) { return dev[i]; }, hist, &sp, &sr, wsum));
-    const double den = 1.4826 * mad + kEps;
-    for (int i = threadIdx.x; i < n; i += blockDim.x) {
-        double z = scale * ((x[i] - med) / den);
-        out[i] = accumulate ? out[i] + z : z;
+    // one fp64 division, then products: fp64 division is slow on this part, and
+    // the product differs from the quotient by at most one rounding
+    const double inv_den = 1.0 / (1.4826 * mad + kEps);
+    for (int i0 = threadIdx.x; i0 < n; i0 += blockDim.x * kSelU) {
+        double xv[kSelU], ov[kSelU];
+#pragma unroll
+        for (int u = 0; u < kSelU; u++) {
+            const int i = i0 + u * blockDim.x;
+            xv[u] = i < n ? x[i] : 0.0;
+            ov[u] = i < n && accumulate ? out[i] : 0.0;
+        }
+#pragma unroll
+        for (int u = 0; u < kSelU; u++) {
+            const int i = i0 + u * blockDim.x;
+            const double z = scale * ((xv[u] - med) * inv_den);
+            if (i < n) out[i] = accumulate ? ov[u] + z : z;
+        }
     }
 }
 
@@ -391,33 +423,80 @@ __global__ void seg_dd_kernel(const Tin *V, const float *hidden, SegArgs a, cons
     if (lane == 0) dd[t] = s;
 }
 
-// Exclusive prefix sum of n doubles (single block, deterministic): out[0] = 0,
-// out[t] = sum_{s<t} in[s], t <= n.
-__global__ void __launch_bounds__(1024) seg_scan_kernel(const double *in, int n, double *out) {
-    __shared__ double part[1024];
-    int tid = threadIdx.x;
-    int per = (n + 1023) / 1024;
-    int b = tid * per, e = min(n, b + per);
-    double s = 0.0;
-    for (int i = b; i < e; i++) s += in[i];
-    part[tid] = s;
+// Exclusive prefix sum of n doubles, deterministic: out[0] = 0,
+// out[t] = sum_{s<t} in[s], t <= n.  Block b owns elements [b C, (b + 1) C),
+// C = kScanC; the first kernel reduces each block's elements, the second
+// adds the totals of the blocks before it (in order, by one warp) to the
+// block's own scan.  Sums of one block follow a fixed tree (thread-local
+// runs of kScanPer elements, then warp and block scans).
+constexpr int kScanT = 256, kScanPer = 8, kScanC = kScanT * kScanPer;
+
+__device__ double block_scan_excl(double v, double *wtot, double *total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    double incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const double y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) wtot[warp] = incl;
     __syncthreads();
-    if (tid == 0) {
-        double acc = 0.0;
-        for (int k = 0; k < 1024; k++) {
-            double v = part[k];
-            part[k] = acc;
-            acc += v;
+    if (warp == 0) {
+        const double wv = lane < kScanT / 32 ? wtot[lane] : 0.0;
+        double wi = wv;
+#pragma unroll
+        for (int o = 1; o < kScanT / 32; o <<= 1) {
+            const double y = __shfl_up_sync(0xffffffffu, wi, o);
+            if (lane >= o) wi += y;
         }
+        if (lane < kScanT / 32) wtot[lane] = wi - wv;
+        if (lane == kScanT / 32 - 1) *total = wi;
     }
     __syncthreads();
-    double acc = part[tid];
-    for (int i = b; i < e; i++) {
-        out[i] = acc;
-        acc += in[i];
+    return wtot[warp] + (incl - v);
+}
+
+__device__ __forceinline__ double scan_run(const double *in, int n, int base, double r[kScanPer]) {
+    double s = 0.0;
+#pragma unroll
+    for (int j = 0; j < kScanPer; j++) {
+        const int i = base + j;
+        r[j] = i < n ? in[i] : 0.0;
     }
-    if (e == n && b < e) out[n] = acc;
-    if (n == 0 && tid == 0) out[0] = 0.0;
+#pragma unroll
+    for (int j = 0; j < kScanPer; j++) s += r[j];
+    return s;
+}
+
+__global__ void __launch_bounds__(kScanT) seg_scan_part_kernel(const double *in, int n, double *btot) {
+    __shared__ double wtot[kScanT / 32];
+    __shared__ double total;
+    double r[kScanPer];
+    const double s = scan_run(in, n, blockIdx.x * kScanC + threadIdx.x * kScanPer, r);
+    block_scan_excl(s, wtot, &total);
+    if (threadIdx.x == 0) btot[blockIdx.x] = total;
+}
+
+__global__ void __launch_bounds__(kScanT) seg_scan_kernel(const double *in, int n, const double *btot, double *out) {
+    __shared__ double wtot[kScanT / 32];
+    __shared__ double total, off;
+    if (threadIdx.x < 32) {   // the totals of the blocks before this one, in order
+        double o = 0.0;
+        if (threadIdx.x == 0)
+            for (int q = 0; q < (int)blockIdx.x; q++) o += btot[q];
+        if (threadIdx.x == 0) off = o;
+    }
+    double r[kScanPer];
+    const int base = blockIdx.x * kScanC + threadIdx.x * kScanPer;
+    const double s = scan_run(in, n, base, r);
+    double acc = block_scan_excl(s, wtot, &total) + off;
+#pragma unroll
+    for (int j = 0; j < kScanPer; j++) {
+        const int i = base + j;
+        if (i <= n) out[i] = acc;
+        acc += r[j];
+    }
+    if (n == 0 && blockIdx.x == 0 && threadIdx.x == 0) out[0] = 0.0;
 }
 
 // ---------------------------------------------------------------------------
@@ -1090,7 +1169,12 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
         if (bf) seg_dd_kernel<<<nw8, 256, 0, s>>>(Vb, hidden, a, w.inv_norm, w.zbuf);
         else seg_dd_kernel<<<nw8, 256, 0, s>>>(Vf, hidden, a, w.inv_norm, w.zbuf);
     }
-    seg_scan_kernel<<<1, 1024, 0, s>>>(w.zbuf, N > 1 ? N - 1 : 0, w.p2);
+    {
+        const int ns = N > 1 ? N - 1 : 0, nbs = ns / kScanC + 1;   // blocks cover [0, ns]
+        double *btot = reinterpret_cast<double *>(w.zdev);   // free after the robust z (nbs <= T)
+        seg_scan_part_kernel<<<nbs, kScanT, 0, s>>>(w.zbuf, ns, btot);
+        seg_scan_kernel<<<nbs, kScanT, 0, s>>>(w.zbuf, ns, btot, w.p2);
+    }
     // edge weights
     BandArgs b;
     b.s = a;
@@ -1120,12 +1204,11 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
     if (smd > 227 * 1024 - 64 || nb > 32 * kDpLen) return cudaErrorInvalidConfiguration;   // 64: static shared
     cudaFuncSetAttribute(seg_dp_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smc);
     cudaFuncSetAttribute(seg_dp_finish_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smd);
-    if (c.dp_ev) cudaEventRecord(c.dp_ev, s);   // work that overlaps the DP may start here
     df2 *head = reinterpret_cast<df2 *>(w.dp_head), *tail = reinterpret_cast<df2 *>(w.dp_tail);
     seg_dp_chunk_kernel<<<nch, kDpEp * 32, smc, s>>>(w.ew, N, p.n_min, p.n_max, S, Wu, w.dp_len, head, tail);
     seg_dp_finish_kernel<<<1, kDpEp * 32, smd, s>>>(w.ew, w.ewt, N, p.n_min, p.n_max, S, Wu, nch, w.dp_len,
                                                     head, tail, p.ctx_start, w.dp_rev, w.slots, w.dev_int);
-    c.launches += 9 + (surprisal ? 2 : 0) + (N > 1 ? 1 : 0);
+    c.launches += 10 + (surprisal ? 2 : 0) + (N > 1 ? 1 : 0);
     return cudaGetLastError();
 }
 
