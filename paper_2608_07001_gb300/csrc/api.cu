@@ -622,7 +622,7 @@ static cudaError_t build_passes(Ctx &c, const void *K, const void *V, const void
         const float tau_eff = fmaxf(tau, h.cut);
         // everything built so far fits and few units remain: expand them fully at once
         const bool fits = h.all && (long long)c.B_free - (long long)h.total >= (long long)h.pot;
-        const int levels = fits ? 4 * gkv::kMaxUnit : 1;
+        const int levels = fits ? 4 * gkv::kMaxUnit : 2;
         gkv::StageTimer tm(c, 3, s);
         e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 1, 0, levels, tau_eff, w.u_list,
                                    h.count[0], w.u_list + (nu - h.count[1]), h.count[1], s);

@@ -1145,11 +1145,18 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
                     bool chf = false;
                     if (ufl)
                         for (int t = B.ca[q]; t < B.cb[q] && !chf; t++) chf = sm.Ff[t] > -INFINITY;
-                    A.nd_U[gc] = B.cb[q] - B.ca[q] >= 2 ? (chf ? FLT_MAX : fminf(kap, key_bound(om * rq * B.cD[q]))) : 0.f;
+                    const float cbnd = B.cb[q] - B.ca[q] >= 2 ? (chf ? FLT_MAX : fminf(kap, key_bound(om * rq * B.cD[q]))) : 0.f;
+                    A.nd_U[gc] = cbnd;
                     A.nd_kappa[gc] = 0.f; A.nd_sel[gc] = 0;
                     if (B.cb[q] - B.ca[q] >= 2) {
-                        const int pos = atomicAdd(&sm.nlvl[cur ^ 1], 1);
-                        sm.lvl[cur ^ 1][pos] = (short)ci;
+                        if (cbnd >= A.tau) {   // evaluated at the next level of this launch
+                            const int pos = atomicAdd(&sm.nlvl[cur ^ 1], 1);
+                            sm.lvl[cur ^ 1][pos] = (short)ci;
+                        } else {   // its key cannot reach this pass's threshold: it stays pending
+                            ch.nchild = -1;
+                            A.nd_nchild[gc] = -1;
+                            atomicMax(reinterpret_cast<int *>(&sm.pend), __float_as_int(cbnd));
+                        }
                     }
                 }
             }
