@@ -572,8 +572,10 @@ static cudaError_t build_fresh(Ctx &c, const void *K, const void *V, const void 
 // Trees (build.cu).  Every op's key is bounded before it is built: a pending
 // node's split key is at most min(creator key, omega R D).  Each pass derives
 // the threshold tau of the ops built so far (a lower bound of the final one)
-// and expands one level of the pending nodes whose bound reaches it, until
-// none does; nodes left pending can never be selected.  When the budget is
+// and expands the pending nodes whose bound reaches it, up to four levels
+// deep (a child below tau stays pending), until none does; nodes left
+// pending can never be selected.  Four levels per launch save reloading the
+// units that keep expanding; tau is re-derived between launches.  When the budget is
 // smaller than the number of units, the first launch evaluates only the
 // roots' own distortion (their Add ops) and later passes expand the units
 // with the largest bounds first, about 32768 at a time, so that tau rises
@@ -622,7 +624,7 @@ static cudaError_t build_passes(Ctx &c, const void *K, const void *V, const void
         const float tau_eff = fmaxf(tau, h.cut);
         // everything built so far fits and few units remain: expand them fully at once
         const bool fits = h.all && (long long)c.B_free - (long long)h.total >= (long long)h.pot;
-        const int levels = fits ? 4 * gkv::kMaxUnit : 2;
+        const int levels = fits ? 4 * gkv::kMaxUnit : 4;
         gkv::StageTimer tm(c, 3, s);
         e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 1, 0, levels, tau_eff, w.u_list,
                                    h.count[0], w.u_list + (nu - h.count[1]), h.count[1], s);

@@ -32,7 +32,10 @@
 // threshold -- and resumes only the pending nodes whose creator has a key
 // >= tau: a node whose creator's key is below the final threshold never
 // reaches the frontier before the allocation stops, so its own Split is never
-// needed.  Resuming repeats until no pending node qualifies.
+// needed.  Resuming repeats until no pending node qualifies.  Within a launch
+// a child whose bound is below the launch's tau stays pending as well, so a
+// resume launch may build several levels without expanding what its tau
+// already rules out.
 //
 // Layout.  256 threads; thread (p, c) owns the probes p and p + 32 and the
 // elements 4 c + 32 g + j (j < 4) of every d-vector: each value, prototype or
