@@ -251,7 +251,7 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
     gkv::Workspace &w = c.w;
     bool ok = dalloc(x, &w.rope, (size_t)p.T * (p.d / 2)) &&
               dalloc(x, &w.rope_rel, (size_t)(2 * gkv::kMaxSlot - 1) * (p.d / 2)) &&
-              dalloc(x, &w.long_slots, (size_t)Nc + 2) && dalloc(x, &w.long_n, 3) &&
+              dalloc(x, &w.long_slots, (size_t)Nc + 2) && dalloc(x, &w.long_n, 4) &&
               dalloc(x, &w.ent, (size_t)p.budget + (size_t)p.L * p.G * (p.T - Nc)) &&
               dalloc(x, &w.inv_norm, (size_t)c.nseg * p.T) &&
               dalloc(x, &w.nrm2, (size_t)c.nseg * p.T) &&

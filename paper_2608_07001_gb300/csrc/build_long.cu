@@ -89,6 +89,7 @@ struct LongArgs {
     LongRes *res;
     int32_t *u_start, *u_cnt;      // per listed unit: its block of work items
     unsigned int *n_items;         // [3]: work items, small subtrees (<= kShortUnit, <= kMaxUnit tokens)
+    unsigned int *it_next;         // the next work item to take (zero at the level's start)
     int32_t *sub;                  // [2][cap_items] small subtrees' roots (global node indices)
     int64_t cap_items;
     // node records and unit arrays (build.cu's layout)
@@ -373,7 +374,15 @@ __global__ void __launch_bounds__(kLT, 1) long_eval_kernel(LongArgs A) {
     const int c = lane / kLPPW, pp = warp * kLPPW + (lane & (kLPPW - 1));
     const int64_t n_items = min((int64_t)*A.n_items, A.cap_items);
     const float inv_sqrt_d = A.inv_sqrt_d, lamZ = A.lamZ, lamM = A.lamM, epsf = A.eps;
-    for (int64_t it = blockIdx.x; it < n_items; it += gridDim.x) {
+    // work items are taken from a counter, so that CTAs finishing short nodes
+    // take the next ones (the nodes of a level range from 129 to 16384 tokens)
+    __shared__ long long s_it;
+    for (;;) {
+        __syncthreads();   // the previous item's reads of s_it are done
+        if (tid == 0) s_it = (long long)atomicAdd(A.it_next, 1u);
+        __syncthreads();
+        const int64_t it = s_it;
+        if (it >= n_items) break;
         const int64_t gv = A.it_gv[it], uid = A.it_uid[it];
         const int lg = (int)(uid / A.J), l = lg / A.G, g = lg - l * A.G;
         const int a = A.nd_a[gv], b = A.nd_b[gv], n = b - a;
@@ -1093,6 +1102,19 @@ __global__ void long_commit_kernel(LongArgs A) {
     }
 }
 
+// CTAs of long_eval resident per SM (its shared memory set as at launch)
+template <int DH, typename Tin>
+int eval_occupancy() {
+    using S = LongSmem<DH>;
+    if (cudaFuncSetAttribute(long_eval_kernel<DH, Tin>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)sizeof(S)) != cudaSuccess)
+        return 1;
+    int n = 1;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, long_eval_kernel<DH, Tin>, kLT, sizeof(S)) != cudaSuccess)
+        return 1;
+    return n;
+}
+
 template <int DH, typename Tin>
 cudaError_t launch_eval(Ctx &c, const LongArgs &A, unsigned grid, cudaStream_t s) {
     using S = LongSmem<DH>;
@@ -1163,7 +1185,8 @@ cudaError_t launch_long_level(Ctx &c, const void *K, const void *V, const void *
     A.status = w.dev_int + 1;
     A.work = w.work;
     A.sub = w.long_sub;
-    cudaError_t e = cudaMemsetAsync(w.long_n, 0, 3 * sizeof(unsigned int), s);
+    A.it_next = w.long_n + 3;
+    cudaError_t e = cudaMemsetAsync(w.long_n, 0, 4 * sizeof(unsigned int), s);
     if (e != cudaSuccess) return e;
     long_collect_kernel<<<(unsigned)n_units, kLT, 0, s>>>(A);
     c.launches += 1;
@@ -1177,7 +1200,11 @@ cudaError_t launch_long_level(Ctx &c, const void *K, const void *V, const void *
     for (int q = 0; q < 3; q++) cnt[q] = (unsigned)std::min<int64_t>((int64_t)cnt[q], w.long_cap);
     if (n_items_host) *n_items_host = cnt[0] + cnt[1] + cnt[2];
     if (cnt[0] > 0) {
-        const unsigned grid = (unsigned)std::min<int64_t>((int64_t)c.num_sms * 2, (int64_t)cnt[0]);
+        // one resident wave: items are taken dynamically
+        int occ = 1;
+        if (p.d == 128) occ = p.dtype == GKV_BF16 ? eval_occupancy<128, __nv_bfloat16>() : eval_occupancy<128, float>();
+        else occ = p.dtype == GKV_BF16 ? eval_occupancy<64, __nv_bfloat16>() : eval_occupancy<64, float>();
+        const unsigned grid = (unsigned)std::min<int64_t>((int64_t)c.num_sms * std::max(occ, 1), (int64_t)cnt[0]);
         e = p.dtype == GKV_BF16
                 ? (p.d == 128 ? launch_eval<128, __nv_bfloat16>(c, A, grid, s) : launch_eval<64, __nv_bfloat16>(c, A, grid, s))
                 : (p.d == 128 ? launch_eval<128, float>(c, A, grid, s) : launch_eval<64, float>(c, A, grid, s));

@@ -114,7 +114,7 @@ struct Workspace {
     uint8_t *long_ufl = nullptr;
     void *long_res = nullptr;      // [long_cap] results (long_res_bytes() each)
     int32_t *long_start = nullptr, *long_cnt = nullptr;   // [long_units_cap]
-    unsigned int *long_n = nullptr;                       // [3] the level's work items, small subtrees
+    unsigned int *long_n = nullptr;                       // [4] the level's work items, small subtrees, next item
                                                           //     of <= kShortUnit and <= kMaxUnit tokens
     int32_t *long_sub = nullptr;    // [2][long_cap] the small subtrees' root nodes (global indices)
     int32_t *long_slots = nullptr;  // [N_c + 1] slot indices of the long slots
