@@ -203,7 +203,7 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
     int64_t Nc = (int64_t)p.ctx_end - r - p.ctx_start;
     if (Nc < 1) return GKV_EBUDGET;
     if (gkv::dp_smem_bytes(p, (int)std::min<int64_t>(Nc, 1 << 30)) > 227 * 1024 - 64)
-        return GKV_EUNSUPPORTED;   // the DP's backtracking keeps every endpoint's length in shared memory
+        return GKV_EUNSUPPORTED;   // the DP's finish kernel keeps one exit table per chunk in shared memory
     if (p.lambda_graph > 0.0 && Nc > gkv::multihop_max_context()) return GKV_EUNSUPPORTED;
 
     gracekv_ctx *x = new (std::nothrow) gracekv_ctx();
@@ -257,11 +257,12 @@ gkv_status gracekv_create(const gkv_params *pin, gracekv_ctx **out) {
               dalloc(x, &w.nrm2, (size_t)c.nseg * p.T) &&
               dalloc(x, &w.klw, (size_t)c.nseg * c.nwin * p.T) &&
               dalloc(x, &w.kappa, (size_t)p.T) && dalloc(x, &w.bscore, (size_t)p.T) &&
-              dalloc(x, &w.zbuf, (size_t)p.T) && dalloc(x, &w.zdev, (size_t)p.T) && dalloc(x, &w.p2, (size_t)Nc + 1) &&
+              dalloc(x, &w.zbuf, (size_t)p.T) && dalloc(x, &w.zdev, (size_t)p.T) &&
+              dalloc(x, &w.sel_state, 4) && dalloc(x, &w.sel_hist, 2048) && dalloc(x, &w.p2, (size_t)Nc + 1) &&
               dalloc(x, &w.ew, (size_t)(Nc + 1) * ((nb + 3) & ~3)) && dalloc(x, &w.ewt, (size_t)p.n_max + 1) &&
               dalloc(x, &w.slots, (size_t)Nc + 2) && dalloc(x, &w.dp_len, (size_t)Nc + 16) &&
               dalloc(x, &w.dp_head, (size_t)dp_nch * 128) && dalloc(x, &w.dp_tail, (size_t)dp_nch * 256) &&
-              dalloc(x, &w.dp_rev, (size_t)Nc + 1) &&
+              dalloc(x, &w.dp_tab, (size_t)dp_nch * p.n_max) &&
               dalloc(x, &w.dev_int, 16) &&
               dalloc(x, &w.row_m, (size_t)nrow) && dalloc(x, &w.row_Z, (size_t)nrow) &&
               dalloc(x, &w.row_ZC, (size_t)nrow) && dalloc(x, &w.rowp, (size_t)3 * nrow * c.n_chunks) &&

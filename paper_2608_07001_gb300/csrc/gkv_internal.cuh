@@ -45,9 +45,10 @@ struct Workspace {
     uint8_t *dp_len = nullptr;     // [N_c + 16] DP: chosen slot length of every endpoint
     float2 *dp_head = nullptr;     // [chunks][128] DP state (double-float) on the window ending at a chunk's start
     float2 *dp_tail = nullptr;     // [chunks][256] DP state on the window ending at a chunk's end
-    int32_t *dp_rev = nullptr;     // [N_c + 1] DP: the path's endpoints from N down (backtracking)
+    uint8_t *dp_tab = nullptr;     // [chunks][n_max] DP: where the path leaves a chunk, per entry point
     int32_t *dev_int = nullptr;    // [16] small device scalars (J, status, counts, ...)
-    unsigned long long *sel_state = nullptr;   // radix-select state for the median
+    unsigned long long *sel_state = nullptr;   // [4] radix-select state of the robust z
+    unsigned int *sel_hist = nullptr;          // [2048] its global digit histogram
     // row statistics and token values
     float *row_m = nullptr, *row_Z = nullptr, *row_ZC = nullptr;  // [L*Hq*W]
     float *rowp = nullptr;         // [3][L*Hq*W][n_chunks] pass-A partials
@@ -299,7 +300,7 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
                            const float *surprisal, float *kappa_out, cudaStream_t s);
 // chunks of the segmentation DP over N endpoints: endpoints per chunk, warm-up tokens, count
 void dp_chunking(const gkv_params &p, int N, int *S, int *Wu, int *nch);
-// shared memory of the DP's finish kernel (bytes) for N endpoints
+// shared memory of the DP's finish kernel (bytes) for N endpoints (the larger of its two kernels)
 size_t dp_smem_bytes(const gkv_params &p, int N);
 
 // layers [l0, l1) (l1 < 0: all); a partial range needs use_tc(c)

@@ -265,126 +265,147 @@ __device__ __forceinline__ double dkey_inv(unsigned long long k) {
     return __longlong_as_double((long long)u);
 }
 
-// Select the element of ascending rank `rank` of the keys key(i), i < n, by
-// radix select over 11-bit digits (6 passes).  Histogram updates are
-// aggregated per warp (one shared atomic per distinct bin), since the keys of
-// a pass crowd into few bins; the digit is found by a block-wide scan.  Each
-// thread issues the loads of kSelU keys before using any.
-constexpr int kSelBits = 11, kSelBins = 1 << kSelBits, kSelU = 8;
+// Select the element of ascending rank `rank` of n keys by radix select over
+// 11-bit digits (6 passes).  Each pass: every block counts the keys that
+// match the digits fixed so far into a shared-memory histogram (updates
+// aggregated per warp, one atomic per distinct bin, since the keys of a pass
+// crowd into few bins) and adds it to a global one; one block then scans the
+// global histogram, fixes the digit that holds the rank and clears it.  The
+// keys are dkey(x[i]) (the median) or dev[i] (the MAD).
+constexpr int kSelBits = 11, kSelBins = 1 << kSelBits, kSelU = 8, kSelT = 256;
 
-template <typename KeyF>
-__device__ unsigned long long block_select(int n, int rank, KeyF key, unsigned int *hist,
-                                           unsigned long long *shared_prefix, int *shared_rank,
-                                           unsigned int *wsum) {
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    unsigned long long prefix = 0, mask = 0;
-    int r = rank;
-    for (int top = 64; top > 0; top -= kSelBits) {
-        const int shift = top > kSelBits ? top - kSelBits : 0, bits = top - shift;
-        const unsigned int nbin = 1u << bits;
-        for (int b = tid; b < kSelBins; b += blockDim.x) hist[b] = 0;
-        __syncthreads();
-        for (int i0 = warp * 32 * kSelU; i0 < n; i0 += blockDim.x * kSelU) {   // whole warps step together
-            unsigned long long kk[kSelU];
-#pragma unroll
-            for (int u = 0; u < kSelU; u++) {
-                const int i = i0 + 32 * u + lane;
-                kk[u] = i < n ? key(i) : 0ull;
-            }
-#pragma unroll
-            for (int u = 0; u < kSelU; u++) {
-                const int i = i0 + 32 * u + lane;
-                int bin = -1;
-                if (i < n && (kk[u] & mask) == prefix) bin = (int)((kk[u] >> shift) & (nbin - 1));
-                const unsigned grp = __match_any_sync(0xffffffffu, bin);
-                if (bin >= 0 && lane == __ffs(grp) - 1) atomicAdd(&hist[bin], (unsigned)__popc(grp));
-            }
-        }
-        __syncthreads();
-        // inclusive scan of the bins in ascending order: thread t owns bins 2t, 2t + 1
-        const unsigned int h0 = 2 * tid < (int)nbin ? hist[2 * tid] : 0u;
-        const unsigned int h1 = 2 * tid + 1 < (int)nbin ? hist[2 * tid + 1] : 0u;
-        unsigned int incl = h0 + h1;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const unsigned int y = __shfl_up_sync(0xffffffffu, incl, o);
-            if (lane >= o) incl += y;
-        }
-        if (lane == 31) wsum[warp] = incl;
-        __syncthreads();
-        if (warp == 0) {
-            const unsigned int wv = lane < (int)(blockDim.x >> 5) ? wsum[lane] : 0u;
-            unsigned int wi = wv;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const unsigned int y = __shfl_up_sync(0xffffffffu, wi, o);
-                if (lane >= o) wi += y;
-            }
-            wsum[lane] = wi - wv;
-        }
-        __syncthreads();
-        const unsigned int before = wsum[warp] + incl - (h0 + h1);   // keys in lower bins
-        // the bin holding rank r: before <= r < before + count
-        if ((unsigned)r >= before && (unsigned)r < before + h0) {
-            *shared_prefix = prefix | ((unsigned long long)(2 * tid) << shift);
-            *shared_rank = r - (int)before;
-        } else if ((unsigned)r >= before + h0 && (unsigned)r < before + h0 + h1) {
-            *shared_prefix = prefix | ((unsigned long long)(2 * tid + 1) << shift);
-            *shared_rank = r - (int)(before + h0);
-        }
-        __syncthreads();
-        prefix = *shared_prefix;
-        r = *shared_rank;
-        mask |= (unsigned long long)(nbin - 1) << shift;
-        __syncthreads();
-    }
-    return prefix;
-}
+struct SelState {           // in global memory (4 words)
+    unsigned long long prefix, mask;
+    long long rank;
+    double med;
+};
 
-// out[i] (+)= scale * (x[i] - median) / (1.4826 MAD + eps); the lower median
-// of the absolute deviations is selected over keys written once to `dev`.
-__global__ void __launch_bounds__(1024) seg_robust_z_kernel(const double *x, int n, double scale,
-                                                            int accumulate, double *out,
-                                                            unsigned long long *dev) {
+template <bool kDev>
+__global__ void __launch_bounds__(kSelT) zsel_hist_kernel(const double *x, const unsigned long long *dev, int n,
+                                                         const SelState *st, int shift, int bits,
+                                                         unsigned int *ghist) {
     __shared__ unsigned int hist[kSelBins];
-    __shared__ unsigned int wsum[32];
-    __shared__ unsigned long long sp;
-    __shared__ int sr;
-    const int rank = (n - 1) / 2;
-    const double med = dkey_inv(block_select(n, rank, [&](int i) { return dkey(x[i]); }, hist, &sp, &sr, wsum));
-    for (int i0 = threadIdx.x; i0 < n; i0 += blockDim.x * kSelU) {
-        double xv[kSelU];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const unsigned int nbin = 1u << bits;
+    for (int bq = tid; bq < (int)nbin; bq += kSelT) hist[bq] = 0;
+    const unsigned long long prefix = st->prefix, mask = st->mask;
+    __syncthreads();
+    const int per_warp = 32 * kSelU, stride = gridDim.x * (kSelT / 32) * per_warp;
+    for (int i0 = (blockIdx.x * (kSelT / 32) + warp) * per_warp; i0 < n; i0 += stride) {   // whole warps
+        unsigned long long kk[kSelU];
 #pragma unroll
         for (int u = 0; u < kSelU; u++) {
-            const int i = i0 + u * blockDim.x;
-            xv[u] = i < n ? x[i] : 0.0;
+            const int i = i0 + 32 * u + lane;
+            kk[u] = i < n ? (kDev ? dev[i] : dkey(x[i])) : 0ull;
         }
 #pragma unroll
         for (int u = 0; u < kSelU; u++) {
-            const int i = i0 + u * blockDim.x;
-            if (i < n) dev[i] = dkey(fabs(xv[u] - med));
+            const int i = i0 + 32 * u + lane;
+            int bin = -1;
+            if (i < n && (kk[u] & mask) == prefix) bin = (int)((kk[u] >> shift) & (nbin - 1));
+            const unsigned grp = __match_any_sync(0xffffffffu, bin);
+            if (bin >= 0 && lane == __ffs(grp) - 1) atomicAdd(&hist[bin], (unsigned)__popc(grp));
         }
     }
     __syncthreads();
-    const double mad = dkey_inv(block_select(n, rank, [&](int i) { return dev[i]; }, hist, &sp, &sr, wsum));
-    // one fp64 division, then products: fp64 division is slow on this part, and
-    // the product differs from the quotient by at most one rounding
-    const double inv_den = 1.0 / (1.4826 * mad + kEps);
-    for (int i0 = threadIdx.x; i0 < n; i0 += blockDim.x * kSelU) {
-        double xv[kSelU], ov[kSelU];
+    for (int bq = tid; bq < (int)nbin; bq += kSelT)
+        if (hist[bq]) atomicAdd(&ghist[bq], hist[bq]);
+}
+
+// The digit of this pass: thread t owns bins 2t, 2t + 1 (ascending order).
+__global__ void __launch_bounds__(1024) zsel_pick_kernel(SelState *st, unsigned int *ghist, int shift, int bits) {
+    __shared__ unsigned int wsum[32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const unsigned int nbin = 1u << bits;
+    const long long r = st->rank;
+    const unsigned int h0 = 2 * tid < (int)nbin ? ghist[2 * tid] : 0u;
+    const unsigned int h1 = 2 * tid + 1 < (int)nbin ? ghist[2 * tid + 1] : 0u;
+    unsigned int incl = h0 + h1;
 #pragma unroll
-        for (int u = 0; u < kSelU; u++) {
-            const int i = i0 + u * blockDim.x;
-            xv[u] = i < n ? x[i] : 0.0;
-            ov[u] = i < n && accumulate ? out[i] : 0.0;
+    for (int o = 1; o < 32; o <<= 1) {
+        const unsigned int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        const unsigned int wv = lane < (int)(blockDim.x >> 5) ? wsum[lane] : 0u;
+        unsigned int wi = wv;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const unsigned int y = __shfl_up_sync(0xffffffffu, wi, o);
+            if (lane >= o) wi += y;
         }
-#pragma unroll
-        for (int u = 0; u < kSelU; u++) {
-            const int i = i0 + u * blockDim.x;
-            const double z = scale * ((xv[u] - med) * inv_den);
-            if (i < n) out[i] = accumulate ? ov[u] + z : z;
+        wsum[lane] = wi - wv;
+    }
+    __syncthreads();
+    const long long before = (long long)wsum[warp] + incl - (h0 + h1);   // keys in lower bins
+    if (r >= before && r < before + h0) {
+        st->prefix |= (unsigned long long)(2 * tid) << shift;
+        st->rank = r - before;
+    } else if (r >= before + h0 && r < before + h0 + h1) {
+        st->prefix |= (unsigned long long)(2 * tid + 1) << shift;
+        st->rank = r - (before + h0);
+    }
+    if (tid == 0) st->mask |= (unsigned long long)(nbin - 1) << shift;
+    if (2 * tid < (int)nbin) ghist[2 * tid] = 0;
+    if (2 * tid + 1 < (int)nbin) ghist[2 * tid + 1] = 0;
+}
+
+// A fresh select of rank `rank`; with `keep_med`, the median found by the
+// select before it is kept in st->med.
+__global__ void zsel_init_kernel(SelState *st, unsigned int *ghist, long long rank, int keep_med) {
+    if (threadIdx.x == 0) {
+        if (keep_med) st->med = dkey_inv(st->prefix);
+        st->prefix = 0;
+        st->mask = 0;
+        st->rank = rank;
+    }
+    for (int bq = threadIdx.x; bq < kSelBins; bq += blockDim.x) ghist[bq] = 0;
+}
+
+__global__ void zsel_dev_kernel(const double *x, int n, const SelState *st, unsigned long long *dev) {
+    const double med = st->med;
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
+        dev[i] = dkey(fabs(x[i] - med));
+}
+
+// out[i] (+)= scale * (x[i] - median) / (1.4826 MAD + eps), with one fp64
+// division (fp64 division is slow on this part; the product differs from the
+// quotient by at most one rounding).
+__global__ void zsel_z_kernel(const double *x, int n, const SelState *st, double scale, int accumulate,
+                              double *out) {
+    const double med = st->med, inv_den = 1.0 / (1.4826 * dkey_inv(st->prefix) + kEps);
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
+        const double z = scale * ((x[i] - med) * inv_den);
+        out[i] = accumulate ? out[i] + z : z;
+    }
+}
+
+// The robust z of x (Eq. app_robust_z), scaled by `scale`, written to or added
+// to `out`: lower median and lower median of the absolute deviations.
+void robust_z(const double *x, int n, double scale, int accumulate, double *out, unsigned long long *dev,
+              SelState *st, unsigned int *ghist, int n_sms, int64_t *launches, cudaStream_t s) {
+    const long long rank = (n - 1) / 2;
+    const int hb = (int)std::max<long long>(1, std::min<long long>(2LL * n_sms, ((long long)n + kSelT * kSelU - 1) / (kSelT * kSelU)));
+    const int eb = (int)std::max<long long>(1, std::min<long long>(4LL * n_sms, ((long long)n + 255) / 256));
+    zsel_init_kernel<<<1, 256, 0, s>>>(st, ghist, rank, 0);
+    for (int pass = 0; pass < 2; pass++) {
+        for (int top = 64; top > 0; top -= kSelBits) {
+            const int shift = top > kSelBits ? top - kSelBits : 0, bits = top - shift;
+            if (pass == 0) zsel_hist_kernel<false><<<hb, kSelT, 0, s>>>(x, dev, n, st, shift, bits, ghist);
+            else zsel_hist_kernel<true><<<hb, kSelT, 0, s>>>(x, dev, n, st, shift, bits, ghist);
+            zsel_pick_kernel<<<1, 1024, 0, s>>>(st, ghist, shift, bits);
+            *launches += 2;
+        }
+        if (pass == 0) {
+            zsel_init_kernel<<<1, 256, 0, s>>>(st, ghist, rank, 1);
+            zsel_dev_kernel<<<eb, 256, 0, s>>>(x, n, st, dev);
+            *launches += 2;
         }
     }
+    zsel_z_kernel<<<eb, 256, 0, s>>>(x, n, st, scale, accumulate, out);
+    *launches += 2;   // with the first init
 }
 
 __global__ void f32_to_f64_kernel(const float *x, int n, double *y) {
@@ -838,8 +859,15 @@ constexpr double kDpTol = 1e-9;   // boundary check: relative spread of tail - h
 __host__ __device__ constexpr size_t dp_smem_base(int nb) {
     return (size_t)kDpRing * 8 + (size_t)kDpEp * kDpPD * dp_row(nb) * 4;
 }
-__host__ __device__ constexpr size_t dp_smem(int N, int nb, int nch) {
-    return dp_smem_base(nb) + (((size_t)N + 1 + 15) & ~(size_t)15) + (size_t)nch;
+// chunk kernel: the base plus the chunk's chosen lengths [S + 1]
+__host__ __device__ constexpr size_t dp_smem_chunk(int nb, int S) {
+    return dp_smem_base(nb) + (((size_t)S + 1 + 15) & ~(size_t)15);
+}
+// finish kernel: the base, the boundary flags [nch] and the exit table
+// [nch][n_max] (uint8), the chunks' entries and counts [nch] (int32)
+__host__ __device__ constexpr size_t dp_smem(int nb, int nch, int n_max) {
+    return dp_smem_base(nb) + (((size_t)nch + 15) & ~(size_t)15) + (((size_t)nch * n_max + 15) & ~(size_t)15) +
+           (size_t)nch * 8;
 }
 
 __device__ __forceinline__ bool better(df2 v, int a, df2 bv, int ba) {
@@ -855,7 +883,7 @@ __host__ __device__ __forceinline__ bool dp_exact(int c, int S, int Wu) {
 // Runs the recurrence for the endpoints i_lo + 1 .. i_hi, step at a time.  On
 // entry the ring holds F of the positions i_lo - n_max .. i_lo; on exit the
 // positions i_hi - kDpRing + 1 .. i_hi.  The chosen length of endpoint i is
-// stored to len_out[i] for i > len_from.  With head non-null, the kDpWin
+// stored to len_out[i - len_from] for i > len_from.  With head non-null, the kDpWin
 // ring entries ending at head_at are copied there once endpoint head_at is
 // done (head_at - i_lo a multiple of step).  All threads of the block call it.
 __device__ void dp_run(const float *ew, int N, int n_min, int n_max, int i_lo, int i_hi,
@@ -915,7 +943,7 @@ __device__ void dp_run(const float *ew, int N, int n_min, int n_max, int i_lo, i
         }
         if (lane == 0 && act) {
             ring[i & (kDpRing - 1)] = best;
-            if (i > len_from) len_out[i] = best.hi == -INFINITY ? 0 : (uint8_t)(i - ba);
+            if (i > len_from) len_out[i - len_from] = best.hi == -INFINITY ? 0 : (uint8_t)(i - ba);
         }
         __syncthreads();
         if (head && i0 + step - 1 == head_at && tid < kDpWin) {
@@ -936,12 +964,29 @@ __device__ __forceinline__ void dp_save_ring(const df2 *ring, int e, df2 *out) {
     }
 }
 
+// Exit table of chunk c (endpoints (e0, e1]): for q < n_max, following the
+// chosen lengths from z = e1 - q down, the first position <= e0 is
+// e0 - tab[q] (z itself when z <= e0); 255 when the walk meets an
+// unreachable endpoint or z < 0.  len(i) is the chosen length of i in (e0, e1].
+template <typename LenF>
+__device__ __forceinline__ uint8_t dp_exit(int e0, int e1, int q, LenF len) {
+    int z = e1 - q;
+    if (z < 0) return 255;
+    while (z > e0) {
+        const int l = len(z);
+        if (l == 0) return 255;
+        z -= l;
+    }
+    return (uint8_t)(e0 - z);   // < n_max: the last step into (e0 - n_max, e0], or z = 0 with e0 < n_max
+}
+
 __global__ void __launch_bounds__(kDpEp * 32) seg_dp_chunk_kernel(const float *ew, int N, int n_min, int n_max,
                                                                 int S, int Wu, uint8_t *len_g, df2 *head,
-                                                                df2 *tail) {
+                                                                df2 *tail, uint8_t *tab_g) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     df2 *ring = reinterpret_cast<df2 *>(smem_raw);          // [kDpRing]
     float *wbuf = reinterpret_cast<float *>(ring + kDpRing); // [kDpEp][kDpPD][nbp]
+    uint8_t *lloc = smem_raw + dp_smem_base(n_max - n_min + 1);   // [S + 1] lengths of (e0, e1]
     const int c = blockIdx.x;
     const int e0 = c * S, e1 = min(N, e0 + S);
     const bool exact = dp_exact(c, S, Wu);
@@ -949,9 +994,12 @@ __global__ void __launch_bounds__(kDpEp * 32) seg_dp_chunk_kernel(const float *e
     for (int t = threadIdx.x; t < kDpRing; t += blockDim.x)
         ring[t] = exact ? df2{t == 0 ? 0.f : -INFINITY, 0.f} : df2{0.f, 0.f};
     __syncthreads();
-    dp_run(ew, N, n_min, n_max, s0, e1, ring, wbuf, len_g, e0, exact ? -1 : e0,
+    dp_run(ew, N, n_min, n_max, s0, e1, ring, wbuf, lloc, e0, exact ? -1 : e0,
            exact ? nullptr : head + (size_t)c * kDpWin);
     dp_save_ring(ring, e1, tail + (size_t)c * kDpRing);
+    for (int i = e0 + 1 + threadIdx.x; i <= e1; i += blockDim.x) len_g[i] = lloc[i - e0];
+    for (int q = threadIdx.x; q < n_max; q += blockDim.x)
+        tab_g[(size_t)c * n_max + q] = dp_exit(e0, e1, q, [&](int z) { return (int)lloc[z - e0]; });
 }
 
 // Difference of two double-float numbers in double-float (two-sum of the
@@ -1002,18 +1050,19 @@ __device__ bool dp_match(const df2 *a, const df2 *b, int n_max, int lane) {
 
 __global__ void __launch_bounds__(kDpEp * 32) seg_dp_finish_kernel(const float *ew, const float2 *ewt, int N,
                                                                  int n_min, int n_max, int S, int Wu, int nch,
-                                                                 const uint8_t *len_g, const df2 *head,
-                                                                 df2 *tail, int cs, int32_t *rev,
-                                                                 int32_t *slots, int *dev_int) {
+                                                                 uint8_t *len_g, const df2 *head, df2 *tail,
+                                                                 const uint8_t *tab_g, int cs, int32_t *slots,
+                                                                 int *dev_int) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int nb = n_max - n_min + 1;
     df2 *ring = reinterpret_cast<df2 *>(smem_raw);
     float *wbuf = reinterpret_cast<float *>(ring + kDpRing);
-    uint8_t *lenarr = smem_raw + dp_smem_base(nb);                          // [N + 1]
-    uint8_t *ok = lenarr + (((size_t)N + 1 + 15) & ~(size_t)15);            // [nch]
+    uint8_t *ok = smem_raw + dp_smem_base(nb);                                  // [nch]
+    uint8_t *tab = ok + (((size_t)nch + 15) & ~(size_t)15);                      // [nch][n_max]
+    int *ent = reinterpret_cast<int *>(tab + (((size_t)nch * n_max + 15) & ~(size_t)15));   // [nch]
+    int *cnt = ent + nch;                                                       // [nch]
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
-    for (int v = tid; v < (N + 1 + 15) / 16; v += blockDim.x)
-        reinterpret_cast<uint4 *>(lenarr)[v] = reinterpret_cast<const uint4 *>(len_g)[v];
+    for (int q = tid; q < nch * n_max; q += blockDim.x) tab[q] = tab_g[q];
     for (int c = warp; c < nch; c += nw) {
         const bool m = dp_exact(c, S, Wu) ||
                        dp_match(tail + (size_t)(c - 1) * kDpRing + (kDpRing - kDpWin), head + (size_t)c * kDpWin, n_max, lane);
@@ -1039,9 +1088,12 @@ __global__ void __launch_bounds__(kDpEp * 32) seg_dp_finish_kernel(const float *
         for (int t = tid; t < kDpRing; t += blockDim.x)
             ring[(e0 - kDpRing + 1 + t) & (kDpRing - 1)] = tail[(size_t)(c - 1) * kDpRing + t];
         __syncthreads();
-        dp_run(ew, N, n_min, n_max, e0, e1, ring, wbuf, lenarr, e0, -1, nullptr);
+        dp_run(ew, N, n_min, n_max, e0, e1, ring, wbuf, len_g + e0, e0, -1, nullptr);
         dp_save_ring(ring, e1, tail + (size_t)c * kDpRing);
         __threadfence_block();
+        __syncthreads();
+        for (int q = tid; q < n_max; q += blockDim.x)   // the chunk's exit table, from its new lengths
+            tab[(size_t)c * n_max + q] = dp_exit(e0, e1, q, [&](int z) { return (int)len_g[z]; });
         __syncthreads();
         rerun++;
     }
@@ -1062,26 +1114,66 @@ __global__ void __launch_bounds__(kDpEp * 32) seg_dp_finish_kernel(const float *
                 df2 v = df_add(fa, ewt[len]);
                 if (better(v, a, best, ba)) { best = v; ba = a; }
             }
-            lenarr[N] = best.hi == -INFINITY ? 0 : (uint8_t)(N - ba);
+            len_g[N] = best.hi == -INFINITY ? 0 : (uint8_t)(N - ba);
         }
-        // backtracking in one pass: the path's endpoints from N down, into rev
-        int J = 0;
-        for (int i = N; i > 0;) {
-            const int len = lenarr[i];
-            if (len == 0) { J = -1; break; }
-            rev[J++] = i;
-            i -= len;
+        // the path's first endpoint in each chunk, from the top: the last chunk
+        // is walked from N itself (its relaxed length), the others by their tables
+        int z = N, bad = 0;
+        for (int c = nch - 1; c >= 0; c--) {
+            ent[c] = z;
+            if (z == 0) continue;
+            const int e0 = c * S, e1 = min(N, e0 + S), q = e1 - z;
+            if (q < 0 || q >= n_max) { bad = 1; break; }
+            const uint8_t o = c == nch - 1 ? dp_exit(e0, e1, 0, [&](int y) { return (int)len_g[y]; })
+                                           : tab[(size_t)c * n_max + q];
+            if (o == 255) { bad = 1; break; }
+            z = e0 - o;
         }
-        sJ = J;
+        sJ = bad ? -1 : 0;
     }
     __syncthreads();
-    const int J = sJ;
-    if (J < 0) {
+    if (sJ < 0) {
         if (tid == 0) dev_int[0] = -1;
         return;
     }
-    for (int j = tid; j <= J; j += blockDim.x) slots[j] = cs + (j == 0 ? 0 : rev[J - j]);
-    if (tid == 0) dev_int[0] = J;
+    // endpoints of the path inside each chunk, then their offsets from the top
+    for (int c = tid; c < nch; c += blockDim.x) {
+        const int e0 = c * S;
+        int k = 0;
+        for (int z = ent[c]; z > e0 && z > 0;) {   // every length on it is >= 1 (checked above)
+            const int l = len_g[z];
+            if (l == 0) break;
+            k++;
+            z -= l;
+        }
+        cnt[c] = k;
+    }
+    __syncthreads();
+    if (tid == 0) {   // exclusive offsets from the top chunk down; J = all of them
+        int acc = 0;
+        for (int c = nch - 1; c >= 0; c--) {
+            const int k = cnt[c];
+            cnt[c] = acc;
+            acc += k;
+        }
+        sJ = acc;
+    }
+    __syncthreads();
+    const int J = sJ;
+    for (int c = tid; c < nch; c += blockDim.x) {   // the m-th endpoint from the top is slot start J - m
+        const int e0 = c * S;
+        int m = cnt[c];
+        for (int z = ent[c]; z > e0 && z > 0;) {
+            const int l = len_g[z];
+            if (l == 0) break;
+            slots[J - m++] = cs + z;
+            z -= l;
+        }
+    }
+    if (tid == 0) {
+        slots[0] = cs;
+        dev_int[0] = J;
+    }
 }
 
 }  // namespace
@@ -1106,7 +1198,8 @@ void dp_chunking(const gkv_params &p, int N, int *S, int *Wu, int *nch) {
 size_t dp_smem_bytes(const gkv_params &p, int N) {
     int S, Wu, nch;
     dp_chunking(p, N, &S, &Wu, &nch);
-    return dp_smem(N, p.n_max - p.n_min + 1, nch);
+    const int nb = p.n_max - p.n_min + 1;
+    return std::max(dp_smem_chunk(nb, S), dp_smem(nb, nch, p.n_max));
 }
 
 // ---------------------------------------------------------------------------
@@ -1157,10 +1250,11 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
     seg_combine_kernel<<<(p.T + 255) / 256, 256, 0, s>>>(w.klw, c.nseg * c.nwin, p.T, p.lambda_stab,
                                                           w.kappa, kappa_out, w.dev_int + 1);
     // boundary score b = z(kappa) + lambda_s z(surprisal)
-    seg_robust_z_kernel<<<1, 1024, 0, s>>>(w.kappa, p.T, 1.0, 0, w.bscore, w.zdev);
+    SelState *st = reinterpret_cast<SelState *>(w.sel_state);
+    robust_z(w.kappa, p.T, 1.0, 0, w.bscore, w.zdev, st, w.sel_hist, c.num_sms, &c.launches, s);
     if (surprisal) {
         f32_to_f64_kernel<<<(p.T + 255) / 256, 256, 0, s>>>(surprisal, p.T, w.zbuf);
-        seg_robust_z_kernel<<<1, 1024, 0, s>>>(w.zbuf, p.T, p.lambda_s, 1, w.bscore, w.zdev);
+        robust_z(w.zbuf, p.T, p.lambda_s, 1, w.bscore, w.zdev, st, w.sel_hist, c.num_sms, &c.launches, s);
     }
     // prefix of sum_l ||d_t||^2 over the compressible region
     int N = c.Nc;
@@ -1200,15 +1294,16 @@ cudaError_t launch_segment(Ctx &c, const void *V, const float *hidden, int Dh,
     }
     int S, Wu, nch;
     dp_chunking(p, N, &S, &Wu, &nch);
-    const size_t smc = dp_smem_base(nb), smd = dp_smem(N, nb, nch);
-    if (smd > 227 * 1024 - 64 || nb > 32 * kDpLen) return cudaErrorInvalidConfiguration;   // 64: static shared
+    const size_t smc = dp_smem_chunk(nb, S), smd = dp_smem(nb, nch, p.n_max);
+    if (std::max(smc, smd) > 227 * 1024 - 64 || nb > 32 * kDpLen) return cudaErrorInvalidConfiguration;   // 64: static shared
     cudaFuncSetAttribute(seg_dp_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smc);
     cudaFuncSetAttribute(seg_dp_finish_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smd);
     df2 *head = reinterpret_cast<df2 *>(w.dp_head), *tail = reinterpret_cast<df2 *>(w.dp_tail);
-    seg_dp_chunk_kernel<<<nch, kDpEp * 32, smc, s>>>(w.ew, N, p.n_min, p.n_max, S, Wu, w.dp_len, head, tail);
+    seg_dp_chunk_kernel<<<nch, kDpEp * 32, smc, s>>>(w.ew, N, p.n_min, p.n_max, S, Wu, w.dp_len, head, tail,
+                                                      w.dp_tab);
     seg_dp_finish_kernel<<<1, kDpEp * 32, smd, s>>>(w.ew, w.ewt, N, p.n_min, p.n_max, S, Wu, nch, w.dp_len,
-                                                    head, tail, p.ctx_start, w.dp_rev, w.slots, w.dev_int);
-    c.launches += 10 + (surprisal ? 2 : 0) + (N > 1 ? 1 : 0);
+                                                    head, tail, w.dp_tab, p.ctx_start, w.slots, w.dev_int);
+    c.launches += 9 + (surprisal ? 1 : 0) + (N > 1 ? 1 : 0);   // and the robust z's own
     return cudaGetLastError();
 }
 
