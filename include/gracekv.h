@@ -154,8 +154,10 @@ int32_t gracekv_graph_layers(int32_t L, int32_t *out);
  * allocate the device workspace on the current device.  On success *out owns
  * it; release with gracekv_destroy.  Errors: GKV_EINVAL, GKV_EBUDGET,
  * GKV_EUNSUPPORTED (d not in {64, 128}, W > 64, n_max above 128, G d above
- * 2048, N_c above 228,351 tokens; lambda_graph > 0 with fp32 inputs or
- * N_c above 131072; alpha_floor > 0 together with quota_alloc), GKV_ENOMEM,
+ * 2048, a compressible region whose segmentation DP does not fit one CTA's
+ * shared memory -- about 630,000 tokens with the default n_min and n_max,
+ * about 170,000 with a negative dp_warmup; lambda_graph > 0 with fp32 inputs
+ * or N_c above 131072; alpha_floor > 0 together with quota_alloc), GKV_ENOMEM,
  * GKV_ECUDA. */
 gkv_status gracekv_create(const gkv_params *p, gracekv_ctx **out);
 void gracekv_destroy(gracekv_ctx *ctx);
