@@ -101,20 +101,22 @@ __global__ void seg_norm_kernel(const Tin *V, const float *hidden, SegArgs a, fl
 }
 
 // ---------------------------------------------------------------------------
-// Curvature.  Block = 256 threads = 256 consecutive positions (one per
-// thread) of one segmentation layer.  The trajectory channels are staged in
-// chunks of kCurvCC channels, already normalised (hbar = h / max(|h|, eps)),
-// channel-major in shared memory so that the threads of a warp read
-// consecutive rows.  Each thread forms its window sums directly (running sums
-// outward from its position, left window [i-w+1, i], right window [i+1, i+w])
-// and accumulates |d-|^2, |d+|^2 and d-.d+ over all channels in registers: no
-// cross-thread reduction.
+// Curvature.  Block = 256 threads = 512 consecutive positions (two adjacent
+// ones per thread) of one segmentation layer.  The trajectory channels are
+// staged in chunks of kCurvCC channels, already normalised (hbar = h /
+// max(|h|, eps)), channel-major in shared memory so that the threads of a
+// warp read consecutive rows.  A thread loads the 34 rows around its two
+// positions with 8-byte loads, forms each position's window sums directly
+// (running sums outward from the position, left window [i-w+1, i], right
+// window [i+1, i+w]) and accumulates |d-|^2, |d+|^2 and d-.d+ over all
+// channels in registers: no cross-thread reduction.
 // ---------------------------------------------------------------------------
 constexpr int kHalo = 16;                       // largest window
-constexpr int kCurvPT = 256;                    // positions per block
+constexpr int kCurvPP = 2;                      // positions per thread
+constexpr int kCurvPT = 256 * kCurvPP;          // positions per block
 constexpr int kCurvRows = kCurvPT + 2 * kHalo;  // staged rows
-constexpr int kCurvRS = kCurvRows + 1;          // row stride (odd: 2-way staging conflicts at most)
-constexpr int kCurvCC = 64;                     // channels per stage
+constexpr int kCurvRS = kCurvRows + 2;          // row stride (even: 8-byte row loads)
+constexpr int kCurvCC = 32;                     // channels per stage
 constexpr size_t kCurvSmem = ((size_t)kCurvCC * kCurvRS + kCurvRows) * sizeof(float);
 
 // 8 consecutive trajectory channels c .. c+7 (c % 8 == 0) of row t, or zeros
@@ -162,74 +164,106 @@ __global__ void __launch_bounds__(256) seg_curv_kernel(const Tin *V, const float
         wv[wi] = kDefaultWindows ? (4 << wi) : a.windows[wi];
         inv_w[wi] = 1.0f / (float)wv[wi];
     }
-    float acc[kMaxWindows][3];
+    float acc[kCurvPP][kMaxWindows][3];
 #pragma unroll
-    for (int wi = 0; wi < kMaxWindows; wi++) acc[wi][0] = acc[wi][1] = acc[wi][2] = 0.f;
-    const int R = tid + kHalo;   // staged row of this thread's position
+    for (int pp = 0; pp < kCurvPP; pp++)
+#pragma unroll
+        for (int wi = 0; wi < kMaxWindows; wi++) acc[pp][wi][0] = acc[pp][wi][1] = acc[pp][wi][2] = 0.f;
+    // this thread's positions sit at staged rows kHalo + 2 tid (+1); it reads
+    // rows 2 tid .. 2 tid + 33 (x[k] = row 2 tid + k)
+    constexpr int NX = kCurvPP + 2 * kHalo;
     for (int c0 = 0; c0 < a.D; c0 += kCurvCC) {
         const int nq = min(kCurvCC, a.D - c0) >> 3;   // 8-channel chunks in this stage
         __syncthreads();
-        for (int e = tid; e < kCurvRows * nq; e += 256) {
-            const int r = e / nq, q = e - r * nq;
-            float v[8];
-            traj_load8(V, hidden, a, l, li, row0 + r, c0 + 8 * q, v);
-            const float sc = inv_s[r];
+        // stage: the loads of 4 row chunks are issued before any is stored
+        for (int e0 = tid; e0 < kCurvRows * nq; e0 += 256 * 4) {
+            float v[4][8];
 #pragma unroll
-            for (int j = 0; j < 8; j++) P[(size_t)(8 * q + j) * kCurvRS + r] = v[j] * sc;
+            for (int u = 0; u < 4; u++) {
+                const int e = e0 + 256 * u;
+                if (e < kCurvRows * nq) {
+                    const int r = e / nq, q = e - r * nq;
+                    traj_load8(V, hidden, a, l, li, row0 + r, c0 + 8 * q, v[u]);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < 4; u++) {
+                const int e = e0 + 256 * u;
+                if (e < kCurvRows * nq) {
+                    const int r = e / nq, q = e - r * nq;
+                    const float sc = inv_s[r];
+#pragma unroll
+                    for (int j = 0; j < 8; j++) P[(size_t)(8 * q + j) * kCurvRS + r] = v[u][j] * sc;
+                }
+            }
         }
         __syncthreads();
         for (int c = 0; c < 8 * nq; c++) {
-            const float *row = P + (size_t)c * kCurvRS + R;
-            const float h = row[0];
-            float sl = h, sr = 0.f;
-            float SL[kMaxWindows], SR[kMaxWindows];
+            const float2 *rp = reinterpret_cast<const float2 *>(P + (size_t)c * kCurvRS + 2 * tid);
+            float x[NX];
 #pragma unroll
-            for (int wi = 0; wi < kMaxWindows; wi++) SL[wi] = SR[wi] = 0.f;
-#pragma unroll
-            for (int tau = 1; tau <= kHalo; tau++) {
-                // left sum over tau' < tau, right sum over 1 .. tau
-                if (kDefaultWindows) {
-                    if (tau == 4) SL[0] = sl;
-                    if (tau == 8) SL[1] = sl;
-                    if (tau == 16) SL[2] = sl;
-                } else {
-#pragma unroll
-                    for (int wi = 0; wi < kMaxWindows; wi++) SL[wi] = wv[wi] == tau ? sl : SL[wi];
-                }
-                if (tau < kHalo) sl += row[-tau];
-                sr += row[tau];
-                if (kDefaultWindows) {
-                    if (tau == 4) SR[0] = sr;
-                    if (tau == 8) SR[1] = sr;
-                    if (tau == 16) SR[2] = sr;
-                } else {
-#pragma unroll
-                    for (int wi = 0; wi < kMaxWindows; wi++) SR[wi] = wv[wi] == tau ? sr : SR[wi];
-                }
+            for (int k = 0; k < NX / 2; k++) {
+                const float2 y = rp[k];
+                x[2 * k] = y.x;
+                x[2 * k + 1] = y.y;
             }
 #pragma unroll
-            for (int wi = 0; wi < kMaxWindows; wi++) {
-                if (wi >= nw) break;
-                const float dm = h - SL[wi] * inv_w[wi];   // h_i - mean of the left window
-                const float dp = SR[wi] * inv_w[wi] - h;   // mean of the right window - h_i
-                acc[wi][0] = fmaf(dm, dm, acc[wi][0]);
-                acc[wi][1] = fmaf(dp, dp, acc[wi][1]);
-                acc[wi][2] = fmaf(dm, dp, acc[wi][2]);
+            for (int pp = 0; pp < kCurvPP; pp++) {
+                const int R = kHalo + pp;   // the position's index in x
+                const float h = x[R];
+                float sl = h, sr = 0.f;
+                float SL[kMaxWindows], SR[kMaxWindows];
+#pragma unroll
+                for (int wi = 0; wi < kMaxWindows; wi++) SL[wi] = SR[wi] = 0.f;
+#pragma unroll
+                for (int tau = 1; tau <= kHalo; tau++) {
+                    // left sum over tau' < tau, right sum over 1 .. tau
+                    if (kDefaultWindows) {
+                        if (tau == 4) SL[0] = sl;
+                        if (tau == 8) SL[1] = sl;
+                        if (tau == 16) SL[2] = sl;
+                    } else {
+#pragma unroll
+                        for (int wi = 0; wi < kMaxWindows; wi++) SL[wi] = wv[wi] == tau ? sl : SL[wi];
+                    }
+                    if (tau < kHalo) sl += x[R - tau];
+                    sr += x[R + tau];
+                    if (kDefaultWindows) {
+                        if (tau == 4) SR[0] = sr;
+                        if (tau == 8) SR[1] = sr;
+                        if (tau == 16) SR[2] = sr;
+                    } else {
+#pragma unroll
+                        for (int wi = 0; wi < kMaxWindows; wi++) SR[wi] = wv[wi] == tau ? sr : SR[wi];
+                    }
+                }
+#pragma unroll
+                for (int wi = 0; wi < kMaxWindows; wi++) {
+                    if (wi >= nw) break;
+                    const float dm = h - SL[wi] * inv_w[wi];   // h_i - mean of the left window
+                    const float dp = SR[wi] * inv_w[wi] - h;   // mean of the right window - h_i
+                    acc[pp][wi][0] = fmaf(dm, dm, acc[pp][wi][0]);
+                    acc[pp][wi][1] = fmaf(dp, dp, acc[pp][wi][1]);
+                    acc[pp][wi][2] = fmaf(dm, dp, acc[pp][wi][2]);
+                }
             }
         }
     }
-    const int i = i0 + tid;
-    if (i >= a.T) return;
 #pragma unroll
-    for (int wi = 0; wi < kMaxWindows; wi++) {
-        if (wi >= nw) break;
-        const int w = wv[wi];
-        double k = 0.0;
-        if (i >= w && i < a.T - w) {
-            const double x = sqrt((double)acc[wi][0]), y = sqrt((double)acc[wi][1]);
-            k = 1.0 - (double)acc[wi][2] / ((x > kEps ? x : kEps) * (y > kEps ? y : kEps));
+    for (int pp = 0; pp < kCurvPP; pp++) {
+        const int i = i0 + kCurvPP * tid + pp;
+        if (i >= a.T) continue;
+#pragma unroll
+        for (int wi = 0; wi < kMaxWindows; wi++) {
+            if (wi >= nw) break;
+            const int w = wv[wi];
+            double k = 0.0;
+            if (i >= w && i < a.T - w) {
+                const double xv = sqrt((double)acc[pp][wi][0]), yv = sqrt((double)acc[pp][wi][1]);
+                k = 1.0 - (double)acc[pp][wi][2] / ((xv > kEps ? xv : kEps) * (yv > kEps ? yv : kEps));
+            }
+            klw[((size_t)li * nw + wi) * a.T + i] = k;
         }
-        klw[((size_t)li * nw + wi) * a.T + i] = k;
     }
 }
 
