@@ -686,7 +686,7 @@ constexpr int kBNtW = 9;              // column tiles per warp: ceil(18 / 2) for
 __host__ __device__ constexpr int band_ncol_tiles(int nb) { return (kBM + nb - 1 + 7) / 8; }
 __host__ __device__ constexpr size_t band_mma_smem(int nb) {
     return (size_t)2 * (kBM + 8 * band_ncol_tiles(nb)) * kBStride * sizeof(__nv_bfloat16) +
-           (size_t)2 * (kBM + 8 * band_ncol_tiles(nb)) * sizeof(float);
+           (size_t)2 * (kBM + 8 * band_ncol_tiles(nb)) * sizeof(float) + (size_t)3 * 128 * sizeof(double);
 }
 
 __global__ void __launch_bounds__(256) seg_band_mma_kernel(const __nv_bfloat16 *V, BandArgs b,
@@ -701,6 +701,17 @@ __global__ void __launch_bounds__(256) seg_band_mma_kernel(const __nv_bfloat16 *
     __nv_bfloat16 *stg = reinterpret_cast<__nv_bfloat16 *>(smem_raw);   // [2][nrs][kBStride]
     float *inv_r = reinterpret_cast<float *>(stg + (size_t)2 * nrs * kBStride);   // [nrs]
     float *nrm_r = inv_r + nrs;                                                    // [nrs]
+    // per slot length len = n_min + k: 1 / nS, 1 / ((nS - 1) n_seg) (nS = len - 1)
+    // and lambda_n pen^2, so that the edge weights need no fp64 division
+    double *t_ins = reinterpret_cast<double *>(nrm_r + nrs);   // [128] (8-byte aligned: 296 nrs bytes in)
+    double *t_idn = t_ins + 128, *t_pen = t_idn + 128;
+    for (int k = threadIdx.x; k < nb; k += blockDim.x) {
+        const int len = b.n_min + k, nS = len - 1;
+        t_ins[k] = nS >= 1 ? 1.0 / nS : 0.0;
+        t_idn[k] = nS >= 2 ? 1.0 / (double)(nS - 1) / a.nseg : 0.0;
+        const double pen = (double)(len - b.n0) / b.n0;
+        t_pen[k] = b.lambda_n * pen * pen;
+    }
     const int E0 = blockIdx.x * kBM;
     const int a0 = E0 + 1 - b.n_max;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -804,15 +815,14 @@ __global__ void __launch_bounds__(256) seg_band_mma_kernel(const __nv_bfloat16 *
                 ew[(size_t)i * nbp + (len - b.n_min)] = -INFINITY;
                 continue;
             }
-            const int nS = len - 1;
+            const int nS = len - 1, kl = len - b.n_min;
             double disp = 0.0;
             if (nS >= 2) {
                 const double s2 = p2[ep] - p2[ap];     // sum_{t=ap}^{ep-1} ||d_t||^2
-                disp = (s2 - (double)sd[q][h] / nS) / (double)(nS - 1) / a.nseg;
+                disp = (s2 - (double)sd[q][h] * t_ins[kl]) * t_idn[kl];
             }
             const double gam = ap == 0 ? 0.0 : bscore[a.cs + ap - 1] - b.c_cut;
-            const double pen = (double)(len - b.n0) / b.n0;
-            ew[(size_t)i * nbp + (len - b.n_min)] = (float)(gam - b.lambda_d * disp - b.lambda_n * pen * pen);
+            ew[(size_t)i * nbp + kl] = (float)(gam - b.lambda_d * disp - t_pen[kl]);
         }
     }
 }
