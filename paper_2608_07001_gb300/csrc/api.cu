@@ -573,10 +573,10 @@ static cudaError_t build_fresh(Ctx &c, const void *K, const void *V, const void 
 // Trees (build.cu).  Every op's key is bounded before it is built: a pending
 // node's split key is at most min(creator key, omega R D).  Each pass derives
 // the threshold tau of the ops built so far (a lower bound of the final one)
-// and expands the pending nodes whose bound reaches it, up to four levels
-// deep (a child below tau stays pending), until none does; nodes left
-// pending can never be selected.  Four levels per launch save reloading the
-// units that keep expanding; tau is re-derived between launches.  When the budget is
+// and expands the pending nodes whose bound reaches it -- one level while tau
+// still rises, up to four once it has settled (a child below tau stays
+// pending) -- until none does; nodes left pending can never be selected.
+// Several levels per launch save reloading the units that keep expanding.  When the budget is
 // smaller than the number of units, the first launch evaluates only the
 // roots' own distortion (their Add ops) and later passes expand the units
 // with the largest bounds first, about 32768 at a time, so that tau rises
@@ -591,6 +591,7 @@ static cudaError_t build_passes(Ctx &c, const void *K, const void *V, const void
     const int64_t nu = (int64_t)c.p.L * c.p.G * J;
     const bool root_only = c.B_free < nu;
     const int pass_units = 32768;
+    float tau_prev = -INFINITY;   // tau of the previous pass
     cudaError_t e = cudaSuccess;
     for (int it = 0; e == cudaSuccess; it++) {
         struct {
@@ -625,7 +626,15 @@ static cudaError_t build_passes(Ctx &c, const void *K, const void *V, const void
         const float tau_eff = fmaxf(tau, h.cut);
         // everything built so far fits and few units remain: expand them fully at once
         const bool fits = h.all && (long long)c.B_free - (long long)h.total >= (long long)h.pot;
-        const int levels = fits ? 4 * gkv::kMaxUnit : 4;
+        // several levels per launch once tau has settled (within 10 % of the
+        // previous pass's): the children are then checked against a tau close to
+        // the final one; while tau still rises, one level, so that a child it
+        // would rule out next pass is not built.  With long units the passes
+        // follow their levels anyway, and several levels per launch spare the
+        // other units that many reloads.
+        const bool settled = tau_prev > -INFINITY && tau <= tau_prev + 0.1f * fabsf(tau_prev);
+        const int levels = fits ? 4 * gkv::kMaxUnit : ((settled || c.n_long > 0) ? 4 : 1);
+        tau_prev = tau;
         gkv::StageTimer tm(c, 3, s);
         e = gkv::launch_unit_build(c, K, V, Q, omega, w.slots, J, 1, 0, levels, tau_eff, w.u_list,
                                    h.count[0], w.u_list + (nu - h.count[1]), h.count[1], s);
