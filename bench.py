@@ -40,7 +40,7 @@ FP32_LANES = 128
 # DRAM bytes of one compression in the dominant stage, from an ncu capture
 # (profiles/unit_build_llama128k_2layers_32x.md: the 2-layer slice's 2.31 GB
 # scaled by 16 to 32 layers); reported only for the workload it was taken on
-STAGE_TRAFFIC = {("unit_trees", "llama128k@32x"): (36.994e9, "ncu dram bytes of every unit_build launch "
+STAGE_TRAFFIC = {("unit_trees", "llama128k@32x"): (36.62e9, "ncu dram bytes of every unit_build launch "
                                                            "of one compression on the 2-layer slice x 16")}
 
 
