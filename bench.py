@@ -38,7 +38,7 @@ PEAK_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustaine
                  "sm_max_mhz": 2070.0}
 FP32_LANES = 128
 # DRAM bytes of one compression in the dominant stage, from an ncu capture
-# (profiles/unit_build_llama128k_2layers_32x.md: the 2-layer slice's 2.31 GB
+# (profiles/unit_build_llama128k_2layers_32x.md: the 2-layer slice's 2.29 GB
 # scaled by 16 to 32 layers); reported only for the workload it was taken on
 STAGE_TRAFFIC = {("unit_trees", "llama128k@32x"): (36.62e9, "ncu dram bytes of every unit_build launch "
                                                            "of one compression on the 2-layer slice x 16")}
