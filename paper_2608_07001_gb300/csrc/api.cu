@@ -640,7 +640,7 @@ static cudaError_t build_passes(Ctx &c, const void *K, const void *V, const void
                                    h.count[0], w.u_list + (nu - h.count[1]), h.count[1], s);
         if (e == cudaSuccess && h.count[2] > 0) {   // long units: one level, or all of them when they fit
             e = gkv::launch_long_level(c, K, V, Q, omega, w.slots, J, 0, 0, tau_eff, w.long_list, h.count[2], 0, -1,
-                                       s, nullptr);
+                                       s, nullptr, tau);   // subtrees prune against tau itself, not the cut
             if (e == cudaSuccess && fits) e = long_to_leaves(c, K, V, Q, omega, w.long_list, h.count[2], s);
         }
         c.build_passes = it + 2;

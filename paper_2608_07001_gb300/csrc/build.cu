@@ -1187,7 +1187,7 @@ __global__ void __launch_bounds__(kNT, NMAX <= 64 ? 2 : 1) unit_build_kernel(Bui
     if (lane == 0) { sm.wcnt[warp][0] = w_scan; sm.wcnt[warp][1] = w_eval; sm.wcnt[warp][2] = w_len; }
     __syncthreads();
     if (tid == 0) {
-        if constexpr (!SUB) {   // a subtree is built completely inside its reserved slots
+        if constexpr (!SUB) {   // a subtree stays inside its reserved slots; what it left pending is never needed
             A.u_nnodes[uid] = sm.nnodes;
             A.u_pend[uid] = sm.pend;
         }
@@ -1271,7 +1271,7 @@ cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *
 
 cudaError_t launch_unit_subtrees(Ctx &c, const void *K, const void *V, const void *Q, const float *omega,
                                  const int32_t *slots, int J, const int32_t *list_short, int n_short,
-                                 const int32_t *list_long, int n_long, cudaStream_t s) {
+                                 const int32_t *list_long, int n_long, float tau_prune, cudaStream_t s) {
     if (n_short + n_long == 0) return cudaSuccess;
     cudaError_t e;
     const gkv_params &p = c.p;
@@ -1287,7 +1287,7 @@ cudaError_t launch_unit_subtrees(Ctx &c, const void *K, const void *V, const voi
     A.inv_sqrt_d = (float)(1.0 / sqrt((double)p.d));
     A.lamZ = (float)p.lambda_Z; A.lamM = (float)p.lambda_M; A.eps = (float)p.eps;
     A.lam_kappa = p.lambda_kappa; A.base_frac = p.base_frac;
-    A.resume = 0; A.subtree = 1; A.root_only = 0; A.max_levels = 4 * kMaxUnit; A.tau = -INFINITY;
+    A.resume = 0; A.subtree = 1; A.root_only = 0; A.max_levels = 4 * kMaxUnit; A.tau = tau_prune;
     A.nd_a = c.w.nd_a; A.nd_b = c.w.nd_b; A.nd_child0 = c.w.nd_child0;
     A.nd_parent = c.w.nd_parent; A.nd_unit = c.w.nd_unit;
     A.nd_nchild = c.w.nd_nchild; A.nd_cost = c.w.nd_cost;

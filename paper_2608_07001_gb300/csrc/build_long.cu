@@ -250,7 +250,11 @@ __global__ void __launch_bounds__(kLT) long_collect_kernel(LongArgs A) {
         if (bnd < A.tau) { pend = fmaxf(pend, bnd); continue; }
         const int len = A.nd_b[v] - A.nd_a[v];
         if (len > kMaxUnit) { cnt++; continue; }
-        // a small node: its subtree goes to the unit kernel (subtree mode)
+        // a small node: its subtree goes to the unit kernel (subtree mode), into
+        // the slots reserved for it.  A node the unit kernel left pending inside
+        // a subtree has none, but its bound is below a threshold that only
+        // rises, so it never reaches this point; it is skipped all the same.
+        if (A.nd_child0[v] < 0) continue;
         const int cls = len <= kShortUnit ? 0 : 1;
         const unsigned int pos = atomicAdd(&A.n_items[1 + cls], 1u);
         if ((int64_t)pos < A.cap_items) A.sub[(size_t)cls * A.cap_items + pos] = (int32_t)v;
@@ -1151,7 +1155,7 @@ cudaError_t launch_long_units(Ctx &c, const int32_t *long_slots, int n_long, int
 cudaError_t launch_long_level(Ctx &c, const void *K, const void *V, const void *Q, const float *omega,
                               const int32_t *slots, int J, int fresh, int root_only, float tau,
                               const int32_t *list, int n_list, int lg0, int nlg, cudaStream_t s,
-                              unsigned int *n_items_host) {
+                              unsigned int *n_items_host, float tau_prune) {
     const gkv_params &p = c.p;
     Workspace &w = c.w;
     if (nlg < 0) nlg = p.L * p.G - lg0;
@@ -1216,7 +1220,7 @@ cudaError_t launch_long_level(Ctx &c, const void *K, const void *V, const void *
     }
     // nodes of at most kMaxUnit tokens: their subtrees on the unit kernel
     return launch_unit_subtrees(c, K, V, Q, omega, slots, J, w.long_sub, (int)cnt[1], w.long_sub + w.long_cap,
-                                (int)cnt[2], s);
+                                (int)cnt[2], tau_prune, s);
 }
 
 }  // namespace gkv

@@ -324,10 +324,12 @@ cudaError_t launch_unit_build(Ctx &c, const void *K, const void *V, const void *
 // Subtree mode of the unit kernel (build.cu): the listed pending nodes of
 // long units (global node indices; at most kShortUnit tokens in list_short,
 // at most kMaxUnit in list_long) each get their subtree built to the leaves
-// into the node slots reserved for it (its child0, unit-relative).
+// into the node slots reserved for it (its child0, unit-relative), except the
+// children whose key bound is below tau_prune (the threshold of the ops built
+// so far: it only rises, so they can never be selected); they stay pending.
 cudaError_t launch_unit_subtrees(Ctx &c, const void *K, const void *V, const void *Q, const float *omega,
                                  const int32_t *slots, int J, const int32_t *list_short, int n_short,
-                                 const int32_t *list_long, int n_long, cudaStream_t s);
+                                 const int32_t *list_long, int n_long, float tau_prune, cudaStream_t s);
 // Slot indices split by length class: short ones at list[0, count[0]), those
 // of kShortUnit + 1 .. kMaxUnit tokens at list[J - count[1], J), longer ones
 // at long_slots[0, count[2]); count[3] receives the tokens of the longer ones.
@@ -336,13 +338,16 @@ cudaError_t launch_slot_classes(Ctx &c, const int32_t *slots, int J, int32_t *li
 // One level of the trees of long units (build_long.cu): with fresh = 1 the
 // roots of the listed slots for (l, g) in [lg0, lg0 + nlg) (root_only: their
 // own distortion and Add gain, the split left pending), else the pending
-// nodes of the listed units whose key bound reaches tau.  With n_items_host
-// the level's work-item count is read back (synchronises s) and a level
-// without work launches nothing more.
+// nodes of the listed units whose key bound reaches tau.  The subtrees of
+// its nodes of at most kMaxUnit tokens prune against tau_prune (the
+// allocation threshold of the ops built so far, -inf when none; never a
+// scheduling cut, since a node pruned inside a subtree is not resumed).  With
+// n_items_host the level's work-item count is read back (synchronises s) and
+// a level without work launches nothing more.
 cudaError_t launch_long_level(Ctx &c, const void *K, const void *V, const void *Q, const float *omega,
                               const int32_t *slots, int J, int fresh, int root_only, float tau,
                               const int32_t *list, int n_list, int lg0, int nlg, cudaStream_t s,
-                              unsigned int *n_items_host);
+                              unsigned int *n_items_host, float tau_prune = -INFINITY);
 size_t long_res_bytes();
 // out[q nlg + i] = the unit id of long slot long_slots[q] for (l, g) = lg0 + i.
 cudaError_t launch_long_units(Ctx &c, const int32_t *long_slots, int n_long, int lg0, int nlg, int J,
